@@ -1,0 +1,297 @@
+"""Checks that pin the float64 oracle to facts fixed by the paper and by mathematics.
+
+Each function returns the largest discrepancy it found (a float).  They are used
+by test_oracle_pins.py against the real oracle and by test_oracle_mutants.py
+against deliberately broken copies of it, to show that a plausible mistake in
+the oracle (a sign, an index, a dropped term) makes at least one pin fail.
+
+None of these functions calls the CUDA library.  The reference values are
+computed here from closed forms that differ from the oracle's own formulas.
+"""
+import numpy as np
+
+
+def rng(seed):
+    return np.random.default_rng(seed)
+
+
+def _worst(*vals):
+    """Largest of the discrepancies; NaN counts as an infinite discrepancy."""
+    out = 0.0
+    for x in vals:
+        x = float(x)
+        if x != x:
+            return float("inf")
+        out = max(out, x)
+    return out
+
+
+def _softmax_masked(s, valid):
+    s = np.where(valid, s, -np.inf)
+    mx = s.max(axis=-1, keepdims=True)
+    e = np.where(valid, np.exp(s - mx), 0.0)
+    return e / e.sum(axis=-1, keepdims=True), (mx + np.log(e.sum(axis=-1, keepdims=True)))[..., 0]
+
+
+def dirichlet_sine_ratio(M, w, x):
+    """D_M(x) from the Dirichlet closed form: (2M-1) D_M(x) = sin((M-1/2) w x) / sin(w x / 2),
+    i.e. sum_{m=-N}^{N} e^{i m y} = sin((N+1/2) y)/sin(y/2) at N = M-1, y = w x; value 1 where
+    sin(w x / 2) = 0."""
+    x = np.asarray(x, dtype=np.float64)
+    den = np.sin(w * x / 2.0)
+    num = np.sin((M - 0.5) * w * x)
+    out = np.ones_like(x)
+    nz = np.abs(den) > 1e-12
+    out[nz] = num[nz] / ((2 * M - 1) * den[nz])
+    return out
+
+
+# ---------------------------------------------------------------- P1: kernel
+
+def pin_dirichlet_identity(orc):
+    """(2M-1) D_M(x) = sin((M-1/2)x)/sin(x/2) at omega = 1 (Eq. dirichlet; the identity
+    sum_{m=-N}^{N} e^{imx} = sin((N+1/2)x)/sin(x/2) at N = M-1)."""
+    err = 0.0
+    xs = np.linspace(0.05, 2 * np.pi - 0.05, 97)
+    for M in (1, 2, 3, 6, 17):
+        d = orc.dirichlet(M, xs, 1.0)
+        ref = np.sin((M - 0.5) * xs) / ((2 * M - 1) * np.sin(xs / 2))
+        err = _worst(err, float(np.abs(d - ref).max()))
+    return err
+
+
+def pin_dirichlet_samples(orc):
+    """D_M(0) = 1 and D_M(t) = 0 for t = 1..2M-2 at omega = 2 pi/(2M-1) (text after Eq. dirichlet)."""
+    err = 0.0
+    for M in (1, 2, 4, 9):
+        n = 2 * M - 1
+        d = orc.dirichlet(M, np.arange(n), 2 * np.pi / n)
+        ref = np.zeros(n)
+        ref[0] = 1.0
+        err = _worst(err, float(np.abs(d - ref).max()))
+    return err
+
+
+# ------------------------------------------------------- grid and tables
+
+def pin_grid(orc):
+    """Dilated grid round(j T / S), half to even; the paper's grid at S = 2M-1; clamp T >= 2M-1."""
+    err = 0.0
+    delta, _, _ = orc.tables(3, 4, 10.0)
+    err = _worst(err, float(np.abs(delta - np.array([0.0, 2.0, 5.0, 8.0])).max()))   # 2.5->2, 7.5->8
+    M, T = 4, 14.0
+    delta, _, _ = orc.tables(M, 2 * M - 1, T)
+    ref = np.round(np.arange(2 * M - 1) / (2 * M - 1) * T)
+    err = _worst(err, float(np.abs(delta - ref).max()))
+    err = _worst(err, abs(orc.period(4, 3.0) - 7.0), abs(orc.period(4, 9.0) - 9.0))
+    err = _worst(err, abs(orc.omega_of(4, 3.0) - 2 * np.pi / 7.0), abs(orc.omega_of(4, 3.0, 0.5) - 0.5))
+    return err
+
+
+def pin_translated_coefficients(orc):
+    """App. B: D_M(t - Delta) = sum_m A[Delta,m] cos(m w t) + B[Delta,m] sin(m w t), with D_M
+    from the sine-ratio closed form, for several periods (also T > 2M-1)."""
+    err = 0.0
+    for M, S, T in ((4, 7, 7.0), (4, 7, 14.0), (5, 6, 23.0), (3, 3, 11.0)):
+        delta, A, B = orc.tables(M, S, T)
+        w = 2 * np.pi / orc.period(M, T)
+        t = np.arange(-30, 31, dtype=np.float64)
+        m = np.arange(M)
+        C = np.cos(np.outer(t, m) * w)
+        Sn = np.sin(np.outer(t, m) * w)
+        for j in range(S):
+            lhs = dirichlet_sine_ratio(M, w, t - delta[j])
+            rhs = C @ A[j] + Sn @ B[j]
+            err = _worst(err, float(np.abs(lhs - rhs).max()))
+    return err
+
+
+# ------------------------------------------------------- P2: state closed form
+
+def pin_state_closed_form(orc):
+    """Eq. (states): after tokens 0..t, Kcos[m] = sum_{t'<=t} cos(m w (t-t')) k_t' and
+    Ksin[m] = sum sin(m w (t-t')) k_t'; with an initial state Z0 the rotated Z0
+    e^{i m w (t+1)} is added (App. B induction)."""
+    g = rng(11)
+    err = 0.0
+    for M, S, T, L, d in ((3, 5, 5.0, 9, 4), (4, 3, 17.0, 13, 3)):
+        q, k, v = (g.standard_normal((1, 2, L, d)) for _ in range(3))
+        z0 = g.standard_normal((1, 2, 2, M, 2, d))
+        z0[:, :, :, 0, 1, :] = 0.0
+        w = 2 * np.pi / orc.period(M, T)
+        for init in (None, z0):
+            st = orc.forward(q, k, v, M, S, T, state=init, return_state=True)["state"]
+            lag = (L - 1) - np.arange(L)
+            for kv, x in ((0, k), (1, v)):
+                for m in range(M):
+                    zc = (np.cos(m * w * lag)[None, None, :, None] * x).sum(2)
+                    zs = (np.sin(m * w * lag)[None, None, :, None] * x).sum(2)
+                    if init is not None:
+                        a, b = init[:, :, kv, m, 0], init[:, :, kv, m, 1]
+                        ph = m * w * L
+                        zc = zc + np.cos(ph) * a - np.sin(ph) * b
+                        zs = zs + np.sin(ph) * a + np.cos(ph) * b
+                    err = _worst(err, float(np.abs(st[:, :, kv, m, 0] - zc).max()),
+                              float(np.abs(st[:, :, kv, m, 1] - zs).max()))
+    return err
+
+
+# ------------------------------------------------ P3: full resolution = attention
+
+def pin_causal_attention(orc):
+    """T = S = 2M-1 and L <= 2M-1 give causal softmax attention exactly (Fig. 2b; text after
+    Eq. conv_key); lse is the log-sum-exp of the causal scores."""
+    g = rng(5)
+    err = 0.0
+    for M, L, d in ((4, 7, 5), (6, 9, 3), (1, 1, 2)):
+        n = 2 * M - 1
+        q, k, v = (g.standard_normal((2, 1, L, d)) for _ in range(3))
+        for form in ("naive", "modes", "parallel"):
+            r = orc.forward(q, k, v, M, n, float(n), form=form)
+            s = np.einsum("bhtd,bhud->bhtu", q, k) / np.sqrt(d)
+            valid = np.tril(np.ones((L, L), bool))
+            p, lse = _softmax_masked(s, valid)
+            o = np.einsum("bhtu,bhud->bhtd", p, v)
+            err = _worst(err, float(np.abs(r["o"] - o).max()), float(np.abs(r["lse"] - lse).max()))
+    return err
+
+
+# -------------------------------------------------- P4: aliasing modulo 2M-1
+
+def pin_aliasing(orc):
+    """T = S = 2M-1, L > 2M-1: slot j holds the sum of the keys k_t' with t - t' = j (mod 2M-1)
+    (Eq. conv_key) and is visible once t >= j."""
+    g = rng(7)
+    err = 0.0
+    for M, L, d in ((3, 17, 4), (4, 30, 2)):
+        n = 2 * M - 1
+        q, k, v = (g.standard_normal((1, 1, L, d)) for _ in range(3))
+        r = orc.forward(q, k, v, M, n, float(n), form="naive")
+        for t in range(L):
+            Ks = np.zeros((n, d))
+            Vs = np.zeros((n, d))
+            for u in range(t + 1):
+                Ks[(t - u) % n] += k[0, 0, u]
+                Vs[(t - u) % n] += v[0, 0, u]
+            s = Ks @ q[0, 0, t] / np.sqrt(d)
+            valid = np.arange(n) <= t
+            p, _ = _softmax_masked(s[None], valid[None])
+            err = _worst(err, float(np.abs(r["o"][0, 0, t] - p[0] @ Vs).max()))
+    return err
+
+
+# ------------------------------------------ blurry case (T > 2M-1, S != 2M-1)
+
+def pin_blurry_bruteforce(orc):
+    """T > 2M-1: slots are Dirichlet-blurred lags, K~_t[j] = sum_{t'<=t} D_M(t - t' - Delta_j) k_t'
+    (Eq. compressed with Eq. translated), evaluated by brute force with the sine-ratio D_M and
+    the grid round(j T/S) computed here."""
+    g = rng(9)
+    err = 0.0
+    for M, S, T, L, d in ((3, 4, 10.0, 23, 3), (4, 6, 21.0, 40, 2), (2, 3, 8.0, 11, 5)):
+        q, k, v = (g.standard_normal((1, 1, L, d)) for _ in range(3))
+        r = orc.forward(q, k, v, M, S, T, form="naive")
+        w = 2 * np.pi / T
+        delta = np.round(np.arange(S) * T / S)
+        for t in range(L):
+            u = np.arange(t + 1)
+            W = dirichlet_sine_ratio(M, w, (t - u)[None, :] - delta[:, None])   # [S, t+1]
+            Ks = W @ k[0, 0, : t + 1]
+            Vs = W @ v[0, 0, : t + 1]
+            s = Ks @ q[0, 0, t] / np.sqrt(d)
+            valid = t >= delta
+            p, lse = _softmax_masked(s[None], valid[None])
+            err = _worst(err, float(np.abs(r["o"][0, 0, t] - p[0] @ Vs).max()),
+                      float(abs(r["lse"][0, 0, t] - lse[0])))
+    return err
+
+
+# --------------------------------------------- P5: the oracle's forms agree
+
+def pin_forms_agree(orc):
+    """Alg. 2 recurrence = mode read-out = parallel closed form, also for T > 2M-1 and S != 2M-1."""
+    g = rng(3)
+    err = 0.0
+    for M, S, T, L, d in ((4, 4, 16.0, 37, 5), (3, 5, 11.0, 20, 3), (5, 9, 9.0, 25, 4), (2, 2, 6.5, 19, 2)):
+        q, k, v = (g.standard_normal((2, 2, L, d)) for _ in range(3))
+        ref = orc.forward(q, k, v, M, S, T, form="naive")
+        for form in ("modes", "parallel"):
+            r = orc.forward(q, k, v, M, S, T, form=form)
+            err = _worst(err, float(np.abs(r["o"] - ref["o"]).max()), float(np.abs(r["lse"] - ref["lse"]).max()))
+    return err
+
+
+# ------------------------------------- P6: lag form vs absolute (Alg. 1) form
+
+def lag_vs_absolute(orc, M, S, T, L=40, d=4, seed=13):
+    g = rng(seed)
+    q, k, v = (g.standard_normal((1, 2, L, d)) for _ in range(3))
+    a = orc.forward(q, k, v, M, S, T, form="naive")["o"]
+    b = orc.forward(q, k, v, M, S, T, form="absolute")["o"]
+    return float(np.linalg.norm(a - b) / np.linalg.norm(a))
+
+
+# ----------------------------------------------------------- P7: one mode
+
+def pin_single_mode(orc):
+    """M = 1 (one slot): D_1 = 1, so o_t = sum_{t'<=t} v_t' (Eq. dirichlet with M = 1)."""
+    g = rng(17)
+    q, k, v = (g.standard_normal((1, 3, 12, 4)) for _ in range(3))
+    r = orc.forward(q, k, v, 1, 1, 5.0, form="naive")
+    return float(np.abs(r["o"] - np.cumsum(v, axis=2)).max())
+
+
+# ---------------------------------------------- P9: gradients vs differences
+
+def pin_backward_fd(orc, h=1e-6):
+    """Analytic VJP = central finite differences of the Alg. 2 forward, loss = sum(dO * O)."""
+    g = rng(21)
+    err = 0.0
+    for M, S, T, L, d in ((3, 4, 9.0, 7, 3), (3, 5, 5.0, 12, 2)):
+        q, k, v, do = (g.standard_normal((1, 1, L, d)) for _ in range(4))
+        dq, dk, dv = orc.backward(q, k, v, do, M, S, T)
+        for x, gx in ((q, dq), (k, dk), (v, dv)):
+            fd = np.zeros_like(x)
+            for idx in np.ndindex(x.shape):
+                x0 = x[idx]
+                x[idx] = x0 + h
+                lp = float((orc.forward(q, k, v, M, S, T)["o"] * do).sum())
+                x[idx] = x0 - h
+                lm = float((orc.forward(q, k, v, M, S, T)["o"] * do).sum())
+                x[idx] = x0
+                fd[idx] = (lp - lm) / (2 * h)
+            err = _worst(err, float(np.abs(fd - gx).max() / (np.abs(gx).max() + 1e-30)))
+    return err
+
+
+# ------------------------------------------------- P10: state hand-off
+
+def pin_state_handoff(orc):
+    """Prefill of L1 tokens, then the remaining tokens from the returned state with pos0 = L1,
+    equals one pass over all tokens (Eq. recurrence is a one-step map)."""
+    g = rng(23)
+    M, S, T, L1, L2, d = 4, 5, 13.0, 11, 9, 3
+    q, k, v = (g.standard_normal((1, 2, L1 + L2, d)) for _ in range(3))
+    full = orc.forward(q, k, v, M, S, T, return_state=True)
+    a = orc.forward(q[:, :, :L1], k[:, :, :L1], v[:, :, :L1], M, S, T, return_state=True)
+    b = orc.forward(q[:, :, L1:], k[:, :, L1:], v[:, :, L1:], M, S, T, state=a["state"], pos0=L1,
+                    return_state=True)
+    return _worst(float(np.abs(b["o"] - full["o"][:, :, L1:]).max()),
+               float(np.abs(b["state"] - full["state"]).max()),
+               float(np.abs(a["o"] - full["o"][:, :, :L1]).max()))
+
+
+ALL_PINS = {
+    "dirichlet_identity": (pin_dirichlet_identity, 1e-12),
+    "dirichlet_samples": (pin_dirichlet_samples, 1e-13),
+    "grid": (pin_grid, 0.0),
+    "translated_coefficients": (pin_translated_coefficients, 1e-12),
+    "state_closed_form": (pin_state_closed_form, 1e-11),
+    "causal_attention": (pin_causal_attention, 1e-12),
+    "aliasing": (pin_aliasing, 1e-11),
+    "blurry_bruteforce": (pin_blurry_bruteforce, 1e-11),
+    "forms_agree": (pin_forms_agree, 1e-11),
+    "single_mode": (pin_single_mode, 1e-12),
+    "backward_fd": (pin_backward_fd, 1e-6),
+    "state_handoff": (pin_state_handoff, 1e-12),
+}

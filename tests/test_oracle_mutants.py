@@ -1,0 +1,66 @@
+"""Planted mistakes in the oracle must be caught by the pins (CPU only).
+
+Each case copies oracle/bla_oracle.c, plants one plausible mistake (a wrong sign,
+a dropped term, an index or grid error, a transposed operand), compiles the copy
+and runs every pin against it; at least one pin must fail.  This shows the pins
+constrain every part of the oracle, not only the parts they were written for.
+"""
+import ctypes
+import os
+import subprocess
+import sys
+
+import pytest
+
+sys.path.insert(0, os.path.dirname(os.path.abspath(__file__)))
+import oracle_pins as P  # noqa: E402
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SRC = os.path.join(ROOT, "oracle", "bla_oracle.c")
+
+MUTANTS = {
+    "rotation_sign": ("xc[i] = cw * a - sw * b + x[i];", "xc[i] = cw * a + sw * b + x[i];"),
+    "input_into_sin_row": ("xc[i] = cw * a - sw * b + x[i];\n            xs[i] = sw * a + cw * b;",
+                           "xc[i] = cw * a - sw * b;\n            xs[i] = sw * a + cw * b + x[i];"),
+    "coefficient_factor": ("A[j * M + m] = 2.0 * cos", "A[j * M + m] = 1.0 * cos"),
+    "sin_coefficient_sign": ("B[j * M + m] = 2.0 * sin", "B[j * M + m] = -2.0 * sin"),
+    "mode0_coefficient": ("A[j * M + 0] = 1.0 / n;", "A[j * M + 0] = 2.0 / n;"),
+    "mask_strict": ("(double)tabs >= delta[j]", "(double)tabs > delta[j]"),
+    "grid_floor": ("nearbyint((double)j * Te / (double)S)", "floor((double)j * Te / (double)S)"),
+    "no_period_clamp": ("return T < r ? r : T;", "return T;"),
+    "scale_1_over_d": ("1.0 / sqrt((double)dk)", "1.0 / (double)dk"),
+    "swapped_A_B_readout": ("acc += A[j * M + m] * Kc[m * dk + i] + B[j * M + m] * Ks[m * dk + i];",
+                            "acc += B[j * M + m] * Kc[m * dk + i] + A[j * M + m] * Ks[m * dk + i];"),
+    "read_before_update": ("rotate_add(M, dk, c->w, Kc, Ks, k + (size_t)t * dk);\n        rotate_add(M, dv, c->w, Vc, Vs, v + (size_t)t * dv);\n        if (want && !want[t]) continue;\n        /* \"Compute",
+                           "rotate_add(M, dk, c->w, Kc, Ks, k + (size_t)(t > 0 ? t - 1 : 0) * dk);\n        rotate_add(M, dv, c->w, Vc, Vs, v + (size_t)t * dv);\n        if (want && !want[t]) continue;\n        /* \"Compute"),
+    "backward_no_scale": ("dP *= c->scale;", "dP *= 1.0;"),
+    "backward_no_centering": ("p[j] * (dp[j] - pdp) * wgt", "p[j] * dp[j] * wgt"),
+    "dirichlet_no_factor2": ("acc += 2.0 / n * cos(m * w * x);", "acc += 1.0 / n * cos(m * w * x);"),
+}
+
+
+@pytest.fixture(scope="module")
+def src_text():
+    with open(SRC) as f:
+        return f.read()
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, src_text, tmp_path, monkeypatch):
+    import oracle.oracle as oo
+    old, new = MUTANTS[name]
+    assert src_text.count(old) >= 1, "mutation anchor not found: " + name
+    (tmp_path / "m.c").write_text(src_text.replace(old, new))
+    lib_path = str(tmp_path / "libm.so")
+    subprocess.run(["gcc", "-O1", "-fPIC", "-shared", "-fopenmp", "-std=c11", "-o", lib_path,
+                    str(tmp_path / "m.c"), "-lm"], check=True)
+    monkeypatch.setattr(oo, "_lib", oo._configure(ctypes.CDLL(lib_path)))
+    failed = []
+    for pname, (fn, tol) in sorted(P.ALL_PINS.items()):
+        try:
+            err = fn(oo)
+        except Exception:            # a crash or rejected argument also counts as caught
+            err = float("inf")
+        if not err <= tol:
+            failed.append(pname)
+    assert failed, "planted mistake %r passed every pin" % name
