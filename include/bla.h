@@ -1,0 +1,143 @@
+/*
+ * bla.h -- C ABI of the GB300 (sm_103a) Blurry Window Attention library, libbla_gb300.so.
+ *
+ * The operator (arxiv 2606.09862, "Blurry Window Attention", Sec. 3.1):
+ * per batch element b and head h, keys and values are written into a finite
+ * frequency window of M Fourier modes, a rotating state advanced by e^{i m w}
+ * (Eq. recurrence):
+ *     Kcos[m] <- cos(m w) Kcos[m] - sin(m w) Ksin[m] + k_t
+ *     Ksin[m] <- sin(m w) Kcos[m] + cos(m w) Ksin[m]          (V likewise)
+ * S blurry slots are rebuilt from the state with the translated Dirichlet
+ * coefficients A, B of Eq. (translated) at the dilated lags Delta_j (Eq. compressed),
+ *     K~[j] = sum_m A[j,m] Kcos[m] + B[j,m] Ksin[m],
+ * and the query attends over the slots with a softmax whose mask hides slots
+ * before the start of the sequence, t >= Delta_j (Eq. output; Alg. 2):
+ *     o_t = softmax_j(scale * q_t . K~[j] + mask) . V~.
+ *
+ * Conventions shared by every entry point
+ *   - All tensor arguments are DEVICE pointers owned by the caller; the library
+ *     allocates no device memory.  Scratch memory, where needed, is the
+ *     caller's `workspace` of at least bla_workspace_bytes() bytes, 256-byte
+ *     aligned.  Tensor pointers must be 16-byte aligned.
+ *   - q, k: [B][H][L][d_k]; v, o, dout: [B][H][L][d_v]; contiguous, element type
+ *     `dtype` (fp32 or bf16).  lse: [B][H][L] fp32 (natural-log log-sum-exp of the
+ *     unmasked slot scores).
+ *   - Recurrent state: fp32 [B][H][2 (K then V)][M][2 (cos, sin)][d], d = d_k for
+ *     the K half and d_v for the V half.  Row (m, sin) at m = 0 is the sine of the
+ *     zero frequency: it is always 0 and is neither read nor written.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Every call is
+ *     asynchronous on that stream; argument errors are detected on the host
+ *     before any launch.
+ *   - Nothing is thrown across the ABI; every function returns a bla_status.
+ *     bla_last_error_string() describes the most recent failure of the calling
+ *     thread.
+ *   - Bounded device waits: every wait inside a kernel gives up after a fixed
+ *     number of polls, records a code in the library's device error word and
+ *     returns.  bla_device_error() synchronises the stream and reports it as
+ *     BLA_ERR_TIMEOUT.
+ */
+#ifndef BLA_GB300_H
+#define BLA_GB300_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    BLA_OK = 0,
+    BLA_ERR_INVALID = 1,      /* bad argument (null pointer, size, alignment, range) */
+    BLA_ERR_UNSUPPORTED = 2,  /* valid but outside what the kernels implement */
+    BLA_ERR_CUDA = 3,         /* a CUDA runtime/driver call or a launch failed */
+    BLA_ERR_TIMEOUT = 4       /* a bounded device wait gave up (see bla_device_error) */
+} bla_status;
+
+typedef enum { BLA_F32 = 0, BLA_BF16 = 1 } bla_dtype;
+
+/* Operator parameters (Alg. 1-3 inputs: Q, K, V, period T, interpolation
+ * matrices A, B built from M, S and T, chunk size C). */
+typedef struct {
+    int B, H, L;        /* batch, heads, sequence length (L ignored by bla_decode_step) */
+    int d_k, d_v;       /* head dimensions */
+    int M;              /* Fourier modes, m = 0..M-1; 2M-1 live state rows per K and V */
+    int S;              /* slots; 1 <= S <= T.  The paper uses S = 2M-1 */
+    double window;      /* period T (> 0); clamped to max(T, 2M-1) as in Alg. 1 and 3 */
+    double omega;       /* <= 0: 2*pi/T (Sec. 3.1); > 0: used as the mode frequency w */
+    int chunk;          /* chunk length C of the fp32 path; 0 = default (64).  The bf16
+                           path always tiles by 128 tokens.  Results do not depend on it
+                           beyond rounding. */
+    double scale;       /* softmax scale; <= 0: 1/sqrt(d_k) (Eq. output, per head) */
+    int dtype;          /* bla_dtype of q, k, v, o, dout, dq, dk, dv */
+} bla_params;
+
+/* Which entry point a workspace size is asked for. */
+typedef enum { BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2 } bla_ws_kind;
+
+/*
+ * Bytes of device workspace the entry point `which` (a bla_ws_kind) needs for
+ * these parameters.  The workspace holds the interpolation tables (built on the
+ * device at every call) and, for the chunked paths, per-segment states and
+ * inter-pass intermediates.  Returns 0 for invalid parameters; call the entry
+ * point to get the error.
+ */
+size_t bla_workspace_bytes(const bla_params *p, int which);
+
+/*
+ * Chunked forward (prefill) over L tokens from the zero state (Sec. 3.1: "These
+ * states are initialized to zero"; Alg. 3 chunk form, computed in the lag frame of
+ * Eq. recurrence).
+ *   q, k, v    inputs as described above (device).
+ *   o          output [B][H][L][d_v] (device), dtype of the inputs.
+ *   lse        optional [B][H][L] fp32 (device) or NULL; needed by bla_backward.
+ *   state_out  optional fp32 state after the last token (device) or NULL; it is
+ *              the state bla_decode_step continues from with pos = L.
+ *   workspace  device scratch of >= bla_workspace_bytes(p, BLA_WS_FORWARD) bytes.
+ * dtype BLA_F32: fp32 SIMT path.  dtype BLA_BF16: tcgen05 tensor-core path with
+ * bf16 operands and fp32 accumulation; requires d_k = d_v in {64, 128},
+ * 2M in {64, 128, 256} and S in {32, 64, 128} (else BLA_ERR_UNSUPPORTED).
+ */
+bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k, const void *v,
+                               void *o, float *lse, float *state_out,
+                               void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * One single-token decode step for B*H independent sequences (Alg. 2 loop body).
+ *   pos        0-based absolute index of this token in its sequence (>= 0); the
+ *              slot mask keeps slot j iff pos >= Delta_j.
+ *   q, k, v    [B][H][d_k] / [B][H][d_k] / [B][H][d_v] (device), dtype p->dtype.
+ *   state      fp32 state (device), read and updated in place: on return it
+ *              includes this token.
+ *   o          [B][H][d_v] (device), dtype p->dtype.
+ *   workspace  device scratch of >= bla_workspace_bytes(p, BLA_WS_DECODE) bytes.
+ * p->L is ignored.  Requires d_k = d_v in {32, 64, 128} and S <= 256.
+ */
+bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, const void *k,
+                           const void *v, float *state, void *o, void *workspace, size_t ws_bytes,
+                           void *stream);
+
+/*
+ * Backward pass of bla_forward_chunked: given dout = dL/do, writes dq, dk, dv
+ * (same shapes and dtype as q, k, v).  o and lse are the forward's outputs.
+ * The vector-Jacobian product of the operator defined by Eqs. (recurrence),
+ * (compressed) and (output); the paper trains through it but prints no formula.
+ */
+bla_status bla_backward(const bla_params *p, const void *q, const void *k, const void *v,
+                        const void *o, const void *dout, const float *lse,
+                        void *dq, void *dk, void *dv, void *workspace, size_t ws_bytes, void *stream);
+
+/* Synchronise `stream` and report (then clear) the library's device error word:
+ * BLA_OK, or BLA_ERR_TIMEOUT if a bounded wait gave up since the last call. */
+bla_status bla_device_error(void *stream);
+
+/* Static description of a status code. */
+const char *bla_status_string(bla_status s);
+
+/* Description of the most recent failure on the calling thread ("" if none). */
+const char *bla_last_error_string(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BLA_GB300_H */

@@ -1,0 +1,166 @@
+"""Thin ctypes binding of libbla_gb300.so (C ABI in include/bla.h).
+
+The functions keep the C names.  They only marshal arguments: take torch CUDA
+tensors (PyTorch supplies device memory and streams), allocate outputs and the
+workspace with torch, pass raw pointers and the current stream to the library,
+and raise BlaError on any non-OK status.  All computation happens in the CUDA
+library; if it is missing this module raises instead of falling back.
+"""
+import ctypes
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libbla_gb300.so")
+
+BLA_OK, BLA_ERR_INVALID, BLA_ERR_UNSUPPORTED, BLA_ERR_CUDA, BLA_ERR_TIMEOUT = range(5)
+BLA_F32, BLA_BF16 = 0, 1
+BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE = 0, 1, 2
+
+EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
+            "bla_device_error", "bla_status_string", "bla_last_error_string")
+
+
+class BlaError(RuntimeError):
+    def __init__(self, status, msg):
+        super().__init__("%s (status %d)" % (msg, status))
+        self.status = status
+
+
+class Params(ctypes.Structure):
+    """Mirror of bla_params."""
+    _fields_ = [("B", ctypes.c_int), ("H", ctypes.c_int), ("L", ctypes.c_int),
+                ("d_k", ctypes.c_int), ("d_v", ctypes.c_int), ("M", ctypes.c_int), ("S", ctypes.c_int),
+                ("window", ctypes.c_double), ("omega", ctypes.c_double), ("chunk", ctypes.c_int),
+                ("scale", ctypes.c_double), ("dtype", ctypes.c_int)]
+
+
+_lib = None
+
+
+def load():
+    """Load the CUDA library (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError("libbla_gb300.so is missing at %s; run __graft_entry__.build() "
+                           "(there is no CPU fallback)" % LIB_PATH)
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, sz, P = ctypes.c_void_p, ctypes.c_size_t, ctypes.POINTER(Params)
+    lib.bla_workspace_bytes.restype = sz
+    lib.bla_workspace_bytes.argtypes = [P, ctypes.c_int]
+    lib.bla_forward_chunked.restype = ctypes.c_int
+    lib.bla_forward_chunked.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_decode_step.restype = ctypes.c_int
+    lib.bla_decode_step.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_backward.restype = ctypes.c_int
+    lib.bla_backward.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_device_error.restype = ctypes.c_int
+    lib.bla_device_error.argtypes = [vp]
+    lib.bla_status_string.restype = ctypes.c_char_p
+    lib.bla_status_string.argtypes = [ctypes.c_int]
+    lib.bla_last_error_string.restype = ctypes.c_char_p
+    lib.bla_last_error_string.argtypes = []
+    _lib = lib
+    return lib
+
+
+def _check(status):
+    if status != BLA_OK:
+        lib = load()
+        msg = lib.bla_last_error_string().decode() or lib.bla_status_string(status).decode()
+        raise BlaError(status, msg)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _dtype_code(dt):
+    if dt == torch.float32:
+        return BLA_F32
+    if dt == torch.bfloat16:
+        return BLA_BF16
+    raise BlaError(BLA_ERR_INVALID, "dtype must be float32 or bfloat16, got %s" % dt)
+
+
+def make_params(B, H, L, d_k, d_v, M, S, window, omega=0.0, chunk=0, scale=0.0, dtype=torch.bfloat16):
+    return Params(int(B), int(H), int(L), int(d_k), int(d_v), int(M), int(S), float(window), float(omega),
+                  int(chunk), float(scale), _dtype_code(dtype))
+
+
+def bla_workspace_bytes(params, which):
+    return int(load().bla_workspace_bytes(ctypes.byref(params), int(which)))
+
+
+def _workspace(params, which, device, workspace):
+    n = bla_workspace_bytes(params, which)
+    if workspace is not None:
+        return workspace, workspace.numel() * workspace.element_size()
+    if n == 0:
+        return None, 0
+    return torch.empty(n, dtype=torch.uint8, device=device), n
+
+
+def _need_cuda(*ts):
+    for t in ts:
+        if t is not None and (not t.is_cuda or not t.is_contiguous()):
+            raise BlaError(BLA_ERR_INVALID, "tensors must be contiguous CUDA tensors")
+
+
+def bla_forward_chunked(q, k, v, M, S, window, omega=0.0, chunk=0, scale=0.0, want_lse=True,
+                        want_state=False, workspace=None, out=None, stream=None):
+    """Chunked forward over q, k: [B,H,L,d_k], v: [B,H,L,d_v] (float32 or bfloat16 CUDA tensors).
+
+    Returns (o, lse or None, state or None); state is [B,H,2,M,2,d] fp32 (needs d_k == d_v).
+    """
+    _need_cuda(q, k, v)
+    B, H, L, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, L, dk, dv, M, S, window, omega, chunk, scale, q.dtype)
+    o = out if out is not None else torch.empty((B, H, L, dv), dtype=q.dtype, device=q.device)
+    lse = torch.empty((B, H, L), dtype=torch.float32, device=q.device) if want_lse else None
+    st = torch.empty((B, H, 2, M, 2, dk), dtype=torch.float32, device=q.device) if want_state else None
+    ws, n = _workspace(p, BLA_WS_FORWARD, q.device, workspace)
+    _check(load().bla_forward_chunked(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(st),
+                                      _ptr(ws), n, _stream(stream)))
+    return o, lse, st
+
+
+def bla_decode_step(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, workspace=None, out=None,
+                    stream=None):
+    """One decode step; q, k, v: [B,H,d]; state [B,H,2,M,2,d] fp32 is updated in place. Returns o."""
+    _need_cuda(q, k, v, state)
+    B, H, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, 1, dk, dv, M, S, window, omega, 0, scale, q.dtype)
+    o = out if out is not None else torch.empty((B, H, dv), dtype=q.dtype, device=q.device)
+    ws, n = _workspace(p, BLA_WS_DECODE, q.device, workspace)
+    _check(load().bla_decode_step(ctypes.byref(p), int(pos), _ptr(q), _ptr(k), _ptr(v), _ptr(state), _ptr(o),
+                                  _ptr(ws), n, _stream(stream)))
+    return o
+
+
+def bla_backward(q, k, v, o, dout, lse, M, S, window, omega=0.0, scale=0.0, workspace=None, stream=None):
+    """Gradients (dq, dk, dv) of the chunked forward for upstream gradient dout."""
+    _need_cuda(q, k, v, o, dout, lse)
+    B, H, L, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, L, dk, dv, M, S, window, omega, 0, scale, q.dtype)
+    dq, dkk, dvv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    ws, n = _workspace(p, BLA_WS_BACKWARD, q.device, workspace)
+    _check(load().bla_backward(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout), _ptr(lse),
+                               _ptr(dq), _ptr(dkk), _ptr(dvv), _ptr(ws), n, _stream(stream)))
+    return dq, dkk, dvv
+
+
+def bla_device_error(stream=None):
+    """Synchronise and raise BlaError if a bounded device wait gave up."""
+    _check(load().bla_device_error(_stream(stream)))

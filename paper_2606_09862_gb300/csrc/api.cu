@@ -1,0 +1,214 @@
+// api.cu -- the C ABI of libbla_gb300.so: argument checking, workspace layout, dispatch.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "common.cuh"
+#include "fwd_bf16.cuh"
+
+namespace bla {
+
+__device__ int g_dev_error = 0;
+
+int *device_error_word() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+    static int *cache[64] = {nullptr};
+    if (dev < 0 || dev >= 64) return nullptr;
+    if (!cache[dev]) {
+        void *ptr = nullptr;
+        if (cudaGetSymbolAddress(&ptr, g_dev_error) != cudaSuccess) return nullptr;
+        cache[dev] = static_cast<int *>(ptr);
+    }
+    return cache[dev];
+}
+
+namespace {
+
+thread_local char t_last_error[512] = "";
+
+bla_status fail(bla_status s, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
+bla_status fail(bla_status s, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(t_last_error, sizeof(t_last_error), fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+bla_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(BLA_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+constexpr double kPi = 3.14159265358979323846;
+constexpr int kDefaultChunkF32 = 64;
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Common parameter checks; fills the derived dimensions.
+bla_status check_params(const bla_params *p, OpDims *d) {
+    if (!p) return fail(BLA_ERR_INVALID, "params is NULL");
+    if (p->B < 1 || p->H < 1) return fail(BLA_ERR_INVALID, "B and H must be >= 1 (got %d, %d)", p->B, p->H);
+    if (p->L < 0) return fail(BLA_ERR_INVALID, "L must be >= 0 (got %d)", p->L);
+    if (p->d_k < 1 || p->d_v < 1) return fail(BLA_ERR_INVALID, "d_k and d_v must be >= 1");
+    if (p->M < 1) return fail(BLA_ERR_INVALID, "M must be >= 1 (got %d)", p->M);
+    if (!(p->window > 0.0) || !isfinite(p->window)) return fail(BLA_ERR_INVALID, "window (period T) must be > 0");
+    if (!isfinite(p->omega) || !isfinite(p->scale)) return fail(BLA_ERR_INVALID, "omega and scale must be finite");
+    if (p->dtype != BLA_F32 && p->dtype != BLA_BF16) return fail(BLA_ERR_INVALID, "dtype must be BLA_F32 or BLA_BF16");
+    const double Te = fmax(p->window, 2.0 * p->M - 1.0);
+    if (p->S < 1 || (double)p->S > Te) return fail(BLA_ERR_INVALID, "S must be in [1, T] (S=%d, T=%g)", p->S, Te);
+    if (p->chunk < 0) return fail(BLA_ERR_INVALID, "chunk must be >= 0");
+    if ((long long)p->B * p->H > (1ll << 31) - 1) return fail(BLA_ERR_INVALID, "B*H too large");
+    d->B = p->B; d->H = p->H; d->L = p->L; d->dk = p->d_k; d->dv = p->d_v; d->M = p->M; d->S = p->S;
+    d->R2 = 2 * p->M;
+    d->T = Te;
+    d->w = p->omega > 0.0 ? p->omega : 2.0 * kPi / Te;
+    d->scale = (float)(p->scale > 0.0 ? p->scale : 1.0 / sqrt((double)p->d_k));
+    d->dtype = p->dtype;
+    return BLA_OK;
+}
+
+int f32_chunk(const bla_params *p, const OpDims &d) {
+    int C = p->chunk > 0 ? p->chunk : kDefaultChunkF32;
+    if (d.L > 0 && C > d.L) C = d.L;
+    while (C > 1 && forward_f32_smem_bytes(d, C) > 227 * 1024) C /= 2;
+    return C < 1 ? 1 : C;
+}
+
+bla_status check_ws(void *ws, size_t have, size_t need) {
+    if (need == 0) return BLA_OK;
+    if (!ws) return fail(BLA_ERR_INVALID, "workspace is NULL but %zu bytes are needed", need);
+    if ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return fail(BLA_ERR_INVALID, "workspace must be 256-byte aligned");
+    if (have < need) return fail(BLA_ERR_INVALID, "workspace too small: %zu < %zu bytes", have, need);
+    return BLA_OK;
+}
+
+size_t ws_forward(const bla_params *p, const OpDims &d) {
+    if (d.dtype == BLA_F32) {
+        int C = f32_chunk(p, d);
+        return tables_bytes(d, C) + forward_f32_scratch_bytes(d, C);
+    }
+    return fwd_bf16_workspace_bytes(d);
+}
+
+size_t ws_decode(const OpDims &d) { return tables_bytes(d, 0); }
+
+}  // namespace
+}  // namespace bla
+
+using namespace bla;
+
+extern "C" {
+
+const char *bla_status_string(bla_status s) {
+    switch (s) {
+    case BLA_OK: return "ok";
+    case BLA_ERR_INVALID: return "invalid argument";
+    case BLA_ERR_UNSUPPORTED: return "unsupported configuration";
+    case BLA_ERR_CUDA: return "CUDA error";
+    case BLA_ERR_TIMEOUT: return "device wait timed out";
+    default: return "unknown status";
+    }
+}
+
+const char *bla_last_error_string(void) { return t_last_error; }
+
+size_t bla_workspace_bytes(const bla_params *p, int which) {
+    OpDims d;
+    if (check_params(p, &d) != BLA_OK) return 0;
+    switch (which) {
+    case BLA_WS_FORWARD: return ws_forward(p, d);
+    case BLA_WS_DECODE: return ws_decode(d);
+    case BLA_WS_BACKWARD: return fwd_bf16_workspace_bytes(d);
+    default: return 0;
+    }
+}
+
+bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k, const void *v, void *o,
+                               float *lse, float *state_out, void *workspace, size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    OpDims d;
+    bla_status s = check_params(p, &d);
+    if (s != BLA_OK) return s;
+    if (d.L > 0 && (!q || !k || !v || !o)) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse) ||
+        !aligned16(state_out))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (d.dtype == BLA_F32) {
+        const int C = f32_chunk(p, d);
+        size_t need = ws_forward(p, d);
+        if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
+        Tables t;
+        char *rest = tables_carve(d, C, static_cast<char *>(workspace), &t);
+        cudaError_t e = tables_build(d, t, st);
+        if (e != cudaSuccess) return cuda_fail(e, "table build");
+        e = launch_forward_f32(d, C, t, (const float *)q, (const float *)k, (const float *)v, (float *)o, lse,
+                               state_out, reinterpret_cast<float *>(rest), st);
+        if (e != cudaSuccess) return cuda_fail(e, "fp32 forward launch");
+        return BLA_OK;
+    }
+    const char *why = fwd_bf16_unsupported(d);
+    if (why) return fail(BLA_ERR_UNSUPPORTED, "bf16 forward: %s", why);
+    size_t need = fwd_bf16_workspace_bytes(d);
+    if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
+    cudaError_t e = fwd_bf16_run(d, q, k, v, o, lse, state_out, workspace, st);
+    if (e != cudaSuccess) return cuda_fail(e, "bf16 forward");
+    return BLA_OK;
+}
+
+bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
+                           float *state, void *o, void *workspace, size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    OpDims d;
+    bla_status s = check_params(p, &d);
+    if (s != BLA_OK) return s;
+    if (pos < 0) return fail(BLA_ERR_INVALID, "pos must be >= 0 (got %lld)", pos);
+    if (!q || !k || !v || !state || !o) return fail(BLA_ERR_INVALID, "q, k, v, state and o must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(state) || !aligned16(o))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    if (d.dk != d.dv || (d.dk != 32 && d.dk != 64 && d.dk != 128))
+        return fail(BLA_ERR_UNSUPPORTED, "decode needs d_k = d_v in {32, 64, 128} (got %d, %d)", d.dk, d.dv);
+    if (d.S > 256) return fail(BLA_ERR_UNSUPPORTED, "decode needs S <= 256 (got %d)", d.S);
+    size_t need = ws_decode(d);
+    if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    Tables t;
+    tables_carve(d, 0, static_cast<char *>(workspace), &t);
+    cudaError_t e = tables_build(d, t, st);
+    if (e != cudaSuccess) return cuda_fail(e, "table build");
+    e = launch_decode(d, pos, t, q, k, v, state, o, st);
+    if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    return BLA_OK;
+}
+
+bla_status bla_backward(const bla_params *p, const void *q, const void *k, const void *v, const void *o,
+                        const void *dout, const float *lse, void *dq, void *dk, void *dv, void *workspace,
+                        size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    OpDims d;
+    bla_status s = check_params(p, &d);
+    if (s != BLA_OK) return s;
+    (void)q; (void)k; (void)v; (void)o; (void)dout; (void)lse; (void)dq; (void)dk; (void)dv;
+    (void)workspace; (void)ws_bytes; (void)stream;
+    return fail(BLA_ERR_UNSUPPORTED, "backward is not implemented yet");
+}
+
+bla_status bla_device_error(void *stream) {
+    t_last_error[0] = 0;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "stream synchronize");
+    int code = 0, zero = 0;
+    e = cudaMemcpyFromSymbol(&code, g_dev_error, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "read device error word");
+    if (code != 0) {
+        e = cudaMemcpyToSymbol(g_dev_error, &zero, sizeof(int));
+        if (e != cudaSuccess) return cuda_fail(e, "clear device error word");
+        return fail(BLA_ERR_TIMEOUT, "device wait gave up (code %d)", code);
+    }
+    return BLA_OK;
+}
+
+}  // extern "C"

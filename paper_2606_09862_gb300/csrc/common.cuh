@@ -1,0 +1,81 @@
+// common.cuh -- shared definitions of the BLA CUDA library (sm_103a).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+#include "../../include/bla.h"
+
+namespace bla {
+
+// Error codes written to the device error word by bounded waits.
+enum : int {
+    DEVERR_NONE = 0,
+    DEVERR_MBAR_TIMEOUT = 1,   // an mbarrier wait exceeded its poll budget
+};
+
+// Derived operator constants (host side), from bla_params.
+struct OpDims {
+    int B, H, L, dk, dv, M, S, R2;   // R2 = 2M interleaved state rows (cos m, sin m)
+    double T;                        // clamped period
+    double w;                        // mode frequency omega
+    float scale;
+    int dtype;
+};
+
+// Table block (built on the device per call; lives in the caller's workspace).
+//   phi   [S][R2] fp32: phi[j][2m] = c_m cos(m w D_j), phi[j][2m+1] = c_m sin(m w D_j)
+//         with c_0 = 1/(2M-1), c_m = 2/(2M-1) (Eq. translated).
+//   delta [S] int: dilated lags round(j T / S).
+//   rot1  [M][2] fp32: cos(m w), sin(m w) (Eq. recurrence, one step).
+//   erel  [C+1][M][2] fp32: cos(m w tau), sin(m w tau), tau = 0..C (chunk phases).
+struct Tables {
+    float *phi;
+    int *delta;
+    float *rot1;
+    float *erel;
+    int C;
+};
+
+// Bytes taken by the table block for a given chunk length (each part 256-aligned).
+size_t tables_bytes(const OpDims &d, int C);
+// Carve the table block out of `base` (256-aligned) and return the next free byte.
+char *tables_carve(const OpDims &d, int C, char *base, Tables *t);
+// Launch the table builder (fp64 arithmetic, rounded to fp32).
+cudaError_t tables_build(const OpDims &d, const Tables &t, cudaStream_t st);
+
+static inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+__device__ __forceinline__ float bf16_to_f32(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T> __device__ __forceinline__ float load_elem(const T *p, size_t i);
+template <> __device__ __forceinline__ float load_elem<float>(const float *p, size_t i) { return p[i]; }
+template <> __device__ __forceinline__ float load_elem<__nv_bfloat16>(const __nv_bfloat16 *p, size_t i) {
+    return __bfloat162float(p[i]);
+}
+template <typename T> __device__ __forceinline__ void store_elem(T *p, size_t i, float x);
+template <> __device__ __forceinline__ void store_elem<float>(float *p, size_t i, float x) { p[i] = x; }
+template <> __device__ __forceinline__ void store_elem<__nv_bfloat16>(__nv_bfloat16 *p, size_t i, float x) {
+    p[i] = __float2bfloat16_rn(x);
+}
+
+// Device address of the library's error word (a __device__ int of this module, one per
+// device); kernels with bounded waits receive it as an argument.  NULL on failure.
+int *device_error_word();
+
+__device__ __forceinline__ void report_device_error(int *word, int code) {
+    if (word) atomicCAS(word, 0, code);
+}
+
+// Launchers of the individual kernels (defined in their .cu files).
+cudaError_t launch_forward_f32(const OpDims &d, int C, const Tables &t, const float *q, const float *k,
+                               const float *v, float *o, float *lse, float *state_out, float *scratch,
+                               cudaStream_t st);
+size_t forward_f32_scratch_bytes(const OpDims &d, int C);
+int forward_f32_smem_bytes(const OpDims &d, int C);
+
+cudaError_t launch_decode(const OpDims &d, long long pos, const Tables &t, const void *q, const void *k,
+                          const void *v, float *state, void *o, cudaStream_t st);
+
+}  // namespace bla

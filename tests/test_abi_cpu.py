@@ -1,0 +1,106 @@
+"""The C-ABI library loads, exports every declared entry point, and rejects bad
+arguments on the host before touching the GPU (CPU only: no compute calls)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2606_09862_gb300 import build, bla
+    build.build()
+    return bla.load()
+
+
+def declared_functions():
+    names = set()
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names |= set(re.findall(r"\b(bla_\w+)\s*\(", text))
+    return sorted(names)
+
+
+def test_exports_every_declared_symbol(lib):
+    names = declared_functions()
+    assert "bla_forward_chunked" in names and "bla_decode_step" in names and "bla_backward" in names
+    for n in names:
+        assert hasattr(lib, n), "missing export " + n
+
+
+def test_status_strings(lib):
+    assert lib.bla_status_string(0) == b"ok"
+    assert lib.bla_status_string(4) == b"device wait timed out"
+
+
+def _params(**kw):
+    from paper_2606_09862_gb300 import bla
+    base = dict(B=1, H=2, L=16, d_k=32, d_v=32, M=4, S=4, window=16.0, omega=0.0, chunk=0, scale=0.0,
+                dtype=bla.BLA_F32)
+    base.update(kw)
+    return bla.Params(**base)
+
+
+FAKE = ctypes.c_void_p(0x10000)      # aligned, never dereferenced: validation fails first
+
+
+@pytest.mark.parametrize("kw", [dict(B=0), dict(H=0), dict(L=-1), dict(d_k=0), dict(M=0), dict(S=0),
+                                dict(S=17), dict(window=0.0), dict(window=float("nan")), dict(dtype=7),
+                                dict(chunk=-3), dict(omega=float("inf"))])
+def test_invalid_params_rejected_on_host(lib, kw):
+    from paper_2606_09862_gb300 import bla
+    p = _params(**kw)
+    st = lib.bla_forward_chunked(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 30, None)
+    assert st == bla.BLA_ERR_INVALID
+    assert lib.bla_last_error_string() != b""
+    assert lib.bla_workspace_bytes(ctypes.byref(p), 0) == 0
+
+
+def test_null_and_misaligned_pointers_rejected(lib):
+    from paper_2606_09862_gb300 import bla
+    p = _params()
+    assert lib.bla_forward_chunked(None, FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 30, None) == \
+        bla.BLA_ERR_INVALID
+    assert lib.bla_forward_chunked(ctypes.byref(p), None, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 30, None) == \
+        bla.BLA_ERR_INVALID
+    bad = ctypes.c_void_p(0x10004)
+    assert lib.bla_forward_chunked(ctypes.byref(p), bad, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 30, None) == \
+        bla.BLA_ERR_INVALID
+    # workspace too small / misaligned
+    assert lib.bla_forward_chunked(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 8, None) == \
+        bla.BLA_ERR_INVALID
+    assert lib.bla_forward_chunked(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, None, None,
+                                   ctypes.c_void_p(0x10010), 1 << 30, None) == bla.BLA_ERR_INVALID
+
+
+def test_decode_argument_checks(lib):
+    from paper_2606_09862_gb300 import bla
+    p = _params()
+    assert lib.bla_decode_step(ctypes.byref(p), -1, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, None) == \
+        bla.BLA_ERR_INVALID
+    p2 = _params(d_k=48, d_v=48)
+    assert lib.bla_decode_step(ctypes.byref(p2), 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20, None) == \
+        bla.BLA_ERR_UNSUPPORTED
+
+
+def test_workspace_sizes_positive(lib):
+    from paper_2606_09862_gb300 import bla
+    p = _params()
+    assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_FORWARD) > 0
+    assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECODE) > 0
+
+
+def test_product_path_does_not_import_oracle():
+    """The CUDA binding and package never import the oracle."""
+    pkg = os.path.join(ROOT, "paper_2606_09862_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for fn in files:
+            if fn.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, fn)).read()
+                assert "import oracle" not in text and "from oracle" not in text, fn
+                assert "bla_oracle" not in text and "liborc" not in text, fn
