@@ -206,7 +206,8 @@ bla_status bla_device_error(void *stream) {
     if (code != 0) {
         e = cudaMemcpyToSymbol(g_dev_error, &zero, sizeof(int));
         if (e != cudaSuccess) return cuda_fail(e, "clear device error word");
-        return fail(BLA_ERR_TIMEOUT, "device wait gave up (code %d)", code);
+        return fail(BLA_ERR_TIMEOUT, "device wait gave up (code 0x%x: kind %d, kernel %d, barrier %d, parity %d, block %d)",
+                    code, code & 15, (code >> 4) & 15, (code >> 8) & 127, (code >> 15) & 1, (code >> 16) & 0xffff);
     }
     return BLA_OK;
 }

@@ -1,22 +1,1090 @@
-// fwd_bf16.cu -- bf16 tensor-core chunked forward (placeholder until the tcgen05 kernels land).
+// fwd_bf16.cu -- bf16 chunked forward on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
+//
+// Chunk algebra (the same exact rearrangement as the fp32 path, Eqs. (recurrence),
+// (compressed), (output)): for a chunk of C = 128 tokens starting at t0, with W the state
+// carried into the chunk (W_m = e^{i m w} Z_m(t0-1), interleaved rows 2m = Re, 2m+1 = Im):
+//   P  = tril(Q K^T)                                 [C x C]
+//   X  = P EB^T + Q W^T,  EB[2m][u] = cos(m w u), EB[2m+1][u] = -sin(m w u)
+//   Y  = e^{i m w t} X (per row t, per mode pair)    = q_t . Z_m(t0+t)
+//   s  = scale Y PHI^T,   PHI[j][2m] = c_m cos(m w D_j), PHI[j][2m+1] = c_m sin(m w D_j)
+//   p  = softmax over slots with t0+t >= D_j
+//   U  = p PHI;  A'  = rotation of U by -m w t  (real form of U_m e^{i m w t}, imaginary negated)
+//   G  = tril(A' EB),  O = G V + A' WV
+//   W <- e^{i m w C} (W + EB X_chunk)  for X in {K, V}
+//
+// The work runs as four kernels per call:
+//   k_prepass  per (head, segment): segment deltas  F_seg [K|V]  (one GEMM, K-dim = segment)
+//   k_scan     per head: states entering each segment, W_in(g+1) = e^{i m w Lseg} W_in(g) + delta(g)
+//   k_kpass    per (head, segment): carries the K state in TMEM, writes slot probabilities p and lse
+//   k_vpass    per (head, segment): carries the V state in TMEM, reads p, writes o
+// Every CTA runs 6 warps: warps 0-3 drain TMEM (thread = TMEM lane), warp 4 issues TMA loads,
+// warp 5 allocates TMEM and issues the MMAs.  All waits are bounded (tc::mbar_wait).
+#include <math.h>
+
 #include "fwd_bf16.cuh"
+#include "tc.cuh"
+#include "tmap.cuh"
 
 namespace bla {
 
+namespace {
+
+using bf16 = __nv_bfloat16;
+constexpr int kC = 128;          // tokens per chunk (MMA M)
+constexpr int kThreads = 192;
+constexpr int kEpiThreads = 128;
+
+// ------------------------------------------------------------------ geometry
+
+struct Geo {
+    int BH, L, D, M, R2, RH, NH, NB, S, SP, RP;
+    int nchunks, cps, G, Lseg;      // chunks per segment, segments per head, segment length (tokens)
+};
+
+Geo make_geo(const OpDims &d) {
+    Geo g;
+    g.BH = d.B * d.H; g.L = d.L; g.D = d.dk; g.M = d.M; g.R2 = d.R2;
+    g.RH = d.R2 < 128 ? d.R2 : 128;
+    g.NH = d.R2 / g.RH;
+    g.NB = d.R2 <= 128 ? 1 : d.R2 / 128;
+    g.RP = g.NB * 128;
+    g.S = d.S;
+    g.SP = d.S < 64 ? 64 : d.S;
+    g.nchunks = (d.L + kC - 1) / kC;
+    int want = (2 * 152 + g.BH / 2) / (g.BH > 0 ? g.BH : 1);
+    if (want < 1) want = 1;
+    if (want > g.nchunks) want = g.nchunks > 0 ? g.nchunks : 1;
+    g.cps = (g.nchunks + want - 1) / want;
+    if (g.cps < 1) g.cps = 1;
+    g.G = g.nchunks > 0 ? (g.nchunks + g.cps - 1) / g.cps : 1;
+    g.Lseg = g.cps * kC;
+    return g;
+}
+
+struct WsLayout {
+    size_t tables, eb, phi, fseg, deltas, win, pbuf, total;
+};
+
+WsLayout ws_layout(const OpDims &d, const Geo &g) {
+    WsLayout w;
+    size_t off = 0;
+    w.tables = off; off += tables_bytes(d, kC);
+    w.eb = off;     off += align_up(sizeof(bf16) * (size_t)g.RP * kC, 1024);
+    w.phi = off;    off += align_up(sizeof(bf16) * (size_t)g.SP * g.R2, 1024);
+    w.fseg = off;   off += g.G > 1 ? align_up(sizeof(bf16) * (size_t)g.RP * g.Lseg, 1024) : 0;
+    w.deltas = off; off += g.G > 1 ? align_up(sizeof(float) * (size_t)g.BH * g.G * 2 * g.RP * g.D, 1024) : 0;
+    w.win = off;    off += g.G > 1 ? align_up(sizeof(float) * (size_t)g.BH * g.G * 2 * g.RP * g.D, 1024) : 0;
+    w.pbuf = off;   off += align_up(sizeof(bf16) * (size_t)g.BH * (g.L > 0 ? g.L : 1) * g.SP, 1024);
+    w.total = off;
+    return w;
+}
+
+// ------------------------------------------------------------------ bf16 tables
+
+// EB [RP][C], PHI [SP][R2], FSEG [RP][Lseg] in bf16, from fp64 phases (rows beyond 2M and
+// slots beyond S are zero).
+__global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, double T, double w, bf16 *eb, bf16 *phi,
+                              bf16 *fseg) {
+    const int R2 = 2 * M;
+    const long long n_eb = (long long)RP * kC, n_phi = (long long)SP * R2;
+    const long long n_f = fseg ? (long long)RP * Lseg : 0;
+    const long long total = n_eb + n_phi + n_f;
+    const double n = 2.0 * M - 1.0;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        if (i < n_eb) {
+            int r = (int)(i / kC), u = (int)(i % kC), m = r >> 1;
+            double v = 0.0;
+            if (r < R2) {
+                double s, c;
+                sincos((double)m * w * (double)u, &s, &c);
+                v = (r & 1) ? -s : c;
+            }
+            eb[i] = __float2bfloat16_rn((float)v);
+        } else if (i < n_eb + n_phi) {
+            long long e = i - n_eb;
+            int j = (int)(e / R2), r = (int)(e % R2), m = r >> 1;
+            double v = 0.0;
+            if (j < S) {
+                double dj = rint((double)j * T / (double)S);
+                double cm = (m == 0) ? 1.0 / n : 2.0 / n;
+                double s, c;
+                sincos((double)m * w * dj, &s, &c);
+                v = cm * ((r & 1) ? s : c);
+            }
+            phi[e] = __float2bfloat16_rn((float)v);
+        } else {
+            long long e = i - n_eb - n_phi;
+            int r = (int)(e / Lseg), u = (int)(e % Lseg), m = r >> 1;
+            double v = 0.0;
+            if (r < R2) {
+                double s, c;
+                sincos((double)m * w * (double)(Lseg - u), &s, &c);
+                v = (r & 1) ? s : c;
+            }
+            fseg[e] = __float2bfloat16_rn((float)v);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ kernel arguments
+
+struct Args {
+    Geo g;
+    float scale;
+    double w;
+    const float *erel;   // [C+1][M][2] fp32 (cos, sin)(m w tau)
+    const int *delta;    // [S]
+    const float *deltas; // [BH][G][2][RP][D] segment deltas (prepass output)
+    float *win;          // [BH][G][2][RP][D] states entering each segment (or null if G == 1)
+    bf16 *pbuf;          // [BH][L][SP]
+    float *lse;          // [BH][L] or null
+    bf16 *o;             // [BH][L][D]
+    float *state_out;    // [BH][2][M][2][D] or null
+    float *deltas_out;   // prepass output (same buffer as deltas)
+    int *err;
+};
+
+// Bounded-wait bookkeeping shared by the roles of one CTA.
+struct Ctl {
+    volatile int abort;
+    int kernel;            // 1 prepass, 2 K pass, 3 V pass
+    uint64_t *bar0;        // first barrier of the CTA (for error reports)
+};
+
+// Bounded wait on `bar` for the phase of parity `phase` (flipped after the call).  On a
+// timeout the CTA's abort flag is raised and the error word records
+//   DEVERR_MBAR_TIMEOUT | kernel << 4 | barrier index << 8 | parity << 15 | block << 16.
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t &phase, Ctl *ctl, int *err) {
+    if (ctl->abort) return false;
+    bool ok = tc::mbar_wait(bar, phase);
+    if (!ok) {
+        ctl->abort = 1;
+        report_device_error(err, DEVERR_MBAR_TIMEOUT | (ctl->kernel << 4) |
+                                     ((int)(bar - ctl->bar0) << 8) | ((int)phase << 15) | ((int)blockIdx.x << 16));
+    }
+    phase ^= 1u;
+    return ok;
+}
+
+__device__ __forceinline__ uint32_t tmem_addr(uint32_t base, int lane_base, int col) {
+    return base + ((uint32_t)lane_base << 16) + (uint32_t)col;
+}
+
+// Store 32 fp32 values of one tile row as bf16 into a [rows][64]-blocked 128B-swizzled tile,
+// columns [col0, col0+32) (col0 a multiple of 32).
+__device__ __forceinline__ void st_row32_bf16(uint8_t *tile, int rows_per_block, int row, int col0, const float *v) {
+    uint8_t *blk = tile + (size_t)(col0 >> 6) * rows_per_block * 128;
+    const int c = col0 & 63;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 pk;
+        pk.x = tc::pack_bf16x2(v[q * 8 + 0], v[q * 8 + 1]);
+        pk.y = tc::pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]);
+        pk.z = tc::pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]);
+        pk.w = tc::pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]);
+        *reinterpret_cast<uint4 *>(blk + tc::sw128_offset(row, c + q * 8)) = pk;
+    }
+}
+
+// MMA helpers: one K-step of 16 on 128B-swizzled tiles.
+//   K-major tile: blocks of [rows][64] (block bytes = rows*128); step k -> block k/4, +32B*(k%4).
+__device__ __forceinline__ uint64_t kmaj_desc(const uint8_t *tile, int rows, int k) {
+    uint32_t a = tc::smem_u32(tile) + (uint32_t)((k >> 2) * rows * 128) + (uint32_t)((k & 3) * 32);
+    return tc::sdesc_sw128(a, 16, 1024);
+}
+//   MN-major tile: [K rows][64 MN] blocks, block bytes = krows*128 (LBO); step k -> +16 rows.
+__device__ __forceinline__ uint64_t mnmaj_desc(const uint8_t *tile, int krows, int k) {
+    uint32_t a = tc::smem_u32(tile) + (uint32_t)(k * 16 * 128);
+    return tc::sdesc_sw128(a, (uint32_t)krows * 128u, 1024);
+}
+
+// Rotate the state block held in TMEM (rows = lanes, interleaved cos/sin pairs) by
+// e^{i m w adv} and optionally write it back, also emitting the bf16 copy into a
+// [RH rows][64 d] blocked tile (rows >= RH skipped) and/or an fp32 copy to global.
+// Executed by the 128 epilogue threads; `row` is this thread's lane = local state row.
+__device__ void state_pass(uint32_t tbase, int col0, int D, int row, int mode_base, int RH, int R2row_limit,
+                           int R2, const float *erel, int M, int adv, bool rotate, bool write_back, uint8_t *wtile,
+                           float *gout) {
+    (void)R2;
+    const int lane_base = (row >> 5) << 5;
+    const int m = mode_base + (row >> 1);
+    float c = 1.f, s = 0.f;
+    if (rotate && m < M) {
+        c = erel[((size_t)adv * M + m) * 2];
+        s = erel[((size_t)adv * M + m) * 2 + 1];
+    }
+    const bool odd = row & 1;
+    for (int g = 0; g < D; g += 32) {
+        float v[32];
+        tc::tmem_ld32(tmem_addr(tbase, lane_base, col0 + g), v);
+        if (rotate) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                float partner = __shfl_xor_sync(0xffffffffu, v[i], 1);
+                // even row: Re' = c Re - s Im ; odd row: Im' = s Re + c Im
+                v[i] = odd ? fmaf(s, partner, c * v[i]) : fmaf(-s, partner, c * v[i]);
+            }
+            if (write_back) tc::tmem_st32(tmem_addr(tbase, lane_base, col0 + g), v);
+        }
+        if (wtile && row < RH) st_row32_bf16(wtile, RH, row, g, v);
+        if (gout && row < R2row_limit) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4)
+                *reinterpret_cast<float4 *>(gout + g + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+        }
+    }
+}
+
+// Load 128 rows x D fp32 (global, row stride D) into a TMEM state block; rows at or beyond
+// `live_rows` (padding beyond 2M) and a NULL source give zeros.
+__device__ void state_init(uint32_t tbase, int col0, int D, int row, const float *src, int live_rows) {
+    const int lane_base = (row >> 5) << 5;
+    for (int g = 0; g < D; g += 32) {
+        float v[32];
+        if (src && row < live_rows) {
+#pragma unroll
+            for (int i = 0; i < 32; i += 4) {
+                float4 t = *reinterpret_cast<const float4 *>(src + (size_t)row * D + g + i);
+                v[i] = t.x; v[i + 1] = t.y; v[i + 2] = t.z; v[i + 3] = t.w;
+            }
+        } else {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) v[i] = 0.f;
+        }
+        tc::tmem_st32(tmem_addr(tbase, lane_base, col0 + g), v);
+    }
+}
+
+// ================================================================== prepass
+//
+// delta_seg[K|V][RP][D] = F_seg [RP x Lseg] . X_seg [Lseg x D] for every full segment but the last.
+// Pipelined over half-chunks of 64 tokens with 3 smem stages.
+
+constexpr int kPreStages = 3;
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_prepass(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+              const __grid_constant__ CUtensorMap tm_f, Args a) {
+    const Geo &g = a.g;
+    const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
+    if (seg >= g.G - 1) return;   // the last segment's delta is never used
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const int D = g.D, NB = g.NB;
+    const size_t f_bytes = (size_t)NB * 128 * 64 * 2, x_bytes = (size_t)64 * D * 2;
+    const size_t stage_bytes = f_bytes + 2 * x_bytes;
+    uint8_t *stage0 = sm;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(sm + kPreStages * stage_bytes);
+    uint64_t *full = bars, *empty = bars + kPreStages, *done = bars + 2 * kPreStages;
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bars + 2 * kPreStages + 1);
+    Ctl *ctl = reinterpret_cast<Ctl *>(bars + 2 * kPreStages + 2);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t ncols = (uint32_t)(2 * NB * D) <= 128 ? 128u : (uint32_t)(2 * NB * D) <= 256 ? 256u : 512u;
+    // (the host requests shared memory so that CTAs whose column counts would not fit together
+    //  are never co-resident)
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < kPreStages; ++i) { tc::mbar_init(&full[i], 1); tc::mbar_init(&empty[i], 1); }
+        tc::mbar_init(done, 1);
+        ctl->abort = 0;
+        ctl->kernel = 1;
+        ctl->bar0 = bars;
+        tc::fence_barrier_init();
+    }
+    if (warp == 5) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tb = *tslot;
+    const int steps = g.cps * 2;          // half-chunks in the segment
+    const int t_seg = seg * g.Lseg;
+
+    if (warp == 4 && lane == 0) {
+        uint32_t ph[kPreStages] = {0, 0, 0};
+        for (int it = 0; it < steps; ++it) {
+            const int st = it % kPreStages;
+            if (it >= kPreStages && !wait_bar(&empty[st], ph[st], ctl, a.err)) break;
+            uint8_t *base = stage0 + st * stage_bytes;
+            tc::mbar_arrive_expect_tx(&full[st], (uint32_t)stage_bytes);
+            for (int b = 0; b < NB; ++b) tc::tma_load_2d(base + b * 128 * 128, &tm_f, &full[st], it * 64, b * 128);
+            for (int db = 0; db < D / 64; ++db) {
+                tc::tma_load_3d(base + f_bytes + db * 64 * 128, &tm_k, &full[st], db * 64, t_seg + it * 64, bh);
+                tc::tma_load_3d(base + f_bytes + x_bytes + db * 64 * 128, &tm_v, &full[st], db * 64, t_seg + it * 64,
+                                bh);
+            }
+        }
+    } else if (warp == 5 && lane == 0) {
+        uint32_t ph[kPreStages] = {0, 0, 0};
+        const uint32_t idesc = tc::idesc_bf16(128, D, false, true);
+        for (int it = 0; it < steps; ++it) {
+            const int st = it % kPreStages;
+            if (!wait_bar(&full[st], ph[st], ctl, a.err)) break;
+            tc::tc_fence_after();
+            uint8_t *base = stage0 + st * stage_bytes;
+            for (int x = 0; x < 2; ++x)
+                for (int b = 0; b < NB; ++b)
+                    for (int k = 0; k < 4; ++k) {
+                        uint64_t ad = kmaj_desc(base + b * 128 * 128, 128, k);
+                        uint64_t bd = mnmaj_desc(base + f_bytes + x * x_bytes, 64, k);
+                        tc::mma_bf16(tb + (uint32_t)((x * NB + b) * D), ad, bd, idesc, (it > 0 || k > 0) ? 1u : 0u);
+                    }
+            tc::mma_commit(&empty[st]);
+        }
+        tc::mma_commit(done);
+    } else if (warp < 4) {
+        uint32_t ph = 0;
+        bool ok = wait_bar(done, ph, ctl, a.err);
+        tc::tc_fence_after();
+        if (ok) {
+            const int row = threadIdx.x;
+            for (int x = 0; x < 2; ++x)
+                for (int b = 0; b < NB; ++b) {
+                    float *dst = a.deltas_out + ((((size_t)bh * g.G + seg) * 2 + x) * g.RP + b * 128 + row) * D;
+                    state_pass(tb, (x * NB + b) * D, D, row, 0, 0, 1 << 30, g.R2, a.erel, g.M, 0, false, false, nullptr,
+                               dst);
+                }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 5) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tb, ncols);
+    }
+}
+
+// ================================================================== segment scan
+// W_in(0) = 0; W_in(g+1) = e^{i m w Lseg} W_in(g) + delta(g).  One thread per (head, K|V, mode, d).
+__global__ void k_scan(Args a) {
+    const Geo &g = a.g;
+    const long long total = (long long)g.BH * 2 * g.M * g.D;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int e = (int)(i % g.D);
+        long long r = i / g.D;
+        const int m = (int)(r % g.M);
+        r /= g.M;
+        const int x = (int)(r % 2);
+        const int bh = (int)(r / 2);
+        double sn, cs;
+        sincos((double)m * a.w * (double)g.Lseg, &sn, &cs);
+        const float c = (float)cs, s = (float)sn;
+        float re = 0.f, im = 0.f;
+        for (int seg = 0; seg < g.G; ++seg) {
+            const size_t base = (((size_t)bh * g.G + seg) * 2 + x) * g.RP;
+            a.win[(base + 2 * m) * g.D + e] = re;
+            a.win[(base + 2 * m + 1) * g.D + e] = im;
+            if (seg + 1 < g.G) {
+                const float dre = a.deltas[(base + 2 * m) * g.D + e], dim = a.deltas[(base + 2 * m + 1) * g.D + e];
+                const float nre = c * re - s * im + dre;
+                const float nim = s * re + c * im + dim;
+                re = nre;
+                im = nim;
+            }
+        }
+    }
+}
+
+// ================================================================== K pass
+
+struct KLayout {
+    size_t q, k, p, w, y, eb, phi, bars, total;
+};
+
+__host__ __device__ inline KLayout k_layout(const Geo &g) {
+    KLayout l;
+    size_t off = 0;
+    l.q = off;   off += (size_t)kC * g.D * 2;
+    l.k = off;   off += (size_t)kC * g.D * 2;
+    l.p = off;   off += (size_t)kC * kC * 2;
+    l.w = off;   off += (size_t)g.RH * g.D * 2;
+    l.y = off;   off += (size_t)kC * g.RH * 2;
+    l.eb = off;  off += (size_t)128 * kC * 2;
+    l.phi = off; off += (size_t)g.SP * g.RH * 2;
+    l.bars = off; off += 1024;
+    l.total = off + 1024;   // slack for 1024-byte alignment of the dynamic smem base
+    return l;
+}
+
+// One barrier per use and per mode half: a barrier is never committed twice without the
+// waiter's hand-back in between, so a parity wait can never fall two phases behind.
+enum KBar {
+    KB_QK_FULL, KB_QK_FREE, KB_EB_FULL, KB_EB_FREE, KB_PHI_FULL, KB_PHI_FREE,
+    KB_ACC_FULL_A, KB_ACC_FULL_B, KB_ACC_FREE_A, KB_ACC_FREE_B,
+    KB_P_READY, KB_W_READY, KB_W_FREE, KB_STATE_DONE, KB_STATE_DONE1, KB_Y_READY, KB_Y_FREE, KB_EXIT, KB_COUNT
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_kpass(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+            const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi, Args a) {
+    const Geo &g = a.g;
+    const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
+    const int c_begin = seg * g.cps, c_end = min(g.nchunks, c_begin + g.cps);
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const KLayout lay = k_layout(g);
+    uint8_t *sQ = sm + lay.q, *sK = sm + lay.k, *sP = sm + lay.p, *sW = sm + lay.w, *sY = sm + lay.y;
+    uint8_t *sEB = sm + lay.eb, *sPHI = sm + lay.phi;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + lay.bars);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + KB_COUNT);
+    Ctl *ctl = reinterpret_cast<Ctl *>(bar + KB_COUNT + 1);
+    int *sdelta = reinterpret_cast<int *>(bar + KB_COUNT + 4);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int D = g.D, RH = g.RH, NH = g.NH, S = g.S, SP = g.SP;
+    // TMEM columns: [0, NB*D) state; accA at NB*D (128 cols); accB after it (RH cols).
+    const int colA = g.NB * D, colB = colA + 128;
+    const uint32_t ncols = (uint32_t)(colB + RH) <= 256 ? 256u : 512u;   // host: pow2_cols(NB*D + 128 + RH)
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < KB_COUNT; ++i) {
+            const bool epi = i == KB_P_READY || i == KB_W_READY || i == KB_Y_READY || i == KB_ACC_FREE_A ||
+                             i == KB_ACC_FREE_B;
+            tc::mbar_init(&bar[i], epi ? kEpiThreads : 1);
+        }
+        ctl->abort = 0;
+        ctl->kernel = 2;
+        ctl->bar0 = bar;
+        tc::fence_barrier_init();
+    }
+    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
+    if (warp == 5) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tb = *tslot;
+
+    if (warp == 4) {
+        if (lane == 0) {
+            tc::tma_prefetch_desc(&tm_q); tc::tma_prefetch_desc(&tm_k);
+            tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
+            uint32_t ph_qk = 0, ph_eb = 0, ph_phi = 0;
+            bool first_eb = true, first_phi = true;
+            for (int c = c_begin; c < c_end && !ctl->abort; ++c) {
+                if (c > c_begin && !wait_bar(&bar[KB_QK_FREE], ph_qk, ctl, a.err)) break;
+                tc::mbar_arrive_expect_tx(&bar[KB_QK_FULL], (uint32_t)(2 * kC * D * 2));
+                for (int db = 0; db < D / 64; ++db) {
+                    tc::tma_load_3d(sQ + db * kC * 128, &tm_q, &bar[KB_QK_FULL], db * 64, c * kC, bh);
+                    tc::tma_load_3d(sK + db * kC * 128, &tm_k, &bar[KB_QK_FULL], db * 64, c * kC, bh);
+                }
+                for (int h = 0; h < NH; ++h) {
+                    if (!first_eb && !wait_bar(&bar[KB_EB_FREE], ph_eb, ctl, a.err)) break;
+                    first_eb = false;
+                    tc::mbar_arrive_expect_tx(&bar[KB_EB_FULL], (uint32_t)(128 * kC * 2));
+                    for (int kb = 0; kb < 2; ++kb)
+                        tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[KB_EB_FULL], kb * 64, h * 128);
+                    if (!first_phi && !wait_bar(&bar[KB_PHI_FREE], ph_phi, ctl, a.err)) break;
+                    first_phi = false;
+                    tc::mbar_arrive_expect_tx(&bar[KB_PHI_FULL], (uint32_t)(SP * RH * 2));
+                    for (int kb = 0; kb < RH / 64; ++kb)
+                        tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[KB_PHI_FULL], h * RH + kb * 64, 0);
+                }
+            }
+        }
+    } else if (warp == 5) {
+        if (lane == 0) {
+            uint32_t ph_qk = 0, ph_eb = 0, ph_phi = 0, ph_freeA = 0, ph_freeB = 0, ph_p = 0, ph_w = 0, ph_y = 0;
+            const uint32_t id_P = tc::idesc_bf16(128, kC, false, false);
+            const uint32_t id_X = tc::idesc_bf16(128, RH, false, false);
+            const uint32_t id_S = tc::idesc_bf16(128, S, false, false);
+            const uint32_t id_U = tc::idesc_bf16(128, D, false, true);
+            // Each accumulator region is handed back by the epilogue after every drain; every use
+            // but the very first waits for that hand-back.
+            bool usedA = false, usedB = false;
+            auto acquire = [&](bool inB) -> bool {
+                bool &used = inB ? usedB : usedA;
+                if (used && !wait_bar(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A], inB ? ph_freeB : ph_freeA, ctl, a.err))
+                    return false;
+                used = true;
+                return true;
+            };
+            for (int c = c_begin; c < c_end; ++c) {
+                if (!wait_bar(&bar[KB_QK_FULL], ph_qk, ctl, a.err)) break;
+                if (!acquire(false)) break;
+                tc::tc_fence_after();
+                for (int k = 0; k < D / 16; ++k)
+                    tc::mma_bf16(tb + colA, kmaj_desc(sQ, kC, k), kmaj_desc(sK, kC, k), id_P, k > 0);
+                tc::mma_commit(&bar[KB_ACC_FULL_A]);
+                bool bad = false;
+                for (int h = 0; h < NH && !bad; ++h) {
+                    // X_h = Q W_h^T + P EB_h^T  -> acc (h even: B, odd: A)
+                    const bool inB = (h & 1) == 0;
+                    if (!wait_bar(&bar[KB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
+                    if (!wait_bar(&bar[KB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
+                    if (h == 0 && !wait_bar(&bar[KB_P_READY], ph_p, ctl, a.err)) { bad = true; break; }
+                    if (!acquire(inB)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    const uint32_t dX = tb + (inB ? colB : colA);
+                    for (int k = 0; k < D / 16; ++k)
+                        tc::mma_bf16(dX, kmaj_desc(sQ, kC, k), kmaj_desc(sW, RH, k), id_X, k > 0);
+                    for (int k = 0; k < kC / 16; ++k)
+                        tc::mma_bf16(dX, kmaj_desc(sP, kC, k), kmaj_desc(sEB, 128, k), id_X, 1);
+                    tc::mma_commit(&bar[inB ? KB_ACC_FULL_B : KB_ACC_FULL_A]);
+                    tc::mma_commit(&bar[KB_W_FREE]);
+                    // state block h += EB_h (A, 128 rows) . K_chunk (B, MN-major, N = D)
+                    for (int k = 0; k < kC / 16; ++k)
+                        tc::mma_bf16(tb + h * D, kmaj_desc(sEB, 128, k), mnmaj_desc(sK, kC, k), id_U, 1);
+                    tc::mma_commit(&bar[KB_STATE_DONE + h]);
+                    tc::mma_commit(&bar[KB_EB_FREE]);
+                    if (h == NH - 1) tc::mma_commit(&bar[KB_QK_FREE]);
+                }
+                if (bad) break;
+                // s = sum_h Y_h PHI_h^T -> acc (NH == 2: B after X_0 drained; NH == 1: A after P drained)
+                const bool sInB = NH == 2;
+                if (!acquire(sInB)) break;
+                for (int h = 0; h < NH && !bad; ++h) {
+                    if (!wait_bar(&bar[KB_PHI_FULL], ph_phi, ctl, a.err)) { bad = true; break; }
+                    if (!wait_bar(&bar[KB_Y_READY], ph_y, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    const uint32_t dS = tb + (sInB ? colB : colA);
+                    for (int k = 0; k < RH / 16; ++k)
+                        tc::mma_bf16(dS, kmaj_desc(sY, kC, k), kmaj_desc(sPHI, SP, k), id_S, (h > 0 || k > 0) ? 1u : 0u);
+                    tc::mma_commit(&bar[KB_Y_FREE]);
+                    tc::mma_commit(&bar[KB_PHI_FREE]);
+                }
+                if (bad) break;
+                tc::mma_commit(&bar[sInB ? KB_ACC_FULL_B : KB_ACC_FULL_A]);
+            }
+            tc::mma_commit(&bar[KB_EXIT]);
+            uint32_t ph_exit = 0;
+            tc::mbar_wait(&bar[KB_EXIT], ph_exit);
+        }
+    } else {
+        // ---------------- epilogue warps 0-3: thread = TMEM lane = token row / state row
+        const int row = threadIdx.x, lane_base = warp * 32;
+        uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0;
+        uint32_t ph_state[2] = {0, 0};
+        const int M = g.M;
+        const float *erel = a.erel;
+        // state entering the segment
+        for (int b = 0; b < g.NB; ++b) {
+            const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
+            state_init(tb, b * D, D, row, src, g.R2 - b * 128);
+        }
+        bool bad = false;
+        for (int c = c_begin; c < c_end && !bad; ++c) {
+            const int t0 = c * kC;
+            const int n = min(kC, g.L - t0);
+            const bool rot = c > c_begin;
+            for (int h = 0; h < NH && !bad; ++h) {
+                // W_h extraction: state block h (holding W + EB X of the previous chunk) is rotated by
+                // e^{i m w C} into the state carried into this chunk, written back, and copied to bf16.
+                if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+                tc::tc_fence_after();
+                state_pass(tb, h * D, D, row, h * 64, RH, 0, g.R2, erel, M, kC, rot, rot, sW, nullptr);
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bar[KB_W_READY]);
+                if (h == 0) {
+                    // P drain: mask u <= t, bf16 -> sP
+                    if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    for (int g0 = 0; g0 < kC; g0 += 32) {
+                        float v[32];
+                        tc::tmem_ld32(tmem_addr(tb, lane_base, colA + g0), v);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (g0 + i > row) v[i] = 0.f;
+                        st_row32_bf16(sP, kC, row, g0, v);
+                    }
+                    tc::fence_proxy_async_smem();
+                    tc::tc_fence_before();
+                    tc::mbar_arrive(&bar[KB_P_READY]);
+                    tc::mbar_arrive(&bar[KB_ACC_FREE_A]);
+                }
+                // drain X_h -> Y_h (rotate by e^{i m w t}, t = row)
+                const bool inB = (h & 1) == 0;
+                if (!wait_bar(&bar[inB ? KB_ACC_FULL_B : KB_ACC_FULL_A], inB ? ph_fullB : ph_fullA, ctl, a.err)) {
+                    bad = true;
+                    break;
+                }
+                // X_h complete => W tile free for the next half
+                if (!wait_bar(&bar[KB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
+                if (h > 0 && !wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
+                tc::tc_fence_after();
+                const float c1 = erel[((size_t)row * M + 1) * 2], s1 = erel[((size_t)row * M + 1) * 2 + 1];
+                for (int g0 = 0; g0 < RH; g0 += 32) {
+                    float v[32];
+                    tc::tmem_ld32(tmem_addr(tb, lane_base, (inB ? colB : colA) + g0), v);
+                    const int m0 = h * (RH / 2) + g0 / 2;
+                    float cc = erel[((size_t)row * M + m0) * 2], ss = erel[((size_t)row * M + m0) * 2 + 1];
+#pragma unroll
+                    for (int i = 0; i < 32; i += 2) {
+                        const float xr = v[i], xi = v[i + 1];
+                        v[i] = cc * xr - ss * xi;
+                        v[i + 1] = ss * xr + cc * xi;
+                        const float nc = cc * c1 - ss * s1, ns = ss * c1 + cc * s1;
+                        cc = nc;
+                        ss = ns;
+                    }
+                    st_row32_bf16(sY, kC, row, g0, v);
+                }
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bar[KB_Y_READY]);
+                tc::mbar_arrive(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
+            }
+            if (bad) break;
+            // softmax over slots
+            const bool sInB = NH == 2;
+            if (!wait_bar(&bar[sInB ? KB_ACC_FULL_B : KB_ACC_FULL_A], sInB ? ph_fullB : ph_fullA, ctl, a.err)) {
+                bad = true;
+                break;
+            }
+            if (!wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
+            tc::tc_fence_after();
+            const int cs = sInB ? colB : colA;
+            const int t = t0 + row;
+            float mx = -INFINITY;
+            for (int g0 = 0; g0 < S; g0 += 32) {
+                float v[32];
+                tc::tmem_ld32(tmem_addr(tb, lane_base, cs + g0), v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (g0 + i < S && t >= sdelta[g0 + i]) mx = fmaxf(mx, v[i] * a.scale);
+            }
+            float sum = 0.f;
+            for (int g0 = 0; g0 < S; g0 += 32) {
+                float v[32];
+                tc::tmem_ld32(tmem_addr(tb, lane_base, cs + g0), v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (g0 + i < S && t >= sdelta[g0 + i]) sum += __expf(v[i] * a.scale - mx);
+            }
+            const float inv = 1.f / sum;
+            bf16 *prow = a.pbuf + ((size_t)bh * g.L + t) * SP;
+            for (int g0 = 0; g0 < SP; g0 += 32) {
+                float v[32];
+                if (g0 < S) tc::tmem_ld32(tmem_addr(tb, lane_base, cs + g0), v);
+                uint32_t pk[16];
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                    float p0 = (g0 < S && g0 + i < S && t >= sdelta[g0 + i]) ? __expf(v[i] * a.scale - mx) * inv : 0.f;
+                    float p1 = (g0 < S && g0 + i + 1 < S && t >= sdelta[g0 + i + 1])
+                                   ? __expf(v[i + 1] * a.scale - mx) * inv
+                                   : 0.f;
+                    pk[i / 2] = tc::pack_bf16x2(p0, p1);
+                }
+                if (row < n) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        *reinterpret_cast<uint4 *>(prow + g0 + q * 8) =
+                            make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
+                }
+            }
+            if (row < n && a.lse) a.lse[(size_t)bh * g.L + t] = mx + logf(sum);
+            tc::tc_fence_before();
+            tc::mbar_arrive(&bar[sInB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
+        }
+        // final K state (lag frame at t = L-1) after the last chunk of the last segment
+        if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
+            for (int h = 0; h < NH; ++h)
+                if (!wait_bar(&bar[KB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+            if (!bad) {
+                tc::tc_fence_after();
+                const int n_last = g.L - (c_end - 1) * kC;
+                for (int b = 0; b < g.NB; ++b) {
+                    const int r = b * 128 + row;
+                    float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + r) * D : nullptr;
+                    state_pass(tb, b * D, D, row, b * 64, 0, g.R2 - b * 128, g.R2, erel, M, n_last - 1, true, false,
+                               nullptr, dst);
+                }
+            }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 5) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tb, ncols);
+    }
+}
+
+// ================================================================== V pass
+
+struct VLayout {
+    size_t pg, v, a2, w, phi, eb, bars, total;
+};
+
+__host__ __device__ inline VLayout v_layout(const Geo &g) {
+    VLayout l;
+    size_t off = 0;
+    const size_t pbytes = (size_t)kC * g.SP * 2, gbytes = (size_t)kC * kC * 2;
+    l.pg = off;  off += pbytes > gbytes ? pbytes : gbytes;
+    l.v = off;   off += (size_t)kC * g.D * 2;
+    l.a2 = off;  off += (size_t)g.NH * kC * g.RH * 2;
+    l.w = off;   off += (size_t)g.RH * g.D * 2;
+    l.phi = off; off += (size_t)g.SP * g.RH * 2;
+    l.eb = off;  off += (size_t)128 * kC * 2;
+    l.bars = off; off += 1024;
+    l.total = off + 1024;
+    return l;
+}
+
+enum VBar {
+    VB_PV_FULL, VB_PV_FREE, VB_EB_FULL, VB_EB_FREE, VB_PHI_FULL, VB_PHI_FREE,
+    VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_G_READY, VB_W_READY, VB_W_FREE,
+    VB_STATE_DONE, VB_STATE_DONE1, VB_O_FULL, VB_EXIT, VB_COUNT
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    k_vpass(const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_v,
+            const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi, Args a) {
+    const Geo &g = a.g;
+    const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
+    const int c_begin = seg * g.cps, c_end = min(g.nchunks, c_begin + g.cps);
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const VLayout lay = v_layout(g);
+    uint8_t *sPG = sm + lay.pg, *sV = sm + lay.v, *sA = sm + lay.a2, *sW = sm + lay.w;
+    uint8_t *sPHI = sm + lay.phi, *sEB = sm + lay.eb;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + lay.bars);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + VB_COUNT);
+    Ctl *ctl = reinterpret_cast<Ctl *>(bar + VB_COUNT + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int D = g.D, RH = g.RH, NH = g.NH, SP = g.SP;
+    const size_t a_tile = (size_t)kC * RH * 2;
+    // TMEM: [0, NB*D) state; colU (128 cols: U_h, then O); colG (128 cols).
+    const int colU = g.NB * D, colG = colU + 128;
+    const uint32_t ncols = (uint32_t)(colG + 128) <= 256 ? 256u : 512u;  // host: pow2_cols(NB*D + 256)
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < VB_COUNT; ++i) {
+            const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_G_READY || i == VB_W_READY;
+            tc::mbar_init(&bar[i], epi ? kEpiThreads : 1);
+        }
+        ctl->abort = 0;
+        ctl->kernel = 3;
+        ctl->bar0 = bar;
+        tc::fence_barrier_init();
+    }
+    if (warp == 5) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tb = *tslot;
+
+    if (warp == 4) {
+        if (lane == 0) {
+            tc::tma_prefetch_desc(&tm_p); tc::tma_prefetch_desc(&tm_v);
+            tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
+            uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0;
+            bool first_eb = true, first_phi = true;
+            bool bad = false;
+            for (int c = c_begin; c < c_end && !bad; ++c) {
+                if (c > c_begin && !wait_bar(&bar[VB_PV_FREE], ph_pv, ctl, a.err)) break;
+                tc::mbar_arrive_expect_tx(&bar[VB_PV_FULL], (uint32_t)(kC * SP * 2 + kC * D * 2));
+                for (int kb = 0; kb < SP / 64; ++kb)
+                    tc::tma_load_3d(sPG + kb * kC * 128, &tm_p, &bar[VB_PV_FULL], kb * 64, c * kC, bh);
+                for (int db = 0; db < D / 64; ++db)
+                    tc::tma_load_3d(sV + db * kC * 128, &tm_v, &bar[VB_PV_FULL], db * 64, c * kC, bh);
+                // phase 1: PHI_h and EB_h per half; phase 3: EB_h again per half
+                for (int rep = 0; rep < 2 && !bad; ++rep)
+                    for (int h = 0; h < NH; ++h) {
+                        if (rep == 0) {
+                            if (!first_phi && !wait_bar(&bar[VB_PHI_FREE], ph_phi, ctl, a.err)) { bad = true; break; }
+                            first_phi = false;
+                            tc::mbar_arrive_expect_tx(&bar[VB_PHI_FULL], (uint32_t)(SP * RH * 2));
+                            for (int kb = 0; kb < RH / 64; ++kb)
+                                tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PHI_FULL], h * RH + kb * 64, 0);
+                        }
+                        if (!first_eb && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) { bad = true; break; }
+                        first_eb = false;
+                        tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
+                        for (int kb = 0; kb < 2; ++kb)
+                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, h * 128);
+                    }
+            }
+        }
+    } else if (warp == 5) {
+        if (lane == 0) {
+            uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0, ph_w = 0;
+            const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
+            const uint32_t id_G = tc::idesc_bf16(128, kC, false, true);
+            const uint32_t id_O = tc::idesc_bf16(128, D, false, true);
+            bool firstU = true, firstG = true;
+            bool bad = false;
+            for (int c = c_begin; c < c_end && !bad; ++c) {
+                if (!wait_bar(&bar[VB_PV_FULL], ph_pv, ctl, a.err)) break;
+                // phase 1
+                for (int h = 0; h < NH; ++h) {
+                    if (!wait_bar(&bar[VB_PHI_FULL], ph_phi, ctl, a.err)) { bad = true; break; }
+                    if (!(firstU && h == 0) && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    for (int k = 0; k < SP / 16; ++k)
+                        tc::mma_bf16(tb + colU, kmaj_desc(sPG, kC, k), mnmaj_desc(sPHI, SP, k), id_U, k > 0);
+                    tc::mma_commit(&bar[VB_U_FULL]);
+                    tc::mma_commit(&bar[VB_PHI_FREE]);
+                    if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
+                    if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) { bad = true; break; }
+                    if (h == 0 && !firstG && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    for (int k = 0; k < RH / 16; ++k)
+                        tc::mma_bf16(tb + colG, kmaj_desc(sA + h * a_tile, kC, k), mnmaj_desc(sEB, 128, k), id_G,
+                                     (h > 0 || k > 0) ? 1u : 0u);
+                    tc::mma_commit(&bar[VB_EB_FREE]);
+                }
+                firstU = false;
+                firstG = false;
+                if (bad) break;
+                tc::mma_commit(&bar[VB_G_FULL]);
+                // phase 2: O = G V (G written over p by the epilogue)
+                if (!wait_bar(&bar[VB_G_READY], ph_gready, ctl, a.err)) break;
+                if (!wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
+                tc::tc_fence_after();
+                for (int k = 0; k < kC / 16; ++k)
+                    tc::mma_bf16(tb + colU, kmaj_desc(sPG, kC, k), mnmaj_desc(sV, kC, k), id_O, k > 0);
+                // phase 3: O += A'_h W_h ; state_h += EB_h V
+                for (int h = 0; h < NH; ++h) {
+                    if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
+                    if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    for (int k = 0; k < RH / 16; ++k)
+                        tc::mma_bf16(tb + colU, kmaj_desc(sA + h * a_tile, kC, k), mnmaj_desc(sW, RH, k), id_O, 1);
+                    tc::mma_commit(&bar[VB_W_FREE]);
+                    for (int k = 0; k < kC / 16; ++k)
+                        tc::mma_bf16(tb + h * D, kmaj_desc(sEB, 128, k), mnmaj_desc(sV, kC, k), id_O, 1);
+                    tc::mma_commit(&bar[VB_STATE_DONE + h]);
+                    tc::mma_commit(&bar[VB_EB_FREE]);
+                }
+                if (bad) break;
+                tc::mma_commit(&bar[VB_O_FULL]);
+                tc::mma_commit(&bar[VB_PV_FREE]);
+            }
+            tc::mma_commit(&bar[VB_EXIT]);
+            uint32_t ph_exit = 0;
+            tc::mbar_wait(&bar[VB_EXIT], ph_exit);
+        }
+    } else {
+        const int row = threadIdx.x, lane_base = warp * 32;
+        const int M = g.M;
+        const float *erel = a.erel;
+        uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0;
+        uint32_t ph_state[2] = {0, 0};
+        for (int b = 0; b < g.NB; ++b) {
+            const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
+            state_init(tb, b * D, D, row, src, g.R2 - b * 128);
+        }
+        bool bad = false;
+        for (int c = c_begin; c < c_end && !bad; ++c) {
+            const int t0 = c * kC;
+            const int n = min(kC, g.L - t0);
+            const bool rot = c > c_begin;
+            // phase 1: U_h -> A'_h (rotation by -m w t of (sum_j p A, sum_j p B))
+            for (int h = 0; h < NH; ++h) {
+                if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
+                tc::tc_fence_after();
+                for (int g0 = 0; g0 < RH; g0 += 32) {
+                    float v[32];
+                    tc::tmem_ld32(tmem_addr(tb, lane_base, colU + g0), v);
+                    const int m0 = h * (RH / 2) + g0 / 2;
+                    const float c1 = erel[((size_t)row * M + 1) * 2], s1 = erel[((size_t)row * M + 1) * 2 + 1];
+                    float cc = erel[((size_t)row * M + m0) * 2], ss = erel[((size_t)row * M + m0) * 2 + 1];
+#pragma unroll
+                    for (int i = 0; i < 32; i += 2) {
+                        const float uc = v[i], us = v[i + 1];
+                        v[i] = cc * uc + ss * us;
+                        v[i + 1] = cc * us - ss * uc;
+                        const float nc = cc * c1 - ss * s1, ns = ss * c1 + cc * s1;
+                        cc = nc;
+                        ss = ns;
+                    }
+                    st_row32_bf16(sA + h * a_tile, kC, row, g0, v);
+                }
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bar[VB_A_READY]);
+                tc::mbar_arrive(&bar[VB_U_FREE]);
+            }
+            if (bad) break;
+            // phase 2: G drain -> mask -> bf16 over p's tile
+            if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
+            tc::tc_fence_after();
+            for (int g0 = 0; g0 < kC; g0 += 32) {
+                float v[32];
+                tc::tmem_ld32(tmem_addr(tb, lane_base, colG + g0), v);
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (g0 + i > row) v[i] = 0.f;
+                st_row32_bf16(sPG, kC, row, g0, v);
+            }
+            tc::fence_proxy_async_smem();
+            tc::tc_fence_before();
+            tc::mbar_arrive(&bar[VB_G_READY]);
+            tc::mbar_arrive(&bar[VB_G_FREE]);
+            // phase 3: W_h extraction (state read before this chunk's V update)
+            for (int h = 0; h < NH; ++h) {
+                if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
+                if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+                tc::tc_fence_after();
+                state_pass(tb, h * D, D, row, h * 64, RH, 0, g.R2, erel, M, kC, rot, rot, sW, nullptr);
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bar[VB_W_READY]);
+            }
+            if (bad) break;
+            if (!wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) break;
+            // phase 4: O drain -> global
+            if (!wait_bar(&bar[VB_O_FULL], ph_o, ctl, a.err)) break;
+            tc::tc_fence_after();
+            bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D;
+            for (int g0 = 0; g0 < D; g0 += 32) {
+                float v[32];
+                tc::tmem_ld32(tmem_addr(tb, lane_base, colU + g0), v);
+                if (row < n) {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        uint4 pk = make_uint4(tc::pack_bf16x2(v[q * 8], v[q * 8 + 1]), tc::pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]),
+                                              tc::pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]),
+                                              tc::pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]));
+                        *reinterpret_cast<uint4 *>(orow + g0 + q * 8) = pk;
+                    }
+                }
+            }
+            tc::tc_fence_before();
+            tc::mbar_arrive(&bar[VB_U_FREE]);
+        }
+        if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
+            for (int h = 0; h < NH; ++h)
+                if (!wait_bar(&bar[VB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+            if (!bad) {
+                tc::tc_fence_after();
+                const int n_last = g.L - (c_end - 1) * kC;
+                for (int b = 0; b < g.NB; ++b) {
+                    const int r = b * 128 + row;
+                    float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + g.R2 + r) * D : nullptr;
+                    state_pass(tb, b * D, D, row, b * 64, 0, g.R2 - b * 128, g.R2, erel, M, n_last - 1, true, false,
+                               nullptr, dst);
+                }
+            }
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 5) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tb, ncols);
+    }
+}
+
+}  // namespace
+
+// ================================================================== host side
+
 const char *fwd_bf16_unsupported(const OpDims &d) {
-    (void)d;
-    return "the tcgen05 chunked forward is not built yet";
+    if (d.dk != d.dv) return "d_k must equal d_v";
+    if (d.dk != 64 && d.dk != 128) return "d_k must be 64 or 128";
+    if (d.R2 != 64 && d.R2 != 128 && d.R2 != 256) return "2M must be 64, 128 or 256";
+    if (d.S != 32 && d.S != 64 && d.S != 128) return "S must be 32, 64 or 128";
+    return nullptr;
 }
 
 size_t fwd_bf16_workspace_bytes(const OpDims &d) {
-    (void)d;
-    return 0;
+    if (fwd_bf16_unsupported(d)) return 0;
+    Geo g = make_geo(d);
+    return ws_layout(d, g).total;
 }
+
+// Dynamic shared memory to request: at least `bytes`, and when the kernel allocates all 512
+// TMEM columns, enough to keep a second CTA of it off the same SM.
+static int smem_request(size_t bytes, int tmem_cols) {
+    const size_t one_per_sm = 120 * 1024;
+    if (tmem_cols >= 512 && bytes < one_per_sm) bytes = one_per_sm;
+    return (int)bytes;
+}
+
+static int pow2_cols(int n) { return n <= 32 ? 32 : n <= 64 ? 64 : n <= 128 ? 128 : n <= 256 ? 256 : 512; }
 
 cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const void *v, void *o, float *lse,
                          float *state_out, void *workspace, cudaStream_t st) {
-    (void)d; (void)q; (void)k; (void)v; (void)o; (void)lse; (void)state_out; (void)workspace; (void)st;
-    return cudaErrorNotSupported;
+    Geo g = make_geo(d);
+    if (g.L == 0) {
+        if (state_out)
+            return cudaMemsetAsync(state_out, 0, sizeof(float) * (size_t)g.BH * 2 * g.R2 * g.D, st);
+        return cudaSuccess;
+    }
+    WsLayout wl = ws_layout(d, g);
+    char *ws = static_cast<char *>(workspace);
+    Tables t;
+    tables_carve(d, kC, ws + wl.tables, &t);
+    cudaError_t e = tables_build(d, t, st);
+    if (e != cudaSuccess) return e;
+    bf16 *eb = reinterpret_cast<bf16 *>(ws + wl.eb), *phi = reinterpret_cast<bf16 *>(ws + wl.phi);
+    bf16 *fseg = g.G > 1 ? reinterpret_cast<bf16 *>(ws + wl.fseg) : nullptr;
+    {
+        long long total = (long long)g.RP * kC + (long long)g.SP * g.R2 + (fseg ? (long long)g.RP * g.Lseg : 0);
+        int blocks = (int)((total + 255) / 256);
+        if (blocks > 2048) blocks = 2048;
+        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, d.T, d.w, eb, phi, fseg);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    Args a;
+    a.g = g;
+    a.scale = d.scale;
+    a.w = d.w;
+    a.erel = t.erel;
+    a.delta = t.delta;
+    a.deltas = g.G > 1 ? reinterpret_cast<float *>(ws + wl.deltas) : nullptr;
+    a.deltas_out = const_cast<float *>(a.deltas);
+    a.win = g.G > 1 ? reinterpret_cast<float *>(ws + wl.win) : nullptr;
+    a.pbuf = reinterpret_cast<bf16 *>(ws + wl.pbuf);
+    a.lse = lse;
+    a.o = static_cast<bf16 *>(o);
+    a.state_out = state_out;
+    a.err = device_error_word();
+
+    // tensor maps
+    CUtensorMap tq, tk, tv, tp, teb, tphi, tf;
+    const uint64_t dq[3] = {(uint64_t)g.D, (uint64_t)g.L, (uint64_t)g.BH};
+    const uint64_t sq[2] = {(uint64_t)g.D * 2, (uint64_t)g.L * g.D * 2};
+    const uint32_t bq[3] = {64, (uint32_t)kC, 1};
+    const uint32_t bx[3] = {64, 64, 1};
+    const uint64_t dp[3] = {(uint64_t)g.SP, (uint64_t)g.L, (uint64_t)g.BH};
+    const uint64_t sp[2] = {(uint64_t)g.SP * 2, (uint64_t)g.L * g.SP * 2};
+    const uint64_t deb[2] = {(uint64_t)kC, (uint64_t)g.RP}, seb[1] = {(uint64_t)kC * 2};
+    const uint32_t beb[2] = {64, 128};
+    const uint64_t dph[2] = {(uint64_t)g.R2, (uint64_t)g.SP}, sph[1] = {(uint64_t)g.R2 * 2};
+    const uint32_t bph[2] = {64, (uint32_t)g.SP};
+    if (!make_tmap_bf16(&tq, q, 3, dq, sq, bq) || !make_tmap_bf16(&tp, a.pbuf, 3, dp, sp, bq) ||
+        !make_tmap_bf16(&teb, eb, 2, deb, seb, beb) || !make_tmap_bf16(&tphi, phi, 2, dph, sph, bph))
+        return cudaErrorInvalidValue;
+    const int nblk = g.BH * g.G;
+    if (g.G > 1) {
+        // prepass uses half-chunk boxes (64 rows) for K and V
+        if (!make_tmap_bf16(&tk, k, 3, dq, sq, bx) || !make_tmap_bf16(&tv, v, 3, dq, sq, bx)) return cudaErrorInvalidValue;
+        const uint64_t df[2] = {(uint64_t)g.Lseg, (uint64_t)g.RP}, sf[1] = {(uint64_t)g.Lseg * 2};
+        const uint32_t bf[2] = {64, 128};
+        if (!make_tmap_bf16(&tf, fseg, 2, df, sf, bf)) return cudaErrorInvalidValue;
+        const size_t stage_bytes = (size_t)g.NB * 128 * 64 * 2 + 2 * (size_t)64 * g.D * 2;
+        const int smem = smem_request(kPreStages * stage_bytes + 256 + 1024, pow2_cols(2 * g.NB * g.D));
+        if ((e = cudaFuncSetAttribute(k_prepass, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+            return e;
+        k_prepass<<<nblk, kThreads, smem, st>>>(tk, tv, tf, a);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        long long tot = (long long)g.BH * 2 * g.M * g.D;
+        int blocks = (int)((tot + 255) / 256);
+        if (blocks > 4096) blocks = 4096;
+        k_scan<<<blocks, 256, 0, st>>>(a);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    if (!make_tmap_bf16(&tk, k, 3, dq, sq, bq) || !make_tmap_bf16(&tv, v, 3, dq, sq, bq)) return cudaErrorInvalidValue;
+    {
+        KLayout kl = k_layout(g);
+        const int smem = smem_request(kl.total, pow2_cols(g.NB * g.D + 128 + g.RH));
+        if ((e = cudaFuncSetAttribute(k_kpass, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+            return e;
+        k_kpass<<<nblk, kThreads, smem, st>>>(tq, tk, teb, tphi, a);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    {
+        VLayout vl = v_layout(g);
+        const int smem = smem_request(vl.total, pow2_cols(g.NB * g.D + 256));
+        if ((e = cudaFuncSetAttribute(k_vpass, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+            return e;
+        k_vpass<<<nblk, kThreads, smem, st>>>(tp, tv, teb, tphi, a);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace bla

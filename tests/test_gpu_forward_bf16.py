@@ -1,0 +1,98 @@
+"""bf16 tensor-core chunked forward (tcgen05/TMEM/TMA) against the float64 oracle."""
+import numpy as np
+import pytest
+
+from gpu_util import TOL_BF16, rel, require_cuda, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def run(q, k, v, M, S, T, want_state=True, omega=0.0):
+    import torch
+    from paper_2606_09862_gb300 import bla
+    dev = require_cuda()
+    o, lse, st = bla.bla_forward_chunked(to_dev(q, dev, torch.bfloat16), to_dev(k, dev, torch.bfloat16),
+                                         to_dev(v, dev, torch.bfloat16), M, S, T, omega=omega,
+                                         want_state=want_state)
+    bla.bla_device_error()
+    return o.float().cpu().numpy(), lse.cpu().numpy(), (st.cpu().numpy() if st is not None else None)
+
+
+@pytest.mark.parametrize("B,H,L,d,M,S,T", [
+    (2, 2, 300, 64, 32, 32, 256.0),      # 2M = 64, one segment per head, ragged tail
+    (1, 2, 1000, 128, 64, 64, 1024.0),   # 2M = 128, many one-chunk segments (prepass + scan)
+    (1, 1, 777, 128, 128, 128, 4096.0),  # 2M = 256 (two mode halves), ragged, multi-segment
+    (3, 1, 129, 64, 128, 32, 512.0),     # 2M = 256 with d = 64, S = 32
+    (1, 3, 128, 128, 64, 128, 200.0),    # exactly one chunk
+    (2, 1, 1, 64, 32, 64, 100.0),        # a single token
+])
+def test_shapes_against_oracle(orc, B, H, L, d, M, S, T):
+    from paper_2606_09862_gb300.inputs import make_qkv
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=L + M)
+    o, lse, st = run(q, k, v, M, S, T)
+    ref = orc.forward(q, k, v, M, S, T, form="modes", return_state=True)
+    assert rel(o, ref["o"]) <= TOL_BF16, rel(o, ref["o"])
+    assert np.abs(lse - ref["lse"]).max() <= 5e-2
+    assert rel(st, ref["state"]) <= TOL_BF16
+
+
+def test_sharp_softmax(orc):
+    from paper_2606_09862_gb300.inputs import make_qkv
+    q, k, v = make_qkv(1, 2, 2000, 128, dtype="bf16", seed=3, sharp=True)
+    o, lse, st = run(q, k, v, 128, 128, 4096.0)
+    ref = orc.forward(q, k, v, 128, 128, 4096.0, form="modes", return_state=True)
+    assert rel(o, ref["o"]) <= TOL_BF16, rel(o, ref["o"])
+    assert rel(st, ref["state"]) <= TOL_BF16
+
+
+def test_recall_workload_full(orc):
+    """B=64, H=4, L=512, d=64, M=32, S=32, T=256; 10% of keys duplicated earlier: every output."""
+    from paper_2606_09862_gb300.inputs import WORKLOADS, workload_inputs
+    w = WORKLOADS["fwd_bf16_recall"]
+    x = workload_inputs(w, seed=0)
+    o, lse, st = run(x["q"], x["k"], x["v"], w.M, w.S, w.T)
+    ref = orc.forward(x["q"], x["k"], x["v"], w.M, w.S, w.T, form="modes", return_state=True)
+    assert rel(o, ref["o"]) <= TOL_BF16, rel(o, ref["o"])
+    assert rel(st, ref["state"]) <= TOL_BF16
+
+
+def test_lm_layer_workload_forward_full(orc):
+    """B=8, H=8, L=4096, d=128, M=64, S=64, T=1024: every output and the final state."""
+    from paper_2606_09862_gb300.inputs import WORKLOADS, workload_inputs
+    w = WORKLOADS["fwdbwd_bf16_lm"]
+    x = workload_inputs(w, seed=0)
+    o, lse, st = run(x["q"], x["k"], x["v"], w.M, w.S, w.T)
+    ref = orc.forward(x["q"], x["k"], x["v"], w.M, w.S, w.T, form="modes", return_state=True)
+    assert rel(o, ref["o"]) <= TOL_BF16, rel(o, ref["o"])
+    assert rel(st, ref["state"]) <= TOL_BF16
+
+
+def test_long_prefill_workload_sampled(orc):
+    """B=1, H=16, L=65536, d=128, M=128, S=128, T=4096 in the bench's launch configuration:
+    outputs at sampled tokens (every 61st, plus chunk and segment edges and the tail) and the
+    final state of every head, against the oracle recurrence over the full sequence."""
+    from paper_2606_09862_gb300.inputs import WORKLOADS, workload_inputs
+    w = WORKLOADS["prefill_bf16_long"]
+    x = workload_inputs(w, seed=0)
+    o, lse, st = run(x["q"], x["k"], x["v"], w.M, w.S, w.T)
+    want = np.zeros(w.L, bool)
+    want[::61] = True
+    want[127::128] = True
+    want[128::128] = True
+    want[-5:] = True
+    ref = orc.forward(x["q"], x["k"], x["v"], w.M, w.S, w.T, form="modes", want=want, return_state=True)
+    assert rel(o[:, :, want], ref["o"][:, :, want]) <= TOL_BF16, rel(o[:, :, want], ref["o"][:, :, want])
+    assert np.abs(lse[:, :, want] - ref["lse"][:, :, want]).max() <= 5e-2
+    assert rel(st, ref["state"]) <= TOL_BF16
+
+
+def test_repeated_calls_are_deterministic():
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    q, k, v = (to_dev(x, dev, torch.bfloat16) for x in make_qkv(1, 4, 3000, 128, dtype="bf16", seed=11))
+    a = bla.bla_forward_chunked(q, k, v, 128, 128, 4096.0)[0]
+    b = bla.bla_forward_chunked(q, k, v, 128, 128, 4096.0)[0]
+    torch.cuda.synchronize()
+    assert torch.equal(a, b)
