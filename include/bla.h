@@ -126,6 +126,33 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
                         const void *o, const void *dout, const float *lse,
                         void *dq, void *dk, void *dv, void *workspace, size_t ws_bytes, void *stream);
 
+/* ---------------------------------------------------------------- instrumentation
+ * (no paper counterpart: measurement support for benchmarks and tests)
+ * Kernels of this library, as counted and timed below. */
+typedef enum {
+    BLA_K_TABLES = 0,      /* fp32 interpolation/phase tables (every call) */
+    BLA_K_TABLES_BF16,     /* bf16 operand tables of the tensor-core path */
+    BLA_K_PREPASS,         /* per-segment state deltas (tcgen05 GEMM) */
+    BLA_K_SCAN,            /* states entering each segment */
+    BLA_K_KPASS,           /* K pass: scores, softmax, slot probabilities (tcgen05) */
+    BLA_K_VPASS,           /* V pass: outputs (tcgen05) */
+    BLA_K_FWD_F32,         /* fp32 chunked forward (CUDA cores) */
+    BLA_K_DECODE,          /* decode step */
+    BLA_K_BWD,             /* backward kernels */
+    BLA_K_COUNT
+} bla_kernel_id;
+
+/* Kernels launched by this library in this process so far. */
+long long bla_kernel_launches(void);
+
+/* on != 0: from now on record a CUDA event pair around every kernel launch, on the
+ * launch's stream (two event records per launch; off by default). */
+bla_status bla_profile_enable(int on);
+
+/* Synchronise the recorded events, add each launch's duration (ms) to ms[kernel] and
+ * 1 to launches[kernel] (arrays of BLA_K_COUNT, zeroed by the caller), then forget them. */
+bla_status bla_profile_collect(double *ms, int *launches);
+
 /* Synchronise `stream` and report (then clear) the library's device error word:
  * BLA_OK, or BLA_ERR_TIMEOUT if a bounded wait gave up since the last call. */
 bla_status bla_device_error(void *stream);

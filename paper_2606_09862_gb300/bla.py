@@ -19,7 +19,11 @@ BLA_F32, BLA_BF16 = 0, 1
 BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE = 0, 1, 2
 
 EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
-            "bla_device_error", "bla_status_string", "bla_last_error_string")
+            "bla_device_error", "bla_status_string", "bla_last_error_string", "bla_kernel_launches",
+            "bla_profile_enable", "bla_profile_collect")
+
+# bla_kernel_id
+KERNELS = ("tables", "tables_bf16", "prepass", "scan", "kpass", "vpass", "fwd_f32", "decode", "bwd")
 
 
 class BlaError(RuntimeError):
@@ -63,6 +67,12 @@ def load():
     lib.bla_status_string.argtypes = [ctypes.c_int]
     lib.bla_last_error_string.restype = ctypes.c_char_p
     lib.bla_last_error_string.argtypes = []
+    lib.bla_kernel_launches.restype = ctypes.c_longlong
+    lib.bla_kernel_launches.argtypes = []
+    lib.bla_profile_enable.restype = ctypes.c_int
+    lib.bla_profile_enable.argtypes = [ctypes.c_int]
+    lib.bla_profile_collect.restype = ctypes.c_int
+    lib.bla_profile_collect.argtypes = [ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)]
     _lib = lib
     return lib
 
@@ -164,3 +174,54 @@ def bla_backward(q, k, v, o, dout, lse, M, S, window, omega=0.0, scale=0.0, work
 def bla_device_error(stream=None):
     """Synchronise and raise BlaError if a bounded device wait gave up."""
     _check(load().bla_device_error(_stream(stream)))
+
+
+def bla_kernel_launches():
+    """Kernels this library has launched in this process."""
+    return int(load().bla_kernel_launches())
+
+
+def bla_profile_enable(on=True):
+    """Record a CUDA event pair around every launch (on the launch stream) from now on."""
+    _check(load().bla_profile_enable(1 if on else 0))
+
+
+def bla_profile_collect():
+    """{kernel name: (total ms, launches)} for the launches recorded since the last collect."""
+    n = len(KERNELS)
+    ms = (ctypes.c_double * n)()
+    cnt = (ctypes.c_int * n)()
+    _check(load().bla_profile_collect(ms, cnt))
+    return {KERNELS[i]: (float(ms[i]), int(cnt[i])) for i in range(n) if cnt[i] > 0}
+
+
+def forward_from_host(q_host, k_host, v_host, M, S, window, omega=0.0, scale=0.0, device=None, bufs=None,
+                      out_host=None, stream=None):
+    """bla_forward_chunked on host tensors: copies q, k, v (pinned for asynchronous copies) to the
+    device, runs the chunked forward and copies o back into `out_host` (allocated if None).
+    `bufs` (dict) caches the device buffers and workspace between calls.  Returns out_host; the
+    copy back is asynchronous on the current stream."""
+    dev = torch.device("cuda") if device is None else device
+    bufs = {} if bufs is None else bufs
+    for name, h in (("q", q_host), ("k", k_host), ("v", v_host)):
+        t = bufs.get(name)
+        if t is None or t.shape != h.shape or t.dtype != h.dtype:
+            bufs[name] = torch.empty(h.shape, dtype=h.dtype, device=dev)
+        bufs[name].copy_(h, non_blocking=True)
+    B, H, L, _ = q_host.shape
+    dv = v_host.shape[-1]
+    if "o" not in bufs or bufs["o"].shape != (B, H, L, dv):
+        bufs["o"] = torch.empty((B, H, L, dv), dtype=q_host.dtype, device=dev)
+        bufs["lse"] = torch.empty((B, H, L), dtype=torch.float32, device=dev)
+    p = make_params(B, H, L, q_host.shape[-1], dv, M, S, window, omega, 0, scale, q_host.dtype)
+    if "ws" not in bufs:
+        n = bla_workspace_bytes(p, BLA_WS_FORWARD)
+        bufs["ws"] = torch.empty(max(n, 1), dtype=torch.uint8, device=dev)
+    ws = bufs["ws"]
+    _check(load().bla_forward_chunked(ctypes.byref(p), _ptr(bufs["q"]), _ptr(bufs["k"]), _ptr(bufs["v"]),
+                                      _ptr(bufs["o"]), _ptr(bufs["lse"]), None, _ptr(ws), ws.numel(),
+                                      _stream(stream)))
+    if out_host is None:
+        out_host = torch.empty(bufs["o"].shape, dtype=bufs["o"].dtype, pin_memory=True)
+    out_host.copy_(bufs["o"], non_blocking=True)
+    return out_host

@@ -4,10 +4,55 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
+#include <mutex>
+#include <vector>
+
 #include "common.cuh"
 #include "fwd_bf16.cuh"
 
 namespace bla {
+
+// ------------------------------------------------------------------ launch accounting
+namespace {
+std::atomic<long long> g_launches{0};
+std::atomic<bool> g_prof_on{false};
+struct ProfRec {
+    int kid;
+    cudaEvent_t a, b;
+};
+std::mutex g_prof_mu;
+std::vector<ProfRec> g_prof_recs;       // recorded, not yet collected
+std::vector<cudaEvent_t> g_prof_pool;   // idle events
+
+cudaEvent_t pool_get() {
+    if (!g_prof_pool.empty()) {
+        cudaEvent_t e = g_prof_pool.back();
+        g_prof_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+}
+}  // namespace
+
+ProfScope::ProfScope(int kernel_id, cudaStream_t st) : kid(kernel_id), stream(st), slot(-1) {
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    if (!g_prof_on.load(std::memory_order_relaxed)) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    ProfRec r{kernel_id, pool_get(), pool_get()};
+    if (!r.a || !r.b) return;
+    cudaEventRecord(r.a, st);
+    g_prof_recs.push_back(r);
+    slot = (int)g_prof_recs.size() - 1;
+}
+
+ProfScope::~ProfScope() {
+    if (slot < 0) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (slot < (int)g_prof_recs.size()) cudaEventRecord(g_prof_recs[slot].b, stream);
+}
 
 __device__ int g_dev_error = 0;
 
@@ -193,6 +238,36 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
     (void)q; (void)k; (void)v; (void)o; (void)dout; (void)lse; (void)dq; (void)dk; (void)dv;
     (void)workspace; (void)ws_bytes; (void)stream;
     return fail(BLA_ERR_UNSUPPORTED, "backward is not implemented yet");
+}
+
+long long bla_kernel_launches(void) { return g_launches.load(); }
+
+bla_status bla_profile_enable(int on) {
+    t_last_error[0] = 0;
+    g_prof_on.store(on != 0);
+    return BLA_OK;
+}
+
+bla_status bla_profile_collect(double *ms, int *launches) {
+    t_last_error[0] = 0;
+    if (!ms || !launches) return fail(BLA_ERR_INVALID, "ms and launches must be non-NULL");
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    bla_status st = BLA_OK;
+    for (auto &r : g_prof_recs) {
+        float t = 0.f;
+        cudaError_t e = cudaEventSynchronize(r.b);
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&t, r.a, r.b);
+        if (e != cudaSuccess) {
+            st = cuda_fail(e, "profile event");
+        } else if (r.kid >= 0 && r.kid < BLA_K_COUNT) {
+            ms[r.kid] += t;
+            launches[r.kid] += 1;
+        }
+        g_prof_pool.push_back(r.a);
+        g_prof_pool.push_back(r.b);
+    }
+    g_prof_recs.clear();
+    return st;
 }
 
 bla_status bla_device_error(void *stream) {

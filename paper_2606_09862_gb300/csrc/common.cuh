@@ -68,6 +68,16 @@ __device__ __forceinline__ void report_device_error(int *word, int code) {
     if (word) atomicCAS(word, 0, code);
 }
 
+// Launch accounting and optional per-launch event timing (api.cu).  Construct a ProfScope
+// immediately before a kernel launch and let it go out of scope right after it.
+struct ProfScope {
+    ProfScope(int kernel_id, cudaStream_t st);
+    ~ProfScope();
+    int kid;
+    cudaStream_t stream;
+    int slot;
+};
+
 // Launchers of the individual kernels (defined in their .cu files).
 cudaError_t launch_forward_f32(const OpDims &d, int C, const Tables &t, const float *q, const float *k,
                                const float *v, float *o, float *lse, float *state_out, float *scratch,

@@ -211,6 +211,7 @@ template <typename T, int D>
 cudaError_t launch_decode_t(const OpDims &d, long long pos, const Tables &t, const void *q, const void *k,
                             const void *v, float *state, void *o, cudaStream_t st) {
     int smem = (int)(sizeof(float) * (d.R2 + d.S + kWarps * D));
+    ProfScope ps(BLA_K_DECODE, st);
     k_decode<T, D><<<d.B * d.H, kThreads, smem, st>>>(d, pos, t, (const T *)q, (const T *)k, (const T *)v, state,
                                                      (T *)o);
     return cudaGetLastError();

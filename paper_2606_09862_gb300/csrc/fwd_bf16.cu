@@ -199,61 +199,55 @@ __device__ __forceinline__ uint64_t mnmaj_desc(const uint8_t *tile, int krows, i
     return tc::sdesc_sw128(a, (uint32_t)krows * 128u, 1024);
 }
 
-// Rotate the state block held in TMEM (rows = lanes, interleaved cos/sin pairs) by
-// e^{i m w adv} and optionally write it back, also emitting the bf16 copy into a
-// [RH rows][64 d] blocked tile (rows >= RH skipped) and/or an fp32 copy to global.
+// Rotate the state block held in TMEM (rows = lanes, interleaved cos/sin pairs) by the
+// phase (c, s) of this thread's mode, optionally write it back, and emit a bf16 copy into
+// a [RH rows][64 d]-blocked tile (rows >= RH skipped) and/or an fp32 copy to global.
 // Executed by the 128 epilogue threads; `row` is this thread's lane = local state row.
-__device__ void state_pass(uint32_t tbase, int col0, int D, int row, int mode_base, int RH, int R2row_limit,
-                           int R2, const float *erel, int M, int adv, bool rotate, bool write_back, uint8_t *wtile,
-                           float *gout) {
-    (void)R2;
+template <int D>
+__device__ __forceinline__ void state_pass(uint32_t tbase, int col0, int row, bool rotate, float c, float s,
+                                           bool write_back, uint8_t *wtile, int RH, float *gout) {
     const int lane_base = (row >> 5) << 5;
-    const int m = mode_base + (row >> 1);
-    float c = 1.f, s = 0.f;
-    if (rotate && m < M) {
-        c = erel[((size_t)adv * M + m) * 2];
-        s = erel[((size_t)adv * M + m) * 2 + 1];
+    const uint32_t addr = tmem_addr(tbase, lane_base, col0);
+    float v[D];
+    tc::tmem_ld<D>(addr, v);
+    if (rotate) {
+        const bool odd = row & 1;
+#pragma unroll
+        for (int i = 0; i < D; ++i) {
+            const float partner = __shfl_xor_sync(0xffffffffu, v[i], 1);
+            // even row: Re' = c Re - s Im ; odd row: Im' = s Re + c Im
+            v[i] = odd ? fmaf(s, partner, c * v[i]) : fmaf(-s, partner, c * v[i]);
+        }
+        if (write_back) tc::tmem_st<D>(addr, v);
     }
-    const bool odd = row & 1;
-    for (int g = 0; g < D; g += 32) {
-        float v[32];
-        tc::tmem_ld32(tmem_addr(tbase, lane_base, col0 + g), v);
-        if (rotate) {
+    if (wtile && row < RH) {
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                float partner = __shfl_xor_sync(0xffffffffu, v[i], 1);
-                // even row: Re' = c Re - s Im ; odd row: Im' = s Re + c Im
-                v[i] = odd ? fmaf(s, partner, c * v[i]) : fmaf(-s, partner, c * v[i]);
-            }
-            if (write_back) tc::tmem_st32(tmem_addr(tbase, lane_base, col0 + g), v);
-        }
-        if (wtile && row < RH) st_row32_bf16(wtile, RH, row, g, v);
-        if (gout && row < R2row_limit) {
+        for (int g = 0; g < D; g += 32) st_row32_bf16(wtile, RH, row, g, v + g);
+    }
+    if (gout) {
 #pragma unroll
-            for (int i = 0; i < 32; i += 4)
-                *reinterpret_cast<float4 *>(gout + g + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
-        }
+        for (int i = 0; i < D; i += 4) *reinterpret_cast<float4 *>(gout + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
     }
 }
 
 // Load 128 rows x D fp32 (global, row stride D) into a TMEM state block; rows at or beyond
 // `live_rows` (padding beyond 2M) and a NULL source give zeros.
-__device__ void state_init(uint32_t tbase, int col0, int D, int row, const float *src, int live_rows) {
+template <int D>
+__device__ __forceinline__ void state_init(uint32_t tbase, int col0, int row, const float *src, int live_rows) {
     const int lane_base = (row >> 5) << 5;
-    for (int g = 0; g < D; g += 32) {
-        float v[32];
-        if (src && row < live_rows) {
+    float v[D];
 #pragma unroll
-            for (int i = 0; i < 32; i += 4) {
-                float4 t = *reinterpret_cast<const float4 *>(src + (size_t)row * D + g + i);
-                v[i] = t.x; v[i + 1] = t.y; v[i + 2] = t.z; v[i + 3] = t.w;
-            }
-        } else {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) v[i] = 0.f;
-        }
-        tc::tmem_st32(tmem_addr(tbase, lane_base, col0 + g), v);
+    for (int i = 0; i < D; i += 4) {
+        float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (src && row < live_rows) t = *reinterpret_cast<const float4 *>(src + (size_t)row * D + i);
+        v[i] = t.x; v[i + 1] = t.y; v[i + 2] = t.z; v[i + 3] = t.w;
     }
+    tc::tmem_st<D>(tmem_addr(tbase, lane_base, col0), v);
+}
+
+// Phase (cos, sin)(m w tau) from the fp32 table [C+1][M][2].
+__device__ __forceinline__ float2 phase(const float *erel, int M, int tau, int m) {
+    return make_float2(erel[((size_t)tau * M + m) * 2], erel[((size_t)tau * M + m) * 2 + 1]);
 }
 
 // ================================================================== prepass
@@ -341,8 +335,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int x = 0; x < 2; ++x)
                 for (int b = 0; b < NB; ++b) {
                     float *dst = a.deltas_out + ((((size_t)bh * g.G + seg) * 2 + x) * g.RP + b * 128 + row) * D;
-                    state_pass(tb, (x * NB + b) * D, D, row, 0, 0, 1 << 30, g.R2, a.erel, g.M, 0, false, false, nullptr,
-                               dst);
+                    if (D == 128)
+                        state_pass<128>(tb, (x * NB + b) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
+                    else
+                        state_pass<64>(tb, (x * NB + b) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
                 }
         }
     }
@@ -415,6 +411,7 @@ enum KBar {
     KB_P_READY, KB_W_READY, KB_W_FREE, KB_STATE_DONE, KB_STATE_DONE1, KB_Y_READY, KB_Y_FREE, KB_EXIT, KB_COUNT
 };
 
+template <int D, int RH, int S>
 __global__ void __launch_bounds__(kThreads, 1)
     k_kpass(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
             const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi, Args a) {
@@ -431,7 +428,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     Ctl *ctl = reinterpret_cast<Ctl *>(bar + KB_COUNT + 1);
     int *sdelta = reinterpret_cast<int *>(bar + KB_COUNT + 4);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int D = g.D, RH = g.RH, NH = g.NH, S = g.S, SP = g.SP;
+    const int NH = g.NH, SP = g.SP;
     // TMEM columns: [0, NB*D) state; accA at NB*D (128 cols); accB after it (RH cols).
     const int colA = g.NB * D, colB = colA + 128;
     const uint32_t ncols = (uint32_t)(colB + RH) <= 256 ? 256u : 512u;   // host: pow2_cols(NB*D + 128 + RH)
@@ -556,10 +553,19 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint32_t ph_state[2] = {0, 0};
         const int M = g.M;
         const float *erel = a.erel;
-        // state entering the segment
+        // phase constants of this thread, fixed for the whole CTA: the per-mode step e^{i w t}
+        // of token row t, the start phase of each mode half, and e^{i m w C} of its state row
+        const float2 e1 = phase(erel, M, row, 1);
+        float2 ph0[2], rotC[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            ph0[h] = (h < NH) ? phase(erel, M, row, h * (RH / 2)) : make_float2(1.f, 0.f);
+            const int m = (h * 128 + row) >> 1;
+            rotC[h] = (h < g.NB && m < M) ? phase(erel, M, kC, m) : make_float2(1.f, 0.f);
+        }
         for (int b = 0; b < g.NB; ++b) {
             const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
-            state_init(tb, b * D, D, row, src, g.R2 - b * 128);
+            state_init<D>(tb, b * D, row, src, g.R2 - b * 128);
         }
         bool bad = false;
         for (int c = c_begin; c < c_end && !bad; ++c) {
@@ -567,57 +573,54 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int n = min(kC, g.L - t0);
             const bool rot = c > c_begin;
             for (int h = 0; h < NH && !bad; ++h) {
-                // W_h extraction: state block h (holding W + EB X of the previous chunk) is rotated by
-                // e^{i m w C} into the state carried into this chunk, written back, and copied to bf16.
+                // W_h: state block h (W + EB X of the previous chunk) rotated by e^{i m w C} into the
+                // state carried into this chunk, written back, and copied to bf16 for the MMA.
                 if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                state_pass(tb, h * D, D, row, h * 64, RH, 0, g.R2, erel, M, kC, rot, rot, sW, nullptr);
+                state_pass<D>(tb, h * D, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 tc::mbar_arrive(&bar[KB_W_READY]);
                 if (h == 0) {
-                    // P drain: mask u <= t, bf16 -> sP
+                    // P drain: causal mask u <= t, bf16 -> sP
                     if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
-                    for (int g0 = 0; g0 < kC; g0 += 32) {
-                        float v[32];
-                        tc::tmem_ld32(tmem_addr(tb, lane_base, colA + g0), v);
+                    float v[kC];
+                    tc::tmem_ld<kC>(tmem_addr(tb, lane_base, colA), v);
 #pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (g0 + i > row) v[i] = 0.f;
-                        st_row32_bf16(sP, kC, row, g0, v);
-                    }
+                    for (int i = 0; i < kC; ++i)
+                        if (i > row) v[i] = 0.f;
+#pragma unroll
+                    for (int g0 = 0; g0 < kC; g0 += 32) st_row32_bf16(sP, kC, row, g0, v + g0);
                     tc::fence_proxy_async_smem();
                     tc::tc_fence_before();
                     tc::mbar_arrive(&bar[KB_P_READY]);
                     tc::mbar_arrive(&bar[KB_ACC_FREE_A]);
                 }
-                // drain X_h -> Y_h (rotate by e^{i m w t}, t = row)
+                // X_h drain -> Y_h = e^{i m w t} X_h (t = row), modes advanced by e1
                 const bool inB = (h & 1) == 0;
                 if (!wait_bar(&bar[inB ? KB_ACC_FULL_B : KB_ACC_FULL_A], inB ? ph_fullB : ph_fullA, ctl, a.err)) {
                     bad = true;
                     break;
                 }
-                // X_h complete => W tile free for the next half
                 if (!wait_bar(&bar[KB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
                 if (h > 0 && !wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                const float c1 = erel[((size_t)row * M + 1) * 2], s1 = erel[((size_t)row * M + 1) * 2 + 1];
-                for (int g0 = 0; g0 < RH; g0 += 32) {
-                    float v[32];
-                    tc::tmem_ld32(tmem_addr(tb, lane_base, (inB ? colB : colA) + g0), v);
-                    const int m0 = h * (RH / 2) + g0 / 2;
-                    float cc = erel[((size_t)row * M + m0) * 2], ss = erel[((size_t)row * M + m0) * 2 + 1];
+                {
+                    float v[RH];
+                    tc::tmem_ld<RH>(tmem_addr(tb, lane_base, inB ? colB : colA), v);
+                    float cc = ph0[h].x, ss = ph0[h].y;
 #pragma unroll
-                    for (int i = 0; i < 32; i += 2) {
+                    for (int i = 0; i < RH; i += 2) {
                         const float xr = v[i], xi = v[i + 1];
                         v[i] = cc * xr - ss * xi;
                         v[i + 1] = ss * xr + cc * xi;
-                        const float nc = cc * c1 - ss * s1, ns = ss * c1 + cc * s1;
+                        const float nc = cc * e1.x - ss * e1.y, ns = ss * e1.x + cc * e1.y;
                         cc = nc;
                         ss = ns;
                     }
-                    st_row32_bf16(sY, kC, row, g0, v);
+#pragma unroll
+                    for (int g0 = 0; g0 < RH; g0 += 32) st_row32_bf16(sY, kC, row, g0, v + g0);
                 }
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
@@ -625,7 +628,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::mbar_arrive(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
             }
             if (bad) break;
-            // softmax over slots
+            // masked softmax over the S slots, one TMEM pass
             const bool sInB = NH == 2;
             if (!wait_bar(&bar[sInB ? KB_ACC_FULL_B : KB_ACC_FULL_A], sInB ? ph_fullB : ph_fullA, ctl, a.err)) {
                 bad = true;
@@ -633,48 +636,39 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             if (!wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
             tc::tc_fence_after();
-            const int cs = sInB ? colB : colA;
-            const int t = t0 + row;
-            float mx = -INFINITY;
-            for (int g0 = 0; g0 < S; g0 += 32) {
-                float v[32];
-                tc::tmem_ld32(tmem_addr(tb, lane_base, cs + g0), v);
+            {
+                float v[S];
+                tc::tmem_ld<S>(tmem_addr(tb, lane_base, sInB ? colB : colA), v);
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bar[sInB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
+                const int t = t0 + row;
+                float mx = -INFINITY;
 #pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (g0 + i < S && t >= sdelta[g0 + i]) mx = fmaxf(mx, v[i] * a.scale);
-            }
-            float sum = 0.f;
-            for (int g0 = 0; g0 < S; g0 += 32) {
-                float v[32];
-                tc::tmem_ld32(tmem_addr(tb, lane_base, cs + g0), v);
-#pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (g0 + i < S && t >= sdelta[g0 + i]) sum += __expf(v[i] * a.scale - mx);
-            }
-            const float inv = 1.f / sum;
-            bf16 *prow = a.pbuf + ((size_t)bh * g.L + t) * SP;
-            for (int g0 = 0; g0 < SP; g0 += 32) {
-                float v[32];
-                if (g0 < S) tc::tmem_ld32(tmem_addr(tb, lane_base, cs + g0), v);
-                uint32_t pk[16];
-#pragma unroll
-                for (int i = 0; i < 32; i += 2) {
-                    float p0 = (g0 < S && g0 + i < S && t >= sdelta[g0 + i]) ? __expf(v[i] * a.scale - mx) * inv : 0.f;
-                    float p1 = (g0 < S && g0 + i + 1 < S && t >= sdelta[g0 + i + 1])
-                                   ? __expf(v[i + 1] * a.scale - mx) * inv
-                                   : 0.f;
-                    pk[i / 2] = tc::pack_bf16x2(p0, p1);
+                for (int j = 0; j < S; ++j) {
+                    v[j] = (t >= sdelta[j]) ? v[j] * a.scale : -INFINITY;
+                    mx = fmaxf(mx, v[j]);
                 }
+                float sum = 0.f;
+#pragma unroll
+                for (int j = 0; j < S; ++j) {
+                    v[j] = (v[j] == -INFINITY) ? 0.f : __expf(v[j] - mx);
+                    sum += v[j];
+                }
+                const float inv = 1.f / sum;
                 if (row < n) {
+                    bf16 *prow = a.pbuf + ((size_t)bh * g.L + t) * SP;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        *reinterpret_cast<uint4 *>(prow + g0 + q * 8) =
-                            make_uint4(pk[q * 4], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
+                    for (int j = 0; j < S; j += 8) {
+                        uint4 pk = make_uint4(tc::pack_bf16x2(v[j] * inv, v[j + 1] * inv),
+                                              tc::pack_bf16x2(v[j + 2] * inv, v[j + 3] * inv),
+                                              tc::pack_bf16x2(v[j + 4] * inv, v[j + 5] * inv),
+                                              tc::pack_bf16x2(v[j + 6] * inv, v[j + 7] * inv));
+                        *reinterpret_cast<uint4 *>(prow + j) = pk;
+                    }
+                    for (int j = S; j < SP; j += 8) *reinterpret_cast<uint4 *>(prow + j) = make_uint4(0, 0, 0, 0);
+                    if (a.lse) a.lse[(size_t)bh * g.L + t] = mx + logf(sum);
                 }
             }
-            if (row < n && a.lse) a.lse[(size_t)bh * g.L + t] = mx + logf(sum);
-            tc::tc_fence_before();
-            tc::mbar_arrive(&bar[sInB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
         }
         // final K state (lag frame at t = L-1) after the last chunk of the last segment
         if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
@@ -684,10 +678,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::tc_fence_after();
                 const int n_last = g.L - (c_end - 1) * kC;
                 for (int b = 0; b < g.NB; ++b) {
-                    const int r = b * 128 + row;
+                    const int r = b * 128 + row, m = r >> 1;
                     float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + r) * D : nullptr;
-                    state_pass(tb, b * D, D, row, b * 64, 0, g.R2 - b * 128, g.R2, erel, M, n_last - 1, true, false,
-                               nullptr, dst);
+                    const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
+                    state_pass<D>(tb, b * D, row, true, f.x, f.y, false, nullptr, 0, dst);
                 }
             }
         }
@@ -727,6 +721,7 @@ enum VBar {
     VB_STATE_DONE, VB_STATE_DONE1, VB_O_FULL, VB_EXIT, VB_COUNT
 };
 
+template <int D, int RH>
 __global__ void __launch_bounds__(kThreads, 1)
     k_vpass(const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_v,
             const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi, Args a) {
@@ -742,7 +737,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + VB_COUNT);
     Ctl *ctl = reinterpret_cast<Ctl *>(bar + VB_COUNT + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int D = g.D, RH = g.RH, NH = g.NH, SP = g.SP;
+    const int NH = g.NH, SP = g.SP;
     const size_t a_tile = (size_t)kC * RH * 2;
     // TMEM: [0, NB*D) state; colU (128 cols: U_h, then O); colG (128 cols).
     const int colU = g.NB * D, colG = colU + 128;
@@ -861,63 +856,69 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float *erel = a.erel;
         uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0;
         uint32_t ph_state[2] = {0, 0};
+        const float2 e1 = phase(erel, M, row, 1);
+        float2 ph0[2], rotC[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            ph0[h] = (h < NH) ? phase(erel, M, row, h * (RH / 2)) : make_float2(1.f, 0.f);
+            const int m = (h * 128 + row) >> 1;
+            rotC[h] = (h < g.NB && m < M) ? phase(erel, M, kC, m) : make_float2(1.f, 0.f);
+        }
         for (int b = 0; b < g.NB; ++b) {
             const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
-            state_init(tb, b * D, D, row, src, g.R2 - b * 128);
+            state_init<D>(tb, b * D, row, src, g.R2 - b * 128);
         }
         bool bad = false;
         for (int c = c_begin; c < c_end && !bad; ++c) {
             const int t0 = c * kC;
             const int n = min(kC, g.L - t0);
             const bool rot = c > c_begin;
-            // phase 1: U_h -> A'_h (rotation by -m w t of (sum_j p A, sum_j p B))
+            // phase 1: U_h -> A'_h, the rotation by -m w t of (sum_j p A, sum_j p B)
             for (int h = 0; h < NH; ++h) {
                 if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                for (int g0 = 0; g0 < RH; g0 += 32) {
-                    float v[32];
-                    tc::tmem_ld32(tmem_addr(tb, lane_base, colU + g0), v);
-                    const int m0 = h * (RH / 2) + g0 / 2;
-                    const float c1 = erel[((size_t)row * M + 1) * 2], s1 = erel[((size_t)row * M + 1) * 2 + 1];
-                    float cc = erel[((size_t)row * M + m0) * 2], ss = erel[((size_t)row * M + m0) * 2 + 1];
+                float v[RH];
+                tc::tmem_ld<RH>(tmem_addr(tb, lane_base, colU), v);
+                float cc = ph0[h].x, ss = ph0[h].y;
 #pragma unroll
-                    for (int i = 0; i < 32; i += 2) {
-                        const float uc = v[i], us = v[i + 1];
-                        v[i] = cc * uc + ss * us;
-                        v[i + 1] = cc * us - ss * uc;
-                        const float nc = cc * c1 - ss * s1, ns = ss * c1 + cc * s1;
-                        cc = nc;
-                        ss = ns;
-                    }
-                    st_row32_bf16(sA + h * a_tile, kC, row, g0, v);
+                for (int i = 0; i < RH; i += 2) {
+                    const float uc = v[i], us = v[i + 1];
+                    v[i] = cc * uc + ss * us;
+                    v[i + 1] = cc * us - ss * uc;
+                    const float nc = cc * e1.x - ss * e1.y, ns = ss * e1.x + cc * e1.y;
+                    cc = nc;
+                    ss = ns;
                 }
+#pragma unroll
+                for (int g0 = 0; g0 < RH; g0 += 32) st_row32_bf16(sA + h * a_tile, kC, row, g0, v + g0);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 tc::mbar_arrive(&bar[VB_A_READY]);
                 tc::mbar_arrive(&bar[VB_U_FREE]);
             }
             if (bad) break;
-            // phase 2: G drain -> mask -> bf16 over p's tile
+            // phase 2: G drain -> causal mask -> bf16 over p's tile
             if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
             tc::tc_fence_after();
-            for (int g0 = 0; g0 < kC; g0 += 32) {
-                float v[32];
-                tc::tmem_ld32(tmem_addr(tb, lane_base, colG + g0), v);
+            {
+                float v[kC];
+                tc::tmem_ld<kC>(tmem_addr(tb, lane_base, colG), v);
 #pragma unroll
-                for (int i = 0; i < 32; ++i)
-                    if (g0 + i > row) v[i] = 0.f;
-                st_row32_bf16(sPG, kC, row, g0, v);
+                for (int i = 0; i < kC; ++i)
+                    if (i > row) v[i] = 0.f;
+#pragma unroll
+                for (int g0 = 0; g0 < kC; g0 += 32) st_row32_bf16(sPG, kC, row, g0, v + g0);
             }
             tc::fence_proxy_async_smem();
             tc::tc_fence_before();
             tc::mbar_arrive(&bar[VB_G_READY]);
             tc::mbar_arrive(&bar[VB_G_FREE]);
-            // phase 3: W_h extraction (state read before this chunk's V update)
+            // phase 3: W_h (the V state read before this chunk's update)
             for (int h = 0; h < NH; ++h) {
                 if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
                 if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                state_pass(tb, h * D, D, row, h * 64, RH, 0, g.R2, erel, M, kC, rot, rot, sW, nullptr);
+                state_pass<D>(tb, h * D, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 tc::mbar_arrive(&bar[VB_W_READY]);
@@ -927,22 +928,21 @@ __global__ void __launch_bounds__(kThreads, 1)
             // phase 4: O drain -> global
             if (!wait_bar(&bar[VB_O_FULL], ph_o, ctl, a.err)) break;
             tc::tc_fence_after();
-            bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D;
-            for (int g0 = 0; g0 < D; g0 += 32) {
-                float v[32];
-                tc::tmem_ld32(tmem_addr(tb, lane_base, colU + g0), v);
+            {
+                float v[D];
+                tc::tmem_ld<D>(tmem_addr(tb, lane_base, colU), v);
+                tc::tc_fence_before();
+                tc::mbar_arrive(&bar[VB_U_FREE]);
                 if (row < n) {
+                    bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        uint4 pk = make_uint4(tc::pack_bf16x2(v[q * 8], v[q * 8 + 1]), tc::pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]),
-                                              tc::pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]),
-                                              tc::pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]));
-                        *reinterpret_cast<uint4 *>(orow + g0 + q * 8) = pk;
+                    for (int j = 0; j < D; j += 8) {
+                        uint4 pk = make_uint4(tc::pack_bf16x2(v[j], v[j + 1]), tc::pack_bf16x2(v[j + 2], v[j + 3]),
+                                              tc::pack_bf16x2(v[j + 4], v[j + 5]), tc::pack_bf16x2(v[j + 6], v[j + 7]));
+                        *reinterpret_cast<uint4 *>(orow + j) = pk;
                     }
                 }
             }
-            tc::tc_fence_before();
-            tc::mbar_arrive(&bar[VB_U_FREE]);
         }
         if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
             for (int h = 0; h < NH; ++h)
@@ -951,10 +951,10 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc::tc_fence_after();
                 const int n_last = g.L - (c_end - 1) * kC;
                 for (int b = 0; b < g.NB; ++b) {
-                    const int r = b * 128 + row;
+                    const int r = b * 128 + row, m = r >> 1;
                     float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + g.R2 + r) * D : nullptr;
-                    state_pass(tb, b * D, D, row, b * 64, 0, g.R2 - b * 128, g.R2, erel, M, n_last - 1, true, false,
-                               nullptr, dst);
+                    const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
+                    state_pass<D>(tb, b * D, row, true, f.x, f.y, false, nullptr, 0, dst);
                 }
             }
         }
@@ -995,6 +995,56 @@ static int smem_request(size_t bytes, int tmem_cols) {
 
 static int pow2_cols(int n) { return n <= 32 ? 32 : n <= 64 ? 64 : n <= 128 ? 128 : n <= 256 ? 256 : 512; }
 
+
+template <int D, int RH, int S>
+static cudaError_t launch_kpass_t(int smem, int nblk, cudaStream_t st, const CUtensorMap &tq, const CUtensorMap &tk,
+                                  const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+    cudaError_t e = cudaFuncSetAttribute(k_kpass<D, RH, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    ProfScope ps(BLA_K_KPASS, st);
+    k_kpass<D, RH, S><<<nblk, kThreads, smem, st>>>(tq, tk, teb, tphi, a);
+    return cudaGetLastError();
+}
+
+template <int D, int RH>
+static cudaError_t launch_kpass_s(const Geo &g, int smem, int nblk, cudaStream_t st, const CUtensorMap &tq,
+                                  const CUtensorMap &tk, const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+    switch (g.S) {
+    case 32: return launch_kpass_t<D, RH, 32>(smem, nblk, st, tq, tk, teb, tphi, a);
+    case 64: return launch_kpass_t<D, RH, 64>(smem, nblk, st, tq, tk, teb, tphi, a);
+    case 128: return launch_kpass_t<D, RH, 128>(smem, nblk, st, tq, tk, teb, tphi, a);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+static cudaError_t launch_kpass(const Geo &g, int smem, int nblk, cudaStream_t st, const CUtensorMap &tq,
+                                const CUtensorMap &tk, const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+    if (g.D == 64 && g.RH == 64) return launch_kpass_s<64, 64>(g, smem, nblk, st, tq, tk, teb, tphi, a);
+    if (g.D == 64 && g.RH == 128) return launch_kpass_s<64, 128>(g, smem, nblk, st, tq, tk, teb, tphi, a);
+    if (g.D == 128 && g.RH == 64) return launch_kpass_s<128, 64>(g, smem, nblk, st, tq, tk, teb, tphi, a);
+    if (g.D == 128 && g.RH == 128) return launch_kpass_s<128, 128>(g, smem, nblk, st, tq, tk, teb, tphi, a);
+    return cudaErrorInvalidValue;
+}
+
+template <int D, int RH>
+static cudaError_t launch_vpass_t(int smem, int nblk, cudaStream_t st, const CUtensorMap &tp, const CUtensorMap &tv,
+                                  const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+    cudaError_t e = cudaFuncSetAttribute(k_vpass<D, RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    ProfScope ps(BLA_K_VPASS, st);
+    k_vpass<D, RH><<<nblk, kThreads, smem, st>>>(tp, tv, teb, tphi, a);
+    return cudaGetLastError();
+}
+
+static cudaError_t launch_vpass(const Geo &g, int smem, int nblk, cudaStream_t st, const CUtensorMap &tp,
+                                const CUtensorMap &tv, const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+    if (g.D == 64 && g.RH == 64) return launch_vpass_t<64, 64>(smem, nblk, st, tp, tv, teb, tphi, a);
+    if (g.D == 64 && g.RH == 128) return launch_vpass_t<64, 128>(smem, nblk, st, tp, tv, teb, tphi, a);
+    if (g.D == 128 && g.RH == 64) return launch_vpass_t<128, 64>(smem, nblk, st, tp, tv, teb, tphi, a);
+    if (g.D == 128 && g.RH == 128) return launch_vpass_t<128, 128>(smem, nblk, st, tp, tv, teb, tphi, a);
+    return cudaErrorInvalidValue;
+}
+
 cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const void *v, void *o, float *lse,
                          float *state_out, void *workspace, cudaStream_t st) {
     Geo g = make_geo(d);
@@ -1015,6 +1065,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
         long long total = (long long)g.RP * kC + (long long)g.SP * g.R2 + (fseg ? (long long)g.RP * g.Lseg : 0);
         int blocks = (int)((total + 255) / 256);
         if (blocks > 2048) blocks = 2048;
+        ProfScope ps(BLA_K_TABLES_BF16, st);
         k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, d.T, d.w, eb, phi, fseg);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
@@ -1059,30 +1110,30 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
         const int smem = smem_request(kPreStages * stage_bytes + 256 + 1024, pow2_cols(2 * g.NB * g.D));
         if ((e = cudaFuncSetAttribute(k_prepass, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
             return e;
-        k_prepass<<<nblk, kThreads, smem, st>>>(tk, tv, tf, a);
+        {
+            ProfScope ps(BLA_K_PREPASS, st);
+            k_prepass<<<nblk, kThreads, smem, st>>>(tk, tv, tf, a);
+        }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         long long tot = (long long)g.BH * 2 * g.M * g.D;
         int blocks = (int)((tot + 255) / 256);
         if (blocks > 4096) blocks = 4096;
-        k_scan<<<blocks, 256, 0, st>>>(a);
+        {
+            ProfScope ps(BLA_K_SCAN, st);
+            k_scan<<<blocks, 256, 0, st>>>(a);
+        }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     if (!make_tmap_bf16(&tk, k, 3, dq, sq, bq) || !make_tmap_bf16(&tv, v, 3, dq, sq, bq)) return cudaErrorInvalidValue;
     {
         KLayout kl = k_layout(g);
         const int smem = smem_request(kl.total, pow2_cols(g.NB * g.D + 128 + g.RH));
-        if ((e = cudaFuncSetAttribute(k_kpass, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
-            return e;
-        k_kpass<<<nblk, kThreads, smem, st>>>(tq, tk, teb, tphi, a);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if ((e = launch_kpass(g, smem, nblk, st, tq, tk, teb, tphi, a)) != cudaSuccess) return e;
     }
     {
         VLayout vl = v_layout(g);
         const int smem = smem_request(vl.total, pow2_cols(g.NB * g.D + 256));
-        if ((e = cudaFuncSetAttribute(k_vpass, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
-            return e;
-        k_vpass<<<nblk, kThreads, smem, st>>>(tp, tv, teb, tphi, a);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+        if ((e = launch_vpass(g, smem, nblk, st, tp, tv, teb, tphi, a)) != cudaSuccess) return e;
     }
     return cudaSuccess;
 }

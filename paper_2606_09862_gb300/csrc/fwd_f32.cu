@@ -188,6 +188,7 @@ cudaError_t launch_forward_f32(const OpDims &d, int C, const Tables &t, const fl
     cudaError_t e = cudaFuncSetAttribute(k_forward_f32, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     float *state = state_out ? state_out : scratch;
+    ProfScope ps(BLA_K_FWD_F32, st);
     k_forward_f32<<<d.B * d.H, 256, smem, st>>>(d, C, t, q, k, v, o, lse, state);
     return cudaGetLastError();
 }

@@ -71,6 +71,7 @@ cudaError_t tables_build(const OpDims &d, const Tables &t, cudaStream_t st) {
     int threads = 256;
     int blocks = (int)((total + threads - 1) / threads);
     if (blocks > 1024) blocks = 1024;
+    ProfScope ps(BLA_K_TABLES, st);
     k_tables<<<blocks, threads, 0, st>>>(d.M, d.S, d.T, d.w, t.C, t.phi, t.delta, t.rot1, t.erel);
     return cudaGetLastError();
 }
