@@ -33,6 +33,12 @@ using bf16 = __nv_bfloat16;
 constexpr int kC = 128;          // tokens per chunk (MMA M)
 constexpr int kThreads = 192;
 constexpr int kEpiThreads = 128;
+constexpr int kEpiWarps = 4;   // epilogue hand-off barriers count one arrival per epilogue warp
+// The K and V passes run 10 warps: 0-7 drain TMEM as two warpgroups that split every row's
+// columns in halves (warp w reads TMEM lanes 32(w%4)..), 8 issues TMA, 9 issues the MMAs.
+constexpr int kPassThreads = 320;
+constexpr int kPassEpiWarps = 8;
+
 
 // ------------------------------------------------------------------ geometry
 
@@ -167,6 +173,20 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t &phase, Ctl *ct
     return ok;
 }
 
+// Epilogue hand-off: every thread has finished its TMEM reads/writes and shared-memory
+// stores (fenced by the caller); the warp converges and its lane 0 arrives once.
+__device__ __forceinline__ void epi_arrive(uint64_t *bar) {
+    __syncwarp();
+    if ((threadIdx.x & 31) == 0) tc::mbar_arrive(bar);
+}
+
+// Bounded barrier among the epilogue warps (an mbarrier counting one arrival per warp):
+// every epilogue thread arrives through its warp and waits for the phase to complete.
+__device__ __forceinline__ bool epi_sync(uint64_t *bar, uint32_t &phase, Ctl *ctl, int *err) {
+    epi_arrive(bar);
+    return wait_bar(bar, phase, ctl, err);
+}
+
 __device__ __forceinline__ uint32_t tmem_addr(uint32_t base, int lane_base, int col) {
     return base + ((uint32_t)lane_base << 16) + (uint32_t)col;
 }
@@ -205,7 +225,7 @@ __device__ __forceinline__ uint64_t mnmaj_desc(const uint8_t *tile, int krows, i
 // Executed by the 128 epilogue threads; `row` is this thread's lane = local state row.
 template <int D>
 __device__ __forceinline__ void state_pass(uint32_t tbase, int col0, int row, bool rotate, float c, float s,
-                                           bool write_back, uint8_t *wtile, int RH, float *gout) {
+                                           bool write_back, uint8_t *wtile, int RH, float *gout, int ccol = 0) {
     const int lane_base = (row >> 5) << 5;
     const uint32_t addr = tmem_addr(tbase, lane_base, col0);
     float v[D];
@@ -222,24 +242,26 @@ __device__ __forceinline__ void state_pass(uint32_t tbase, int col0, int row, bo
     }
     if (wtile && row < RH) {
 #pragma unroll
-        for (int g = 0; g < D; g += 32) st_row32_bf16(wtile, RH, row, g, v + g);
+        for (int g = 0; g < D; g += 32) st_row32_bf16(wtile, RH, row, ccol + g, v + g);
     }
     if (gout) {
 #pragma unroll
-        for (int i = 0; i < D; i += 4) *reinterpret_cast<float4 *>(gout + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
+        for (int i = 0; i < D; i += 4)
+            *reinterpret_cast<float4 *>(gout + ccol + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
     }
 }
 
 // Load 128 rows x D fp32 (global, row stride D) into a TMEM state block; rows at or beyond
 // `live_rows` (padding beyond 2M) and a NULL source give zeros.
 template <int D>
-__device__ __forceinline__ void state_init(uint32_t tbase, int col0, int row, const float *src, int live_rows) {
+__device__ __forceinline__ void state_init(uint32_t tbase, int col0, int row, const float *src, int live_rows,
+                                           int stride = D) {
     const int lane_base = (row >> 5) << 5;
     float v[D];
 #pragma unroll
     for (int i = 0; i < D; i += 4) {
         float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (src && row < live_rows) t = *reinterpret_cast<const float4 *>(src + (size_t)row * D + i);
+        if (src && row < live_rows) t = *reinterpret_cast<const float4 *>(src + (size_t)row * stride + i);
         v[i] = t.x; v[i + 1] = t.y; v[i + 2] = t.z; v[i + 3] = t.w;
     }
     tc::tmem_st<D>(tmem_addr(tbase, lane_base, col0), v);
@@ -398,7 +420,7 @@ __host__ __device__ inline KLayout k_layout(const Geo &g) {
     l.y = off;   off += (size_t)kC * g.RH * 2;
     l.eb = off;  off += (size_t)128 * kC * 2;
     l.phi = off; off += (size_t)g.SP * g.RH * 2;
-    l.bars = off; off += 1024;
+    l.bars = off; off += 2048;   // barriers, TMEM slot, control, slot lags, softmax partials
     l.total = off + 1024;   // slack for 1024-byte alignment of the dynamic smem base
     return l;
 }
@@ -408,13 +430,15 @@ __host__ __device__ inline KLayout k_layout(const Geo &g) {
 enum KBar {
     KB_QK_FULL, KB_QK_FREE, KB_EB_FULL, KB_EB_FREE, KB_PHI_FULL, KB_PHI_FREE,
     KB_ACC_FULL_A, KB_ACC_FULL_B, KB_ACC_FREE_A, KB_ACC_FREE_B,
-    KB_P_READY, KB_W_READY, KB_W_FREE, KB_STATE_DONE, KB_STATE_DONE1, KB_Y_READY, KB_Y_FREE, KB_EXIT, KB_COUNT
+    KB_P_READY, KB_W_READY, KB_W_FREE, KB_STATE_DONE, KB_STATE_DONE1, KB_Y_READY, KB_Y_FREE, KB_EPI_SYNC, KB_EXIT,
+    KB_COUNT
 };
 
 template <int D, int RH, int S>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kPassThreads, 1)
     k_kpass(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-            const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi, Args a) {
+            const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi,
+            const __grid_constant__ CUtensorMap tm_p, Args a) {
     const Geo &g = a.g;
     const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
     const int c_begin = seg * g.cps, c_end = min(g.nchunks, c_begin + g.cps);
@@ -436,8 +460,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < KB_COUNT; ++i) {
             const bool epi = i == KB_P_READY || i == KB_W_READY || i == KB_Y_READY || i == KB_ACC_FREE_A ||
-                             i == KB_ACC_FREE_B;
-            tc::mbar_init(&bar[i], epi ? kEpiThreads : 1);
+                             i == KB_ACC_FREE_B || i == KB_EPI_SYNC;
+            tc::mbar_init(&bar[i], epi ? kPassEpiWarps : 1);
         }
         ctl->abort = 0;
         ctl->kernel = 2;
@@ -445,13 +469,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc::fence_barrier_init();
     }
     for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
-    if (warp == 5) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
+    if (warp == 9) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
 
-    if (warp == 4) {
+    if (warp == 8) {
         if (lane == 0) {
             tc::tma_prefetch_desc(&tm_q); tc::tma_prefetch_desc(&tm_k);
             tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
@@ -478,7 +502,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
             }
         }
-    } else if (warp == 5) {
+    } else if (warp == 9) {
         if (lane == 0) {
             uint32_t ph_qk = 0, ph_eb = 0, ph_phi = 0, ph_freeA = 0, ph_freeB = 0, ph_p = 0, ph_w = 0, ph_y = 0;
             const uint32_t id_P = tc::idesc_bf16(128, kC, false, false);
@@ -547,25 +571,33 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mbar_wait(&bar[KB_EXIT], ph_exit);
         }
     } else {
-        // ---------------- epilogue warps 0-3: thread = TMEM lane = token row / state row
-        const int row = threadIdx.x, lane_base = warp * 32;
-        uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0;
+        // ---------------- epilogue warps 0-7: thread = TMEM lane = token row / state row;
+        // warpgroup wg handles columns [wg*N/2, (wg+1)*N/2) of every N-column drain
+        const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
+        float *red = reinterpret_cast<float *>(sdelta + 128);   // [2][128] softmax partials
+        uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0, ph_sync = 0;
         uint32_t ph_state[2] = {0, 0};
         const int M = g.M;
         const float *erel = a.erel;
-        // phase constants of this thread, fixed for the whole CTA: the per-mode step e^{i w t}
-        // of token row t, the start phase of each mode half, and e^{i m w C} of its state row
+        constexpr int XH = RH / 2;        // X columns per warpgroup (XH/2 modes)
+        constexpr int DH = D / 2;         // state columns per warpgroup
+        constexpr int SH = S >= 64 ? S / 2 : S;   // slot columns per warpgroup (S = 32: warpgroup 0 only)
+        // phase constants of this thread, fixed for the whole CTA: e^{i 2 w t} (two interleaved
+        // mode chains), the start phases of its mode range in each half, e^{i m w C} of its state row
         const float2 e1 = phase(erel, M, row, 1);
-        float2 ph0[2], rotC[2];
+        const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
+        float2 ph0[2], ph1[2], rotC[2];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            ph0[h] = (h < NH) ? phase(erel, M, row, h * (RH / 2)) : make_float2(1.f, 0.f);
+            const int m0 = h * (RH / 2) + wg * (XH / 2);
+            ph0[h] = (h < NH) ? phase(erel, M, row, m0) : make_float2(1.f, 0.f);
+            ph1[h] = (h < NH) ? phase(erel, M, row, m0 + 1) : make_float2(1.f, 0.f);
             const int m = (h * 128 + row) >> 1;
             rotC[h] = (h < g.NB && m < M) ? phase(erel, M, kC, m) : make_float2(1.f, 0.f);
         }
         for (int b = 0; b < g.NB; ++b) {
             const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
-            state_init<D>(tb, b * D, row, src, g.R2 - b * 128);
+            state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
         }
         bool bad = false;
         for (int c = c_begin; c < c_end && !bad; ++c) {
@@ -577,27 +609,27 @@ __global__ void __launch_bounds__(kThreads, 1)
                 // state carried into this chunk, written back, and copied to bf16 for the MMA.
                 if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                state_pass<D>(tb, h * D, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr);
+                state_pass<DH>(tb, h * D + wg * DH, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr, wg * DH);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
-                tc::mbar_arrive(&bar[KB_W_READY]);
+                epi_arrive(&bar[KB_W_READY]);
                 if (h == 0) {
                     // P drain: causal mask u <= t, bf16 -> sP
                     if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
-                    float v[kC];
-                    tc::tmem_ld<kC>(tmem_addr(tb, lane_base, colA), v);
+                    float v[64];
+                    tc::tmem_ld<64>(tmem_addr(tb, lane_base, colA + wg * 64), v);
 #pragma unroll
-                    for (int i = 0; i < kC; ++i)
-                        if (i > row) v[i] = 0.f;
+                    for (int i = 0; i < 64; ++i)
+                        if (wg * 64 + i > row) v[i] = 0.f;
 #pragma unroll
-                    for (int g0 = 0; g0 < kC; g0 += 32) st_row32_bf16(sP, kC, row, g0, v + g0);
+                    for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(sP, kC, row, wg * 64 + g0, v + g0);
                     tc::fence_proxy_async_smem();
                     tc::tc_fence_before();
-                    tc::mbar_arrive(&bar[KB_P_READY]);
-                    tc::mbar_arrive(&bar[KB_ACC_FREE_A]);
+                    epi_arrive(&bar[KB_P_READY]);
+                    epi_arrive(&bar[KB_ACC_FREE_A]);
                 }
-                // X_h drain -> Y_h = e^{i m w t} X_h (t = row), modes advanced by e1
+                // X_h drain -> Y_h = e^{i m w t} X_h (t = row), two interleaved mode chains
                 const bool inB = (h & 1) == 0;
                 if (!wait_bar(&bar[inB ? KB_ACC_FULL_B : KB_ACC_FULL_A], inB ? ph_fullB : ph_fullA, ctl, a.err)) {
                     bad = true;
@@ -605,30 +637,43 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 if (!wait_bar(&bar[KB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
                 if (h > 0 && !wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
+                if (h == 0) {
+                    // the previous chunk's probabilities left the Y tile through a bulk store
+                    if (threadIdx.x == 0) tc::bulk_wait_read0();
+                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                }
                 tc::tc_fence_after();
                 {
-                    float v[RH];
-                    tc::tmem_ld<RH>(tmem_addr(tb, lane_base, inB ? colB : colA), v);
-                    float cc = ph0[h].x, ss = ph0[h].y;
+                    float v[XH];
+                    tc::tmem_ld<XH>(tmem_addr(tb, lane_base, (inB ? colB : colA) + wg * XH), v);
+                    float ca = ph0[h].x, sa = ph0[h].y, cb = ph1[h].x, sb = ph1[h].y;
 #pragma unroll
-                    for (int i = 0; i < RH; i += 2) {
-                        const float xr = v[i], xi = v[i + 1];
-                        v[i] = cc * xr - ss * xi;
-                        v[i + 1] = ss * xr + cc * xi;
-                        const float nc = cc * e1.x - ss * e1.y, ns = ss * e1.x + cc * e1.y;
-                        cc = nc;
-                        ss = ns;
+                    for (int i = 0; i < XH; i += 4) {
+                        float xr = v[i], xi = v[i + 1];
+                        v[i] = ca * xr - sa * xi;
+                        v[i + 1] = sa * xr + ca * xi;
+                        xr = v[i + 2];
+                        xi = v[i + 3];
+                        v[i + 2] = cb * xr - sb * xi;
+                        v[i + 3] = sb * xr + cb * xi;
+                        float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
+                        ca = t1;
+                        sa = t2;
+                        t1 = cb * e2.x - sb * e2.y;
+                        t2 = sb * e2.x + cb * e2.y;
+                        cb = t1;
+                        sb = t2;
                     }
 #pragma unroll
-                    for (int g0 = 0; g0 < RH; g0 += 32) st_row32_bf16(sY, kC, row, g0, v + g0);
+                    for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sY, kC, row, wg * XH + g0, v + g0);
                 }
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
-                tc::mbar_arrive(&bar[KB_Y_READY]);
-                tc::mbar_arrive(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
+                epi_arrive(&bar[KB_Y_READY]);
+                epi_arrive(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
             }
             if (bad) break;
-            // masked softmax over the S slots, one TMEM pass
+            // masked softmax over the S slots; the two warpgroups combine row max and sum through smem
             const bool sInB = NH == 2;
             if (!wait_bar(&bar[sInB ? KB_ACC_FULL_B : KB_ACC_FULL_A], sInB ? ph_fullB : ph_fullA, ctl, a.err)) {
                 bad = true;
@@ -637,36 +682,61 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
             tc::tc_fence_after();
             {
-                float v[S];
-                tc::tmem_ld<S>(tmem_addr(tb, lane_base, sInB ? colB : colA), v);
-                tc::tc_fence_before();
-                tc::mbar_arrive(&bar[sInB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
+                const bool active = wg == 0 || S >= 64;
+                const int j0 = (S >= 64) ? wg * SH : 0;
                 const int t = t0 + row;
-                float mx = -INFINITY;
+                float v[SH];
+                if (active) tc::tmem_ld<SH>(tmem_addr(tb, lane_base, (sInB ? colB : colA) + j0), v);
+                tc::tc_fence_before();
+                epi_arrive(&bar[sInB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
+                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                if (active) {
 #pragma unroll
-                for (int j = 0; j < S; ++j) {
-                    v[j] = (t >= sdelta[j]) ? v[j] * a.scale : -INFINITY;
-                    mx = fmaxf(mx, v[j]);
+                    for (int j = 0; j < SH; ++j) {
+                        v[j] = (t >= sdelta[j0 + j]) ? v[j] * a.scale : -INFINITY;
+                        m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                    }
                 }
-                float sum = 0.f;
+                float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+                if (S >= 64) {
+                    red[wg * 128 + row] = mx;
+                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                    mx = fmaxf(red[row], red[128 + row]);
+                }
+                float s4[4] = {0.f, 0.f, 0.f, 0.f};
+                if (active) {
 #pragma unroll
-                for (int j = 0; j < S; ++j) {
-                    v[j] = (v[j] == -INFINITY) ? 0.f : __expf(v[j] - mx);
-                    sum += v[j];
+                    for (int j = 0; j < SH; ++j) {
+                        v[j] = (v[j] == -INFINITY) ? 0.f : __expf(v[j] - mx);
+                        s4[j & 3] += v[j];
+                    }
+                }
+                float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+                if (S >= 64) {
+                    // every max is read before the sums overwrite it
+                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                    red[wg * 128 + row] = sum;
+                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                    sum = red[row] + red[128 + row];
                 }
                 const float inv = 1.f / sum;
-                if (row < n) {
-                    bf16 *prow = a.pbuf + ((size_t)bh * g.L + t) * SP;
+                if (active) {
 #pragma unroll
-                    for (int j = 0; j < S; j += 8) {
-                        uint4 pk = make_uint4(tc::pack_bf16x2(v[j] * inv, v[j + 1] * inv),
-                                              tc::pack_bf16x2(v[j + 2] * inv, v[j + 3] * inv),
-                                              tc::pack_bf16x2(v[j + 4] * inv, v[j + 5] * inv),
-                                              tc::pack_bf16x2(v[j + 6] * inv, v[j + 7] * inv));
-                        *reinterpret_cast<uint4 *>(prow + j) = pk;
-                    }
-                    for (int j = S; j < SP; j += 8) *reinterpret_cast<uint4 *>(prow + j) = make_uint4(0, 0, 0, 0);
-                    if (a.lse) a.lse[(size_t)bh * g.L + t] = mx + logf(sum);
+                    for (int j = 0; j < SH; ++j) v[j] *= inv;
+#pragma unroll
+                    for (int g0 = 0; g0 < SH; g0 += 32) st_row32_bf16(sY, kC, row, j0 + g0, v + g0);
+                } else if (SP > S) {
+                    float z[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) z[i] = 0.f;
+                    for (int g0 = S; g0 < SP; g0 += 32) st_row32_bf16(sY, kC, row, g0, z);
+                }
+                if (wg == 0 && row < n && a.lse) a.lse[(size_t)bh * g.L + t] = mx + logf(sum);
+                tc::fence_proxy_async_smem();
+                if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                if (threadIdx.x == 0) {
+                    for (int kb = 0; kb < SP / 64; ++kb) tc::tma_store_3d(&tm_p, sY + kb * kC * 128, kb * 64, t0, bh);
+                    tc::bulk_commit();
                 }
             }
         }
@@ -681,14 +751,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int r = b * 128 + row, m = r >> 1;
                     float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + r) * D : nullptr;
                     const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
-                    state_pass<D>(tb, b * D, row, true, f.x, f.y, false, nullptr, 0, dst);
+                    state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
                 }
             }
         }
+        if (threadIdx.x == 0) tc::bulk_wait0();
     }
     tc::tc_fence_before();
     __syncthreads();
-    if (warp == 5) {
+    if (warp == 9) {
         tc::tc_fence_after();
         tc::tmem_dealloc(tb, ncols);
     }
@@ -722,7 +793,7 @@ enum VBar {
 };
 
 template <int D, int RH>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kPassThreads, 1)
     k_vpass(const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_v,
             const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi, Args a) {
     const Geo &g = a.g;
@@ -746,20 +817,20 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < VB_COUNT; ++i) {
             const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_G_READY || i == VB_W_READY;
-            tc::mbar_init(&bar[i], epi ? kEpiThreads : 1);
+            tc::mbar_init(&bar[i], epi ? kPassEpiWarps : 1);
         }
         ctl->abort = 0;
         ctl->kernel = 3;
         ctl->bar0 = bar;
         tc::fence_barrier_init();
     }
-    if (warp == 5) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
+    if (warp == 9) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
 
-    if (warp == 4) {
+    if (warp == 8) {
         if (lane == 0) {
             tc::tma_prefetch_desc(&tm_p); tc::tma_prefetch_desc(&tm_v);
             tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
@@ -791,7 +862,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     }
             }
         }
-    } else if (warp == 5) {
+    } else if (warp == 9) {
         if (lane == 0) {
             uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0, ph_w = 0;
             const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
@@ -851,22 +922,26 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc::mbar_wait(&bar[VB_EXIT], ph_exit);
         }
     } else {
-        const int row = threadIdx.x, lane_base = warp * 32;
+        const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
         const int M = g.M;
         const float *erel = a.erel;
+        constexpr int XH = RH / 2, DH = D / 2;
         uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0;
         uint32_t ph_state[2] = {0, 0};
         const float2 e1 = phase(erel, M, row, 1);
-        float2 ph0[2], rotC[2];
+        const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
+        float2 ph0[2], ph1[2], rotC[2];
 #pragma unroll
         for (int h = 0; h < 2; ++h) {
-            ph0[h] = (h < NH) ? phase(erel, M, row, h * (RH / 2)) : make_float2(1.f, 0.f);
+            const int m0 = h * (RH / 2) + wg * (XH / 2);
+            ph0[h] = (h < NH) ? phase(erel, M, row, m0) : make_float2(1.f, 0.f);
+            ph1[h] = (h < NH) ? phase(erel, M, row, m0 + 1) : make_float2(1.f, 0.f);
             const int m = (h * 128 + row) >> 1;
             rotC[h] = (h < g.NB && m < M) ? phase(erel, M, kC, m) : make_float2(1.f, 0.f);
         }
         for (int b = 0; b < g.NB; ++b) {
             const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
-            state_init<D>(tb, b * D, row, src, g.R2 - b * 128);
+            state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
         }
         bool bad = false;
         for (int c = c_begin; c < c_end && !bad; ++c) {
@@ -877,51 +952,59 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int h = 0; h < NH; ++h) {
                 if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                float v[RH];
-                tc::tmem_ld<RH>(tmem_addr(tb, lane_base, colU), v);
-                float cc = ph0[h].x, ss = ph0[h].y;
+                float v[XH];
+                tc::tmem_ld<XH>(tmem_addr(tb, lane_base, colU + wg * XH), v);
+                float ca = ph0[h].x, sa = ph0[h].y, cb = ph1[h].x, sb = ph1[h].y;
 #pragma unroll
-                for (int i = 0; i < RH; i += 2) {
-                    const float uc = v[i], us = v[i + 1];
-                    v[i] = cc * uc + ss * us;
-                    v[i + 1] = cc * us - ss * uc;
-                    const float nc = cc * e1.x - ss * e1.y, ns = ss * e1.x + cc * e1.y;
-                    cc = nc;
-                    ss = ns;
+                for (int i = 0; i < XH; i += 4) {
+                    float uc = v[i], us = v[i + 1];
+                    v[i] = ca * uc + sa * us;
+                    v[i + 1] = ca * us - sa * uc;
+                    uc = v[i + 2];
+                    us = v[i + 3];
+                    v[i + 2] = cb * uc + sb * us;
+                    v[i + 3] = cb * us - sb * uc;
+                    float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
+                    ca = t1;
+                    sa = t2;
+                    t1 = cb * e2.x - sb * e2.y;
+                    t2 = sb * e2.x + cb * e2.y;
+                    cb = t1;
+                    sb = t2;
                 }
 #pragma unroll
-                for (int g0 = 0; g0 < RH; g0 += 32) st_row32_bf16(sA + h * a_tile, kC, row, g0, v + g0);
+                for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sA + h * a_tile, kC, row, wg * XH + g0, v + g0);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
-                tc::mbar_arrive(&bar[VB_A_READY]);
-                tc::mbar_arrive(&bar[VB_U_FREE]);
+                epi_arrive(&bar[VB_A_READY]);
+                epi_arrive(&bar[VB_U_FREE]);
             }
             if (bad) break;
             // phase 2: G drain -> causal mask -> bf16 over p's tile
             if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
             tc::tc_fence_after();
             {
-                float v[kC];
-                tc::tmem_ld<kC>(tmem_addr(tb, lane_base, colG), v);
+                float v[64];
+                tc::tmem_ld<64>(tmem_addr(tb, lane_base, colG + wg * 64), v);
 #pragma unroll
-                for (int i = 0; i < kC; ++i)
-                    if (i > row) v[i] = 0.f;
+                for (int i = 0; i < 64; ++i)
+                    if (wg * 64 + i > row) v[i] = 0.f;
 #pragma unroll
-                for (int g0 = 0; g0 < kC; g0 += 32) st_row32_bf16(sPG, kC, row, g0, v + g0);
+                for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(sPG, kC, row, wg * 64 + g0, v + g0);
             }
             tc::fence_proxy_async_smem();
             tc::tc_fence_before();
-            tc::mbar_arrive(&bar[VB_G_READY]);
-            tc::mbar_arrive(&bar[VB_G_FREE]);
+            epi_arrive(&bar[VB_G_READY]);
+            epi_arrive(&bar[VB_G_FREE]);
             // phase 3: W_h (the V state read before this chunk's update)
             for (int h = 0; h < NH; ++h) {
                 if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
                 if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                state_pass<D>(tb, h * D, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr);
+                state_pass<DH>(tb, h * D + wg * DH, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr, wg * DH);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
-                tc::mbar_arrive(&bar[VB_W_READY]);
+                epi_arrive(&bar[VB_W_READY]);
             }
             if (bad) break;
             if (!wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) break;
@@ -929,14 +1012,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!wait_bar(&bar[VB_O_FULL], ph_o, ctl, a.err)) break;
             tc::tc_fence_after();
             {
-                float v[D];
-                tc::tmem_ld<D>(tmem_addr(tb, lane_base, colU), v);
+                float v[DH];
+                tc::tmem_ld<DH>(tmem_addr(tb, lane_base, colU + wg * DH), v);
                 tc::tc_fence_before();
-                tc::mbar_arrive(&bar[VB_U_FREE]);
+                epi_arrive(&bar[VB_U_FREE]);
                 if (row < n) {
-                    bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D;
+                    bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D + wg * DH;
 #pragma unroll
-                    for (int j = 0; j < D; j += 8) {
+                    for (int j = 0; j < DH; j += 8) {
                         uint4 pk = make_uint4(tc::pack_bf16x2(v[j], v[j + 1]), tc::pack_bf16x2(v[j + 2], v[j + 3]),
                                               tc::pack_bf16x2(v[j + 4], v[j + 5]), tc::pack_bf16x2(v[j + 6], v[j + 7]));
                         *reinterpret_cast<uint4 *>(orow + j) = pk;
@@ -954,14 +1037,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                     const int r = b * 128 + row, m = r >> 1;
                     float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + g.R2 + r) * D : nullptr;
                     const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
-                    state_pass<D>(tb, b * D, row, true, f.x, f.y, false, nullptr, 0, dst);
+                    state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
                 }
             }
         }
     }
     tc::tc_fence_before();
     __syncthreads();
-    if (warp == 5) {
+    if (warp == 9) {
         tc::tc_fence_after();
         tc::tmem_dealloc(tb, ncols);
     }
@@ -976,6 +1059,7 @@ const char *fwd_bf16_unsupported(const OpDims &d) {
     if (d.dk != 64 && d.dk != 128) return "d_k must be 64 or 128";
     if (d.R2 != 64 && d.R2 != 128 && d.R2 != 256) return "2M must be 64, 128 or 256";
     if (d.S != 32 && d.S != 64 && d.S != 128) return "S must be 32, 64 or 128";
+    if (d.S > (d.R2 < 64 ? 64 : d.R2)) return "S must not exceed max(2M, 64)";
     return nullptr;
 }
 
@@ -998,31 +1082,33 @@ static int pow2_cols(int n) { return n <= 32 ? 32 : n <= 64 ? 64 : n <= 128 ? 12
 
 template <int D, int RH, int S>
 static cudaError_t launch_kpass_t(int smem, int nblk, cudaStream_t st, const CUtensorMap &tq, const CUtensorMap &tk,
-                                  const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+                                  const CUtensorMap &teb, const CUtensorMap &tphi, const CUtensorMap &tp, const Args &a) {
     cudaError_t e = cudaFuncSetAttribute(k_kpass<D, RH, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_KPASS, st);
-    k_kpass<D, RH, S><<<nblk, kThreads, smem, st>>>(tq, tk, teb, tphi, a);
+    k_kpass<D, RH, S><<<nblk, kPassThreads, smem, st>>>(tq, tk, teb, tphi, tp, a);
     return cudaGetLastError();
 }
 
 template <int D, int RH>
 static cudaError_t launch_kpass_s(const Geo &g, int smem, int nblk, cudaStream_t st, const CUtensorMap &tq,
-                                  const CUtensorMap &tk, const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+                                  const CUtensorMap &tk, const CUtensorMap &teb, const CUtensorMap &tphi,
+                                  const CUtensorMap &tp, const Args &a) {
     switch (g.S) {
-    case 32: return launch_kpass_t<D, RH, 32>(smem, nblk, st, tq, tk, teb, tphi, a);
-    case 64: return launch_kpass_t<D, RH, 64>(smem, nblk, st, tq, tk, teb, tphi, a);
-    case 128: return launch_kpass_t<D, RH, 128>(smem, nblk, st, tq, tk, teb, tphi, a);
+    case 32: return launch_kpass_t<D, RH, 32>(smem, nblk, st, tq, tk, teb, tphi, tp, a);
+    case 64: return launch_kpass_t<D, RH, 64>(smem, nblk, st, tq, tk, teb, tphi, tp, a);
+    case 128: return launch_kpass_t<D, RH, 128>(smem, nblk, st, tq, tk, teb, tphi, tp, a);
     default: return cudaErrorInvalidValue;
     }
 }
 
 static cudaError_t launch_kpass(const Geo &g, int smem, int nblk, cudaStream_t st, const CUtensorMap &tq,
-                                const CUtensorMap &tk, const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
-    if (g.D == 64 && g.RH == 64) return launch_kpass_s<64, 64>(g, smem, nblk, st, tq, tk, teb, tphi, a);
-    if (g.D == 64 && g.RH == 128) return launch_kpass_s<64, 128>(g, smem, nblk, st, tq, tk, teb, tphi, a);
-    if (g.D == 128 && g.RH == 64) return launch_kpass_s<128, 64>(g, smem, nblk, st, tq, tk, teb, tphi, a);
-    if (g.D == 128 && g.RH == 128) return launch_kpass_s<128, 128>(g, smem, nblk, st, tq, tk, teb, tphi, a);
+                                const CUtensorMap &tk, const CUtensorMap &teb, const CUtensorMap &tphi,
+                                const CUtensorMap &tp, const Args &a) {
+    if (g.D == 64 && g.RH == 64) return launch_kpass_s<64, 64>(g, smem, nblk, st, tq, tk, teb, tphi, tp, a);
+    if (g.D == 64 && g.RH == 128) return launch_kpass_s<64, 128>(g, smem, nblk, st, tq, tk, teb, tphi, tp, a);
+    if (g.D == 128 && g.RH == 64) return launch_kpass_s<128, 64>(g, smem, nblk, st, tq, tk, teb, tphi, tp, a);
+    if (g.D == 128 && g.RH == 128) return launch_kpass_s<128, 128>(g, smem, nblk, st, tq, tk, teb, tphi, tp, a);
     return cudaErrorInvalidValue;
 }
 
@@ -1032,7 +1118,7 @@ static cudaError_t launch_vpass_t(int smem, int nblk, cudaStream_t st, const CUt
     cudaError_t e = cudaFuncSetAttribute(k_vpass<D, RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_VPASS, st);
-    k_vpass<D, RH><<<nblk, kThreads, smem, st>>>(tp, tv, teb, tphi, a);
+    k_vpass<D, RH><<<nblk, kPassThreads, smem, st>>>(tp, tv, teb, tphi, a);
     return cudaGetLastError();
 }
 
@@ -1128,7 +1214,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     {
         KLayout kl = k_layout(g);
         const int smem = smem_request(kl.total, pow2_cols(g.NB * g.D + 128 + g.RH));
-        if ((e = launch_kpass(g, smem, nblk, st, tq, tk, teb, tphi, a)) != cudaSuccess) return e;
+        if ((e = launch_kpass(g, smem, nblk, st, tq, tk, teb, tphi, tp, a)) != cudaSuccess) return e;
     }
     {
         VLayout vl = v_layout(g);
