@@ -117,6 +117,23 @@ bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, co
                            void *stream);
 
 /*
+ * bla_decode_step for callers that may not allocate device memory (the paper has no
+ * counterpart; this is a deployment convenience).  Same arguments and results as
+ * bla_decode_step, without the workspace: the step's tables live in a fixed 512 KiB
+ * device array owned by the library (reserved on every GPU that loads it, until exit).
+ * Meant for callers that run within a fixed, pre-reserved memory budget or must not
+ * call the allocator mid-step (cudaMalloc can synchronise the device).
+ *   - Parameters whose tables exceed the array are rejected with BLA_ERR_UNSUPPORTED
+ *     before any launch.
+ *   - The array's device address is looked up on the first call made on each device;
+ *     make that first call before any stream capture.
+ *   - All calls share the array (it keeps the last call's tables, rewritten in full by
+ *     every call): calls that overlap on the GPU race and must be ordered by the caller.
+ */
+bla_status bla_decode_step_noalloc(const bla_params *p, long long pos, const void *q, const void *k,
+                                   const void *v, float *state, void *o, void *stream);
+
+/*
  * Backward pass of bla_forward_chunked: given dout = dL/do, writes dq, dk, dv
  * (same shapes and dtype as q, k, v).  o and lse are the forward's outputs.
  * The vector-Jacobian product of the operator defined by Eqs. (recurrence),

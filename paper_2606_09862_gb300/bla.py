@@ -20,7 +20,7 @@ BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE = 0, 1, 2
 
 EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
             "bla_device_error", "bla_status_string", "bla_last_error_string", "bla_kernel_launches",
-            "bla_profile_enable", "bla_profile_collect")
+            "bla_profile_enable", "bla_profile_collect", "bla_decode_step_noalloc")
 
 # bla_kernel_id
 KERNELS = ("tables", "tables_bf16", "prepass", "scan", "kpass", "vpass", "fwd_f32", "decode", "bwd")
@@ -59,6 +59,8 @@ def load():
     lib.bla_forward_chunked.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_decode_step.restype = ctypes.c_int
     lib.bla_decode_step.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_decode_step_noalloc.restype = ctypes.c_int
+    lib.bla_decode_step_noalloc.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp]
     lib.bla_backward.restype = ctypes.c_int
     lib.bla_backward.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_device_error.restype = ctypes.c_int
@@ -155,6 +157,19 @@ def bla_decode_step(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, wor
     ws, n = _workspace(p, BLA_WS_DECODE, q.device, workspace)
     _check(load().bla_decode_step(ctypes.byref(p), int(pos), _ptr(q), _ptr(k), _ptr(v), _ptr(state), _ptr(o),
                                   _ptr(ws), n, _stream(stream)))
+    return o
+
+
+def bla_decode_step_noalloc(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, out=None, stream=None):
+    """bla_decode_step without a workspace: the library's own fixed device scratch holds the
+    tables, so the call allocates nothing (the output is allocated here unless `out` is given)."""
+    _need_cuda(q, k, v, state)
+    B, H, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, 1, dk, dv, M, S, window, omega, 0, scale, q.dtype)
+    o = out if out is not None else torch.empty((B, H, dv), dtype=q.dtype, device=q.device)
+    _check(load().bla_decode_step_noalloc(ctypes.byref(p), int(pos), _ptr(q), _ptr(k), _ptr(v), _ptr(state),
+                                          _ptr(o), _stream(stream)))
     return o
 
 

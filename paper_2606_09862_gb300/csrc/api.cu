@@ -70,8 +70,14 @@ int *device_error_word() {
 }
 
 namespace {
-
 thread_local char t_last_error[512] = "";
+}  // namespace
+
+void set_last_error(const char *msg) {
+    snprintf(t_last_error, sizeof(t_last_error), "%s", msg ? msg : "");
+}
+
+namespace {
 
 bla_status fail(bla_status s, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
 bla_status fail(bla_status s, const char *fmt, ...) {

@@ -60,6 +60,9 @@ template <> __device__ __forceinline__ void store_elem<__nv_bfloat16>(__nv_bfloa
     p[i] = __float2bfloat16_rn(x);
 }
 
+// Replace the calling thread's bla_last_error_string() text.
+void set_last_error(const char *msg);
+
 // Device address of the library's error word (a __device__ int of this module, one per
 // device); kernels with bounded waits receive it as an argument.  NULL on failure.
 int *device_error_word();
