@@ -9,6 +9,7 @@
 #include <vector>
 
 #include "common.cuh"
+#include "bwd.cuh"
 #include "fwd_bf16.cuh"
 
 namespace bla {
@@ -171,7 +172,7 @@ size_t bla_workspace_bytes(const bla_params *p, int which) {
     switch (which) {
     case BLA_WS_FORWARD: return ws_forward(p, d);
     case BLA_WS_DECODE: return ws_decode(d);
-    case BLA_WS_BACKWARD: return fwd_bf16_workspace_bytes(d);
+    case BLA_WS_BACKWARD: return bwd_workspace_bytes(d);
     default: return 0;
     }
 }
@@ -241,9 +242,18 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
     OpDims d;
     bla_status s = check_params(p, &d);
     if (s != BLA_OK) return s;
-    (void)q; (void)k; (void)v; (void)o; (void)dout; (void)lse; (void)dq; (void)dk; (void)dv;
-    (void)workspace; (void)ws_bytes; (void)stream;
-    return fail(BLA_ERR_UNSUPPORTED, "backward is not implemented yet");
+    if (d.L > 0 && (!q || !k || !v || !o || !dout || !lse || !dq || !dk || !dv))
+        return fail(BLA_ERR_INVALID, "q, k, v, o, dout, lse, dq, dk and dv must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(dout) || !aligned16(lse) ||
+        !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    const char *why = bwd_unsupported(d);
+    if (why) return fail(BLA_ERR_UNSUPPORTED, "backward: %s", why);
+    size_t need = bwd_workspace_bytes(d);
+    if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
+    cudaError_t e = bwd_run(d, q, k, v, o, dout, lse, dq, dk, dv, workspace, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "backward");
+    return BLA_OK;
 }
 
 long long bla_kernel_launches(void) { return g_launches.load(); }

@@ -1054,6 +1054,15 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 
 // ================================================================== host side
 
+cudaError_t build_bf16_tables(const OpDims &d, int RP, int SP, bf16 *eb, bf16 *phi, cudaStream_t st) {
+    long long total = (long long)RP * kC + (long long)SP * d.R2;
+    int blocks = (int)((total + 255) / 256);
+    if (blocks > 2048) blocks = 2048;
+    ProfScope ps(BLA_K_TABLES_BF16, st);
+    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, d.T, d.w, eb, phi, nullptr);
+    return cudaGetLastError();
+}
+
 const char *fwd_bf16_unsupported(const OpDims &d) {
     if (d.dk != d.dv) return "d_k must equal d_v";
     if (d.dk != 64 && d.dk != 128) return "d_k must be 64 or 128";
