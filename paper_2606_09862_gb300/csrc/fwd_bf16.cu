@@ -89,8 +89,22 @@ WsLayout ws_layout(const OpDims &d, const Geo &g) {
 
 // EB [RP][C], PHI [SP][R2], FSEG [RP][Lseg] in bf16, from fp64 phases (rows beyond 2M and
 // slots beyond S are zero).
-__global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, double T, double w, bf16 *eb, bf16 *phi,
-                              bf16 *fseg) {
+// (cos, sin)(m w u): with w = 2 pi / T and an integer period tint > 0 the angle is reduced
+// exactly, 2 pi ((m u) mod T) / T, and evaluated by sincospi in fp32; otherwise in fp64.
+__device__ __forceinline__ void mode_phase(long long mu, double w, int tint, float *c, float *s) {
+    if (tint > 0) {
+        const long long kk = mu % tint;
+        sincospif(2.0f * (float)kk / (float)tint, s, c);
+    } else {
+        double sd, cd;
+        sincos((double)mu * w, &sd, &cd);
+        *s = (float)sd;
+        *c = (float)cd;
+    }
+}
+
+__global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, double T, double w, int tint, bf16 *eb,
+                              bf16 *phi, bf16 *fseg) {
     const int R2 = 2 * M;
     const long long n_eb = (long long)RP * kC, n_phi = (long long)SP * R2;
     const long long n_f = fseg ? (long long)RP * Lseg : 0;
@@ -100,13 +114,13 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, double T, 
          i += (long long)gridDim.x * blockDim.x) {
         if (i < n_eb) {
             int r = (int)(i / kC), u = (int)(i % kC), m = r >> 1;
-            double v = 0.0;
+            float v = 0.f;
             if (r < R2) {
-                double s, c;
-                sincos((double)m * w * (double)u, &s, &c);
+                float s, c;
+                mode_phase((long long)m * u, w, tint, &c, &s);
                 v = (r & 1) ? -s : c;
             }
-            eb[i] = __float2bfloat16_rn((float)v);
+            eb[i] = __float2bfloat16_rn(v);
         } else if (i < n_eb + n_phi) {
             long long e = i - n_eb;
             int j = (int)(e / R2), r = (int)(e % R2), m = r >> 1;
@@ -122,13 +136,13 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, double T, 
         } else {
             long long e = i - n_eb - n_phi;
             int r = (int)(e / Lseg), u = (int)(e % Lseg), m = r >> 1;
-            double v = 0.0;
+            float v = 0.f;
             if (r < R2) {
-                double s, c;
-                sincos((double)m * w * (double)(Lseg - u), &s, &c);
+                float s, c;
+                mode_phase((long long)m * (Lseg - u), w, tint, &c, &s);
                 v = (r & 1) ? s : c;
             }
-            fseg[e] = __float2bfloat16_rn((float)v);
+            fseg[e] = __float2bfloat16_rn(v);
         }
     }
 }
@@ -148,6 +162,7 @@ struct Args {
     bf16 *o;             // [BH][L][D]
     float *state_out;    // [BH][2][M][2][D] or null
     float *deltas_out;   // prepass output (same buffer as deltas)
+    int tint;            // integer period for exact phase reduction (0: use fp64 phases)
     int *err;
 };
 
@@ -385,9 +400,8 @@ __global__ void k_scan(Args a) {
         r /= g.M;
         const int x = (int)(r % 2);
         const int bh = (int)(r / 2);
-        double sn, cs;
-        sincos((double)m * a.w * (double)g.Lseg, &sn, &cs);
-        const float c = (float)cs, s = (float)sn;
+        float c, s;
+        mode_phase((long long)m * g.Lseg, a.w, a.tint, &c, &s);
         float re = 0.f, im = 0.f;
         for (int seg = 0; seg < g.G; ++seg) {
             const size_t base = (((size_t)bh * g.G + seg) * 2 + x) * g.RP;
@@ -420,7 +434,7 @@ __host__ __device__ inline KLayout k_layout(const Geo &g) {
     l.y = off;   off += (size_t)kC * g.RH * 2;
     l.eb = off;  off += (size_t)128 * kC * 2;
     l.phi = off; off += (size_t)g.SP * g.RH * 2;
-    l.bars = off; off += 2048;   // barriers, TMEM slot, control, slot lags, softmax partials
+    l.bars = off; off += 2048;   // barriers, TMEM slot, control, slot lags
     l.total = off + 1024;   // slack for 1024-byte alignment of the dynamic smem base
     return l;
 }
@@ -430,8 +444,8 @@ __host__ __device__ inline KLayout k_layout(const Geo &g) {
 enum KBar {
     KB_QK_FULL, KB_QK_FREE, KB_EB_FULL, KB_EB_FREE, KB_PHI_FULL, KB_PHI_FREE,
     KB_ACC_FULL_A, KB_ACC_FULL_B, KB_ACC_FREE_A, KB_ACC_FREE_B,
-    KB_P_READY, KB_W_READY, KB_W_FREE, KB_STATE_DONE, KB_STATE_DONE1, KB_Y_READY, KB_Y_FREE, KB_EPI_SYNC, KB_EXIT,
-    KB_COUNT
+    KB_P_READY, KB_W_READY, KB_W_FREE, KB_STATE_DONE, KB_STATE_DONE1, KB_Y_READY, KB_Y_FREE, KB_EPI_SYNC, KB_Y_STORED,
+    KB_EXIT, KB_COUNT
 };
 
 template <int D, int RH, int S>
@@ -574,8 +588,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         // ---------------- epilogue warps 0-7: thread = TMEM lane = token row / state row;
         // warpgroup wg handles columns [wg*N/2, (wg+1)*N/2) of every N-column drain
         const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
-        float *red = reinterpret_cast<float *>(sdelta + 128);   // [2][128] softmax partials
-        uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0, ph_sync = 0;
+        // softmax partials [2 (max, sum)][2 (warpgroup)][128 rows] live in the P tile, which is idle
+        // between the X_1 MMA (its last reader) and the next chunk's P drain
+        float *red = reinterpret_cast<float *>(sP);
+        uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0, ph_sync = 0, ph_ystored = 0;
         uint32_t ph_state[2] = {0, 0};
         const int M = g.M;
         const float *erel = a.erel;
@@ -637,10 +653,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 }
                 if (!wait_bar(&bar[KB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
                 if (h > 0 && !wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
-                if (h == 0) {
-                    // the previous chunk's probabilities left the Y tile through a bulk store
-                    if (threadIdx.x == 0) tc::bulk_wait_read0();
-                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                if (h == 0 && c > c_begin) {
+                    // the previous chunk's probabilities have left the Y tile (bulk store read done)
+                    if (!wait_bar(&bar[KB_Y_STORED], ph_ystored, ctl, a.err)) { bad = true; break; }
                 }
                 tc::tc_fence_after();
                 {
@@ -673,7 +688,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 epi_arrive(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
             }
             if (bad) break;
-            // masked softmax over the S slots; the two warpgroups combine row max and sum through smem
+            // masked softmax over the S slots; the two warpgroups exchange their (max, sum) pairs once
             const bool sInB = NH == 2;
             if (!wait_bar(&bar[sInB ? KB_ACC_FULL_B : KB_ACC_FULL_A], sInB ? ph_fullB : ph_fullA, ctl, a.err)) {
                 bad = true;
@@ -685,44 +700,53 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 const bool active = wg == 0 || S >= 64;
                 const int j0 = (S >= 64) ? wg * SH : 0;
                 const int t = t0 + row;
+                // slots are visible when t >= D_j; past the largest lag of the grid every slot is
+                const bool all_visible = t0 >= sdelta[S - 1];
+                const float sl2 = a.scale * 1.4426950408889634f;   // scores in log2 units
                 float v[SH];
                 if (active) tc::tmem_ld<SH>(tmem_addr(tb, lane_base, (sInB ? colB : colA) + j0), v);
                 tc::tc_fence_before();
                 epi_arrive(&bar[sInB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
-                float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                float mx = -INFINITY, sum = 0.f;
                 if (active) {
+                    float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                    if (all_visible) {
 #pragma unroll
-                    for (int j = 0; j < SH; ++j) {
-                        v[j] = (t >= sdelta[j0 + j]) ? v[j] * a.scale : -INFINITY;
-                        m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                        for (int j = 0; j < SH; ++j) {
+                            v[j] *= sl2;
+                            m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                        }
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < SH; ++j) {
+                            v[j] = (t >= sdelta[j0 + j]) ? v[j] * sl2 : -INFINITY;
+                            m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                        }
                     }
-                }
-                float mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-                if (S >= 64) {
-                    red[wg * 128 + row] = mx;
-                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
-                    mx = fmaxf(red[row], red[128 + row]);
-                }
-                float s4[4] = {0.f, 0.f, 0.f, 0.f};
-                if (active) {
+                    mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+                    // a half whose slots are all hidden has mx = -inf: exponentiate against 0 instead
+                    const float mref = (mx == -INFINITY) ? 0.f : mx;
+                    float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                     for (int j = 0; j < SH; ++j) {
-                        v[j] = (v[j] == -INFINITY) ? 0.f : __expf(v[j] - mx);
+                        v[j] = exp2f(v[j] - mref);          // exp2(-inf) = 0 on masked slots
                         s4[j & 3] += v[j];
                     }
+                    sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
                 }
-                float sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+                float gmx = mx, gsum = sum;
                 if (S >= 64) {
-                    // every max is read before the sums overwrite it
+                    red[wg * 128 + row] = mx;
+                    red[256 + wg * 128 + row] = sum;
                     if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
-                    red[wg * 128 + row] = sum;
-                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
-                    sum = red[row] + red[128 + row];
+                    const float m0 = red[row], m1 = red[128 + row];
+                    gmx = fmaxf(m0, m1);
+                    gsum = red[256 + row] * exp2f(m0 - gmx) + red[384 + row] * exp2f(m1 - gmx);
                 }
-                const float inv = 1.f / sum;
                 if (active) {
+                    const float f = exp2f(mx - gmx) / gsum;
 #pragma unroll
-                    for (int j = 0; j < SH; ++j) v[j] *= inv;
+                    for (int j = 0; j < SH; ++j) v[j] *= f;
 #pragma unroll
                     for (int g0 = 0; g0 < SH; g0 += 32) st_row32_bf16(sY, kC, row, j0 + g0, v + g0);
                 } else if (SP > S) {
@@ -731,12 +755,14 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     for (int i = 0; i < 32; ++i) z[i] = 0.f;
                     for (int g0 = S; g0 < SP; g0 += 32) st_row32_bf16(sY, kC, row, g0, z);
                 }
-                if (wg == 0 && row < n && a.lse) a.lse[(size_t)bh * g.L + t] = mx + logf(sum);
+                if (wg == 0 && row < n && a.lse) a.lse[(size_t)bh * g.L + t] = (gmx + log2f(gsum)) * 0.6931471805599453f;
                 tc::fence_proxy_async_smem();
                 if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
                 if (threadIdx.x == 0) {
                     for (int kb = 0; kb < SP / 64; ++kb) tc::tma_store_3d(&tm_p, sY + kb * kC * 128, kb * 64, t0, bh);
                     tc::bulk_commit();
+                    tc::bulk_wait_read0();
+                    tc::mbar_arrive(&bar[KB_Y_STORED]);
                 }
             }
         }
@@ -789,13 +815,14 @@ __host__ __device__ inline VLayout v_layout(const Geo &g) {
 enum VBar {
     VB_PV_FULL, VB_PV_FREE, VB_EB_FULL, VB_EB_FREE, VB_PHI_FULL, VB_PHI_FREE,
     VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_G_READY, VB_W_READY, VB_W_FREE,
-    VB_STATE_DONE, VB_STATE_DONE1, VB_O_FULL, VB_EXIT, VB_COUNT
+    VB_STATE_DONE, VB_STATE_DONE1, VB_O_FULL, VB_EPI_SYNC, VB_O_STORED, VB_EXIT, VB_COUNT
 };
 
 template <int D, int RH>
 __global__ void __launch_bounds__(kPassThreads, 1)
     k_vpass(const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_v,
-            const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi, Args a) {
+            const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi,
+            const __grid_constant__ CUtensorMap tm_o, Args a) {
     const Geo &g = a.g;
     const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
     const int c_begin = seg * g.cps, c_end = min(g.nchunks, c_begin + g.cps);
@@ -816,7 +843,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < VB_COUNT; ++i) {
-            const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_G_READY || i == VB_W_READY;
+            const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_G_READY || i == VB_W_READY ||
+                             i == VB_EPI_SYNC;
             tc::mbar_init(&bar[i], epi ? kPassEpiWarps : 1);
         }
         ctl->abort = 0;
@@ -926,8 +954,11 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         const int M = g.M;
         const float *erel = a.erel;
         constexpr int XH = RH / 2, DH = D / 2;
-        uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0;
+        uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0, ph_sync = 0, ph_ostored = 0;
         uint32_t ph_state[2] = {0, 0};
+        // the output tile is staged in A'_0's buffer (idle between the last MMA of a chunk and the
+        // next chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
+        const bool stage_o = NH * RH >= D;
         const float2 e1 = phase(erel, M, row, 1);
         const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
         float2 ph0[2], ph1[2], rotC[2];
@@ -949,6 +980,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             const int n = min(kC, g.L - t0);
             const bool rot = c > c_begin;
             // phase 1: U_h -> A'_h, the rotation by -m w t of (sum_j p A, sum_j p B)
+            if (stage_o && c > c_begin && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
             for (int h = 0; h < NH; ++h) {
                 if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
@@ -1016,7 +1048,18 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 tc::tmem_ld<DH>(tmem_addr(tb, lane_base, colU + wg * DH), v);
                 tc::tc_fence_before();
                 epi_arrive(&bar[VB_U_FREE]);
-                if (row < n) {
+                if (stage_o) {
+#pragma unroll
+                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16(sA, kC, row, wg * DH + g0, v + g0);
+                    tc::fence_proxy_async_smem();
+                    if (!epi_sync(&bar[VB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                    if (threadIdx.x == 0) {
+                        for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sA + db * kC * 128, db * 64, t0, bh);
+                        tc::bulk_commit();
+                        tc::bulk_wait_read0();
+                        tc::mbar_arrive(&bar[VB_O_STORED]);
+                    }
+                } else if (row < n) {
                     bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D + wg * DH;
 #pragma unroll
                     for (int j = 0; j < DH; j += 8) {
@@ -1041,6 +1084,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 }
             }
         }
+        if (threadIdx.x == 0) tc::bulk_wait0();
     }
     tc::tc_fence_before();
     __syncthreads();
@@ -1054,12 +1098,21 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 
 // ================================================================== host side
 
+// The period as an integer when w = 2 pi / T and T is a whole number below 2^24 (exact phase
+// reduction applies), else 0.
+static int integer_period(const OpDims &d) {
+    const double kPi2 = 6.283185307179586;
+    if (d.T >= 16777216.0 || d.T != floor(d.T)) return 0;
+    if (fabs(d.w - kPi2 / d.T) > 1e-15 * kPi2 / d.T) return 0;
+    return (int)d.T;
+}
+
 cudaError_t build_bf16_tables(const OpDims &d, int RP, int SP, bf16 *eb, bf16 *phi, cudaStream_t st) {
     long long total = (long long)RP * kC + (long long)SP * d.R2;
     int blocks = (int)((total + 255) / 256);
     if (blocks > 2048) blocks = 2048;
     ProfScope ps(BLA_K_TABLES_BF16, st);
-    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, d.T, d.w, eb, phi, nullptr);
+    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, d.T, d.w, integer_period(d), eb, phi, nullptr);
     return cudaGetLastError();
 }
 
@@ -1123,20 +1176,22 @@ static cudaError_t launch_kpass(const Geo &g, int smem, int nblk, cudaStream_t s
 
 template <int D, int RH>
 static cudaError_t launch_vpass_t(int smem, int nblk, cudaStream_t st, const CUtensorMap &tp, const CUtensorMap &tv,
-                                  const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
+                                  const CUtensorMap &teb, const CUtensorMap &tphi, const CUtensorMap &to,
+                                  const Args &a) {
     cudaError_t e = cudaFuncSetAttribute(k_vpass<D, RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_VPASS, st);
-    k_vpass<D, RH><<<nblk, kPassThreads, smem, st>>>(tp, tv, teb, tphi, a);
+    k_vpass<D, RH><<<nblk, kPassThreads, smem, st>>>(tp, tv, teb, tphi, to, a);
     return cudaGetLastError();
 }
 
 static cudaError_t launch_vpass(const Geo &g, int smem, int nblk, cudaStream_t st, const CUtensorMap &tp,
-                                const CUtensorMap &tv, const CUtensorMap &teb, const CUtensorMap &tphi, const Args &a) {
-    if (g.D == 64 && g.RH == 64) return launch_vpass_t<64, 64>(smem, nblk, st, tp, tv, teb, tphi, a);
-    if (g.D == 64 && g.RH == 128) return launch_vpass_t<64, 128>(smem, nblk, st, tp, tv, teb, tphi, a);
-    if (g.D == 128 && g.RH == 64) return launch_vpass_t<128, 64>(smem, nblk, st, tp, tv, teb, tphi, a);
-    if (g.D == 128 && g.RH == 128) return launch_vpass_t<128, 128>(smem, nblk, st, tp, tv, teb, tphi, a);
+                                const CUtensorMap &tv, const CUtensorMap &teb, const CUtensorMap &tphi,
+                                const CUtensorMap &to, const Args &a) {
+    if (g.D == 64 && g.RH == 64) return launch_vpass_t<64, 64>(smem, nblk, st, tp, tv, teb, tphi, to, a);
+    if (g.D == 64 && g.RH == 128) return launch_vpass_t<64, 128>(smem, nblk, st, tp, tv, teb, tphi, to, a);
+    if (g.D == 128 && g.RH == 64) return launch_vpass_t<128, 64>(smem, nblk, st, tp, tv, teb, tphi, to, a);
+    if (g.D == 128 && g.RH == 128) return launch_vpass_t<128, 128>(smem, nblk, st, tp, tv, teb, tphi, to, a);
     return cudaErrorInvalidValue;
 }
 
@@ -1161,7 +1216,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
         int blocks = (int)((total + 255) / 256);
         if (blocks > 2048) blocks = 2048;
         ProfScope ps(BLA_K_TABLES_BF16, st);
-        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, d.T, d.w, eb, phi, fseg);
+        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, d.T, d.w, integer_period(d), eb, phi, fseg);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     Args a;
@@ -1177,6 +1232,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     a.lse = lse;
     a.o = static_cast<bf16 *>(o);
     a.state_out = state_out;
+    a.tint = integer_period(d);
     a.err = device_error_word();
 
     // tensor maps
@@ -1228,7 +1284,9 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     {
         VLayout vl = v_layout(g);
         const int smem = smem_request(vl.total, pow2_cols(g.NB * g.D + 256));
-        if ((e = launch_vpass(g, smem, nblk, st, tp, tv, teb, tphi, a)) != cudaSuccess) return e;
+        CUtensorMap to;
+        if (!make_tmap_bf16(&to, o, 3, dq, sq, bq)) return cudaErrorInvalidValue;
+        if ((e = launch_vpass(g, smem, nblk, st, tp, tv, teb, tphi, to, a)) != cudaSuccess) return e;
     }
     return cudaSuccess;
 }
