@@ -236,6 +236,7 @@ def main():
     ap.add_argument("--no-decode", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--seq", type=int, default=0, help="override L (profiling captures of a smaller case)")
+    ap.add_argument("--decode-batch", type=int, default=0, help="override the decode batch (profiling captures)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -338,6 +339,9 @@ def main():
     decode = None
     if not args.no_decode:
         dw = WORKLOADS[DECODE_WORKLOAD]
+        if args.decode_batch > 0:
+            import dataclasses
+            dw = dataclasses.replace(dw, B=args.decode_batch)
         del q, k, v, o, ws
         torch.cuda.empty_cache()
         st = torch.from_numpy(make_state(dw.B, dw.H, dw.M, dw.d, dw.state_std, seed=rank)).to(dev)
@@ -362,7 +366,7 @@ def main():
         k_ms = dprof["decode"][0] / max(dprof["decode"][1], 1)
         state_bytes = 2 * (2 * dw.d) * (2 * dw.M - 1) * 4 * dw.B * dw.H
         gbs = state_bytes / (k_ms / 1000.0) / 1e9
-        decode = {"workload": DECODE_WORKLOAD + ": 256 seqs x 16 heads, d=128, M=128, S=128, T=4096",
+        decode = {"workload": DECODE_WORKLOAD + ": %d seqs x 16 heads, d=128, M=128, S=128, T=4096" % dw.B,
                   "tokens_per_s": dw.B / (d_ms / 1000.0), "ms_per_step": d_ms, "kernel_ms": k_ms,
                   "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                                "frac": gbs / peaks["hbm_gbs"], "bytes_per_launch": state_bytes}}
