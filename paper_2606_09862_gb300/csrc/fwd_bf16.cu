@@ -188,6 +188,14 @@ __device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t &phase, Ctl *ct
     return ok;
 }
 
+// wait_bar on the parity stored in bit `bit` of `bits` (flipped afterwards).
+__device__ __forceinline__ bool wait_bar(uint64_t *bar, uint32_t &bits, int bit, Ctl *ctl, int *err) {
+    uint32_t ph = (bits >> bit) & 1u;
+    const bool ok = wait_bar(bar, ph, ctl, err);
+    bits ^= 1u << bit;
+    return ok;
+}
+
 // Epilogue hand-off: every thread has finished its TMEM reads/writes and shared-memory
 // stores (fenced by the caller); the warp converges and its lane 0 arrives once.
 __device__ __forceinline__ void epi_arrive(uint64_t *bar) {
@@ -448,7 +456,7 @@ enum KBar {
     KB_EXIT, KB_COUNT
 };
 
-template <int D, int RH, int S>
+template <int D, int RH, int S, int NH>
 __global__ void __launch_bounds__(kPassThreads, 1)
     k_kpass(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
             const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi,
@@ -466,7 +474,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     Ctl *ctl = reinterpret_cast<Ctl *>(bar + KB_COUNT + 1);
     int *sdelta = reinterpret_cast<int *>(bar + KB_COUNT + 4);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int NH = g.NH, SP = g.SP;
+    const int SP = g.SP;
     // TMEM columns: [0, NB*D) state; accA at NB*D (128 cols); accB after it (RH cols).
     const int colA = g.NB * D, colB = colA + 128;
     const uint32_t ncols = (uint32_t)(colB + RH) <= 256 ? 256u : 512u;   // host: pow2_cols(NB*D + 128 + RH)
@@ -592,7 +600,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         // between the X_1 MMA (its last reader) and the next chunk's P drain
         float *red = reinterpret_cast<float *>(sP);
         uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0, ph_sync = 0, ph_ystored = 0;
-        uint32_t ph_state[2] = {0, 0};
+        uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
         const int M = g.M;
         const float *erel = a.erel;
         constexpr int XH = RH / 2;        // X columns per warpgroup (XH/2 modes)
@@ -602,15 +610,14 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         // mode chains), the start phases of its mode range in each half, e^{i m w C} of its state row
         const float2 e1 = phase(erel, M, row, 1);
         const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
-        float2 ph0[2], ph1[2], rotC[2];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int m0 = h * (RH / 2) + wg * (XH / 2);
-            ph0[h] = (h < NH) ? phase(erel, M, row, m0) : make_float2(1.f, 0.f);
-            ph1[h] = (h < NH) ? phase(erel, M, row, m0 + 1) : make_float2(1.f, 0.f);
-            const int m = (h * 128 + row) >> 1;
-            rotC[h] = (h < g.NB && m < M) ? phase(erel, M, kC, m) : make_float2(1.f, 0.f);
-        }
+        // per-half constants held in scalars (selected by h) so nothing is indexed at run time
+        const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
+        const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
+        const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
+        const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
+        const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
+        const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
+        const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
         for (int b = 0; b < g.NB; ++b) {
             const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
             state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
@@ -620,12 +627,13 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             const int t0 = c * kC;
             const int n = min(kC, g.L - t0);
             const bool rot = c > c_begin;
-            for (int h = 0; h < NH && !bad; ++h) {
+            for (int h = 0; h < NH; ++h) {
+                if (bad) break;
                 // W_h: state block h (W + EB X of the previous chunk) rotated by e^{i m w C} into the
                 // state carried into this chunk, written back, and copied to bf16 for the MMA.
-                if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+                if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                state_pass<DH>(tb, h * D + wg * DH, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr, wg * DH);
+                state_pass<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, rot, sW, RH, nullptr, wg * DH);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 epi_arrive(&bar[KB_W_READY]);
@@ -661,7 +669,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 {
                     float v[XH];
                     tc::tmem_ld<XH>(tmem_addr(tb, lane_base, (inB ? colB : colA) + wg * XH), v);
-                    float ca = ph0[h].x, sa = ph0[h].y, cb = ph1[h].x, sb = ph1[h].y;
+                    const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
+                    float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
 #pragma unroll
                     for (int i = 0; i < XH; i += 4) {
                         float xr = v[i], xi = v[i + 1];
@@ -769,7 +778,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         // final K state (lag frame at t = L-1) after the last chunk of the last segment
         if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
             for (int h = 0; h < NH; ++h)
-                if (!wait_bar(&bar[KB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+                if (!wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
             if (!bad) {
                 tc::tc_fence_after();
                 const int n_last = g.L - (c_end - 1) * kC;
@@ -818,7 +827,7 @@ enum VBar {
     VB_STATE_DONE, VB_STATE_DONE1, VB_O_FULL, VB_EPI_SYNC, VB_O_STORED, VB_EXIT, VB_COUNT
 };
 
-template <int D, int RH>
+template <int D, int RH, int NH>
 __global__ void __launch_bounds__(kPassThreads, 1)
     k_vpass(const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_v,
             const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi,
@@ -835,7 +844,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + VB_COUNT);
     Ctl *ctl = reinterpret_cast<Ctl *>(bar + VB_COUNT + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int NH = g.NH, SP = g.SP;
+    const int SP = g.SP;
     const size_t a_tile = (size_t)kC * RH * 2;
     // TMEM: [0, NB*D) state; colU (128 cols: U_h, then O); colG (128 cols).
     const int colU = g.NB * D, colG = colU + 128;
@@ -955,21 +964,20 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         const float *erel = a.erel;
         constexpr int XH = RH / 2, DH = D / 2;
         uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0, ph_sync = 0, ph_ostored = 0;
-        uint32_t ph_state[2] = {0, 0};
+        uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
         // the output tile is staged in A'_0's buffer (idle between the last MMA of a chunk and the
         // next chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
         const bool stage_o = NH * RH >= D;
         const float2 e1 = phase(erel, M, row, 1);
         const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
-        float2 ph0[2], ph1[2], rotC[2];
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int m0 = h * (RH / 2) + wg * (XH / 2);
-            ph0[h] = (h < NH) ? phase(erel, M, row, m0) : make_float2(1.f, 0.f);
-            ph1[h] = (h < NH) ? phase(erel, M, row, m0 + 1) : make_float2(1.f, 0.f);
-            const int m = (h * 128 + row) >> 1;
-            rotC[h] = (h < g.NB && m < M) ? phase(erel, M, kC, m) : make_float2(1.f, 0.f);
-        }
+        // per-half constants held in scalars (selected by h) so nothing is indexed at run time
+        const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
+        const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
+        const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
+        const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
+        const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
+        const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
+        const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
         for (int b = 0; b < g.NB; ++b) {
             const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
             state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
@@ -986,7 +994,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 tc::tc_fence_after();
                 float v[XH];
                 tc::tmem_ld<XH>(tmem_addr(tb, lane_base, colU + wg * XH), v);
-                float ca = ph0[h].x, sa = ph0[h].y, cb = ph1[h].x, sb = ph1[h].y;
+                const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
+                    float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
 #pragma unroll
                 for (int i = 0; i < XH; i += 4) {
                     float uc = v[i], us = v[i + 1];
@@ -1031,9 +1040,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             // phase 3: W_h (the V state read before this chunk's update)
             for (int h = 0; h < NH; ++h) {
                 if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
-                if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+                if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                state_pass<DH>(tb, h * D + wg * DH, row, rot, rotC[h].x, rotC[h].y, rot, sW, RH, nullptr, wg * DH);
+                state_pass<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, rot, sW, RH, nullptr, wg * DH);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 epi_arrive(&bar[VB_W_READY]);
@@ -1072,7 +1081,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         }
         if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
             for (int h = 0; h < NH; ++h)
-                if (!wait_bar(&bar[VB_STATE_DONE + h], ph_state[h], ctl, a.err)) { bad = true; break; }
+                if (!wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
             if (!bad) {
                 tc::tc_fence_after();
                 const int n_last = g.L - (c_end - 1) * kC;
@@ -1142,14 +1151,23 @@ static int smem_request(size_t bytes, int tmem_cols) {
 static int pow2_cols(int n) { return n <= 32 ? 32 : n <= 64 ? 64 : n <= 128 ? 128 : n <= 256 ? 256 : 512; }
 
 
+template <int D, int RH, int S, int NH>
+static cudaError_t launch_kpass_n(int smem, int nblk, cudaStream_t st, const CUtensorMap &tq, const CUtensorMap &tk,
+                                  const CUtensorMap &teb, const CUtensorMap &tphi, const CUtensorMap &tp, const Args &a) {
+    cudaError_t e = cudaFuncSetAttribute(k_kpass<D, RH, S, NH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    ProfScope ps(BLA_K_KPASS, st);
+    k_kpass<D, RH, S, NH><<<nblk, kPassThreads, smem, st>>>(tq, tk, teb, tphi, tp, a);
+    return cudaGetLastError();
+}
+
 template <int D, int RH, int S>
 static cudaError_t launch_kpass_t(int smem, int nblk, cudaStream_t st, const CUtensorMap &tq, const CUtensorMap &tk,
                                   const CUtensorMap &teb, const CUtensorMap &tphi, const CUtensorMap &tp, const Args &a) {
-    cudaError_t e = cudaFuncSetAttribute(k_kpass<D, RH, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    ProfScope ps(BLA_K_KPASS, st);
-    k_kpass<D, RH, S><<<nblk, kPassThreads, smem, st>>>(tq, tk, teb, tphi, tp, a);
-    return cudaGetLastError();
+    if constexpr (RH == 128) {
+        if (a.g.NH == 2) return launch_kpass_n<D, RH, S, 2>(smem, nblk, st, tq, tk, teb, tphi, tp, a);
+    }
+    return launch_kpass_n<D, RH, S, 1>(smem, nblk, st, tq, tk, teb, tphi, tp, a);
 }
 
 template <int D, int RH>
@@ -1174,15 +1192,25 @@ static cudaError_t launch_kpass(const Geo &g, int smem, int nblk, cudaStream_t s
     return cudaErrorInvalidValue;
 }
 
+template <int D, int RH, int NH>
+static cudaError_t launch_vpass_n(int smem, int nblk, cudaStream_t st, const CUtensorMap &tp, const CUtensorMap &tv,
+                                  const CUtensorMap &teb, const CUtensorMap &tphi, const CUtensorMap &to,
+                                  const Args &a) {
+    cudaError_t e = cudaFuncSetAttribute(k_vpass<D, RH, NH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    ProfScope ps(BLA_K_VPASS, st);
+    k_vpass<D, RH, NH><<<nblk, kPassThreads, smem, st>>>(tp, tv, teb, tphi, to, a);
+    return cudaGetLastError();
+}
+
 template <int D, int RH>
 static cudaError_t launch_vpass_t(int smem, int nblk, cudaStream_t st, const CUtensorMap &tp, const CUtensorMap &tv,
                                   const CUtensorMap &teb, const CUtensorMap &tphi, const CUtensorMap &to,
                                   const Args &a) {
-    cudaError_t e = cudaFuncSetAttribute(k_vpass<D, RH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    ProfScope ps(BLA_K_VPASS, st);
-    k_vpass<D, RH><<<nblk, kPassThreads, smem, st>>>(tp, tv, teb, tphi, to, a);
-    return cudaGetLastError();
+    if constexpr (RH == 128) {
+        if (a.g.NH == 2) return launch_vpass_n<D, RH, 2>(smem, nblk, st, tp, tv, teb, tphi, to, a);
+    }
+    return launch_vpass_n<D, RH, 1>(smem, nblk, st, tp, tv, teb, tphi, to, a);
 }
 
 static cudaError_t launch_vpass(const Geo &g, int smem, int nblk, cudaStream_t st, const CUtensorMap &tp,
