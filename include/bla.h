@@ -171,7 +171,9 @@ bla_status bla_profile_enable(int on);
 bla_status bla_profile_collect(double *ms, int *launches);
 
 /* Synchronise `stream` and report (then clear) the library's device error word:
- * BLA_OK, or BLA_ERR_TIMEOUT if a bounded wait gave up since the last call. */
+ * BLA_OK; BLA_ERR_TIMEOUT if a bounded wait gave up since the last call; or
+ * BLA_ERR_CUDA if a kernel refused to run because its dynamic shared memory base
+ * was not 1024-byte aligned. */
 bla_status bla_device_error(void *stream);
 
 /* Static description of a status code. */

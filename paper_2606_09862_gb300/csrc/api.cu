@@ -297,6 +297,9 @@ bla_status bla_device_error(void *stream) {
     if (code != 0) {
         e = cudaMemcpyToSymbol(g_dev_error, &zero, sizeof(int));
         if (e != cudaSuccess) return cuda_fail(e, "clear device error word");
+        if ((code & 15) == DEVERR_SMEM_ALIGN)
+            return fail(BLA_ERR_CUDA, "kernel %d found its dynamic shared memory base misaligned (block %d)",
+                        (code >> 4) & 15, (code >> 16) & 0xffff);
         return fail(BLA_ERR_TIMEOUT, "device wait gave up (code 0x%x: kind %d, kernel %d, barrier %d, parity %d, block %d)",
                     code, code & 15, (code >> 4) & 15, (code >> 8) & 127, (code >> 15) & 1, (code >> 16) & 0xffff);
     }

@@ -13,6 +13,7 @@ namespace bla {
 enum : int {
     DEVERR_NONE = 0,
     DEVERR_MBAR_TIMEOUT = 1,   // an mbarrier wait exceeded its poll budget
+    DEVERR_SMEM_ALIGN = 2,     // a kernel found its dynamic shared memory base misaligned
 };
 
 // Derived operator constants (host side), from bla_params.

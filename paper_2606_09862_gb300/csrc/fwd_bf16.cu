@@ -32,11 +32,16 @@ namespace {
 using bf16 = __nv_bfloat16;
 constexpr int kC = 128;          // tokens per chunk (MMA M)
 constexpr int kThreads = 192;
-constexpr int kEpiThreads = 128;
-constexpr int kEpiWarps = 4;   // epilogue hand-off barriers count one arrival per epilogue warp
-// The K and V passes run 10 warps: 0-7 drain TMEM as two warpgroups that split every row's
-// columns in halves (warp w reads TMEM lanes 32(w%4)..), 8 issues TMA, 9 issues the MMAs.
-constexpr int kPassThreads = 320;
+// The K and V passes run 12 warps: 0-7 drain TMEM as two warpgroups that split every row's
+// columns in halves (warp w reads TMEM lanes 32(w%4)..), 8 issues TMA loads, 9 issues the MMAs,
+// 10 issues the bulk stores of finished output tiles (K pass), 11 only completes the third
+// warpgroup.  In the K pass the third warpgroup hands registers to the first two: launched with
+// kLaunchRegs each (65536 / 384 rounded down to the allocation granule), it drops to kCtlRegs and
+// the epilogue warpgroups rise to kEpiRegs, within the launch's total.  (The V pass measured
+// slower with the same split and keeps kLaunchRegs everywhere.)
+constexpr int kPassThreads = 384;
+constexpr int kLaunchRegs = 168, kCtlRegs = 40, kEpiRegs = 232;
+static_assert(128 * kCtlRegs + 256 * kEpiRegs <= kPassThreads * kLaunchRegs, "register split exceeds the launch");
 constexpr int kPassEpiWarps = 8;
 
 
@@ -242,6 +247,71 @@ __device__ __forceinline__ uint64_t mnmaj_desc(const uint8_t *tile, int krows, i
     return tc::sdesc_sw128(a, (uint32_t)krows * 128u, 1024);
 }
 
+// Load DH columns of this thread's state row from TMEM, optionally rotate them by the phase
+// (c, s) of its mode (partner row = lane ^ 1) and write them back, and pack them to bf16 pairs.
+template <int DH>
+__device__ __forceinline__ void state_rotate_pack(uint32_t tbase, int col0, int row, bool rotate, float c, float s,
+                                                  uint32_t *pk) {
+    const int lane_base = (row >> 5) << 5;
+    const bool odd = row & 1;
+    // 32-column pieces keep the loaded values and their partners within the register budget
+#pragma unroll
+    for (int p0 = 0; p0 < DH; p0 += 32) {
+        const uint32_t addr = tmem_addr(tbase, lane_base, col0 + p0);
+        float v[32];
+        tc::tmem_ld<32>(addr, v);
+        if (rotate) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+                const float partner = __shfl_xor_sync(0xffffffffu, v[i], 1);
+                v[i] = odd ? fmaf(s, partner, c * v[i]) : fmaf(-s, partner, c * v[i]);
+            }
+            tc::tmem_st<32>(addr, v);
+        }
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) pk[(p0 + i) / 2] = tc::pack_bf16x2(v[i], v[i + 1]);
+    }
+}
+
+// Store 32 bf16 values (16 packed words) of one tile row, like st_row32_bf16.
+__device__ __forceinline__ void st_row32_packed(uint8_t *tile, int rows_per_block, int row, int col0,
+                                                const uint32_t *pk) {
+    uint8_t *blk = tile + (size_t)(col0 >> 6) * rows_per_block * 128;
+    const int c = col0 & 63;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+        *reinterpret_cast<uint4 *>(blk + tc::sw128_offset(row, c + q * 8)) =
+            make_uint4(pk[q * 4 + 0], pk[q * 4 + 1], pk[q * 4 + 2], pk[q * 4 + 3]);
+}
+
+// Descriptor offset of K-step k from step 0, in the 16-byte units of the address field (tiles
+// lie below 256 KiB, so the sum never carries out of the field).
+__device__ __forceinline__ uint64_t kmaj_step(int rows, int k) {
+    return (uint64_t)((((k >> 2) * rows * 128) + (k & 3) * 32) >> 4);
+}
+__device__ __forceinline__ uint64_t mnmaj_step(int k) { return (uint64_t)(k * 128); }   // 16 rows x 128 B
+
+// An opaque copy of x: values derived from it cannot be hoisted above this point.
+__device__ __forceinline__ uint64_t opaque(uint64_t x) {
+    asm volatile("" : "+l"(x));
+    return x;
+}
+
+// acc (+)= A B^T over nk K-steps of 16.  A is a K-major tile of `arows` rows; B is K-major with
+// `brows` rows, or MN-major (MN_B) with `brows` K rows per block.  The first step accumulates only
+// if acc0.  Each step's descriptors are the base descriptors plus a constant, formed at the issue,
+// so that the issuing thread holds two descriptors rather than one per step.
+template <bool MN_B>
+__device__ __forceinline__ void mma_steps(uint32_t acc, const uint8_t *a, int arows, const uint8_t *b, int brows,
+                                          uint32_t idesc, int nk, bool acc0) {
+    const uint64_t da = opaque(kmaj_desc(a, arows, 0));
+    const uint64_t db = opaque(MN_B ? mnmaj_desc(b, brows, 0) : kmaj_desc(b, brows, 0));
+#pragma unroll
+    for (int k = 0; k < nk; ++k)
+        tc::mma_bf16(acc, da + kmaj_step(arows, k), db + (MN_B ? mnmaj_step(k) : kmaj_step(brows, k)), idesc,
+                     (acc0 || k > 0) ? 1u : 0u);
+}
+
 // Rotate the state block held in TMEM (rows = lanes, interleaved cos/sin pairs) by the
 // phase (c, s) of this thread's mode, optionally write it back, and emit a bf16 copy into
 // a [RH rows][64 d]-blocked tile (rows >= RH skipped) and/or an fp32 copy to global.
@@ -442,8 +512,8 @@ __host__ __device__ inline KLayout k_layout(const Geo &g) {
     l.y = off;   off += (size_t)kC * g.RH * 2;
     l.eb = off;  off += (size_t)128 * kC * 2;
     l.phi = off; off += (size_t)g.SP * g.RH * 2;
-    l.bars = off; off += 2048;   // barriers, TMEM slot, control, slot lags
-    l.total = off + 1024;   // slack for 1024-byte alignment of the dynamic smem base
+    l.bars = off; off += 3072;   // barriers, TMEM slot, control, slot lags [0, 1024); softmax exchange
+    l.total = off;               // the dynamic shared memory base is 1024-aligned (checked by the kernel)
     return l;
 }
 
@@ -453,7 +523,7 @@ enum KBar {
     KB_QK_FULL, KB_QK_FREE, KB_EB_FULL, KB_EB_FREE, KB_PHI_FULL, KB_PHI_FREE,
     KB_ACC_FULL_A, KB_ACC_FULL_B, KB_ACC_FREE_A, KB_ACC_FREE_B,
     KB_P_READY, KB_W_READY, KB_W_FREE, KB_STATE_DONE, KB_STATE_DONE1, KB_Y_READY, KB_Y_FREE, KB_EPI_SYNC, KB_Y_STORED,
-    KB_EXIT, KB_COUNT
+    KB_P_SMEM, KB_EXIT, KB_COUNT
 };
 
 template <int D, int RH, int S, int NH>
@@ -464,8 +534,13 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     const Geo &g = a.g;
     const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
     const int c_begin = seg * g.cps, c_end = min(g.nchunks, c_begin + g.cps);
-    extern __shared__ uint8_t smem_raw[];
-    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    // the 128-byte-swizzled tiles need a 1024-aligned base; the layout reserves no slack for it
+    if (tc::smem_u32(smem_raw) & 1023u) {
+        if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (2 << 4) | ((int)blockIdx.x << 16));
+        return;
+    }
+    uint8_t *sm = smem_raw;
     const KLayout lay = k_layout(g);
     uint8_t *sQ = sm + lay.q, *sK = sm + lay.k, *sP = sm + lay.p, *sW = sm + lay.w, *sY = sm + lay.y;
     uint8_t *sEB = sm + lay.eb, *sPHI = sm + lay.phi;
@@ -482,7 +557,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < KB_COUNT; ++i) {
             const bool epi = i == KB_P_READY || i == KB_W_READY || i == KB_Y_READY || i == KB_ACC_FREE_A ||
-                             i == KB_ACC_FREE_B || i == KB_EPI_SYNC;
+                             i == KB_ACC_FREE_B || i == KB_EPI_SYNC || i == KB_P_SMEM;
             tc::mbar_init(&bar[i], epi ? kPassEpiWarps : 1);
         }
         ctl->abort = 0;
@@ -497,150 +572,229 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
 
-    if (warp == 8) {
-        if (lane == 0) {
-            tc::tma_prefetch_desc(&tm_q); tc::tma_prefetch_desc(&tm_k);
-            tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
-            uint32_t ph_qk = 0, ph_eb = 0, ph_phi = 0;
-            bool first_eb = true, first_phi = true;
-            for (int c = c_begin; c < c_end && !ctl->abort; ++c) {
-                if (c > c_begin && !wait_bar(&bar[KB_QK_FREE], ph_qk, ctl, a.err)) break;
-                tc::mbar_arrive_expect_tx(&bar[KB_QK_FULL], (uint32_t)(2 * kC * D * 2));
-                for (int db = 0; db < D / 64; ++db) {
-                    tc::tma_load_3d(sQ + db * kC * 128, &tm_q, &bar[KB_QK_FULL], db * 64, c * kC, bh);
-                    tc::tma_load_3d(sK + db * kC * 128, &tm_k, &bar[KB_QK_FULL], db * 64, c * kC, bh);
-                }
-                for (int h = 0; h < NH; ++h) {
-                    if (!first_eb && !wait_bar(&bar[KB_EB_FREE], ph_eb, ctl, a.err)) break;
-                    first_eb = false;
-                    tc::mbar_arrive_expect_tx(&bar[KB_EB_FULL], (uint32_t)(128 * kC * 2));
-                    for (int kb = 0; kb < 2; ++kb)
-                        tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[KB_EB_FULL], kb * 64, h * 128);
-                    if (!first_phi && !wait_bar(&bar[KB_PHI_FREE], ph_phi, ctl, a.err)) break;
-                    first_phi = false;
-                    tc::mbar_arrive_expect_tx(&bar[KB_PHI_FULL], (uint32_t)(SP * RH * 2));
-                    for (int kb = 0; kb < RH / 64; ++kb)
-                        tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[KB_PHI_FULL], h * RH + kb * 64, 0);
+    if (warp >= 8) {
+        tc::reg_dealloc<kCtlRegs>();
+        if (warp == 8) {
+            // ---------------- TMA producer: per chunk Q, K, then (EB_h, PHI_h) for each mode half, in
+            // the order the MMA issuer consumes them
+            if (lane == 0) {
+                tc::tma_prefetch_desc(&tm_q); tc::tma_prefetch_desc(&tm_k);
+                tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
+                uint32_t ph_qk = 0, ph_eb = 0, ph_phi = 0;
+                bool first_eb = true, first_phi = true;
+                for (int c = c_begin; c < c_end && !ctl->abort; ++c) {
+                    if (c > c_begin && !wait_bar(&bar[KB_QK_FREE], ph_qk, ctl, a.err)) break;
+                    tc::mbar_arrive_expect_tx(&bar[KB_QK_FULL], (uint32_t)(2 * kC * D * 2));
+                    for (int db = 0; db < D / 64; ++db) {
+                        tc::tma_load_3d(sQ + db * kC * 128, &tm_q, &bar[KB_QK_FULL], db * 64, c * kC, bh);
+                        tc::tma_load_3d(sK + db * kC * 128, &tm_k, &bar[KB_QK_FULL], db * 64, c * kC, bh);
+                    }
+                    for (int h = 0; h < NH; ++h) {
+                        if (!first_eb && !wait_bar(&bar[KB_EB_FREE], ph_eb, ctl, a.err)) break;
+                        first_eb = false;
+                        tc::mbar_arrive_expect_tx(&bar[KB_EB_FULL], (uint32_t)(128 * kC * 2));
+                        for (int kb = 0; kb < 2; ++kb)
+                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[KB_EB_FULL], kb * 64, h * 128);
+                        if (!first_phi && !wait_bar(&bar[KB_PHI_FREE], ph_phi, ctl, a.err)) break;
+                        first_phi = false;
+                        tc::mbar_arrive_expect_tx(&bar[KB_PHI_FULL], (uint32_t)(SP * RH * 2));
+                        for (int kb = 0; kb < RH / 64; ++kb)
+                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[KB_PHI_FULL], h * RH + kb * 64, 0);
+                    }
                 }
             }
-        }
-    } else if (warp == 9) {
-        if (lane == 0) {
-            uint32_t ph_qk = 0, ph_eb = 0, ph_phi = 0, ph_freeA = 0, ph_freeB = 0, ph_p = 0, ph_w = 0, ph_y = 0;
-            const uint32_t id_P = tc::idesc_bf16(128, kC, false, false);
-            const uint32_t id_X = tc::idesc_bf16(128, RH, false, false);
-            const uint32_t id_S = tc::idesc_bf16(128, S, false, false);
-            const uint32_t id_U = tc::idesc_bf16(128, D, false, true);
-            // Each accumulator region is handed back by the epilogue after every drain; every use
-            // but the very first waits for that hand-back.
-            bool usedA = false, usedB = false;
-            auto acquire = [&](bool inB) -> bool {
-                bool &used = inB ? usedB : usedA;
-                if (used && !wait_bar(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A], inB ? ph_freeB : ph_freeA, ctl, a.err))
-                    return false;
-                used = true;
-                return true;
-            };
-            for (int c = c_begin; c < c_end; ++c) {
-                if (!wait_bar(&bar[KB_QK_FULL], ph_qk, ctl, a.err)) break;
-                if (!acquire(false)) break;
-                tc::tc_fence_after();
-                for (int k = 0; k < D / 16; ++k)
-                    tc::mma_bf16(tb + colA, kmaj_desc(sQ, kC, k), kmaj_desc(sK, kC, k), id_P, k > 0);
-                tc::mma_commit(&bar[KB_ACC_FULL_A]);
-                bool bad = false;
-                for (int h = 0; h < NH && !bad; ++h) {
-                    // X_h = Q W_h^T + P EB_h^T  -> acc (h even: B, odd: A)
-                    const bool inB = (h & 1) == 0;
-                    if (!wait_bar(&bar[KB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
-                    if (!wait_bar(&bar[KB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
-                    if (h == 0 && !wait_bar(&bar[KB_P_READY], ph_p, ctl, a.err)) { bad = true; break; }
-                    if (!acquire(inB)) { bad = true; break; }
-                    tc::tc_fence_after();
-                    const uint32_t dX = tb + (inB ? colB : colA);
-                    for (int k = 0; k < D / 16; ++k)
-                        tc::mma_bf16(dX, kmaj_desc(sQ, kC, k), kmaj_desc(sW, RH, k), id_X, k > 0);
-                    for (int k = 0; k < kC / 16; ++k)
-                        tc::mma_bf16(dX, kmaj_desc(sP, kC, k), kmaj_desc(sEB, 128, k), id_X, 1);
-                    tc::mma_commit(&bar[inB ? KB_ACC_FULL_B : KB_ACC_FULL_A]);
-                    tc::mma_commit(&bar[KB_W_FREE]);
-                    // state block h += EB_h (A, 128 rows) . K_chunk (B, MN-major, N = D)
-                    for (int k = 0; k < kC / 16; ++k)
-                        tc::mma_bf16(tb + h * D, kmaj_desc(sEB, 128, k), mnmaj_desc(sK, kC, k), id_U, 1);
+        } else if (warp == 9) {
+            // ---------------- MMA issuer.  X_h = Q W_h^T + P EB_h^T is issued in two parts so that the
+            // tensor pipe has work while P is drained and while EB_1 is loaded.  Per chunk:
+            //   Q W_0^T -> B;  P EB_0^T -> B;  state_0 += EB_0 K;
+            //   Q W_1^T -> A (once P is drained);  P EB_1^T -> A;  s_0 -> B (once Y_0 is out of B);
+            //   state_1 += EB_1 K;  s_1 -> B;  P of the next chunk -> A.
+            // With one half the scores go to A once P is drained (B holds only RH columns).
+            if (lane == 0) {
+                uint32_t ph_qk = 0, ph_eb = 0, ph_phi = 0, ph_freeA = 0, ph_freeB = 0, ph_p = 0, ph_w = 0, ph_y = 0;
+                const uint32_t id_P = tc::idesc_bf16(128, kC, false, false);
+                const uint32_t id_X = tc::idesc_bf16(128, RH, false, false);
+                const uint32_t id_S = tc::idesc_bf16(128, S, false, false);
+                const uint32_t id_U = tc::idesc_bf16(128, D, false, true);
+                const uint32_t accA = tb + colA, accB = tb + colB;
+                constexpr bool sB = NH == 2;
+                const uint32_t accS = sB ? accB : accA;
+                auto peb = [&](uint32_t dX) {
+                    // X_h += P EB_h^T
+                    mma_steps<false>(dX, sP, kC, sEB, 128, id_X, kC / 16, true);
+                    tc::mma_commit(&bar[dX == accA ? KB_ACC_FULL_A : KB_ACC_FULL_B]);
+                };
+                auto state_update = [&](int h) {
+                    // state block h += EB_h (A, 128 rows) . K (B, MN-major)
+                    mma_steps<true>(tb + h * D, sEB, 128, sK, kC, id_U, kC / 16, true);
                     tc::mma_commit(&bar[KB_STATE_DONE + h]);
                     tc::mma_commit(&bar[KB_EB_FREE]);
                     if (h == NH - 1) tc::mma_commit(&bar[KB_QK_FREE]);
-                }
-                if (bad) break;
-                // s = sum_h Y_h PHI_h^T -> acc (NH == 2: B after X_0 drained; NH == 1: A after P drained)
-                const bool sInB = NH == 2;
-                if (!acquire(sInB)) break;
-                for (int h = 0; h < NH && !bad; ++h) {
-                    if (!wait_bar(&bar[KB_PHI_FULL], ph_phi, ctl, a.err)) { bad = true; break; }
-                    if (!wait_bar(&bar[KB_Y_READY], ph_y, ctl, a.err)) { bad = true; break; }
+                };
+                auto s_part = [&](int h) -> bool {
+                    // s (+)= Y_h PHI_h^T
+                    if (!wait_bar(&bar[KB_PHI_FULL], ph_phi, ctl, a.err)) return false;
+                    if (!wait_bar(&bar[KB_Y_READY], ph_y, ctl, a.err)) return false;
                     tc::tc_fence_after();
-                    const uint32_t dS = tb + (sInB ? colB : colA);
-                    for (int k = 0; k < RH / 16; ++k)
-                        tc::mma_bf16(dS, kmaj_desc(sY, kC, k), kmaj_desc(sPHI, SP, k), id_S, (h > 0 || k > 0) ? 1u : 0u);
+                    mma_steps<false>(accS, sY, kC, sPHI, SP, id_S, RH / 16, h > 0);
                     tc::mma_commit(&bar[KB_Y_FREE]);
                     tc::mma_commit(&bar[KB_PHI_FREE]);
+                    return true;
+                };
+                // P of the first chunk; every later P is issued at the end of the chunk before it
+                auto issue_p = [&](bool first) -> bool {
+                    if (!wait_bar(&bar[KB_QK_FULL], ph_qk, ctl, a.err)) return false;
+                    // A: last read by the previous chunk's Y_1 drain (two halves) or softmax (one half)
+                    if (!first && !wait_bar(&bar[KB_ACC_FREE_A], ph_freeA, ctl, a.err)) return false;
+                    tc::tc_fence_after();
+                    mma_steps<false>(accA, sQ, kC, sK, kC, id_P, D / 16, false);
+                    tc::mma_commit(&bar[KB_ACC_FULL_A]);
+                    return true;
+                };
+                bool ok = c_begin < c_end && issue_p(true);
+                for (int c = c_begin; c < c_end && ok; ++c) {
+                    ok = false;
+                    const bool first = c == c_begin;
+                    // X_0 -> B: last read by the previous chunk's softmax (two halves) or Y_0 drain (one)
+                    if (!wait_bar(&bar[KB_W_READY], ph_w, ctl, a.err)) break;
+                    if (!first && !wait_bar(&bar[KB_ACC_FREE_B], ph_freeB, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    mma_steps<false>(accB, sQ, kC, sW, RH, id_X, D / 16, false);
+                    tc::mma_commit(&bar[KB_W_FREE]);
+                    if (!wait_bar(&bar[KB_EB_FULL], ph_eb, ctl, a.err)) break;
+                    if (!wait_bar(&bar[KB_P_READY], ph_p, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    peb(accB);
+                    state_update(0);
+                    if (NH == 2) {
+                        // X_1 -> A once P has been drained
+                        if (!wait_bar(&bar[KB_W_READY], ph_w, ctl, a.err)) break;
+                        if (!wait_bar(&bar[KB_ACC_FREE_A], ph_freeA, ctl, a.err)) break;
+                        tc::tc_fence_after();
+                        mma_steps<false>(accA, sQ, kC, sW, RH, id_X, D / 16, false);
+                        tc::mma_commit(&bar[KB_W_FREE]);
+                        if (!wait_bar(&bar[KB_EB_FULL], ph_eb, ctl, a.err)) break;
+                        tc::tc_fence_after();
+                        peb(accA);
+                    }
+                    // s_0 once its region has been drained (X_0 into Y, or P)
+                    if (sB ? !wait_bar(&bar[KB_ACC_FREE_B], ph_freeB, ctl, a.err)
+                           : !wait_bar(&bar[KB_ACC_FREE_A], ph_freeA, ctl, a.err))
+                        break;
+                    if (!s_part(0)) break;
+                    if (NH == 2) {
+                        state_update(1);
+                        if (!s_part(1)) break;
+                    }
+                    tc::mma_commit(&bar[sB ? KB_ACC_FULL_B : KB_ACC_FULL_A]);
+                    ok = c + 1 >= c_end || issue_p(false);
                 }
-                if (bad) break;
-                tc::mma_commit(&bar[sInB ? KB_ACC_FULL_B : KB_ACC_FULL_A]);
+                tc::mma_commit(&bar[KB_EXIT]);
+                uint32_t ph_exit = 0;
+                tc::mbar_wait(&bar[KB_EXIT], ph_exit);
             }
-            tc::mma_commit(&bar[KB_EXIT]);
-            uint32_t ph_exit = 0;
-            tc::mbar_wait(&bar[KB_EXIT], ph_exit);
+        } else if (warp == 10) {
+            // ---------------- p store: once the epilogue has written a chunk's probabilities into the
+            // Y tile, bulk-store them and hand the tile back when the copy has read it
+            if (lane == 0) {
+                uint32_t ph_psmem = 0;
+                for (int c = c_begin; c < c_end; ++c) {
+                    if (!wait_bar(&bar[KB_P_SMEM], ph_psmem, ctl, a.err)) break;
+                    for (int kb = 0; kb < SP / 64; ++kb) tc::tma_store_3d(&tm_p, sY + kb * kC * 128, kb * 64, c * kC, bh);
+                    tc::bulk_commit();
+                    tc::bulk_wait_read0();
+                    tc::mbar_arrive(&bar[KB_Y_STORED]);
+                }
+                tc::bulk_wait0();
+            }
         }
     } else {
-        // ---------------- epilogue warps 0-7: thread = TMEM lane = token row / state row;
-        // warpgroup wg handles columns [wg*N/2, (wg+1)*N/2) of every N-column drain
-        const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
-        // softmax partials [2 (max, sum)][2 (warpgroup)][128 rows] live in the P tile, which is idle
-        // between the X_1 MMA (its last reader) and the next chunk's P drain
-        float *red = reinterpret_cast<float *>(sP);
-        uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0, ph_sync = 0, ph_ystored = 0;
-        uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
-        const int M = g.M;
-        const float *erel = a.erel;
-        constexpr int XH = RH / 2;        // X columns per warpgroup (XH/2 modes)
-        constexpr int DH = D / 2;         // state columns per warpgroup
-        constexpr int SH = S >= 64 ? S / 2 : S;   // slot columns per warpgroup (S = 32: warpgroup 0 only)
-        // phase constants of this thread, fixed for the whole CTA: e^{i 2 w t} (two interleaved
-        // mode chains), the start phases of its mode range in each half, e^{i m w C} of its state row
-        const float2 e1 = phase(erel, M, row, 1);
-        const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
-        // per-half constants held in scalars (selected by h) so nothing is indexed at run time
-        const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
-        const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
-        const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
-        const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
-        const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
-        const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
-        const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
-        for (int b = 0; b < g.NB; ++b) {
-            const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
-            state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
-        }
-        bool bad = false;
-        for (int c = c_begin; c < c_end && !bad; ++c) {
-            const int t0 = c * kC;
-            const int n = min(kC, g.L - t0);
-            const bool rot = c > c_begin;
-            for (int h = 0; h < NH; ++h) {
-                if (bad) break;
-                // W_h: state block h (W + EB X of the previous chunk) rotated by e^{i m w C} into the
-                // state carried into this chunk, written back, and copied to bf16 for the MMA.
-                if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
+        tc::reg_alloc<kEpiRegs>();
+        {
+            // ---------------- epilogue warps 0-7: thread = TMEM lane = token row / state row;
+            // warpgroup wg handles columns [wg*N/2, (wg+1)*N/2) of every N-column drain.
+            // Per chunk: W_1; Y_0; Y_1; W_0 (and W_1 into registers) of the next chunk; P of the next
+            // chunk; softmax (one half: softmax, then P).
+            const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
+            // softmax partials [2 (max, sum)][2 (warpgroup)][128 rows] in the control area
+            float *red = reinterpret_cast<float *>(sm + lay.bars + 1024);
+            uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0, ph_sync = 0, ph_ystored = 0;
+            uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
+            const int M = g.M;
+            const float *erel = a.erel;
+            constexpr int XH = RH / 2;        // X columns per warpgroup (XH/2 modes)
+            constexpr int DH = D / 2;         // state columns per warpgroup
+            constexpr int SH = S >= 64 ? S / 2 : S;   // slot columns per warpgroup (S = 32: warpgroup 0 only)
+            // phase constants of this thread, fixed for the whole CTA: e^{i 2 w t} (two interleaved
+            // mode chains), the start phases of its mode range in each half, e^{i m w C} of its state row
+            const float2 e1 = phase(erel, M, row, 1);
+            const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
+            // per-half constants held in scalars (selected by h) so nothing is indexed at run time
+            const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
+            const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
+            const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
+            const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
+            const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
+            const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
+            const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
+            for (int b = 0; b < g.NB; ++b) {
+                const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
+                state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
+            }
+            // W_h: state block h (W + EB K of the previous chunk) rotated by e^{i m w C} into the state
+            // carried into the next chunk and written back (w_compute, into packed bf16 registers);
+            // then copied into the W tile once the MMA that read the previous W_h' is done (w_store).
+            auto w_compute = [&](int h, bool rot, uint32_t *pk) -> bool {
+                if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) return false;
                 tc::tc_fence_after();
-                state_pass<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, rot, sW, RH, nullptr, wg * DH);
+                state_rotate_pack<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, pk);
+                return true;
+            };
+            auto w_store = [&](bool wait_free, const uint32_t *pk) -> bool {
+                if (wait_free && !wait_bar(&bar[KB_W_FREE], ph_wfree, ctl, a.err)) return false;
+                if (row < RH) {
+#pragma unroll
+                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_packed(sW, RH, row, wg * DH + g0, pk + g0 / 2);
+                }
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 epi_arrive(&bar[KB_W_READY]);
-                if (h == 0) {
-                    // P drain: causal mask u <= t, bf16 -> sP
-                    if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
-                    tc::tc_fence_after();
+                return true;
+            };
+            // Y_h = e^{i m w t} X_h (t = row) from accumulator region `col`, two interleaved mode chains
+            auto y_drain = [&](int h, int col) {
+                float v[XH];
+                tc::tmem_ld<XH>(tmem_addr(tb, lane_base, col + wg * XH), v);
+                const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
+                float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
+#pragma unroll
+                for (int i = 0; i < XH; i += 4) {
+                    float xr = v[i], xi = v[i + 1];
+                    v[i] = ca * xr - sa * xi;
+                    v[i + 1] = sa * xr + ca * xi;
+                    xr = v[i + 2];
+                    xi = v[i + 3];
+                    v[i + 2] = cb * xr - sb * xi;
+                    v[i + 3] = sb * xr + cb * xi;
+                    float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
+                    ca = t1;
+                    sa = t2;
+                    t1 = cb * e2.x - sb * e2.y;
+                    t2 = sb * e2.x + cb * e2.y;
+                    cb = t1;
+                    sb = t2;
+                }
+#pragma unroll
+                for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sY, kC, row, wg * XH + g0, v + g0);
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                epi_arrive(&bar[KB_Y_READY]);
+            };
+            // P drain: causal mask u <= t, bf16 -> sP
+            auto p_drain = [&]() -> bool {
+                if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) return false;
+                tc::tc_fence_after();
+                {
                     float v[64];
                     tc::tmem_ld<64>(tmem_addr(tb, lane_base, colA + wg * 64), v);
 #pragma unroll
@@ -648,149 +802,144 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         if (wg * 64 + i > row) v[i] = 0.f;
 #pragma unroll
                     for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(sP, kC, row, wg * 64 + g0, v + g0);
-                    tc::fence_proxy_async_smem();
-                    tc::tc_fence_before();
-                    epi_arrive(&bar[KB_P_READY]);
+                }
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                epi_arrive(&bar[KB_P_READY]);
+                epi_arrive(&bar[KB_ACC_FREE_A]);
+                return true;
+            };
+            // W_0 and W_1 of the first chunk (the carried-in state as it is) and its P
+            uint32_t pk1[DH / 2];   // W_1 of the coming chunk, stored once that chunk's Q W_0^T is done
+            bool bad = false;
+            if (c_begin < c_end) {
+                uint32_t pk0[DH / 2];
+                bad = !w_compute(0, false, pk0) || !w_store(false, pk0) || (NH == 2 && !w_compute(1, false, pk1)) ||
+                      !p_drain();
+            }
+            for (int c = c_begin; c < c_end && !bad; ++c) {
+                const int t0 = c * kC;
+                const int n = min(kC, g.L - t0);
+                const bool rot = c > c_begin, more = c + 1 < c_end;
+                // W_1 (computed at the end of the previous chunk) once Q W_0^T has read W_0
+                if (NH == 2 && !w_store(true, pk1)) { bad = true; break; }
+                // Y_0 from B; the previous chunk's probabilities must have left the Y tile
+                if (!wait_bar(&bar[KB_ACC_FULL_B], ph_fullB, ctl, a.err)) { bad = true; break; }
+                if (rot && !wait_bar(&bar[KB_Y_STORED], ph_ystored, ctl, a.err)) { bad = true; break; }
+                tc::tc_fence_after();
+                y_drain(0, colB);
+                epi_arrive(&bar[KB_ACC_FREE_B]);
+                if (NH == 2) {
+                    // Y_1 from A once s_0 has read Y_0
+                    if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
+                    if (!wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    y_drain(1, colA);
                     epi_arrive(&bar[KB_ACC_FREE_A]);
                 }
-                // X_h drain -> Y_h = e^{i m w t} X_h (t = row), two interleaved mode chains
-                const bool inB = (h & 1) == 0;
-                if (!wait_bar(&bar[inB ? KB_ACC_FULL_B : KB_ACC_FULL_A], inB ? ph_fullB : ph_fullA, ctl, a.err)) {
+                // W_0 of the next chunk (stored once Q W_1^T, or with one half Q W_0^T, has read the W
+                // tile) and W_1 of the next chunk into registers, while the last s MMA runs
+                if (more) {
+                    uint32_t pk0[DH / 2];
+                    if (!w_compute(0, true, pk0) || !w_store(true, pk0) || (NH == 2 && !w_compute(1, true, pk1))) {
+                        bad = true;
+                        break;
+                    }
+                }
+                // two halves: the next chunk's P (A is free once Y_1 is drained) before this chunk's
+                // softmax, so that the next chunk's X MMAs run during the softmax
+                if (NH == 2 && more && !p_drain()) { bad = true; break; }
+                // masked softmax over the S slots; the two warpgroups exchange their (max, sum) pairs once
+                constexpr bool sB = NH == 2;
+                if (sB ? !wait_bar(&bar[KB_ACC_FULL_B], ph_fullB, ctl, a.err)
+                       : !wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) {
                     bad = true;
                     break;
                 }
-                if (!wait_bar(&bar[KB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
-                if (h > 0 && !wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
-                if (h == 0 && c > c_begin) {
-                    // the previous chunk's probabilities have left the Y tile (bulk store read done)
-                    if (!wait_bar(&bar[KB_Y_STORED], ph_ystored, ctl, a.err)) { bad = true; break; }
-                }
+                if (!wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
                 {
-                    float v[XH];
-                    tc::tmem_ld<XH>(tmem_addr(tb, lane_base, (inB ? colB : colA) + wg * XH), v);
-                    const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
-                    float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
+                    const bool active = wg == 0 || S >= 64;
+                    const int j0 = (S >= 64) ? wg * SH : 0;
+                    const int t = t0 + row;
+                    // slots are visible when t >= D_j; past the largest lag of the grid every slot is
+                    const bool all_visible = t0 >= sdelta[S - 1];
+                    const float sl2 = a.scale * 1.4426950408889634f;   // scores in log2 units
+                    float v[SH];
+                    if (active) tc::tmem_ld<SH>(tmem_addr(tb, lane_base, (sB ? colB : colA) + j0), v);
+                    tc::tc_fence_before();
+                    epi_arrive(&bar[sB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
+                    float mx = -INFINITY, sum = 0.f;
+                    if (active) {
+                        float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                        if (all_visible) {
 #pragma unroll
-                    for (int i = 0; i < XH; i += 4) {
-                        float xr = v[i], xi = v[i + 1];
-                        v[i] = ca * xr - sa * xi;
-                        v[i + 1] = sa * xr + ca * xi;
-                        xr = v[i + 2];
-                        xi = v[i + 3];
-                        v[i + 2] = cb * xr - sb * xi;
-                        v[i + 3] = sb * xr + cb * xi;
-                        float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
-                        ca = t1;
-                        sa = t2;
-                        t1 = cb * e2.x - sb * e2.y;
-                        t2 = sb * e2.x + cb * e2.y;
-                        cb = t1;
-                        sb = t2;
-                    }
+                            for (int j = 0; j < SH; ++j) {
+                                v[j] *= sl2;
+                                m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                            }
+                        } else {
 #pragma unroll
-                    for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sY, kC, row, wg * XH + g0, v + g0);
-                }
-                tc::fence_proxy_async_smem();
-                tc::tc_fence_before();
-                epi_arrive(&bar[KB_Y_READY]);
-                epi_arrive(&bar[inB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
-            }
-            if (bad) break;
-            // masked softmax over the S slots; the two warpgroups exchange their (max, sum) pairs once
-            const bool sInB = NH == 2;
-            if (!wait_bar(&bar[sInB ? KB_ACC_FULL_B : KB_ACC_FULL_A], sInB ? ph_fullB : ph_fullA, ctl, a.err)) {
-                bad = true;
-                break;
-            }
-            if (!wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
-            tc::tc_fence_after();
-            {
-                const bool active = wg == 0 || S >= 64;
-                const int j0 = (S >= 64) ? wg * SH : 0;
-                const int t = t0 + row;
-                // slots are visible when t >= D_j; past the largest lag of the grid every slot is
-                const bool all_visible = t0 >= sdelta[S - 1];
-                const float sl2 = a.scale * 1.4426950408889634f;   // scores in log2 units
-                float v[SH];
-                if (active) tc::tmem_ld<SH>(tmem_addr(tb, lane_base, (sInB ? colB : colA) + j0), v);
-                tc::tc_fence_before();
-                epi_arrive(&bar[sInB ? KB_ACC_FREE_B : KB_ACC_FREE_A]);
-                float mx = -INFINITY, sum = 0.f;
-                if (active) {
-                    float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                    if (all_visible) {
+                            for (int j = 0; j < SH; ++j) {
+                                v[j] = (t >= sdelta[j0 + j]) ? v[j] * sl2 : -INFINITY;
+                                m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                            }
+                        }
+                        mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
+                        // a half whose slots are all hidden has mx = -inf: exponentiate against 0 instead
+                        const float mref = (mx == -INFINITY) ? 0.f : mx;
+                        float s4[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                         for (int j = 0; j < SH; ++j) {
-                            v[j] *= sl2;
-                            m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                            v[j] = exp2f(v[j] - mref);          // exp2(-inf) = 0 on masked slots
+                            s4[j & 3] += v[j];
                         }
-                    } else {
-#pragma unroll
-                        for (int j = 0; j < SH; ++j) {
-                            v[j] = (t >= sdelta[j0 + j]) ? v[j] * sl2 : -INFINITY;
-                            m4[j & 3] = fmaxf(m4[j & 3], v[j]);
-                        }
+                        sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
                     }
-                    mx = fmaxf(fmaxf(m4[0], m4[1]), fmaxf(m4[2], m4[3]));
-                    // a half whose slots are all hidden has mx = -inf: exponentiate against 0 instead
-                    const float mref = (mx == -INFINITY) ? 0.f : mx;
-                    float s4[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-                    for (int j = 0; j < SH; ++j) {
-                        v[j] = exp2f(v[j] - mref);          // exp2(-inf) = 0 on masked slots
-                        s4[j & 3] += v[j];
+                    float gmx = mx, gsum = sum;
+                    if (S >= 64) {
+                        red[wg * 128 + row] = mx;
+                        red[256 + wg * 128 + row] = sum;
+                        if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                        const float m0 = red[row], m1 = red[128 + row];
+                        gmx = fmaxf(m0, m1);
+                        gsum = red[256 + row] * exp2f(m0 - gmx) + red[384 + row] * exp2f(m1 - gmx);
                     }
-                    sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
-                }
-                float gmx = mx, gsum = sum;
-                if (S >= 64) {
-                    red[wg * 128 + row] = mx;
-                    red[256 + wg * 128 + row] = sum;
-                    if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
-                    const float m0 = red[row], m1 = red[128 + row];
-                    gmx = fmaxf(m0, m1);
-                    gsum = red[256 + row] * exp2f(m0 - gmx) + red[384 + row] * exp2f(m1 - gmx);
-                }
-                if (active) {
-                    const float f = exp2f(mx - gmx) / gsum;
+                    if (active) {
+                        const float f = exp2f(mx - gmx) / gsum;
 #pragma unroll
-                    for (int j = 0; j < SH; ++j) v[j] *= f;
+                        for (int j = 0; j < SH; ++j) v[j] *= f;
 #pragma unroll
-                    for (int g0 = 0; g0 < SH; g0 += 32) st_row32_bf16(sY, kC, row, j0 + g0, v + g0);
-                } else if (SP > S) {
-                    float z[32];
+                        for (int g0 = 0; g0 < SH; g0 += 32) st_row32_bf16(sY, kC, row, j0 + g0, v + g0);
+                    } else if (SP > S) {
+                        float z[32];
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) z[i] = 0.f;
-                    for (int g0 = S; g0 < SP; g0 += 32) st_row32_bf16(sY, kC, row, g0, z);
+                        for (int i = 0; i < 32; ++i) z[i] = 0.f;
+                        for (int g0 = S; g0 < SP; g0 += 32) st_row32_bf16(sY, kC, row, g0, z);
+                    }
+                    if (wg == 0 && row < n && a.lse) a.lse[(size_t)bh * g.L + t] = (gmx + log2f(gsum)) * 0.6931471805599453f;
+                    tc::fence_proxy_async_smem();
+                    epi_arrive(&bar[KB_P_SMEM]);
                 }
-                if (wg == 0 && row < n && a.lse) a.lse[(size_t)bh * g.L + t] = (gmx + log2f(gsum)) * 0.6931471805599453f;
-                tc::fence_proxy_async_smem();
-                if (!epi_sync(&bar[KB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
-                if (threadIdx.x == 0) {
-                    for (int kb = 0; kb < SP / 64; ++kb) tc::tma_store_3d(&tm_p, sY + kb * kC * 128, kb * 64, t0, bh);
-                    tc::bulk_commit();
-                    tc::bulk_wait_read0();
-                    tc::mbar_arrive(&bar[KB_Y_STORED]);
+                // one half: the scores occupy A until the softmax has loaded them
+                if (NH == 1 && more && !p_drain()) { bad = true; break; }
+            }
+            // final K state (lag frame at t = L-1) after the last chunk of the last segment
+            if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
+                for (int h = 0; h < NH; ++h)
+                    if (!wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
+                if (!bad) {
+                    tc::tc_fence_after();
+                    const int n_last = g.L - (c_end - 1) * kC;
+                    for (int b = 0; b < g.NB; ++b) {
+                        const int r = b * 128 + row, m = r >> 1;
+                        float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + r) * D : nullptr;
+                        const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
+                        state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
+                    }
                 }
             }
         }
-        // final K state (lag frame at t = L-1) after the last chunk of the last segment
-        if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
-            for (int h = 0; h < NH; ++h)
-                if (!wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
-            if (!bad) {
-                tc::tc_fence_after();
-                const int n_last = g.L - (c_end - 1) * kC;
-                for (int b = 0; b < g.NB; ++b) {
-                    const int r = b * 128 + row, m = r >> 1;
-                    float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + r) * D : nullptr;
-                    const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
-                    state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
-                }
-            }
-        }
-        if (threadIdx.x == 0) tc::bulk_wait0();
     }
     tc::tc_fence_before();
     __syncthreads();
@@ -867,233 +1016,231 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
 
-    if (warp == 8) {
-        if (lane == 0) {
-            tc::tma_prefetch_desc(&tm_p); tc::tma_prefetch_desc(&tm_v);
-            tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
-            uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0;
-            bool first_eb = true, first_phi = true;
-            bool bad = false;
-            for (int c = c_begin; c < c_end && !bad; ++c) {
-                if (c > c_begin && !wait_bar(&bar[VB_PV_FREE], ph_pv, ctl, a.err)) break;
-                tc::mbar_arrive_expect_tx(&bar[VB_PV_FULL], (uint32_t)(kC * SP * 2 + kC * D * 2));
-                for (int kb = 0; kb < SP / 64; ++kb)
-                    tc::tma_load_3d(sPG + kb * kC * 128, &tm_p, &bar[VB_PV_FULL], kb * 64, c * kC, bh);
-                for (int db = 0; db < D / 64; ++db)
-                    tc::tma_load_3d(sV + db * kC * 128, &tm_v, &bar[VB_PV_FULL], db * 64, c * kC, bh);
-                // phase 1: PHI_h and EB_h per half; phase 3: EB_h again per half
-                for (int rep = 0; rep < 2 && !bad; ++rep)
-                    for (int h = 0; h < NH; ++h) {
-                        if (rep == 0) {
-                            if (!first_phi && !wait_bar(&bar[VB_PHI_FREE], ph_phi, ctl, a.err)) { bad = true; break; }
-                            first_phi = false;
-                            tc::mbar_arrive_expect_tx(&bar[VB_PHI_FULL], (uint32_t)(SP * RH * 2));
-                            for (int kb = 0; kb < RH / 64; ++kb)
-                                tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PHI_FULL], h * RH + kb * 64, 0);
+    if (warp >= 8) {
+        if (warp == 8) {
+            if (lane == 0) {
+                tc::tma_prefetch_desc(&tm_p); tc::tma_prefetch_desc(&tm_v);
+                tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
+                uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0;
+                bool first_eb = true, first_phi = true;
+                bool bad = false;
+                for (int c = c_begin; c < c_end && !bad; ++c) {
+                    if (c > c_begin && !wait_bar(&bar[VB_PV_FREE], ph_pv, ctl, a.err)) break;
+                    tc::mbar_arrive_expect_tx(&bar[VB_PV_FULL], (uint32_t)(kC * SP * 2 + kC * D * 2));
+                    for (int kb = 0; kb < SP / 64; ++kb)
+                        tc::tma_load_3d(sPG + kb * kC * 128, &tm_p, &bar[VB_PV_FULL], kb * 64, c * kC, bh);
+                    for (int db = 0; db < D / 64; ++db)
+                        tc::tma_load_3d(sV + db * kC * 128, &tm_v, &bar[VB_PV_FULL], db * 64, c * kC, bh);
+                    // phase 1: PHI_h and EB_h per half; phase 3: EB_h again per half
+                    for (int rep = 0; rep < 2 && !bad; ++rep)
+                        for (int h = 0; h < NH; ++h) {
+                            if (rep == 0) {
+                                if (!first_phi && !wait_bar(&bar[VB_PHI_FREE], ph_phi, ctl, a.err)) { bad = true; break; }
+                                first_phi = false;
+                                tc::mbar_arrive_expect_tx(&bar[VB_PHI_FULL], (uint32_t)(SP * RH * 2));
+                                for (int kb = 0; kb < RH / 64; ++kb)
+                                    tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PHI_FULL], h * RH + kb * 64, 0);
+                            }
+                            if (!first_eb && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) { bad = true; break; }
+                            first_eb = false;
+                            tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
+                            for (int kb = 0; kb < 2; ++kb)
+                                tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, h * 128);
                         }
-                        if (!first_eb && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) { bad = true; break; }
-                        first_eb = false;
-                        tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
-                        for (int kb = 0; kb < 2; ++kb)
-                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, h * 128);
+                }
+            }
+        } else if (warp == 9) {
+            if (lane == 0) {
+                uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0, ph_w = 0;
+                const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
+                const uint32_t id_G = tc::idesc_bf16(128, kC, false, true);
+                const uint32_t id_O = tc::idesc_bf16(128, D, false, true);
+                bool firstU = true, firstG = true;
+                bool bad = false;
+                for (int c = c_begin; c < c_end && !bad; ++c) {
+                    if (!wait_bar(&bar[VB_PV_FULL], ph_pv, ctl, a.err)) break;
+                    // phase 1
+                    for (int h = 0; h < NH; ++h) {
+                        if (!wait_bar(&bar[VB_PHI_FULL], ph_phi, ctl, a.err)) { bad = true; break; }
+                        if (!(firstU && h == 0) && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
+                        tc::tc_fence_after();
+                        mma_steps<true>(tb + colU, sPG, kC, sPHI, SP, id_U, SP / 16, false);
+                        tc::mma_commit(&bar[VB_U_FULL]);
+                        tc::mma_commit(&bar[VB_PHI_FREE]);
+                        if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
+                        if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) { bad = true; break; }
+                        if (h == 0 && !firstG && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) { bad = true; break; }
+                        tc::tc_fence_after();
+                        mma_steps<true>(tb + colG, sA + h * a_tile, kC, sEB, 128, id_G, RH / 16, h > 0);
+                        tc::mma_commit(&bar[VB_EB_FREE]);
                     }
-            }
-        }
-    } else if (warp == 9) {
-        if (lane == 0) {
-            uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0, ph_w = 0;
-            const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
-            const uint32_t id_G = tc::idesc_bf16(128, kC, false, true);
-            const uint32_t id_O = tc::idesc_bf16(128, D, false, true);
-            bool firstU = true, firstG = true;
-            bool bad = false;
-            for (int c = c_begin; c < c_end && !bad; ++c) {
-                if (!wait_bar(&bar[VB_PV_FULL], ph_pv, ctl, a.err)) break;
-                // phase 1
-                for (int h = 0; h < NH; ++h) {
-                    if (!wait_bar(&bar[VB_PHI_FULL], ph_phi, ctl, a.err)) { bad = true; break; }
-                    if (!(firstU && h == 0) && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
+                    firstU = false;
+                    firstG = false;
+                    if (bad) break;
+                    tc::mma_commit(&bar[VB_G_FULL]);
+                    // phase 2: O = G V (G written over p by the epilogue)
+                    if (!wait_bar(&bar[VB_G_READY], ph_gready, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
                     tc::tc_fence_after();
-                    for (int k = 0; k < SP / 16; ++k)
-                        tc::mma_bf16(tb + colU, kmaj_desc(sPG, kC, k), mnmaj_desc(sPHI, SP, k), id_U, k > 0);
-                    tc::mma_commit(&bar[VB_U_FULL]);
-                    tc::mma_commit(&bar[VB_PHI_FREE]);
-                    if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
-                    if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) { bad = true; break; }
-                    if (h == 0 && !firstG && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) { bad = true; break; }
-                    tc::tc_fence_after();
-                    for (int k = 0; k < RH / 16; ++k)
-                        tc::mma_bf16(tb + colG, kmaj_desc(sA + h * a_tile, kC, k), mnmaj_desc(sEB, 128, k), id_G,
-                                     (h > 0 || k > 0) ? 1u : 0u);
-                    tc::mma_commit(&bar[VB_EB_FREE]);
+                    mma_steps<true>(tb + colU, sPG, kC, sV, kC, id_O, kC / 16, false);
+                    // phase 3: O += A'_h W_h ; state_h += EB_h V
+                    for (int h = 0; h < NH; ++h) {
+                        if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
+                        if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
+                        tc::tc_fence_after();
+                        mma_steps<true>(tb + colU, sA + h * a_tile, kC, sW, RH, id_O, RH / 16, true);
+                        tc::mma_commit(&bar[VB_W_FREE]);
+                        mma_steps<true>(tb + h * D, sEB, 128, sV, kC, id_O, kC / 16, true);
+                        tc::mma_commit(&bar[VB_STATE_DONE + h]);
+                        tc::mma_commit(&bar[VB_EB_FREE]);
+                    }
+                    if (bad) break;
+                    tc::mma_commit(&bar[VB_O_FULL]);
+                    tc::mma_commit(&bar[VB_PV_FREE]);
                 }
-                firstU = false;
-                firstG = false;
-                if (bad) break;
-                tc::mma_commit(&bar[VB_G_FULL]);
-                // phase 2: O = G V (G written over p by the epilogue)
-                if (!wait_bar(&bar[VB_G_READY], ph_gready, ctl, a.err)) break;
-                if (!wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
-                tc::tc_fence_after();
-                for (int k = 0; k < kC / 16; ++k)
-                    tc::mma_bf16(tb + colU, kmaj_desc(sPG, kC, k), mnmaj_desc(sV, kC, k), id_O, k > 0);
-                // phase 3: O += A'_h W_h ; state_h += EB_h V
-                for (int h = 0; h < NH; ++h) {
-                    if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
-                    if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
-                    tc::tc_fence_after();
-                    for (int k = 0; k < RH / 16; ++k)
-                        tc::mma_bf16(tb + colU, kmaj_desc(sA + h * a_tile, kC, k), mnmaj_desc(sW, RH, k), id_O, 1);
-                    tc::mma_commit(&bar[VB_W_FREE]);
-                    for (int k = 0; k < kC / 16; ++k)
-                        tc::mma_bf16(tb + h * D, kmaj_desc(sEB, 128, k), mnmaj_desc(sV, kC, k), id_O, 1);
-                    tc::mma_commit(&bar[VB_STATE_DONE + h]);
-                    tc::mma_commit(&bar[VB_EB_FREE]);
-                }
-                if (bad) break;
-                tc::mma_commit(&bar[VB_O_FULL]);
-                tc::mma_commit(&bar[VB_PV_FREE]);
+                tc::mma_commit(&bar[VB_EXIT]);
+                uint32_t ph_exit = 0;
+                tc::mbar_wait(&bar[VB_EXIT], ph_exit);
             }
-            tc::mma_commit(&bar[VB_EXIT]);
-            uint32_t ph_exit = 0;
-            tc::mbar_wait(&bar[VB_EXIT], ph_exit);
         }
     } else {
-        const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
-        const int M = g.M;
-        const float *erel = a.erel;
-        constexpr int XH = RH / 2, DH = D / 2;
-        uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0, ph_sync = 0, ph_ostored = 0;
-        uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
-        // the output tile is staged in A'_0's buffer (idle between the last MMA of a chunk and the
-        // next chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
-        const bool stage_o = NH * RH >= D;
-        const float2 e1 = phase(erel, M, row, 1);
-        const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
-        // per-half constants held in scalars (selected by h) so nothing is indexed at run time
-        const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
-        const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
-        const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
-        const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
-        const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
-        const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
-        const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
-        for (int b = 0; b < g.NB; ++b) {
-            const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
-            state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
-        }
-        bool bad = false;
-        for (int c = c_begin; c < c_end && !bad; ++c) {
-            const int t0 = c * kC;
-            const int n = min(kC, g.L - t0);
-            const bool rot = c > c_begin;
-            // phase 1: U_h -> A'_h, the rotation by -m w t of (sum_j p A, sum_j p B)
-            if (stage_o && c > c_begin && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
-            for (int h = 0; h < NH; ++h) {
-                if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
-                tc::tc_fence_after();
-                float v[XH];
-                tc::tmem_ld<XH>(tmem_addr(tb, lane_base, colU + wg * XH), v);
-                const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
-                    float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
-#pragma unroll
-                for (int i = 0; i < XH; i += 4) {
-                    float uc = v[i], us = v[i + 1];
-                    v[i] = ca * uc + sa * us;
-                    v[i + 1] = ca * us - sa * uc;
-                    uc = v[i + 2];
-                    us = v[i + 3];
-                    v[i + 2] = cb * uc + sb * us;
-                    v[i + 3] = cb * us - sb * uc;
-                    float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
-                    ca = t1;
-                    sa = t2;
-                    t1 = cb * e2.x - sb * e2.y;
-                    t2 = sb * e2.x + cb * e2.y;
-                    cb = t1;
-                    sb = t2;
-                }
-#pragma unroll
-                for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sA + h * a_tile, kC, row, wg * XH + g0, v + g0);
-                tc::fence_proxy_async_smem();
-                tc::tc_fence_before();
-                epi_arrive(&bar[VB_A_READY]);
-                epi_arrive(&bar[VB_U_FREE]);
+        {
+            const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
+            const int M = g.M;
+            const float *erel = a.erel;
+            constexpr int XH = RH / 2, DH = D / 2;
+            uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0, ph_sync = 0, ph_ostored = 0;
+            uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
+            // the output tile is staged in A'_0's buffer (idle between the last MMA of a chunk and the
+            // next chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
+            const bool stage_o = NH * RH >= D;
+            const float2 e1 = phase(erel, M, row, 1);
+            const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
+            // per-half constants held in scalars (selected by h) so nothing is indexed at run time
+            const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
+            const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
+            const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
+            const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
+            const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
+            const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
+            const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
+            for (int b = 0; b < g.NB; ++b) {
+                const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
+                state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
             }
-            if (bad) break;
-            // phase 2: G drain -> causal mask -> bf16 over p's tile
-            if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
-            tc::tc_fence_after();
-            {
-                float v[64];
-                tc::tmem_ld<64>(tmem_addr(tb, lane_base, colG + wg * 64), v);
+            bool bad = false;
+            for (int c = c_begin; c < c_end && !bad; ++c) {
+                const int t0 = c * kC;
+                const int n = min(kC, g.L - t0);
+                const bool rot = c > c_begin;
+                // phase 1: U_h -> A'_h, the rotation by -m w t of (sum_j p A, sum_j p B)
+                if (stage_o && c > c_begin && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
+                for (int h = 0; h < NH; ++h) {
+                    if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    float v[XH];
+                    tc::tmem_ld<XH>(tmem_addr(tb, lane_base, colU + wg * XH), v);
+                    const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
+                        float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
 #pragma unroll
-                for (int i = 0; i < 64; ++i)
-                    if (wg * 64 + i > row) v[i] = 0.f;
+                    for (int i = 0; i < XH; i += 4) {
+                        float uc = v[i], us = v[i + 1];
+                        v[i] = ca * uc + sa * us;
+                        v[i + 1] = ca * us - sa * uc;
+                        uc = v[i + 2];
+                        us = v[i + 3];
+                        v[i + 2] = cb * uc + sb * us;
+                        v[i + 3] = cb * us - sb * uc;
+                        float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
+                        ca = t1;
+                        sa = t2;
+                        t1 = cb * e2.x - sb * e2.y;
+                        t2 = sb * e2.x + cb * e2.y;
+                        cb = t1;
+                        sb = t2;
+                    }
 #pragma unroll
-                for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(sPG, kC, row, wg * 64 + g0, v + g0);
-            }
-            tc::fence_proxy_async_smem();
-            tc::tc_fence_before();
-            epi_arrive(&bar[VB_G_READY]);
-            epi_arrive(&bar[VB_G_FREE]);
-            // phase 3: W_h (the V state read before this chunk's update)
-            for (int h = 0; h < NH; ++h) {
-                if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
-                if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
-                tc::tc_fence_after();
-                state_pass<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, rot, sW, RH, nullptr, wg * DH);
-                tc::fence_proxy_async_smem();
-                tc::tc_fence_before();
-                epi_arrive(&bar[VB_W_READY]);
-            }
-            if (bad) break;
-            if (!wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) break;
-            // phase 4: O drain -> global
-            if (!wait_bar(&bar[VB_O_FULL], ph_o, ctl, a.err)) break;
-            tc::tc_fence_after();
-            {
-                float v[DH];
-                tc::tmem_ld<DH>(tmem_addr(tb, lane_base, colU + wg * DH), v);
-                tc::tc_fence_before();
-                epi_arrive(&bar[VB_U_FREE]);
-                if (stage_o) {
-#pragma unroll
-                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16(sA, kC, row, wg * DH + g0, v + g0);
+                    for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sA + h * a_tile, kC, row, wg * XH + g0, v + g0);
                     tc::fence_proxy_async_smem();
-                    if (!epi_sync(&bar[VB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
-                    if (threadIdx.x == 0) {
-                        for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sA + db * kC * 128, db * 64, t0, bh);
-                        tc::bulk_commit();
-                        tc::bulk_wait_read0();
-                        tc::mbar_arrive(&bar[VB_O_STORED]);
-                    }
-                } else if (row < n) {
-                    bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D + wg * DH;
-#pragma unroll
-                    for (int j = 0; j < DH; j += 8) {
-                        uint4 pk = make_uint4(tc::pack_bf16x2(v[j], v[j + 1]), tc::pack_bf16x2(v[j + 2], v[j + 3]),
-                                              tc::pack_bf16x2(v[j + 4], v[j + 5]), tc::pack_bf16x2(v[j + 6], v[j + 7]));
-                        *reinterpret_cast<uint4 *>(orow + j) = pk;
-                    }
+                    tc::tc_fence_before();
+                    epi_arrive(&bar[VB_A_READY]);
+                    epi_arrive(&bar[VB_U_FREE]);
                 }
-            }
-        }
-        if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
-            for (int h = 0; h < NH; ++h)
-                if (!wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
-            if (!bad) {
+                if (bad) break;
+                // phase 2: G drain -> causal mask -> bf16 over p's tile
+                if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
                 tc::tc_fence_after();
-                const int n_last = g.L - (c_end - 1) * kC;
-                for (int b = 0; b < g.NB; ++b) {
-                    const int r = b * 128 + row, m = r >> 1;
-                    float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + g.R2 + r) * D : nullptr;
-                    const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
-                    state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
+                {
+                    float v[64];
+                    tc::tmem_ld<64>(tmem_addr(tb, lane_base, colG + wg * 64), v);
+#pragma unroll
+                    for (int i = 0; i < 64; ++i)
+                        if (wg * 64 + i > row) v[i] = 0.f;
+#pragma unroll
+                    for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(sPG, kC, row, wg * 64 + g0, v + g0);
+                }
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                epi_arrive(&bar[VB_G_READY]);
+                epi_arrive(&bar[VB_G_FREE]);
+                // phase 3: W_h (the V state read before this chunk's update)
+                for (int h = 0; h < NH; ++h) {
+                    if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
+                    if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
+                    tc::tc_fence_after();
+                    state_pass<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, rot, sW, RH, nullptr, wg * DH);
+                    tc::fence_proxy_async_smem();
+                    tc::tc_fence_before();
+                    epi_arrive(&bar[VB_W_READY]);
+                }
+                if (bad) break;
+                if (!wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) break;
+                // phase 4: O drain -> global
+                if (!wait_bar(&bar[VB_O_FULL], ph_o, ctl, a.err)) break;
+                tc::tc_fence_after();
+                {
+                    float v[DH];
+                    tc::tmem_ld<DH>(tmem_addr(tb, lane_base, colU + wg * DH), v);
+                    tc::tc_fence_before();
+                    epi_arrive(&bar[VB_U_FREE]);
+                    if (stage_o) {
+#pragma unroll
+                        for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16(sA, kC, row, wg * DH + g0, v + g0);
+                        tc::fence_proxy_async_smem();
+                        if (!epi_sync(&bar[VB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
+                        if (threadIdx.x == 0) {
+                            for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sA + db * kC * 128, db * 64, t0, bh);
+                            tc::bulk_commit();
+                            tc::bulk_wait_read0();
+                            tc::mbar_arrive(&bar[VB_O_STORED]);
+                        }
+                    } else if (row < n) {
+                        bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D + wg * DH;
+#pragma unroll
+                        for (int j = 0; j < DH; j += 8) {
+                            uint4 pk = make_uint4(tc::pack_bf16x2(v[j], v[j + 1]), tc::pack_bf16x2(v[j + 2], v[j + 3]),
+                                                  tc::pack_bf16x2(v[j + 4], v[j + 5]), tc::pack_bf16x2(v[j + 6], v[j + 7]));
+                            *reinterpret_cast<uint4 *>(orow + j) = pk;
+                        }
+                    }
                 }
             }
+            if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
+                for (int h = 0; h < NH; ++h)
+                    if (!wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
+                if (!bad) {
+                    tc::tc_fence_after();
+                    const int n_last = g.L - (c_end - 1) * kC;
+                    for (int b = 0; b < g.NB; ++b) {
+                        const int r = b * 128 + row, m = r >> 1;
+                        float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + g.R2 + r) * D : nullptr;
+                        const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
+                        state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
+                    }
+                }
+            }
+            if (threadIdx.x == 0) tc::bulk_wait0();
         }
-        if (threadIdx.x == 0) tc::bulk_wait0();
     }
     tc::tc_fence_before();
     __syncthreads();
@@ -1150,12 +1297,23 @@ static int smem_request(size_t bytes, int tmem_cols) {
 
 static int pow2_cols(int n) { return n <= 32 ? 32 : n <= 64 ? 64 : n <= 128 ? 128 : n <= 256 ? 256 : 512; }
 
+// The pass kernels move registers between warpgroups (setmaxnreg); an increase that the launch
+// cannot cover would wait forever, so launch only if every thread starts with kLaunchRegs.
+static cudaError_t check_register_split(const void *fn) {
+    cudaFuncAttributes fa;
+    cudaError_t e = cudaFuncGetAttributes(&fa, fn);
+    if (e != cudaSuccess) return e;
+    if (fa.numRegs < kLaunchRegs || fa.maxThreadsPerBlock < kPassThreads) return cudaErrorLaunchOutOfResources;
+    return cudaSuccess;
+}
+
 
 template <int D, int RH, int S, int NH>
 static cudaError_t launch_kpass_n(int smem, int nblk, cudaStream_t st, const CUtensorMap &tq, const CUtensorMap &tk,
                                   const CUtensorMap &teb, const CUtensorMap &tphi, const CUtensorMap &tp, const Args &a) {
     cudaError_t e = cudaFuncSetAttribute(k_kpass<D, RH, S, NH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
+    if ((e = check_register_split((const void *)k_kpass<D, RH, S, NH>)) != cudaSuccess) return e;
     ProfScope ps(BLA_K_KPASS, st);
     k_kpass<D, RH, S, NH><<<nblk, kPassThreads, smem, st>>>(tq, tk, teb, tphi, tp, a);
     return cudaGetLastError();
