@@ -80,7 +80,7 @@ WsLayout ws_layout(const OpDims &d, const Geo &g) {
     WsLayout w;
     size_t off = 0;
     w.tables = off; off += tables_bytes(d, kC);
-    w.eb = off;     off += align_up(sizeof(bf16) * (size_t)g.RP * kC, 1024);
+    w.eb = off;     off += align_up(sizeof(bf16) * (size_t)g.nchunks * g.RP * kC, 1024);   // EB per chunk
     w.phi = off;    off += align_up(sizeof(bf16) * (size_t)g.SP * g.R2, 1024);
     w.fseg = off;   off += g.G > 1 ? align_up(sizeof(bf16) * (size_t)g.RP * g.Lseg, 1024) : 0;
     w.deltas = off; off += g.G > 1 ? align_up(sizeof(float) * (size_t)g.BH * g.G * 2 * g.RP * g.D, 1024) : 0;
@@ -98,7 +98,7 @@ WsLayout ws_layout(const OpDims &d, const Geo &g) {
 // exactly, 2 pi ((m u) mod T) / T, and evaluated by sincospi in fp32; otherwise in fp64.
 __device__ __forceinline__ void mode_phase(long long mu, double w, int tint, float *c, float *s) {
     if (tint > 0) {
-        const long long kk = mu % tint;
+        const int kk = mu < 0x7fffffffLL ? (int)((unsigned)mu % (unsigned)tint) : (int)(mu % tint);
         sincospif(2.0f * (float)kk / (float)tint, s, c);
     } else {
         double sd, cd;
@@ -149,6 +149,42 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, double T, 
             }
             fseg[e] = __float2bfloat16_rn(v);
         }
+    }
+}
+
+// Per-chunk EB for the forward passes, whose states are kept in the absolute frame:
+//   EB_c [RP][C]: EB_c[2m][u] = cos(m w (cC + u)), EB_c[2m+1][u] = -sin(m w (cC + u)), rows >= 2M zero.
+// One thread per (c, m, 8 consecutive u), u fastest so that a warp writes whole rows: the first
+// phase is reduced exactly (mode_phase), the next seven follow by products with e^{i m w}.
+__global__ void k_eb_chunks(int M, int RP, int nch, double w, int tint, bf16 *ebc) {
+    const int MP = RP / 2;
+    const long long per_c = (long long)MP * (kC / 8);
+    const long long total = (long long)nch * per_c;
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
+         i += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(i / per_c), rem = (int)(i % per_c);
+        const int m = rem / (kC / 8), u0 = (rem % (kC / 8)) * 8;
+        bf16 *rc = ebc + ((size_t)c * RP + 2 * m) * kC + u0, *rs = rc + kC;
+        uint32_t wc[4] = {0u, 0u, 0u, 0u}, ws[4] = {0u, 0u, 0u, 0u};
+        if (m < M) {
+            float bc, bs, ec, es;
+            mode_phase((long long)m * ((long long)c * kC + u0), w, tint, &bc, &bs);
+            mode_phase((long long)m, w, tint, &ec, &es);
+#pragma unroll
+            for (int j = 0; j < 8; j += 2) {
+                const float c0 = bc, s0 = bs;
+                float t = bc * ec - bs * es;
+                bs = bc * es + bs * ec;
+                bc = t;
+                wc[j / 2] = tc::pack_bf16x2(c0, bc);
+                ws[j / 2] = tc::pack_bf16x2(-s0, -bs);
+                t = bc * ec - bs * es;
+                bs = bc * es + bs * ec;
+                bc = t;
+            }
+        }
+        *reinterpret_cast<uint4 *>(rc) = make_uint4(wc[0], wc[1], wc[2], wc[3]);
+        *reinterpret_cast<uint4 *>(rs) = make_uint4(ws[0], ws[1], ws[2], ws[3]);
     }
 }
 
@@ -247,27 +283,72 @@ __device__ __forceinline__ uint64_t mnmaj_desc(const uint8_t *tile, int krows, i
     return tc::sdesc_sw128(a, (uint32_t)krows * 128u, 1024);
 }
 
-// Load DH columns of this thread's state row from TMEM, optionally rotate them by the phase
-// (c, s) of its mode (partner row = lane ^ 1) and write them back, and pack them to bf16 pairs.
+// (cos, sin)(m w t) for the product mt = m t, reduced exactly when w = 2 pi / tint.
+__device__ __forceinline__ float2 abs_phase(long long mt, double w, int tint) {
+    float c, s;
+    mode_phase(mt, w, tint, &c, &s);
+    return make_float2(c, s);
+}
+
+__device__ __forceinline__ float2 cmul(float2 a, float2 b) {
+    return make_float2(a.x * b.x - a.y * b.y, a.x * b.y + a.y * b.x);
+}
+
+// Phases of token t for the drains of one chunk: e^{i m0 w t} for the first mode of this thread's
+// range in each half (h0, h1), e^{i w t} (start offset of the second interleaved chain) and
+// e^{i 2 w t} (step of both chains).
+struct RowPhases {
+    float2 e1, e2, h0, h1;
+};
+__device__ __forceinline__ RowPhases row_phases(long long t, int m00, int m10, bool two, double w, int tint) {
+    RowPhases p;
+    p.e1 = abs_phase(t, w, tint);
+    p.e2 = abs_phase(2 * t, w, tint);
+    p.h0 = abs_phase((long long)m00 * t, w, tint);
+    p.h1 = two ? abs_phase((long long)m10 * t, w, tint) : make_float2(1.f, 0.f);
+    return p;
+}
+// The phases of token t + C from those of t and the phases of C (one complex product each; over
+// the chunks of one segment the rounding stays orders of magnitude below bf16 resolution).
+__device__ __forceinline__ void advance(RowPhases &p, const RowPhases &step) {
+    p.e1 = cmul(p.e1, step.e1);
+    p.e2 = cmul(p.e2, step.e2);
+    p.h0 = cmul(p.h0, step.h0);
+    p.h1 = cmul(p.h1, step.h1);
+}
+
+// Initial state block in the absolute frame: the carried-in lag-frame state S (rows [rows][stride],
+// interleaved (Re, Im) row pairs; null = zero) rotated to A = e^{-i m w t0} S, written to TMEM.
+// (c, s) = (cos, sin)(m w t0) of this thread's mode; the partner row is read from global memory.
 template <int DH>
-__device__ __forceinline__ void state_rotate_pack(uint32_t tbase, int col0, int row, bool rotate, float c, float s,
-                                                  uint32_t *pk) {
+__device__ __forceinline__ void state_init_abs(uint32_t tbase, int col0, int row, const float *src, int live_rows,
+                                               int stride, float c, float s) {
     const int lane_base = (row >> 5) << 5;
-    const bool odd = row & 1;
-    // 32-column pieces keep the loaded values and their partners within the register budget
+    const float sg = (row & 1) ? -s : s;   // Re' = c Re + s Im ; Im' = c Im - s Re
+    float v[DH];
+#pragma unroll
+    for (int i = 0; i < DH; i += 4) {
+        float4 own = make_float4(0.f, 0.f, 0.f, 0.f), par = own;
+        if (src && row < live_rows) {
+            own = *reinterpret_cast<const float4 *>(src + (size_t)row * stride + i);
+            par = *reinterpret_cast<const float4 *>(src + (size_t)(row ^ 1) * stride + i);
+        }
+        v[i] = c * own.x + sg * par.x;
+        v[i + 1] = c * own.y + sg * par.y;
+        v[i + 2] = c * own.z + sg * par.z;
+        v[i + 3] = c * own.w + sg * par.w;
+    }
+    tc::tmem_st<DH>(tmem_addr(tbase, lane_base, col0), v);
+}
+
+// Load DH columns of this thread's state row from TMEM and pack them to bf16 pairs.
+template <int DH>
+__device__ __forceinline__ void state_pack(uint32_t tbase, int col0, int row, uint32_t *pk) {
+    const int lane_base = (row >> 5) << 5;
 #pragma unroll
     for (int p0 = 0; p0 < DH; p0 += 32) {
-        const uint32_t addr = tmem_addr(tbase, lane_base, col0 + p0);
         float v[32];
-        tc::tmem_ld<32>(addr, v);
-        if (rotate) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) {
-                const float partner = __shfl_xor_sync(0xffffffffu, v[i], 1);
-                v[i] = odd ? fmaf(s, partner, c * v[i]) : fmaf(-s, partner, c * v[i]);
-            }
-            tc::tmem_st<32>(addr, v);
-        }
+        tc::tmem_ld<32>(tmem_addr(tbase, lane_base, col0 + p0), v);
 #pragma unroll
         for (int i = 0; i < 32; i += 2) pk[(p0 + i) / 2] = tc::pack_bf16x2(v[i], v[i + 1]);
     }
@@ -342,27 +423,6 @@ __device__ __forceinline__ void state_pass(uint32_t tbase, int col0, int row, bo
         for (int i = 0; i < D; i += 4)
             *reinterpret_cast<float4 *>(gout + ccol + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
     }
-}
-
-// Load 128 rows x D fp32 (global, row stride D) into a TMEM state block; rows at or beyond
-// `live_rows` (padding beyond 2M) and a NULL source give zeros.
-template <int D>
-__device__ __forceinline__ void state_init(uint32_t tbase, int col0, int row, const float *src, int live_rows,
-                                           int stride = D) {
-    const int lane_base = (row >> 5) << 5;
-    float v[D];
-#pragma unroll
-    for (int i = 0; i < D; i += 4) {
-        float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
-        if (src && row < live_rows) t = *reinterpret_cast<const float4 *>(src + (size_t)row * stride + i);
-        v[i] = t.x; v[i + 1] = t.y; v[i + 2] = t.z; v[i + 3] = t.w;
-    }
-    tc::tmem_st<D>(tmem_addr(tbase, lane_base, col0), v);
-}
-
-// Phase (cos, sin)(m w tau) from the fp32 table [C+1][M][2].
-__device__ __forceinline__ float2 phase(const float *erel, int M, int tau, int m) {
-    return make_float2(erel[((size_t)tau * M + m) * 2], erel[((size_t)tau * M + m) * 2 + 1]);
 }
 
 // ================================================================== prepass
@@ -594,7 +654,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         first_eb = false;
                         tc::mbar_arrive_expect_tx(&bar[KB_EB_FULL], (uint32_t)(128 * kC * 2));
                         for (int kb = 0; kb < 2; ++kb)
-                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[KB_EB_FULL], kb * 64, h * 128);
+                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[KB_EB_FULL], kb * 64, c * g.RP + h * 128);
                         if (!first_phi && !wait_bar(&bar[KB_PHI_FREE], ph_phi, ctl, a.err)) break;
                         first_phi = false;
                         tc::mbar_arrive_expect_tx(&bar[KB_PHI_FULL], (uint32_t)(SP * RH * 2));
@@ -721,33 +781,27 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             uint32_t ph_fullA = 0, ph_fullB = 0, ph_wfree = 0, ph_yfree = 0, ph_sync = 0, ph_ystored = 0;
             uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
             const int M = g.M;
-            const float *erel = a.erel;
             constexpr int XH = RH / 2;        // X columns per warpgroup (XH/2 modes)
             constexpr int DH = D / 2;         // state columns per warpgroup
             constexpr int SH = S >= 64 ? S / 2 : S;   // slot columns per warpgroup (S = 32: warpgroup 0 only)
-            // phase constants of this thread, fixed for the whole CTA: e^{i 2 w t} (two interleaved
-            // mode chains), the start phases of its mode range in each half, e^{i m w C} of its state row
-            const float2 e1 = phase(erel, M, row, 1);
-            const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
-            // per-half constants held in scalars (selected by h) so nothing is indexed at run time
+            // first mode of this thread's range in each half (two interleaved chains per range), and
+            // the drain phases of this row: exact at the CTA's first chunk, then advanced per chunk
             const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
-            const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
-            const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
-            const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
-            const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
-            const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
-            const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
+            RowPhases rp = row_phases((long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
+            const RowPhases rp_step = row_phases(kC, m00, m10, NH == 2, a.w, a.tint);
+            // the state is kept in the absolute frame, A = sum_{u < t0} e^{-i m w u} k_u: it needs no
+            // rotation between chunks; the carried-in lag-frame state is rotated once
             for (int b = 0; b < g.NB; ++b) {
                 const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
-                state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
+                const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
+                state_init_abs<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D, f.x, f.y);
             }
-            // W_h: state block h (W + EB K of the previous chunk) rotated by e^{i m w C} into the state
-            // carried into the next chunk and written back (w_compute, into packed bf16 registers);
-            // then copied into the W tile once the MMA that read the previous W_h' is done (w_store).
-            auto w_compute = [&](int h, bool rot, uint32_t *pk) -> bool {
-                if (rot && !wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) return false;
+            // W_h: state block h after the previous chunk's update, packed to bf16 in registers
+            // (w_compute); copied into the W tile once the MMA that read the previous W is done (w_store).
+            auto w_compute = [&](int h, bool wait_update, uint32_t *pk) -> bool {
+                if (wait_update && !wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) return false;
                 tc::tc_fence_after();
-                state_rotate_pack<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, pk);
+                state_pack<DH>(tb, h * D + wg * DH, row, pk);
                 return true;
             };
             auto w_store = [&](bool wait_free, const uint32_t *pk) -> bool {
@@ -761,11 +815,12 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 epi_arrive(&bar[KB_W_READY]);
                 return true;
             };
-            // Y_h = e^{i m w t} X_h (t = row) from accumulator region `col`, two interleaved mode chains
-            auto y_drain = [&](int h, int col) {
+            // Y_h = e^{i m w t} X_h (t = absolute token of this row) from accumulator region `col`,
+            // two interleaved mode chains
+            auto y_drain = [&](int h, int col, const RowPhases &rp) {
                 float v[XH];
                 tc::tmem_ld<XH>(tmem_addr(tb, lane_base, col + wg * XH), v);
-                const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
+                const float2 pa = h ? rp.h1 : rp.h0, pb = cmul(pa, rp.e1), e2 = rp.e2;
                 float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
 #pragma unroll
                 for (int i = 0; i < XH; i += 4) {
@@ -821,20 +876,21 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 const int t0 = c * kC;
                 const int n = min(kC, g.L - t0);
                 const bool rot = c > c_begin, more = c + 1 < c_end;
+                if (rot) advance(rp, rp_step);
                 // W_1 (computed at the end of the previous chunk) once Q W_0^T has read W_0
                 if (NH == 2 && !w_store(true, pk1)) { bad = true; break; }
                 // Y_0 from B; the previous chunk's probabilities must have left the Y tile
                 if (!wait_bar(&bar[KB_ACC_FULL_B], ph_fullB, ctl, a.err)) { bad = true; break; }
                 if (rot && !wait_bar(&bar[KB_Y_STORED], ph_ystored, ctl, a.err)) { bad = true; break; }
                 tc::tc_fence_after();
-                y_drain(0, colB);
+                y_drain(0, colB, rp);
                 epi_arrive(&bar[KB_ACC_FREE_B]);
                 if (NH == 2) {
                     // Y_1 from A once s_0 has read Y_0
                     if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
                     if (!wait_bar(&bar[KB_Y_FREE], ph_yfree, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
-                    y_drain(1, colA);
+                    y_drain(1, colA, rp);
                     epi_arrive(&bar[KB_ACC_FREE_A]);
                 }
                 // W_0 of the next chunk (stored once Q W_1^T, or with one half Q W_0^T, has read the W
@@ -930,11 +986,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     if (!wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
                 if (!bad) {
                     tc::tc_fence_after();
-                    const int n_last = g.L - (c_end - 1) * kC;
                     for (int b = 0; b < g.NB; ++b) {
                         const int r = b * 128 + row, m = r >> 1;
                         float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + r) * D : nullptr;
-                        const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
+                        const float2 f = (m < M) ? abs_phase((long long)m * (g.L - 1), a.w, a.tint) : make_float2(1.f, 0.f);
                         state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
                     }
                 }
@@ -1045,7 +1100,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                             first_eb = false;
                             tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
                             for (int kb = 0; kb < 2; ++kb)
-                                tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, h * 128);
+                                tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP + h * 128);
                         }
                 }
             }
@@ -1107,41 +1162,37 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         {
             const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
             const int M = g.M;
-            const float *erel = a.erel;
             constexpr int XH = RH / 2, DH = D / 2;
             uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0, ph_sync = 0, ph_ostored = 0;
             uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
             // the output tile is staged in A'_0's buffer (idle between the last MMA of a chunk and the
             // next chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
             const bool stage_o = NH * RH >= D;
-            const float2 e1 = phase(erel, M, row, 1);
-            const float2 e2 = make_float2(e1.x * e1.x - e1.y * e1.y, 2.f * e1.x * e1.y);
-            // per-half constants held in scalars (selected by h) so nothing is indexed at run time
+            // first mode of this thread's range in each half, and the drain phases of this row
             const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
-            const float2 ph0_0 = phase(erel, M, row, m00), ph1_0 = phase(erel, M, row, m00 + 1);
-            const float2 ph0_1 = (NH > 1) ? phase(erel, M, row, m10) : make_float2(1.f, 0.f);
-            const float2 ph1_1 = (NH > 1) ? phase(erel, M, row, m10 + 1) : make_float2(1.f, 0.f);
-            const int mr0 = row >> 1, mr1 = (128 + row) >> 1;
-            const float2 rotC_0 = (mr0 < M) ? phase(erel, M, kC, mr0) : make_float2(1.f, 0.f);
-            const float2 rotC_1 = (g.NB > 1 && mr1 < M) ? phase(erel, M, kC, mr1) : make_float2(1.f, 0.f);
+            RowPhases rp = row_phases((long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
+            const RowPhases rp_step = row_phases(kC, m00, m10, NH == 2, a.w, a.tint);
+            // V state in the absolute frame (see the K pass)
             for (int b = 0; b < g.NB; ++b) {
                 const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
-                state_init<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D);
+                const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
+                state_init_abs<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D, f.x, f.y);
             }
             bool bad = false;
             for (int c = c_begin; c < c_end && !bad; ++c) {
                 const int t0 = c * kC;
                 const int n = min(kC, g.L - t0);
                 const bool rot = c > c_begin;
-                // phase 1: U_h -> A'_h, the rotation by -m w t of (sum_j p A, sum_j p B)
+                if (rot) advance(rp, rp_step);
+                // phase 1: U_h -> A'_h, the rotation by -m w t (t absolute) of (sum_j p A, sum_j p B)
                 if (stage_o && c > c_begin && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
                 for (int h = 0; h < NH; ++h) {
                     if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
                     float v[XH];
                     tc::tmem_ld<XH>(tmem_addr(tb, lane_base, colU + wg * XH), v);
-                    const float2 pa = h ? ph0_1 : ph0_0, pb = h ? ph1_1 : ph1_0;
-                        float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
+                    const float2 pa = h ? rp.h1 : rp.h0, pb = cmul(pa, rp.e1), e2 = rp.e2;
+                    float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
 #pragma unroll
                     for (int i = 0; i < XH; i += 4) {
                         float uc = v[i], us = v[i + 1];
@@ -1188,7 +1239,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
                     if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
-                    state_pass<DH>(tb, h * D + wg * DH, row, rot, (h ? rotC_1 : rotC_0).x, (h ? rotC_1 : rotC_0).y, rot, sW, RH, nullptr, wg * DH);
+                    state_pass<DH>(tb, h * D + wg * DH, row, false, 1.f, 0.f, false, sW, RH, nullptr, wg * DH);
                     tc::fence_proxy_async_smem();
                     tc::tc_fence_before();
                     epi_arrive(&bar[VB_W_READY]);
@@ -1230,11 +1281,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     if (!wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
                 if (!bad) {
                     tc::tc_fence_after();
-                    const int n_last = g.L - (c_end - 1) * kC;
                     for (int b = 0; b < g.NB; ++b) {
                         const int r = b * 128 + row, m = r >> 1;
                         float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + g.R2 + r) * D : nullptr;
-                        const float2 f = (m < M) ? phase(erel, M, n_last - 1, m) : make_float2(1.f, 0.f);
+                        const float2 f = (m < M) ? abs_phase((long long)m * (g.L - 1), a.w, a.tint) : make_float2(1.f, 0.f);
                         state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
                     }
                 }
@@ -1405,6 +1455,14 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
         k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, d.T, d.w, integer_period(d), eb, phi, fseg);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
+    {
+        // EB of every chunk (absolute phases) over the single-chunk table written above
+        const long long total = (long long)g.nchunks * (g.RP / 2) * (kC / 8);
+        const int blocks = (int)(total < 4096 * 256 ? (total + 255) / 256 : 4096);
+        ProfScope ps(BLA_K_TABLES_BF16, st);
+        k_eb_chunks<<<blocks, 256, 0, st>>>(g.M, g.RP, g.nchunks, d.w, integer_period(d), eb);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     Args a;
     a.g = g;
     a.scale = d.scale;
@@ -1429,7 +1487,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     const uint32_t bx[3] = {64, 64, 1};
     const uint64_t dp[3] = {(uint64_t)g.SP, (uint64_t)g.L, (uint64_t)g.BH};
     const uint64_t sp[2] = {(uint64_t)g.SP * 2, (uint64_t)g.L * g.SP * 2};
-    const uint64_t deb[2] = {(uint64_t)kC, (uint64_t)g.RP}, seb[1] = {(uint64_t)kC * 2};
+    const uint64_t deb[2] = {(uint64_t)kC, (uint64_t)g.nchunks * g.RP}, seb[1] = {(uint64_t)kC * 2};
     const uint32_t beb[2] = {64, 128};
     const uint64_t dph[2] = {(uint64_t)g.R2, (uint64_t)g.SP}, sph[1] = {(uint64_t)g.R2 * 2};
     const uint32_t bph[2] = {64, (uint32_t)g.SP};
