@@ -1028,7 +1028,7 @@ __host__ __device__ inline VLayout v_layout(const Geo &g) {
 enum VBar {
     VB_PV_FULL, VB_PV_FREE, VB_EB_FULL, VB_EB_FREE, VB_PHI_FULL, VB_PHI_FREE,
     VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_G_READY, VB_W_READY, VB_W_FREE,
-    VB_STATE_DONE, VB_STATE_DONE1, VB_O_FULL, VB_EPI_SYNC, VB_O_STORED, VB_EXIT, VB_COUNT
+    VB_STATE_DONE, VB_STATE_DONE1, VB_STATE_READ, VB_O_FULL, VB_O_SMEM, VB_O_STORED, VB_EXIT, VB_COUNT
 };
 
 template <int D, int RH, int NH>
@@ -1050,6 +1050,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int SP = g.SP;
     const size_t a_tile = (size_t)kC * RH * 2;
+    // the output tile is staged in A'_0's buffer (idle between the chunk's last MMA and the next
+    // chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
+    const bool stage_o = NH * RH >= D;
     // TMEM: [0, NB*D) state; colU (128 cols: U_h, then O); colG (128 cols).
     const int colU = g.NB * D, colG = colU + 128;
     const uint32_t ncols = (uint32_t)(colG + 128) <= 256 ? 256u : 512u;  // host: pow2_cols(NB*D + 256)
@@ -1057,7 +1060,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < VB_COUNT; ++i) {
             const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_G_READY || i == VB_W_READY ||
-                             i == VB_EPI_SYNC;
+                             i == VB_STATE_READ || i == VB_O_SMEM;
             tc::mbar_init(&bar[i], epi ? kPassEpiWarps : 1);
         }
         ctl->abort = 0;
@@ -1073,6 +1076,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 
     if (warp >= 8) {
         if (warp == 8) {
+            // ---------------- TMA producer: per chunk p and V, then PHI_0, EB_0, PHI_1, EB_1 in the
+            // order the MMA issuer consumes them
             if (lane == 0) {
                 tc::tma_prefetch_desc(&tm_p); tc::tma_prefetch_desc(&tm_v);
                 tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
@@ -1086,70 +1091,72 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         tc::tma_load_3d(sPG + kb * kC * 128, &tm_p, &bar[VB_PV_FULL], kb * 64, c * kC, bh);
                     for (int db = 0; db < D / 64; ++db)
                         tc::tma_load_3d(sV + db * kC * 128, &tm_v, &bar[VB_PV_FULL], db * 64, c * kC, bh);
-                    // phase 1: PHI_h and EB_h per half; phase 3: EB_h again per half
-                    for (int rep = 0; rep < 2 && !bad; ++rep)
-                        for (int h = 0; h < NH; ++h) {
-                            if (rep == 0) {
-                                if (!first_phi && !wait_bar(&bar[VB_PHI_FREE], ph_phi, ctl, a.err)) { bad = true; break; }
-                                first_phi = false;
-                                tc::mbar_arrive_expect_tx(&bar[VB_PHI_FULL], (uint32_t)(SP * RH * 2));
-                                for (int kb = 0; kb < RH / 64; ++kb)
-                                    tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PHI_FULL], h * RH + kb * 64, 0);
-                            }
-                            if (!first_eb && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) { bad = true; break; }
-                            first_eb = false;
-                            tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
-                            for (int kb = 0; kb < 2; ++kb)
-                                tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP + h * 128);
-                        }
+                    for (int h = 0; h < NH; ++h) {
+                        if (!first_phi && !wait_bar(&bar[VB_PHI_FREE], ph_phi, ctl, a.err)) { bad = true; break; }
+                        first_phi = false;
+                        tc::mbar_arrive_expect_tx(&bar[VB_PHI_FULL], (uint32_t)(SP * RH * 2));
+                        for (int kb = 0; kb < RH / 64; ++kb)
+                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PHI_FULL], h * RH + kb * 64, 0);
+                        if (!first_eb && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) { bad = true; break; }
+                        first_eb = false;
+                        tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
+                        for (int kb = 0; kb < 2; ++kb)
+                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP + h * 128);
+                    }
                 }
             }
         } else if (warp == 9) {
+            // ---------------- MMA issuer.  Per chunk and half h: U_h = p PHI_h -> U; once A'_h is
+            // drained, G (+)= A'_h EB_h -> G and state_h += EB_h V (EB_h is loaded once for both).
+            // Then O = A'_0 W_0 (+ A'_1 W_1) + G V -> U.
             if (lane == 0) {
                 uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0, ph_w = 0;
+                uint32_t ph_sread = 0;
                 const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
                 const uint32_t id_G = tc::idesc_bf16(128, kC, false, true);
                 const uint32_t id_O = tc::idesc_bf16(128, D, false, true);
-                bool firstU = true, firstG = true;
+                const uint32_t accU = tb + colU, accG = tb + colG;
                 bool bad = false;
                 for (int c = c_begin; c < c_end && !bad; ++c) {
+                    const bool first = c == c_begin;
                     if (!wait_bar(&bar[VB_PV_FULL], ph_pv, ctl, a.err)) break;
-                    // phase 1
                     for (int h = 0; h < NH; ++h) {
+                        // U_h -> U: last read by the previous chunk's O drain, or by A'_0's drain
                         if (!wait_bar(&bar[VB_PHI_FULL], ph_phi, ctl, a.err)) { bad = true; break; }
-                        if (!(firstU && h == 0) && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
+                        if (!(first && h == 0) && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
                         tc::tc_fence_after();
-                        mma_steps<true>(tb + colU, sPG, kC, sPHI, SP, id_U, SP / 16, false);
+                        mma_steps<true>(accU, sPG, kC, sPHI, SP, id_U, SP / 16, false);
                         tc::mma_commit(&bar[VB_U_FULL]);
                         tc::mma_commit(&bar[VB_PHI_FREE]);
+                        // G (+)= A'_h EB_h once A'_h is in shared memory (G: last read by the previous
+                        // chunk's G drain)
                         if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
                         if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) { bad = true; break; }
-                        if (h == 0 && !firstG && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) { bad = true; break; }
+                        if (h == 0 && !first && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) { bad = true; break; }
                         tc::tc_fence_after();
-                        mma_steps<true>(tb + colG, sA + h * a_tile, kC, sEB, 128, id_G, RH / 16, h > 0);
-                        tc::mma_commit(&bar[VB_EB_FREE]);
-                    }
-                    firstU = false;
-                    firstG = false;
-                    if (bad) break;
-                    tc::mma_commit(&bar[VB_G_FULL]);
-                    // phase 2: O = G V (G written over p by the epilogue)
-                    if (!wait_bar(&bar[VB_G_READY], ph_gready, ctl, a.err)) break;
-                    if (!wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
-                    tc::tc_fence_after();
-                    mma_steps<true>(tb + colU, sPG, kC, sV, kC, id_O, kC / 16, false);
-                    // phase 3: O += A'_h W_h ; state_h += EB_h V
-                    for (int h = 0; h < NH; ++h) {
-                        if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
-                        if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
+                        mma_steps<true>(accG, sA + h * a_tile, kC, sEB, 128, id_G, RH / 16, h > 0);
+                        if (h == NH - 1) tc::mma_commit(&bar[VB_G_FULL]);
+                        // state_h += EB_h V once this chunk's W tiles have been read from the state
+                        if (h == 0 && !wait_bar(&bar[VB_STATE_READ], ph_sread, ctl, a.err)) { bad = true; break; }
                         tc::tc_fence_after();
-                        mma_steps<true>(tb + colU, sA + h * a_tile, kC, sW, RH, id_O, RH / 16, true);
-                        tc::mma_commit(&bar[VB_W_FREE]);
                         mma_steps<true>(tb + h * D, sEB, 128, sV, kC, id_O, kC / 16, true);
                         tc::mma_commit(&bar[VB_STATE_DONE + h]);
                         tc::mma_commit(&bar[VB_EB_FREE]);
                     }
                     if (bad) break;
+                    // O = sum_h A'_h W_h -> U once the last A' has been drained
+                    for (int h = 0; h < NH; ++h) {
+                        if (h == 0 && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
+                        if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
+                        tc::tc_fence_after();
+                        mma_steps<true>(accU, sA + h * a_tile, kC, sW, RH, id_O, RH / 16, h > 0);
+                        tc::mma_commit(&bar[VB_W_FREE]);
+                    }
+                    if (bad) break;
+                    // O += G V (G written over p by the epilogue)
+                    if (!wait_bar(&bar[VB_G_READY], ph_gready, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    mma_steps<true>(accU, sPG, kC, sV, kC, id_O, kC / 16, true);
                     tc::mma_commit(&bar[VB_O_FULL]);
                     tc::mma_commit(&bar[VB_PV_FREE]);
                 }
@@ -1157,17 +1164,31 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 uint32_t ph_exit = 0;
                 tc::mbar_wait(&bar[VB_EXIT], ph_exit);
             }
+        } else if (warp == 10) {
+            // ---------------- O store: bulk-store each output tile staged in A'_0's buffer and hand
+            // the buffer back once the copy has read it
+            if (lane == 0 && stage_o) {
+                uint32_t ph_osmem = 0;
+                for (int c = c_begin; c < c_end; ++c) {
+                    if (!wait_bar(&bar[VB_O_SMEM], ph_osmem, ctl, a.err)) break;
+                    for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sA + db * kC * 128, db * 64, c * kC, bh);
+                    tc::bulk_commit();
+                    tc::bulk_wait_read0();
+                    tc::mbar_arrive(&bar[VB_O_STORED]);
+                }
+                tc::bulk_wait0();
+            }
         }
     } else {
         {
+            // ---------------- epilogue warps 0-7 (thread = TMEM lane = token row / state row; warpgroup
+            // wg handles half of the columns of every drain).  Per chunk: read W_0, W_1 from the state
+            // (letting the state updates proceed) and store W_0; A'_0; A'_1; W_1; G; O.
             const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
             const int M = g.M;
             constexpr int XH = RH / 2, DH = D / 2;
-            uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0, ph_sync = 0, ph_ostored = 0;
+            uint32_t ph_u = 0, ph_g = 0, ph_wfree = 0, ph_o = 0, ph_ostored = 0;
             uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
-            // the output tile is staged in A'_0's buffer (idle between the last MMA of a chunk and the
-            // next chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
-            const bool stage_o = NH * RH >= D;
             // first mode of this thread's range in each half, and the drain phases of this row
             const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
             RowPhases rp = row_phases((long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
@@ -1178,14 +1199,37 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
                 state_init_abs<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D, f.x, f.y);
             }
+            auto w_store = [&](bool wait_free, const uint32_t *pk) -> bool {
+                if (wait_free && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) return false;
+                if (row < RH) {
+#pragma unroll
+                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_packed(sW, RH, row, wg * DH + g0, pk + g0 / 2);
+                }
+                tc::fence_proxy_async_smem();
+                tc::tc_fence_before();
+                epi_arrive(&bar[VB_W_READY]);
+                return true;
+            };
             bool bad = false;
             for (int c = c_begin; c < c_end && !bad; ++c) {
                 const int t0 = c * kC;
                 const int n = min(kC, g.L - t0);
                 const bool rot = c > c_begin;
                 if (rot) advance(rp, rp_step);
-                // phase 1: U_h -> A'_h, the rotation by -m w t (t absolute) of (sum_j p A, sum_j p B)
-                if (stage_o && c > c_begin && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
+                // W_h: the V state before this chunk's update, into registers
+                uint32_t pk0[DH / 2], pk1[DH / 2];
+                for (int h = 0; h < NH; ++h)
+                    if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
+                if (bad) break;
+                tc::tc_fence_after();
+                state_pack<DH>(tb, wg * DH, row, pk0);
+                if (NH == 2) state_pack<DH>(tb, D + wg * DH, row, pk1);
+                tc::tc_fence_before();
+                epi_arrive(&bar[VB_STATE_READ]);
+                if (!w_store(rot, pk0)) { bad = true; break; }
+                // A'_h = e^{-i m w t} U_h (t absolute) -> its shared tile; A'_0's tile held the previous
+                // chunk's output tile until the store read it
+                if (stage_o && rot && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
                 for (int h = 0; h < NH; ++h) {
                     if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
@@ -1218,7 +1262,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     epi_arrive(&bar[VB_U_FREE]);
                 }
                 if (bad) break;
-                // phase 2: G drain -> causal mask -> bf16 over p's tile
+                // W_1 once O = A'_0 W_0 has read W_0
+                if (NH == 2 && !w_store(true, pk1)) { bad = true; break; }
+                // G drain -> causal mask -> bf16 over p's tile
                 if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
                 tc::tc_fence_after();
                 {
@@ -1234,19 +1280,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 tc::tc_fence_before();
                 epi_arrive(&bar[VB_G_READY]);
                 epi_arrive(&bar[VB_G_FREE]);
-                // phase 3: W_h (the V state read before this chunk's update)
-                for (int h = 0; h < NH; ++h) {
-                    if (h > 0 && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) { bad = true; break; }
-                    if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
-                    tc::tc_fence_after();
-                    state_pass<DH>(tb, h * D + wg * DH, row, false, 1.f, 0.f, false, sW, RH, nullptr, wg * DH);
-                    tc::fence_proxy_async_smem();
-                    tc::tc_fence_before();
-                    epi_arrive(&bar[VB_W_READY]);
-                }
-                if (bad) break;
-                if (!wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) break;
-                // phase 4: O drain -> global
+                // O drain -> staged in A'_0's tile for the store warp, or straight to global
                 if (!wait_bar(&bar[VB_O_FULL], ph_o, ctl, a.err)) break;
                 tc::tc_fence_after();
                 {
@@ -1258,13 +1292,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 #pragma unroll
                         for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16(sA, kC, row, wg * DH + g0, v + g0);
                         tc::fence_proxy_async_smem();
-                        if (!epi_sync(&bar[VB_EPI_SYNC], ph_sync, ctl, a.err)) { bad = true; break; }
-                        if (threadIdx.x == 0) {
-                            for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sA + db * kC * 128, db * 64, t0, bh);
-                            tc::bulk_commit();
-                            tc::bulk_wait_read0();
-                            tc::mbar_arrive(&bar[VB_O_STORED]);
-                        }
+                        epi_arrive(&bar[VB_O_SMEM]);
                     } else if (row < n) {
                         bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D + wg * DH;
 #pragma unroll
@@ -1289,7 +1317,6 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     }
                 }
             }
-            if (threadIdx.x == 0) tc::bulk_wait0();
         }
     }
     tc::tc_fence_before();
