@@ -73,13 +73,13 @@ Geo make_geo(const OpDims &d) {
 }
 
 struct WsLayout {
-    size_t tables, eb, phi, fseg, deltas, win, pbuf, total;
+    size_t delta, eb, phi, fseg, deltas, win, pbuf, total;
 };
 
 WsLayout ws_layout(const OpDims &d, const Geo &g) {
     WsLayout w;
     size_t off = 0;
-    w.tables = off; off += tables_bytes(d, kC);
+    w.delta = off;  off += align_up(sizeof(int) * (size_t)g.S, 1024);
     w.eb = off;     off += align_up(sizeof(bf16) * (size_t)g.nchunks * g.RP * kC, 1024);   // EB per chunk
     w.phi = off;    off += align_up(sizeof(bf16) * (size_t)g.SP * g.R2, 1024);
     w.fseg = off;   off += g.G > 1 ? align_up(sizeof(bf16) * (size_t)g.RP * g.Lseg, 1024) : 0;
@@ -92,8 +92,6 @@ WsLayout ws_layout(const OpDims &d, const Geo &g) {
 
 // ------------------------------------------------------------------ bf16 tables
 
-// EB [RP][C], PHI [SP][R2], FSEG [RP][Lseg] in bf16, from fp64 phases (rows beyond 2M and
-// slots beyond S are zero).
 // (cos, sin)(m w u): with w = 2 pi / T and an integer period tint > 0 the angle is reduced
 // exactly, 2 pi ((m u) mod T) / T, and evaluated by sincospi in fp32; otherwise in fp64.
 __device__ __forceinline__ void mode_phase(long long mu, double w, int tint, float *c, float *s) {
@@ -108,83 +106,75 @@ __device__ __forceinline__ void mode_phase(long long mu, double w, int tint, flo
     }
 }
 
-__global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, double T, double w, int tint, bf16 *eb,
-                              bf16 *phi, bf16 *fseg) {
-    const int R2 = 2 * M;
-    const long long n_eb = (long long)RP * kC, n_phi = (long long)SP * R2;
-    const long long n_f = fseg ? (long long)RP * Lseg : 0;
-    const long long total = n_eb + n_phi + n_f;
+// Operand tables of the tensor-core path, in bf16 (rows beyond 2M and slots beyond S are zero):
+//   EB    [nch][RP][C]: EB_c[2m][u] = cos(m w (cC + u)), EB_c[2m+1][u] = -sin(m w (cC + u));
+//         with nch = 1 this is the in-chunk table (c = 0) of the lag frame
+//   PHI   [SP][R2]: PHI[j][2m] = c_m cos(m w D_j), PHI[j][2m+1] = c_m sin(m w D_j), D_j = round(j T / S),
+//         c_0 = 1/(2M-1), c_m = 2/(2M-1)
+//   FSEG  [RP][Lseg] (optional): FSEG[2m][u] = cos(m w (Lseg - u)), FSEG[2m+1][u] = sin(m w (Lseg - u))
+//   delta [S] (optional): the slot lags D_j
+// EB is written by one thread per (c, m, 8 consecutive u), u fastest so that a warp writes whole
+// rows: the first phase is reduced exactly, the next seven follow by products with e^{i m w}.
+__global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, double T, double w, int tint,
+                              bf16 *eb, bf16 *phi, bf16 *fseg, int *delta) {
+    const int R2 = 2 * M, MP = RP / 2;
+    const long long n_eb = (long long)nch * MP * (kC / 8), n_phi = (long long)SP * R2;
+    const long long n_f = fseg ? (long long)RP * Lseg : 0, n_d = delta ? S : 0;
+    const long long total = n_eb + n_phi + n_f + n_d;
     const double n = 2.0 * M - 1.0;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
         if (i < n_eb) {
-            int r = (int)(i / kC), u = (int)(i % kC), m = r >> 1;
-            float v = 0.f;
-            if (r < R2) {
-                float s, c;
-                mode_phase((long long)m * u, w, tint, &c, &s);
-                v = (r & 1) ? -s : c;
+            const long long per_c = (long long)MP * (kC / 8);
+            const int c = (int)(i / per_c), rem = (int)(i % per_c);
+            const int m = rem / (kC / 8), u0 = (rem % (kC / 8)) * 8;
+            bf16 *rc = eb + ((size_t)c * RP + 2 * m) * kC + u0, *rs = rc + kC;
+            uint32_t wc[4] = {0u, 0u, 0u, 0u}, ws[4] = {0u, 0u, 0u, 0u};
+            if (m < M) {
+                float bc, bs, ec, es;
+                mode_phase((long long)m * ((long long)c * kC + u0), w, tint, &bc, &bs);
+                mode_phase((long long)m, w, tint, &ec, &es);
+#pragma unroll
+                for (int j = 0; j < 8; j += 2) {
+                    const float c0 = bc, s0 = bs;
+                    float t = bc * ec - bs * es;
+                    bs = bc * es + bs * ec;
+                    bc = t;
+                    wc[j / 2] = tc::pack_bf16x2(c0, bc);
+                    ws[j / 2] = tc::pack_bf16x2(-s0, -bs);
+                    t = bc * ec - bs * es;
+                    bs = bc * es + bs * ec;
+                    bc = t;
+                }
             }
-            eb[i] = __float2bfloat16_rn(v);
+            *reinterpret_cast<uint4 *>(rc) = make_uint4(wc[0], wc[1], wc[2], wc[3]);
+            *reinterpret_cast<uint4 *>(rs) = make_uint4(ws[0], ws[1], ws[2], ws[3]);
         } else if (i < n_eb + n_phi) {
-            long long e = i - n_eb;
-            int j = (int)(e / R2), r = (int)(e % R2), m = r >> 1;
-            double v = 0.0;
+            const long long e = i - n_eb;
+            const int j = (int)(e / R2), r = (int)(e % R2), m = r >> 1;
+            float v = 0.f;
             if (j < S) {
-                double dj = rint((double)j * T / (double)S);
-                double cm = (m == 0) ? 1.0 / n : 2.0 / n;
-                double s, c;
-                sincos((double)m * w * dj, &s, &c);
-                v = cm * ((r & 1) ? s : c);
+                const long long dj = (long long)rint((double)j * T / (double)S);
+                const float cm = (m == 0) ? (float)(1.0 / n) : (float)(2.0 / n);
+                float c, sn;
+                mode_phase((long long)m * dj, w, tint, &c, &sn);
+                v = cm * ((r & 1) ? sn : c);
             }
-            phi[e] = __float2bfloat16_rn((float)v);
-        } else {
-            long long e = i - n_eb - n_phi;
-            int r = (int)(e / Lseg), u = (int)(e % Lseg), m = r >> 1;
+            phi[e] = __float2bfloat16_rn(v);
+        } else if (i < n_eb + n_phi + n_f) {
+            const long long e = i - n_eb - n_phi;
+            const int r = (int)(e / Lseg), u = (int)(e % Lseg), m = r >> 1;
             float v = 0.f;
             if (r < R2) {
-                float s, c;
-                mode_phase((long long)m * (Lseg - u), w, tint, &c, &s);
-                v = (r & 1) ? s : c;
+                float c, sn;
+                mode_phase((long long)m * (Lseg - u), w, tint, &c, &sn);
+                v = (r & 1) ? sn : c;
             }
             fseg[e] = __float2bfloat16_rn(v);
+        } else {
+            const int j = (int)(i - n_eb - n_phi - n_f);
+            delta[j] = (int)rint((double)j * T / (double)S);
         }
-    }
-}
-
-// Per-chunk EB for the forward passes, whose states are kept in the absolute frame:
-//   EB_c [RP][C]: EB_c[2m][u] = cos(m w (cC + u)), EB_c[2m+1][u] = -sin(m w (cC + u)), rows >= 2M zero.
-// One thread per (c, m, 8 consecutive u), u fastest so that a warp writes whole rows: the first
-// phase is reduced exactly (mode_phase), the next seven follow by products with e^{i m w}.
-__global__ void k_eb_chunks(int M, int RP, int nch, double w, int tint, bf16 *ebc) {
-    const int MP = RP / 2;
-    const long long per_c = (long long)MP * (kC / 8);
-    const long long total = (long long)nch * per_c;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int c = (int)(i / per_c), rem = (int)(i % per_c);
-        const int m = rem / (kC / 8), u0 = (rem % (kC / 8)) * 8;
-        bf16 *rc = ebc + ((size_t)c * RP + 2 * m) * kC + u0, *rs = rc + kC;
-        uint32_t wc[4] = {0u, 0u, 0u, 0u}, ws[4] = {0u, 0u, 0u, 0u};
-        if (m < M) {
-            float bc, bs, ec, es;
-            mode_phase((long long)m * ((long long)c * kC + u0), w, tint, &bc, &bs);
-            mode_phase((long long)m, w, tint, &ec, &es);
-#pragma unroll
-            for (int j = 0; j < 8; j += 2) {
-                const float c0 = bc, s0 = bs;
-                float t = bc * ec - bs * es;
-                bs = bc * es + bs * ec;
-                bc = t;
-                wc[j / 2] = tc::pack_bf16x2(c0, bc);
-                ws[j / 2] = tc::pack_bf16x2(-s0, -bs);
-                t = bc * ec - bs * es;
-                bs = bc * es + bs * ec;
-                bc = t;
-            }
-        }
-        *reinterpret_cast<uint4 *>(rc) = make_uint4(wc[0], wc[1], wc[2], wc[3]);
-        *reinterpret_cast<uint4 *>(rs) = make_uint4(ws[0], ws[1], ws[2], ws[3]);
     }
 }
 
@@ -194,7 +184,6 @@ struct Args {
     Geo g;
     float scale;
     double w;
-    const float *erel;   // [C+1][M][2] fp32 (cos, sin)(m w tau)
     const int *delta;    // [S]
     const float *deltas; // [BH][G][2][RP][D] segment deltas (prepass output)
     float *win;          // [BH][G][2][RP][D] states entering each segment (or null if G == 1)
@@ -485,19 +474,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     } else if (warp == 5 && lane == 0) {
         uint32_t ph[kPreStages] = {0, 0, 0};
-        const uint32_t idesc = tc::idesc_bf16(128, D, false, true);
+        // K and V of a stage are adjacent MN-major blocks of [64 tokens][64 d] (LBO = 8 KB), so one
+        // N = 2D MMA covers both: accumulator columns [b*2D, b*2D + D) for K, [b*2D + D, (b+1)*2D) for V
+        const uint32_t idesc = tc::idesc_bf16(128, 2 * D, false, true);
         for (int it = 0; it < steps; ++it) {
             const int st = it % kPreStages;
             if (!wait_bar(&full[st], ph[st], ctl, a.err)) break;
             tc::tc_fence_after();
             uint8_t *base = stage0 + st * stage_bytes;
-            for (int x = 0; x < 2; ++x)
-                for (int b = 0; b < NB; ++b)
-                    for (int k = 0; k < 4; ++k) {
-                        uint64_t ad = kmaj_desc(base + b * 128 * 128, 128, k);
-                        uint64_t bd = mnmaj_desc(base + f_bytes + x * x_bytes, 64, k);
-                        tc::mma_bf16(tb + (uint32_t)((x * NB + b) * D), ad, bd, idesc, (it > 0 || k > 0) ? 1u : 0u);
-                    }
+            for (int b = 0; b < NB; ++b)
+                for (int k = 0; k < 4; ++k) {
+                    uint64_t ad = kmaj_desc(base + b * 128 * 128, 128, k);
+                    uint64_t bd = mnmaj_desc(base + f_bytes, 64, k);
+                    tc::mma_bf16(tb + (uint32_t)(b * 2 * D), ad, bd, idesc, (it > 0 || k > 0) ? 1u : 0u);
+                }
             tc::mma_commit(&empty[st]);
         }
         tc::mma_commit(done);
@@ -511,9 +501,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                 for (int b = 0; b < NB; ++b) {
                     float *dst = a.deltas_out + ((((size_t)bh * g.G + seg) * 2 + x) * g.RP + b * 128 + row) * D;
                     if (D == 128)
-                        state_pass<128>(tb, (x * NB + b) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
+                        state_pass<128>(tb, (b * 2 + x) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
                     else
-                        state_pass<64>(tb, (x * NB + b) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
+                        state_pass<64>(tb, (b * 2 + x) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
                 }
         }
     }
@@ -541,14 +531,28 @@ __global__ void k_scan(Args a) {
         float c, s;
         mode_phase((long long)m * g.Lseg, a.w, a.tint, &c, &s);
         float re = 0.f, im = 0.f;
-        for (int seg = 0; seg < g.G; ++seg) {
-            const size_t base = (((size_t)bh * g.G + seg) * 2 + x) * g.RP;
-            a.win[(base + 2 * m) * g.D + e] = re;
-            a.win[(base + 2 * m + 1) * g.D + e] = im;
-            if (seg + 1 < g.G) {
-                const float dre = a.deltas[(base + 2 * m) * g.D + e], dim = a.deltas[(base + 2 * m + 1) * g.D + e];
-                const float nre = c * re - s * im + dre;
-                const float nim = s * re + c * im + dim;
+        // the deltas of eight segments are loaded before they are used, so that their latencies overlap
+        for (int s0 = 0; s0 < g.G; s0 += 8) {
+            float dre[8], dim[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int seg = s0 + j;
+                dre[j] = dim[j] = 0.f;
+                if (seg + 1 < g.G) {
+                    const size_t base = (((size_t)bh * g.G + seg) * 2 + x) * g.RP;
+                    dre[j] = a.deltas[(base + 2 * m) * g.D + e];
+                    dim[j] = a.deltas[(base + 2 * m + 1) * g.D + e];
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                const int seg = s0 + j;
+                if (seg >= g.G) break;
+                const size_t base = (((size_t)bh * g.G + seg) * 2 + x) * g.RP;
+                a.win[(base + 2 * m) * g.D + e] = re;
+                a.win[(base + 2 * m + 1) * g.D + e] = im;
+                const float nre = c * re - s * im + dre[j];
+                const float nim = s * re + c * im + dim[j];
                 re = nre;
                 im = nim;
             }
@@ -1341,11 +1345,11 @@ static int integer_period(const OpDims &d) {
 }
 
 cudaError_t build_bf16_tables(const OpDims &d, int RP, int SP, bf16 *eb, bf16 *phi, cudaStream_t st) {
-    long long total = (long long)RP * kC + (long long)SP * d.R2;
+    long long total = (long long)(RP / 2) * (kC / 8) + (long long)SP * d.R2;
     int blocks = (int)((total + 255) / 256);
     if (blocks > 2048) blocks = 2048;
     ProfScope ps(BLA_K_TABLES_BF16, st);
-    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, d.T, d.w, integer_period(d), eb, phi, nullptr);
+    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, 1, d.T, d.w, integer_period(d), eb, phi, nullptr, nullptr);
     return cudaGetLastError();
 }
 
@@ -1468,34 +1472,25 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     }
     WsLayout wl = ws_layout(d, g);
     char *ws = static_cast<char *>(workspace);
-    Tables t;
-    tables_carve(d, kC, ws + wl.tables, &t);
-    cudaError_t e = tables_build(d, t, st);
-    if (e != cudaSuccess) return e;
+    cudaError_t e;
     bf16 *eb = reinterpret_cast<bf16 *>(ws + wl.eb), *phi = reinterpret_cast<bf16 *>(ws + wl.phi);
     bf16 *fseg = g.G > 1 ? reinterpret_cast<bf16 *>(ws + wl.fseg) : nullptr;
+    int *delta = reinterpret_cast<int *>(ws + wl.delta);
     {
-        long long total = (long long)g.RP * kC + (long long)g.SP * g.R2 + (fseg ? (long long)g.RP * g.Lseg : 0);
-        int blocks = (int)((total + 255) / 256);
-        if (blocks > 2048) blocks = 2048;
-        ProfScope ps(BLA_K_TABLES_BF16, st);
-        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, d.T, d.w, integer_period(d), eb, phi, fseg);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-    {
-        // EB of every chunk (absolute phases) over the single-chunk table written above
-        const long long total = (long long)g.nchunks * (g.RP / 2) * (kC / 8);
+        // EB of every chunk (absolute phases), PHI, FSEG and the slot lags in one launch
+        const long long total = (long long)g.nchunks * (g.RP / 2) * (kC / 8) + (long long)g.SP * g.R2 +
+                                (fseg ? (long long)g.RP * g.Lseg : 0) + g.S;
         const int blocks = (int)(total < 4096 * 256 ? (total + 255) / 256 : 4096);
         ProfScope ps(BLA_K_TABLES_BF16, st);
-        k_eb_chunks<<<blocks, 256, 0, st>>>(g.M, g.RP, g.nchunks, d.w, integer_period(d), eb);
+        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, g.nchunks, d.T, d.w, integer_period(d), eb,
+                                              phi, fseg, delta);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     Args a;
     a.g = g;
     a.scale = d.scale;
     a.w = d.w;
-    a.erel = t.erel;
-    a.delta = t.delta;
+    a.delta = delta;
     a.deltas = g.G > 1 ? reinterpret_cast<float *>(ws + wl.deltas) : nullptr;
     a.deltas_out = const_cast<float *>(a.deltas);
     a.win = g.G > 1 ? reinterpret_cast<float *>(ws + wl.win) : nullptr;
