@@ -596,7 +596,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi,
             const __grid_constant__ CUtensorMap tm_p, Args a) {
     const Geo &g = a.g;
-    const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
+    // heads fastest: the CTAs of one segment run in the same wave and share its EB tables in L2
+    const int bh = blockIdx.x % g.BH, seg = blockIdx.x / g.BH;
     const int c_begin = seg * g.cps, c_end = min(g.nchunks, c_begin + g.cps);
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     // the 128-byte-swizzled tiles need a 1024-aligned base; the layout reserves no slack for it
@@ -1041,7 +1042,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_phi,
             const __grid_constant__ CUtensorMap tm_o, Args a) {
     const Geo &g = a.g;
-    const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
+    // heads fastest: the CTAs of one segment run in the same wave and share its EB tables in L2
+    const int bh = blockIdx.x % g.BH, seg = blockIdx.x / g.BH;
     const int c_begin = seg * g.cps, c_end = min(g.nchunks, c_begin + g.cps);
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
