@@ -1012,30 +1012,38 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 // ================================================================== V pass
 
 struct VLayout {
-    size_t pg, v, a2, w, phi, eb, bars, total;
+    size_t v, y0, bx, bz, w, phi, eb, bars, total;
 };
 
+// Every 128-row tile buffer holds 32 KB: p (128 x SP), G (128 x C), A'_h (128 x RH) or O (128 x d).
 __host__ __device__ inline VLayout v_layout(const Geo &g) {
     VLayout l;
     size_t off = 0;
-    const size_t pbytes = (size_t)kC * g.SP * 2, gbytes = (size_t)kC * kC * 2;
-    l.pg = off;  off += pbytes > gbytes ? pbytes : gbytes;
+    const size_t tile = (size_t)kC * 128 * 2;
     l.v = off;   off += (size_t)kC * g.D * 2;
-    l.a2 = off;  off += (size_t)g.NH * kC * g.RH * 2;
+    l.y0 = off;  off += tile;   // A'_0, then the staged output tile
+    l.bx = off;  off += tile;   // p then G, and A'_1, alternating with bz from chunk to chunk
+    l.bz = off;  off += tile;
     l.w = off;   off += (size_t)g.RH * g.D * 2;
-    l.phi = off; off += (size_t)g.SP * g.RH * 2;
-    l.eb = off;  off += (size_t)128 * kC * 2;
+    l.phi = off; off += tile;   // PHI_0, PHI_1, then EB_1
+    l.eb = off;  off += tile;   // EB_0
     l.bars = off; off += 1024;
     l.total = off + 1024;
     return l;
 }
 
+// One barrier per hand-off (see the K pass).
 enum VBar {
-    VB_PV_FULL, VB_PV_FREE, VB_EB_FULL, VB_EB_FREE, VB_PHI_FULL, VB_PHI_FREE,
+    VB_P_FULL, VB_P_FREE, VB_V_FULL, VB_V_FREE, VB_EB_FULL, VB_EB_FREE, VB_PH_FULL, VB_PH_FREE,
     VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_G_READY, VB_W_READY, VB_W_FREE,
     VB_STATE_DONE, VB_STATE_DONE1, VB_STATE_READ, VB_O_FULL, VB_O_SMEM, VB_O_STORED, VB_EXIT, VB_COUNT
 };
 
+// V pass.  Per chunk and mode half h: U_h = p PHI_h; A'_h = e^{-i m w t} U_h (t absolute) into shared
+// memory; G = sum_h A'_h EB_h (causal mask on drain, written over p); state_h += EB_h V; and
+// O = sum_h A'_h W_h + G V.  Buffers: A'_0 and the staged output in y0; p/G and A'_1 alternate
+// between bx and bz from chunk to chunk, so the next chunk's p can load as soon as A'_1 W_1 is
+// done; the PHI tile takes EB_1 once U_1 has read PHI_1, so that EB_0 and EB_1 are both resident.
 template <int D, int RH, int NH>
 __global__ void __launch_bounds__(kPassThreads, 1)
     k_vpass(const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_v,
@@ -1048,17 +1056,16 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const VLayout lay = v_layout(g);
-    uint8_t *sPG = sm + lay.pg, *sV = sm + lay.v, *sA = sm + lay.a2, *sW = sm + lay.w;
+    uint8_t *sV = sm + lay.v, *sY0 = sm + lay.y0, *sBX = sm + lay.bx, *sBZ = sm + lay.bz, *sW = sm + lay.w;
     uint8_t *sPHI = sm + lay.phi, *sEB = sm + lay.eb;
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + lay.bars);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + VB_COUNT);
     Ctl *ctl = reinterpret_cast<Ctl *>(bar + VB_COUNT + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int SP = g.SP;
-    const size_t a_tile = (size_t)kC * RH * 2;
-    // the output tile is staged in A'_0's buffer (idle between the chunk's last MMA and the next
-    // chunk's A'_0) when that buffer holds 128 x d bf16, and leaves by a bulk tensor store
-    const bool stage_o = NH * RH >= D;
+    // chunk i (from c_begin) keeps p/G in pbuf(i) and A'_1 in a1buf(i) (two halves: alternating)
+    auto pbuf = [&](int i) { return (NH == 2 && (i & 1)) ? sBZ : sBX; };
+    auto a1buf = [&](int i) { return (i & 1) ? sBX : sBZ; };
     // TMEM: [0, NB*D) state; colU (128 cols: U_h, then O); colG (128 cols).
     const int colU = g.NB * D, colG = colU + 128;
     const uint32_t ncols = (uint32_t)(colG + 128) <= 256 ? 256u : 512u;  // host: pow2_cols(NB*D + 256)
@@ -1082,102 +1089,135 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 
     if (warp >= 8) {
         if (warp == 8) {
-            // ---------------- TMA producer: per chunk p and V, then PHI_0, EB_0, PHI_1, EB_1 in the
-            // order the MMA issuer consumes them
+            // ---------------- TMA producer, in the order of first use: p, PHI_0, EB_0, V, PHI_1, EB_1
             if (lane == 0) {
                 tc::tma_prefetch_desc(&tm_p); tc::tma_prefetch_desc(&tm_v);
                 tc::tma_prefetch_desc(&tm_eb); tc::tma_prefetch_desc(&tm_phi);
-                uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0;
-                bool first_eb = true, first_phi = true;
-                bool bad = false;
-                for (int c = c_begin; c < c_end && !bad; ++c) {
-                    if (c > c_begin && !wait_bar(&bar[VB_PV_FREE], ph_pv, ctl, a.err)) break;
-                    tc::mbar_arrive_expect_tx(&bar[VB_PV_FULL], (uint32_t)(kC * SP * 2 + kC * D * 2));
+                uint32_t ph_p = 0, ph_v = 0, ph_eb = 0, ph_ph = 0;
+                for (int c = c_begin; c < c_end; ++c) {
+                    const int i = c - c_begin;
+                    const bool first = i == 0;
+                    // p: the buffer held the previous chunk's A'_1 (two halves) or G (one half)
+                    if (!first && !wait_bar(&bar[VB_P_FREE], ph_p, ctl, a.err)) break;
+                    tc::mbar_arrive_expect_tx(&bar[VB_P_FULL], (uint32_t)(kC * SP * 2));
                     for (int kb = 0; kb < SP / 64; ++kb)
-                        tc::tma_load_3d(sPG + kb * kC * 128, &tm_p, &bar[VB_PV_FULL], kb * 64, c * kC, bh);
+                        tc::tma_load_3d(pbuf(i) + kb * kC * 128, &tm_p, &bar[VB_P_FULL], kb * 64, c * kC, bh);
+                    // PHI_0 (the PHI tile last held the previous chunk's EB_1, or PHI_0 with one half)
+                    if (!first && !wait_bar(&bar[VB_PH_FREE], ph_ph, ctl, a.err)) break;
+                    tc::mbar_arrive_expect_tx(&bar[VB_PH_FULL], (uint32_t)(SP * RH * 2));
+                    for (int kb = 0; kb < RH / 64; ++kb)
+                        tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PH_FULL], kb * 64, 0);
+                    if (!first && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) break;
+                    tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
+                    for (int kb = 0; kb < 2; ++kb)
+                        tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP);
+                    if (!first && !wait_bar(&bar[VB_V_FREE], ph_v, ctl, a.err)) break;
+                    tc::mbar_arrive_expect_tx(&bar[VB_V_FULL], (uint32_t)(kC * D * 2));
                     for (int db = 0; db < D / 64; ++db)
-                        tc::tma_load_3d(sV + db * kC * 128, &tm_v, &bar[VB_PV_FULL], db * 64, c * kC, bh);
-                    for (int h = 0; h < NH; ++h) {
-                        if (!first_phi && !wait_bar(&bar[VB_PHI_FREE], ph_phi, ctl, a.err)) { bad = true; break; }
-                        first_phi = false;
-                        tc::mbar_arrive_expect_tx(&bar[VB_PHI_FULL], (uint32_t)(SP * RH * 2));
+                        tc::tma_load_3d(sV + db * kC * 128, &tm_v, &bar[VB_V_FULL], db * 64, c * kC, bh);
+                    if (NH == 2) {
+                        // PHI_1 once U_0 has read PHI_0; EB_1 into the PHI tile once U_1 has read PHI_1
+                        if (!wait_bar(&bar[VB_PH_FREE], ph_ph, ctl, a.err)) break;
+                        tc::mbar_arrive_expect_tx(&bar[VB_PH_FULL], (uint32_t)(SP * RH * 2));
                         for (int kb = 0; kb < RH / 64; ++kb)
-                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PHI_FULL], h * RH + kb * 64, 0);
-                        if (!first_eb && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) { bad = true; break; }
-                        first_eb = false;
-                        tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
+                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PH_FULL], RH + kb * 64, 0);
+                        if (!wait_bar(&bar[VB_PH_FREE], ph_ph, ctl, a.err)) break;
+                        tc::mbar_arrive_expect_tx(&bar[VB_PH_FULL], (uint32_t)(128 * kC * 2));
                         for (int kb = 0; kb < 2; ++kb)
-                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP + h * 128);
+                            tc::tma_load_2d(sPHI + kb * 128 * 128, &tm_eb, &bar[VB_PH_FULL], kb * 64, c * g.RP + 128);
                     }
                 }
             }
         } else if (warp == 9) {
-            // ---------------- MMA issuer.  Per chunk and half h: U_h = p PHI_h -> U; once A'_h is
-            // drained, G (+)= A'_h EB_h -> G and state_h += EB_h V (EB_h is loaded once for both).
-            // Then O = A'_0 W_0 (+ A'_1 W_1) + G V -> U.
+            // ---------------- MMA issuer.  Per chunk: U_0; U_1 (once A'_0 is drained); G = A'_0 EB_0;
+            // state_0 += EB_0 V; G += A'_1 EB_1; state_1 += EB_1 V; O = A'_0 W_0 (+ A'_1 W_1); O += G V.
             if (lane == 0) {
-                uint32_t ph_pv = 0, ph_eb = 0, ph_phi = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0, ph_w = 0;
-                uint32_t ph_sread = 0;
+                uint32_t ph_p = 0, ph_v = 0, ph_eb = 0, ph_ph = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0;
+                uint32_t ph_w = 0, ph_sread = 0;
                 const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
                 const uint32_t id_G = tc::idesc_bf16(128, kC, false, true);
                 const uint32_t id_O = tc::idesc_bf16(128, D, false, true);
                 const uint32_t accU = tb + colU, accG = tb + colG;
-                bool bad = false;
-                for (int c = c_begin; c < c_end && !bad; ++c) {
-                    const bool first = c == c_begin;
-                    if (!wait_bar(&bar[VB_PV_FULL], ph_pv, ctl, a.err)) break;
-                    for (int h = 0; h < NH; ++h) {
-                        // U_h -> U: last read by the previous chunk's O drain, or by A'_0's drain
-                        if (!wait_bar(&bar[VB_PHI_FULL], ph_phi, ctl, a.err)) { bad = true; break; }
-                        if (!(first && h == 0) && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
+                for (int c = c_begin; c < c_end; ++c) {
+                    const int i = c - c_begin;
+                    const bool first = i == 0;
+                    uint8_t *sP = pbuf(i), *sA1 = a1buf(i);
+                    // U_0 -> U (last read by the previous chunk's O drain)
+                    if (!wait_bar(&bar[VB_P_FULL], ph_p, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_PH_FULL], ph_ph, ctl, a.err)) break;
+                    if (!first && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    mma_steps<true>(accU, sP, kC, sPHI, SP, id_U, SP / 16, false);
+                    tc::mma_commit(&bar[VB_U_FULL]);
+                    tc::mma_commit(&bar[VB_PH_FREE]);
+                    if (NH == 2) {
+                        // U_1 -> U once A'_0 is drained
+                        if (!wait_bar(&bar[VB_PH_FULL], ph_ph, ctl, a.err)) break;
+                        if (!wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
                         tc::tc_fence_after();
-                        mma_steps<true>(accU, sPG, kC, sPHI, SP, id_U, SP / 16, false);
+                        mma_steps<true>(accU, sP, kC, sPHI, SP, id_U, SP / 16, false);
                         tc::mma_commit(&bar[VB_U_FULL]);
-                        tc::mma_commit(&bar[VB_PHI_FREE]);
-                        // G (+)= A'_h EB_h once A'_h is in shared memory (G: last read by the previous
-                        // chunk's G drain)
-                        if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) { bad = true; break; }
-                        if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) { bad = true; break; }
-                        if (h == 0 && !first && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) { bad = true; break; }
-                        tc::tc_fence_after();
-                        mma_steps<true>(accG, sA + h * a_tile, kC, sEB, 128, id_G, RH / 16, h > 0);
-                        if (h == NH - 1) tc::mma_commit(&bar[VB_G_FULL]);
-                        // state_h += EB_h V once this chunk's W tiles have been read from the state
-                        if (h == 0 && !wait_bar(&bar[VB_STATE_READ], ph_sread, ctl, a.err)) { bad = true; break; }
-                        tc::tc_fence_after();
-                        mma_steps<true>(tb + h * D, sEB, 128, sV, kC, id_O, kC / 16, true);
-                        tc::mma_commit(&bar[VB_STATE_DONE + h]);
-                        tc::mma_commit(&bar[VB_EB_FREE]);
+                        tc::mma_commit(&bar[VB_PH_FREE]);
                     }
-                    if (bad) break;
-                    // O = sum_h A'_h W_h -> U once the last A' has been drained
-                    for (int h = 0; h < NH; ++h) {
-                        if (h == 0 && !wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) { bad = true; break; }
-                        if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) { bad = true; break; }
+                    // G = A'_0 EB_0 -> G (last read by the previous chunk's G drain)
+                    if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) break;
+                    if (!first && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    mma_steps<true>(accG, sY0, kC, sEB, 128, id_G, RH / 16, false);
+                    if (NH == 1) tc::mma_commit(&bar[VB_G_FULL]);
+                    // state_0 += EB_0 V once this chunk's W tiles have been read from the state
+                    if (!wait_bar(&bar[VB_STATE_READ], ph_sread, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_V_FULL], ph_v, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    mma_steps<true>(tb, sEB, 128, sV, kC, id_O, kC / 16, true);
+                    tc::mma_commit(&bar[VB_STATE_DONE]);
+                    tc::mma_commit(&bar[VB_EB_FREE]);
+                    if (NH == 2) {
+                        // G += A'_1 EB_1 (EB_1 in the PHI tile); state_1 += EB_1 V
+                        if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) break;
+                        if (!wait_bar(&bar[VB_PH_FULL], ph_ph, ctl, a.err)) break;
                         tc::tc_fence_after();
-                        mma_steps<true>(accU, sA + h * a_tile, kC, sW, RH, id_O, RH / 16, h > 0);
+                        mma_steps<true>(accG, sA1, kC, sPHI, 128, id_G, RH / 16, true);
+                        tc::mma_commit(&bar[VB_G_FULL]);
+                        mma_steps<true>(tb + D, sPHI, 128, sV, kC, id_O, kC / 16, true);
+                        tc::mma_commit(&bar[VB_STATE_DONE1]);
+                        tc::mma_commit(&bar[VB_PH_FREE]);
+                    }
+                    // O = A'_0 W_0 -> U once the last A' has been drained
+                    if (!wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    mma_steps<true>(accU, sY0, kC, sW, RH, id_O, RH / 16, false);
+                    tc::mma_commit(&bar[VB_W_FREE]);
+                    if (NH == 2) {
+                        // O += A'_1 W_1; A'_1's buffer then takes the next chunk's p
+                        if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) break;
+                        tc::tc_fence_after();
+                        mma_steps<true>(accU, sA1, kC, sW, RH, id_O, RH / 16, true);
                         tc::mma_commit(&bar[VB_W_FREE]);
+                        tc::mma_commit(&bar[VB_P_FREE]);
                     }
-                    if (bad) break;
                     // O += G V (G written over p by the epilogue)
                     if (!wait_bar(&bar[VB_G_READY], ph_gready, ctl, a.err)) break;
                     tc::tc_fence_after();
-                    mma_steps<true>(accU, sPG, kC, sV, kC, id_O, kC / 16, true);
+                    mma_steps<true>(accU, sP, kC, sV, kC, id_O, kC / 16, true);
                     tc::mma_commit(&bar[VB_O_FULL]);
-                    tc::mma_commit(&bar[VB_PV_FREE]);
+                    tc::mma_commit(&bar[VB_V_FREE]);
+                    if (NH == 1) tc::mma_commit(&bar[VB_P_FREE]);
                 }
                 tc::mma_commit(&bar[VB_EXIT]);
                 uint32_t ph_exit = 0;
                 tc::mbar_wait(&bar[VB_EXIT], ph_exit);
             }
         } else if (warp == 10) {
-            // ---------------- O store: bulk-store each output tile staged in A'_0's buffer and hand
-            // the buffer back once the copy has read it
-            if (lane == 0 && stage_o) {
+            // ---------------- O store: bulk-store each output tile staged in y0 and hand the buffer
+            // back once the copy has read it
+            if (lane == 0) {
                 uint32_t ph_osmem = 0;
                 for (int c = c_begin; c < c_end; ++c) {
                     if (!wait_bar(&bar[VB_O_SMEM], ph_osmem, ctl, a.err)) break;
-                    for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sA + db * kC * 128, db * 64, c * kC, bh);
+                    for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sY0 + db * kC * 128, db * 64, c * kC, bh);
                     tc::bulk_commit();
                     tc::bulk_wait_read0();
                     tc::mbar_arrive(&bar[VB_O_STORED]);
@@ -1218,9 +1258,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             };
             bool bad = false;
             for (int c = c_begin; c < c_end && !bad; ++c) {
-                const int t0 = c * kC;
-                const int n = min(kC, g.L - t0);
-                const bool rot = c > c_begin;
+                const int i = c - c_begin;
+                const bool rot = i > 0;
                 if (rot) advance(rp, rp_step);
                 // W_h: the V state before this chunk's update, into registers
                 uint32_t pk0[DH / 2], pk1[DH / 2];
@@ -1233,25 +1272,27 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 tc::tc_fence_before();
                 epi_arrive(&bar[VB_STATE_READ]);
                 if (!w_store(rot, pk0)) { bad = true; break; }
-                // A'_h = e^{-i m w t} U_h (t absolute) -> its shared tile; A'_0's tile held the previous
-                // chunk's output tile until the store read it
-                if (stage_o && rot && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
+                // A'_h = e^{-i m w t} U_h (t absolute); y0 held the previous chunk's output tile until
+                // the store read it
+                if (rot && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
                 for (int h = 0; h < NH; ++h) {
                     if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
                     float v[XH];
                     tc::tmem_ld<XH>(tmem_addr(tb, lane_base, colU + wg * XH), v);
+                    tc::tc_fence_before();
+                    epi_arrive(&bar[VB_U_FREE]);
                     const float2 pa = h ? rp.h1 : rp.h0, pb = cmul(pa, rp.e1), e2 = rp.e2;
                     float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
 #pragma unroll
-                    for (int i = 0; i < XH; i += 4) {
-                        float uc = v[i], us = v[i + 1];
-                        v[i] = ca * uc + sa * us;
-                        v[i + 1] = ca * us - sa * uc;
-                        uc = v[i + 2];
-                        us = v[i + 3];
-                        v[i + 2] = cb * uc + sb * us;
-                        v[i + 3] = cb * us - sb * uc;
+                    for (int q = 0; q < XH; q += 4) {
+                        float uc = v[q], us = v[q + 1];
+                        v[q] = ca * uc + sa * us;
+                        v[q + 1] = ca * us - sa * uc;
+                        uc = v[q + 2];
+                        us = v[q + 3];
+                        v[q + 2] = cb * uc + sb * us;
+                        v[q + 3] = cb * us - sb * uc;
                         float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
                         ca = t1;
                         sa = t2;
@@ -1260,33 +1301,32 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         cb = t1;
                         sb = t2;
                     }
+                    uint8_t *dstA = h ? a1buf(i) : sY0;
 #pragma unroll
-                    for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sA + h * a_tile, kC, row, wg * XH + g0, v + g0);
+                    for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(dstA, kC, row, wg * XH + g0, v + g0);
                     tc::fence_proxy_async_smem();
-                    tc::tc_fence_before();
                     epi_arrive(&bar[VB_A_READY]);
-                    epi_arrive(&bar[VB_U_FREE]);
                 }
                 if (bad) break;
                 // W_1 once O = A'_0 W_0 has read W_0
                 if (NH == 2 && !w_store(true, pk1)) { bad = true; break; }
-                // G drain -> causal mask -> bf16 over p's tile
+                // G drain -> causal mask -> bf16 over p (U_0 and U_1 are done once G is full)
                 if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
                 tc::tc_fence_after();
                 {
                     float v[64];
                     tc::tmem_ld<64>(tmem_addr(tb, lane_base, colG + wg * 64), v);
 #pragma unroll
-                    for (int i = 0; i < 64; ++i)
-                        if (wg * 64 + i > row) v[i] = 0.f;
+                    for (int q = 0; q < 64; ++q)
+                        if (wg * 64 + q > row) v[q] = 0.f;
 #pragma unroll
-                    for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(sPG, kC, row, wg * 64 + g0, v + g0);
+                    for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(pbuf(i), kC, row, wg * 64 + g0, v + g0);
                 }
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 epi_arrive(&bar[VB_G_READY]);
                 epi_arrive(&bar[VB_G_FREE]);
-                // O drain -> staged in A'_0's tile for the store warp, or straight to global
+                // O drain -> staged in y0 for the store warp
                 if (!wait_bar(&bar[VB_O_FULL], ph_o, ctl, a.err)) break;
                 tc::tc_fence_after();
                 {
@@ -1294,20 +1334,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     tc::tmem_ld<DH>(tmem_addr(tb, lane_base, colU + wg * DH), v);
                     tc::tc_fence_before();
                     epi_arrive(&bar[VB_U_FREE]);
-                    if (stage_o) {
 #pragma unroll
-                        for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16(sA, kC, row, wg * DH + g0, v + g0);
-                        tc::fence_proxy_async_smem();
-                        epi_arrive(&bar[VB_O_SMEM]);
-                    } else if (row < n) {
-                        bf16 *orow = a.o + ((size_t)bh * g.L + t0 + row) * D + wg * DH;
-#pragma unroll
-                        for (int j = 0; j < DH; j += 8) {
-                            uint4 pk = make_uint4(tc::pack_bf16x2(v[j], v[j + 1]), tc::pack_bf16x2(v[j + 2], v[j + 3]),
-                                                  tc::pack_bf16x2(v[j + 4], v[j + 5]), tc::pack_bf16x2(v[j + 6], v[j + 7]));
-                            *reinterpret_cast<uint4 *>(orow + j) = pk;
-                        }
-                    }
+                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16(sY0, kC, row, wg * DH + g0, v + g0);
+                    tc::fence_proxy_async_smem();
+                    epi_arrive(&bar[VB_O_SMEM]);
                 }
             }
             if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
