@@ -308,24 +308,29 @@ __device__ __forceinline__ void advance(RowPhases &p, const RowPhases &step) {
 
 // Initial state block in the absolute frame: the carried-in lag-frame state S (rows [rows][stride],
 // interleaved (Re, Im) row pairs; null = zero) rotated to A = e^{-i m w t0} S, written to TMEM.
-// (c, s) = (cos, sin)(m w t0) of this thread's mode; the partner row is read from global memory.
+// (c, s) = (cos, sin)(m w t0) of this thread's mode.  Each thread loads only its own row, all
+// loads issued before any use (one memory latency per block); the partner row of the pair is
+// the neighbouring lane's.
 template <int DH>
 __device__ __forceinline__ void state_init_abs(uint32_t tbase, int col0, int row, const float *src, int live_rows,
                                                int stride, float c, float s) {
     const int lane_base = (row >> 5) << 5;
     const float sg = (row & 1) ? -s : s;   // Re' = c Re + s Im ; Im' = c Im - s Re
+    const bool live = src != nullptr && row < live_rows;   // same for both rows of a pair
     float v[DH];
 #pragma unroll
     for (int i = 0; i < DH; i += 4) {
-        float4 own = make_float4(0.f, 0.f, 0.f, 0.f), par = own;
-        if (src && row < live_rows) {
-            own = *reinterpret_cast<const float4 *>(src + (size_t)row * stride + i);
-            par = *reinterpret_cast<const float4 *>(src + (size_t)(row ^ 1) * stride + i);
-        }
-        v[i] = c * own.x + sg * par.x;
-        v[i + 1] = c * own.y + sg * par.y;
-        v[i + 2] = c * own.z + sg * par.z;
-        v[i + 3] = c * own.w + sg * par.w;
+        float4 t = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (live) t = __ldg(reinterpret_cast<const float4 *>(src + (size_t)row * stride + i));
+        v[i] = t.x;
+        v[i + 1] = t.y;
+        v[i + 2] = t.z;
+        v[i + 3] = t.w;
+    }
+#pragma unroll
+    for (int i = 0; i < DH; ++i) {
+        const float par = __shfl_xor_sync(0xffffffffu, v[i], 1);
+        v[i] = c * v[i] + sg * par;
     }
     tc::tmem_st<DH>(tmem_addr(tbase, lane_base, col0), v);
 }
@@ -1032,10 +1037,11 @@ __host__ __device__ inline VLayout v_layout(const Geo &g) {
     return l;
 }
 
-// One barrier per hand-off (see the K pass).
+// One barrier per hand-off (see the K pass).  A'_0 and A'_1 each have their own ready barrier:
+// U_1 is issued before G waits for A'_0, so one barrier could complete twice before that wait.
 enum VBar {
     VB_P_FULL, VB_P_FREE, VB_V_FULL, VB_V_FREE, VB_EB_FULL, VB_EB_FREE, VB_PH_FULL, VB_PH_FREE,
-    VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_G_READY, VB_W_READY, VB_W_FREE,
+    VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_A_READY1, VB_G_READY, VB_W_READY, VB_W_FREE,
     VB_STATE_DONE, VB_STATE_DONE1, VB_STATE_READ, VB_O_FULL, VB_O_SMEM, VB_O_STORED, VB_EXIT, VB_COUNT
 };
 
@@ -1072,8 +1078,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < VB_COUNT; ++i) {
-            const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_G_READY || i == VB_W_READY ||
-                             i == VB_STATE_READ || i == VB_O_SMEM;
+            const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_A_READY1 || i == VB_G_READY ||
+                             i == VB_W_READY || i == VB_STATE_READ || i == VB_O_SMEM;
             tc::mbar_init(&bar[i], epi ? kPassEpiWarps : 1);
         }
         ctl->abort = 0;
@@ -1132,7 +1138,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             // ---------------- MMA issuer.  Per chunk: U_0; U_1 (once A'_0 is drained); G = A'_0 EB_0;
             // state_0 += EB_0 V; G += A'_1 EB_1; state_1 += EB_1 V; O = A'_0 W_0 (+ A'_1 W_1); O += G V.
             if (lane == 0) {
-                uint32_t ph_p = 0, ph_v = 0, ph_eb = 0, ph_ph = 0, ph_ufree = 0, ph_gfree = 0, ph_a = 0, ph_gready = 0;
+                uint32_t ph_p = 0, ph_v = 0, ph_eb = 0, ph_ph = 0, ph_ufree = 0, ph_gfree = 0, ph_a0 = 0, ph_a1 = 0, ph_gready = 0;
                 uint32_t ph_w = 0, ph_sread = 0;
                 const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
                 const uint32_t id_G = tc::idesc_bf16(128, kC, false, true);
@@ -1160,7 +1166,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         tc::mma_commit(&bar[VB_PH_FREE]);
                     }
                     // G = A'_0 EB_0 -> G (last read by the previous chunk's G drain)
-                    if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_A_READY], ph_a0, ctl, a.err)) break;
                     if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) break;
                     if (!first && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) break;
                     tc::tc_fence_after();
@@ -1175,7 +1181,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     tc::mma_commit(&bar[VB_EB_FREE]);
                     if (NH == 2) {
                         // G += A'_1 EB_1 (EB_1 in the PHI tile); state_1 += EB_1 V
-                        if (!wait_bar(&bar[VB_A_READY], ph_a, ctl, a.err)) break;
+                        if (!wait_bar(&bar[VB_A_READY1], ph_a1, ctl, a.err)) break;
                         if (!wait_bar(&bar[VB_PH_FULL], ph_ph, ctl, a.err)) break;
                         tc::tc_fence_after();
                         mma_steps<true>(accG, sA1, kC, sPHI, 128, id_G, RH / 16, true);
@@ -1275,6 +1281,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 // A'_h = e^{-i m w t} U_h (t absolute); y0 held the previous chunk's output tile until
                 // the store read it
                 if (rot && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
+#pragma unroll
                 for (int h = 0; h < NH; ++h) {
                     if (!wait_bar(&bar[VB_U_FULL], ph_u, ctl, a.err)) { bad = true; break; }
                     tc::tc_fence_after();
@@ -1305,7 +1312,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 #pragma unroll
                     for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(dstA, kC, row, wg * XH + g0, v + g0);
                     tc::fence_proxy_async_smem();
-                    epi_arrive(&bar[VB_A_READY]);
+                    epi_arrive(&bar[VB_A_READY + h]);
                 }
                 if (bad) break;
                 // W_1 once O = A'_0 W_0 has read W_0
