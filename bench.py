@@ -237,6 +237,7 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--seq", type=int, default=0, help="override L (profiling captures of a smaller case)")
     ap.add_argument("--decode-batch", type=int, default=0, help="override the decode batch (profiling captures)")
+    ap.add_argument("--no-configs", action="store_true", help="skip the timing of the other parity configs")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -371,6 +372,11 @@ def main():
                   "roofline": {"bound": "hbm", "achieved": gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
                                "frac": gbs / peaks["hbm_gbs"], "bytes_per_launch": state_bytes}}
 
+    # ---- the other parity configs (rank 0, N = 1 only)
+    configs = None
+    if rank == 0 and world == 1 and not args.no_configs and args.seq == 0:
+        configs = measure_configs(bla, torch, dev, stream, peaks)
+
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -385,11 +391,78 @@ def main():
                            "inputs": "q,k,v bf16 805 MB resident, larger than the 129 MB L2 (no flush)",
                            "accumulate": "fp32 (TMEM), state fp32"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
-                "clocks": sampler.summary(), "decode": decode}
+                "clocks": sampler.summary(), "decode": decode, "configs": configs}
         print(json.dumps(line))
     if world > 1:
         torch.distributed.destroy_process_group()
     return 0
+
+
+def measure_configs(bla, torch, dev, stream, peaks, iters=20):
+    """The other parity configs, timed through the same ABI: config 2 (recall-shaped forward) and
+    config 3 (LM-layer forward and backward).  Each call is timed alone with CUDA events after an
+    L2 flush (config 2's inputs fit in L2); FLOPs are the canonical counts at chunk 64, the chunk
+    the survey fixes for these configs' accounting; bytes are the tensors the call must read and
+    write once."""
+    from paper_2606_09862_gb300.inputs import WORKLOADS, make_qkv, make_dout
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)   # 256 MB > 129 MB L2
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        tot = 0.0
+        for _ in range(iters):
+            flush.zero_()
+            a = torch.cuda.Event(enable_timing=True)
+            b = torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            fn()
+            b.record(stream)
+            torch.cuda.synchronize()
+            tot += a.elapsed_time(b)
+        bla.bla_device_error()
+        return tot / iters
+
+    def roof(flops, nbytes, ms, tokens):
+        tf = flops / (ms / 1000.0) / 1e12
+        gbs = nbytes / (ms / 1000.0) / 1e9
+        return {"ms": ms, "tokens_per_s": tokens / (ms / 1000.0), "tflops": tf, "gbs": gbs,
+                "frac_tensor": tf / peaks["bf16_tflops"], "frac_hbm": gbs / peaks["hbm_gbs"],
+                "bound": "hbm" if flops / nbytes < peaks["bf16_tflops"] * 1e3 / peaks["hbm_gbs"] else "tensor",
+                "flops": flops, "bytes": nbytes}
+
+    out = {}
+    for name in ("fwd_bf16_recall", "fwdbwd_bf16_lm"):
+        w = WORKLOADS[name]
+        q, k, v = (torch.from_numpy(x).to(torch.bfloat16).to(dev)
+                   for x in make_qkv(w.B, w.H, w.L, w.d, "bf16", seed=0, recall_dup=getattr(w, "recall_dup", 0.0)))
+        par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16)
+        ws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_FORWARD), dtype=torch.uint8, device=dev)
+        res = {}
+
+        def fwd():
+            return bla.bla_forward_chunked(q, k, v, w.M, w.S, w.T, workspace=ws, stream=stream)
+
+        tok = w.B * w.L
+        F = canonical_flops(w, C=64)["total"] * w.B * w.H * w.L
+        elem = w.B * w.H * w.L * w.d
+        res["forward"] = roof(F, 4 * elem * 2 + w.B * w.H * w.L * 4, timed(fwd), tok)
+        if getattr(w, "backward", False):
+            o, lse, _ = fwd()
+            do = torch.from_numpy(make_dout(w.B, w.H, w.L, w.d, "bf16", seed=0)).to(torch.bfloat16).to(dev)
+            bws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_BACKWARD), dtype=torch.uint8, device=dev)
+
+            def bwd():
+                return bla.bla_backward(q, k, v, o, do, lse, w.M, w.S, w.T, workspace=bws, stream=stream)
+
+            res["backward"] = roof(2 * F, 8 * elem * 2 + w.B * w.H * w.L * 4, timed(bwd), tok)
+            del o, lse, do, bws
+        res["shape"] = "B=%d H=%d L=%d d=%d M=%d S=%d T=%d" % (w.B, w.H, w.L, w.d, w.M, w.S, w.T)
+        out[name] = res
+        del q, k, v, ws
+    del flush
+    torch.cuda.empty_cache()
+    return out
 
 
 def stored_traffic(kernel, L):

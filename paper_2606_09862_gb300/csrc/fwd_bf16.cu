@@ -52,6 +52,19 @@ struct Geo {
     int nchunks, cps, G, Lseg;      // chunks per segment, segments per head, segment length (tokens)
 };
 
+// Multiprocessors of the current device (queried once per device).
+static int sm_count() {
+    static int cached[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+    if (cached[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
+        cached[dev] = n;
+    }
+    return cached[dev];
+}
+
 Geo make_geo(const OpDims &d) {
     Geo g;
     g.BH = d.B * d.H; g.L = d.L; g.D = d.dk; g.M = d.M; g.R2 = d.R2;
@@ -62,11 +75,24 @@ Geo make_geo(const OpDims &d) {
     g.S = d.S;
     g.SP = d.S < 64 ? 64 : d.S;
     g.nchunks = (d.L + kC - 1) / kC;
-    int want = (2 * 152 + g.BH / 2) / (g.BH > 0 ? g.BH : 1);
-    if (want < 1) want = 1;
-    if (want > g.nchunks) want = g.nchunks > 0 ? g.nchunks : 1;
-    g.cps = (g.nchunks + want - 1) / want;
-    if (g.cps < 1) g.cps = 1;
+    // Segments per head.  The passes run one CTA per SM; a CTA costs about (chunks + 2) chunk
+    // periods (state entry and pipeline fill come to ~2), both passes run on the same grid, and
+    // with more than one segment the prepass adds ~0.3 chunk period per chunk.  Pick the count
+    // that minimises waves x that cost.
+    const int nsm = sm_count();
+    g.cps = g.nchunks > 0 ? g.nchunks : 1;
+    double best = 1e300;
+    for (int G = 1; G <= g.nchunks && G <= 256; ++G) {
+        const int cps = (g.nchunks + G - 1) / G;
+        const int Geff = (g.nchunks + cps - 1) / cps;
+        if (Geff != G) continue;
+        const long long waves = ((long long)g.BH * G + nsm - 1) / nsm;
+        const double cost = (double)waves * (2.0 * (cps + 2) + (G > 1 ? 0.3 * cps : 0.0));
+        if (cost < best - 1e-9) {
+            best = cost;
+            g.cps = cps;
+        }
+    }
     g.G = g.nchunks > 0 ? (g.nchunks + g.cps - 1) / g.cps : 1;
     g.Lseg = g.cps * kC;
     return g;
