@@ -276,28 +276,45 @@ __global__ void k_state_scan(int BH, int nch, int M, int D, const float *erel, c
         const int R2 = 2 * M;
         const float cs = erel[((size_t)kC * M + m) * 2], sn = erel[((size_t)kC * M + m) * 2 + 1];
         float re = 0.f, im = 0.f;
-        for (int s = 0; s < nch; ++s) {
-            const int c = reverse ? nch - 1 - s : s;
-            const size_t base = (((size_t)bh * nch + c) * 2 + x) * R2;
-            wout[(base + 2 * m) * D + e] = __float2bfloat16_rn(re);
-            wout[(base + 2 * m + 1) * D + e] = __float2bfloat16_rn(im);
-            const float ar = re + contrib[(base + 2 * m) * D + e], ai = im + contrib[(base + 2 * m + 1) * D + e];
-            if (!reverse) {          // rot by +m w C
-                re = cs * ar - sn * ai;
-                im = sn * ar + cs * ai;
-            } else {                 // transpose: rot by -m w C
-                re = cs * ar + sn * ai;
-                im = -sn * ar + cs * ai;
+        // the contributions of eight chunks are loaded before they are used, so that their
+        // latencies overlap
+        for (int s0 = 0; s0 < nch; s0 += 8) {
+            float cr[8], ci[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                cr[j] = ci[j] = 0.f;
+                if (s0 + j < nch) {
+                    const int c = reverse ? nch - 1 - (s0 + j) : s0 + j;
+                    const size_t base = (((size_t)bh * nch + c) * 2 + x) * R2;
+                    cr[j] = __ldg(contrib + (base + 2 * m) * D + e);
+                    ci[j] = __ldg(contrib + (base + 2 * m + 1) * D + e);
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                if (s0 + j >= nch) break;
+                const int c = reverse ? nch - 1 - (s0 + j) : s0 + j;
+                const size_t base = (((size_t)bh * nch + c) * 2 + x) * R2;
+                wout[(base + 2 * m) * D + e] = __float2bfloat16_rn(re);
+                wout[(base + 2 * m + 1) * D + e] = __float2bfloat16_rn(im);
+                const float ar = re + cr[j], ai = im + ci[j];
+                if (!reverse) {          // rot by +m w C
+                    re = cs * ar - sn * ai;
+                    im = sn * ar + cs * ai;
+                } else {                 // transpose: rot by -m w C
+                    re = cs * ar + sn * ai;
+                    im = -sn * ar + cs * ai;
+                }
             }
         }
     }
 }
-
-// rowsum(dO * O) per chunk row: dl[z][row], zero beyond L.
+// rowsum(dO o) per token: one warp per row, each lane reading D/32 consecutive elements.
 __global__ void k_rowdot(int BH, int L, int nch, int D, const bf16 *dout, const bf16 *o, float *dl) {
-    const long long total = (long long)BH * nch * kC;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
+    const long long rows = (long long)BH * nch * kC;
+    const int lane = threadIdx.x & 31;
+    const long long warps = (long long)gridDim.x * (blockDim.x >> 5);
+    for (long long i = blockIdx.x * (long long)(blockDim.x >> 5) + (threadIdx.x >> 5); i < rows; i += warps) {
         const int row = (int)(i % kC);
         const long long z = i / kC;
         const int bh = (int)(z / nch), c = (int)(z % nch);
@@ -305,9 +322,15 @@ __global__ void k_rowdot(int BH, int L, int nch, int D, const bf16 *dout, const 
         float acc = 0.f;
         if (t < L) {
             const bf16 *a = dout + ((size_t)bh * L + t) * D, *b = o + ((size_t)bh * L + t) * D;
-            for (int j = 0; j < D; ++j) acc = fmaf(__bfloat162float(a[j]), __bfloat162float(b[j]), acc);
+            for (int j = lane * 2; j < D; j += 64) {
+                const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(a + j));
+                const float2 y = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(b + j));
+                acc = fmaf(x.x, y.x, fmaf(x.y, y.y, acc));
+            }
         }
-        dl[i] = acc;
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+        if (lane == 0) dl[i] = acc;
     }
 }
 
@@ -514,8 +537,8 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     if ((e = gemm(g, 1, R2, dGK, ZK, ebKR, SHK, kC, &dOK, &SEQK, &wbK, &WV_K, D, ep, st))) return e;
     {
         long long total = (long long)Z * kC;
-        int blocks = (int)((total + 255) / 256);
-        if (blocks > 8192) blocks = 8192;
+        int blocks = (int)((total + 7) / 8);   // eight rows (warps) per block
+        if (blocks > 16384) blocks = 16384;
         ProfScope ps(BLA_K_BWD, st);
         k_rowdot<<<blocks, 256, 0, st>>>(g.BH, g.L, g.nch, D, (const bf16 *)dout, (const bf16 *)o, dl);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
