@@ -209,14 +209,21 @@ __global__ void __launch_bounds__(kThreads, 1)
                         for (int i = 0; i < 32; ++i)
                             if (g0 + i > row) v[i] = 0.f;
                     } else if (e.op == EP_ROT) {
+                        // e^{i m w row} for the 16 modes of this block: the table's first phase, then
+                        // products with e^{i w row} (16 steps; rounding far below bf16 resolution)
+                        const int m0 = g0 >> 1;
+                        float cs = e.erel[((size_t)row * e.M + m0) * 2];
+                        float sn = e.erel[((size_t)row * e.M + m0) * 2 + 1];
+                        const float c1 = e.erel[((size_t)row * e.M + 1) * 2], s1 = e.erel[((size_t)row * e.M + 1) * 2 + 1];
 #pragma unroll
                         for (int i = 0; i < 32; i += 2) {
-                            const int m = (g0 + i) >> 1;
-                            const float cs = e.erel[((size_t)row * e.M + m) * 2];
-                            const float sn = e.rot_sign * e.erel[((size_t)row * e.M + m) * 2 + 1];
+                            const float sg = e.rot_sign * sn;
                             const float xr = v[i], xi = v[i + 1];
-                            v[i] = e.scale * (cs * xr - sn * xi);
-                            v[i + 1] = e.scale * (sn * xr + cs * xi);
+                            v[i] = e.scale * (cs * xr - sg * xi);
+                            v[i + 1] = e.scale * (sg * xr + cs * xi);
+                            const float t = cs * c1 - sn * s1;
+                            sn = sn * c1 + cs * s1;
+                            cs = t;
                         }
                     } else if (e.op == EP_PROB) {
 #pragma unroll
@@ -227,11 +234,26 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else if (e.op == EP_DS) {
                         const bf16 *pr = e.pbuf + ((size_t)z * kC + row) * e.ldp + g0;
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = __bfloat162float(pr[i]) * (v[i] - dl);
+                        for (int i = 0; i < 32; i += 8) {
+                            const uint4 pk = __ldg(reinterpret_cast<const uint4 *>(pr + i));
+                            const uint32_t w[4] = {pk.x, pk.y, pk.z, pk.w};
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) {
+                                const float2 pf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[q]));
+                                v[i + 2 * q] = pf.x * (v[i + 2 * q] - dl);
+                                v[i + 2 * q + 1] = pf.y * (v[i + 2 * q + 1] - dl);
+                            }
+                        }
                     } else if (e.op == EP_ADD) {
                         const float *ad = e.addend + ((size_t)z * kC + row) * e.ldo + g0;
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] += ad[i];
+                        for (int i = 0; i < 32; i += 4) {
+                            const float4 a4 = __ldg(reinterpret_cast<const float4 *>(ad + i));
+                            v[i] += a4.x;
+                            v[i + 1] += a4.y;
+                            v[i + 2] += a4.z;
+                            v[i + 3] += a4.w;
+                        }
                     }
                 }
                 if (!live) continue;
