@@ -117,11 +117,14 @@ __device__ __forceinline__ void load_block(const CUtensorMap *map, const Operand
 
 constexpr int kMaxStages = 4;
 
+// Persistent: CTA i takes tiles i, i + gridDim.x, ... (tile = (z, 128-row M tile), z fastest
+// within an M tile).  The producer streams every tile's K blocks through one shared-memory ring;
+// the MMA issuer alternates between two TMEM accumulators, so the epilogue drains tile j while
+// the MMAs of tile j+1 run.
 __global__ void __launch_bounds__(kThreads, 1)
     k_bgemm(const __grid_constant__ CUtensorMap mA0, const __grid_constant__ CUtensorMap mB0,
-            const __grid_constant__ CUtensorMap mA1, const __grid_constant__ CUtensorMap mB1, GemmArgs g, int stages) {
-    const int z = blockIdx.x, mt = blockIdx.y;
-    const int bh = z / g.nchunks, c = z % g.nchunks;
+            const __grid_constant__ CUtensorMap mA1, const __grid_constant__ CUtensorMap mB1, GemmArgs g, int stages,
+            int ntiles) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const int N = g.N;
@@ -129,16 +132,18 @@ __global__ void __launch_bounds__(kThreads, 1)
     const size_t stage_bytes = a_bytes + b_bytes;
     uint64_t *full = reinterpret_cast<uint64_t *>(sm + stages * stage_bytes);
     uint64_t *empty = full + kMaxStages;
-    uint64_t *done = empty + kMaxStages;
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(done + 1);
-    Ctl *ctl = reinterpret_cast<Ctl *>(done + 2);
+    uint64_t *acc_full = empty + kMaxStages;   // [2]
+    uint64_t *acc_empty = acc_full + 2;        // [2], one arrival per epilogue warp
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(acc_empty + 2);
+    Ctl *ctl = reinterpret_cast<Ctl *>(acc_empty + 3);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const uint32_t ncols = N <= 32 ? 32u : N <= 64 ? 64u : N <= 128 ? 128u : 256u;
+    const uint32_t ncols = N <= 16 ? 32u : N <= 32 ? 64u : N <= 64 ? 128u : N <= 128 ? 256u : 512u;   // 2 x N
     const int kb0 = g.t[0].K / 64, nkb = kb0 + (g.nterms > 1 ? g.t[1].K / 64 : 0);
+    const int Z = g.BH * g.nchunks;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < stages; ++i) { tc::mbar_init(&full[i], 1); tc::mbar_init(&empty[i], 1); }
-        tc::mbar_init(done, 1);
+        for (int i = 0; i < 2; ++i) { tc::mbar_init(&acc_full[i], 1); tc::mbar_init(&acc_empty[i], 4); }
         ctl->abort = 0;
         tc::fence_barrier_init();
     }
@@ -150,39 +155,58 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (warp == 4 && lane == 0) {
         uint32_t ph[kMaxStages] = {0, 0, 0, 0};
-        for (int it = 0; it < nkb; ++it) {
-            const int st = it % stages;
-            if (it >= stages && !wait_bar(&empty[st], ph[st], ctl, g.err, 1)) break;
-            const int term = it < kb0 ? 0 : 1, kb = it < kb0 ? it : it - kb0;
-            const Term &t = g.t[term];
-            uint8_t *base = sm + st * stage_bytes;
-            tc::mbar_arrive_expect_tx(&full[st], (uint32_t)stage_bytes);
-            load_block(term ? &mA1 : &mA0, t.A, kC, kb, mt * kC, z, bh, c, base, &full[st]);
-            load_block(term ? &mB1 : &mB0, t.B, N, kb, 0, z, bh, c, base + a_bytes, &full[st]);
+        long long it = 0;   // K blocks issued so far, over all tiles of this CTA
+        bool bad = false;
+        for (int tile = blockIdx.x; tile < ntiles && !bad; tile += gridDim.x) {
+            const int z = tile % Z, mt = tile / Z;
+            const int bh = z / g.nchunks, c = z % g.nchunks;
+            for (int kk = 0; kk < nkb; ++kk, ++it) {
+                const int st = (int)(it % stages);
+                if (it >= stages && !wait_bar(&empty[st], ph[st], ctl, g.err, 1)) { bad = true; break; }
+                const int term = kk < kb0 ? 0 : 1, kb = kk < kb0 ? kk : kk - kb0;
+                const Term &t = g.t[term];
+                uint8_t *base = sm + st * stage_bytes;
+                tc::mbar_arrive_expect_tx(&full[st], (uint32_t)stage_bytes);
+                load_block(term ? &mA1 : &mA0, t.A, kC, kb, mt * kC, z, bh, c, base, &full[st]);
+                load_block(term ? &mB1 : &mB0, t.B, N, kb, 0, z, bh, c, base + a_bytes, &full[st]);
+            }
         }
     } else if (warp == 5 && lane == 0) {
-        uint32_t ph[kMaxStages] = {0, 0, 0, 0};
-        for (int it = 0; it < nkb; ++it) {
-            const int st = it % stages;
-            if (!wait_bar(&full[st], ph[st], ctl, g.err, 2)) break;
-            tc::tc_fence_after();
-            const int term = it < kb0 ? 0 : 1;
-            const Term &t = g.t[term];
-            const uint32_t idesc = tc::idesc_bf16(128, N, !t.A.kmajor, !t.B.kmajor);
-            const uint32_t a = tc::smem_u32(sm + st * stage_bytes), b = a + (uint32_t)a_bytes;
-            for (int k = 0; k < 4; ++k)
-                tc::mma_bf16(tb, t.A.kmajor ? kmaj_desc(a, k) : mnmaj_desc(a, k),
-                             t.B.kmajor ? kmaj_desc(b, k) : mnmaj_desc(b, k), idesc, (it > 0 || k > 0) ? 1u : 0u);
-            tc::mma_commit(&empty[st]);
+        uint32_t ph[kMaxStages] = {0, 0, 0, 0}, ph_ae[2] = {0, 0};
+        long long it = 0;
+        int j = 0;   // tiles of this CTA so far
+        bool bad = false;
+        for (int tile = blockIdx.x; tile < ntiles && !bad; tile += gridDim.x, ++j) {
+            const int buf = j & 1;
+            // the accumulator's previous tile (j - 2) must have been drained
+            if (j >= 2 && !wait_bar(&acc_empty[buf], ph_ae[buf], ctl, g.err, 4)) break;
+            const uint32_t acc = tb + (uint32_t)(buf * N);
+            for (int kk = 0; kk < nkb; ++kk, ++it) {
+                const int st = (int)(it % stages);
+                if (!wait_bar(&full[st], ph[st], ctl, g.err, 2)) { bad = true; break; }
+                tc::tc_fence_after();
+                const int term = kk < kb0 ? 0 : 1;
+                const Term &t = g.t[term];
+                const uint32_t idesc = tc::idesc_bf16(128, N, !t.A.kmajor, !t.B.kmajor);
+                const uint32_t a = tc::smem_u32(sm + st * stage_bytes), b = a + (uint32_t)a_bytes;
+                for (int k = 0; k < 4; ++k)
+                    tc::mma_bf16(acc, t.A.kmajor ? kmaj_desc(a, k) : mnmaj_desc(a, k),
+                                 t.B.kmajor ? kmaj_desc(b, k) : mnmaj_desc(b, k), idesc, (kk > 0 || k > 0) ? 1u : 0u);
+                tc::mma_commit(&empty[st]);
+            }
+            tc::mma_commit(&acc_full[buf]);
         }
-        tc::mma_commit(done);
-        uint32_t ph_done = 0;
-        tc::mbar_wait(done, ph_done);
     } else if (warp < 4) {
-        uint32_t ph = 0;
-        const bool ok = wait_bar(done, ph, ctl, g.err, 3);
-        tc::tc_fence_after();
-        if (ok) {
+        uint32_t ph_af[2] = {0, 0};
+        int j = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++j) {
+            const int buf = j & 1;
+            const int z = tile % Z, mt = tile / Z;
+            const int bh = z / g.nchunks, c = z % g.nchunks;
+            if (!wait_bar(&acc_full[buf], ph_af[buf], ctl, g.err, 3)) break;
+            tc::tc_fence_after();
+            const uint32_t tacc = tb + (uint32_t)(buf * N);
+            {
             const Epi &e = g.e;
             const int row = threadIdx.x, lane_base = warp * 32;
             const int orow = mt * kC + row;
@@ -198,7 +222,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const float dl = (e.op == EP_DS) ? e.dl[(size_t)z * kC + row] : 0.f;
             for (int g0 = 0; g0 < e.ncols_out; g0 += 32) {
                 float v[32];
-                if (g0 < N) tc::tmem_ld32(tb + ((uint32_t)lane_base << 16) + (uint32_t)g0, v);
+                if (g0 < N) tc::tmem_ld32(tacc + ((uint32_t)lane_base << 16) + (uint32_t)g0, v);
                 else {
 #pragma unroll
                     for (int i = 0; i < 32; ++i) v[i] = 0.f;
@@ -270,6 +294,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                                        tc::pack_bf16x2(v[i + 4], v[i + 5]), tc::pack_bf16x2(v[i + 6], v[i + 7]));
                 }
             }
+            }
+            // the accumulator may take tile j + 2
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&acc_empty[buf]);
         }
     }
     tc::tc_fence_before();
@@ -438,6 +467,14 @@ Epi epi_base(int op, void *out, int out_mode, int out_f32, int ldo, int ncols_ou
     return e;
 }
 
+static int bwd_sm_count() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+        n <= 0)
+        return 152;
+    return n;
+}
+
 cudaError_t gemm(const BwdGeo &g, int mtiles, int N, const CUtensorMap &a0, const Operand &A0, const CUtensorMap &b0,
                  const Operand &B0, int K0, const CUtensorMap *a1, const Operand *A1, const CUtensorMap *b1,
                  const Operand *B1, int K1, const Epi &e, cudaStream_t st) {
@@ -455,9 +492,17 @@ cudaError_t gemm(const BwdGeo &g, int mtiles, int N, const CUtensorMap &a0, cons
     const int smem = (int)(stages * stage + 256 + 1024);
     cudaError_t err = cudaFuncSetAttribute(k_bgemm, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (err != cudaSuccess) return err;
-    dim3 grid(g.Z, mtiles);
+    // persistent grid: as many CTAs as fit on the device at once (shared memory and TMEM: 2N
+    // columns each), at most one per tile
+    const int ntiles = g.Z * mtiles;
+    int per_sm = (int)((227 * 1024) / smem);
+    const int cols = N <= 16 ? 32 : N <= 32 ? 64 : N <= 64 ? 128 : N <= 128 ? 256 : 512;
+    if (per_sm > 512 / cols) per_sm = 512 / cols;
+    if (per_sm < 1) per_sm = 1;
+    int nblk = bwd_sm_count() * per_sm;
+    if (nblk > ntiles) nblk = ntiles;
     ProfScope ps(BLA_K_BWD, st);
-    k_bgemm<<<grid, kThreads, smem, st>>>(a0, b0, a1 ? *a1 : a0, b1 ? *b1 : b0, ga, stages);
+    k_bgemm<<<nblk, kThreads, smem, st>>>(a0, b0, a1 ? *a1 : a0, b1 ? *b1 : b0, ga, stages, ntiles);
     return cudaGetLastError();
 }
 
