@@ -117,26 +117,37 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
-def dist_setup(n_gpus):
+def dist_setup(n_gpus, backend="nccl"):
+    """World size, rank and local rank from the torchrun environment; joins the process group
+    (NCCL on GPUs; the CPU tests use gloo).  The group carries only timing reductions."""
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     if world > 1:
         import torch.distributed as dist
-        torch.cuda.set_device(local)
-        dist.init_process_group("nccl")
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
     return world, rank, local
 
 
 def barrier_max(value, world):
+    """The maximum of `value` over the ranks (the slowest rank's time)."""
     if world <= 1:
         return value
     import torch
     import torch.distributed as dist
-    t = torch.tensor([value], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_rate(world, units_per_rank, ms_max):
+    """Weak scaling: every rank processes its own units; the job rate is all ranks' units over the
+    slowest rank's time."""
+    return world * units_per_rank / (ms_max / 1000.0)
 
 
 def oracle_sample(w, budget_s, seed=0, form="naive"):
@@ -290,7 +301,7 @@ def main():
     bla.bla_device_error()
     ms = barrier_max(ms, world)
     tokens_per_step = w.B * w.L
-    value = world * tokens_per_step / (ms / 1000.0)
+    value = whole_job_rate(world, tokens_per_step, ms)
 
     # ---- per-kernel launch times (same steps, CUDA events on the launch stream)
     bla.bla_profile_enable(True)
@@ -331,7 +342,7 @@ def main():
             torch.cuda.synchronize()      # the step's result is on the host
         e_ms = 1000.0 * (time.perf_counter() - t0) / e_steps
         e_ms = barrier_max(e_ms, world)
-        e2e = {"value": world * tokens_per_step / (e_ms / 1000.0), "unit": "tokens/s",
+        e2e = {"value": whole_job_rate(world, tokens_per_step, e_ms), "unit": "tokens/s",
                "h2d_bytes_per_step": int(sum(x.numel() * x.element_size() for x in (qp, kp, vp))),
                "d2h_bytes_per_step": int(oh.numel() * oh.element_size()), "ms_per_step": e_ms}
         del bufs
