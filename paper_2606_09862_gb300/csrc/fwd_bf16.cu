@@ -971,9 +971,18 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                                 m4[j & 3] = fmaxf(m4[j & 3], v[j]);
                             }
                         } else {
+                            // the lags D_j do not decrease, so the visible slots are j < nvis(t): one
+                            // binary search instead of a lag load per slot
+                            int lo = 0, hi = S;
+                            while (lo < hi) {
+                                const int mid = (lo + hi) >> 1;
+                                if (sdelta[mid] <= t) lo = mid + 1;
+                                else hi = mid;
+                            }
+                            const int nvis = lo - j0;
 #pragma unroll
                             for (int j = 0; j < SH; ++j) {
-                                v[j] = (t >= sdelta[j0 + j]) ? v[j] * sl2 : -INFINITY;
+                                v[j] = (j < nvis) ? v[j] * sl2 : -INFINITY;
                                 m4[j & 3] = fmaxf(m4[j & 3], v[j]);
                             }
                         }
