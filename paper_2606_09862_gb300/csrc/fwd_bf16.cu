@@ -1052,39 +1052,41 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 // ================================================================== V pass
 
 struct VLayout {
-    size_t v, y0, bx, bz, w, phi, eb, bars, total;
+    size_t v, y0, a1, bx, bz, w, phi, bars, total;
 };
 
-// Every 128-row tile buffer holds 32 KB: p (128 x SP), G (128 x C), A'_h (128 x RH) or O (128 x d).
+// Every 128-row tile buffer holds 32 KB: p (128 x SP), G (128 x C), EB_h (128 x C), A'_h
+// (128 x RH), W_h (RH x d) or O (128 x d).
 __host__ __device__ inline VLayout v_layout(const Geo &g) {
     VLayout l;
     size_t off = 0;
     const size_t tile = (size_t)kC * 128 * 2;
     l.v = off;   off += (size_t)kC * g.D * 2;
     l.y0 = off;  off += tile;   // A'_0, then the staged output tile
-    l.bx = off;  off += tile;   // p then G, and A'_1, alternating with bz from chunk to chunk
+    l.a1 = off;  off += tile;   // A'_1
+    l.bx = off;  off += tile;   // p then G, and EB_0, alternating with bz from chunk to chunk
     l.bz = off;  off += tile;
-    l.w = off;   off += (size_t)g.RH * g.D * 2;
-    l.phi = off; off += tile;   // PHI_0, PHI_1, then EB_1
-    l.eb = off;  off += tile;   // EB_0
+    l.w = off;   off += tile;   // W_0
+    l.phi = off; off += tile;   // PHI_0, PHI_1, EB_1, then W_1
     l.bars = off; off += 1024;
     l.total = off + 1024;
     return l;
 }
 
-// One barrier per hand-off (see the K pass).  A'_0 and A'_1 each have their own ready barrier:
-// U_1 is issued before G waits for A'_0, so one barrier could complete twice before that wait.
+// One barrier per hand-off (see the K pass).  A'_0 / A'_1 and W_0 / W_1 each have their own ready
+// barrier: the second of each pair can be signalled before the MMA issuer has waited for the first.
 enum VBar {
     VB_P_FULL, VB_P_FREE, VB_V_FULL, VB_V_FREE, VB_EB_FULL, VB_EB_FREE, VB_PH_FULL, VB_PH_FREE,
-    VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_A_READY1, VB_G_READY, VB_W_READY, VB_W_FREE,
+    VB_U_FULL, VB_U_FREE, VB_G_FULL, VB_G_FREE, VB_A_READY, VB_A_READY1, VB_G_READY, VB_W_READY, VB_W_READY1, VB_W_FREE,
     VB_STATE_DONE, VB_STATE_DONE1, VB_STATE_READ, VB_O_FULL, VB_O_SMEM, VB_O_STORED, VB_EXIT, VB_COUNT
 };
 
 // V pass.  Per chunk and mode half h: U_h = p PHI_h; A'_h = e^{-i m w t} U_h (t absolute) into shared
 // memory; G = sum_h A'_h EB_h (causal mask on drain, written over p); state_h += EB_h V; and
-// O = sum_h A'_h W_h + G V.  Buffers: A'_0 and the staged output in y0; p/G and A'_1 alternate
-// between bx and bz from chunk to chunk, so the next chunk's p can load as soon as A'_1 W_1 is
-// done; the PHI tile takes EB_1 once U_1 has read PHI_1, so that EB_0 and EB_1 are both resident.
+// O = sum_h A'_h W_h + G V.  Buffers: A'_0 and the staged output in y0, A'_1 in a1; p/G and EB_0
+// alternate between bx and bz from chunk to chunk, so the next chunk's p loads into this chunk's
+// EB_0 buffer as soon as state_0 has read it; the PHI tile takes EB_1 once U_1 has read PHI_1, and
+// W_1 once state_1 has read EB_1, so O = A'_0 W_0 + A'_1 W_1 runs without a wait in between.
 template <int D, int RH, int NH>
 __global__ void __launch_bounds__(kPassThreads, 1)
     k_vpass(const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_v,
@@ -1097,16 +1099,16 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const VLayout lay = v_layout(g);
-    uint8_t *sV = sm + lay.v, *sY0 = sm + lay.y0, *sBX = sm + lay.bx, *sBZ = sm + lay.bz, *sW = sm + lay.w;
-    uint8_t *sPHI = sm + lay.phi, *sEB = sm + lay.eb;
+    uint8_t *sV = sm + lay.v, *sY0 = sm + lay.y0, *sA1 = sm + lay.a1, *sBX = sm + lay.bx, *sBZ = sm + lay.bz;
+    uint8_t *sW = sm + lay.w, *sPHI = sm + lay.phi;
     uint64_t *bar = reinterpret_cast<uint64_t *>(sm + lay.bars);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + VB_COUNT);
     Ctl *ctl = reinterpret_cast<Ctl *>(bar + VB_COUNT + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int SP = g.SP;
-    // chunk i (from c_begin) keeps p/G in pbuf(i) and A'_1 in a1buf(i) (two halves: alternating)
-    auto pbuf = [&](int i) { return (NH == 2 && (i & 1)) ? sBZ : sBX; };
-    auto a1buf = [&](int i) { return (i & 1) ? sBX : sBZ; };
+    // chunk i (from c_begin) keeps p/G in pbuf(i) and EB_0 in ebuf(i), alternating
+    auto pbuf = [&](int i) { return (i & 1) ? sBZ : sBX; };
+    auto ebuf = [&](int i) { return (i & 1) ? sBX : sBZ; };
     // TMEM: [0, NB*D) state; colU (128 cols: U_h, then O); colG (128 cols).
     const int colU = g.NB * D, colG = colU + 128;
     const uint32_t ncols = (uint32_t)(colG + 128) <= 256 ? 256u : 512u;  // host: pow2_cols(NB*D + 256)
@@ -1114,7 +1116,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     if (threadIdx.x == 0) {
         for (int i = 0; i < VB_COUNT; ++i) {
             const bool epi = i == VB_U_FREE || i == VB_G_FREE || i == VB_A_READY || i == VB_A_READY1 || i == VB_G_READY ||
-                             i == VB_W_READY || i == VB_STATE_READ || i == VB_O_SMEM;
+                             i == VB_W_READY || i == VB_W_READY1 || i == VB_STATE_READ || i == VB_O_SMEM;
             tc::mbar_init(&bar[i], epi ? kPassEpiWarps : 1);
         }
         ctl->abort = 0;
@@ -1138,20 +1140,21 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 for (int c = c_begin; c < c_end; ++c) {
                     const int i = c - c_begin;
                     const bool first = i == 0;
-                    // p: the buffer held the previous chunk's A'_1 (two halves) or G (one half)
+                    // p: the buffer held the previous chunk's EB_0 (freed once state_0 has read it)
                     if (!first && !wait_bar(&bar[VB_P_FREE], ph_p, ctl, a.err)) break;
                     tc::mbar_arrive_expect_tx(&bar[VB_P_FULL], (uint32_t)(kC * SP * 2));
                     for (int kb = 0; kb < SP / 64; ++kb)
                         tc::tma_load_3d(pbuf(i) + kb * kC * 128, &tm_p, &bar[VB_P_FULL], kb * 64, c * kC, bh);
-                    // PHI_0 (the PHI tile last held the previous chunk's EB_1, or PHI_0 with one half)
+                    // PHI_0 (the PHI tile last held the previous chunk's W_1, or PHI_0 with one half)
                     if (!first && !wait_bar(&bar[VB_PH_FREE], ph_ph, ctl, a.err)) break;
                     tc::mbar_arrive_expect_tx(&bar[VB_PH_FULL], (uint32_t)(SP * RH * 2));
                     for (int kb = 0; kb < RH / 64; ++kb)
                         tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PH_FULL], kb * 64, 0);
+                    // EB_0 into the buffer of the previous chunk's p/G (freed once G V has read it)
                     if (!first && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) break;
                     tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
                     for (int kb = 0; kb < 2; ++kb)
-                        tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP);
+                        tc::tma_load_2d(ebuf(i) + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP);
                     if (!first && !wait_bar(&bar[VB_V_FREE], ph_v, ctl, a.err)) break;
                     tc::mbar_arrive_expect_tx(&bar[VB_V_FULL], (uint32_t)(kC * D * 2));
                     for (int db = 0; db < D / 64; ++db)
@@ -1174,7 +1177,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             // state_0 += EB_0 V; G += A'_1 EB_1; state_1 += EB_1 V; O = A'_0 W_0 (+ A'_1 W_1); O += G V.
             if (lane == 0) {
                 uint32_t ph_p = 0, ph_v = 0, ph_eb = 0, ph_ph = 0, ph_ufree = 0, ph_gfree = 0, ph_a0 = 0, ph_a1 = 0, ph_gready = 0;
-                uint32_t ph_w = 0, ph_sread = 0;
+                uint32_t ph_w0 = 0, ph_w1 = 0, ph_sread = 0;
                 const uint32_t id_U = tc::idesc_bf16(128, RH, false, true);
                 const uint32_t id_G = tc::idesc_bf16(128, kC, false, true);
                 const uint32_t id_O = tc::idesc_bf16(128, D, false, true);
@@ -1182,7 +1185,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 for (int c = c_begin; c < c_end; ++c) {
                     const int i = c - c_begin;
                     const bool first = i == 0;
-                    uint8_t *sP = pbuf(i), *sA1 = a1buf(i);
+                    uint8_t *sP = pbuf(i), *sE0 = ebuf(i);
                     // U_0 -> U (last read by the previous chunk's O drain)
                     if (!wait_bar(&bar[VB_P_FULL], ph_p, ctl, a.err)) break;
                     if (!wait_bar(&bar[VB_PH_FULL], ph_ph, ctl, a.err)) break;
@@ -1205,15 +1208,15 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) break;
                     if (!first && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) break;
                     tc::tc_fence_after();
-                    mma_steps<true>(accG, sY0, kC, sEB, 128, id_G, RH / 16, false);
+                    mma_steps<true>(accG, sY0, kC, sE0, 128, id_G, RH / 16, false);
                     if (NH == 1) tc::mma_commit(&bar[VB_G_FULL]);
                     // state_0 += EB_0 V once this chunk's W tiles have been read from the state
                     if (!wait_bar(&bar[VB_STATE_READ], ph_sread, ctl, a.err)) break;
                     if (!wait_bar(&bar[VB_V_FULL], ph_v, ctl, a.err)) break;
                     tc::tc_fence_after();
-                    mma_steps<true>(tb, sEB, 128, sV, kC, id_O, kC / 16, true);
+                    mma_steps<true>(tb, sE0, 128, sV, kC, id_O, kC / 16, true);
                     tc::mma_commit(&bar[VB_STATE_DONE]);
-                    tc::mma_commit(&bar[VB_EB_FREE]);
+                    tc::mma_commit(&bar[VB_P_FREE]);   // EB_0's buffer takes the next chunk's p
                     if (NH == 2) {
                         // G += A'_1 EB_1 (EB_1 in the PHI tile); state_1 += EB_1 V
                         if (!wait_bar(&bar[VB_A_READY1], ph_a1, ctl, a.err)) break;
@@ -1222,22 +1225,20 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         mma_steps<true>(accG, sA1, kC, sPHI, 128, id_G, RH / 16, true);
                         tc::mma_commit(&bar[VB_G_FULL]);
                         mma_steps<true>(tb + D, sPHI, 128, sV, kC, id_O, kC / 16, true);
-                        tc::mma_commit(&bar[VB_STATE_DONE1]);
-                        tc::mma_commit(&bar[VB_PH_FREE]);
+                        tc::mma_commit(&bar[VB_STATE_DONE1]);   // the PHI tile may take W_1
                     }
                     // O = A'_0 W_0 -> U once the last A' has been drained
                     if (!wait_bar(&bar[VB_U_FREE], ph_ufree, ctl, a.err)) break;
-                    if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_W_READY], ph_w0, ctl, a.err)) break;
                     tc::tc_fence_after();
                     mma_steps<true>(accU, sY0, kC, sW, RH, id_O, RH / 16, false);
                     tc::mma_commit(&bar[VB_W_FREE]);
                     if (NH == 2) {
-                        // O += A'_1 W_1; A'_1's buffer then takes the next chunk's p
-                        if (!wait_bar(&bar[VB_W_READY], ph_w, ctl, a.err)) break;
+                        // O += A'_1 W_1 (W_1 in the PHI tile, which then takes the next PHI_0)
+                        if (!wait_bar(&bar[VB_W_READY1], ph_w1, ctl, a.err)) break;
                         tc::tc_fence_after();
-                        mma_steps<true>(accU, sA1, kC, sW, RH, id_O, RH / 16, true);
-                        tc::mma_commit(&bar[VB_W_FREE]);
-                        tc::mma_commit(&bar[VB_P_FREE]);
+                        mma_steps<true>(accU, sA1, kC, sPHI, RH, id_O, RH / 16, true);
+                        tc::mma_commit(&bar[VB_PH_FREE]);
                     }
                     // O += G V (G written over p by the epilogue)
                     if (!wait_bar(&bar[VB_G_READY], ph_gready, ctl, a.err)) break;
@@ -1245,7 +1246,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     mma_steps<true>(accU, sP, kC, sV, kC, id_O, kC / 16, true);
                     tc::mma_commit(&bar[VB_O_FULL]);
                     tc::mma_commit(&bar[VB_V_FREE]);
-                    if (NH == 1) tc::mma_commit(&bar[VB_P_FREE]);
+                    tc::mma_commit(&bar[VB_EB_FREE]);   // p/G's buffer takes the next chunk's EB_0
                 }
                 tc::mma_commit(&bar[VB_EXIT]);
                 uint32_t ph_exit = 0;
@@ -1286,15 +1287,19 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
                 state_init_abs<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D, f.x, f.y);
             }
-            auto w_store = [&](bool wait_free, const uint32_t *pk) -> bool {
-                if (wait_free && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) return false;
+            // W_0 goes to the W tile once the previous chunk's O = A'_0 W_0 has read it; W_1 goes to the
+            // PHI tile once state_1 has read EB_1 there
+            auto w_store = [&](int h, bool wait_free, const uint32_t *pk) -> bool {
+                if (h == 0 && wait_free && !wait_bar(&bar[VB_W_FREE], ph_wfree, ctl, a.err)) return false;
+                if (h == 1 && !wait_bar(&bar[VB_STATE_DONE1], ph_states, 1, ctl, a.err)) return false;
+                uint8_t *dst = h ? sPHI : sW;
                 if (row < RH) {
 #pragma unroll
-                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_packed(sW, RH, row, wg * DH + g0, pk + g0 / 2);
+                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_packed(dst, RH, row, wg * DH + g0, pk + g0 / 2);
                 }
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
-                epi_arrive(&bar[VB_W_READY]);
+                epi_arrive(&bar[VB_W_READY + h]);
                 return true;
             };
             bool bad = false;
@@ -1302,17 +1307,16 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 const int i = c - c_begin;
                 const bool rot = i > 0;
                 if (rot) advance(rp, rp_step);
-                // W_h: the V state before this chunk's update, into registers
+                // W_h: the V state before this chunk's update, into registers (state_1's previous update
+                // was awaited before the previous chunk's W_1 store)
                 uint32_t pk0[DH / 2], pk1[DH / 2];
-                for (int h = 0; h < NH; ++h)
-                    if (rot && !wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
-                if (bad) break;
+                if (rot && !wait_bar(&bar[VB_STATE_DONE], ph_states, 0, ctl, a.err)) break;
                 tc::tc_fence_after();
                 state_pack<DH>(tb, wg * DH, row, pk0);
                 if (NH == 2) state_pack<DH>(tb, D + wg * DH, row, pk1);
                 tc::tc_fence_before();
                 epi_arrive(&bar[VB_STATE_READ]);
-                if (!w_store(rot, pk0)) { bad = true; break; }
+                if (!w_store(0, rot, pk0)) { bad = true; break; }
                 // A'_h = e^{-i m w t} U_h (t absolute); y0 held the previous chunk's output tile until
                 // the store read it
                 if (rot && !wait_bar(&bar[VB_O_STORED], ph_ostored, ctl, a.err)) break;
@@ -1343,15 +1347,15 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         cb = t1;
                         sb = t2;
                     }
-                    uint8_t *dstA = h ? a1buf(i) : sY0;
+                    uint8_t *dstA = h ? sA1 : sY0;
 #pragma unroll
                     for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(dstA, kC, row, wg * XH + g0, v + g0);
                     tc::fence_proxy_async_smem();
                     epi_arrive(&bar[VB_A_READY + h]);
                 }
                 if (bad) break;
-                // W_1 once O = A'_0 W_0 has read W_0
-                if (NH == 2 && !w_store(true, pk1)) { bad = true; break; }
+                // W_1 into the PHI tile once state_1 has read EB_1 there
+                if (NH == 2 && !w_store(1, true, pk1)) { bad = true; break; }
                 // G drain -> causal mask -> bf16 over p (U_0 and U_1 are done once G is full)
                 if (!wait_bar(&bar[VB_G_FULL], ph_g, ctl, a.err)) break;
                 tc::tc_fence_after();
@@ -1383,8 +1387,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 }
             }
             if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
-                for (int h = 0; h < NH; ++h)
-                    if (!wait_bar(&bar[VB_STATE_DONE + h], ph_states, h, ctl, a.err)) { bad = true; break; }
+                // the last chunk's state_1 update was awaited before its W_1 store
+                if (!wait_bar(&bar[VB_STATE_DONE], ph_states, 0, ctl, a.err)) bad = true;
                 if (!bad) {
                     tc::tc_fence_after();
                     for (int b = 0; b < g.NB; ++b) {
