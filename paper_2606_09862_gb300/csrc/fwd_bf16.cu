@@ -685,6 +685,14 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         tc::tma_load_3d(sQ + db * kC * 128, &tm_q, &bar[KB_QK_FULL], db * 64, c * kC, bh);
                         tc::tma_load_3d(sK + db * kC * 128, &tm_k, &bar[KB_QK_FULL], db * 64, c * kC, bh);
                     }
+                    // the next chunk's q and k into L2 now: their loads wait for this chunk's state_1
+                    // update and would otherwise pay the full memory latency on the chunk's critical path
+                    if (c + 1 < c_end) {
+                        for (int db = 0; db < D / 64; ++db) {
+                            tc::tma_prefetch_3d(&tm_q, db * 64, (c + 1) * kC, bh);
+                            tc::tma_prefetch_3d(&tm_k, db * 64, (c + 1) * kC, bh);
+                        }
+                    }
                     for (int h = 0; h < NH; ++h) {
                         if (!first_eb && !wait_bar(&bar[KB_EB_FREE], ph_eb, ctl, a.err)) break;
                         first_eb = false;
