@@ -137,7 +137,8 @@ __device__ __forceinline__ void mode_phase(long long mu, double w, int tint, flo
 //         with nch = 1 this is the in-chunk table (c = 0) of the lag frame
 //   PHI   [SP][R2]: PHI[j][2m] = c_m cos(m w D_j), PHI[j][2m+1] = c_m sin(m w D_j), D_j = round(j T / S),
 //         c_0 = 1/(2M-1), c_m = 2/(2M-1)
-//   FSEG  [RP][Lseg] (optional): FSEG[2m][u] = cos(m w (Lseg - u)), FSEG[2m+1][u] = sin(m w (Lseg - u))
+//   FSEG  [RP][Lseg] (optional): FSEG[2m][u] = cos(m w (Lseg - u)), FSEG[2m+1][u] = sin(m w (Lseg - u)),
+//         eight entries per thread as for EB
 //   delta [S] (optional): the slot lags D_j
 // EB is written by one thread per (c, m, 8 consecutive u), u fastest so that a warp writes whole
 // rows: the first phase is reduced exactly, the next seven follow by products with e^{i m w}.
@@ -145,7 +146,7 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, d
                               bf16 *eb, bf16 *phi, bf16 *fseg, int *delta) {
     const int R2 = 2 * M, MP = RP / 2;
     const long long n_eb = (long long)nch * MP * (kC / 8), n_phi = (long long)SP * R2;
-    const long long n_f = fseg ? (long long)RP * Lseg : 0, n_d = delta ? S : 0;
+    const long long n_f = fseg ? (long long)MP * ((Lseg + 7) / 8) : 0, n_d = delta ? S : 0;
     const long long total = n_eb + n_phi + n_f + n_d;
     const double n = 2.0 * M - 1.0;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
@@ -188,15 +189,23 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, d
             }
             phi[e] = __float2bfloat16_rn(v);
         } else if (i < n_eb + n_phi + n_f) {
+            // FSEG rows 2m, 2m+1 for 8 consecutive u: e^{i m w (Lseg - u)}, stepping by e^{-i m w}
             const long long e = i - n_eb - n_phi;
-            const int r = (int)(e / Lseg), u = (int)(e % Lseg), m = r >> 1;
-            float v = 0.f;
-            if (r < R2) {
-                float c, sn;
-                mode_phase((long long)m * (Lseg - u), w, tint, &c, &sn);
-                v = (r & 1) ? sn : c;
+            const int per_m = (Lseg + 7) / 8;
+            const int m = (int)(e / per_m), u0 = (int)(e % per_m) * 8;
+            bf16 *rc = fseg + (size_t)(2 * m) * Lseg + u0, *rs = rc + Lseg;
+            float bc = 0.f, bs = 0.f, ec = 1.f, es = 0.f;
+            if (m < M) {
+                mode_phase((long long)m * (Lseg - u0), w, tint, &bc, &bs);
+                mode_phase((long long)m, w, tint, &ec, &es);
             }
-            fseg[e] = __float2bfloat16_rn(v);
+            for (int j = 0; j < 8 && u0 + j < Lseg; ++j) {
+                rc[j] = __float2bfloat16_rn(bc);
+                rs[j] = __float2bfloat16_rn(bs);
+                const float t = bc * ec + bs * es;   // times e^{-i m w}
+                bs = bs * ec - bc * es;
+                bc = t;
+            }
         } else {
             const int j = (int)(i - n_eb - n_phi - n_f);
             delta[j] = (int)rint((double)j * T / (double)S);
@@ -1565,7 +1574,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     {
         // EB of every chunk (absolute phases), PHI, FSEG and the slot lags in one launch
         const long long total = (long long)g.nchunks * (g.RP / 2) * (kC / 8) + (long long)g.SP * g.R2 +
-                                (fseg ? (long long)g.RP * g.Lseg : 0) + g.S;
+                                (fseg ? (long long)(g.RP / 2) * ((g.Lseg + 7) / 8) : 0) + g.S;
         const int blocks = (int)(total < 4096 * 256 ? (total + 255) / 256 : 4096);
         ProfScope ps(BLA_K_TABLES_BF16, st);
         k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, g.nchunks, d.T, d.w, integer_period(d), eb,
