@@ -1007,10 +1007,15 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         // a half whose slots are all hidden has mx = -inf: exponentiate against 0 instead
                         const float mref = (mx == -INFINITY) ? 0.f : mx;
                         float s4[4] = {0.f, 0.f, 0.f, 0.f};
+                        // exponents in pairs through packed fp16 ex2: the probabilities are stored in
+                        // bf16, whose resolution (2^-8) is coarser than the fp16 path's error
 #pragma unroll
-                        for (int j = 0; j < SH; ++j) {
-                            v[j] = exp2f(v[j] - mref);          // exp2(-inf) = 0 on masked slots
-                            s4[j & 3] += v[j];
+                        for (int j = 0; j < SH; j += 2) {
+                            const float2 e2 = tc::exp2_pair_f16(v[j] - mref, v[j + 1] - mref);   // -inf -> 0
+                            v[j] = e2.x;
+                            v[j + 1] = e2.y;
+                            s4[j & 3] += e2.x;
+                            s4[(j + 1) & 3] += e2.y;
                         }
                         sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
                     }
