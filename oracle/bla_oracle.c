@@ -37,6 +37,10 @@
  *   orc_backward_parallel vector-Jacobian product of the parallel form, written out
  *                         by the chain rule (no paper counterpart; pinned to central
  *                         finite differences of orc_forward_naive by the tests).
+ *                         With form 3 it is the VJP of the absolute form instead: the
+ *                         same chain rule with the weight D_M(t' - Delta_j) of Alg. 1's
+ *                         "interpolate" in place of D_M(t - t' - Delta_j) (pinned to
+ *                         finite differences of orc_forward_absolute).
  */
 #include <math.h>
 #include <stdlib.h>
@@ -347,7 +351,7 @@ static void head_absolute(const orc_cfg *c, const double *A, const double *B, co
 
 /* ------------------------------------ VJP of the parallel form (chain rule)
  *
- *   W[t,t',j] = D_M(t - t' - Delta_j)            (t' <= t)
+ *   W[t,t',j] = D_M(t - t' - Delta_j)            (t' <= t; absolute form: D_M(t' - Delta_j))
  *   s[t,j]    = scale sum_t' W (q_t . k_t'),     p = masked softmax_j(s)
  *   G[t,t']   = sum_j p[t,j] W[t,t',j],          o_t = sum_t' G[t,t'] v_t'
  * Given do:
@@ -356,7 +360,13 @@ static void head_absolute(const orc_cfg *c, const double *A, const double *B, co
  *   dP[t,t']  = scale sum_j ds[t,j] W[t,t',j]
  *   dq_t = sum_t' dP[t,t'] k_t',  dk_t' = sum_t dP[t,t'] q_t,  dv_t' = sum_t G[t,t'] do_t
  */
-static void head_backward(const orc_cfg *c, const double *delta,
+/* Index of D_M in the weight W[t,t',j]: lag form t - t' - Delta_j, absolute form t' - Delta_j. */
+static int weight_arg(int absolute, int t, int u, int dj)
+{
+    return absolute ? u - dj : t - u - dj;
+}
+
+static void head_backward(const orc_cfg *c, const double *delta, int absolute,
                           const double *q, const double *k, const double *v, const double *dout,
                           double *dq, double *dk_, double *dv_)
 {
@@ -378,7 +388,7 @@ static void head_backward(const orc_cfg *c, const double *delta,
         for (int j = 0; j < S; ++j) {
             double a = 0.0, b = 0.0;
             for (int u = 0; u <= t; ++u) {
-                double wgt = Dt[t - u - (int)delta[j] + off];
+                double wgt = Dt[weight_arg(absolute, t, u, (int)delta[j]) + off];
                 a += wgt * qk[u]; b += wgt * dov[u];
             }
             s[j] = c->scale * a; dp[j] = b;
@@ -389,7 +399,7 @@ static void head_backward(const orc_cfg *c, const double *delta,
         for (int u = 0; u <= t; ++u) {
             double g = 0.0, dP = 0.0;
             for (int j = 0; j < S; ++j) {
-                double wgt = Dt[t - u - (int)delta[j] + off];
+                double wgt = Dt[weight_arg(absolute, t, u, (int)delta[j]) + off];
                 g += p[j] * wgt;
                 dP += p[j] * (dp[j] - pdp) * wgt;
             }
@@ -449,18 +459,19 @@ int orc_forward(int form, int NH, int L, int dk, int dv, int M, int S, double T,
     return (form >= 0 && form <= 3) ? 0 : 3;
 }
 
-int orc_backward(int NH, int L, int dk, int dv, int M, int S, double T, double omega, double scale,
+int orc_backward(int form, int NH, int L, int dk, int dv, int M, int S, double T, double omega, double scale,
                  const double *q, const double *k, const double *v, const double *dout,
                  double *dq, double *dk_, double *dv_)
 {
     if (NH < 0 || L < 0 || dk < 1 || dv < 1 || M < 1 || S < 1) return 1;
+    if (form != 2 && form != 3) return 3;
     orc_cfg c = make_cfg(L, dk, dv, M, S, T, omega, scale, 0);
     double *delta = malloc(sizeof(double) * S);
     orc_delta(M, S, T, delta);
     #pragma omp parallel for schedule(dynamic, 1)
     for (int h = 0; h < NH; ++h) {
         size_t ok = (size_t)h * L * dk, ov = (size_t)h * L * dv;
-        head_backward(&c, delta, q + ok, k + ok, v + ov, dout + ov, dq + ok, dk_ + ok, dv_ + ov);
+        head_backward(&c, delta, form == 3, q + ok, k + ok, v + ov, dout + ov, dq + ok, dk_ + ok, dv_ + ov);
     }
     free(delta);
     return 0;

@@ -36,7 +36,7 @@ def _configure(lib):
     lib.orc_forward.argtypes = [ctypes.c_int] * 7 + [ctypes.c_double] * 3 + [ctypes.c_longlong] + \
         [_dp] * 6 + [ctypes.c_void_p]
     lib.orc_backward.restype = ctypes.c_int
-    lib.orc_backward.argtypes = [ctypes.c_int] * 6 + [ctypes.c_double] * 3 + [_dp] * 7
+    lib.orc_backward.argtypes = [ctypes.c_int] * 7 + [ctypes.c_double] * 3 + [_dp] * 7
     lib.orc_max_threads.restype = ctypes.c_int
     return lib
 
@@ -129,15 +129,19 @@ def forward(q, k, v, M, S, T, omega=0.0, scale=0.0, form="naive", state=None, po
     return out
 
 
-def backward(q, k, v, dout, M, S, T, omega=0.0, scale=0.0):
-    """Vector-Jacobian product (dq, dk, dv) of the forward for upstream gradient dout."""
+def backward(q, k, v, dout, M, S, T, omega=0.0, scale=0.0, form="parallel"):
+    """Vector-Jacobian product (dq, dk, dv) of the forward for upstream gradient dout.
+
+    ``form`` "parallel" (any of the lag-form forwards; they agree) or "absolute" (Alg. 1)."""
+    if form not in ("parallel", "absolute"):
+        raise ValueError("backward form must be 'parallel' or 'absolute', got %r" % (form,))
     q, k, v, dout = _f64(q), _f64(k), _f64(v), _f64(dout)
     Bn, Hn, L, dk = q.shape
     dv = v.shape[-1]
     dq = np.zeros_like(q)
     dkk = np.zeros_like(k)
     dvv = np.zeros_like(v)
-    rc = _load().orc_backward(Bn * Hn, L, dk, dv, int(M), int(S), float(T), float(omega), float(scale),
+    rc = _load().orc_backward(FORMS[form], Bn * Hn, L, dk, dv, int(M), int(S), float(T), float(omega), float(scale),
                               _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(dq), _ptr(dkk), _ptr(dvv))
     if rc != 0:
         raise ValueError("oracle backward rejected its arguments (code %d)" % rc)

@@ -231,6 +231,30 @@ def lag_vs_absolute(orc, M, S, T, L=40, d=4, seed=13):
     return float(np.linalg.norm(a - b) / np.linalg.norm(a))
 
 
+def pin_absolute_bruteforce(orc):
+    """Absolute form (Alg. 1, Sec. 3.2): slot j of token t holds sum_{t'<=t} D_M(t' - Delta_j) k_t',
+    the Dirichlet kernel anchored at absolute phase Delta_j, here by brute force with the
+    sine-ratio D_M, the grid round(j T/S) and the mask t >= Delta_j computed in this file."""
+    g = rng(31)
+    err = 0.0
+    for M, S, T, L, d in ((3, 4, 10.0, 23, 3), (4, 6, 21.0, 40, 2), (3, 5, 5.0, 17, 4)):
+        q, k, v = (g.standard_normal((1, 1, L, d)) for _ in range(3))
+        r = orc.forward(q, k, v, M, S, T, form="absolute")
+        w = 2 * np.pi / T
+        delta = np.round(np.arange(S) * T / S)
+        for t in range(L):
+            u = np.arange(t + 1)
+            W = dirichlet_sine_ratio(M, w, u[None, :] - delta[:, None])   # [S, t+1]
+            Ks = W @ k[0, 0, : t + 1]
+            Vs = W @ v[0, 0, : t + 1]
+            s = Ks @ q[0, 0, t] / np.sqrt(d)
+            valid = t >= delta
+            p, lse = _softmax_masked(s[None], valid[None])
+            err = _worst(err, float(np.abs(r["o"][0, 0, t] - p[0] @ Vs).max()),
+                      float(abs(r["lse"][0, 0, t] - lse[0])))
+    return err
+
+
 # ----------------------------------------------------------- P7: one mode
 
 def pin_single_mode(orc):
@@ -258,6 +282,27 @@ def pin_backward_fd(orc, h=1e-6):
                 lp = float((orc.forward(q, k, v, M, S, T)["o"] * do).sum())
                 x[idx] = x0 - h
                 lm = float((orc.forward(q, k, v, M, S, T)["o"] * do).sum())
+                x[idx] = x0
+                fd[idx] = (lp - lm) / (2 * h)
+            err = _worst(err, float(np.abs(fd - gx).max() / (np.abs(gx).max() + 1e-30)))
+    return err
+
+
+def pin_backward_fd_absolute(orc, h=1e-6):
+    """The absolute form's VJP = central finite differences of its Alg. 1 forward, loss = sum(dO * O)."""
+    g = rng(37)
+    err = 0.0
+    for M, S, T, L, d in ((3, 4, 9.0, 8, 3), (2, 3, 7.0, 11, 2)):
+        q, k, v, do = (g.standard_normal((1, 1, L, d)) for _ in range(4))
+        dq, dk, dv = orc.backward(q, k, v, do, M, S, T, form="absolute")
+        for x, gx in ((q, dq), (k, dk), (v, dv)):
+            fd = np.zeros_like(x)
+            for idx in np.ndindex(x.shape):
+                x0 = x[idx]
+                x[idx] = x0 + h
+                lp = float((orc.forward(q, k, v, M, S, T, form="absolute")["o"] * do).sum())
+                x[idx] = x0 - h
+                lm = float((orc.forward(q, k, v, M, S, T, form="absolute")["o"] * do).sum())
                 x[idx] = x0
                 fd[idx] = (lp - lm) / (2 * h)
             err = _worst(err, float(np.abs(fd - gx).max() / (np.abs(gx).max() + 1e-30)))
@@ -293,5 +338,7 @@ ALL_PINS = {
     "forms_agree": (pin_forms_agree, 1e-11),
     "single_mode": (pin_single_mode, 1e-12),
     "backward_fd": (pin_backward_fd, 1e-6),
+    "absolute_bruteforce": (pin_absolute_bruteforce, 1e-11),
+    "backward_fd_absolute": (pin_backward_fd_absolute, 1e-6),
     "state_handoff": (pin_state_handoff, 1e-12),
 }

@@ -36,6 +36,8 @@ MUTANTS = {
     "backward_no_scale": ("dP *= c->scale;", "dP *= 1.0;"),
     "backward_no_centering": ("p[j] * (dp[j] - pdp) * wgt", "p[j] * dp[j] * wgt"),
     "dirichlet_no_factor2": ("acc += 2.0 / n * cos(m * w * x);", "acc += 1.0 / n * cos(m * w * x);"),
+    "absolute_interp_sign": ("+ sin(t * m * c->w) * B[j * M + m];", "- sin(t * m * c->w) * B[j * M + m];"),
+    "absolute_backward_lag_weight": ("return absolute ? u - dj : t - u - dj;", "return t - u - dj;"),
 }
 
 
