@@ -443,34 +443,42 @@ def measure_configs(bla, torch, dev, stream, peaks, iters=20):
                 "flops": flops, "bytes": nbytes}
 
     out = {}
-    for name in ("fwd_bf16_recall", "fwdbwd_bf16_lm"):
+    # the two parity configs in the lag form; config 3 and the long prefill also in the absolute
+    # form (phase_mode "absolute", Alg. 1), which runs the same kernels with other tables
+    for name, modes in (("fwd_bf16_recall", ("lag",)), ("fwdbwd_bf16_lm", ("lag", "absolute")),
+                        ("prefill_bf16_long", ("absolute",))):
         w = WORKLOADS[name]
         q, k, v = (torch.from_numpy(x).to(torch.bfloat16).to(dev)
                    for x in make_qkv(w.B, w.H, w.L, w.d, "bf16", seed=0, recall_dup=getattr(w, "recall_dup", 0.0)))
-        par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16)
-        ws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_FORWARD), dtype=torch.uint8, device=dev)
         res = {}
-
-        def fwd():
-            return bla.bla_forward_chunked(q, k, v, w.M, w.S, w.T, workspace=ws, stream=stream)
-
+        C = 64 if name != "prefill_bf16_long" else 128
         tok = w.B * w.L
-        F = canonical_flops(w, C=64)["total"] * w.B * w.H * w.L
+        F = canonical_flops(w, C=C)["total"] * w.B * w.H * w.L
         elem = w.B * w.H * w.L * w.d
-        res["forward"] = roof(F, 4 * elem * 2 + w.B * w.H * w.L * 4, timed(fwd), tok)
-        if getattr(w, "backward", False):
-            o, lse, _ = fwd()
-            do = torch.from_numpy(make_dout(w.B, w.H, w.L, w.d, "bf16", seed=0)).to(torch.bfloat16).to(dev)
-            bws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_BACKWARD), dtype=torch.uint8, device=dev)
+        for mode in modes:
+            sfx = "" if mode == "lag" else "_absolute"
+            par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16, phase_mode=mode)
+            ws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_FORWARD), dtype=torch.uint8, device=dev)
 
-            def bwd():
-                return bla.bla_backward(q, k, v, o, do, lse, w.M, w.S, w.T, workspace=bws, stream=stream)
+            def fwd():
+                return bla.bla_forward_chunked(q, k, v, w.M, w.S, w.T, workspace=ws, stream=stream, phase_mode=mode)
 
-            res["backward"] = roof(2 * F, 8 * elem * 2 + w.B * w.H * w.L * 4, timed(bwd), tok)
-            del o, lse, do, bws
+            res["forward" + sfx] = roof(F, 4 * elem * 2 + w.B * w.H * w.L * 4, timed(fwd), tok)
+            if getattr(w, "backward", False):
+                o, lse, _ = fwd()
+                do = torch.from_numpy(make_dout(w.B, w.H, w.L, w.d, "bf16", seed=0)).to(torch.bfloat16).to(dev)
+                bws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_BACKWARD), dtype=torch.uint8, device=dev)
+
+                def bwd():
+                    return bla.bla_backward(q, k, v, o, do, lse, w.M, w.S, w.T, workspace=bws, stream=stream,
+                                            phase_mode=mode)
+
+                res["backward" + sfx] = roof(2 * F, 8 * elem * 2 + w.B * w.H * w.L * 4, timed(bwd), tok)
+                del o, lse, do, bws
+            del ws
         res["shape"] = "B=%d H=%d L=%d d=%d M=%d S=%d T=%d" % (w.B, w.H, w.L, w.d, w.M, w.S, w.T)
         out[name] = res
-        del q, k, v, ws
+        del q, k, v
     del flush
     torch.cuda.empty_cache()
     return out

@@ -69,7 +69,21 @@ typedef struct {
                            beyond rounding. */
     double scale;       /* softmax scale; <= 0: 1/sqrt(d_k) (Eq. output, per head) */
     int dtype;          /* bla_dtype of q, k, v, o, dout, dq, dk, dv */
+    int phase_mode;     /* bla_phase_mode: how the slots index time (0 = the lag form) */
 } bla_params;
+
+/* How a slot reads the past (bla_params.phase_mode).
+ *   BLA_PHASE_LAG       the recurrent definition (Eq. recurrence, Eq. compressed, Alg. 2):
+ *                       slot j of token t weights key u by D_M(t - u - Delta_j), a window
+ *                       at lag Delta_j behind t.
+ *   BLA_PHASE_ABSOLUTE  the time-rolling form the paper runs in practice (Sec. 3.2, Alg. 1,
+ *                       Alg. 3): slot j weights key u by D_M(u - Delta_j), a kernel anchored
+ *                       at absolute phase Delta_j (mod T).  The two agree only when
+ *                       T = S = 2M-1.
+ * D_M is the translated Dirichlet kernel of Eq. (translated); the slot mask (keep slot j
+ * of token t iff t >= Delta_j) and the state (the lag-frame mode state of Eq. recurrence,
+ * so a prefill hands over to decode identically) are the same in both modes. */
+typedef enum { BLA_PHASE_LAG = 0, BLA_PHASE_ABSOLUTE = 1 } bla_phase_mode;
 
 /* Which entry point a workspace size is asked for. */
 typedef enum { BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2 } bla_ws_kind;

@@ -17,6 +17,8 @@ LIB_PATH = os.path.join(_HERE, "libbla_gb300.so")
 BLA_OK, BLA_ERR_INVALID, BLA_ERR_UNSUPPORTED, BLA_ERR_CUDA, BLA_ERR_TIMEOUT = range(5)
 BLA_F32, BLA_BF16 = 0, 1
 BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE = 0, 1, 2
+BLA_PHASE_LAG, BLA_PHASE_ABSOLUTE = 0, 1
+PHASE_MODES = {"lag": BLA_PHASE_LAG, "absolute": BLA_PHASE_ABSOLUTE}
 
 EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
             "bla_device_error", "bla_status_string", "bla_last_error_string", "bla_kernel_launches",
@@ -37,7 +39,7 @@ class Params(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("H", ctypes.c_int), ("L", ctypes.c_int),
                 ("d_k", ctypes.c_int), ("d_v", ctypes.c_int), ("M", ctypes.c_int), ("S", ctypes.c_int),
                 ("window", ctypes.c_double), ("omega", ctypes.c_double), ("chunk", ctypes.c_int),
-                ("scale", ctypes.c_double), ("dtype", ctypes.c_int)]
+                ("scale", ctypes.c_double), ("dtype", ctypes.c_int), ("phase_mode", ctypes.c_int)]
 
 
 _lib = None
@@ -103,9 +105,19 @@ def _dtype_code(dt):
     raise BlaError(BLA_ERR_INVALID, "dtype must be float32 or bfloat16, got %s" % dt)
 
 
-def make_params(B, H, L, d_k, d_v, M, S, window, omega=0.0, chunk=0, scale=0.0, dtype=torch.bfloat16):
+def _phase_code(phase_mode):
+    if isinstance(phase_mode, str):
+        if phase_mode not in PHASE_MODES:
+            raise BlaError(BLA_ERR_INVALID, "phase_mode must be one of %s, got %r" % (sorted(PHASE_MODES), phase_mode))
+        return PHASE_MODES[phase_mode]
+    return int(phase_mode)
+
+
+def make_params(B, H, L, d_k, d_v, M, S, window, omega=0.0, chunk=0, scale=0.0, dtype=torch.bfloat16,
+                phase_mode="lag"):
+    """bla_params; phase_mode is "lag" (Alg. 2, the default) or "absolute" (Alg. 1), or its code."""
     return Params(int(B), int(H), int(L), int(d_k), int(d_v), int(M), int(S), float(window), float(omega),
-                  int(chunk), float(scale), _dtype_code(dtype))
+                  int(chunk), float(scale), _dtype_code(dtype), _phase_code(phase_mode))
 
 
 def bla_workspace_bytes(params, which):
@@ -128,7 +140,7 @@ def _need_cuda(*ts):
 
 
 def bla_forward_chunked(q, k, v, M, S, window, omega=0.0, chunk=0, scale=0.0, want_lse=True,
-                        want_state=False, workspace=None, out=None, stream=None):
+                        want_state=False, workspace=None, out=None, stream=None, phase_mode="lag"):
     """Chunked forward over q, k: [B,H,L,d_k], v: [B,H,L,d_v] (float32 or bfloat16 CUDA tensors).
 
     Returns (o, lse or None, state or None); state is [B,H,2,M,2,d] fp32 (needs d_k == d_v).
@@ -136,7 +148,7 @@ def bla_forward_chunked(q, k, v, M, S, window, omega=0.0, chunk=0, scale=0.0, wa
     _need_cuda(q, k, v)
     B, H, L, dk = q.shape
     dv = v.shape[-1]
-    p = make_params(B, H, L, dk, dv, M, S, window, omega, chunk, scale, q.dtype)
+    p = make_params(B, H, L, dk, dv, M, S, window, omega, chunk, scale, q.dtype, phase_mode)
     o = out if out is not None else torch.empty((B, H, L, dv), dtype=q.dtype, device=q.device)
     lse = torch.empty((B, H, L), dtype=torch.float32, device=q.device) if want_lse else None
     st = torch.empty((B, H, 2, M, 2, dk), dtype=torch.float32, device=q.device) if want_state else None
@@ -147,12 +159,12 @@ def bla_forward_chunked(q, k, v, M, S, window, omega=0.0, chunk=0, scale=0.0, wa
 
 
 def bla_decode_step(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, workspace=None, out=None,
-                    stream=None):
+                    stream=None, phase_mode="lag"):
     """One decode step; q, k, v: [B,H,d]; state [B,H,2,M,2,d] fp32 is updated in place. Returns o."""
     _need_cuda(q, k, v, state)
     B, H, dk = q.shape
     dv = v.shape[-1]
-    p = make_params(B, H, 1, dk, dv, M, S, window, omega, 0, scale, q.dtype)
+    p = make_params(B, H, 1, dk, dv, M, S, window, omega, 0, scale, q.dtype, phase_mode)
     o = out if out is not None else torch.empty((B, H, dv), dtype=q.dtype, device=q.device)
     ws, n = _workspace(p, BLA_WS_DECODE, q.device, workspace)
     _check(load().bla_decode_step(ctypes.byref(p), int(pos), _ptr(q), _ptr(k), _ptr(v), _ptr(state), _ptr(o),
@@ -160,25 +172,27 @@ def bla_decode_step(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, wor
     return o
 
 
-def bla_decode_step_noalloc(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, out=None, stream=None):
+def bla_decode_step_noalloc(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, out=None, stream=None,
+                            phase_mode="lag"):
     """bla_decode_step without a workspace: the library's own fixed device scratch holds the
     tables, so the call allocates nothing (the output is allocated here unless `out` is given)."""
     _need_cuda(q, k, v, state)
     B, H, dk = q.shape
     dv = v.shape[-1]
-    p = make_params(B, H, 1, dk, dv, M, S, window, omega, 0, scale, q.dtype)
+    p = make_params(B, H, 1, dk, dv, M, S, window, omega, 0, scale, q.dtype, phase_mode)
     o = out if out is not None else torch.empty((B, H, dv), dtype=q.dtype, device=q.device)
     _check(load().bla_decode_step_noalloc(ctypes.byref(p), int(pos), _ptr(q), _ptr(k), _ptr(v), _ptr(state),
                                           _ptr(o), _stream(stream)))
     return o
 
 
-def bla_backward(q, k, v, o, dout, lse, M, S, window, omega=0.0, scale=0.0, workspace=None, stream=None):
+def bla_backward(q, k, v, o, dout, lse, M, S, window, omega=0.0, scale=0.0, workspace=None, stream=None,
+                 phase_mode="lag"):
     """Gradients (dq, dk, dv) of the chunked forward for upstream gradient dout."""
     _need_cuda(q, k, v, o, dout, lse)
     B, H, L, dk = q.shape
     dv = v.shape[-1]
-    p = make_params(B, H, L, dk, dv, M, S, window, omega, 0, scale, q.dtype)
+    p = make_params(B, H, L, dk, dv, M, S, window, omega, 0, scale, q.dtype, phase_mode)
     dq, dkk, dvv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
     ws, n = _workspace(p, BLA_WS_BACKWARD, q.device, workspace)
     _check(load().bla_backward(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout), _ptr(lse),
@@ -211,7 +225,7 @@ def bla_profile_collect():
 
 
 def forward_from_host(q_host, k_host, v_host, M, S, window, omega=0.0, scale=0.0, device=None, bufs=None,
-                      out_host=None, stream=None):
+                      out_host=None, stream=None, phase_mode="lag"):
     """bla_forward_chunked on host tensors: copies q, k, v (pinned for asynchronous copies) to the
     device, runs the chunked forward and copies o back into `out_host` (allocated if None).
     `bufs` (dict) caches the device buffers and workspace between calls.  Returns out_host; the
@@ -228,7 +242,7 @@ def forward_from_host(q_host, k_host, v_host, M, S, window, omega=0.0, scale=0.0
     if "o" not in bufs or bufs["o"].shape != (B, H, L, dv):
         bufs["o"] = torch.empty((B, H, L, dv), dtype=q_host.dtype, device=dev)
         bufs["lse"] = torch.empty((B, H, L), dtype=torch.float32, device=dev)
-    p = make_params(B, H, L, q_host.shape[-1], dv, M, S, window, omega, 0, scale, q_host.dtype)
+    p = make_params(B, H, L, q_host.shape[-1], dv, M, S, window, omega, 0, scale, q_host.dtype, phase_mode)
     if "ws" not in bufs:
         n = bla_workspace_bytes(p, BLA_WS_FORWARD)
         bufs["ws"] = torch.empty(max(n, 1), dtype=torch.uint8, device=dev)

@@ -111,6 +111,8 @@ bla_status check_params(const bla_params *p, OpDims *d) {
     const double Te = fmax(p->window, 2.0 * p->M - 1.0);
     if (p->S < 1 || (double)p->S > Te) return fail(BLA_ERR_INVALID, "S must be in [1, T] (S=%d, T=%g)", p->S, Te);
     if (p->chunk < 0) return fail(BLA_ERR_INVALID, "chunk must be >= 0");
+    if (p->phase_mode != BLA_PHASE_LAG && p->phase_mode != BLA_PHASE_ABSOLUTE)
+        return fail(BLA_ERR_INVALID, "phase_mode must be BLA_PHASE_LAG or BLA_PHASE_ABSOLUTE (got %d)", p->phase_mode);
     if ((long long)p->B * p->H > (1ll << 31) - 1) return fail(BLA_ERR_INVALID, "B*H too large");
     d->B = p->B; d->H = p->H; d->L = p->L; d->dk = p->d_k; d->dv = p->d_v; d->M = p->M; d->S = p->S;
     d->R2 = 2 * p->M;
@@ -118,6 +120,7 @@ bla_status check_params(const bla_params *p, OpDims *d) {
     d->w = p->omega > 0.0 ? p->omega : 2.0 * kPi / Te;
     d->scale = (float)(p->scale > 0.0 ? p->scale : 1.0 / sqrt((double)p->d_k));
     d->dtype = p->dtype;
+    d->absolute = p->phase_mode == BLA_PHASE_ABSOLUTE;
     return BLA_OK;
 }
 

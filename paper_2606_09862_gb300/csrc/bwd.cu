@@ -15,6 +15,11 @@
 // 64-wide K blocks through a shared-memory ring, accumulates in TMEM and applies a fused
 // epilogue (causal mask, per-mode phase rotation, probability recompute from lse, dS, addend).
 // The forward chunk states and the adjoint states come from element-wise scans on CUDA cores.
+//
+// Absolute form (Alg. 1): the forward's two per-row rotations by m w tau become one rotation by
+// -m w t0 (t0 = the chunk's first token) and PHI has its sine half negated (see fwd_f32.cu).  The
+// adjoint rotations are the transposes at the same angle, so every EP_ROT epilogue takes its
+// phase from a per-chunk table instead of the per-row one; the rest of the backward is shared.
 #include <math.h>
 #include <string.h>
 
@@ -62,6 +67,7 @@ struct Epi {
     const float *dl;         // EP_DS: [Z][128]
     const float *addend;     // EP_ADD: [Z][128][ldo] fp32
     const float *erel;       // EP_ROT: (cos, sin)(m w tau), [C+1][M][2]
+    const float *cphase;     // EP_ROT, absolute form: (cos, sin)(-m w c C), [nchunks][M][2] (else null)
     int M;
 };
 
@@ -235,10 +241,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else if (e.op == EP_ROT) {
                         // e^{i m w row} for the 16 modes of this block: the table's first phase, then
                         // products with e^{i w row} (16 steps; rounding far below bf16 resolution)
+                        // (absolute form: e^{-i m w t0} of the chunk, stepped by e^{-i w t0})
                         const int m0 = g0 >> 1;
-                        float cs = e.erel[((size_t)row * e.M + m0) * 2];
-                        float sn = e.erel[((size_t)row * e.M + m0) * 2 + 1];
-                        const float c1 = e.erel[((size_t)row * e.M + 1) * 2], s1 = e.erel[((size_t)row * e.M + 1) * 2 + 1];
+                        const float *ptab = e.cphase ? e.cphase + (size_t)c * e.M * 2 : e.erel + (size_t)row * e.M * 2;
+                        float cs = ptab[m0 * 2], sn = ptab[m0 * 2 + 1];
+                        const float c1 = ptab[2], s1 = ptab[3];
 #pragma unroll
                         for (int i = 0; i < 32; i += 2) {
                             const float sg = e.rot_sign * sn;
@@ -360,6 +367,17 @@ __global__ void k_state_scan(int BH, int nch, int M, int D, const float *erel, c
         }
     }
 }
+// Absolute form: (cos, sin)(-m w c C) for every chunk c and mode m, in fp64 rounded to fp32.
+__global__ void k_chunk_phase(int M, int nch, double w, float *out) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nch * M; i += gridDim.x * blockDim.x) {
+        const int c = i / M, m = i % M;
+        double sn, cs;
+        sincos((double)m * w * ((double)c * kC), &sn, &cs);
+        out[2 * i] = (float)cs;
+        out[2 * i + 1] = (float)-sn;
+    }
+}
+
 // rowsum(dO o) per token: one warp per row, each lane reading D/32 consecutive elements.
 __global__ void k_rowdot(int BH, int L, int nch, int D, const bf16 *dout, const bf16 *o, float *dl) {
     const long long rows = (long long)BH * nch * kC;
@@ -402,7 +420,7 @@ BwdGeo bwd_geo(const OpDims &d) {
 }
 
 struct BwdWs {
-    size_t tables, eb, phi, cb, wb, lb, P, Y, p, A, G, dG, dU, ds, dX, dP, dKi, dVi, dl, total;
+    size_t tables, eb, phi, cphase, cb, wb, lb, P, Y, p, A, G, dG, dU, ds, dX, dP, dKi, dVi, dl, total;
 };
 
 BwdWs bwd_ws(const OpDims &d, const BwdGeo &g) {
@@ -413,6 +431,7 @@ BwdWs bwd_ws(const OpDims &d, const BwdGeo &g) {
     w.tables = take(tables_bytes(d, kC));
     w.eb = take(2 * (size_t)g.RP * kC);
     w.phi = take(2 * (size_t)g.SP * g.R2);
+    w.cphase = take(d.absolute ? 4 * (size_t)g.nch * g.M * 2 : 0);
     w.cb = take(4 * Z * 2 * g.R2 * g.D);
     w.wb = take(2 * Z * 2 * g.R2 * g.D);
     w.lb = take(2 * Z * 2 * g.R2 * g.D);
@@ -531,6 +550,14 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     if (e != cudaSuccess) return e;
     bf16 *eb = reinterpret_cast<bf16 *>(ws + w.eb), *phi = reinterpret_cast<bf16 *>(ws + w.phi);
     if ((e = build_bf16_tables(d, g.RP, g.SP, eb, phi, st)) != cudaSuccess) return e;
+    float *cphase = nullptr;
+    if (d.absolute) {
+        cphase = reinterpret_cast<float *>(ws + w.cphase);
+        const int n = g.nch * g.M;
+        ProfScope ps(BLA_K_BWD, st);
+        k_chunk_phase<<<(n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024, 256, 0, st>>>(g.M, g.nch, d.w, cphase);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
     float *cb = reinterpret_cast<float *>(ws + w.cb), *dKi = reinterpret_cast<float *>(ws + w.dKi);
     float *dVi = reinterpret_cast<float *>(ws + w.dVi), *dl = reinterpret_cast<float *>(ws + w.dl);
     bf16 *wb = reinterpret_cast<bf16 *>(ws + w.wb), *lb = reinterpret_cast<bf16 *>(ws + w.lb);
@@ -588,19 +615,19 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     // ---- 1. recompute the chunk's forward quantities
     ep = epi_base(EP_CAUSAL, Pb, OUT_Z, 0, kC, kC);                                   // P = tril(Q K^T)
     if ((e = gemm(g, 1, kC, qK, SEQK, kK, SEQK, D, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_ROT, Yb, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.M = g.M;         // Y = rot+(P EB^T + Q W_K^T)
+    ep = epi_base(EP_ROT, Yb, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.cphase = cphase; ep.M = g.M;         // Y = rot+(P EB^T + Q W_K^T)
     if ((e = gemm(g, 1, R2, PK, ZK, ebKR, SHK, kC, &qK, &SEQK, &wbK, &WK_K, D, ep, st))) return e;
     ep = epi_base(EP_PROB, pb, OUT_Z, 0, SP, SP);                                      // p from lse
     ep.scale = d.scale; ep.lse = lse; ep.delta = t.delta; ep.S = S;
     if ((e = gemm(g, 1, S, YK, ZK, phiK, SHK, R2, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_ROT, Ab, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.M = g.M; ep.rot_sign = -1;   // A' = rot-(p PHI)
+    ep = epi_base(EP_ROT, Ab, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.cphase = cphase; ep.M = g.M; ep.rot_sign = -1;   // A' = rot-(p PHI)
     if ((e = gemm(g, 1, R2, pK, ZK, phiM, SHM, SP, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
     ep = epi_base(EP_CAUSAL, Gb, OUT_Z, 0, kC, kC);                                   // G = tril(A' EB)
     if ((e = gemm(g, 1, kC, AK, ZK, ebM, SHM, R2, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
     // ---- 2. local adjoints
     ep = epi_base(EP_CAUSAL, dGb, OUT_Z, 0, kC, kC);                                  // dG = tril(dO V^T)
     if ((e = gemm(g, 1, kC, dOK, SEQK, vK, SEQK, D, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_ROT, dUb, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.M = g.M;        // dU = rot+(dG EB^T + dO W_V^T)
+    ep = epi_base(EP_ROT, dUb, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.cphase = cphase; ep.M = g.M;        // dU = rot+(dG EB^T + dO W_V^T)
     if ((e = gemm(g, 1, R2, dGK, ZK, ebKR, SHK, kC, &dOK, &SEQK, &wbK, &WV_K, D, ep, st))) return e;
     {
         long long total = (long long)Z * kC;
@@ -612,7 +639,7 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     }
     ep = epi_base(EP_DS, dsb, OUT_Z, 0, SP, SP); ep.pbuf = pb; ep.ldp = SP; ep.dl = dl;  // ds = p (dU PHI^T - dl)
     if ((e = gemm(g, 1, S, dUK, ZK, phiK, SHK, R2, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_ROT, dXb, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.M = g.M;        // dX = rot-(scale ds PHI)
+    ep = epi_base(EP_ROT, dXb, OUT_Z, 0, R2, R2); ep.erel = t.erel; ep.cphase = cphase; ep.M = g.M;        // dX = rot-(scale ds PHI)
     ep.rot_sign = -1; ep.scale = d.scale;
     if ((e = gemm(g, 1, R2, dsK, ZK, phiM, SHM, SP, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
     ep = epi_base(EP_CAUSAL, dPb, OUT_Z, 0, kC, kC);                                  // dP = tril(dX EB)

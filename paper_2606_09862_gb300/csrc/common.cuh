@@ -23,11 +23,14 @@ struct OpDims {
     double w;                        // mode frequency omega
     float scale;
     int dtype;
+    int absolute;                    // 1: absolute-phase slots (Alg. 1), 0: lag form (Alg. 2)
 };
 
 // Table block (built on the device per call; lives in the caller's workspace).
-//   phi   [S][R2] fp32: phi[j][2m] = c_m cos(m w D_j), phi[j][2m+1] = c_m sin(m w D_j)
-//         with c_0 = 1/(2M-1), c_m = 2/(2M-1) (Eq. translated).
+//   phi   [S][R2] fp32: phi[j][2m] = c_m cos(m w D_j), phi[j][2m+1] = sigma c_m sin(m w D_j)
+//         with c_0 = 1/(2M-1), c_m = 2/(2M-1) (Eq. translated); sigma = +1 in the lag form,
+//         -1 in the absolute form (its slots read e^{+i m w D_j} where the lag form reads
+//         e^{-i m w D_j}).
 //   delta [S] int: dilated lags round(j T / S).
 //   rot1  [M][2] fp32: cos(m w), sin(m w) (Eq. recurrence, one step).
 //   erel  [C+1][M][2] fp32: cos(m w tau), sin(m w tau), tau = 0..C (chunk phases).

@@ -9,6 +9,9 @@
 //   V pass: Z_m <- e^{i m w} Z_m + v, o = sum_m u_m^c Re Z_m + u_m^s Im Z_m,
 //           u_m = sum_j p_j (A[j,m], B[j,m])  (= sum_j p_j V~[j] with the sums exchanged)
 // The sine row of mode 0 never changes (sin(0) = 0) and is neither read nor written.
+// Absolute form (Alg. 1): the slots read q . Zabs_m = e^{-i m w pos} y_m through c_m e^{+i m w D_j}
+// (the phi table with its sine half negated), and the output coefficient u_m is multiplied by
+// e^{-i m w pos}; the state and its update are the same as in the lag form.
 #include "common.cuh"
 
 namespace bla {
@@ -55,6 +58,13 @@ __device__ __forceinline__ float warp_max(float x) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
     return x;
+}
+
+// (cos, sin)(m w pos) in fp64, rounded to fp32.
+__device__ __forceinline__ float2 pos_phase(int m, long long pos, double w) {
+    double sn, cs;
+    sincos((double)m * w * (double)pos, &sn, &cs);
+    return make_float2((float)cs, (float)sn);
 }
 
 // Modes handled per warp per batch of independent loads.
@@ -125,6 +135,16 @@ __global__ void __launch_bounds__(kThreads) k_decode(OpDims d, long long pos, Ta
         }
     }
     __syncthreads();
+    // absolute form: y_m <- e^{-i m w pos} y_m
+    if (d.absolute) {
+        for (int m = threadIdx.x; m < M; m += kThreads) {
+            const float2 f = pos_phase(m, pos, d.w);
+            const float yc = y[2 * m], ys = y[2 * m + 1];
+            y[2 * m] = f.x * yc + f.y * ys;
+            y[2 * m + 1] = f.x * ys - f.y * yc;
+        }
+        __syncthreads();
+    }
 
     // ---- slot scores: warp per slot, lanes across the R2 state rows (coalesced table reads)
     for (int j = warp; j < S; j += kWarps) {
@@ -159,6 +179,16 @@ __global__ void __launch_bounds__(kThreads) k_decode(OpDims d, long long pos, Ta
         y[r] = acc;
     }
     __syncthreads();
+    // absolute form: the coefficient uc - i us is multiplied by e^{-i m w pos}
+    if (d.absolute) {
+        for (int m = threadIdx.x; m < M; m += kThreads) {
+            const float2 f = pos_phase(m, pos, d.w);
+            const float uc = y[2 * m], us = y[2 * m + 1];
+            y[2 * m] = f.x * uc - f.y * us;
+            y[2 * m + 1] = f.y * uc + f.x * us;
+        }
+        __syncthreads();
+    }
 
     // ---- V pass
     float oacc[VEC];

@@ -82,12 +82,16 @@ extern "C" bla_status bla_decode_step_noalloc(const bla_params *p, long long pos
     if (p->d_k != p->d_v || (p->d_k != 32 && p->d_k != 64 && p->d_k != 128))
         return reject(BLA_ERR_UNSUPPORTED, "decode needs d_k = d_v in {32, 64, 128} (got %lld, %lld)", p->d_k, p->d_v);
     if (p->S > 256) return reject(BLA_ERR_UNSUPPORTED, "decode needs S <= 256 (got %lld)", p->S);
+    if (p->phase_mode != BLA_PHASE_LAG && p->phase_mode != BLA_PHASE_ABSOLUTE)
+        return reject(BLA_ERR_INVALID, "phase_mode must be BLA_PHASE_LAG or BLA_PHASE_ABSOLUTE (got %lld)",
+                      (long long)p->phase_mode);
     OpDims d;
     d.B = p->B; d.H = p->H; d.L = 1; d.dk = p->d_k; d.dv = p->d_v; d.M = p->M; d.S = p->S; d.R2 = 2 * p->M;
     d.T = Te;
     d.w = p->omega > 0.0 ? p->omega : 2.0 * kPi / Te;
     d.scale = (float)(p->scale > 0.0 ? p->scale : 1.0 / sqrt((double)p->d_k));
     d.dtype = p->dtype;
+    d.absolute = p->phase_mode == BLA_PHASE_ABSOLUTE;
     const size_t need = tables_bytes(d, 0);
     if (need > kNoAllocScratchBytes)
         return reject(BLA_ERR_UNSUPPORTED,

@@ -1,23 +1,27 @@
 // fwd_bf16.cu -- bf16 chunked forward on the 5th-generation tensor cores (tcgen05 + TMEM + TMA).
 //
 // Chunk algebra (the same exact rearrangement as the fp32 path, Eqs. (recurrence),
-// (compressed), (output)): for a chunk of C = 128 tokens starting at t0, with W the state
-// carried into the chunk (W_m = e^{i m w} Z_m(t0-1), interleaved rows 2m = Re, 2m+1 = Im):
+// (compressed), (output)), with the states kept in the absolute frame
+// A_m = sum_{u < t0} e^{-i m w u} x_u (interleaved rows 2m = Re, 2m+1 = Im), for a chunk of
+// C = 128 tokens starting at t0:
 //   P  = tril(Q K^T)                                 [C x C]
-//   X  = P EB^T + Q W^T,  EB[2m][u] = cos(m w u), EB[2m+1][u] = -sin(m w u)
-//   Y  = e^{i m w t} X (per row t, per mode pair)    = q_t . Z_m(t0+t)
+//   X  = P EB_c^T + Q A^T,  EB_c[2m][u] = cos(m w (t0+u)), EB_c[2m+1][u] = -sin(m w (t0+u))
+//   Y  = e^{i m w t} X (per row, t = t0 + row)       = q_t . Z_m(t)   (lag-frame state)
 //   s  = scale Y PHI^T,   PHI[j][2m] = c_m cos(m w D_j), PHI[j][2m+1] = c_m sin(m w D_j)
-//   p  = softmax over slots with t0+t >= D_j
+//   p  = softmax over slots with t >= D_j
 //   U  = p PHI;  A'  = rotation of U by -m w t  (real form of U_m e^{i m w t}, imaginary negated)
-//   G  = tril(A' EB),  O = G V + A' WV
-//   W <- e^{i m w C} (W + EB X_chunk)  for X in {K, V}
+//   G  = tril(A' EB_c),  O = G V + A' A_V
+//   A <- A + EB_c X_chunk  for X in {K, V}   (no rotation between chunks)
+// The absolute-phase form (Alg. 1) differs only in its read-out: Y = X and A' = U (no per-row
+// rotation) with the sine half of PHI negated.  The state is the same in both forms.
 //
-// The work runs as four kernels per call:
+// The work runs as five kernels per call:
+//   k_tables_bf16  EB_c of every chunk, PHI, the segment phase table and the slot lags
 //   k_prepass  per (head, segment): segment deltas  F_seg [K|V]  (one GEMM, K-dim = segment)
 //   k_scan     per head: states entering each segment, W_in(g+1) = e^{i m w Lseg} W_in(g) + delta(g)
 //   k_kpass    per (head, segment): carries the K state in TMEM, writes slot probabilities p and lse
 //   k_vpass    per (head, segment): carries the V state in TMEM, reads p, writes o
-// Every CTA runs 6 warps: warps 0-3 drain TMEM (thread = TMEM lane), warp 4 issues TMA loads,
+// The prepass runs 6 warps: warps 0-3 drain TMEM (thread = TMEM lane), warp 4 issues TMA loads,
 // warp 5 allocates TMEM and issues the MMAs.  All waits are bounded (tc::mbar_wait).
 #include <math.h>
 
@@ -135,15 +139,15 @@ __device__ __forceinline__ void mode_phase(long long mu, double w, int tint, flo
 // Operand tables of the tensor-core path, in bf16 (rows beyond 2M and slots beyond S are zero):
 //   EB    [nch][RP][C]: EB_c[2m][u] = cos(m w (cC + u)), EB_c[2m+1][u] = -sin(m w (cC + u));
 //         with nch = 1 this is the in-chunk table (c = 0) of the lag frame
-//   PHI   [SP][R2]: PHI[j][2m] = c_m cos(m w D_j), PHI[j][2m+1] = c_m sin(m w D_j), D_j = round(j T / S),
-//         c_0 = 1/(2M-1), c_m = 2/(2M-1)
+//   PHI   [SP][R2]: PHI[j][2m] = c_m cos(m w D_j), PHI[j][2m+1] = sigma c_m sin(m w D_j), D_j = round(j T / S),
+//         c_0 = 1/(2M-1), c_m = 2/(2M-1); sigma = +1 (lag form) or -1 (absolute form, Alg. 1)
 //   FSEG  [RP][Lseg] (optional): FSEG[2m][u] = cos(m w (Lseg - u)), FSEG[2m+1][u] = sin(m w (Lseg - u)),
 //         eight entries per thread as for EB
 //   delta [S] (optional): the slot lags D_j
 // EB is written by one thread per (c, m, 8 consecutive u), u fastest so that a warp writes whole
 // rows: the first phase is reduced exactly, the next seven follow by products with e^{i m w}.
 __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, double T, double w, int tint,
-                              bf16 *eb, bf16 *phi, bf16 *fseg, int *delta) {
+                              float sin_sign, bf16 *eb, bf16 *phi, bf16 *fseg, int *delta) {
     const int R2 = 2 * M, MP = RP / 2;
     const long long n_eb = (long long)nch * MP * (kC / 8), n_phi = (long long)SP * R2;
     const long long n_f = fseg ? (long long)MP * ((Lseg + 7) / 8) : 0, n_d = delta ? S : 0;
@@ -185,7 +189,7 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, d
                 const float cm = (m == 0) ? (float)(1.0 / n) : (float)(2.0 / n);
                 float c, sn;
                 mode_phase((long long)m * dj, w, tint, &c, &sn);
-                v = cm * ((r & 1) ? sn : c);
+                v = cm * ((r & 1) ? sin_sign * sn : c);
             }
             phi[e] = __float2bfloat16_rn(v);
         } else if (i < n_eb + n_phi + n_f) {
@@ -228,6 +232,7 @@ struct Args {
     float *state_out;    // [BH][2][M][2][D] or null
     float *deltas_out;   // prepass output (same buffer as deltas)
     int tint;            // integer period for exact phase reduction (0: use fp64 phases)
+    int absolute;        // absolute form (Alg. 1): the drains do not rotate rows by e^{i m w t}
     int *err;
 };
 
@@ -840,8 +845,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             // first mode of this thread's range in each half (two interleaved chains per range), and
             // the drain phases of this row: exact at the CTA's first chunk, then advanced per chunk
             const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
-            RowPhases rp = row_phases((long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
-            const RowPhases rp_step = row_phases(kC, m00, m10, NH == 2, a.w, a.tint);
+            // (the absolute form reads the absolute-frame products as they are: every phase is 1)
+            RowPhases rp = row_phases(a.absolute ? 0 : (long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
+            const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, a.w, a.tint);
             // the state is kept in the absolute frame, A = sum_{u < t0} e^{-i m w u} k_u: it needs no
             // rotation between chunks; the carried-in lag-frame state is rotated once
             for (int b = 0; b < g.NB; ++b) {
@@ -1301,8 +1307,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
             // first mode of this thread's range in each half, and the drain phases of this row
             const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
-            RowPhases rp = row_phases((long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
-            const RowPhases rp_step = row_phases(kC, m00, m10, NH == 2, a.w, a.tint);
+            RowPhases rp = row_phases(a.absolute ? 0 : (long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
+            const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, a.w, a.tint);
             // V state in the absolute frame (see the K pass)
             for (int b = 0; b < g.NB; ++b) {
                 const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
@@ -1449,7 +1455,8 @@ cudaError_t build_bf16_tables(const OpDims &d, int RP, int SP, bf16 *eb, bf16 *p
     int blocks = (int)((total + 255) / 256);
     if (blocks > 2048) blocks = 2048;
     ProfScope ps(BLA_K_TABLES_BF16, st);
-    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, 1, d.T, d.w, integer_period(d), eb, phi, nullptr, nullptr);
+    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, 1, d.T, d.w, integer_period(d), d.absolute ? -1.f : 1.f,
+                                          eb, phi, nullptr, nullptr);
     return cudaGetLastError();
 }
 
@@ -1582,8 +1589,8 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
                                 (fseg ? (long long)(g.RP / 2) * ((g.Lseg + 7) / 8) : 0) + g.S;
         const int blocks = (int)(total < 4096 * 256 ? (total + 255) / 256 : 4096);
         ProfScope ps(BLA_K_TABLES_BF16, st);
-        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, g.nchunks, d.T, d.w, integer_period(d), eb,
-                                              phi, fseg, delta);
+        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, g.nchunks, d.T, d.w, integer_period(d),
+                                              d.absolute ? -1.f : 1.f, eb, phi, fseg, delta);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     Args a;
@@ -1599,6 +1606,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     a.o = static_cast<bf16 *>(o);
     a.state_out = state_out;
     a.tint = integer_period(d);
+    a.absolute = d.absolute;
     a.err = device_error_word();
 
     // tensor maps

@@ -16,6 +16,12 @@
 // This is Alg. 2's per-token read-out with the sums over slots, modes and past
 // tokens exchanged; every term is an exact rearrangement of Eqs. (recurrence),
 // (compressed) and (output).
+//
+// Absolute form (Alg. 1): slot j weights key u by D_M(u - D_j) instead of D_M(t - u - D_j).
+// Its scores read q_t . Zabs_m(t) = e^{-i m w (t0+t)} Y_m(t) = e^{-i m w t0} X_m(t) through
+// the coefficients c_m e^{+i m w D_j} (the phi table with its sine half negated), and its
+// output coefficient is U'_m(t) e^{-i m w t0}.  So both per-row rotations e^{i m w t} become
+// the chunk-constant e^{-i m w t0}; everything else is unchanged.
 #include "common.cuh"
 
 namespace bla {
@@ -23,7 +29,7 @@ namespace bla {
 namespace {
 
 struct F32Smem {
-    float *Q, *K, *V, *P, *X, *Sc;
+    float *Q, *K, *V, *P, *X, *Sc, *Ph;
 };
 
 __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb, const float *__restrict__ q,
@@ -41,6 +47,7 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
     sm.P = sm.V + C * dv;
     sm.X = sm.P + C * C;
     sm.Sc = sm.X + C * R2;
+    sm.Ph = sm.Sc + C * S;   // [M][2] absolute form: (cos, sin)(-m w t0) of the current chunk
 
     const float *qh = q + (size_t)bh * L * dk, *kh = k + (size_t)bh * L * dk, *vh = v + (size_t)bh * L * dv;
     float *oh = o + (size_t)bh * L * dv;
@@ -60,6 +67,14 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
             sm.K[i] = kh[(size_t)t0 * dk + i];
         }
         for (int i = tid; i < n * dv; i += nt) sm.V[i] = vh[(size_t)t0 * dv + i];
+        if (d.absolute) {
+            for (int m = tid; m < M; m += nt) {
+                double sn, cs;
+                sincos((double)m * d.w * (double)t0, &sn, &cs);
+                sm.Ph[2 * m] = (float)cs;
+                sm.Ph[2 * m + 1] = (float)-sn;
+            }
+        }
         __syncthreads();
         // P = tril(Q K^T)
         for (int i = tid; i < n * n; i += nt) {
@@ -84,7 +99,8 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
                 xc = fmaf(sm.Q[t * dk + e], wc[e], xc);
                 xs = fmaf(sm.Q[t * dk + e], ws[e], xs);
             }
-            float c = erel[(t * M + m) * 2], s = erel[(t * M + m) * 2 + 1];
+            const float *ph = d.absolute ? sm.Ph + 2 * m : erel + (t * M + m) * 2;
+            float c = ph[0], s = ph[1];
             sm.X[t * R2 + 2 * m] = c * xc - s * xs;
             sm.X[t * R2 + 2 * m + 1] = s * xc + c * xs;
         }
@@ -121,7 +137,8 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
                 uc = fmaf(pj, phi[j * R2 + 2 * m], uc);
                 us = fmaf(pj, phi[j * R2 + 2 * m + 1], us);
             }
-            float c = erel[(t * M + m) * 2], s = erel[(t * M + m) * 2 + 1];
+            const float *ph = d.absolute ? sm.Ph + 2 * m : erel + (t * M + m) * 2;
+            float c = ph[0], s = ph[1];
             sm.X[t * R2 + 2 * m] = c * uc + s * us;
             sm.X[t * R2 + 2 * m + 1] = c * us - s * uc;
         }
@@ -172,7 +189,8 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
 }  // namespace
 
 int forward_f32_smem_bytes(const OpDims &d, int C) {
-    size_t f = (size_t)C * d.dk * 2 + (size_t)C * d.dv + (size_t)C * C + (size_t)C * d.R2 + (size_t)C * d.S;
+    size_t f = (size_t)C * d.dk * 2 + (size_t)C * d.dv + (size_t)C * C + (size_t)C * d.R2 + (size_t)C * d.S +
+               (size_t)d.R2;
     return (int)(f * sizeof(float));
 }
 

@@ -4,7 +4,8 @@
 //   dilated lags   D_j = round(j T / S)       (Alg. 1-3 "dilated_time", generalised to S slots;
 //                                              round half to even)
 //   coefficients   A[j,m] = c_m cos(m w D_j), B[j,m] = c_m sin(m w D_j), c_0 = 1/(2M-1),
-//                  c_{m>0} = 2/(2M-1)          (Eq. translated)
+//                  c_{m>0} = 2/(2M-1)          (Eq. translated); B is negated for the
+//                  absolute form (Alg. 1), whose slots read e^{+i m w D_j}
 //   one-step rotation cos(m w), sin(m w)       (Eq. recurrence)
 //   chunk phases   cos(m w tau), sin(m w tau), tau = 0..C
 #include "common.cuh"
@@ -30,8 +31,8 @@ char *tables_carve(const OpDims &d, int C, char *base, Tables *t) {
     return p;
 }
 
-__global__ void k_tables(int M, int S, double T, double w, int C, float *phi, int *delta, float *rot1,
-                         float *erel) {
+__global__ void k_tables(int M, int S, double T, double w, int C, float sin_sign, float *phi, int *delta,
+                         float *rot1, float *erel) {
     const int R2 = 2 * M;
     const double n = 2.0 * M - 1.0;
     const long long n_phi = (long long)S * R2;
@@ -45,7 +46,7 @@ __global__ void k_tables(int M, int S, double T, double w, int C, float *phi, in
             double dj = rint((double)j * T / (double)S);
             double c = (m == 0) ? 1.0 / n : 2.0 / n;
             double ang = (double)m * w * dj;
-            phi[i] = (float)(c * ((r & 1) ? sin(ang) : cos(ang)));
+            phi[i] = (float)(c * ((r & 1) ? sin_sign * sin(ang) : cos(ang)));
         } else if (i < n_phi + S) {
             int j = (int)(i - n_phi);
             delta[j] = (int)rint((double)j * T / (double)S);
@@ -72,7 +73,8 @@ cudaError_t tables_build(const OpDims &d, const Tables &t, cudaStream_t st) {
     int blocks = (int)((total + threads - 1) / threads);
     if (blocks > 1024) blocks = 1024;
     ProfScope ps(BLA_K_TABLES, st);
-    k_tables<<<blocks, threads, 0, st>>>(d.M, d.S, d.T, d.w, t.C, t.phi, t.delta, t.rot1, t.erel);
+    k_tables<<<blocks, threads, 0, st>>>(d.M, d.S, d.T, d.w, t.C, d.absolute ? -1.f : 1.f, t.phi, t.delta, t.rot1,
+                                         t.erel);
     return cudaGetLastError();
 }
 

@@ -51,7 +51,8 @@ FAKE = ctypes.c_void_p(0x10000)      # aligned, never dereferenced: validation f
 
 @pytest.mark.parametrize("kw", [dict(B=0), dict(H=0), dict(L=-1), dict(d_k=0), dict(M=0), dict(S=0),
                                 dict(S=17), dict(window=0.0), dict(window=float("nan")), dict(dtype=7),
-                                dict(chunk=-3), dict(omega=float("inf"))])
+                                dict(chunk=-3), dict(omega=float("inf")), dict(phase_mode=2),
+                                dict(phase_mode=-1)])
 def test_invalid_params_rejected_on_host(lib, kw):
     from paper_2606_09862_gb300 import bla
     p = _params(**kw)
@@ -93,6 +94,24 @@ def test_workspace_sizes_positive(lib):
     p = _params()
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_FORWARD) > 0
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECODE) > 0
+
+
+def test_phase_mode_accepted(lib):
+    """Both phase modes are valid parameters; the absolute form's backward needs its per-chunk
+    phase table on top of the lag form's workspace."""
+    from paper_2606_09862_gb300 import bla
+    for mode in (bla.BLA_PHASE_LAG, bla.BLA_PHASE_ABSOLUTE):
+        p = _params(phase_mode=mode)
+        assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_FORWARD) > 0
+        assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECODE) > 0
+    kw = dict(L=300, d_k=64, d_v=64, M=32, S=32, window=256.0, dtype=bla.BLA_BF16)
+    lag = lib.bla_workspace_bytes(ctypes.byref(_params(**kw)), bla.BLA_WS_BACKWARD)
+    ab = lib.bla_workspace_bytes(ctypes.byref(_params(phase_mode=bla.BLA_PHASE_ABSOLUTE, **kw)),
+                                 bla.BLA_WS_BACKWARD)
+    assert lag > 0 and ab > lag
+    assert bla.make_params(1, 1, 8, 32, 32, 4, 4, 16.0, phase_mode="absolute").phase_mode == 1
+    with pytest.raises(bla.BlaError):
+        bla.make_params(1, 1, 8, 32, 32, 4, 4, 16.0, phase_mode="relative")
 
 
 def test_product_path_does_not_import_oracle():
