@@ -10,11 +10,14 @@
 // where the adjoint states L of the chunk sums (W + EB X) run backwards over the chunks:
 //   L_{c-1} = rot_C^T (X_c^T + L_c) with X_c^T = dX^T Q (K) or A'^T dO (V), L_last = 0.
 //
-// Every contraction runs on the tensor cores through one batched kernel, k_bgemm: one CTA per
-// (chunk, 128-row tile) computes sum_t A_t B_t (up to two terms) with A, B streamed by TMA in
-// 64-wide K blocks through a shared-memory ring, accumulates in TMEM and applies a fused
-// epilogue (causal mask, per-mode phase rotation, probability recompute from lse, dS, addend).
-// The forward chunk states and the adjoint states come from element-wise scans on CUDA cores.
+// The chunk-local contractions run on the tensor cores through one batched kernel, k_bgemm: a
+// persistent CTA walks (chunk, 128-row tile) tiles and computes sum_t A_t B_t (up to two terms)
+// with A, B streamed by TMA in 64-wide K blocks through a shared-memory ring, accumulates in TMEM
+// and applies a fused epilogue (causal mask, per-mode phase rotation, probability recompute from
+// lse, dS).  The states run through two chunk-sequential kernels, one CTA per (head, K or V):
+// k_fwd_states rebuilds the forward's chunk states, k_adj_states carries the adjoint states
+// backwards and writes dK and dV on the way; both keep the state in registers and take each
+// chunk's contribution from the tensor cores.
 //
 // Absolute form (Alg. 1): the forward's two per-row rotations by m w tau become one rotation by
 // -m w t0 (t0 = the chunk's first token) and PHI has its sine half negated (see fwd_f32.cu).  The
@@ -37,7 +40,7 @@ constexpr int kC = 128;
 constexpr int kThreads = 192;
 
 enum OpMode { OP_SHARED = 0, OP_Z = 1, OP_SEQ = 2 };
-enum EpiOp { EP_PLAIN = 0, EP_CAUSAL, EP_ROT, EP_PROB, EP_DS, EP_ADD };
+enum EpiOp { EP_PLAIN = 0, EP_CAUSAL, EP_ROT, EP_PROB, EP_DS };
 enum OutMode { OUT_Z = 0, OUT_SEQ = 1 };
 
 struct Operand {
@@ -65,7 +68,6 @@ struct Epi {
     const bf16 *pbuf;        // EP_DS: [Z][128][ldp]
     int ldp;
     const float *dl;         // EP_DS: [Z][128]
-    const float *addend;     // EP_ADD: [Z][128][ldo] fp32
     const float *erel;       // EP_ROT: (cos, sin)(m w tau), [C+1][M][2]
     const float *cphase;     // EP_ROT, absolute form: (cos, sin)(-m w c C), [nchunks][M][2] (else null)
     int M;
@@ -275,16 +277,6 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 v[i + 2 * q + 1] = pf.y * (v[i + 2 * q + 1] - dl);
                             }
                         }
-                    } else if (e.op == EP_ADD) {
-                        const float *ad = e.addend + ((size_t)z * kC + row) * e.ldo + g0;
-#pragma unroll
-                        for (int i = 0; i < 32; i += 4) {
-                            const float4 a4 = __ldg(reinterpret_cast<const float4 *>(ad + i));
-                            v[i] += a4.x;
-                            v[i + 1] += a4.y;
-                            v[i + 2] += a4.z;
-                            v[i + 3] += a4.w;
-                        }
                     }
                 }
                 if (!live) continue;
@@ -318,55 +310,6 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // ------------------------------------------------------------------ scans (CUDA cores)
 
-// Forward chunk states: W_0 = 0, W_{c+1} = rot_C (W_c + contrib_c); writes bf16 W_c for every chunk.
-// contrib, wout: [Z][2][R2][D] with Z = BH * nchunks.  One thread per (bh, x, m, e).
-__global__ void k_state_scan(int BH, int nch, int M, int D, const float *erel, const float *contrib, bf16 *wout,
-                             int reverse) {
-    const long long total = (long long)BH * 2 * M * D;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int e = (int)(i % D);
-        long long r = i / D;
-        const int m = (int)(r % M);
-        r /= M;
-        const int x = (int)(r % 2);
-        const int bh = (int)(r / 2);
-        const int R2 = 2 * M;
-        const float cs = erel[((size_t)kC * M + m) * 2], sn = erel[((size_t)kC * M + m) * 2 + 1];
-        float re = 0.f, im = 0.f;
-        // the contributions of eight chunks are loaded before they are used, so that their
-        // latencies overlap
-        for (int s0 = 0; s0 < nch; s0 += 8) {
-            float cr[8], ci[8];
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                cr[j] = ci[j] = 0.f;
-                if (s0 + j < nch) {
-                    const int c = reverse ? nch - 1 - (s0 + j) : s0 + j;
-                    const size_t base = (((size_t)bh * nch + c) * 2 + x) * R2;
-                    cr[j] = __ldg(contrib + (base + 2 * m) * D + e);
-                    ci[j] = __ldg(contrib + (base + 2 * m + 1) * D + e);
-                }
-            }
-#pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                if (s0 + j >= nch) break;
-                const int c = reverse ? nch - 1 - (s0 + j) : s0 + j;
-                const size_t base = (((size_t)bh * nch + c) * 2 + x) * R2;
-                wout[(base + 2 * m) * D + e] = __float2bfloat16_rn(re);
-                wout[(base + 2 * m + 1) * D + e] = __float2bfloat16_rn(im);
-                const float ar = re + cr[j], ai = im + ci[j];
-                if (!reverse) {          // rot by +m w C
-                    re = cs * ar - sn * ai;
-                    im = sn * ar + cs * ai;
-                } else {                 // transpose: rot by -m w C
-                    re = cs * ar + sn * ai;
-                    im = -sn * ar + cs * ai;
-                }
-            }
-        }
-    }
-}
 // Absolute form: (cos, sin)(-m w c C) for every chunk c and mode m, in fp64 rounded to fp32.
 __global__ void k_chunk_phase(int M, int nch, double w, float *out) {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < nch * M; i += gridDim.x * blockDim.x) {
@@ -403,6 +346,365 @@ __global__ void k_rowdot(int BH, int L, int nch, int D, const bf16 *dout, const 
     }
 }
 
+// ------------------------------------------------------------------ chunk-sequential state kernels
+//
+// One CTA per (head, x) with x = 0 (K) or 1 (V) walks the chunks in order and keeps the fp32 state
+// in the registers of its eight epilogue warps (thread = state row r, warpgroup wg = columns
+// [wg D/2, (wg+1) D/2)); the tensor cores compute each chunk's contribution into TMEM.
+//   k_fwd_states  W_0 = 0, W_{c+1} = rot_C (W_c + EB X_c): the forward's chunk states (bf16, every c)
+//   k_adj_states  L_last = 0, L_{c-1} = rot_C^T (L_c + X_c^T), X_c^T = dX^T Q (K) or A'^T dO (V),
+//                 and the gradient dK_c = dP^T Q + EB^T L_c (K) or dV_c = G^T dO + EB^T L_c (V)
+// Warps 0-7 are the epilogue, 8 issues TMA loads, 9 allocates TMEM and issues the MMAs.
+
+constexpr int kSeqThreads = 320;
+constexpr int kSeqEpiWarps = 8;
+
+// SW128 descriptors of the chunk kernels' tiles.  A K-major tile stores [K/64][rows][64] (row =
+// M or N index); an MN-major tile stores [MN/64][krows][64] (row = K index).
+__device__ __forceinline__ uint64_t seq_kmaj(uint32_t base, int rows, int blk, int k) {
+    return tc::sdesc_sw128(base + (uint32_t)((k >> 2) * rows * 128 + blk * 128 * 128 + (k & 3) * 32), 16, 1024);
+}
+__device__ __forceinline__ uint64_t seq_mnmaj(uint32_t base, int krows, int blk, int k) {
+    return tc::sdesc_sw128(base + (uint32_t)(blk * 2 * krows * 128 + k * 16 * 128), (uint32_t)krows * 128u, 1024);
+}
+
+// 64 (or 32) bf16 values of one row into global memory (16-byte stores).
+template <int N>
+__device__ __forceinline__ void st_row_global(bf16 *dst, const float *v) {
+#pragma unroll
+    for (int i = 0; i < N; i += 8)
+        *reinterpret_cast<uint4 *>(dst + i) =
+            make_uint4(tc::pack_bf16x2(v[i], v[i + 1]), tc::pack_bf16x2(v[i + 2], v[i + 3]),
+                       tc::pack_bf16x2(v[i + 4], v[i + 5]), tc::pack_bf16x2(v[i + 6], v[i + 7]));
+}
+
+// One step of rot_C (sign +1) or its transpose (sign -1) on interleaved (Re, Im) rows held by
+// lane pairs (2m, 2m+1) of a warp.
+template <int N>
+__device__ __forceinline__ void rot_rows(float (&s)[N], bool odd, float cs, float sn, float sign) {
+    const float sg = sign * sn;
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        const float partner = __shfl_xor_sync(0xffffffffu, s[i], 1);
+        s[i] = odd ? fmaf(sg, partner, cs * s[i]) : fmaf(-sg, partner, cs * s[i]);
+    }
+}
+
+// 32 values of one row of a [cols/64][rows_per_block][64] bf16 tile in the 128-byte-swizzled layout.
+__device__ __forceinline__ void st_row32_bf16_seq(uint8_t *tile, int rows_per_block, int row, int col0, const float *v) {
+    uint8_t *blk = tile + (size_t)(col0 >> 6) * rows_per_block * 128;
+    const int c = col0 & 63;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        uint4 pk;
+        pk.x = tc::pack_bf16x2(v[q * 8 + 0], v[q * 8 + 1]);
+        pk.y = tc::pack_bf16x2(v[q * 8 + 2], v[q * 8 + 3]);
+        pk.z = tc::pack_bf16x2(v[q * 8 + 4], v[q * 8 + 5]);
+        pk.w = tc::pack_bf16x2(v[q * 8 + 6], v[q * 8 + 7]);
+        *reinterpret_cast<uint4 *>(blk + tc::sw128_offset(row, c + q * 8)) = pk;
+    }
+}
+
+struct SeqArgs {
+    int BH, L, nch, M, R2, RP, D;
+    const float *erel;   // (cos, sin)(m w tau), [C+1][M][2]
+    bf16 *wout;          // k_fwd_states: [BH][nch][2][R2][D]
+    bf16 *gout[2];       // k_adj_states: dk, dv [BH][L][D]
+    int *err;
+};
+
+enum FsBar { FS_EB, FS_FULL0, FS_EMPTY0 = FS_FULL0 + 4, FS_DFULL0 = FS_EMPTY0 + 4, FS_DEMPTY0 = FS_DFULL0 + 2,
+             FS_COUNT = FS_DEMPTY0 + 2 };
+constexpr int kFsStages = 3;
+
+template <int D, int NB>
+__global__ void __launch_bounds__(kSeqThreads, 1)
+    k_fwd_states(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+                 const __grid_constant__ CUtensorMap tm_eb, SeqArgs a) {
+    constexpr int DH = D / 2, RP = NB * 128;
+    const int x = blockIdx.x & 1, bh = blockIdx.x >> 1;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sEB = sm;                                   // [2][RP][64] K-major A (rows r, K = u)
+    uint8_t *sX = sEB + RP * 256;                        // kFsStages x [D/64][128 u][64] MN-major B
+    constexpr int x_bytes = 128 * D * 2;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sX + kFsStages * x_bytes);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + FS_COUNT);
+    Ctl *ctl = reinterpret_cast<Ctl *>(bar + FS_COUNT + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nupd = a.nch - 1;                          // chunks whose contribution is needed
+
+    if (threadIdx.x == 0) {
+        tc::mbar_init(&bar[FS_EB], 1);
+        for (int i = 0; i < kFsStages; ++i) { tc::mbar_init(&bar[FS_FULL0 + i], 1); tc::mbar_init(&bar[FS_EMPTY0 + i], 1); }
+        for (int i = 0; i < 2; ++i) { tc::mbar_init(&bar[FS_DFULL0 + i], 1); tc::mbar_init(&bar[FS_DEMPTY0 + i], kSeqEpiWarps); }
+        ctl->abort = 0;
+        tc::fence_barrier_init();
+    }
+    if (warp == 9) { tc::tmem_alloc(tslot, 512); tc::tmem_relinquish(); }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tb = *tslot;
+
+    if (warp == 8) {
+        if (lane == 0 && nupd > 0) {
+            const CUtensorMap *mx = x ? &tm_v : &tm_k;
+            tc::mbar_arrive_expect_tx(&bar[FS_EB], (uint32_t)(RP * 256));
+            for (int b = 0; b < NB; ++b)
+                for (int ub = 0; ub < 2; ++ub)
+                    tc::tma_load_2d(sEB + ub * RP * 128 + b * 128 * 128, &tm_eb, &bar[FS_EB], ub * 64, b * 128);
+            uint32_t ph[kFsStages] = {0, 0, 0};
+            for (int c = 0; c < nupd && !ctl->abort; ++c) {
+                const int st = c % kFsStages;
+                if (c >= kFsStages && !wait_bar(&bar[FS_EMPTY0 + st], ph[st], ctl, a.err, 10)) break;
+                tc::mbar_arrive_expect_tx(&bar[FS_FULL0 + st], (uint32_t)x_bytes);
+                for (int db = 0; db < D / 64; ++db)
+                    tc::tma_load_3d(sX + st * x_bytes + db * 128 * 128, mx, &bar[FS_FULL0 + st], db * 64, c * kC, bh);
+            }
+        }
+    } else if (warp == 9) {
+        if (lane == 0 && nupd > 0) {
+            uint32_t ph_eb = 0, ph[kFsStages] = {0, 0, 0}, ph_de[2] = {0, 0};
+            const uint32_t idesc = tc::idesc_bf16(128, D, false, true);
+            bool ok = wait_bar(&bar[FS_EB], ph_eb, ctl, a.err, 11);
+            for (int c = 0; c < nupd && ok; ++c) {
+                const int st = c % kFsStages, buf = c & 1;
+                if (c >= 2 && !wait_bar(&bar[FS_DEMPTY0 + buf], ph_de[buf], ctl, a.err, 12)) break;
+                if (!wait_bar(&bar[FS_FULL0 + st], ph[st], ctl, a.err, 13)) break;
+                tc::tc_fence_after();
+                const uint32_t xs = tc::smem_u32(sX + st * x_bytes), es = tc::smem_u32(sEB);
+                for (int b = 0; b < NB; ++b)
+                    for (int k = 0; k < 8; ++k)
+                        tc::mma_bf16(tb + (uint32_t)((buf * NB + b) * D), seq_kmaj(es, RP, b, k), seq_mnmaj(xs, 128, 0, k),
+                                     idesc, k > 0 ? 1u : 0u);
+                tc::mma_commit(&bar[FS_EMPTY0 + st]);
+                tc::mma_commit(&bar[FS_DFULL0 + buf]);
+            }
+        }
+    } else {
+        const int wg = warp >> 2, lane_base = (warp & 3) * 32, row = lane_base + lane;
+        const bool odd = row & 1;
+        float s[NB][DH];
+        float cs[NB], sn[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            const int m = (b * 128 + row) >> 1;
+            cs[b] = m < a.M ? a.erel[((size_t)kC * a.M + m) * 2] : 1.f;
+            sn[b] = m < a.M ? a.erel[((size_t)kC * a.M + m) * 2 + 1] : 0.f;
+#pragma unroll
+            for (int i = 0; i < DH; ++i) s[b][i] = 0.f;
+        }
+        uint32_t ph_df[2] = {0, 0};
+        for (int c = 0; c < a.nch; ++c) {
+            // W_c
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                const int r = b * 128 + row;
+                if (r < a.R2)
+                    st_row_global<DH>(a.wout + ((((size_t)bh * a.nch + c) * 2 + x) * a.R2 + r) * D + wg * DH, s[b]);
+            }
+            if (c == nupd) break;
+            const int buf = c & 1;
+            if (!wait_bar(&bar[FS_DFULL0 + buf], ph_df[buf], ctl, a.err, 14)) break;
+            tc::tc_fence_after();
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                float v[DH];
+                tc::tmem_ld<DH>(tb + ((uint32_t)lane_base << 16) + (uint32_t)((buf * NB + b) * D + wg * DH), v);
+#pragma unroll
+                for (int i = 0; i < DH; ++i) s[b][i] += v[i];
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[FS_DEMPTY0 + buf]);
+#pragma unroll
+            for (int b = 0; b < NB; ++b) rot_rows<DH>(s[b], odd, cs[b], sn[b], 1.f);
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tb, 512);
+    }
+}
+
+enum AsBar { AS_EB, AS_FULL0, AS_FREE0 = AS_FULL0 + 2, AS_CFULL0 = AS_FREE0 + 2, AS_CEMPTY0 = AS_CFULL0 + 2,
+             AS_LB = AS_CEMPTY0 + 2, AS_DKFULL, AS_DKEMPTY, AS_COUNT };
+
+// Shared memory of k_adj_states: EB, then `stages` x (Xa [RP/64][128 t][64], Bq [D/64][128 t][64],
+// Pa [2][128 t][64]); L_c (bf16, [D/64][R2][64]) is written over the stage's Xa once its MMA is done.
+__host__ __device__ inline int adj_stage_bytes(int RP, int D) { return RP * 256 + D * 256 + 2 * 128 * 128; }
+
+template <int D, int NB>
+__global__ void __launch_bounds__(kSeqThreads, 1)
+    k_adj_states(const __grid_constant__ CUtensorMap tm_dx, const __grid_constant__ CUtensorMap tm_ap,
+                 const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_do,
+                 const __grid_constant__ CUtensorMap tm_dp, const __grid_constant__ CUtensorMap tm_g,
+                 const __grid_constant__ CUtensorMap tm_eb, SeqArgs a, int stages) {
+    constexpr int DH = D / 2, RP = NB * 128;
+    constexpr int NCB = NB == 1 ? 2 : 1;                 // contribution buffers in TMEM
+    const int x = blockIdx.x & 1, bh = blockIdx.x >> 1;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *sEB = sm;                                   // [2][RP][64]: MN-major A of EB^T (M = u, K = r)
+    uint8_t *sStage = sEB + RP * 256;
+    const int sbytes = adj_stage_bytes(RP, D);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sStage + stages * sbytes);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + AS_COUNT);
+    Ctl *ctl = reinterpret_cast<Ctl *>(bar + AS_COUNT + 1);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nch = a.nch, R2 = a.R2;
+    const uint32_t colDK = (uint32_t)(NCB * NB * D);
+    // chunk i of the walk is c = nch - 1 - i
+
+    if (threadIdx.x == 0) {
+        tc::mbar_init(&bar[AS_EB], 1);
+        for (int i = 0; i < 2; ++i) {
+            tc::mbar_init(&bar[AS_FULL0 + i], 1);
+            tc::mbar_init(&bar[AS_FREE0 + i], 1);
+            tc::mbar_init(&bar[AS_CFULL0 + i], 1);
+            tc::mbar_init(&bar[AS_CEMPTY0 + i], kSeqEpiWarps);
+        }
+        tc::mbar_init(&bar[AS_LB], kSeqEpiWarps);
+        tc::mbar_init(&bar[AS_DKFULL], 1);
+        tc::mbar_init(&bar[AS_DKEMPTY], kSeqEpiWarps);
+        ctl->abort = 0;
+        tc::fence_barrier_init();
+    }
+    if (warp == 9) { tc::tmem_alloc(tslot, 512); tc::tmem_relinquish(); }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tb = *tslot;
+
+    if (warp == 8) {
+        if (lane == 0) {
+            const CUtensorMap *ma = x ? &tm_ap : &tm_dx, *mb = x ? &tm_do : &tm_q, *mp = x ? &tm_g : &tm_dp;
+            tc::mbar_arrive_expect_tx(&bar[AS_EB], (uint32_t)(RP * 256));
+            for (int b = 0; b < NB; ++b)
+                for (int ub = 0; ub < 2; ++ub)
+                    tc::tma_load_2d(sEB + ub * RP * 128 + b * 128 * 128, &tm_eb, &bar[AS_EB], ub * 64, b * 128);
+            uint32_t ph[2] = {0, 0};
+            for (int i = 0; i < nch && !ctl->abort; ++i) {
+                const int c = nch - 1 - i, st = i % stages;
+                if (i >= stages && !wait_bar(&bar[AS_FREE0 + st], ph[st], ctl, a.err, 20)) break;
+                uint8_t *base = sStage + st * sbytes;
+                tc::mbar_arrive_expect_tx(&bar[AS_FULL0 + st], (uint32_t)sbytes);
+                const int z = bh * nch + c;
+                for (int rb = 0; rb < RP / 64; ++rb)            // beyond R2: zero fill
+                    tc::tma_load_3d(base + rb * 128 * 128, ma, &bar[AS_FULL0 + st], rb * 64, 0, z);
+                for (int db = 0; db < D / 64; ++db)
+                    tc::tma_load_3d(base + RP * 256 + db * 128 * 128, mb, &bar[AS_FULL0 + st], db * 64, c * kC, bh);
+                for (int ub = 0; ub < 2; ++ub)
+                    tc::tma_load_3d(base + RP * 256 + D * 256 + ub * 128 * 128, mp, &bar[AS_FULL0 + st], ub * 64, 0, z);
+            }
+        }
+    } else if (warp == 9) {
+        if (lane == 0) {
+            uint32_t ph_eb = 0, ph[2] = {0, 0}, ph_ce[2] = {0, 0}, ph_lb = 0, ph_dke = 0;
+            const uint32_t id_c = tc::idesc_bf16(128, D, true, true);   // A = (dX or A')^T, B = Q or dO: MN-major
+            bool ok = wait_bar(&bar[AS_EB], ph_eb, ctl, a.err, 21);
+            for (int i = 0; i < nch && ok; ++i) {
+                ok = false;
+                const int st = i % stages, cb = i % NCB;
+                if (!wait_bar(&bar[AS_FULL0 + st], ph[st], ctl, a.err, 22)) break;
+                if (i >= NCB && !wait_bar(&bar[AS_CEMPTY0 + cb], ph_ce[cb], ctl, a.err, 23)) break;
+                tc::tc_fence_after();
+                const uint32_t base = tc::smem_u32(sStage + st * sbytes);
+                const uint32_t xa = base, bq = base + RP * 256, pa = bq + D * 256, es = tc::smem_u32(sEB);
+                // X_c^T = (dX or A')^T (Q or dO): M = state rows, K = the chunk's tokens
+                for (int b = 0; b < NB; ++b)
+                    for (int k = 0; k < 8; ++k)
+                        tc::mma_bf16(tb + (uint32_t)((cb * NB + b) * D), seq_mnmaj(xa, 128, b, k), seq_mnmaj(bq, 128, 0, k),
+                                     id_c, k > 0 ? 1u : 0u);
+                tc::mma_commit(&bar[AS_CFULL0 + cb]);
+                // dK_c = dP^T Q + EB^T L_c (or dV_c = G^T dO + EB^T L_c): M = the chunk's tokens u
+                if (i > 0 && !wait_bar(&bar[AS_DKEMPTY], ph_dke, ctl, a.err, 24)) break;
+                tc::tc_fence_after();
+                for (int k = 0; k < 8; ++k)
+                    tc::mma_bf16(tb + colDK, seq_mnmaj(pa, 128, 0, k), seq_mnmaj(bq, 128, 0, k), id_c, k > 0 ? 1u : 0u);
+                if (!wait_bar(&bar[AS_LB], ph_lb, ctl, a.err, 25)) break;
+                tc::tc_fence_after();
+                for (int k = 0; k < R2 / 16; ++k)
+                    tc::mma_bf16(tb + colDK, seq_mnmaj(es, RP, 0, k), seq_mnmaj(xa, R2, 0, k), id_c, 1u);
+                tc::mma_commit(&bar[AS_DKFULL]);
+                tc::mma_commit(&bar[AS_FREE0 + st]);
+                ok = true;
+            }
+        }
+    } else {
+        const int wg = warp >> 2, lane_base = (warp & 3) * 32, row = lane_base + lane;
+        const bool odd = row & 1;
+        float s[NB][DH];
+        float cs[NB], sn[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            const int m = (b * 128 + row) >> 1;
+            cs[b] = m < a.M ? a.erel[((size_t)kC * a.M + m) * 2] : 1.f;
+            sn[b] = m < a.M ? a.erel[((size_t)kC * a.M + m) * 2 + 1] : 0.f;
+#pragma unroll
+            for (int i = 0; i < DH; ++i) s[b][i] = 0.f;
+        }
+        uint32_t ph_cf[2] = {0, 0}, ph_dkf = 0;
+        bf16 *gout = a.gout[x];
+        for (int i = 0; i < nch; ++i) {
+            const int c = nch - 1 - i, st = i % stages, cb = i % NCB;
+            // L_c (bf16) over the stage's Xa once the contribution MMA has read it
+            if (!wait_bar(&bar[AS_CFULL0 + cb], ph_cf[cb], ctl, a.err, 26)) break;
+            tc::tc_fence_after();
+            uint8_t *lb = sStage + st * sbytes;
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                const int r = b * 128 + row;
+                if (r < R2) {
+#pragma unroll
+                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16_seq(lb, R2, r, wg * DH + g0, s[b] + g0);
+                }
+            }
+            tc::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[AS_LB]);
+            // L_{c-1} = rot_C^T (L_c + X_c^T)
+            if (c > 0) {
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    float v[DH];
+                    tc::tmem_ld<DH>(tb + ((uint32_t)lane_base << 16) + (uint32_t)((cb * NB + b) * D + wg * DH), v);
+#pragma unroll
+                    for (int j = 0; j < DH; ++j) s[b][j] += v[j];
+                }
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[AS_CEMPTY0 + cb]);
+            if (c > 0) {
+#pragma unroll
+                for (int b = 0; b < NB; ++b) rot_rows<DH>(s[b], odd, cs[b], sn[b], -1.f);
+            }
+            // the chunk's gradient rows
+            if (!wait_bar(&bar[AS_DKFULL], ph_dkf, ctl, a.err, 27)) break;
+            tc::tc_fence_after();
+            {
+                float v[DH];
+                tc::tmem_ld<DH>(tb + ((uint32_t)lane_base << 16) + colDK + (uint32_t)(wg * DH), v);
+                const int t = c * kC + row;
+                if (t < a.L) st_row_global<DH>(gout + ((size_t)bh * a.L + t) * D + wg * DH, v);
+            }
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[AS_DKEMPTY]);
+        }
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tb, 512);
+    }
+}
+
 // ------------------------------------------------------------------ host side
 
 struct BwdGeo {
@@ -420,7 +722,7 @@ BwdGeo bwd_geo(const OpDims &d) {
 }
 
 struct BwdWs {
-    size_t tables, eb, phi, cphase, cb, wb, lb, P, Y, p, A, G, dG, dU, ds, dX, dP, dKi, dVi, dl, total;
+    size_t tables, eb, phi, cphase, wb, P, Y, p, A, G, dG, dU, ds, dX, dP, dl, total;
 };
 
 BwdWs bwd_ws(const OpDims &d, const BwdGeo &g) {
@@ -432,9 +734,7 @@ BwdWs bwd_ws(const OpDims &d, const BwdGeo &g) {
     w.eb = take(2 * (size_t)g.RP * kC);
     w.phi = take(2 * (size_t)g.SP * g.R2);
     w.cphase = take(d.absolute ? 4 * (size_t)g.nch * g.M * 2 : 0);
-    w.cb = take(4 * Z * 2 * g.R2 * g.D);
     w.wb = take(2 * Z * 2 * g.R2 * g.D);
-    w.lb = take(2 * Z * 2 * g.R2 * g.D);
     w.P = take(2 * Z * kC * kC);
     w.Y = take(2 * Z * kC * g.R2);
     w.p = take(2 * Z * kC * g.SP);
@@ -445,8 +745,6 @@ BwdWs bwd_ws(const OpDims &d, const BwdGeo &g) {
     w.ds = take(2 * Z * kC * g.SP);
     w.dX = take(2 * Z * kC * g.R2);
     w.dP = take(2 * Z * kC * kC);
-    w.dKi = take(4 * Z * kC * g.D);
-    w.dVi = take(4 * Z * kC * g.D);
     w.dl = take(4 * Z * kC);
     w.total = off;
     return w;
@@ -525,6 +823,58 @@ cudaError_t gemm(const BwdGeo &g, int mtiles, int N, const CUtensorMap &a0, cons
     return cudaGetLastError();
 }
 
+template <int D, int NB>
+cudaError_t launch_fwd_states_t(const BwdGeo &g, const CUtensorMap &mk, const CUtensorMap &mv, const CUtensorMap &meb,
+                                const SeqArgs &sa, cudaStream_t st) {
+    // (both chunk kernels allocate all 512 TMEM columns: at least 120 KB of shared memory keeps a
+    //  second CTA off the SM, so an allocation never waits for another CTA to finish)
+    int smem = NB * 128 * 256 + kFsStages * 128 * D * 2 + 256 + 1024;
+    if (smem < 120 * 1024) smem = 120 * 1024;
+    cudaError_t e = cudaFuncSetAttribute(k_fwd_states<D, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    ProfScope ps(BLA_K_BWD, st);
+    k_fwd_states<D, NB><<<g.BH * 2, kSeqThreads, smem, st>>>(mk, mv, meb, sa);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fwd_states(const BwdGeo &g, const CUtensorMap &mk, const CUtensorMap &mv, const CUtensorMap &meb,
+                              const SeqArgs &sa, cudaStream_t st) {
+    const int NB = g.RP / 128;
+    if (g.D == 128) return NB == 1 ? launch_fwd_states_t<128, 1>(g, mk, mv, meb, sa, st)
+                                   : launch_fwd_states_t<128, 2>(g, mk, mv, meb, sa, st);
+    if (g.D == 64) return NB == 1 ? launch_fwd_states_t<64, 1>(g, mk, mv, meb, sa, st)
+                                  : launch_fwd_states_t<64, 2>(g, mk, mv, meb, sa, st);
+    return cudaErrorInvalidValue;
+}
+
+template <int D, int NB>
+cudaError_t launch_adj_states_t(const BwdGeo &g, const CUtensorMap &mdx, const CUtensorMap &map_, const CUtensorMap &mq,
+                                const CUtensorMap &mdo, const CUtensorMap &mdp, const CUtensorMap &mg,
+                                const CUtensorMap &meb, const SeqArgs &sa, cudaStream_t st) {
+    const int RP = NB * 128, sbytes = adj_stage_bytes(RP, D);
+    int stages = (227 * 1024 - 1024 - 256 - RP * 256) / sbytes;
+    if (stages > 2) stages = 2;
+    if (stages < 1) return cudaErrorInvalidValue;
+    int smem = RP * 256 + stages * sbytes + 256 + 1024;
+    if (smem < 120 * 1024) smem = 120 * 1024;
+    cudaError_t e = cudaFuncSetAttribute(k_adj_states<D, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    ProfScope ps(BLA_K_BWD, st);
+    k_adj_states<D, NB><<<g.BH * 2, kSeqThreads, smem, st>>>(mdx, map_, mq, mdo, mdp, mg, meb, sa, stages);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_adj_states(const BwdGeo &g, const CUtensorMap &mdx, const CUtensorMap &map_, const CUtensorMap &mq,
+                              const CUtensorMap &mdo, const CUtensorMap &mdp, const CUtensorMap &mg,
+                              const CUtensorMap &meb, const SeqArgs &sa, cudaStream_t st) {
+    const int NB = g.RP / 128;
+    if (g.D == 128) return NB == 1 ? launch_adj_states_t<128, 1>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st)
+                                   : launch_adj_states_t<128, 2>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st);
+    if (g.D == 64) return NB == 1 ? launch_adj_states_t<64, 1>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st)
+                                  : launch_adj_states_t<64, 2>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st);
+    return cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 const char *bwd_unsupported(const OpDims &d) {
@@ -558,9 +908,8 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
         k_chunk_phase<<<(n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024, 256, 0, st>>>(g.M, g.nch, d.w, cphase);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
-    float *cb = reinterpret_cast<float *>(ws + w.cb), *dKi = reinterpret_cast<float *>(ws + w.dKi);
-    float *dVi = reinterpret_cast<float *>(ws + w.dVi), *dl = reinterpret_cast<float *>(ws + w.dl);
-    bf16 *wb = reinterpret_cast<bf16 *>(ws + w.wb), *lb = reinterpret_cast<bf16 *>(ws + w.lb);
+    float *dl = reinterpret_cast<float *>(ws + w.dl);
+    bf16 *wb = reinterpret_cast<bf16 *>(ws + w.wb);
     bf16 *Pb = reinterpret_cast<bf16 *>(ws + w.P), *Yb = reinterpret_cast<bf16 *>(ws + w.Y);
     bf16 *pb = reinterpret_cast<bf16 *>(ws + w.p), *Ab = reinterpret_cast<bf16 *>(ws + w.A);
     bf16 *Gb = reinterpret_cast<bf16 *>(ws + w.G), *dGb = reinterpret_cast<bf16 *>(ws + w.dG);
@@ -570,47 +919,32 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     const int rt = g.R2 <= 128 ? 1 : g.R2 / 128;   // 128-row tiles of an [R2 x D] result
 
     // ---- tensor maps
-    CUtensorMap qK, qM, kK, kM, vK, vM, dOK, dOM, ebK128, ebKR, ebM, phiK, phiM;
-    CUtensorMap wbK, wbM, lbM, PK, YK, pK, AK, AM, GK, GM, dGK, dUK, dsK, dXK, dXM, dPK, dPM;
-    bool ok = map_seq(&qK, q, g, D, true, kC) && map_seq(&qM, q, g, D, false, 0) && map_seq(&kK, k, g, D, true, kC) &&
-              map_seq(&kM, k, g, D, false, 0) && map_seq(&vK, v, g, D, true, kC) && map_seq(&vM, v, g, D, false, 0) &&
-              map_seq(&dOK, dout, g, D, true, kC) && map_seq(&dOM, dout, g, D, false, 0) &&
+    CUtensorMap qK, kK, kM, vK, dOK, ebK128, ebKR, ebM, phiK, phiM;
+    CUtensorMap wbK, wbM, PK, YK, pK, AK, GK, dGK, dUK, dsK, dXK, dPK;
+    bool ok = map_seq(&qK, q, g, D, true, kC) && map_seq(&kK, k, g, D, true, kC) && map_seq(&kM, k, g, D, false, 0) &&
+              map_seq(&vK, v, g, D, true, kC) && map_seq(&dOK, dout, g, D, true, kC) &&
               map_2d(&ebK128, eb, kC, g.RP, true, 128) && map_2d(&ebKR, eb, kC, g.RP, true, R2) &&
               map_2d(&ebM, eb, kC, g.RP, false, 0) && map_2d(&phiK, phi, R2, SP, true, S) &&
               map_2d(&phiM, phi, R2, SP, false, 0) && map_z(&wbK, wb, D, R2, 2 * Z, true, R2) &&
-              map_z(&wbM, wb, D, R2, 2 * Z, false, 0) && map_z(&lbM, lb, D, R2, 2 * Z, false, 0) &&
+              map_z(&wbM, wb, D, R2, 2 * Z, false, 0) &&
               map_z(&PK, Pb, kC, kC, Z, true, kC) && map_z(&YK, Yb, R2, kC, Z, true, kC) &&
               map_z(&pK, pb, SP, kC, Z, true, kC) && map_z(&AK, Ab, R2, kC, Z, true, kC) &&
-              map_z(&AM, Ab, R2, kC, Z, false, 0) && map_z(&GK, Gb, kC, kC, Z, true, kC) &&
-              map_z(&GM, Gb, kC, kC, Z, false, 0) && map_z(&dGK, dGb, kC, kC, Z, true, kC) &&
+              map_z(&GK, Gb, kC, kC, Z, true, kC) && map_z(&dGK, dGb, kC, kC, Z, true, kC) &&
               map_z(&dUK, dUb, R2, kC, Z, true, kC) && map_z(&dsK, dsb, SP, kC, Z, true, kC) &&
-              map_z(&dXK, dXb, R2, kC, Z, true, kC) && map_z(&dXM, dXb, R2, kC, Z, false, 0) &&
-              map_z(&dPK, dPb, kC, kC, Z, true, kC) && map_z(&dPM, dPb, kC, kC, Z, false, 0);
-    (void)GK;
+              map_z(&dXK, dXb, R2, kC, Z, true, kC) && map_z(&dPK, dPb, kC, kC, Z, true, kC);
     if (!ok) return cudaErrorInvalidValue;
     const Operand SEQK = opnd(OP_SEQ, 1), SEQM = opnd(OP_SEQ, 0);
     const Operand ZK = opnd(OP_Z, 1), ZM = opnd(OP_Z, 0);
     const Operand SHK = opnd(OP_SHARED, 1), SHM = opnd(OP_SHARED, 0);
     const Operand WK_K = opnd(OP_Z, 1, 2, 0), WV_K = opnd(OP_Z, 1, 2, 1);
-    const Operand WK_M = opnd(OP_Z, 0, 2, 0), LK_M = opnd(OP_Z, 0, 2, 0), LV_M = opnd(OP_Z, 0, 2, 1);
+    const Operand WK_M = opnd(OP_Z, 0, 2, 0);
 
-    // ---- 0. forward chunk states: contrib = EB X_c, then the scan
-    for (int x = 0; x < 2; ++x) {
-        Epi ep = epi_base(EP_PLAIN, cb, OUT_Z, 1, D, D, R2);
-        ep.out_zmul = 2; ep.out_zoff = x;
-        // A = EB (rows r, K = tau'), B = X_c MN-major (K rows tau', N = d)
-        if ((e = gemm(g, rt, D, ebK128, SHK, x ? vM : kM, SEQM, kC, nullptr, nullptr, nullptr, nullptr, 0, ep, st)) !=
-            cudaSuccess)
-            return e;
-    }
-    {
-        long long total = (long long)g.BH * 2 * g.M * D;
-        int blocks = (int)((total + 255) / 256);
-        if (blocks > 4096) blocks = 4096;
-        ProfScope ps(BLA_K_BWD, st);
-        k_state_scan<<<blocks, 256, 0, st>>>(g.BH, g.nch, g.M, D, t.erel, cb, wb, 0);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
+    // ---- 0. forward chunk states W_c (bf16), scanned over the chunks of each head in registers
+    SeqArgs sa;
+    sa.BH = g.BH; sa.L = g.L; sa.nch = g.nch; sa.M = g.M; sa.R2 = R2; sa.RP = g.RP; sa.D = D;
+    sa.erel = t.erel; sa.wout = wb; sa.gout[0] = static_cast<bf16 *>(dk); sa.gout[1] = static_cast<bf16 *>(dv);
+    sa.err = device_error_word();
+    if ((e = launch_fwd_states(g, kK, vK, ebK128, sa, st)) != cudaSuccess) return e;
     Epi ep;
     // ---- 1. recompute the chunk's forward quantities
     ep = epi_base(EP_CAUSAL, Pb, OUT_Z, 0, kC, kC);                                   // P = tril(Q K^T)
@@ -646,28 +980,9 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     if ((e = gemm(g, 1, kC, dXK, ZK, ebM, SHM, R2, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
     ep = epi_base(EP_PLAIN, dq, OUT_SEQ, 0, D, D);                                     // dQ = dP K + dX W_K
     if ((e = gemm(g, 1, D, dPK, ZK, kM, SEQM, kC, &dXK, &ZK, &wbM, &WK_M, R2, ep, st))) return e;
-    ep = epi_base(EP_PLAIN, dKi, OUT_Z, 1, D, D);                                      // dK intra = dP^T Q
-    if ((e = gemm(g, 1, D, dPM, ZM, qM, SEQM, kC, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_PLAIN, dVi, OUT_Z, 1, D, D);                                      // dV intra = G^T dO
-    if ((e = gemm(g, 1, D, GM, ZM, dOM, SEQM, kC, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_PLAIN, cb, OUT_Z, 1, D, D, R2); ep.out_zmul = 2; ep.out_zoff = 0;   // contrib K = dX^T Q
-    if ((e = gemm(g, rt, D, dXM, ZM, qM, SEQM, kC, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_PLAIN, cb, OUT_Z, 1, D, D, R2); ep.out_zmul = 2; ep.out_zoff = 1;   // contrib V = A'^T dO
-    if ((e = gemm(g, rt, D, AM, ZM, dOM, SEQM, kC, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    // ---- 3. adjoint states, backwards over the chunks
-    {
-        long long total = (long long)g.BH * 2 * g.M * D;
-        int blocks = (int)((total + 255) / 256);
-        if (blocks > 4096) blocks = 4096;
-        ProfScope ps(BLA_K_BWD, st);
-        k_state_scan<<<blocks, 256, 0, st>>>(g.BH, g.nch, g.M, D, t.erel, cb, lb, 1);
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-    }
-    // ---- 4. dK = dK intra + EB^T Lk, dV = dV intra + EB^T Lv
-    ep = epi_base(EP_ADD, dk, OUT_SEQ, 0, D, D); ep.addend = dKi;
-    if ((e = gemm(g, 1, D, ebM, SHM, lbM, LK_M, R2, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
-    ep = epi_base(EP_ADD, dv, OUT_SEQ, 0, D, D); ep.addend = dVi;
-    if ((e = gemm(g, 1, D, ebM, SHM, lbM, LV_M, R2, nullptr, nullptr, nullptr, nullptr, 0, ep, st))) return e;
+    // ---- 3. adjoint states backwards over the chunks, with dK = dP^T Q + EB^T Lk and
+    //         dV = G^T dO + EB^T Lv for every chunk on the way
+    if ((e = launch_adj_states(g, dXK, AK, qK, dOK, dPK, GK, ebK128, sa, st)) != cudaSuccess) return e;
     return cudaSuccess;
 }
 
