@@ -705,6 +705,594 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     }
 }
 
+// ------------------------------------------------------------------ fused chunk chains
+//
+// For 2M <= 128 and S <= 64 the chunk-local part of the backward runs as two persistent kernels,
+// one CTA per SM walking chunks, whose intermediates stay on chip (TMEM accumulators drained into
+// bf16 shared-memory tiles that feed the next MMA):
+//   k_chain_fwd  P = tril(Q K^T) -> Y = rot+(P EB^T + Q W_K^T) -> p -> A' = rot-(p PHI) -> G = tril(A' EB)
+//                writes p, A' and G
+//   k_chain_adj  dG = tril(dO V^T) -> dU = rot+(dG EB^T + dO W_V^T) -> ds = p (dU PHI^T - rowsum(dO o))
+//                -> dX = rot-(scale ds PHI) -> dP = tril(dX EB) -> dQ = dP K + dX W_K
+//                writes dX, dP and dQ
+// Shared-memory tiles are 128B-swizzled [cols/64][rows][64]: K-major when rows index M or N, and
+// the same bytes serve as an MN-major B operand whose K index is the row (EB, PHI, K, W).
+// Warps 0-7 drain TMEM in 32-column chunks (warpgroup wg takes chunks wg, wg + 2, ...), warp 8
+// issues TMA loads, warp 9 issues the MMAs.  Outputs are written as bf16 tiles in shared memory
+// and stored by TMA (thread 0 issues the stores after an epilogue barrier, and waits for them to
+// have read their tiles before the next chunk overwrites any tile).
+
+struct ChainArgs {
+    int BH, L, nch, Z, M, R2, S, SP, D;
+    float scale;
+    const float *erel;    // (cos, sin)(m w tau), [C+1][M][2]
+    const float *cphase;  // absolute form: (cos, sin)(-m w c C), [nch][M][2]; else null
+    const float *lse;     // [BH][L]
+    const int *delta;     // [S]
+    const bf16 *o;        // [BH][L][D]
+    int *err;
+};
+
+// Phases of one thread's column range in a chunk: e^{i m0 w tau} for its first mode m0 and the step
+// e^{i w tau} between consecutive modes (tau = the row's offset in the chunk), or in the absolute
+// form the chunk's e^{-i m0 w t0} and e^{-i w t0}.
+struct RotPh {
+    float c0, s0, c1, s1;
+};
+
+__device__ __forceinline__ RotPh chain_phases(const ChainArgs &a, int c, int row, int m0) {
+    const float *ptab = a.cphase ? a.cphase + (size_t)c * a.M * 2 : a.erel + (size_t)row * a.M * 2;
+    RotPh r;
+    r.c0 = __ldg(ptab + m0 * 2);
+    r.s0 = __ldg(ptab + m0 * 2 + 1);
+    r.c1 = __ldg(ptab + 2);
+    r.s1 = __ldg(ptab + 3);
+    return r;
+}
+
+// Rotation of N interleaved (Re, Im) columns by the phases of `ph` (sign +1) or their transposes
+// (sign -1), times `scale`.
+template <int N>
+__device__ __forceinline__ void chain_rot(float (&v)[N], const RotPh &ph, float sign, float scale) {
+    float cs = ph.c0, sn = ph.s0;
+#pragma unroll
+    for (int i = 0; i < N; i += 2) {
+        const float sg = sign * sn, xr = v[i], xi = v[i + 1];
+        v[i] = scale * (cs * xr - sg * xi);
+        v[i + 1] = scale * (sg * xr + cs * xi);
+        const float t = cs * ph.c1 - sn * ph.s1;
+        sn = sn * ph.c1 + cs * ph.s1;
+        cs = t;
+    }
+}
+
+template <int N>
+__device__ __forceinline__ void chain_causal(float (&v)[N], int row, int col0) {
+#pragma unroll
+    for (int i = 0; i < N; ++i)
+        if (col0 + i > row) v[i] = 0.f;
+}
+
+template <int N>
+__device__ __forceinline__ void st_tile_row(uint8_t *tile, int row, int col0, const float (&v)[N]) {
+#pragma unroll
+    for (int g = 0; g < N; g += 32) st_row32_bf16_seq(tile, 128, row, col0 + g, v + g);
+}
+
+__device__ __forceinline__ uint32_t tm_addr(uint32_t tb, int lane_base, int col) {
+    return tb + ((uint32_t)lane_base << 16) + (uint32_t)col;
+}
+
+// ---- k_chain_fwd
+enum CfBar { CF_TAB, CF_IN_FULL, CF_IN_FREE, CF_ACC1, CF_ACC2, CF_ACC3, CF_ACC4, CF_ACC5, CF_T1, CF_T2, CF_SP, CF_A,
+             CF_TFREE, CF_ESYNC, CF_COUNT };
+
+struct ChainLayout {
+    int eb, phi, t0, t1, t2, t3, t4, sp, bars, total;
+};
+
+// k_chain_fwd: t0 = Q, t1 = K, t2 = W_K, t3 = T1 (P, then A'), t4 = T2 (Y, then G), sp = p.
+// k_chain_adj: t0 = dO, t1 = V then K, t2 = W_V then W_K, t3 = T1 (dG, then dP), t4 = T2 (dU, then
+//              dX, then dQ), sp = p, then ds.
+// The last 1 KB holds the barriers, the slot lags and the rows' rowsum(dO o).
+__host__ __device__ inline ChainLayout chain_layout(int R2, int S, int SP, int D) {
+    ChainLayout l;
+    int off = 0;
+    l.eb = off;  off += R2 * 256;
+    l.phi = off; off += R2 * S * 2;
+    off = (off + 1023) & ~1023;
+    l.t0 = off;  off += 256 * D;
+    l.t1 = off;  off += 256 * D;
+    l.t2 = off;  off += R2 * D * 2;
+    l.t3 = off;  off += 128 * 256;
+    l.t4 = off;  off += 128 * 256;
+    l.sp = off;  off += SP * 256;
+    l.bars = off; off += 1024;
+    l.total = off;
+    return l;
+}
+
+template <int R2, int S, int D>
+__global__ void __launch_bounds__(kSeqThreads, 1)
+    k_chain_fwd(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+                const __grid_constant__ CUtensorMap tm_w, const __grid_constant__ CUtensorMap tm_eb,
+                const __grid_constant__ CUtensorMap tm_phi, const __grid_constant__ CUtensorMap tm_po,
+                const __grid_constant__ CUtensorMap tm_ao, const __grid_constant__ CUtensorMap tm_go, ChainArgs a) {
+    constexpr int SP = S < 64 ? 64 : S, HX = R2 / 2, HS = S >= 64 ? S / 2 : S;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const ChainLayout lay = chain_layout(R2, S, SP, D);
+    uint8_t *sEB = sm + lay.eb, *sPHI = sm + lay.phi, *sQ = sm + lay.t0, *sK = sm + lay.t1, *sW = sm + lay.t2;
+    uint8_t *sT1 = sm + lay.t3, *sT2 = sm + lay.t4, *sP = sm + lay.sp;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + lay.bars);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + CF_COUNT);
+    Ctl *ctl = reinterpret_cast<Ctl *>(bar + CF_COUNT + 1);
+    int *sdelta = reinterpret_cast<int *>(bar + CF_COUNT + 2);   // [S]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int colP = 0, colX = 128, colS = 0, colU = 0, colG = 128;   // s after P is drained; U after s
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < CF_COUNT; ++i) {
+            const bool epi = i == CF_T1 || i == CF_T2 || i == CF_SP || i == CF_A || i == CF_TFREE || i == CF_ESYNC;
+            tc::mbar_init(&bar[i], epi ? kSeqEpiWarps : 1);
+        }
+        ctl->abort = 0;
+        tc::fence_barrier_init();
+    }
+    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
+    if (warp == 9) { tc::tmem_alloc(tslot, 256); tc::tmem_relinquish(); }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tb = *tslot;
+
+    if (warp == 8) {
+        if (lane == 0) {
+            tc::mbar_arrive_expect_tx(&bar[CF_TAB], (uint32_t)(R2 * 256 + R2 * S * 2));
+            for (int ub = 0; ub < 2; ++ub) tc::tma_load_2d(sEB + ub * R2 * 128, &tm_eb, &bar[CF_TAB], ub * 64, 0);
+            for (int rb = 0; rb < R2 / 64; ++rb) tc::tma_load_2d(sPHI + rb * S * 128, &tm_phi, &bar[CF_TAB], rb * 64, 0);
+            uint32_t ph_free = 0;
+            for (int z = blockIdx.x, i = 0; z < a.Z && !ctl->abort; z += gridDim.x, ++i) {
+                const int bh = z / a.nch, c = z % a.nch;
+                if (i > 0 && !wait_bar(&bar[CF_IN_FREE], ph_free, ctl, a.err, 30)) break;
+                tc::mbar_arrive_expect_tx(&bar[CF_IN_FULL], (uint32_t)(2 * 256 * D + R2 * D * 2));
+                for (int db = 0; db < D / 64; ++db) {
+                    tc::tma_load_3d(sQ + db * 128 * 128, &tm_q, &bar[CF_IN_FULL], db * 64, c * kC, bh);
+                    tc::tma_load_3d(sK + db * 128 * 128, &tm_k, &bar[CF_IN_FULL], db * 64, c * kC, bh);
+                    tc::tma_load_3d(sW + db * R2 * 128, &tm_w, &bar[CF_IN_FULL], db * 64, 0, 2 * z);
+                }
+            }
+        }
+    } else if (warp == 9) {
+        if (lane == 0) {
+            uint32_t ph[CF_COUNT] = {};
+            constexpr uint32_t id_P = tc::idesc_bf16(128, 128, false, false), id_X = tc::idesc_bf16(128, R2, false, false);
+            constexpr uint32_t id_S = tc::idesc_bf16(128, S, false, false), id_U = tc::idesc_bf16(128, R2, false, true);
+            constexpr uint32_t id_G = tc::idesc_bf16(128, 128, false, true);
+            const uint32_t q = tc::smem_u32(sQ), k = tc::smem_u32(sK), w = tc::smem_u32(sW), eb = tc::smem_u32(sEB);
+            const uint32_t phi = tc::smem_u32(sPHI), t1 = tc::smem_u32(sT1), t2 = tc::smem_u32(sT2), sp = tc::smem_u32(sP);
+            bool ok = wait_bar(&bar[CF_TAB], ph[CF_TAB], ctl, a.err, 31);
+            for (int z = blockIdx.x, i = 0; z < a.Z && ok; z += gridDim.x, ++i) {
+                ok = false;
+                if (!wait_bar(&bar[CF_IN_FULL], ph[CF_IN_FULL], ctl, a.err, 32)) break;
+                if (i > 0 && !wait_bar(&bar[CF_TFREE], ph[CF_TFREE], ctl, a.err, 33)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)                 // P = Q K^T
+                    tc::mma_bf16(tb + colP, seq_kmaj(q, 128, 0, kk), seq_kmaj(k, 128, 0, kk), id_P, kk > 0);
+                tc::mma_commit(&bar[CF_ACC1]);
+                if (!wait_bar(&bar[CF_T1], ph[CF_T1], ctl, a.err, 34)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk)                      // X = P EB^T + Q W_K^T
+                    tc::mma_bf16(tb + colX, seq_kmaj(t1, 128, 0, kk), seq_kmaj(eb, R2, 0, kk), id_X, kk > 0);
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)
+                    tc::mma_bf16(tb + colX, seq_kmaj(q, 128, 0, kk), seq_kmaj(w, R2, 0, kk), id_X, 1u);
+                tc::mma_commit(&bar[CF_ACC2]);
+                tc::mma_commit(&bar[CF_IN_FREE]);
+                if (!wait_bar(&bar[CF_T2], ph[CF_T2], ctl, a.err, 35)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < R2 / 16; ++kk)                // s = Y PHI^T
+                    tc::mma_bf16(tb + colS, seq_kmaj(t2, 128, 0, kk), seq_kmaj(phi, S, 0, kk), id_S, kk > 0);
+                tc::mma_commit(&bar[CF_ACC3]);
+                if (!wait_bar(&bar[CF_SP], ph[CF_SP], ctl, a.err, 36)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < S / 16; ++kk)                 // U = p PHI
+                    tc::mma_bf16(tb + colU, seq_kmaj(sp, 128, 0, kk), seq_mnmaj(phi, S, 0, kk), id_U, kk > 0);
+                tc::mma_commit(&bar[CF_ACC4]);
+                if (!wait_bar(&bar[CF_A], ph[CF_A], ctl, a.err, 37)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < R2 / 16; ++kk)                // G = A' EB
+                    tc::mma_bf16(tb + colG, seq_kmaj(t1, 128, 0, kk), seq_mnmaj(eb, R2, 0, kk), id_G, kk > 0);
+                tc::mma_commit(&bar[CF_ACC5]);
+                ok = true;
+            }
+        }
+    } else {
+        // warpgroup wg drains columns [wg N/2, (wg+1) N/2) of each N-column result (N = S = 32: wg 0 only)
+        const int wg = warp >> 2, lane_base = (warp & 3) * 32, row = lane_base + lane;
+        uint32_t ph[CF_COUNT] = {};
+        auto arrive = [&](int b) {
+            tc::fence_proxy_async_smem();
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[b]);
+        };
+        auto esync = [&](int which) -> bool {
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[CF_ESYNC]);
+            return wait_bar(&bar[CF_ESYNC], ph[CF_ESYNC], ctl, a.err, which);
+        };
+        for (int z = blockIdx.x; z < a.Z; z += gridDim.x) {
+            const int bh = z / a.nch, c = z % a.nch, t = c * kC + row;
+            const bool live = t < a.L;
+            const float lse = live ? __ldg(a.lse + (size_t)bh * a.L + t) : 0.f;
+            const RotPh rp = chain_phases(a, c, row, wg * HX / 2);
+            // the previous chunk's stores must have read their tiles
+            if (threadIdx.x == 0) tc::bulk_wait_read0();
+            if (!esync(45)) break;
+            // P = tril(Q K^T)
+            if (!wait_bar(&bar[CF_ACC1], ph[CF_ACC1], ctl, a.err, 40)) break;
+            tc::tc_fence_after();
+            {
+                float v[64];
+                tc::tmem_ld<64>(tm_addr(tb, lane_base, colP + wg * 64), v);
+                chain_causal<64>(v, row, wg * 64);
+                st_tile_row<64>(sT1, row, wg * 64, v);
+            }
+            arrive(CF_T1);
+            // Y = rot+(X)
+            if (!wait_bar(&bar[CF_ACC2], ph[CF_ACC2], ctl, a.err, 41)) break;
+            tc::tc_fence_after();
+            {
+                float v[HX];
+                tc::tmem_ld<HX>(tm_addr(tb, lane_base, colX + wg * HX), v);
+                chain_rot<HX>(v, rp, 1.f, 1.f);
+                st_tile_row<HX>(sT2, row, wg * HX, v);
+            }
+            arrive(CF_T2);
+            // p = exp(scale s - lse), masked; slots beyond S are zero
+            if (!wait_bar(&bar[CF_ACC3], ph[CF_ACC3], ctl, a.err, 42)) break;
+            tc::tc_fence_after();
+            if (S >= 64 || wg == 0) {
+                float v[HS];
+                tc::tmem_ld<HS>(tm_addr(tb, lane_base, colS + wg * HS), v);
+#pragma unroll
+                for (int j = 0; j < HS; ++j) {
+                    const int jj = wg * HS + j;
+                    v[j] = (live && t >= sdelta[jj]) ? __expf(a.scale * v[j] - lse) : 0.f;
+                }
+                st_tile_row<HS>(sP, row, wg * HS, v);
+            } else {
+                float v[32];
+#pragma unroll
+                for (int j = 0; j < 32; ++j) v[j] = 0.f;
+                st_tile_row<32>(sP, row, 32, v);
+            }
+            tc::fence_proxy_async_smem();
+            if (!esync(46)) break;
+            if (threadIdx.x == 0) {
+                for (int jb = 0; jb < SP / 64; ++jb) tc::tma_store_3d(&tm_po, sP + jb * 128 * 128, jb * 64, 0, z);
+                tc::bulk_commit();
+            }
+            arrive(CF_SP);
+            // A' = rot-(p PHI)
+            if (!wait_bar(&bar[CF_ACC4], ph[CF_ACC4], ctl, a.err, 43)) break;
+            tc::tc_fence_after();
+            {
+                float v[HX];
+                tc::tmem_ld<HX>(tm_addr(tb, lane_base, colU + wg * HX), v);
+                chain_rot<HX>(v, rp, -1.f, 1.f);
+                st_tile_row<HX>(sT1, row, wg * HX, v);
+            }
+            tc::fence_proxy_async_smem();
+            if (!esync(47)) break;
+            if (threadIdx.x == 0) {
+                for (int rb = 0; rb < R2 / 64; ++rb) tc::tma_store_3d(&tm_ao, sT1 + rb * 128 * 128, rb * 64, 0, z);
+                tc::bulk_commit();
+            }
+            arrive(CF_A);
+            // G = tril(A' EB), staged in the Y tile (read by s long before)
+            if (!wait_bar(&bar[CF_ACC5], ph[CF_ACC5], ctl, a.err, 44)) break;
+            tc::tc_fence_after();
+            {
+                float v[64];
+                tc::tmem_ld<64>(tm_addr(tb, lane_base, colG + wg * 64), v);
+                chain_causal<64>(v, row, wg * 64);
+                st_tile_row<64>(sT2, row, wg * 64, v);
+            }
+            tc::fence_proxy_async_smem();
+            if (!esync(48)) break;
+            if (threadIdx.x == 0) {
+                for (int ub = 0; ub < 2; ++ub) tc::tma_store_3d(&tm_go, sT2 + ub * 128 * 128, ub * 64, 0, z);
+                tc::bulk_commit();
+            }
+            arrive(CF_TFREE);
+        }
+        if (threadIdx.x == 0) tc::bulk_wait0();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tb, 256);
+    }
+}
+
+// ---- k_chain_adj
+enum CaBar { CA_TAB, CA_IN_FULL, CA_VW_FREE, CA_KW_FULL, CA_KW_FREE, CA_ACC1, CA_ACC2, CA_ACC3, CA_ACC4, CA_ACC5,
+             CA_ACC6, CA_T1, CA_T2, CA_DS, CA_DX, CA_DP, CA_TFREE, CA_ESYNC, CA_COUNT };
+
+template <int R2, int S, int D>
+__global__ void __launch_bounds__(kSeqThreads, 1)
+    k_chain_adj(const __grid_constant__ CUtensorMap tm_do, const __grid_constant__ CUtensorMap tm_v,
+                const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_w,
+                const __grid_constant__ CUtensorMap tm_p, const __grid_constant__ CUtensorMap tm_eb,
+                const __grid_constant__ CUtensorMap tm_phi, const __grid_constant__ CUtensorMap tm_dxo,
+                const __grid_constant__ CUtensorMap tm_dpo, const __grid_constant__ CUtensorMap tm_dqo, ChainArgs a) {
+    constexpr int SP = S < 64 ? 64 : S, HX = R2 / 2, HS = S >= 64 ? S / 2 : S, HD = D / 2;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const ChainLayout lay = chain_layout(R2, S, SP, D);
+    uint8_t *sEB = sm + lay.eb, *sPHI = sm + lay.phi, *sDO = sm + lay.t0, *sVK = sm + lay.t1, *sWW = sm + lay.t2;
+    uint8_t *sT1 = sm + lay.t3, *sT2 = sm + lay.t4, *sP = sm + lay.sp;
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sm + lay.bars);
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + CA_COUNT);
+    Ctl *ctl = reinterpret_cast<Ctl *>(bar + CA_COUNT + 1);
+    float *sdl = reinterpret_cast<float *>(bar + CA_COUNT + 2);   // [128] rowsum(dO o)
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int colA = 0, colB = 128, colC = 256, colD = 384;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < CA_COUNT; ++i) {
+            const bool epi = i == CA_T1 || i == CA_T2 || i == CA_DS || i == CA_DX || i == CA_DP || i == CA_TFREE ||
+                             i == CA_ESYNC;
+            tc::mbar_init(&bar[i], i == CA_VW_FREE ? 1 + kSeqEpiWarps : (epi ? kSeqEpiWarps : 1));
+        }
+        ctl->abort = 0;
+        tc::fence_barrier_init();
+    }
+    if (warp == 9) { tc::tmem_alloc(tslot, 512); tc::tmem_relinquish(); }
+    tc::tc_fence_before();
+    __syncthreads();
+    tc::tc_fence_after();
+    const uint32_t tb = *tslot;
+
+    if (warp == 8) {
+        if (lane == 0) {
+            tc::mbar_arrive_expect_tx(&bar[CA_TAB], (uint32_t)(R2 * 256 + R2 * S * 2));
+            for (int ub = 0; ub < 2; ++ub) tc::tma_load_2d(sEB + ub * R2 * 128, &tm_eb, &bar[CA_TAB], ub * 64, 0);
+            for (int rb = 0; rb < R2 / 64; ++rb) tc::tma_load_2d(sPHI + rb * S * 128, &tm_phi, &bar[CA_TAB], rb * 64, 0);
+            uint32_t ph_kwf = 0, ph_vwf = 0;
+            for (int z = blockIdx.x, i = 0; z < a.Z && !ctl->abort; z += gridDim.x, ++i) {
+                const int bh = z / a.nch, c = z % a.nch;
+                if (i > 0 && !wait_bar(&bar[CA_KW_FREE], ph_kwf, ctl, a.err, 50)) break;
+                tc::mbar_arrive_expect_tx(&bar[CA_IN_FULL], (uint32_t)(2 * 256 * D + R2 * D * 2 + SP * 256));
+                for (int db = 0; db < D / 64; ++db) {
+                    tc::tma_load_3d(sDO + db * 128 * 128, &tm_do, &bar[CA_IN_FULL], db * 64, c * kC, bh);
+                    tc::tma_load_3d(sVK + db * 128 * 128, &tm_v, &bar[CA_IN_FULL], db * 64, c * kC, bh);
+                    tc::tma_load_3d(sWW + db * R2 * 128, &tm_w, &bar[CA_IN_FULL], db * 64, 0, 2 * z + 1);
+                }
+                for (int jb = 0; jb < SP / 64; ++jb)
+                    tc::tma_load_3d(sP + jb * 128 * 128, &tm_p, &bar[CA_IN_FULL], jb * 64, 0, z);
+                // K and W_K over V and W_V once dU has read them
+                if (!wait_bar(&bar[CA_VW_FREE], ph_vwf, ctl, a.err, 51)) break;
+                tc::mbar_arrive_expect_tx(&bar[CA_KW_FULL], (uint32_t)(256 * D + R2 * D * 2));
+                for (int db = 0; db < D / 64; ++db) {
+                    tc::tma_load_3d(sVK + db * 128 * 128, &tm_k, &bar[CA_KW_FULL], db * 64, c * kC, bh);
+                    tc::tma_load_3d(sWW + db * R2 * 128, &tm_w, &bar[CA_KW_FULL], db * 64, 0, 2 * z);
+                }
+            }
+        }
+    } else if (warp == 9) {
+        if (lane == 0) {
+            uint32_t ph[CA_COUNT] = {};
+            constexpr uint32_t id_G = tc::idesc_bf16(128, 128, false, false), id_U = tc::idesc_bf16(128, R2, false, false);
+            constexpr uint32_t id_S = tc::idesc_bf16(128, S, false, false), id_X = tc::idesc_bf16(128, R2, false, true);
+            constexpr uint32_t id_P = tc::idesc_bf16(128, 128, false, true), id_Q = tc::idesc_bf16(128, D, false, true);
+            const uint32_t dO = tc::smem_u32(sDO), vk = tc::smem_u32(sVK), ww = tc::smem_u32(sWW), eb = tc::smem_u32(sEB);
+            const uint32_t phi = tc::smem_u32(sPHI), t1 = tc::smem_u32(sT1), t2 = tc::smem_u32(sT2), sp = tc::smem_u32(sP);
+            bool ok = wait_bar(&bar[CA_TAB], ph[CA_TAB], ctl, a.err, 52);
+            for (int z = blockIdx.x, i = 0; z < a.Z && ok; z += gridDim.x, ++i) {
+                ok = false;
+                if (!wait_bar(&bar[CA_IN_FULL], ph[CA_IN_FULL], ctl, a.err, 53)) break;
+                if (i > 0 && !wait_bar(&bar[CA_TFREE], ph[CA_TFREE], ctl, a.err, 54)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)                 // dG = dO V^T
+                    tc::mma_bf16(tb + colA, seq_kmaj(dO, 128, 0, kk), seq_kmaj(vk, 128, 0, kk), id_G, kk > 0);
+                tc::mma_commit(&bar[CA_ACC1]);
+                if (!wait_bar(&bar[CA_T1], ph[CA_T1], ctl, a.err, 55)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk)                      // dU = dG EB^T + dO W_V^T
+                    tc::mma_bf16(tb + colB, seq_kmaj(t1, 128, 0, kk), seq_kmaj(eb, R2, 0, kk), id_U, kk > 0);
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk)
+                    tc::mma_bf16(tb + colB, seq_kmaj(dO, 128, 0, kk), seq_kmaj(ww, R2, 0, kk), id_U, 1u);
+                tc::mma_commit(&bar[CA_ACC2]);
+                tc::mma_commit(&bar[CA_VW_FREE]);
+                if (!wait_bar(&bar[CA_T2], ph[CA_T2], ctl, a.err, 56)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < R2 / 16; ++kk)                // dp = dU PHI^T
+                    tc::mma_bf16(tb + colC, seq_kmaj(t2, 128, 0, kk), seq_kmaj(phi, S, 0, kk), id_S, kk > 0);
+                tc::mma_commit(&bar[CA_ACC3]);
+                if (!wait_bar(&bar[CA_DS], ph[CA_DS], ctl, a.err, 57)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < S / 16; ++kk)                 // ds PHI
+                    tc::mma_bf16(tb + colA, seq_kmaj(sp, 128, 0, kk), seq_mnmaj(phi, S, 0, kk), id_X, kk > 0);
+                tc::mma_commit(&bar[CA_ACC4]);
+                if (!wait_bar(&bar[CA_DX], ph[CA_DX], ctl, a.err, 58)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < R2 / 16; ++kk)                // dP = dX EB
+                    tc::mma_bf16(tb + colB, seq_kmaj(t2, 128, 0, kk), seq_mnmaj(eb, R2, 0, kk), id_P, kk > 0);
+                tc::mma_commit(&bar[CA_ACC5]);
+                if (!wait_bar(&bar[CA_DP], ph[CA_DP], ctl, a.err, 59)) break;
+                if (!wait_bar(&bar[CA_KW_FULL], ph[CA_KW_FULL], ctl, a.err, 60)) break;
+                tc::tc_fence_after();
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk)                      // dQ = dP K + dX W_K
+                    tc::mma_bf16(tb + colD, seq_kmaj(t1, 128, 0, kk), seq_mnmaj(vk, 128, 0, kk), id_Q, kk > 0);
+#pragma unroll
+                for (int kk = 0; kk < R2 / 16; ++kk)
+                    tc::mma_bf16(tb + colD, seq_kmaj(t2, 128, 0, kk), seq_mnmaj(ww, R2, 0, kk), id_Q, 1u);
+                tc::mma_commit(&bar[CA_ACC6]);
+                tc::mma_commit(&bar[CA_KW_FREE]);
+                ok = true;
+            }
+        }
+    } else {
+        const int wg = warp >> 2, lane_base = (warp & 3) * 32, row = lane_base + lane;
+        uint32_t ph[CA_COUNT] = {};
+        auto arrive = [&](int b) {
+            tc::fence_proxy_async_smem();
+            tc::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[b]);
+        };
+        auto esync = [&](int which) -> bool {
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[CA_ESYNC]);
+            return wait_bar(&bar[CA_ESYNC], ph[CA_ESYNC], ctl, a.err, which);
+        };
+        constexpr int LPR = D / 8;            // lanes per row in the rowsum (8 bf16 each)
+        constexpr int RPI = 32 / LPR;         // rows per warp iteration
+        for (int z = blockIdx.x; z < a.Z; z += gridDim.x) {
+            const int bh = z / a.nch, c = z % a.nch;
+            const RotPh rp = chain_phases(a, c, row, wg * HX / 2);
+            if (threadIdx.x == 0) tc::bulk_wait_read0();
+            if (!esync(68)) break;
+            if (!wait_bar(&bar[CA_IN_FULL], ph[CA_IN_FULL], ctl, a.err, 61)) break;
+            // rowsum(dO o) of 16 rows per warp, loads of o coalesced (LPR lanes per row)
+            for (int r0 = warp * 16; r0 < warp * 16 + 16; r0 += RPI) {
+                const int r = r0 + lane / LPR, d0 = (lane % LPR) * 8, tt = c * kC + r;
+                float acc = 0.f;
+                if (tt < a.L) {
+                    const uint4 ov = __ldg(reinterpret_cast<const uint4 *>(a.o + ((size_t)bh * a.L + tt) * D + d0));
+                    const uint4 gv = *reinterpret_cast<const uint4 *>(sDO + (d0 >> 6) * 128 * 128 + tc::sw128_offset(r, d0 & 63));
+                    const uint32_t ow[4] = {ov.x, ov.y, ov.z, ov.w}, gw[4] = {gv.x, gv.y, gv.z, gv.w};
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&ow[q]));
+                        const float2 y = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&gw[q]));
+                        acc = fmaf(x.x, y.x, fmaf(x.y, y.y, acc));
+                    }
+                }
+#pragma unroll
+                for (int off = LPR / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+                if (lane % LPR == 0) sdl[r] = acc;
+            }
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(&bar[CA_VW_FREE]);
+            if (!esync(73)) break;
+            const float dl = sdl[row];
+            // dG
+            if (!wait_bar(&bar[CA_ACC1], ph[CA_ACC1], ctl, a.err, 62)) break;
+            tc::tc_fence_after();
+            {
+                float v[64];
+                tc::tmem_ld<64>(tm_addr(tb, lane_base, colA + wg * 64), v);
+                chain_causal<64>(v, row, wg * 64);
+                st_tile_row<64>(sT1, row, wg * 64, v);
+            }
+            arrive(CA_T1);
+            // dU
+            if (!wait_bar(&bar[CA_ACC2], ph[CA_ACC2], ctl, a.err, 63)) break;
+            tc::tc_fence_after();
+            {
+                float v[HX];
+                tc::tmem_ld<HX>(tm_addr(tb, lane_base, colB + wg * HX), v);
+                chain_rot<HX>(v, rp, 1.f, 1.f);
+                st_tile_row<HX>(sT2, row, wg * HX, v);
+            }
+            arrive(CA_T2);
+            // ds = p (dp - dl), over p in place
+            if (!wait_bar(&bar[CA_ACC3], ph[CA_ACC3], ctl, a.err, 64)) break;
+            tc::tc_fence_after();
+            if (S >= 64 || wg == 0) {
+                float v[HS];
+                tc::tmem_ld<HS>(tm_addr(tb, lane_base, colC + wg * HS), v);
+#pragma unroll
+                for (int g0 = 0; g0 < HS; g0 += 8) {
+                    const int col = wg * HS + g0;
+                    uint4 *pp = reinterpret_cast<uint4 *>(sP + (col >> 6) * 128 * 128 + tc::sw128_offset(row, col & 63));
+                    const uint4 pk = *pp;
+                    const uint32_t w[4] = {pk.x, pk.y, pk.z, pk.w};
+                    uint32_t o4[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float2 pf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[e]));
+                        o4[e] = tc::pack_bf16x2(pf.x * (v[g0 + 2 * e] - dl), pf.y * (v[g0 + 2 * e + 1] - dl));
+                    }
+                    *pp = make_uint4(o4[0], o4[1], o4[2], o4[3]);
+                }
+            }
+            arrive(CA_DS);
+            // dX = rot-(scale ds PHI)
+            if (!wait_bar(&bar[CA_ACC4], ph[CA_ACC4], ctl, a.err, 65)) break;
+            tc::tc_fence_after();
+            {
+                float v[HX];
+                tc::tmem_ld<HX>(tm_addr(tb, lane_base, colA + wg * HX), v);
+                chain_rot<HX>(v, rp, -1.f, a.scale);
+                st_tile_row<HX>(sT2, row, wg * HX, v);
+            }
+            tc::fence_proxy_async_smem();
+            if (!esync(69)) break;
+            if (threadIdx.x == 0) {
+                for (int rb = 0; rb < R2 / 64; ++rb) tc::tma_store_3d(&tm_dxo, sT2 + rb * 128 * 128, rb * 64, 0, z);
+                tc::bulk_commit();
+            }
+            arrive(CA_DX);
+            // dP = tril(dX EB)
+            if (!wait_bar(&bar[CA_ACC5], ph[CA_ACC5], ctl, a.err, 66)) break;
+            tc::tc_fence_after();
+            {
+                float v[64];
+                tc::tmem_ld<64>(tm_addr(tb, lane_base, colB + wg * 64), v);
+                chain_causal<64>(v, row, wg * 64);
+                st_tile_row<64>(sT1, row, wg * 64, v);
+            }
+            tc::fence_proxy_async_smem();
+            if (!esync(70)) break;
+            if (threadIdx.x == 0) {
+                for (int ub = 0; ub < 2; ++ub) tc::tma_store_3d(&tm_dpo, sT1 + ub * 128 * 128, ub * 64, 0, z);
+                tc::bulk_commit();
+            }
+            arrive(CA_DP);
+            // dQ, staged in the dX tile once dQ's MMA and dX's store have read it
+            if (!wait_bar(&bar[CA_ACC6], ph[CA_ACC6], ctl, a.err, 67)) break;
+            tc::tc_fence_after();
+            float vq[HD];
+            tc::tmem_ld<HD>(tm_addr(tb, lane_base, colD + wg * HD), vq);
+            if (threadIdx.x == 0) tc::bulk_wait_read0();
+            if (!esync(71)) break;
+            st_tile_row<HD>(sT2, row, wg * HD, vq);
+            tc::fence_proxy_async_smem();
+            if (!esync(72)) break;
+            if (threadIdx.x == 0) {
+                for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_dqo, sT2 + db * 128 * 128, db * 64, c * kC, bh);
+                tc::bulk_commit();
+            }
+            arrive(CA_TFREE);
+        }
+        if (threadIdx.x == 0) tc::bulk_wait0();
+    }
+    tc::tc_fence_before();
+    __syncthreads();
+    if (warp == 9) {
+        tc::tc_fence_after();
+        tc::tmem_dealloc(tb, 512);
+    }
+}
+
 // ------------------------------------------------------------------ host side
 
 struct BwdGeo {
@@ -875,6 +1463,47 @@ cudaError_t launch_adj_states(const BwdGeo &g, const CUtensorMap &mdx, const CUt
     return cudaErrorInvalidValue;
 }
 
+// The fused chains hold their tiles in shared memory for 2M <= 128 and S <= 64.
+bool chain_fits(const BwdGeo &g) { return g.R2 >= 64 && g.R2 <= 128 && g.S >= 32 && g.S <= 64; }
+
+template <int R2, int S, int D>
+cudaError_t launch_chains_t(const BwdGeo &g, const ChainArgs &ca, const CUtensorMap &mq, const CUtensorMap &mk,
+                            const CUtensorMap &mv, const CUtensorMap &mdo, const CUtensorMap &mw, const CUtensorMap &mp,
+                            const CUtensorMap &meb, const CUtensorMap &mphi, const CUtensorMap &ma,
+                            const CUtensorMap &mg, const CUtensorMap &mdx, const CUtensorMap &mdp,
+                            const CUtensorMap &mdq, cudaStream_t st) {
+    const ChainLayout lay = chain_layout(R2, S, S < 64 ? 64 : S, D);
+    const int smem = lay.total + 1024;
+    cudaError_t e = cudaFuncSetAttribute(k_chain_fwd<R2, S, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_chain_adj<R2, S, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+    int nblk = bwd_sm_count();
+    if (nblk > g.Z) nblk = g.Z;
+    {
+        ProfScope ps(BLA_K_BWD, st);
+        k_chain_fwd<R2, S, D><<<nblk, kSeqThreads, smem, st>>>(mq, mk, mw, meb, mphi, mp, ma, mg, ca);
+    }
+    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    {
+        ProfScope ps(BLA_K_BWD, st);
+        k_chain_adj<R2, S, D><<<nblk, kSeqThreads, smem, st>>>(mdo, mv, mk, mw, mp, meb, mphi, mdx, mdp, mdq, ca);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_chains(const BwdGeo &g, const ChainArgs &ca, const CUtensorMap &mq, const CUtensorMap &mk,
+                          const CUtensorMap &mv, const CUtensorMap &mdo, const CUtensorMap &mw, const CUtensorMap &mp,
+                          const CUtensorMap &meb, const CUtensorMap &mphi, const CUtensorMap &ma, const CUtensorMap &mg,
+                          const CUtensorMap &mdx, const CUtensorMap &mdp, const CUtensorMap &mdq, cudaStream_t st) {
+#define BLA_CHAIN(R, S_, D_)                                                                                          \
+    if (g.R2 == R && g.S == S_ && g.D == D_)                                                                          \
+        return launch_chains_t<R, S_, D_>(g, ca, mq, mk, mv, mdo, mw, mp, meb, mphi, ma, mg, mdx, mdp, mdq, st);
+    BLA_CHAIN(64, 32, 64) BLA_CHAIN(64, 32, 128) BLA_CHAIN(64, 64, 64) BLA_CHAIN(64, 64, 128)
+    BLA_CHAIN(128, 32, 64) BLA_CHAIN(128, 32, 128) BLA_CHAIN(128, 64, 64) BLA_CHAIN(128, 64, 128)
+#undef BLA_CHAIN
+    return cudaErrorInvalidValue;
+}
+
 }  // namespace
 
 const char *bwd_unsupported(const OpDims &d) {
@@ -945,6 +1574,20 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     sa.erel = t.erel; sa.wout = wb; sa.gout[0] = static_cast<bf16 *>(dk); sa.gout[1] = static_cast<bf16 *>(dv);
     sa.err = device_error_word();
     if ((e = launch_fwd_states(g, kK, vK, ebK128, sa, st)) != cudaSuccess) return e;
+    if (chain_fits(g)) {
+        // ---- 1-2. the chunk-local chains, fused
+        ChainArgs ca;
+        ca.BH = g.BH; ca.L = g.L; ca.nch = g.nch; ca.Z = Z; ca.M = g.M; ca.R2 = R2; ca.S = S; ca.SP = SP; ca.D = D;
+        ca.scale = d.scale; ca.erel = t.erel; ca.cphase = cphase; ca.lse = lse; ca.delta = t.delta;
+        ca.o = static_cast<const bf16 *>(o);
+        ca.err = sa.err;
+        CUtensorMap dqK;
+        if (!map_seq(&dqK, dq, g, D, true, kC)) return cudaErrorInvalidValue;
+        if ((e = launch_chains(g, ca, qK, kK, vK, dOK, wbK, pK, ebKR, phiK, AK, GK, dXK, dPK, dqK, st)) != cudaSuccess)
+            return e;
+        if ((e = launch_adj_states(g, dXK, AK, qK, dOK, dPK, GK, ebK128, sa, st)) != cudaSuccess) return e;
+        return cudaSuccess;
+    }
     Epi ep;
     // ---- 1. recompute the chunk's forward quantities
     ep = epi_base(EP_CAUSAL, Pb, OUT_Z, 0, kC, kC);                                   // P = tril(Q K^T)
