@@ -1024,8 +1024,11 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 }
 
 // ---- k_chain_adj
-enum CaBar { CA_TAB, CA_IN_FULL, CA_VW_FREE, CA_KW_FULL, CA_KW_FREE, CA_ACC1, CA_ACC2, CA_ACC3, CA_ACC4, CA_ACC5,
-             CA_ACC6, CA_T1, CA_T2, CA_DS, CA_DX, CA_DP, CA_TFREE, CA_ESYNC, CA_COUNT };
+// Loads: dO and p of chunk c+1 go in as soon as chunk c has consumed its own (dU and rowsum(dO o);
+// ds PHI), V and W_V once dQ is done; K and W_K replace V and W_V after dU.
+enum CaBar { CA_TAB, CA_DO_FULL, CA_P_FULL, CA_VW_FULL, CA_VW_FREE, CA_SP_FREE, CA_KW_FULL, CA_KW_FREE, CA_ACC1,
+             CA_ACC2, CA_ACC3, CA_ACC4, CA_ACC5, CA_ACC6, CA_T1, CA_T2, CA_DS, CA_DX, CA_DP, CA_TFREE, CA_ESYNC,
+             CA_COUNT };
 
 template <int R2, int S, int D>
 __global__ void __launch_bounds__(kSeqThreads, 1)
@@ -1067,25 +1070,49 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
             tc::mbar_arrive_expect_tx(&bar[CA_TAB], (uint32_t)(R2 * 256 + R2 * S * 2));
             for (int ub = 0; ub < 2; ++ub) tc::tma_load_2d(sEB + ub * R2 * 128, &tm_eb, &bar[CA_TAB], ub * 64, 0);
             for (int rb = 0; rb < R2 / 64; ++rb) tc::tma_load_2d(sPHI + rb * S * 128, &tm_phi, &bar[CA_TAB], rb * 64, 0);
-            uint32_t ph_kwf = 0, ph_vwf = 0;
-            for (int z = blockIdx.x, i = 0; z < a.Z && !ctl->abort; z += gridDim.x, ++i) {
+            uint32_t ph_kwf = 0, ph_vwf = 0, ph_spf = 0;
+            auto load_do = [&](int z) {
                 const int bh = z / a.nch, c = z % a.nch;
-                if (i > 0 && !wait_bar(&bar[CA_KW_FREE], ph_kwf, ctl, a.err, 50)) break;
-                tc::mbar_arrive_expect_tx(&bar[CA_IN_FULL], (uint32_t)(2 * 256 * D + R2 * D * 2 + SP * 256));
-                for (int db = 0; db < D / 64; ++db) {
-                    tc::tma_load_3d(sDO + db * 128 * 128, &tm_do, &bar[CA_IN_FULL], db * 64, c * kC, bh);
-                    tc::tma_load_3d(sVK + db * 128 * 128, &tm_v, &bar[CA_IN_FULL], db * 64, c * kC, bh);
-                    tc::tma_load_3d(sWW + db * R2 * 128, &tm_w, &bar[CA_IN_FULL], db * 64, 0, 2 * z + 1);
-                }
+                tc::mbar_arrive_expect_tx(&bar[CA_DO_FULL], (uint32_t)(256 * D));
+                for (int db = 0; db < D / 64; ++db)
+                    tc::tma_load_3d(sDO + db * 128 * 128, &tm_do, &bar[CA_DO_FULL], db * 64, c * kC, bh);
+            };
+            auto load_p = [&](int z) {
+                tc::mbar_arrive_expect_tx(&bar[CA_P_FULL], (uint32_t)(SP * 256));
                 for (int jb = 0; jb < SP / 64; ++jb)
-                    tc::tma_load_3d(sP + jb * 128 * 128, &tm_p, &bar[CA_IN_FULL], jb * 64, 0, z);
-                // K and W_K over V and W_V once dU has read them
-                if (!wait_bar(&bar[CA_VW_FREE], ph_vwf, ctl, a.err, 51)) break;
+                    tc::tma_load_3d(sP + jb * 128 * 128, &tm_p, &bar[CA_P_FULL], jb * 64, 0, z);
+            };
+            auto load_vw = [&](int z) {
+                const int bh = z / a.nch, c = z % a.nch;
+                tc::mbar_arrive_expect_tx(&bar[CA_VW_FULL], (uint32_t)(256 * D + R2 * D * 2));
+                for (int db = 0; db < D / 64; ++db) {
+                    tc::tma_load_3d(sVK + db * 128 * 128, &tm_v, &bar[CA_VW_FULL], db * 64, c * kC, bh);
+                    tc::tma_load_3d(sWW + db * R2 * 128, &tm_w, &bar[CA_VW_FULL], db * 64, 0, 2 * z + 1);
+                }
+            };
+            auto load_kw = [&](int z) {
+                const int bh = z / a.nch, c = z % a.nch;
                 tc::mbar_arrive_expect_tx(&bar[CA_KW_FULL], (uint32_t)(256 * D + R2 * D * 2));
                 for (int db = 0; db < D / 64; ++db) {
                     tc::tma_load_3d(sVK + db * 128 * 128, &tm_k, &bar[CA_KW_FULL], db * 64, c * kC, bh);
                     tc::tma_load_3d(sWW + db * R2 * 128, &tm_w, &bar[CA_KW_FULL], db * 64, 0, 2 * z);
                 }
+            };
+            const int z0 = blockIdx.x;
+            if (z0 < a.Z) { load_do(z0); load_p(z0); load_vw(z0); }
+            for (int z = z0; z < a.Z && !ctl->abort; z += gridDim.x) {
+                const int zn = z + (int)gridDim.x;
+                // chunk z has read V, W_V and dO: its K, W_K, and the next chunk's dO
+                if (!wait_bar(&bar[CA_VW_FREE], ph_vwf, ctl, a.err, 51)) break;
+                load_kw(z);
+                if (zn < a.Z) load_do(zn);
+                if (zn >= a.Z) break;
+                // chunk z's ds has been read: the next chunk's p
+                if (!wait_bar(&bar[CA_SP_FREE], ph_spf, ctl, a.err, 52)) break;
+                load_p(zn);
+                // chunk z's dQ is done: the next chunk's V and W_V
+                if (!wait_bar(&bar[CA_KW_FREE], ph_kwf, ctl, a.err, 50)) break;
+                load_vw(zn);
             }
         }
     } else if (warp == 9) {
@@ -1099,7 +1126,8 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
             bool ok = wait_bar(&bar[CA_TAB], ph[CA_TAB], ctl, a.err, 52);
             for (int z = blockIdx.x, i = 0; z < a.Z && ok; z += gridDim.x, ++i) {
                 ok = false;
-                if (!wait_bar(&bar[CA_IN_FULL], ph[CA_IN_FULL], ctl, a.err, 53)) break;
+                if (!wait_bar(&bar[CA_DO_FULL], ph[CA_DO_FULL], ctl, a.err, 53)) break;
+                if (!wait_bar(&bar[CA_VW_FULL], ph[CA_VW_FULL], ctl, a.err, 74)) break;
                 if (i > 0 && !wait_bar(&bar[CA_TFREE], ph[CA_TFREE], ctl, a.err, 54)) break;
                 tc::tc_fence_after();
 #pragma unroll
@@ -1128,6 +1156,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
                 for (int kk = 0; kk < S / 16; ++kk)                 // ds PHI
                     tc::mma_bf16(tb + colA, seq_kmaj(sp, 128, 0, kk), seq_mnmaj(phi, S, 0, kk), id_X, kk > 0);
                 tc::mma_commit(&bar[CA_ACC4]);
+                tc::mma_commit(&bar[CA_SP_FREE]);
                 if (!wait_bar(&bar[CA_DX], ph[CA_DX], ctl, a.err, 58)) break;
                 tc::tc_fence_after();
 #pragma unroll
@@ -1169,7 +1198,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
             const RotPh rp = chain_phases(a, c, row, wg * HX / 2);
             if (threadIdx.x == 0) tc::bulk_wait_read0();
             if (!esync(68)) break;
-            if (!wait_bar(&bar[CA_IN_FULL], ph[CA_IN_FULL], ctl, a.err, 61)) break;
+            if (!wait_bar(&bar[CA_DO_FULL], ph[CA_DO_FULL], ctl, a.err, 61)) break;
             // rowsum(dO o) of 16 rows per warp, loads of o coalesced (LPR lanes per row)
             for (int r0 = warp * 16; r0 < warp * 16 + 16; r0 += RPI) {
                 const int r = r0 + lane / LPR, d0 = (lane % LPR) * 8, tt = c * kC + r;
@@ -1214,6 +1243,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
             }
             arrive(CA_T2);
             // ds = p (dp - dl), over p in place
+            if (!wait_bar(&bar[CA_P_FULL], ph[CA_P_FULL], ctl, a.err, 75)) break;
             if (!wait_bar(&bar[CA_ACC3], ph[CA_ACC3], ctl, a.err, 64)) break;
             tc::tc_fence_after();
             if (S >= 64 || wg == 0) {
