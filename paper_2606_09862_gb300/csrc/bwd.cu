@@ -446,6 +446,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
+    tc::pdl_wait();      // the tables
 
     if (warp == 8) {
         if (lane == 0 && nupd > 0) {
@@ -578,6 +579,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
+    tc::pdl_wait();      // the chains' outputs
 
     if (warp == 8) {
         if (lane == 0) {
@@ -839,8 +841,9 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
         ctl->abort = 0;
         tc::fence_barrier_init();
     }
-    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
     if (warp == 9) { tc::tmem_alloc(tslot, 256); tc::tmem_relinquish(); }
+    tc::pdl_wait();      // the chunk states and the tables
+    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
@@ -1064,6 +1067,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
+    tc::pdl_wait();      // p and the chunk states
 
     if (warp == 8) {
         if (lane == 0) {
@@ -1451,8 +1455,7 @@ cudaError_t launch_fwd_states_t(const BwdGeo &g, const CUtensorMap &mk, const CU
     cudaError_t e = cudaFuncSetAttribute(k_fwd_states<D, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_BWD, st);
-    k_fwd_states<D, NB><<<g.BH * 2, kSeqThreads, smem, st>>>(mk, mv, meb, sa);
-    return cudaGetLastError();
+    return launch_pdl(k_fwd_states<D, NB>, dim3(g.BH * 2), dim3(kSeqThreads), (size_t)smem, st, mk, mv, meb, sa);
 }
 
 cudaError_t launch_fwd_states(const BwdGeo &g, const CUtensorMap &mk, const CUtensorMap &mv, const CUtensorMap &meb,
@@ -1478,8 +1481,8 @@ cudaError_t launch_adj_states_t(const BwdGeo &g, const CUtensorMap &mdx, const C
     cudaError_t e = cudaFuncSetAttribute(k_adj_states<D, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_BWD, st);
-    k_adj_states<D, NB><<<g.BH * 2, kSeqThreads, smem, st>>>(mdx, map_, mq, mdo, mdp, mg, meb, sa, stages);
-    return cudaGetLastError();
+    return launch_pdl(k_adj_states<D, NB>, dim3(g.BH * 2), dim3(kSeqThreads), (size_t)smem, st, mdx, map_, mq, mdo,
+                      mdp, mg, meb, sa, stages);
 }
 
 cudaError_t launch_adj_states(const BwdGeo &g, const CUtensorMap &mdx, const CUtensorMap &map_, const CUtensorMap &mq,
@@ -1511,14 +1514,16 @@ cudaError_t launch_chains_t(const BwdGeo &g, const ChainArgs &ca, const CUtensor
     if (nblk > g.Z) nblk = g.Z;
     {
         ProfScope ps(BLA_K_BWD, st);
-        k_chain_fwd<R2, S, D><<<nblk, kSeqThreads, smem, st>>>(mq, mk, mw, meb, mphi, mp, ma, mg, ca);
+        e = launch_pdl(k_chain_fwd<R2, S, D>, dim3(nblk), dim3(kSeqThreads), (size_t)smem, st, mq, mk, mw, meb, mphi,
+                       mp, ma, mg, ca);
     }
-    if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    if (e != cudaSuccess) return e;
     {
         ProfScope ps(BLA_K_BWD, st);
-        k_chain_adj<R2, S, D><<<nblk, kSeqThreads, smem, st>>>(mdo, mv, mk, mw, mp, meb, mphi, mdx, mdp, mdq, ca);
+        e = launch_pdl(k_chain_adj<R2, S, D>, dim3(nblk), dim3(kSeqThreads), (size_t)smem, st, mdo, mv, mk, mw, mp,
+                       meb, mphi, mdx, mdp, mdq, ca);
     }
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_chains(const BwdGeo &g, const ChainArgs &ca, const CUtensorMap &mq, const CUtensorMap &mk,

@@ -85,6 +85,25 @@ struct ProfScope {
     int slot;
 };
 
+// Launch `kernel` so that it may start while the previous kernel in the stream finishes
+// (programmatic stream serialization): the kernel must call tc::pdl_wait() before it reads
+// anything the previous kernels wrote, and write nothing before that.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                       Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<Args &&>(args)...);
+}
+
 // Launchers of the individual kernels (defined in their .cu files).
 cudaError_t launch_forward_f32(const OpDims &d, int C, const Tables &t, const float *q, const float *k,
                                const float *v, float *o, float *lse, float *state_out, float *scratch,

@@ -500,6 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
+    tc::pdl_wait();      // the tables
     const int steps = g.cps * 2;          // half-chunks in the segment
     const int t_seg = seg * g.Lseg;
 
@@ -563,6 +564,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 // ================================================================== segment scan
 // W_in(0) = 0; W_in(g+1) = e^{i m w Lseg} W_in(g) + delta(g).  One thread per (head, K|V, mode, d).
 __global__ void k_scan(Args a) {
+    tc::pdl_wait();      // the segment deltas
     const Geo &g = a.g;
     const long long total = (long long)g.BH * 2 * g.M * g.D;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
@@ -675,8 +677,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         ctl->bar0 = bar;
         tc::fence_barrier_init();
     }
-    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
     if (warp == 9) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
+    // the tables and the entering states come from the kernels before this one
+    tc::pdl_wait();
+    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
@@ -1157,6 +1161,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     __syncthreads();
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
+    tc::pdl_wait();      // p from the K pass, and the tables and states before it
 
     if (warp >= 8) {
         if (warp == 8) {
@@ -1503,7 +1508,8 @@ static cudaError_t launch_kpass_n(int smem, int nblk, cudaStream_t st, const CUt
     if (e != cudaSuccess) return e;
     if ((e = check_register_split((const void *)k_kpass<D, RH, S, NH>)) != cudaSuccess) return e;
     ProfScope ps(BLA_K_KPASS, st);
-    k_kpass<D, RH, S, NH><<<nblk, kPassThreads, smem, st>>>(tq, tk, teb, tphi, tp, a);
+    e = launch_pdl(k_kpass<D, RH, S, NH>, dim3(nblk), dim3(kPassThreads), smem, st, tq, tk, teb, tphi, tp, a);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
@@ -1545,7 +1551,8 @@ static cudaError_t launch_vpass_n(int smem, int nblk, cudaStream_t st, const CUt
     cudaError_t e = cudaFuncSetAttribute(k_vpass<D, RH, NH>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_VPASS, st);
-    k_vpass<D, RH, NH><<<nblk, kPassThreads, smem, st>>>(tp, tv, teb, tphi, to, a);
+    e = launch_pdl(k_vpass<D, RH, NH>, dim3(nblk), dim3(kPassThreads), smem, st, tp, tv, teb, tphi, to, a);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 
@@ -1637,7 +1644,8 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
             return e;
         {
             ProfScope ps(BLA_K_PREPASS, st);
-            k_prepass<<<nblk, kThreads, smem, st>>>(tk, tv, tf, a);
+            if ((e = launch_pdl(k_prepass, dim3(nblk), dim3(kThreads), (size_t)smem, st, tk, tv, tf, a)) != cudaSuccess)
+                return e;
         }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         long long tot = (long long)g.BH * 2 * g.M * g.D;
@@ -1645,7 +1653,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
         if (blocks > 4096) blocks = 4096;
         {
             ProfScope ps(BLA_K_SCAN, st);
-            k_scan<<<blocks, 256, 0, st>>>(a);
+            if ((e = launch_pdl(k_scan, dim3(blocks), dim3(256), 0, st, a)) != cudaSuccess) return e;
         }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }

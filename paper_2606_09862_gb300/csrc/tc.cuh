@@ -123,6 +123,13 @@ __device__ __forceinline__ void named_bar(int id, int count) {
     asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Programmatic dependent launch: block until the grids this one depends on have completed and
+// their memory is visible (returns at once for a kernel launched without the attribute).  No
+// kernel here triggers its dependents early: each CTA's exit does, so a dependent CTA takes the SM
+// a finished CTA leaves and runs its prologue while the rest of the grid completes (measured: an
+// early trigger let dependents crowd the SMs and slowed the long prefill by 5 %).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // Make generic-proxy shared-memory writes visible to the async proxy (TMA, tcgen05.mma).
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
