@@ -86,7 +86,7 @@ typedef struct {
 typedef enum { BLA_PHASE_LAG = 0, BLA_PHASE_ABSOLUTE = 1 } bla_phase_mode;
 
 /* Which entry point a workspace size is asked for. */
-typedef enum { BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2 } bla_ws_kind;
+typedef enum { BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2, BLA_WS_FORWARD_HOST = 3 } bla_ws_kind;
 
 /*
  * Bytes of device workspace the entry point `which` (a bla_ws_kind) needs for
@@ -114,6 +114,26 @@ size_t bla_workspace_bytes(const bla_params *p, int which);
 bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k, const void *v,
                                void *o, float *lse, float *state_out,
                                void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * bla_forward_chunked on tensors in HOST memory (no paper counterpart: a serving convenience).
+ * q, k, v are read from and o is written to host memory, in the layout of bla_forward_chunked.
+ * The B*H heads are independent, so they are processed in groups: each group's host-to-device
+ * copies, its forward and its device-to-host copy run on separate streams (two owned by the
+ * library, created on first use on each device), and copies overlap the other groups' compute.
+ *   - The host buffers should be page-locked (cudaHostAlloc or cudaHostRegister); pageable
+ *     memory gives the same results without the overlap.
+ *   - workspace: device scratch of >= bla_workspace_bytes(p, BLA_WS_FORWARD_HOST) bytes; it holds
+ *     the device copies of q, k, v and o and the forward's own workspace.
+ *   - The call returns once everything is enqueued.  o is complete on the host once `stream` has
+ *     been synchronised (the stream waits for the last copy); the host buffers must stay valid and
+ *     untouched until then.  Calls must be ordered by the caller (they share the library's streams
+ *     and the caller's workspace).
+ * Results equal bla_forward_chunked's to rounding (the heads of a group are one launch, so the
+ * sequence segmentation may differ).  lse and the final state are not returned.
+ */
+bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const void *k, const void *v, void *o,
+                                    void *workspace, size_t ws_bytes, void *stream);
 
 /*
  * One single-token decode step for B*H independent sequences (Alg. 2 loop body).

@@ -16,13 +16,13 @@ LIB_PATH = os.path.join(_HERE, "libbla_gb300.so")
 
 BLA_OK, BLA_ERR_INVALID, BLA_ERR_UNSUPPORTED, BLA_ERR_CUDA, BLA_ERR_TIMEOUT = range(5)
 BLA_F32, BLA_BF16 = 0, 1
-BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE = 0, 1, 2
+BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE, BLA_WS_FORWARD_HOST = 0, 1, 2, 3
 BLA_PHASE_LAG, BLA_PHASE_ABSOLUTE = 0, 1
 PHASE_MODES = {"lag": BLA_PHASE_LAG, "absolute": BLA_PHASE_ABSOLUTE}
 
 EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
             "bla_device_error", "bla_status_string", "bla_last_error_string", "bla_kernel_launches",
-            "bla_profile_enable", "bla_profile_collect", "bla_decode_step_noalloc")
+            "bla_profile_enable", "bla_profile_collect", "bla_decode_step_noalloc", "bla_forward_chunked_host")
 
 # bla_kernel_id
 KERNELS = ("tables", "tables_bf16", "prepass", "scan", "kpass", "vpass", "fwd_f32", "decode", "bwd")
@@ -59,6 +59,8 @@ def load():
     lib.bla_workspace_bytes.argtypes = [P, ctypes.c_int]
     lib.bla_forward_chunked.restype = ctypes.c_int
     lib.bla_forward_chunked.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_forward_chunked_host.restype = ctypes.c_int
+    lib.bla_forward_chunked_host.argtypes = [P, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_decode_step.restype = ctypes.c_int
     lib.bla_decode_step.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_decode_step_noalloc.restype = ctypes.c_int
@@ -224,33 +226,48 @@ def bla_profile_collect():
     return {KERNELS[i]: (float(ms[i]), int(cnt[i])) for i in range(n) if cnt[i] > 0}
 
 
+def _need_host(*ts):
+    for t in ts:
+        if t.is_cuda or not t.is_contiguous():
+            raise BlaError(BLA_ERR_INVALID, "host tensors must be contiguous CPU tensors")
+
+
+def bla_forward_chunked_host(q, k, v, M, S, window, omega=0.0, chunk=0, scale=0.0, out=None, workspace=None,
+                             stream=None, phase_mode="lag", device=None):
+    """bla_forward_chunked_host: q, k, v and the returned o are CPU tensors (page-locked for the
+    copies to overlap the compute).  `workspace` is a CUDA uint8 tensor of at least
+    bla_workspace_bytes(params, BLA_WS_FORWARD_HOST) bytes (allocated if None).  o is complete once
+    `stream` (default: the current stream) has been synchronised."""
+    _need_host(q, k, v)
+    B, H, L, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, L, dk, dv, M, S, window, omega, chunk, scale, q.dtype, phase_mode)
+    o = out if out is not None else torch.empty((B, H, L, dv), dtype=q.dtype, pin_memory=True)
+    _need_host(o)
+    dev = torch.device("cuda") if device is None else device
+    ws, n = _workspace(p, BLA_WS_FORWARD_HOST, dev, workspace)
+    _check(load().bla_forward_chunked_host(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(ws), n,
+                                           _stream(stream)))
+    return o
+
+
 def forward_from_host(q_host, k_host, v_host, M, S, window, omega=0.0, scale=0.0, device=None, bufs=None,
                       out_host=None, stream=None, phase_mode="lag"):
-    """bla_forward_chunked on host tensors: copies q, k, v (pinned for asynchronous copies) to the
-    device, runs the chunked forward and copies o back into `out_host` (allocated if None).
-    `bufs` (dict) caches the device buffers and workspace between calls.  Returns out_host; the
-    copy back is asynchronous on the current stream."""
+    """bla_forward_chunked_host with the workspace (and the output, if `out_host` is None) cached in
+    the dict `bufs` between calls.  Returns the host output; it is complete once the stream has
+    been synchronised."""
     dev = torch.device("cuda") if device is None else device
     bufs = {} if bufs is None else bufs
-    for name, h in (("q", q_host), ("k", k_host), ("v", v_host)):
-        t = bufs.get(name)
-        if t is None or t.shape != h.shape or t.dtype != h.dtype:
-            bufs[name] = torch.empty(h.shape, dtype=h.dtype, device=dev)
-        bufs[name].copy_(h, non_blocking=True)
-    B, H, L, _ = q_host.shape
+    B, H, L, dk = q_host.shape
     dv = v_host.shape[-1]
-    if "o" not in bufs or bufs["o"].shape != (B, H, L, dv):
-        bufs["o"] = torch.empty((B, H, L, dv), dtype=q_host.dtype, device=dev)
-        bufs["lse"] = torch.empty((B, H, L), dtype=torch.float32, device=dev)
-    p = make_params(B, H, L, q_host.shape[-1], dv, M, S, window, omega, 0, scale, q_host.dtype, phase_mode)
-    if "ws" not in bufs:
-        n = bla_workspace_bytes(p, BLA_WS_FORWARD)
-        bufs["ws"] = torch.empty(max(n, 1), dtype=torch.uint8, device=dev)
-    ws = bufs["ws"]
-    _check(load().bla_forward_chunked(ctypes.byref(p), _ptr(bufs["q"]), _ptr(bufs["k"]), _ptr(bufs["v"]),
-                                      _ptr(bufs["o"]), _ptr(bufs["lse"]), None, _ptr(ws), ws.numel(),
-                                      _stream(stream)))
+    key = (B, H, L, dk, dv, M, S, float(window), q_host.dtype, phase_mode)
+    if bufs.get("key") != key:
+        p = make_params(B, H, L, dk, dv, M, S, window, omega, 0, scale, q_host.dtype, phase_mode)
+        bufs["ws"] = torch.empty(max(bla_workspace_bytes(p, BLA_WS_FORWARD_HOST), 1), dtype=torch.uint8, device=dev)
+        bufs["key"] = key
     if out_host is None:
-        out_host = torch.empty(bufs["o"].shape, dtype=bufs["o"].dtype, pin_memory=True)
-    out_host.copy_(bufs["o"], non_blocking=True)
-    return out_host
+        if "o" not in bufs or bufs["o"].shape != (B, H, L, dv) or bufs["o"].dtype != q_host.dtype:
+            bufs["o"] = torch.empty((B, H, L, dv), dtype=q_host.dtype, pin_memory=True)
+        out_host = bufs["o"]
+    return bla_forward_chunked_host(q_host, k_host, v_host, M, S, window, omega, 0, scale, out=out_host,
+                                    workspace=bufs["ws"], stream=stream, phase_mode=phase_mode, device=dev)

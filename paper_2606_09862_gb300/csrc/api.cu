@@ -149,6 +149,100 @@ size_t ws_forward(const bla_params *p, const OpDims &d) {
 
 size_t ws_decode(const OpDims &d) { return tables_bytes(d, 0); }
 
+// ---- host-buffer forward: head groups pipelined over copy streams
+constexpr int kHostGroupsMax = 8;
+constexpr size_t kHostGroupBytes = 64ull << 20;   // split only when a group still moves >= 64 MB
+
+struct HostPipe {
+    cudaStream_t h2d = nullptr, d2h = nullptr;
+    cudaEvent_t start = nullptr, in[kHostGroupsMax] = {}, out[kHostGroupsMax] = {}, done = nullptr;
+    bool ready = false;
+};
+
+// The library's copy streams and events of the current device (created on first use).
+cudaError_t host_pipe(HostPipe **pp) {
+    static HostPipe pipes[64];
+    static std::mutex mu;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(mu);
+    HostPipe &h = pipes[dev];
+    if (!h.ready) {
+        if ((e = cudaStreamCreateWithFlags(&h.h2d, cudaStreamNonBlocking)) != cudaSuccess) return e;
+        if ((e = cudaStreamCreateWithFlags(&h.d2h, cudaStreamNonBlocking)) != cudaSuccess) return e;
+        if ((e = cudaEventCreateWithFlags(&h.start, cudaEventDisableTiming)) != cudaSuccess) return e;
+        if ((e = cudaEventCreateWithFlags(&h.done, cudaEventDisableTiming)) != cudaSuccess) return e;
+        for (int i = 0; i < kHostGroupsMax; ++i) {
+            if ((e = cudaEventCreateWithFlags(&h.in[i], cudaEventDisableTiming)) != cudaSuccess) return e;
+            if ((e = cudaEventCreateWithFlags(&h.out[i], cudaEventDisableTiming)) != cudaSuccess) return e;
+        }
+        h.ready = true;
+    }
+    *pp = &h;
+    return cudaSuccess;
+}
+
+// Head groups of the host-buffer forward: heads [first(g), first(g+1)).
+int host_groups(const OpDims &d) {
+    const long long BH = (long long)d.B * d.H;
+    const size_t elem = d.dtype == BLA_BF16 ? 2 : 4;
+    const size_t total = (size_t)BH * d.L * (2 * d.dk + 2 * d.dv) * elem;
+    long long n = (long long)(total / kHostGroupBytes);
+    if (n > kHostGroupsMax) n = kHostGroupsMax;
+    if (n > BH) n = BH;
+    return n < 1 ? 1 : (int)n;
+}
+long long host_group_first(const OpDims &d, int ngroups, int g) { return (long long)d.B * d.H * g / ngroups; }
+size_t host_elem(const OpDims &d) { return d.dtype == BLA_BF16 ? 2 : 4; }
+
+// Dimensions of one group's launch: its heads as one batch.
+OpDims host_group_dims(const OpDims &d, long long heads) {
+    OpDims g = d;
+    g.B = 1;
+    g.H = (int)heads;
+    return g;
+}
+
+// Workspace of the host-buffer forward: the largest group's forward workspace, then the device
+// copies of q, k, v and o (each 256-aligned).
+size_t ws_forward_host_parts(const bla_params *p, const OpDims &d, size_t *fw) {
+    const int ng = host_groups(d);
+    size_t f = 0;
+    for (int g = 0; g < ng; ++g) {
+        const long long nh = host_group_first(d, ng, g + 1) - host_group_first(d, ng, g);
+        const size_t w = ws_forward(p, host_group_dims(d, nh));
+        if (w > f) f = w;
+    }
+    *fw = align_up(f, 256);
+    const size_t BH = (size_t)d.B * d.H, e = host_elem(d);
+    return *fw + 2 * align_up(BH * d.L * d.dk * e, 256) + 2 * align_up(BH * d.L * d.dv * e, 256);
+}
+size_t ws_forward_host(const bla_params *p, const OpDims &d) {
+    size_t fw;
+    return ws_forward_host_parts(p, d, &fw);
+}
+
+// The forward of a validated problem on device buffers (bla_forward_chunked after its checks).
+bla_status forward_device(const bla_params *p, const OpDims &d, const void *q, const void *k, const void *v, void *o,
+                          float *lse, float *state_out, void *workspace, cudaStream_t st) {
+    if (d.dtype == BLA_F32) {
+        const int C = f32_chunk(p, d);
+        Tables t;
+        char *rest = tables_carve(d, C, static_cast<char *>(workspace), &t);
+        cudaError_t e = tables_build(d, t, st);
+        if (e != cudaSuccess) return cuda_fail(e, "table build");
+        e = launch_forward_f32(d, C, t, (const float *)q, (const float *)k, (const float *)v, (float *)o, lse,
+                               state_out, reinterpret_cast<float *>(rest), st);
+        if (e != cudaSuccess) return cuda_fail(e, "fp32 forward launch");
+        return BLA_OK;
+    }
+    cudaError_t e = fwd_bf16_run(d, q, k, v, o, lse, state_out, workspace, st);
+    if (e != cudaSuccess) return cuda_fail(e, "bf16 forward");
+    return BLA_OK;
+}
+
 }  // namespace
 }  // namespace bla
 
@@ -175,6 +269,7 @@ size_t bla_workspace_bytes(const bla_params *p, int which) {
     switch (which) {
     case BLA_WS_FORWARD: return ws_forward(p, d);
     case BLA_WS_DECODE: return ws_decode(d);
+    case BLA_WS_FORWARD_HOST: return ws_forward_host(p, d);
     case BLA_WS_BACKWARD: return bwd_workspace_bytes(d);
     default: return 0;
     }
@@ -190,26 +285,60 @@ bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(lse) ||
         !aligned16(state_out))
         return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
-    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-    if (d.dtype == BLA_F32) {
-        const int C = f32_chunk(p, d);
-        size_t need = ws_forward(p, d);
-        if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
-        Tables t;
-        char *rest = tables_carve(d, C, static_cast<char *>(workspace), &t);
-        cudaError_t e = tables_build(d, t, st);
-        if (e != cudaSuccess) return cuda_fail(e, "table build");
-        e = launch_forward_f32(d, C, t, (const float *)q, (const float *)k, (const float *)v, (float *)o, lse,
-                               state_out, reinterpret_cast<float *>(rest), st);
-        if (e != cudaSuccess) return cuda_fail(e, "fp32 forward launch");
-        return BLA_OK;
+    if (d.dtype == BLA_BF16) {
+        const char *why = fwd_bf16_unsupported(d);
+        if (why) return fail(BLA_ERR_UNSUPPORTED, "bf16 forward: %s", why);
     }
-    const char *why = fwd_bf16_unsupported(d);
-    if (why) return fail(BLA_ERR_UNSUPPORTED, "bf16 forward: %s", why);
-    size_t need = fwd_bf16_workspace_bytes(d);
-    if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
-    cudaError_t e = fwd_bf16_run(d, q, k, v, o, lse, state_out, workspace, st);
-    if (e != cudaSuccess) return cuda_fail(e, "bf16 forward");
+    if ((s = check_ws(workspace, ws_bytes, ws_forward(p, d))) != BLA_OK) return s;
+    return forward_device(p, d, q, k, v, o, lse, state_out, workspace, reinterpret_cast<cudaStream_t>(stream));
+}
+
+bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const void *k, const void *v, void *o,
+                                    void *workspace, size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    OpDims d;
+    bla_status s = check_params(p, &d);
+    if (s != BLA_OK) return s;
+    if (d.L > 0 && (!q || !k || !v || !o)) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
+    if (d.dtype == BLA_BF16) {
+        const char *why = fwd_bf16_unsupported(d);
+        if (why) return fail(BLA_ERR_UNSUPPORTED, "bf16 forward: %s", why);
+    }
+    size_t fw = 0;
+    if ((s = check_ws(workspace, ws_bytes, ws_forward_host_parts(p, d, &fw))) != BLA_OK) return s;
+    if (d.L == 0) return BLA_OK;
+    HostPipe *hp = nullptr;
+    cudaError_t e = host_pipe(&hp);
+    if (e != cudaSuccess) return cuda_fail(e, "copy streams");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const size_t BH = (size_t)d.B * d.H, es = host_elem(d);
+    const size_t rq = (size_t)d.L * d.dk * es, rv = (size_t)d.L * d.dv * es;   // bytes per head
+    char *ws = static_cast<char *>(workspace);
+    char *qd = ws + fw, *kd = qd + align_up(BH * rq, 256), *vd = kd + align_up(BH * rq, 256);
+    char *od = vd + align_up(BH * rv, 256);
+    const char *qh = static_cast<const char *>(q), *kh = static_cast<const char *>(k), *vh = static_cast<const char *>(v);
+    char *oh = static_cast<char *>(o);
+    // copies start after everything already in `stream` (an earlier call's copies included)
+    if ((e = cudaEventRecord(hp->start, st)) != cudaSuccess || (e = cudaStreamWaitEvent(hp->h2d, hp->start, 0)) != cudaSuccess ||
+        (e = cudaStreamWaitEvent(hp->d2h, hp->start, 0)) != cudaSuccess)
+        return cuda_fail(e, "stream ordering");
+    const int ng = host_groups(d);
+    for (int g = 0; g < ng; ++g) {
+        const long long h0 = host_group_first(d, ng, g), nh = host_group_first(d, ng, g + 1) - h0;
+        if ((e = cudaMemcpyAsync(qd + h0 * rq, qh + h0 * rq, nh * rq, cudaMemcpyHostToDevice, hp->h2d)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(kd + h0 * rq, kh + h0 * rq, nh * rq, cudaMemcpyHostToDevice, hp->h2d)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(vd + h0 * rv, vh + h0 * rv, nh * rv, cudaMemcpyHostToDevice, hp->h2d)) != cudaSuccess ||
+            (e = cudaEventRecord(hp->in[g], hp->h2d)) != cudaSuccess || (e = cudaStreamWaitEvent(st, hp->in[g], 0)) != cudaSuccess)
+            return cuda_fail(e, "host-to-device copy");
+        if ((s = forward_device(p, host_group_dims(d, nh), qd + h0 * rq, kd + h0 * rq, vd + h0 * rv, od + h0 * rv, nullptr,
+                                nullptr, ws, st)) != BLA_OK)
+            return s;
+        if ((e = cudaEventRecord(hp->out[g], st)) != cudaSuccess || (e = cudaStreamWaitEvent(hp->d2h, hp->out[g], 0)) != cudaSuccess ||
+            (e = cudaMemcpyAsync(oh + h0 * rv, od + h0 * rv, nh * rv, cudaMemcpyDeviceToHost, hp->d2h)) != cudaSuccess)
+            return cuda_fail(e, "device-to-host copy");
+    }
+    if ((e = cudaEventRecord(hp->done, hp->d2h)) != cudaSuccess || (e = cudaStreamWaitEvent(st, hp->done, 0)) != cudaSuccess)
+        return cuda_fail(e, "stream ordering");
     return BLA_OK;
 }
 

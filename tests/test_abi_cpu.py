@@ -96,6 +96,19 @@ def test_workspace_sizes_positive(lib):
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECODE) > 0
 
 
+def test_host_forward_argument_checks(lib):
+    """The host-buffer forward validates its arguments before any copy, and its workspace holds the
+    forward's own plus the device copies of q, k, v and o."""
+    from paper_2606_09862_gb300 import bla
+    p = _params(dtype=bla.BLA_BF16, d_k=64, d_v=64, M=32, S=32, window=256.0, L=300)
+    assert lib.bla_forward_chunked_host(ctypes.byref(p), None, FAKE, FAKE, FAKE, FAKE, 1 << 30, None) == \
+        bla.BLA_ERR_INVALID
+    assert lib.bla_forward_chunked_host(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, 8, None) == bla.BLA_ERR_INVALID
+    fw = lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_FORWARD)
+    hw = lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_FORWARD_HOST)
+    assert hw >= fw + 4 * 2 * 300 * 64 * 2
+
+
 def test_phase_mode_accepted(lib):
     """Both phase modes are valid parameters; the absolute form's backward needs its per-chunk
     phase table on top of the lag form's workspace."""
