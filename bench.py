@@ -249,9 +249,14 @@ def main():
     ap.add_argument("--seq", type=int, default=0, help="override L (profiling captures of a smaller case)")
     ap.add_argument("--decode-batch", type=int, default=0, help="override the decode batch (profiling captures)")
     ap.add_argument("--no-configs", action="store_true", help="skip the timing of the other parity configs")
+    ap.add_argument("--configs-only", default="",
+                    help="comma-separated parity configs to time alone (profiling captures); prints their JSON")
+    ap.add_argument("--configs-iters", type=int, default=20, help="timed calls per parity config")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
+    if args.configs_only:
+        return run_configs_only(args)
 
     import torch
     from paper_2606_09862_gb300 import bla
@@ -409,7 +414,20 @@ def main():
     return 0
 
 
-def measure_configs(bla, torch, dev, stream, peaks, iters=20):
+def run_configs_only(args):
+    """Time only the named parity configs (for ncu captures of their kernels) and print the JSON."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    names = tuple(n for n in args.configs_only.split(",") if n)
+    out = measure_configs(bla, torch, dev, torch.cuda.current_stream(dev), load_peaks(), iters=max(1, args.configs_iters),
+                          only=names, warm=max(1, min(3, args.warmup)))
+    print(json.dumps({"configs": out}))
+    return 0
+
+
+def measure_configs(bla, torch, dev, stream, peaks, iters=20, only=None, warm=3):
     """The other parity configs, timed through the same ABI: config 2 (recall-shaped forward) and
     config 3 (LM-layer forward and backward).  Each call is timed alone with CUDA events after an
     L2 flush (config 2's inputs fit in L2); FLOPs are the canonical counts at chunk 64, the chunk
@@ -419,7 +437,7 @@ def measure_configs(bla, torch, dev, stream, peaks, iters=20):
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)   # 256 MB > 129 MB L2
 
     def timed(fn):
-        for _ in range(3):
+        for _ in range(warm):
             fn()
         tot = 0.0
         for _ in range(iters):
@@ -447,6 +465,10 @@ def measure_configs(bla, torch, dev, stream, peaks, iters=20):
     # form (phase_mode "absolute", Alg. 1), which runs the same kernels with other tables
     for name, modes in (("fwd_bf16_recall", ("lag",)), ("fwdbwd_bf16_lm", ("lag", "absolute")),
                         ("prefill_bf16_long", ("absolute",))):
+        if only:
+            if name not in only:
+                continue
+            modes = ("lag",) if name != "prefill_bf16_long" else ("absolute",)
         w = WORKLOADS[name]
         q, k, v = (torch.from_numpy(x).to(torch.bfloat16).to(dev)
                    for x in make_qkv(w.B, w.H, w.L, w.d, "bf16", seed=0, recall_dup=getattr(w, "recall_dup", 0.0)))
