@@ -1109,7 +1109,12 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
                 // chunk z has read V, W_V and dO: its K, W_K, and the next chunk's dO
                 if (!wait_bar(&bar[CA_VW_FREE], ph_vwf, ctl, a.err, 51)) break;
                 load_kw(z);
-                if (zn < a.Z) load_do(zn);
+                if (zn < a.Z) {
+                    load_do(zn);
+                    // the next chunk's o (for rowsum(dO o)) into L2
+                    const int nbh = zn / a.nch, nc = zn % a.nch, rows = min(kC, a.L - nc * kC);
+                    tc::bulk_prefetch_l2(a.o + ((size_t)nbh * a.L + (size_t)nc * kC) * D, (uint32_t)(rows * D * 2));
+                }
                 if (zn >= a.Z) break;
                 // chunk z's ds has been read: the next chunk's p
                 if (!wait_bar(&bar[CA_SP_FREE], ph_spf, ctl, a.err, 52)) break;
@@ -1203,24 +1208,34 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
             if (threadIdx.x == 0) tc::bulk_wait_read0();
             if (!esync(68)) break;
             if (!wait_bar(&bar[CA_DO_FULL], ph[CA_DO_FULL], ctl, a.err, 61)) break;
-            // rowsum(dO o) of 16 rows per warp, loads of o coalesced (LPR lanes per row)
-            for (int r0 = warp * 16; r0 < warp * 16 + 16; r0 += RPI) {
-                const int r = r0 + lane / LPR, d0 = (lane % LPR) * 8, tt = c * kC + r;
-                float acc = 0.f;
-                if (tt < a.L) {
-                    const uint4 ov = __ldg(reinterpret_cast<const uint4 *>(a.o + ((size_t)bh * a.L + tt) * D + d0));
+            // rowsum(dO o) of 16 rows per warp, loads of o coalesced (LPR lanes per row); every load
+            // is issued before the first is used
+            {
+                constexpr int NIT = 16 / RPI;
+                const int d0 = (lane % LPR) * 8;
+                uint4 ov[NIT];
+#pragma unroll
+                for (int it = 0; it < NIT; ++it) {
+                    const int r = warp * 16 + it * RPI + lane / LPR, tt = c * kC + r;
+                    ov[it] = tt < a.L ? __ldg(reinterpret_cast<const uint4 *>(a.o + ((size_t)bh * a.L + tt) * D + d0))
+                                      : make_uint4(0u, 0u, 0u, 0u);
+                }
+#pragma unroll
+                for (int it = 0; it < NIT; ++it) {
+                    const int r = warp * 16 + it * RPI + lane / LPR;
                     const uint4 gv = *reinterpret_cast<const uint4 *>(sDO + (d0 >> 6) * 128 * 128 + tc::sw128_offset(r, d0 & 63));
-                    const uint32_t ow[4] = {ov.x, ov.y, ov.z, ov.w}, gw[4] = {gv.x, gv.y, gv.z, gv.w};
+                    const uint32_t ow[4] = {ov[it].x, ov[it].y, ov[it].z, ov[it].w}, gw[4] = {gv.x, gv.y, gv.z, gv.w};
+                    float acc = 0.f;
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
                         const float2 x = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&ow[q]));
                         const float2 y = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&gw[q]));
                         acc = fmaf(x.x, y.x, fmaf(x.y, y.y, acc));
                     }
-                }
 #pragma unroll
-                for (int off = LPR / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
-                if (lane % LPR == 0) sdl[r] = acc;
+                    for (int off = LPR / 2; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+                    if (lane % LPR == 0) sdl[r] = acc;
+                }
             }
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(&bar[CA_VW_FREE]);

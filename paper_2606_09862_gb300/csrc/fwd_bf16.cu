@@ -156,8 +156,9 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, d
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
         if (i < n_eb) {
-            const long long per_c = (long long)MP * (kC / 8);
-            const int c = (int)(i / per_c), rem = (int)(i % per_c);
+            // (32-bit index arithmetic: n_eb = 16 L < 2^31 for L <= 2^26, which the host checks)
+            const unsigned per_c = (unsigned)MP * (kC / 8), ui = (unsigned)i;
+            const int c = (int)(ui / per_c), rem = (int)(ui - (unsigned)c * per_c);
             const int m = rem / (kC / 8), u0 = (rem % (kC / 8)) * 8;
             bf16 *rc = eb + ((size_t)c * RP + 2 * m) * kC + u0, *rs = rc + kC;
             uint32_t wc[4] = {0u, 0u, 0u, 0u}, ws[4] = {0u, 0u, 0u, 0u};
@@ -181,8 +182,8 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, d
             *reinterpret_cast<uint4 *>(rc) = make_uint4(wc[0], wc[1], wc[2], wc[3]);
             *reinterpret_cast<uint4 *>(rs) = make_uint4(ws[0], ws[1], ws[2], ws[3]);
         } else if (i < n_eb + n_phi) {
-            const long long e = i - n_eb;
-            const int j = (int)(e / R2), r = (int)(e % R2), m = r >> 1;
+            const int e = (int)(i - n_eb);
+            const int j = e / R2, r = e % R2, m = r >> 1;
             float v = 0.f;
             if (j < S) {
                 const long long dj = (long long)rint((double)j * T / (double)S);
@@ -194,9 +195,9 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, d
             phi[e] = __float2bfloat16_rn(v);
         } else if (i < n_eb + n_phi + n_f) {
             // FSEG rows 2m, 2m+1 for 8 consecutive u: e^{i m w (Lseg - u)}, stepping by e^{-i m w}
-            const long long e = i - n_eb - n_phi;
+            const int e = (int)(i - n_eb - n_phi);
             const int per_m = (Lseg + 7) / 8;
-            const int m = (int)(e / per_m), u0 = (int)(e % per_m) * 8;
+            const int m = e / per_m, u0 = (e % per_m) * 8;
             bf16 *rc = fseg + (size_t)(2 * m) * Lseg + u0, *rs = rc + Lseg;
             float bc = 0.f, bs = 0.f, ec = 1.f, es = 0.f;
             if (m < M) {
@@ -1471,6 +1472,7 @@ const char *fwd_bf16_unsupported(const OpDims &d) {
     if (d.R2 != 64 && d.R2 != 128 && d.R2 != 256) return "2M must be 64, 128 or 256";
     if (d.S != 32 && d.S != 64 && d.S != 128) return "S must be 32, 64 or 128";
     if (d.S > (d.R2 < 64 ? 64 : d.R2)) return "S must not exceed max(2M, 64)";
+    if (d.L > (1 << 26)) return "L must not exceed 2^26 tokens (table indices are 32-bit)";
     return nullptr;
 }
 

@@ -102,6 +102,12 @@ __device__ __forceinline__ void tma_prefetch_3d(const CUtensorMap *map, int c0, 
                  : "memory");
 }
 
+// Bring `bytes` (a multiple of 16) of global memory from `gptr` (16-byte aligned) into L2.
+__device__ __forceinline__ void bulk_prefetch_l2(const void *gptr, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(gptr)), "r"(bytes)
+                 : "memory");
+}
+
 // Bulk tensor store shared -> global (3-D map), tracked by this thread's bulk group.
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, const void *src, int c0, int c1, int c2) {
     asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
