@@ -352,6 +352,16 @@ __device__ __forceinline__ void advance(RowPhases &p, const RowPhases &step) {
 // (c, s) = (cos, sin)(m w t0) of this thread's mode.  Each thread loads only its own row, all
 // loads issued before any use (one memory latency per block); the partner row of the pair is
 // the neighbouring lane's.
+// L2 prefetch of this thread's DH columns of one state row (issued before an earlier block is
+// processed, so that the later block's loads do not pay the full memory latency).
+template <int DH>
+__device__ __forceinline__ void state_prefetch_row(const float *src, int row, int live_rows, int stride) {
+    if (src == nullptr || row >= live_rows) return;
+    const float *p = src + (size_t)row * stride;
+#pragma unroll
+    for (int i = 0; i < DH; i += 32) asm volatile("prefetch.global.L2 [%0];" ::"l"(p + i) : "memory");
+}
+
 template <int DH>
 __device__ __forceinline__ void state_init_abs(uint32_t tbase, int col0, int row, const float *src, int live_rows,
                                                int stride, float c, float s) {
@@ -855,6 +865,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, a.w, a.tint);
             // the state is kept in the absolute frame, A = sum_{u < t0} e^{-i m w u} k_u: it needs no
             // rotation between chunks; the carried-in lag-frame state is rotated once
+            if (g.NB > 1 && g.G > 1)
+                state_prefetch_row<DH>(a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + 128) * D + wg * DH, row,
+                                       g.R2 - 128, D);
             for (int b = 0; b < g.NB; ++b) {
                 const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
                 const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
@@ -1316,6 +1329,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             RowPhases rp = row_phases(a.absolute ? 0 : (long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
             const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, a.w, a.tint);
             // V state in the absolute frame (see the K pass)
+            if (g.NB > 1 && g.G > 1)
+                state_prefetch_row<DH>(a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + 128) * D + wg * DH, row,
+                                       g.R2 - 128, D);
             for (int b = 0; b < g.NB; ++b) {
                 const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
                 const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
