@@ -501,9 +501,38 @@ def measure_configs(bla, torch, dev, stream, peaks, iters=20, only=None, warm=3)
         res["shape"] = "B=%d H=%d L=%d d=%d M=%d S=%d T=%d" % (w.B, w.H, w.L, w.d, w.M, w.S, w.T)
         out[name] = res
         del q, k, v
+    if not only or "lm_block_f32" in only:
+        out["lm_block_f32"] = measure_block(bla, torch, dev, timed)
     del flush
     torch.cuda.empty_cache()
     return out
+
+
+def measure_block(bla, torch, dev, timed):
+    """One BLA layer of the RegBench-sized LM block (d_model 128, 4 heads, M = 16, S = 31, T = 62,
+    batch 32, L = 256; fp32): input projections (cuBLAS), token mixing (fp32 path), output projection."""
+    from paper_2606_09862_gb300.inputs import WORKLOADS, make_block_inputs
+    from paper_2606_09862_gb300.layer import bla_block_forward
+    w = WORKLOADS["lm_block_f32"]
+    dm = w.H * w.d
+    x, ws = make_block_inputs(w.B, w.L, dm, seed=0)
+    x = torch.from_numpy(x).to(dev)
+    ws = [torch.from_numpy(a).to(dev) for a in ws]
+    par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.float32)
+    wsp = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_FORWARD), dtype=torch.uint8, device=dev)
+    mix = {}
+
+    def layer():
+        return bla_block_forward(x, *ws, w.H, w.M, w.S, w.T, workspace=wsp)
+
+    def mixing():
+        return bla.bla_forward_chunked(mix["q"], mix["k"], mix["v"], w.M, w.S, w.T, want_lse=False, workspace=wsp)
+
+    mix["q"], mix["k"], mix["v"] = (torch.randn(w.B, w.H, w.L, w.d, device=dev) for _ in range(3))
+    ms = timed(layer)
+    ms_mix = timed(mixing)
+    return {"layer_ms": ms, "mixing_ms": ms_mix, "tokens_per_s": w.B * w.L / (ms / 1000.0),
+            "shape": "B=%d L=%d d_model=%d H=%d d=%d M=%d S=%d T=%g fp32" % (w.B, w.L, dm, w.H, w.d, w.M, w.S, w.T)}
 
 
 def stored_traffic(kernel, L):

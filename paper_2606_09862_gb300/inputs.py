@@ -14,7 +14,7 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-STREAMS = ("q", "k", "v", "dout", "state", "dup")
+STREAMS = ("q", "k", "v", "dout", "state", "dup", "x", "w")
 
 
 @dataclass(frozen=True)
@@ -49,6 +49,11 @@ WORKLOADS = {
                                notes="LM-layer shape, model dim 1024; upstream grad ~ N(0,1)"),
     "prefill_bf16_long": Workload("prefill_bf16_long", "bf16", B=1, H=16, L=65536, d=128, M=128, S=128,
                                   T=4096, chunk=128, notes="long-context prefill"),
+    # a BLA layer of the RegBench-sized LM (model dim 128, 4 heads, batch 32; M = 16 of the searched
+    # 8..64, S = 2M-1 slots, T = 2(2M-1) of the searched [1, 2, 4](2M-1)); the sequence length is
+    # not stated, 256 is assumed.  Odd S and d = 32 run on the fp32 path.
+    "lm_block_f32": Workload("lm_block_f32", "f32", B=32, H=4, L=256, d=32, M=16, S=31, T=62, chunk=64,
+                             notes="x ~ N(0,1) [B, L, 128]; W_q, W_k, W_v, W_o ~ N(0, 1/128)"),
     "decode_bf16": Workload("decode_bf16", "bf16", B=256, H=16, L=1, d=128, M=128, S=128, T=4096,
                             chunk=1, decode_steps=1024, decode_pos0=4096, state_std=0.1,
                             notes="single-token decode, fp32 state ~ N(0, 0.1^2)"),
@@ -147,3 +152,13 @@ def workload_inputs(w: Workload, seed=0, sharp=False):
     if w.backward:
         out["dout"] = make_dout(w.B, w.H, w.L, w.d, w.dtype, seed)
     return out
+
+
+def make_block_inputs(B, L, dm, seed=0):
+    """Input activations x ~ N(0, 1) [B, L, dm] and projection weights W_q, W_k, W_v, W_o ~
+    N(0, 1/dm) [dm, dm] for one LM-block layer (float32)."""
+    st = _streams(seed)
+    sx, sw = st["x"], st["w"]
+    x = sx.standard_normal((B, L, dm)).astype(np.float32)
+    ws = [(sw.standard_normal((dm, dm)) / np.sqrt(dm)).astype(np.float32) for _ in range(4)]
+    return x, ws
