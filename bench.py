@@ -501,6 +501,15 @@ def measure_configs(bla, torch, dev, stream, peaks, iters=20, only=None, warm=3)
         res["shape"] = "B=%d H=%d L=%d d=%d M=%d S=%d T=%d" % (w.B, w.H, w.L, w.d, w.M, w.S, w.T)
         out[name] = res
         del q, k, v
+    if not only or "fwd_f32_small" in only:
+        w = WORKLOADS["fwd_f32_small"]
+        q, k, v = (torch.from_numpy(x).to(dev) for x in make_qkv(w.B, w.H, w.L, w.d, "f32", seed=0))
+        par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, chunk=w.chunk, dtype=torch.float32)
+        wsf = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_FORWARD), dtype=torch.uint8, device=dev)
+        ms = timed(lambda: bla.bla_forward_chunked(q, k, v, w.M, w.S, w.T, chunk=w.chunk, workspace=wsf))
+        out["fwd_f32_small"] = {"forward": {"ms": ms, "tokens_per_s": w.B * w.L / (ms / 1000.0)},
+                                "shape": "B=%d H=%d L=%d d=%d M=%d S=%d T=%g chunk=%d fp32" %
+                                         (w.B, w.H, w.L, w.d, w.M, w.S, w.T, w.chunk)}
     if not only or "lm_block_f32" in only:
         out["lm_block_f32"] = measure_block(bla, torch, dev, timed)
     del flush

@@ -32,41 +32,77 @@ struct F32Smem {
     float *Q, *K, *V, *P, *X, *Sc, *Ph;
 };
 
+// stage != 0: the phase and slot tables (also transposed, for the loops that walk them across
+// rows) and the carried state live in shared memory, copied in at the start, the state written out
+// at the end; otherwise they are read from global memory.  Rows of the q, k, v tiles (and of the
+// staged state) are padded by one float so that loops over rows do not hit one bank.
 __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb, const float *__restrict__ q,
                                                      const float *__restrict__ k, const float *__restrict__ v,
                                                      float *__restrict__ o, float *__restrict__ lse,
-                                                     float *__restrict__ state) {
+                                                     float *__restrict__ state, int stage) {
     extern __shared__ float smem[];
     const int dk = d.dk, dv = d.dv, M = d.M, R2 = d.R2, S = d.S, L = d.L;
+    const int QS = dk + 1, VS = dv + 1;   // padded row strides of the q/k and v tiles
     const int bh = blockIdx.x;
     const int tid = threadIdx.x, nt = blockDim.x;
     F32Smem sm;
     sm.Q = smem;
-    sm.K = sm.Q + C * dk;
-    sm.V = sm.K + C * dk;
-    sm.P = sm.V + C * dv;
+    sm.K = sm.Q + C * QS;
+    sm.V = sm.K + C * QS;
+    sm.P = sm.V + C * VS;
     sm.X = sm.P + C * C;
     sm.Sc = sm.X + C * R2;
     sm.Ph = sm.Sc + C * S;   // [M][2] absolute form: (cos, sin)(-m w t0) of the current chunk
+    float *st_erel = sm.Ph + R2, *st_erelT = st_erel + (C + 1) * M * 2, *st_phi = st_erelT + (C + 1) * M * 2;
+    float *st_phiT = st_phi + S * R2, *st_state = st_phiT + S * R2;
 
     const float *qh = q + (size_t)bh * L * dk, *kh = k + (size_t)bh * L * dk, *vh = v + (size_t)bh * L * dv;
     float *oh = o + (size_t)bh * L * dv;
     float *lh = lse ? lse + (size_t)bh * L : nullptr;
-    float *WK = state + (size_t)bh * R2 * (dk + dv);
-    float *WV = WK + (size_t)R2 * dk;
-    const float *erel = tb.erel, *phi = tb.phi;
+    float *const gstate = state + (size_t)bh * R2 * (dk + dv);
+    // carried state: rows of the K part, then the V part, row strides KS / VSt
+    const int KS = stage ? dk + 1 : dk, VSt = stage ? dv + 1 : dv;
+    float *WK = stage ? st_state : gstate;
+    float *WV = WK + (size_t)R2 * KS;
+    // phase table erel[(u M + m) 2 + c] and slot table phi[j R2 + r]; eT(u, m) and phT(r, j) index
+    // their transposes when staged (the plain tables otherwise)
+    const float *erel = tb.erel, *phi = tb.phi, *erelT = tb.erel, *phiT = tb.phi;
     const int *delta = tb.delta;
+    if (stage) {
+        for (int i = tid; i < (C + 1) * M; i += nt) {
+            const int u = i / M, m = i % M;
+            const float c = tb.erel[2 * i], s = tb.erel[2 * i + 1];
+            st_erel[2 * i] = c;
+            st_erel[2 * i + 1] = s;
+            st_erelT[(m * (C + 1) + u) * 2] = c;
+            st_erelT[(m * (C + 1) + u) * 2 + 1] = s;
+        }
+        for (int i = tid; i < S * R2; i += nt) {
+            const float x = tb.phi[i];
+            st_phi[i] = x;
+            st_phiT[(i % R2) * S + i / R2] = x;
+        }
+        erel = st_erel;
+        phi = st_phi;
+        erelT = st_erelT;
+        phiT = st_phiT;
+    }
+    auto eT = [&](int u, int m, int comp) {
+        return stage ? erelT[(m * (C + 1) + u) * 2 + comp] : erel[(u * M + m) * 2 + comp];
+    };
+    auto phT = [&](int r, int j) { return stage ? phiT[r * S + j] : phi[j * R2 + r]; };
 
-    for (int i = tid; i < R2 * (dk + dv); i += nt) WK[i] = 0.f;
+    for (int i = tid; i < R2 * KS + R2 * VSt; i += nt) WK[i] = 0.f;
     __syncthreads();
 
     for (int t0 = 0; t0 < L; t0 += C) {
         const int n = min(C, L - t0);
         for (int i = tid; i < n * dk; i += nt) {
-            sm.Q[i] = qh[(size_t)t0 * dk + i];
-            sm.K[i] = kh[(size_t)t0 * dk + i];
+            const int r = i / dk, c = i % dk;
+            sm.Q[r * QS + c] = qh[(size_t)t0 * dk + i];
+            sm.K[r * QS + c] = kh[(size_t)t0 * dk + i];
         }
-        for (int i = tid; i < n * dv; i += nt) sm.V[i] = vh[(size_t)t0 * dv + i];
+        for (int i = tid; i < n * dv; i += nt) sm.V[(i / dv) * VS + i % dv] = vh[(size_t)t0 * dv + i];
         if (d.absolute) {
             for (int m = tid; m < M; m += nt) {
                 double sn, cs;
@@ -81,7 +117,7 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
             int t = i / n, u = i % n;
             float acc = 0.f;
             if (u <= t)
-                for (int e = 0; e < dk; ++e) acc = fmaf(sm.Q[t * dk + e], sm.K[u * dk + e], acc);
+                for (int e = 0; e < dk; ++e) acc = fmaf(sm.Q[t * QS + e], sm.K[u * QS + e], acc);
             sm.P[t * C + u] = acc;
         }
         __syncthreads();
@@ -94,10 +130,10 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
                 xc = fmaf(pu, erel[(u * M + m) * 2], xc);
                 xs = fmaf(-pu, erel[(u * M + m) * 2 + 1], xs);
             }
-            const float *wc = WK + (size_t)(2 * m) * dk, *ws = wc + dk;
+            const float *wc = WK + (size_t)(2 * m) * KS, *ws = wc + KS;
             for (int e = 0; e < dk; ++e) {
-                xc = fmaf(sm.Q[t * dk + e], wc[e], xc);
-                xs = fmaf(sm.Q[t * dk + e], ws[e], xs);
+                xc = fmaf(sm.Q[t * QS + e], wc[e], xc);
+                xs = fmaf(sm.Q[t * QS + e], ws[e], xs);
             }
             const float *ph = d.absolute ? sm.Ph + 2 * m : erel + (t * M + m) * 2;
             float c = ph[0], s = ph[1];
@@ -109,7 +145,7 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
         for (int i = tid; i < n * S; i += nt) {
             int t = i / S, j = i % S;
             float acc = 0.f;
-            for (int r = 0; r < R2; ++r) acc = fmaf(phi[j * R2 + r], sm.X[t * R2 + r], acc);
+            for (int r = 0; r < R2; ++r) acc = fmaf(phT(r, j), sm.X[t * R2 + r], acc);
             sm.Sc[t * S + j] = (t0 + t >= delta[j]) ? acc * d.scale : -INFINITY;
         }
         __syncthreads();
@@ -149,8 +185,7 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
             float acc = 0.f;
             if (u <= t)
                 for (int m = 0; m < M; ++m)
-                    acc += sm.X[t * R2 + 2 * m] * erel[(u * M + m) * 2] -
-                           sm.X[t * R2 + 2 * m + 1] * erel[(u * M + m) * 2 + 1];
+                    acc += sm.X[t * R2 + 2 * m] * eT(u, m, 0) - sm.X[t * R2 + 2 * m + 1] * eT(u, m, 1);
             sm.P[t * C + u] = acc;
         }
         __syncthreads();
@@ -158,8 +193,8 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
         for (int i = tid; i < n * dv; i += nt) {
             int t = i / dv, e = i % dv;
             float acc = 0.f;
-            for (int u = 0; u <= t; ++u) acc = fmaf(sm.P[t * C + u], sm.V[u * dv + e], acc);
-            for (int r = 0; r < R2; ++r) acc = fmaf(sm.X[t * R2 + r], WV[(size_t)r * dv + e], acc);
+            for (int u = 0; u <= t; ++u) acc = fmaf(sm.P[t * C + u], sm.V[u * VS + e], acc);
+            for (int r = 0; r < R2; ++r) acc = fmaf(sm.X[t * R2 + r], WV[(size_t)r * VSt + e], acc);
             oh[(size_t)(t0 + t) * dv + e] = acc;
         }
         __syncthreads();
@@ -169,12 +204,12 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
         for (int i = tid; i < M * (dk + dv); i += nt) {
             int m = i / (dk + dv), e = i % (dk + dv);
             const bool isk = e < dk;
-            const int ee = isk ? e : e - dk, dd = isk ? dk : dv;
-            float *Wc = (isk ? WK : WV) + (size_t)(2 * m) * dd + ee, *Ws = Wc + dd;
+            const int ee = isk ? e : e - dk, xs_ = isk ? QS : VS, ws_ = isk ? KS : VSt;
+            float *Wc = (isk ? WK : WV) + (size_t)(2 * m) * ws_ + ee, *Ws = Wc + ws_;
             const float *X = isk ? sm.K : sm.V;
             float ac = *Wc, as = *Ws;
             for (int u = 0; u < n; ++u) {
-                float x = X[u * dd + ee];
+                float x = X[u * xs_ + ee];
                 ac = fmaf(erel[(u * M + m) * 2], x, ac);
                 as = fmaf(-erel[(u * M + m) * 2 + 1], x, as);
             }
@@ -184,13 +219,25 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
         }
         __syncthreads();
     }
+    if (stage) {
+        // out to the global layout [R2][dk] then [R2][dv]
+        for (int i = tid; i < R2 * dk; i += nt) gstate[i] = WK[(i / dk) * KS + i % dk];
+        for (int i = tid; i < R2 * dv; i += nt) gstate[R2 * dk + i] = WV[(i / dv) * VSt + i % dv];
+    }
 }
 
 }  // namespace
 
 int forward_f32_smem_bytes(const OpDims &d, int C) {
-    size_t f = (size_t)C * d.dk * 2 + (size_t)C * d.dv + (size_t)C * C + (size_t)C * d.R2 + (size_t)C * d.S +
-               (size_t)d.R2;
+    size_t f = (size_t)C * (d.dk + 1) * 2 + (size_t)C * (d.dv + 1) + (size_t)C * C + (size_t)C * d.R2 +
+               (size_t)C * d.S + (size_t)d.R2;
+    return (int)(f * sizeof(float));
+}
+
+// Extra shared memory of the staged variant: the phase table and the slot table (each also
+// transposed), and the carried state with padded rows.
+static int forward_f32_stage_bytes(const OpDims &d, int C) {
+    size_t f = 2 * (size_t)(C + 1) * d.M * 2 + 2 * (size_t)d.S * d.R2 + (size_t)d.R2 * (d.dk + 1 + d.dv + 1);
     return (int)(f * sizeof(float));
 }
 
@@ -203,11 +250,14 @@ cudaError_t launch_forward_f32(const OpDims &d, int C, const Tables &t, const fl
                                const float *v, float *o, float *lse, float *state_out, float *scratch,
                                cudaStream_t st) {
     int smem = forward_f32_smem_bytes(d, C);
+    const int staged = smem + forward_f32_stage_bytes(d, C);
+    const int stage = staged <= 227 * 1024;
+    if (stage) smem = staged;
     cudaError_t e = cudaFuncSetAttribute(k_forward_f32, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     float *state = state_out ? state_out : scratch;
     ProfScope ps(BLA_K_FWD_F32, st);
-    k_forward_f32<<<d.B * d.H, 256, smem, st>>>(d, C, t, q, k, v, o, lse, state);
+    k_forward_f32<<<d.B * d.H, 256, smem, st>>>(d, C, t, q, k, v, o, lse, state, stage);
     return cudaGetLastError();
 }
 
