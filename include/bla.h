@@ -210,6 +210,13 @@ bla_status bla_profile_collect(double *ms, int *launches);
  * was not 1024-byte aligned. */
 bla_status bla_device_error(void *stream);
 
+/* Self-test of the failure path (no paper counterpart): launch one CTA whose bounded mbarrier
+ * wait, on a barrier nothing ever arrives at, gives up after about limit_ms milliseconds (1 to
+ * 1000) and records the timeout in the device error word, exactly as a kernel of the library does
+ * when a wait runs out.  The next bla_device_error(stream) then returns BLA_ERR_TIMEOUT, and the
+ * context stays usable.  Returns BLA_ERR_INVALID for a limit out of range. */
+bla_status bla_selftest_wait_timeout(int limit_ms, void *stream);
+
 /* Static description of a status code. */
 const char *bla_status_string(bla_status s);
 

@@ -22,7 +22,8 @@ PHASE_MODES = {"lag": BLA_PHASE_LAG, "absolute": BLA_PHASE_ABSOLUTE}
 
 EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
             "bla_device_error", "bla_status_string", "bla_last_error_string", "bla_kernel_launches",
-            "bla_profile_enable", "bla_profile_collect", "bla_decode_step_noalloc", "bla_forward_chunked_host")
+            "bla_profile_enable", "bla_profile_collect", "bla_decode_step_noalloc", "bla_forward_chunked_host",
+            "bla_selftest_wait_timeout")
 
 # bla_kernel_id
 KERNELS = ("tables", "tables_bf16", "prepass", "scan", "kpass", "vpass", "fwd_f32", "decode", "bwd")
@@ -59,6 +60,8 @@ def load():
     lib.bla_workspace_bytes.argtypes = [P, ctypes.c_int]
     lib.bla_forward_chunked.restype = ctypes.c_int
     lib.bla_forward_chunked.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_selftest_wait_timeout.restype = ctypes.c_int
+    lib.bla_selftest_wait_timeout.argtypes = [ctypes.c_int, vp]
     lib.bla_forward_chunked_host.restype = ctypes.c_int
     lib.bla_forward_chunked_host.argtypes = [P, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_decode_step.restype = ctypes.c_int
@@ -205,6 +208,12 @@ def bla_backward(q, k, v, o, dout, lse, M, S, window, omega=0.0, scale=0.0, work
 def bla_device_error(stream=None):
     """Synchronise and raise BlaError if a bounded device wait gave up."""
     _check(load().bla_device_error(_stream(stream)))
+
+
+def bla_selftest_wait_timeout(limit_ms=20, stream=None):
+    """Launch the library's failure-path self-test (a bounded wait that runs out); the next
+    bla_device_error() raises BlaError with status BLA_ERR_TIMEOUT."""
+    _check(load().bla_selftest_wait_timeout(int(limit_ms), _stream(stream)))
 
 
 def bla_kernel_launches():

@@ -11,6 +11,7 @@
 #include "common.cuh"
 #include "bwd.cuh"
 #include "fwd_bf16.cuh"
+#include "tc.cuh"
 
 namespace bla {
 
@@ -148,6 +149,18 @@ size_t ws_forward(const bla_params *p, const OpDims &d) {
 }
 
 size_t ws_decode(const OpDims &d) { return tables_bytes(d, 0); }
+
+// bla_selftest_wait_timeout: a bounded wait on a barrier nothing arrives at (kernel id 15 in the
+// error word).
+__global__ void k_wait_selftest(uint64_t limit_ns, int *err) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        tc::mbar_init(&bar, 1);
+        tc::fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !tc::mbar_wait(&bar, 0, limit_ns)) report_device_error(err, DEVERR_MBAR_TIMEOUT | (15 << 4));
+}
 
 // ---- host-buffer forward: head groups pipelined over copy streams
 constexpr int kHostGroupsMax = 8;
@@ -385,6 +398,21 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
     if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
     cudaError_t e = bwd_run(d, q, k, v, o, dout, lse, dq, dk, dv, workspace, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "backward");
+    return BLA_OK;
+}
+
+bla_status bla_selftest_wait_timeout(int limit_ms, void *stream) {
+    t_last_error[0] = 0;
+    if (limit_ms < 1 || limit_ms > 1000) return fail(BLA_ERR_INVALID, "limit_ms must be in [1, 1000] (got %d)", limit_ms);
+    int *err = device_error_word();
+    if (!err) return fail(BLA_ERR_CUDA, "device error word unavailable");
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    {
+        ProfScope ps(BLA_K_DECODE, st);   // counted as a launch of the library
+        k_wait_selftest<<<1, 32, 0, st>>>((uint64_t)limit_ms * 1000000ull, err);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "self-test launch");
     return BLA_OK;
 }
 

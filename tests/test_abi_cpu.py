@@ -96,6 +96,12 @@ def test_workspace_sizes_positive(lib):
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECODE) > 0
 
 
+def test_selftest_limit_checked_on_host(lib):
+    from paper_2606_09862_gb300 import bla
+    assert lib.bla_selftest_wait_timeout(0, None) == bla.BLA_ERR_INVALID
+    assert lib.bla_selftest_wait_timeout(5000, None) == bla.BLA_ERR_INVALID
+
+
 def test_host_forward_argument_checks(lib):
     """The host-buffer forward validates its arguments before any copy, and its workspace holds the
     forward's own plus the device copies of q, k, v and o."""
