@@ -787,7 +787,7 @@ __device__ __forceinline__ uint32_t tm_addr(uint32_t tb, int lane_base, int col)
 
 // ---- k_chain_fwd
 enum CfBar { CF_TAB, CF_IN_FULL, CF_IN_FREE, CF_ACC1, CF_ACC2, CF_ACC3, CF_ACC4, CF_ACC5, CF_T1, CF_T2, CF_SP, CF_A,
-             CF_TFREE, CF_ESYNC, CF_COUNT };
+             CF_ESYNC, CF_COUNT };
 
 struct ChainLayout {
     int eb, phi, t0, t1, t2, t3, t4, sp, bars, total;
@@ -835,7 +835,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < CF_COUNT; ++i) {
-            const bool epi = i == CF_T1 || i == CF_T2 || i == CF_SP || i == CF_A || i == CF_TFREE || i == CF_ESYNC;
+            const bool epi = i == CF_T1 || i == CF_T2 || i == CF_SP || i == CF_A || i == CF_ESYNC;
             tc::mbar_init(&bar[i], epi ? kSeqEpiWarps : 1);
         }
         ctl->abort = 0;
@@ -875,15 +875,19 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
             const uint32_t q = tc::smem_u32(sQ), k = tc::smem_u32(sK), w = tc::smem_u32(sW), eb = tc::smem_u32(sEB);
             const uint32_t phi = tc::smem_u32(sPHI), t1 = tc::smem_u32(sT1), t2 = tc::smem_u32(sT2), sp = tc::smem_u32(sP);
             bool ok = wait_bar(&bar[CF_TAB], ph[CF_TAB], ctl, a.err, 31);
-            for (int z = blockIdx.x, i = 0; z < a.Z && ok; z += gridDim.x, ++i) {
-                ok = false;
-                if (!wait_bar(&bar[CF_IN_FULL], ph[CF_IN_FULL], ctl, a.err, 32)) break;
-                if (i > 0 && !wait_bar(&bar[CF_TFREE], ph[CF_TFREE], ctl, a.err, 33)) break;
+            // P = Q K^T of a chunk, into region 0 (free once the previous chunk's A' has been drained)
+            auto issue_p = [&]() -> bool {
+                if (!wait_bar(&bar[CF_IN_FULL], ph[CF_IN_FULL], ctl, a.err, 32)) return false;
                 tc::tc_fence_after();
 #pragma unroll
-                for (int kk = 0; kk < D / 16; ++kk)                 // P = Q K^T
+                for (int kk = 0; kk < D / 16; ++kk)
                     tc::mma_bf16(tb + colP, seq_kmaj(q, 128, 0, kk), seq_kmaj(k, 128, 0, kk), id_P, kk > 0);
                 tc::mma_commit(&bar[CF_ACC1]);
+                return true;
+            };
+            ok = ok && (int)blockIdx.x < a.Z && issue_p();
+            for (int z = blockIdx.x; z < a.Z && ok; z += gridDim.x) {
+                ok = false;
                 if (!wait_bar(&bar[CF_T1], ph[CF_T1], ctl, a.err, 34)) break;
                 tc::tc_fence_after();
 #pragma unroll
@@ -912,7 +916,8 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
                 for (int kk = 0; kk < R2 / 16; ++kk)                // G = A' EB
                     tc::mma_bf16(tb + colG, seq_kmaj(t1, 128, 0, kk), seq_mnmaj(eb, R2, 0, kk), id_G, kk > 0);
                 tc::mma_commit(&bar[CF_ACC5]);
-                ok = true;
+                // the next chunk's P runs while G is drained: region 0 held U, drained before A' arrived
+                ok = z + (int)gridDim.x >= a.Z || issue_p();
             }
         }
     } else {
@@ -1014,7 +1019,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
                 for (int ub = 0; ub < 2; ++ub) tc::tma_store_3d(&tm_go, sT2 + ub * 128 * 128, ub * 64, 0, z);
                 tc::bulk_commit();
             }
-            arrive(CF_TFREE);
+            __syncwarp();
         }
         if (threadIdx.x == 0) tc::bulk_wait0();
     }
