@@ -564,16 +564,20 @@ def stored_traffic(kernel, L):
         return None
 
 
+# The sources the chunked passes (K and V pass) are compiled from.
+PASS_SOURCES = ("common.cuh", "fwd_bf16.cu", "fwd_bf16.cuh", "tc.cuh", "tmap.cu", "tmap.cuh")
+
+
 def _source_digest():
-    """Digest of the CUDA sources; a stored DRAM-traffic figure is used only if it matches."""
+    """Digest of the sources of the chunked passes; a stored DRAM-traffic figure of a pass is used
+    only if it matches (any change to those files may change the pass kernels)."""
     import hashlib
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2606_09862_gb300", "csrc")
-    for fn in sorted(os.listdir(d)):
-        if fn.endswith((".cu", ".cuh")):
-            with open(os.path.join(d, fn), "rb") as f:
-                h.update(fn.encode())
-                h.update(f.read())
+    for fn in PASS_SOURCES:
+        with open(os.path.join(d, fn), "rb") as f:
+            h.update(fn.encode())
+            h.update(f.read())
     return h.hexdigest()[:16]
 
 

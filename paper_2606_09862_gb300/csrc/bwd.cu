@@ -1363,6 +1363,9 @@ BwdGeo bwd_geo(const OpDims &d) {
     return g;
 }
 
+// The fused chains hold their tiles in shared memory for 2M <= 128 and S <= 64.
+bool chain_fits(const BwdGeo &g) { return g.R2 >= 64 && g.R2 <= 128 && g.S >= 32 && g.S <= 64; }
+
 struct BwdWs {
     size_t tables, eb, phi, cphase, wb, P, Y, p, A, G, dG, dU, ds, dX, dP, dl, total;
 };
@@ -1377,17 +1380,19 @@ BwdWs bwd_ws(const OpDims &d, const BwdGeo &g) {
     w.phi = take(2 * (size_t)g.SP * g.R2);
     w.cphase = take(d.absolute ? 4 * (size_t)g.nch * g.M * 2 : 0);
     w.wb = take(2 * Z * 2 * g.R2 * g.D);
-    w.P = take(2 * Z * kC * kC);
-    w.Y = take(2 * Z * kC * g.R2);
+    // P, Y, dG, dU, ds and rowsum(dO o) go through memory only on the unfused route
+    const size_t u = chain_fits(g) ? 0 : 1;
+    w.P = take(u * 2 * Z * kC * kC);
+    w.Y = take(u * 2 * Z * kC * g.R2);
     w.p = take(2 * Z * kC * g.SP);
     w.A = take(2 * Z * kC * g.R2);
     w.G = take(2 * Z * kC * kC);
-    w.dG = take(2 * Z * kC * kC);
-    w.dU = take(2 * Z * kC * g.R2);
-    w.ds = take(2 * Z * kC * g.SP);
+    w.dG = take(u * 2 * Z * kC * kC);
+    w.dU = take(u * 2 * Z * kC * g.R2);
+    w.ds = take(u * 2 * Z * kC * g.SP);
     w.dX = take(2 * Z * kC * g.R2);
     w.dP = take(2 * Z * kC * kC);
-    w.dl = take(4 * Z * kC);
+    w.dl = take(u * 4 * Z * kC);
     w.total = off;
     return w;
 }
@@ -1515,9 +1520,6 @@ cudaError_t launch_adj_states(const BwdGeo &g, const CUtensorMap &mdx, const CUt
                                   : launch_adj_states_t<64, 2>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st);
     return cudaErrorInvalidValue;
 }
-
-// The fused chains hold their tiles in shared memory for 2M <= 128 and S <= 64.
-bool chain_fits(const BwdGeo &g) { return g.R2 >= 64 && g.R2 <= 128 && g.S >= 32 && g.S <= 64; }
 
 template <int R2, int S, int D>
 cudaError_t launch_chains_t(const BwdGeo &g, const ChainArgs &ca, const CUtensorMap &mq, const CUtensorMap &mk,

@@ -120,3 +120,34 @@ def test_host_buffer_forward_pipelined(orc):
     ref = orc.forward(q[:, heads], k[:, heads], v[:, heads], M, S, T, form="modes", want=want)
     got = o_host.float().numpy()[:, heads]
     assert rel(got[:, :, want], ref["o"][:, :, want]) <= TOL_BF16
+
+
+def test_host_buffer_forward_groups_cross_batches():
+    """B=3, H=5, L=12000 (ragged), d=128: 184 MB, so two head groups (heads 0-6, 7-14) that split a
+    batch element; equals the device-buffer forward to bf16 rounding."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    q, k, v = make_qkv(3, 5, 12000, 128, dtype="bf16", seed=23)
+    hq, hk, hv = (torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in (q, k, v))
+    o_host = bla.bla_forward_chunked_host(hq, hk, hv, 64, 64, 1024.0)
+    torch.cuda.synchronize()
+    bla.bla_device_error()
+    o_dev = bla.bla_forward_chunked(hq.to(dev), hk.to(dev), hv.to(dev), 64, 64, 1024.0)[0].cpu()
+    assert rel(o_host.float().numpy(), o_dev.float().numpy()) <= 1e-2
+
+
+def test_host_buffer_forward_f32_is_exact():
+    """fp32 host-buffer forward: each head is one CTA of the fp32 path whatever the grouping, so the
+    result equals the device-buffer forward bit for bit."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    q, k, v = make_qkv(2, 3, 300, 32, dtype="f32", seed=24)
+    hq, hk, hv = (torch.from_numpy(x).pin_memory() for x in (q, k, v))
+    o_host = bla.bla_forward_chunked_host(hq, hk, hv, 16, 16, 64.0, chunk=64)
+    torch.cuda.synchronize()
+    o_dev = bla.bla_forward_chunked(hq.to(dev), hk.to(dev), hv.to(dev), 16, 16, 64.0, chunk=64)[0].cpu()
+    assert torch.equal(o_host, o_dev)
