@@ -8,6 +8,8 @@
 #include <mutex>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 #include "bwd.cuh"
 #include "fwd_bf16.cuh"
@@ -98,6 +100,12 @@ constexpr double kPi = 3.14159265358979323846;
 constexpr int kDefaultChunkF32 = 64;
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// An NVTX range around each entry point (visible in Nsight timelines; free when no tool listens).
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
 
 // Common parameter checks; fills the derived dimensions.
 bla_status check_params(const bla_params *p, OpDims *d) {
@@ -291,6 +299,7 @@ size_t bla_workspace_bytes(const bla_params *p, int which) {
 bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k, const void *v, void *o,
                                float *lse, float *state_out, void *workspace, size_t ws_bytes, void *stream) {
     t_last_error[0] = 0;
+    NvtxRange nvtx("bla_forward_chunked");
     OpDims d;
     bla_status s = check_params(p, &d);
     if (s != BLA_OK) return s;
@@ -309,6 +318,7 @@ bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k
 bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const void *k, const void *v, void *o,
                                     void *workspace, size_t ws_bytes, void *stream) {
     t_last_error[0] = 0;
+    NvtxRange nvtx("bla_forward_chunked_host");
     OpDims d;
     bla_status s = check_params(p, &d);
     if (s != BLA_OK) return s;
@@ -358,6 +368,7 @@ bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const vo
 bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
                            float *state, void *o, void *workspace, size_t ws_bytes, void *stream) {
     t_last_error[0] = 0;
+    NvtxRange nvtx("bla_decode_step");
     OpDims d;
     bla_status s = check_params(p, &d);
     if (s != BLA_OK) return s;
@@ -384,6 +395,7 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
                         const void *dout, const float *lse, void *dq, void *dk, void *dv, void *workspace,
                         size_t ws_bytes, void *stream) {
     t_last_error[0] = 0;
+    NvtxRange nvtx("bla_backward");
     OpDims d;
     bla_status s = check_params(p, &d);
     if (s != BLA_OK) return s;
@@ -403,6 +415,7 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
 
 bla_status bla_selftest_wait_timeout(int limit_ms, void *stream) {
     t_last_error[0] = 0;
+    NvtxRange nvtx("bla_selftest_wait_timeout");
     if (limit_ms < 1 || limit_ms > 1000) return fail(BLA_ERR_INVALID, "limit_ms must be in [1, 1000] (got %d)", limit_ms);
     int *err = device_error_word();
     if (!err) return fail(BLA_ERR_CUDA, "device error word unavailable");

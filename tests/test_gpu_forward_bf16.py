@@ -151,3 +151,20 @@ def test_host_buffer_forward_f32_is_exact():
     torch.cuda.synchronize()
     o_dev = bla.bla_forward_chunked(hq.to(dev), hk.to(dev), hv.to(dev), 16, 16, 64.0, chunk=64)[0].cpu()
     assert torch.equal(o_host, o_dev)
+
+
+@pytest.mark.parametrize("L", [2, 127, 129])
+def test_bf16_outputs_all_written(orc, L):
+    """bf16 path around the 128-token chunk: o and lse prefilled with NaN must come back finite."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    q, k, v = make_qkv(1, 3, L, 64, dtype="bf16", seed=L)
+    out = torch.full((1, 3, L, 64), float("nan"), device=dev, dtype=torch.bfloat16)
+    o, lse, _ = bla.bla_forward_chunked(to_dev(q, dev, torch.bfloat16), to_dev(k, dev, torch.bfloat16),
+                                        to_dev(v, dev, torch.bfloat16), 32, 32, 256.0, out=out)
+    bla.bla_device_error()
+    assert torch.isfinite(o.float()).all() and torch.isfinite(lse).all()
+    ref = orc.forward(q, k, v, 32, 32, 256.0, form="modes")
+    assert rel(o.float().cpu().numpy(), ref["o"]) <= TOL_BF16

@@ -72,3 +72,24 @@ def test_empty_sequence():
     torch.cuda.synchronize()
     assert o.shape == (1, 2, 0, 8)
     assert float(st.abs().max()) == 0.0
+
+
+@pytest.mark.parametrize("L", [1, 2, 63, 65])
+@pytest.mark.parametrize("M,S,T", [(1, 1, 5.0), (4, 7, 7.0), (3, 5, 12.0)])
+def test_tiny_shapes_every_output_written(orc, L, M, S, T):
+    """Tiny shapes around the chunk boundary (C = 64): L in {1, 2, C-1, C+1}, down to one mode and
+    one slot; o is prefilled with NaN so that an element the kernel skips fails the test."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    q, k, v = make_qkv(2, 1, L, 8, dtype="f32", seed=L + 10 * M)
+    out = torch.full((2, 1, L, 8), float("nan"), device=dev)
+    o, lse, st = bla.bla_forward_chunked(to_dev(q, dev, torch.float32), to_dev(k, dev, torch.float32),
+                                         to_dev(v, dev, torch.float32), M, S, T, chunk=64, out=out,
+                                         want_state=True)
+    torch.cuda.synchronize()
+    assert torch.isfinite(o).all() and torch.isfinite(lse).all()
+    ref = orc.forward(q, k, v, M, S, T, form="naive", return_state=True)
+    assert rel(o.cpu().numpy(), ref["o"]) <= TOL_F32
+    assert rel(st.cpu().numpy(), ref["state"]) <= TOL_F32
