@@ -34,6 +34,9 @@
  *                         K~_t[j] = sum_{t'<=t} D_M(t - t' - Delta_j) k_t'.
  *   orc_forward_absolute  Alg. 1 ("Efficient recurrent BLA"), the time-rolling
  *                         cumulative-sum form of Sec. 3.2 (pins only).
+ *   orc_forward_decay     Alg. 1 with the state decay of Sec. 3.3: the previous
+ *                         slot state is multiplied by (1 - D_j(t)) before the token
+ *                         is added with weight D_j(t) (slot-space state [S][d]).
  *   orc_backward_parallel vector-Jacobian product of the parallel form, written out
  *                         by the chain rule (no paper counterpart; pinned to central
  *                         finite differences of orc_forward_naive by the tests).
@@ -349,6 +352,51 @@ static void head_absolute(const orc_cfg *c, const double *A, const double *B, co
     free(Kp); free(Vp); free(ip); free(s); free(p);
 }
 
+/* ------------------------------------------- Sec. 3.3: Alg. 1 with state decay
+ *
+ * The slot-space state of Alg. 1, where the previous state is multiplied by (1 - D_j(t))
+ * before the token's key (value) is added with Alg. 1's weight D_j(t):
+ *     K~[j] <- (1 - D_j(t)) K~[j] + D_j(t) k_t,      V~[j] likewise,
+ * D_j(t) = "interpolate"[j] = cos(t.modes) A^T + sin(t.modes) B^T (Eq. compressed_simplified)
+ * at the absolute token index t = pos0 + i.  Read-out as in Alg. 1: masked softmax of
+ * scale q_t . K~[j] over the slots, output sum_j p_j V~[j].
+ * State (per head, in/out, may be NULL for a zero start): [S][dk] then [S][dv].
+ */
+static void head_decay(const orc_cfg *c, const double *A, const double *B, const double *delta,
+                       const double *q, const double *k, const double *v, double *o, double *lse, double *st)
+{
+    int M = c->M, S = c->S, dk = c->dk, dv = c->dv;
+    double *own = st ? NULL : calloc((size_t)S * (dk + dv), sizeof(double));
+    double *Kp = st ? st : own, *Vp = Kp + (size_t)S * dk;
+    double *ip = malloc(sizeof(double) * S), *s = malloc(sizeof(double) * S), *p = malloc(sizeof(double) * S);
+    for (int i = 0; i < c->L; ++i) {
+        double t = (double)(c->pos0 + i);
+        for (int j = 0; j < S; ++j) {
+            double acc = 0.0;
+            for (int m = 0; m < M; ++m) acc += cos(t * m * c->w) * A[j * M + m] + sin(t * m * c->w) * B[j * M + m];
+            ip[j] = acc;
+        }
+        for (int j = 0; j < S; ++j) {
+            double keep = 1.0 - ip[j];
+            for (int e = 0; e < dk; ++e) Kp[j * dk + e] = keep * Kp[j * dk + e] + ip[j] * k[(size_t)i * dk + e];
+            for (int e = 0; e < dv; ++e) Vp[j * dv + e] = keep * Vp[j * dv + e] + ip[j] * v[(size_t)i * dv + e];
+        }
+        for (int j = 0; j < S; ++j) {
+            double acc = 0.0;
+            for (int e = 0; e < dk; ++e) acc += q[(size_t)i * dk + e] * Kp[j * dk + e];
+            s[j] = c->scale * acc;
+        }
+        double l = masked_softmax(S, s, delta, c->pos0 + i, p);
+        if (lse) lse[i] = l;
+        for (int e = 0; e < dv; ++e) {
+            double acc = 0.0;
+            for (int j = 0; j < S; ++j) acc += p[j] * Vp[j * dv + e];
+            o[(size_t)i * dv + e] = acc;
+        }
+    }
+    free(own); free(ip); free(s); free(p);
+}
+
 /* ------------------------------------ VJP of the parallel form (chain rule)
  *
  *   W[t,t',j] = D_M(t - t' - Delta_j)            (t' <= t; absolute form: D_M(t' - Delta_j))
@@ -457,6 +505,27 @@ int orc_forward(int form, int NH, int L, int dk, int dv, int M, int S, double T,
     }
     free(delta); free(A); free(B);
     return (form >= 0 && form <= 3) ? 0 : 3;
+}
+
+/* Alg. 1 with the state decay of Sec. 3.3.  State is [NH][S*(dk+dv)] (slot-space K~ then
+ * V~), in/out; NULL starts from zero and keeps nothing.  pos0 is the absolute index of
+ * token 0 (it sets both the phase of "interpolate" and the slot mask). */
+int orc_forward_decay(int NH, int L, int dk, int dv, int M, int S, double T, double omega, double scale,
+                      long long pos0, const double *q, const double *k, const double *v,
+                      double *o, double *lse, double *state)
+{
+    if (NH < 0 || L < 0 || dk < 1 || dv < 1 || M < 1 || S < 1 || pos0 < 0) return 1;
+    orc_cfg c = make_cfg(L, dk, dv, M, S, T, omega, scale, pos0);
+    double *delta = malloc(sizeof(double) * S), *A = malloc(sizeof(double) * S * M), *B = malloc(sizeof(double) * S * M);
+    orc_tables(M, S, T, omega, delta, A, B);
+    #pragma omp parallel for schedule(dynamic, 1)
+    for (int h = 0; h < NH; ++h) {
+        size_t ok = (size_t)h * L * dk, ov = (size_t)h * L * dv;
+        head_decay(&c, A, B, delta, q + ok, k + ok, v + ov, o + ov, lse ? lse + (size_t)h * L : NULL,
+                   state ? state + (size_t)h * S * (dk + dv) : NULL);
+    }
+    free(delta); free(A); free(B);
+    return 0;
 }
 
 int orc_backward(int form, int NH, int L, int dk, int dv, int M, int S, double T, double omega, double scale,

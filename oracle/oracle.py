@@ -9,6 +9,7 @@ Forms (see the C header for the paper passage each follows):
   "modes"     same recurrence, read-out through the modes (Eq. conv exchange of sums)
   "parallel"  closed form of Eq. (states) with translated Dirichlet kernels
   "absolute"  Alg. 1 (efficient recurrent BLA, time-rolling slots); pins only
+  forward_decay: Alg. 1 with the state decay of Sec. 3.3 (slot-space state)
 """
 import ctypes
 
@@ -37,6 +38,8 @@ def _configure(lib):
         [_dp] * 6 + [ctypes.c_void_p]
     lib.orc_backward.restype = ctypes.c_int
     lib.orc_backward.argtypes = [ctypes.c_int] * 7 + [ctypes.c_double] * 3 + [_dp] * 7
+    lib.orc_forward_decay.restype = ctypes.c_int
+    lib.orc_forward_decay.argtypes = [ctypes.c_int] * 6 + [ctypes.c_double] * 3 + [ctypes.c_longlong] + [_dp] * 6
     lib.orc_max_threads.restype = ctypes.c_int
     return lib
 
@@ -126,6 +129,33 @@ def forward(q, k, v, M, S, T, omega=0.0, scale=0.0, form="naive", state=None, po
             out["state"] = st.reshape(Bn, Hn, 2, M, 2, dk)
         else:
             out["state"] = st
+    return out
+
+
+def forward_decay(q, k, v, M, S, T, omega=0.0, scale=0.0, state=None, pos0=0, return_state=False):
+    """Alg. 1 with the state decay of Sec. 3.3: K~[j] <- (1 - D_j(t)) K~[j] + D_j(t) k_t.
+
+    q, k: [B, H, L, dk]; v: [B, H, L, dv].  ``state`` (optional) is the slot-space state
+    [B, H, 2, S, d] (K~ then V~; any shape with S*(dk+dv) values per head) and ``pos0`` the
+    absolute index of token 0.  Returns dict(o, lse, state) like ``forward``; the state is
+    [B, H, 2, S, d] when dk == dv.
+    """
+    q, k, v = _f64(q), _f64(k), _f64(v)
+    Bn, Hn, L, dk = q.shape
+    dv = v.shape[-1]
+    o = np.full((Bn, Hn, L, dv), np.nan)
+    lse = np.full((Bn, Hn, L), np.nan)
+    st = None
+    if state is not None or return_state:
+        st = np.zeros((Bn, Hn, S * (dk + dv))) if state is None else _f64(state).reshape(Bn, Hn, -1).copy()
+        assert st.shape[-1] == S * (dk + dv)
+    rc = _load().orc_forward_decay(Bn * Hn, L, dk, dv, int(M), int(S), float(T), float(omega), float(scale),
+                                   int(pos0), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse), _ptr(st))
+    if rc != 0:
+        raise ValueError("oracle decay forward rejected its arguments (code %d)" % rc)
+    out = {"o": o, "lse": lse, "state": None}
+    if st is not None:
+        out["state"] = st.reshape(Bn, Hn, 2, S, dk) if dk == dv else st
     return out
 
 

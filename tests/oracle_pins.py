@@ -326,6 +326,92 @@ def pin_state_handoff(orc):
                float(np.abs(a["o"] - full["o"][:, :, :L1]).max()))
 
 
+# ------------------------------------------------- P8: state decay (Sec. 3.3)
+
+def _latest_in_class(t, dj, T):
+    """Latest token u <= t with u = dj (mod T), for integers t >= dj."""
+    return int(t - ((t - dj) % T))
+
+
+def pin_decay_swa(orc):
+    """Sec. 3.3 at T = 2M-1: D_M(x) is 1 at x = 0 (mod 2M-1) and 0 at other integers, so the
+    decay overwrites slot j with k_t whenever t = Delta_j (mod 2M-1) and leaves it alone
+    otherwise.  Slot j then holds the latest token of its residue class; at S = 2M-1 the slots
+    hold exactly the last 2M-1 tokens, i.e. sliding-window softmax attention, which is checked
+    here against the textbook window [t-2M+2, t] as well."""
+    g = rng(41)
+    err = 0.0
+    for M, S, L, d in ((3, 5, 23, 3), (4, 7, 30, 2), (2, 3, 2, 2), (3, 4, 19, 3), (3, 8, 21, 2)):
+        T = 2 * M - 1
+        q, k, v = (g.standard_normal((1, 1, L, d)) for _ in range(3))
+        r = orc.forward_decay(q, k, v, M, S, float(T))
+        delta = np.round(np.arange(S) * T / S).astype(int)       # half to even, as the grid reading
+        for t in range(L):
+            valid = t >= delta
+            rows = np.array([_latest_in_class(t, dj, T) if ok else 0 for dj, ok in zip(delta, valid)])
+            s = k[0, 0, rows] @ q[0, 0, t] / np.sqrt(d)
+            p, lse = _softmax_masked(s[None], valid[None])
+            err = _worst(err, float(np.abs(r["o"][0, 0, t] - p[0] @ v[0, 0, rows]).max()),
+                         float(abs(r["lse"][0, 0, t] - lse[0])))
+            if S == T:
+                win = np.arange(max(0, t - T + 1), t + 1)
+                sw = k[0, 0, win] @ q[0, 0, t] / np.sqrt(d)
+                pw = np.exp(sw - sw.max())
+                pw /= pw.sum()
+                err = _worst(err, float(np.abs(r["o"][0, 0, t] - pw @ v[0, 0, win]).max()))
+    return err
+
+
+def pin_decay_closed_form(orc):
+    """Unrolled decay recurrence: slot j of token t holds
+    sum_{u<=t} D_j(u) prod_{u<x<=t} (1 - D_j(x)) k_u with D_j(x) = D_M(x - Delta_j), evaluated
+    here with the sine-ratio D_M, for periods above 2M-1 and an explicit omega."""
+    g = rng(43)
+    err = 0.0
+    for M, S, T, om, L, d in ((3, 4, 10.0, 0.0, 17, 3), (4, 6, 21.0, 0.0, 15, 2), (2, 5, 9.0, 0.41, 13, 3)):
+        q, k, v = (g.standard_normal((1, 1, L, d)) for _ in range(3))
+        r = orc.forward_decay(q, k, v, M, S, T, omega=om, return_state=True)
+        w = om if om > 0 else 2 * np.pi / T
+        delta = np.round(np.arange(S) * T / S)
+        Dx = dirichlet_sine_ratio(M, w, np.arange(L)[None, :] - delta[:, None])   # [S, L]
+        for t in range(L):
+            W = np.zeros((S, t + 1))
+            for u in range(t + 1):
+                W[:, u] = Dx[:, u] * np.prod(1.0 - Dx[:, u + 1: t + 1], axis=1)
+            Ks, Vs = W @ k[0, 0, : t + 1], W @ v[0, 0, : t + 1]
+            valid = t >= delta
+            p, lse = _softmax_masked((Ks @ q[0, 0, t] / np.sqrt(d))[None], valid[None])
+            err = _worst(err, float(np.abs(r["o"][0, 0, t] - p[0] @ Vs).max()),
+                         float(abs(r["lse"][0, 0, t] - lse[0])))
+        err = _worst(err, float(np.abs(r["state"][0, 0, 0] - Ks).max()),
+                     float(np.abs(r["state"][0, 0, 1] - Vs).max()))
+    return err
+
+
+def pin_decay_single_mode(orc):
+    """M = 1: D_1 = 1 everywhere, so the decay empties every slot and refills it with the current
+    token; the output is v_t itself."""
+    g = rng(47)
+    q, k, v = (g.standard_normal((2, 2, 11, 3)) for _ in range(3))
+    r = orc.forward_decay(q, k, v, 1, 3, 7.0)
+    return float(np.abs(r["o"] - v).max())
+
+
+def pin_decay_handoff(orc):
+    """Prefill of L1 tokens, then the rest from the returned slot state with pos0 = L1 (which sets
+    both the phase of D_j and the slot mask), equals one pass."""
+    g = rng(53)
+    M, S, T, L1, L2, d = 3, 5, 13.0, 4, 12, 3
+    q, k, v = (g.standard_normal((1, 2, L1 + L2, d)) for _ in range(3))
+    full = orc.forward_decay(q, k, v, M, S, T, return_state=True)
+    a = orc.forward_decay(q[:, :, :L1], k[:, :, :L1], v[:, :, :L1], M, S, T, return_state=True)
+    b = orc.forward_decay(q[:, :, L1:], k[:, :, L1:], v[:, :, L1:], M, S, T, state=a["state"], pos0=L1,
+                          return_state=True)
+    return _worst(float(np.abs(b["o"] - full["o"][:, :, L1:]).max()),
+                  float(np.abs(b["state"] - full["state"]).max()),
+                  float(np.abs(a["o"] - full["o"][:, :, :L1]).max()))
+
+
 ALL_PINS = {
     "dirichlet_identity": (pin_dirichlet_identity, 1e-12),
     "dirichlet_samples": (pin_dirichlet_samples, 1e-13),
@@ -341,4 +427,8 @@ ALL_PINS = {
     "absolute_bruteforce": (pin_absolute_bruteforce, 1e-11),
     "backward_fd_absolute": (pin_backward_fd_absolute, 1e-6),
     "state_handoff": (pin_state_handoff, 1e-12),
+    "decay_swa": (pin_decay_swa, 1e-12),
+    "decay_closed_form": (pin_decay_closed_form, 1e-11),
+    "decay_single_mode": (pin_decay_single_mode, 1e-13),
+    "decay_handoff": (pin_decay_handoff, 1e-12),
 }

@@ -38,6 +38,11 @@ MUTANTS = {
     "dirichlet_no_factor2": ("acc += 2.0 / n * cos(m * w * x);", "acc += 1.0 / n * cos(m * w * x);"),
     "absolute_interp_sign": ("+ sin(t * m * c->w) * B[j * M + m];", "- sin(t * m * c->w) * B[j * M + m];"),
     "absolute_backward_lag_weight": ("return absolute ? u - dj : t - u - dj;", "return t - u - dj;"),
+    "decay_after_add": ("Kp[j * dk + e] = keep * Kp[j * dk + e] + ip[j] * k[(size_t)i * dk + e];",
+                        "Kp[j * dk + e] = keep * (Kp[j * dk + e] + ip[j] * k[(size_t)i * dk + e]);"),
+    "decay_relative_phase": ("double t = (double)(c->pos0 + i);", "double t = (double)i;"),
+    "decay_factor_sign": ("double keep = 1.0 - ip[j];", "double keep = 1.0 + ip[j];"),
+    "decay_value_not_decayed": ("Vp[j * dv + e] = keep * Vp[j * dv + e] + ip[j]", "Vp[j * dv + e] = Vp[j * dv + e] + ip[j]"),
 }
 
 
