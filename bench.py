@@ -512,6 +512,8 @@ def measure_configs(bla, torch, dev, stream, peaks, iters=20, only=None, warm=3)
                                          (w.B, w.H, w.L, w.d, w.M, w.S, w.T, w.chunk)}
     if not only or "lm_block_f32" in only:
         out["lm_block_f32"] = measure_block(bla, torch, dev, timed)
+    if not only or "decay_bf16_lm" in only:
+        out["decay_bf16_lm"] = measure_decay(bla, torch, dev, timed, peaks)
     del flush
     torch.cuda.empty_cache()
     return out
@@ -542,6 +544,49 @@ def measure_block(bla, torch, dev, timed):
     ms_mix = timed(mixing)
     return {"layer_ms": ms, "mixing_ms": ms_mix, "tokens_per_s": w.B * w.L / (ms / 1000.0),
             "shape": "B=%d L=%d d_model=%d H=%d d=%d M=%d S=%d T=%g fp32" % (w.B, w.L, dm, w.H, w.d, w.M, w.S, w.T)}
+
+
+# Nominal fp32 SIMT peak of the part: 152 SMs x 128 fp32 lanes x 2 flops (FMA) x 2.07 GHz.
+FP32_SIMT_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def measure_decay(bla, torch, dev, timed, peaks):
+    """The state decay of Sec. 3.3 (absolute form): the LM-layer prefill (B=8, H=8, L=4096, d=128,
+    M=64, S=64, T=1024, bf16) and one decode step at B=256, H=16, d=128, M=128, S=128, T=4096,
+    pos = 4096, from a random fp32 slot state.  The forward is a scan on the CUDA cores: its flops
+    are 10 S d per token and head (state update 3 + score 2 for K and for V, FMA = 2); the decode
+    reads and writes the whole slot state once."""
+    from paper_2606_09862_gb300.inputs import WORKLOADS, make_decode_step, make_qkv, make_slot_state
+    w = WORKLOADS["decay_bf16_lm"]
+    q, k, v = (torch.from_numpy(x).to(torch.bfloat16).to(dev) for x in make_qkv(w.B, w.H, w.L, w.d, "bf16", seed=0))
+    par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16, phase_mode="absolute")
+    ws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_DECAY_FORWARD), dtype=torch.uint8, device=dev)
+    o = torch.empty_like(v)
+    ms = timed(lambda: bla.bla_decay_forward(q, k, v, w.M, w.S, w.T, workspace=ws, out=o))
+    flops = 10.0 * w.B * w.H * w.L * w.S * w.d
+    tf = flops / (ms / 1000.0) / 1e12
+    res = {"forward": {"ms": ms, "tokens_per_s": w.B * w.L / (ms / 1000.0), "tflops_fp32": tf, "flops": flops,
+                       "bound": "alu", "frac_alu": tf / FP32_SIMT_PEAK_TFLOPS,
+                       "alu_peak_tflops": FP32_SIMT_PEAK_TFLOPS},
+           "shape": "B=%d H=%d L=%d d=%d M=%d S=%d T=%d bf16 absolute+decay" % (w.B, w.H, w.L, w.d, w.M, w.S, w.T)}
+    del q, k, v, ws, o
+    wd = WORKLOADS["decay_decode_bf16"]
+    qd, kd, vd = (torch.from_numpy(x).to(torch.bfloat16).to(dev)
+                  for x in make_decode_step(0, wd.B, wd.H, wd.d, "bf16", seed=0))
+    st = torch.from_numpy(make_slot_state(wd.B, wd.H, wd.S, wd.d, wd.state_std, seed=0)).to(dev)
+    pard = bla.make_params(wd.B, wd.H, 1, wd.d, wd.d, wd.M, wd.S, wd.T, dtype=torch.bfloat16, phase_mode="absolute")
+    wsd = torch.empty(max(bla.bla_workspace_bytes(pard, bla.BLA_WS_DECAY_DECODE), 1), dtype=torch.uint8, device=dev)
+    od = torch.empty((wd.B, wd.H, wd.d), dtype=torch.bfloat16, device=dev)
+    ms_d = timed(lambda: bla.bla_decay_decode_step(qd, kd, vd, st, wd.decode_pos0, wd.M, wd.S, wd.T, workspace=wsd,
+                                                   out=od))
+    nbytes = 2 * st.numel() * 4 + 4 * wd.B * wd.H * wd.d * 2
+    gbs = nbytes / (ms_d / 1000.0) / 1e9
+    res["decode"] = {"ms": ms_d, "tokens_per_s": wd.B / (ms_d / 1000.0), "gbs": gbs, "bytes": nbytes,
+                     "bound": "hbm", "frac_hbm": gbs / peaks["hbm_gbs"],
+                     "shape": "B=%d H=%d d=%d M=%d S=%d T=%d pos=%d bf16, fp32 slot state" %
+                              (wd.B, wd.H, wd.d, wd.M, wd.S, wd.T, wd.decode_pos0)}
+    del qd, kd, vd, st, wsd, od
+    return res
 
 
 def stored_traffic(kernel, L):

@@ -86,7 +86,10 @@ typedef struct {
 typedef enum { BLA_PHASE_LAG = 0, BLA_PHASE_ABSOLUTE = 1 } bla_phase_mode;
 
 /* Which entry point a workspace size is asked for. */
-typedef enum { BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2, BLA_WS_FORWARD_HOST = 3 } bla_ws_kind;
+typedef enum {
+    BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2, BLA_WS_FORWARD_HOST = 3,
+    BLA_WS_DECAY_FORWARD = 4, BLA_WS_DECAY_DECODE = 5
+} bla_ws_kind;
 
 /*
  * Bytes of device workspace the entry point `which` (a bla_ws_kind) needs for
@@ -177,6 +180,45 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
                         const void *o, const void *dout, const float *lse,
                         void *dq, void *dk, void *dv, void *workspace, size_t ws_bytes, void *stream);
 
+/* ---------------------------------------------------------------- state decay (Sec. 3.3)
+ * Alg. 1 (the absolute form) with the decay of Sec. 3.3.  The state is Alg. 1's slot-space state,
+ * fp32 [B][H][2 (K~ then V~)][S][d], and token t (absolute index) updates every slot j as
+ *     K~[j] <- (1 - D_j(t)) K~[j] + D_j(t) k_t,      V~[j] likewise,
+ * with D_j(t) = D_M(t - Delta_j) the weight Alg. 1 adds the token with ("interpolate", Eq.
+ * compressed_simplified); then o_t = softmax_j(scale q_t . K~[j], slots with t >= Delta_j) . V~.
+ * At T = 2M-1 the decay keeps in slot j the latest token t = Delta_j (mod 2M-1), which at S = 2M-1
+ * is sliding-window attention over the last 2M-1 tokens.  Shared requirements: phase_mode =
+ * BLA_PHASE_ABSOLUTE (the decay is defined on that form's slots; BLA_PHASE_LAG returns
+ * BLA_ERR_UNSUPPORTED), d_k = d_v in {32, 64, 128} and S <= 256 (else BLA_ERR_UNSUPPORTED). */
+
+/*
+ * Forward over L tokens, continuing from `state_in` (NULL = zero state) at absolute index pos0
+ * (>= 0; it sets the phase of D_j and the slot mask; 0 for a fresh sequence).
+ *   o          [B][H][L][d_v] (device), dtype of the inputs.
+ *   lse        optional [B][H][L] fp32 (device) or NULL.
+ *   state_in   optional slot-space state (device) the tokens continue from, or NULL.
+ *   state_out  optional slot-space state after the last token (device), or NULL; it may be the
+ *              same pointer as state_in (updated in place) but must not overlap it otherwise.
+ *   workspace  device scratch of >= bla_workspace_bytes(p, BLA_WS_DECAY_FORWARD) bytes (it holds
+ *              the B*H*S*L fp32 slot scores and a table of L + T values of D_M).
+ * dtype BLA_F32 or BLA_BF16 (fp32 state and arithmetic either way).  A period with L + T above
+ * 2^30 returns BLA_ERR_UNSUPPORTED.
+ */
+bla_status bla_decay_forward(const bla_params *p, long long pos0, const void *q, const void *k, const void *v,
+                             void *o, float *lse, const float *state_in, float *state_out, void *workspace,
+                             size_t ws_bytes, void *stream);
+
+/*
+ * One decode step of the decayed form for B*H sequences at absolute index pos (>= 0).
+ *   q, k, v    [B][H][d_k] / [B][H][d_k] / [B][H][d_v] (device), dtype p->dtype.
+ *   state      slot-space state (device), read and updated in place.
+ *   o          [B][H][d_v] (device).
+ *   workspace  device scratch of >= bla_workspace_bytes(p, BLA_WS_DECAY_DECODE) bytes.
+ * p->L is ignored.  A prefill of L tokens by bla_decay_forward hands over with pos = L.
+ */
+bla_status bla_decay_decode_step(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
+                                 float *state, void *o, void *workspace, size_t ws_bytes, void *stream);
+
 /* ---------------------------------------------------------------- instrumentation
  * (no paper counterpart: measurement support for benchmarks and tests)
  * Kernels of this library, as counted and timed below. */
@@ -190,6 +232,7 @@ typedef enum {
     BLA_K_FWD_F32,         /* fp32 chunked forward (CUDA cores) */
     BLA_K_DECODE,          /* decode step */
     BLA_K_BWD,             /* backward kernels */
+    BLA_K_DECAY,           /* state-decay kernels (table, K scan, lse, V scan, decode) */
     BLA_K_COUNT
 } bla_kernel_id;
 

@@ -17,16 +17,17 @@ LIB_PATH = os.path.join(_HERE, "libbla_gb300.so")
 BLA_OK, BLA_ERR_INVALID, BLA_ERR_UNSUPPORTED, BLA_ERR_CUDA, BLA_ERR_TIMEOUT = range(5)
 BLA_F32, BLA_BF16 = 0, 1
 BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE, BLA_WS_FORWARD_HOST = 0, 1, 2, 3
+BLA_WS_DECAY_FORWARD, BLA_WS_DECAY_DECODE = 4, 5
 BLA_PHASE_LAG, BLA_PHASE_ABSOLUTE = 0, 1
 PHASE_MODES = {"lag": BLA_PHASE_LAG, "absolute": BLA_PHASE_ABSOLUTE}
 
 EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
             "bla_device_error", "bla_status_string", "bla_last_error_string", "bla_kernel_launches",
             "bla_profile_enable", "bla_profile_collect", "bla_decode_step_noalloc", "bla_forward_chunked_host",
-            "bla_selftest_wait_timeout")
+            "bla_selftest_wait_timeout", "bla_decay_forward", "bla_decay_decode_step")
 
 # bla_kernel_id
-KERNELS = ("tables", "tables_bf16", "prepass", "scan", "kpass", "vpass", "fwd_f32", "decode", "bwd")
+KERNELS = ("tables", "tables_bf16", "prepass", "scan", "kpass", "vpass", "fwd_f32", "decode", "bwd", "decay")
 
 
 class BlaError(RuntimeError):
@@ -68,6 +69,10 @@ def load():
     lib.bla_decode_step.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_decode_step_noalloc.restype = ctypes.c_int
     lib.bla_decode_step_noalloc.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp]
+    lib.bla_decay_forward.restype = ctypes.c_int
+    lib.bla_decay_forward.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_decay_decode_step.restype = ctypes.c_int
+    lib.bla_decay_decode_step.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_backward.restype = ctypes.c_int
     lib.bla_backward.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_device_error.restype = ctypes.c_int
@@ -203,6 +208,43 @@ def bla_backward(q, k, v, o, dout, lse, M, S, window, omega=0.0, scale=0.0, work
     _check(load().bla_backward(ctypes.byref(p), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout), _ptr(lse),
                                _ptr(dq), _ptr(dkk), _ptr(dvv), _ptr(ws), n, _stream(stream)))
     return dq, dkk, dvv
+
+
+def bla_decay_forward(q, k, v, M, S, window, omega=0.0, scale=0.0, pos0=0, state=None, want_lse=True,
+                      want_state=False, workspace=None, out=None, stream=None, phase_mode="absolute"):
+    """Forward of Alg. 1 with the state decay of Sec. 3.3 over q, k: [B,H,L,d], v: [B,H,L,d].
+
+    ``state`` (optional, [B,H,2,S,d] fp32) is the slot-space state the tokens continue from at
+    absolute index ``pos0``.  Returns (o, lse or None, final state or None); with want_state and
+    a given ``state``, the state is updated in place and returned."""
+    _need_cuda(q, k, v, state)
+    B, H, L, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, L, dk, dv, M, S, window, omega, 0, scale, q.dtype, phase_mode)
+    o = out if out is not None else torch.empty((B, H, L, dv), dtype=q.dtype, device=q.device)
+    lse = torch.empty((B, H, L), dtype=torch.float32, device=q.device) if want_lse else None
+    st_out = None
+    if want_state:
+        st_out = state if state is not None else torch.empty((B, H, 2, S, dk), dtype=torch.float32, device=q.device)
+    ws, n = _workspace(p, BLA_WS_DECAY_FORWARD, q.device, workspace)
+    _check(load().bla_decay_forward(ctypes.byref(p), int(pos0), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(lse),
+                                    _ptr(state), _ptr(st_out), _ptr(ws), n, _stream(stream)))
+    return o, lse, st_out
+
+
+def bla_decay_decode_step(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.0, workspace=None, out=None,
+                          stream=None, phase_mode="absolute"):
+    """One decode step of the decayed form; q, k, v: [B,H,d]; state [B,H,2,S,d] fp32 is updated in
+    place.  Returns o."""
+    _need_cuda(q, k, v, state)
+    B, H, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, 1, dk, dv, M, S, window, omega, 0, scale, q.dtype, phase_mode)
+    o = out if out is not None else torch.empty((B, H, dv), dtype=q.dtype, device=q.device)
+    ws, n = _workspace(p, BLA_WS_DECAY_DECODE, q.device, workspace)
+    _check(load().bla_decay_decode_step(ctypes.byref(p), int(pos), _ptr(q), _ptr(k), _ptr(v), _ptr(state), _ptr(o),
+                                        _ptr(ws), n, _stream(stream)))
+    return o
 
 
 def bla_device_error(stream=None):

@@ -158,6 +158,21 @@ size_t ws_forward(const bla_params *p, const OpDims &d) {
 
 size_t ws_decode(const OpDims &d) { return tables_bytes(d, 0); }
 
+// Checks shared by the state-decay entry points (Sec. 3.3 on Alg. 1's slot state).
+bla_status check_decay(const bla_params *p, OpDims *d, bool forward) {
+    bla_status s = check_params(p, d);
+    if (s != BLA_OK) return s;
+    if (p->phase_mode != BLA_PHASE_ABSOLUTE)
+        return fail(BLA_ERR_UNSUPPORTED, "the state decay is defined on the absolute form's slots (Alg. 1): "
+                                         "phase_mode must be BLA_PHASE_ABSOLUTE");
+    if (d->dk != d->dv || (d->dk != 32 && d->dk != 64 && d->dk != 128))
+        return fail(BLA_ERR_UNSUPPORTED, "the decay path needs d_k = d_v in {32, 64, 128} (got %d, %d)", d->dk, d->dv);
+    if (d->S > 256) return fail(BLA_ERR_UNSUPPORTED, "the decay path needs S <= 256 (got %d)", d->S);
+    if (forward && decay_table_entries(*d) > (size_t(1) << 30))
+        return fail(BLA_ERR_UNSUPPORTED, "L + T too large for the decay table (L=%d, T=%g)", d->L, d->T);
+    return BLA_OK;
+}
+
 // bla_selftest_wait_timeout: a bounded wait on a barrier nothing arrives at (kernel id 15 in the
 // error word).
 __global__ void k_wait_selftest(uint64_t limit_ns, int *err) {
@@ -292,6 +307,8 @@ size_t bla_workspace_bytes(const bla_params *p, int which) {
     case BLA_WS_DECODE: return ws_decode(d);
     case BLA_WS_FORWARD_HOST: return ws_forward_host(p, d);
     case BLA_WS_BACKWARD: return bwd_workspace_bytes(d);
+    case BLA_WS_DECAY_FORWARD: return check_decay(p, &d, true) == BLA_OK ? decay_workspace_bytes(d, false) : 0;
+    case BLA_WS_DECAY_DECODE: return check_decay(p, &d, false) == BLA_OK ? decay_workspace_bytes(d, true) : 0;
     default: return 0;
     }
 }
@@ -388,6 +405,43 @@ bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, co
     if (e != cudaSuccess) return cuda_fail(e, "table build");
     e = launch_decode(d, pos, t, q, k, v, state, o, st);
     if (e != cudaSuccess) return cuda_fail(e, "decode launch");
+    return BLA_OK;
+}
+
+bla_status bla_decay_forward(const bla_params *p, long long pos0, const void *q, const void *k, const void *v,
+                             void *o, float *lse, const float *state_in, float *state_out, void *workspace,
+                             size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    NvtxRange nvtx("bla_decay_forward");
+    OpDims d;
+    bla_status s = check_decay(p, &d, true);
+    if (s != BLA_OK) return s;
+    if (pos0 < 0) return fail(BLA_ERR_INVALID, "pos0 must be >= 0 (got %lld)", pos0);
+    if (!q || !k || !v || !o) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)) ||
+        (state_in && !aligned16(state_in)) || (state_out && !aligned16(state_out)))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    if ((s = check_ws(workspace, ws_bytes, decay_workspace_bytes(d, false))) != BLA_OK) return s;
+    cudaError_t e = launch_decay_forward(d, pos0, q, k, v, o, lse, state_in, state_out, workspace,
+                                         reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "decay forward launch");
+    return BLA_OK;
+}
+
+bla_status bla_decay_decode_step(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
+                                 float *state, void *o, void *workspace, size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    NvtxRange nvtx("bla_decay_decode_step");
+    OpDims d;
+    bla_status s = check_decay(p, &d, false);
+    if (s != BLA_OK) return s;
+    if (pos < 0) return fail(BLA_ERR_INVALID, "pos must be >= 0 (got %lld)", pos);
+    if (!q || !k || !v || !state || !o) return fail(BLA_ERR_INVALID, "q, k, v, state and o must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(state) || !aligned16(o))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    if ((s = check_ws(workspace, ws_bytes, decay_workspace_bytes(d, true))) != BLA_OK) return s;
+    cudaError_t e = launch_decay_decode(d, pos, q, k, v, state, o, workspace, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "decay decode launch");
     return BLA_OK;
 }
 

@@ -57,6 +57,13 @@ WORKLOADS = {
     "decode_bf16": Workload("decode_bf16", "bf16", B=256, H=16, L=1, d=128, M=128, S=128, T=4096,
                             chunk=1, decode_steps=1024, decode_pos0=4096, state_std=0.1,
                             notes="single-token decode, fp32 state ~ N(0, 0.1^2)"),
+    # the state decay of Sec. 3.3 (absolute form): the LM-layer prefill shape, and the decode shape
+    # with a random slot-space state [B, H, 2, S, d]
+    "decay_bf16_lm": Workload("decay_bf16_lm", "bf16", B=8, H=8, L=4096, d=128, M=64, S=64, T=1024,
+                              chunk=128, notes="LM-layer shape with state decay; q,k,v ~ N(0,1)/sqrt(d)"),
+    "decay_decode_bf16": Workload("decay_decode_bf16", "bf16", B=256, H=16, L=1, d=128, M=128, S=128,
+                                  T=4096, chunk=1, decode_steps=1, decode_pos0=4096, state_std=0.1,
+                                  notes="decode with state decay, fp32 slot state ~ N(0, 0.1^2)"),
 }
 
 
@@ -126,6 +133,12 @@ def make_state(B, H, M, d, std=0.1, seed=0):
     st = (g["state"].standard_normal((B, H, 2, M, 2, d)) * std).astype(np.float32)
     st[:, :, :, 0, 1, :] = 0.0
     return st
+
+
+def make_slot_state(B, H, S, d, std=0.1, seed=0):
+    """Random fp32 slot-space state [B, H, 2, S, d] ~ N(0, std^2) (the decayed form's state)."""
+    g = _streams(seed)
+    return (g["state"].standard_normal((B, H, 2, S, d)) * std).astype(np.float32)
 
 
 def make_decode_step(step, B, H, d, dtype="bf16", seed=0):

@@ -142,3 +142,31 @@ def test_product_path_does_not_import_oracle():
                 text = open(os.path.join(dirpath, fn)).read()
                 assert "import oracle" not in text and "from oracle" not in text, fn
                 assert "bla_oracle" not in text and "liborc" not in text, fn
+
+
+def test_decay_argument_checks(lib):
+    """The state-decay entry points refuse the lag form, unsupported shapes and bad positions on the
+    host, and size their workspace from the B*H*S*L slot scores."""
+    from paper_2606_09862_gb300 import bla
+    ab = bla.BLA_PHASE_ABSOLUTE
+
+    def fwd(p, pos0=0, ws=1 << 30):
+        return lib.bla_decay_forward(ctypes.byref(p), pos0, FAKE, FAKE, FAKE, FAKE, None, None, None, FAKE, ws, None)
+
+    def dec(p, pos=0):
+        return lib.bla_decay_decode_step(ctypes.byref(p), pos, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30, None)
+
+    assert fwd(_params()) == bla.BLA_ERR_UNSUPPORTED                     # lag form
+    assert dec(_params()) == bla.BLA_ERR_UNSUPPORTED
+    assert fwd(_params(phase_mode=ab), pos0=-1) == bla.BLA_ERR_INVALID
+    assert dec(_params(phase_mode=ab), pos=-1) == bla.BLA_ERR_INVALID
+    assert fwd(_params(phase_mode=ab, d_k=48, d_v=48)) == bla.BLA_ERR_UNSUPPORTED
+    assert fwd(_params(phase_mode=ab, d_k=32, d_v=64)) == bla.BLA_ERR_UNSUPPORTED
+    assert fwd(_params(phase_mode=ab, S=300, window=1000.0)) == bla.BLA_ERR_UNSUPPORTED
+    assert fwd(_params(phase_mode=ab), ws=8) == bla.BLA_ERR_INVALID
+    assert lib.bla_decay_forward(ctypes.byref(_params(phase_mode=ab)), 0, None, FAKE, FAKE, FAKE, None, None, None,
+                                 FAKE, 1 << 30, None) == bla.BLA_ERR_INVALID
+    p = _params(phase_mode=ab, B=2, H=3, L=100, S=8, window=40.0)
+    assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_FORWARD) >= 2 * 3 * 8 * 100 * 4
+    assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_DECODE) > 0
+    assert lib.bla_workspace_bytes(ctypes.byref(_params()), bla.BLA_WS_DECAY_FORWARD) == 0

@@ -1,0 +1,159 @@
+"""The state decay of Sec. 3.3 (Alg. 1's slot state multiplied by 1 - D_j(t) before each token is
+added) on the GPU, through the C ABI, against the oracle's decayed Alg. 1."""
+import numpy as np
+import pytest
+
+from gpu_util import TOL_BF16, TOL_F32, rel, require_cuda, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+def gpu_forward(q, k, v, M, S, T, dtype, pos0=0, state=None):
+    import torch
+    from paper_2606_09862_gb300 import bla
+    dev = require_cuda()
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    st = None if state is None else to_dev(state, dev, torch.float32)
+    o, lse, st = bla.bla_decay_forward(to_dev(q, dev, tdt), to_dev(k, dev, tdt), to_dev(v, dev, tdt), M, S, T,
+                                       pos0=pos0, state=st, want_state=True)
+    bla.bla_device_error()
+    return o.float().cpu().numpy(), lse.cpu().numpy(), st.cpu().numpy()
+
+
+def check(got, ref, tol, lse_tol):
+    o, lse, st = got
+    assert rel(o, ref["o"]) <= tol, rel(o, ref["o"])
+    assert np.abs(lse - ref["lse"]).max() <= lse_tol
+    assert rel(st, ref["state"]) <= tol, rel(st, ref["state"])
+
+
+@pytest.mark.parametrize("B,H,L,d,M,S,T", [
+    (1, 2, 203, 32, 16, 16, 64.0),     # ragged tails of the 32-token score and 16-token value tiles
+    (2, 1, 100, 64, 4, 7, 7.0),        # T = S = 2M-1: sliding-window attention over 7 tokens
+    (1, 2, 77, 128, 32, 32, 256.0),
+    (1, 1, 50, 64, 8, 200, 300.0),     # 25 slot groups, a partial block of slot warps
+    (1, 1, 1, 32, 4, 5, 9.0),          # a single token
+])
+def test_f32_forward(orc, B, H, L, d, M, S, T):
+    from paper_2606_09862_gb300.inputs import make_qkv
+    q, k, v = make_qkv(B, H, L, d, dtype="f32", seed=L + S)
+    check(gpu_forward(q, k, v, M, S, T, "f32"), orc.forward_decay(q, k, v, M, S, T, return_state=True),
+          TOL_F32, 1e-4)
+
+
+@pytest.mark.parametrize("B,H,L,d,M,S,T", [
+    (1, 2, 300, 128, 64, 64, 1024.0),   # the LM-layer (M, S, T), shortened
+    (2, 2, 257, 64, 32, 32, 256.0),
+    (1, 1, 129, 128, 128, 128, 4096.0),
+    (1, 1, 64, 128, 8, 256, 512.0),     # S = 256, the largest slot count (1024-thread value blocks)
+])
+def test_bf16_forward(orc, B, H, L, d, M, S, T):
+    from paper_2606_09862_gb300.inputs import make_qkv
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=L + M)
+    check(gpu_forward(q, k, v, M, S, T, "bf16"), orc.forward_decay(q, k, v, M, S, T, return_state=True),
+          TOL_BF16, 5e-2)
+
+
+def test_bf16_sharp_softmax(orc):
+    from paper_2606_09862_gb300.inputs import make_qkv
+    q, k, v = make_qkv(1, 2, 400, 128, dtype="bf16", seed=3, sharp=True)
+    check(gpu_forward(q, k, v, 64, 64, 1024.0, "bf16"),
+          orc.forward_decay(q, k, v, 64, 64, 1024.0, return_state=True), TOL_BF16, 5e-2)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_prefill_continue_and_decode(orc, dtype):
+    """Prefill of L1 tokens, a second forward from its state at pos0 = L1, and decode steps from
+    the prefill's state at pos = L1, L1 + 1, ... all equal one pass over the whole sequence."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    B, H, L, L1, d, M, S, T = 2, 2, 90, 61, 64, 16, 24, 100.0
+    q, k, v = make_qkv(B, H, L, d, dtype=dtype, seed=7)
+    tol = TOL_F32 if dtype == "f32" else TOL_BF16
+    full = orc.forward_decay(q, k, v, M, S, T, return_state=True)
+    o1, _, st1 = gpu_forward(q[:, :, :L1], k[:, :, :L1], v[:, :, :L1], M, S, T, dtype)
+    o2, _, st2 = gpu_forward(q[:, :, L1:], k[:, :, L1:], v[:, :, L1:], M, S, T, dtype, pos0=L1, state=st1)
+    assert rel(np.concatenate([o1, o2], 2), full["o"]) <= tol
+    assert rel(st2, full["state"]) <= tol
+    st = to_dev(st1, dev, torch.float32)
+    outs = []
+    for t in range(L1, L):
+        o = bla.bla_decay_decode_step(to_dev(q[:, :, t], dev, tdt), to_dev(k[:, :, t], dev, tdt),
+                                      to_dev(v[:, :, t], dev, tdt), st, t, M, S, T)
+        outs.append(o.float().cpu().numpy())
+    bla.bla_device_error()
+    assert rel(np.stack(outs, 2), full["o"][:, :, L1:]) <= tol
+    assert rel(st.cpu().numpy(), full["state"]) <= tol
+
+
+def test_swa_limit_decode(orc):
+    """Decode at T = S = 2M-1 from a zero state reproduces sliding-window attention (the oracle's
+    pinned limit) step by step, including the first 2M-2 steps where slots are still masked."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    B, H, L, d, M = 1, 3, 20, 32, 4
+    q, k, v = make_qkv(B, H, L, d, dtype="f32", seed=11)
+    ref = orc.forward_decay(q, k, v, M, 7, 7.0)
+    st = torch.zeros((B, H, 2, 7, d), dtype=torch.float32, device=dev)
+    outs = [bla.bla_decay_decode_step(to_dev(q[:, :, t], dev, torch.float32), to_dev(k[:, :, t], dev, torch.float32),
+                                      to_dev(v[:, :, t], dev, torch.float32), st, t, M, 7, 7.0).cpu().numpy()
+            for t in range(L)]
+    bla.bla_device_error()
+    assert rel(np.stack(outs, 2), ref["o"]) <= TOL_F32
+
+
+def test_full_size_forward_sampled(orc):
+    """The bench's decay workload (B=8, H=8, L=4096, d=128, M=64, S=64, T=1024, bf16) in one call;
+    head (0, 0) against the oracle on the same seeded draw, all outputs finite."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import WORKLOADS, make_qkv
+    dev = require_cuda()
+    w = WORKLOADS["decay_bf16_lm"]
+    q, k, v = make_qkv(w.B, w.H, w.L, w.d, dtype="bf16", seed=0)
+    o, lse, _ = bla.bla_decay_forward(*(to_dev(x, dev, torch.bfloat16) for x in (q, k, v)), w.M, w.S, w.T)
+    bla.bla_device_error()
+    o = o.float().cpu().numpy()
+    assert np.isfinite(o).all() and np.isfinite(lse.cpu().numpy()).all()
+    ref = orc.forward_decay(q[:1, :1], k[:1, :1], v[:1, :1], w.M, w.S, w.T)
+    assert rel(o[:1, :1], ref["o"]) <= TOL_BF16, rel(o[:1, :1], ref["o"])
+
+
+def test_full_size_decode_sampled(orc):
+    """The decay decode workload (B=256, H=16, d=128, M=128, S=128, T=4096, pos = 4096, random slot
+    state) in one call; three heads against the oracle's one-token forward from the same state."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import WORKLOADS, make_decode_step, make_slot_state
+    dev = require_cuda()
+    w = WORKLOADS["decay_decode_bf16"]
+    q, k, v = make_decode_step(0, w.B, w.H, w.d, "bf16", seed=0)
+    st0 = make_slot_state(w.B, w.H, w.S, w.d, w.state_std, seed=0)
+    st = torch.from_numpy(st0).to(dev)
+    o = bla.bla_decay_decode_step(*(to_dev(x, dev, torch.bfloat16) for x in (q, k, v)), st, w.decode_pos0,
+                                  w.M, w.S, w.T)
+    bla.bla_device_error()
+    o = o.float().cpu().numpy()
+    stn = st.cpu().numpy()
+    assert np.isfinite(o).all()
+    for b, h in ((0, 0), (17, 5), (255, 15)):
+        ref = orc.forward_decay(q[b:b + 1, h:h + 1, None], k[b:b + 1, h:h + 1, None], v[b:b + 1, h:h + 1, None],
+                                w.M, w.S, w.T, state=st0[b:b + 1, h:h + 1], pos0=w.decode_pos0, return_state=True)
+        assert rel(o[b, h], ref["o"][0, 0, 0]) <= TOL_BF16
+        assert rel(stn[b, h], ref["state"][0, 0]) <= TOL_F32
+
+
+def test_lag_form_rejected():
+    """The decay is defined on the absolute form's slots; the lag form is refused before any launch."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    dev = require_cuda()
+    x = torch.zeros((1, 1, 8, 32), dtype=torch.float32, device=dev)
+    with pytest.raises(bla.BlaError) as e:
+        bla.bla_decay_forward(x, x, x, 4, 4, 16.0, phase_mode="lag")
+    assert e.value.status == bla.BLA_ERR_UNSUPPORTED
