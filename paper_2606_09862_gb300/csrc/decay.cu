@@ -19,8 +19,8 @@
 //                  transposing butterfly, so lane l ends with token t0 + l's score.
 //   k_decay_lse    one thread per token: masked log-sum-exp over the slots.
 //   k_decay_vscan  one CTA per (head, 32 value columns): thread (g, c) holds column c of the 8
-//                  slots of group g; p and D for 16 tokens are staged in shared memory and the
-//                  groups' partial outputs are summed there.
+//                  slots of group g; p, D and the value columns of 16 tokens are staged in shared
+//                  memory and the groups' partial outputs are summed there.
 //   k_decay_decode one CTA per head for a single token: K rows updated and scored, softmax,
 //                  V rows updated and accumulated; every state row is read and written once.
 #include <math.h>
@@ -35,6 +35,7 @@ constexpr unsigned kFull = 0xffffffffu;
 constexpr int kSlotsPerWarpGroup = 8;   // slots per thread in the V scan
 constexpr int kVTile = 16;              // tokens per V-scan shared-memory tile
 constexpr int kDecodeWarps = 8;
+constexpr int kKBatch = 8;              // tokens whose q, k rows the K scan loads ahead
 
 // D_M(x) at mode frequency w, Eq. (dirichlet) in its closed form.  w x is reduced to (-pi, pi]
 // first, where the ratio is well conditioned; at the kernel's peak (|sin| below 1e-9) D = 1 to
@@ -120,24 +121,32 @@ __global__ void __launch_bounds__(256) k_decay_kscan(const T *__restrict__ q, co
     }
     float *srow = sc + ((size_t)bh * S + j) * L;
     for (int t0 = 0; t0 < L; t0 += 32) {
+        // D = 0 past the end of the sequence: those steps leave the state as it is.
         const float Dl = (t0 + lane < L) ? Dx[t0 + lane + off] : 0.f;
         float part[32];
 #pragma unroll
-        for (int u = 0; u < 32; ++u) {
-            const float D = __shfl_sync(kFull, Dl, u);
-            float dot = 0.f;
-            if (t0 + u < L) {
-                float kv[CPL], qv[CPL];
-                load_cols<T, CPL>(k + row0 + (size_t)(t0 + u) * d, kv);
-                load_cols<T, CPL>(q + row0 + (size_t)(t0 + u) * d, qv);
+        for (int u8 = 0; u8 < 32; u8 += kKBatch) {
+            // The rows of kKBatch tokens are loaded before any is used (rows past the end repeat the
+            // last one), so a warp has 2 kKBatch loads in flight instead of two.
+            float kv[kKBatch][CPL], qv[kKBatch][CPL];
+#pragma unroll
+            for (int i = 0; i < kKBatch; ++i) {
+                const size_t r = (size_t)min(t0 + u8 + i, L - 1) * d;
+                load_cols<T, CPL>(k + row0 + r, kv[i]);
+                load_cols<T, CPL>(q + row0 + r, qv[i]);
+            }
+#pragma unroll
+            for (int i = 0; i < kKBatch; ++i) {
+                const float D = __shfl_sync(kFull, Dl, u8 + i);
                 const float keep = 1.f - D;
+                float dot = 0.f;
 #pragma unroll
                 for (int e = 0; e < CPL; ++e) {
-                    K[e] = fmaf(keep, K[e], D * kv[e]);
-                    dot = fmaf(qv[e], K[e], dot);
+                    K[e] = fmaf(keep, K[e], D * kv[i][e]);
+                    dot = fmaf(qv[i][e], K[e], dot);
                 }
+                part[u8 + i] = dot;
             }
-            part[u] = dot;
         }
         // Transposing butterfly: after the stage of width o, a lane with bit o set holds the sums of
         // entries i + o in part[i]; after all five, lane l holds entry l summed over the 32 lanes.
@@ -191,7 +200,8 @@ __global__ void __launch_bounds__(1024) k_decay_vscan(const T *__restrict__ v, c
     float *Dt = reinterpret_cast<float *>(smem4);      // [TT][sp]
     float *Pt = Dt + TT * sp;                          // [TT][sp]
     float *red = Pt + TT * sp;                         // [TT][ng][32]
-    int *dl = reinterpret_cast<int *>(red + TT * ng * 32);   // [spad]
+    float *Vt = red + TT * ng * 32;                    // [TT][32]: the block's value columns
+    int *dl = reinterpret_cast<int *>(Vt + TT * 32);   // [spad]
     const int g = threadIdx.x >> 5, lane = threadIdx.x & 31, nthr = blockDim.x;
     const long long bh = blockIdx.x / ncb;
     const int c = (blockIdx.x % ncb) * 32 + lane;
@@ -204,7 +214,7 @@ __global__ void __launch_bounds__(1024) k_decay_vscan(const T *__restrict__ v, c
         V[jj] = (state_in && j < S) ? state_in[vst + (size_t)j * dv] : 0.f;
     }
     __syncthreads();
-    const T *vh = v + (size_t)bh * L * dv + c;
+    const T *vb = v + (size_t)bh * L * dv + (c - lane);   // first column of the block
     T *oh = o + (size_t)bh * L * dv + c;
     const float *sh = sc + (size_t)bh * S * L;
     const float *lh = lse + (size_t)bh * L;
@@ -219,10 +229,15 @@ __global__ void __launch_bounds__(1024) k_decay_vscan(const T *__restrict__ v, c
             Dt[tt * sp + j] = D;
             Pt[tt * sp + j] = P;
         }
+        for (int idx = threadIdx.x; idx < TT * 32; idx += nthr) {
+            const int t = t0 + (idx >> 5);
+            Vt[idx] = t < L ? load_elem<T>(vb, (size_t)t * dv + (idx & 31)) : 0.f;
+        }
         __syncthreads();
         const int nt = min(TT, L - t0);
+#pragma unroll 4
         for (int tt = 0; tt < nt; ++tt) {
-            const float x = load_elem<T>(vh, (size_t)(t0 + tt) * dv);
+            const float x = Vt[tt * 32 + lane];
             const float4 *d4 = reinterpret_cast<const float4 *>(Dt + tt * sp + g * G);
             const float4 *p4 = reinterpret_cast<const float4 *>(Pt + tt * sp + g * G);
             const float4 da = d4[0], db = d4[1], pa = p4[0], pb = p4[1];
@@ -397,7 +412,8 @@ cudaError_t kscan_dispatch(const OpDims &d, const DecayWs &w, const void *q, con
 
 size_t vscan_smem(int ng) {
     const int spad = ng * kSlotsPerWarpGroup, sp = spad + 4;
-    return sizeof(float) * ((size_t)2 * kVTile * sp + (size_t)kVTile * ng * 32) + sizeof(int) * (size_t)spad;
+    return sizeof(float) * ((size_t)2 * kVTile * sp + (size_t)kVTile * ng * 32 + (size_t)kVTile * 32) +
+           sizeof(int) * (size_t)spad;
 }
 
 template <typename T>
