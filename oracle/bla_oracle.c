@@ -37,6 +37,9 @@
  *   orc_forward_decay     Alg. 1 with the state decay of Sec. 3.3: the previous
  *                         slot state is multiplied by (1 - D_j(t)) before the token
  *                         is added with weight D_j(t) (slot-space state [S][d]).
+ *   orc_backward_decay    its vector-Jacobian product: the chain rule below with the
+ *                         unrolled decay weight D_j(u) prod_{u<x<=t} (1 - D_j(x)) (pinned
+ *                         to finite differences of orc_forward_decay).
  *   orc_backward_parallel vector-Jacobian product of the parallel form, written out
  *                         by the chain rule (no paper counterpart; pinned to central
  *                         finite differences of orc_forward_naive by the tests).
@@ -462,6 +465,78 @@ static void head_backward(const orc_cfg *c, const double *delta, int absolute,
     free(Dt); free(qk); free(dov); free(s); free(p); free(dp);
 }
 
+/* ------------------------------------------- VJP of the decayed form (Sec. 3.3)
+ *
+ * Unrolled, the decayed slot state is a fixed linear map of the past tokens:
+ *     K~_t[j] = sum_{u<=t} Wd[t,u,j] k_u,     Wd[t,u,j] = D_j(u) prod_{u<x<=t} (1 - D_j(x)),
+ * with D_j(x) Alg. 1's "interpolate" at the absolute index pos0 + x (V~ likewise).  With Wd in
+ * place of the weight W, the chain rule written out above head_backward applies as it stands
+ * (zero initial state).
+ */
+static void head_backward_decay(const orc_cfg *c, const double *A, const double *B, const double *delta,
+                                const double *q, const double *k, const double *v, const double *dout,
+                                double *dq, double *dk_, double *dv_)
+{
+    int M = c->M, S = c->S, dk = c->dk, dv = c->dv, L = c->L;
+    size_t nls = (size_t)(L > 0 ? L : 1) * S;
+    double *ip = malloc(sizeof(double) * nls), *Wt = malloc(sizeof(double) * nls);
+    double *qk = malloc(sizeof(double) * (L > 0 ? L : 1)), *dov = malloc(sizeof(double) * (L > 0 ? L : 1));
+    double *s = malloc(sizeof(double) * S), *p = malloc(sizeof(double) * S), *dp = malloc(sizeof(double) * S);
+    memset(dq, 0, sizeof(double) * (size_t)L * dk);
+    memset(dk_, 0, sizeof(double) * (size_t)L * dk);
+    memset(dv_, 0, sizeof(double) * (size_t)L * dv);
+    for (int x = 0; x < L; ++x) {
+        double tx = (double)(c->pos0 + x);
+        for (int j = 0; j < S; ++j) {
+            double acc = 0.0;
+            for (int m = 0; m < M; ++m) acc += cos(tx * m * c->w) * A[j * M + m] + sin(tx * m * c->w) * B[j * M + m];
+            ip[(size_t)x * S + j] = acc;
+        }
+    }
+    for (int t = 0; t < L; ++t) {
+        const double *qt = q + (size_t)t * dk, *dot = dout + (size_t)t * dv;
+        for (int j = 0; j < S; ++j) {          /* Wd[t,u,j] for u = t down to 0 */
+            double prod = 1.0;
+            for (int u = t; u >= 0; --u) {
+                Wt[(size_t)u * S + j] = ip[(size_t)u * S + j] * prod;
+                prod *= 1.0 - ip[(size_t)u * S + j];
+            }
+        }
+        for (int u = 0; u <= t; ++u) {
+            double a = 0.0, b = 0.0;
+            for (int i = 0; i < dk; ++i) a += qt[i] * k[(size_t)u * dk + i];
+            for (int i = 0; i < dv; ++i) b += dot[i] * v[(size_t)u * dv + i];
+            qk[u] = a; dov[u] = b;
+        }
+        for (int j = 0; j < S; ++j) {
+            double a = 0.0, b = 0.0;
+            for (int u = 0; u <= t; ++u) {
+                a += Wt[(size_t)u * S + j] * qk[u];
+                b += Wt[(size_t)u * S + j] * dov[u];
+            }
+            s[j] = c->scale * a; dp[j] = b;
+        }
+        masked_softmax(S, s, delta, c->pos0 + t, p);
+        double pdp = 0.0;
+        for (int j = 0; j < S; ++j) pdp += p[j] * dp[j];
+        for (int u = 0; u <= t; ++u) {
+            double g = 0.0, dP = 0.0;
+            for (int j = 0; j < S; ++j) {
+                double wgt = Wt[(size_t)u * S + j];
+                g += p[j] * wgt;
+                dP += p[j] * (dp[j] - pdp) * wgt;
+            }
+            dP *= c->scale;
+            for (int i = 0; i < dk; ++i) {
+                dq[(size_t)t * dk + i] += dP * k[(size_t)u * dk + i];
+                dk_[(size_t)u * dk + i] += dP * qt[i];
+            }
+            for (int i = 0; i < dv; ++i) dv_[(size_t)u * dv + i] += g * dot[i];
+        }
+    }
+    free(ip); free(Wt); free(qk); free(dov); free(s); free(p); free(dp);
+}
+
 /* ------------------------------------------------------------ entry points
  * Arrays are [NH][L][d] with NH = batch*heads, contiguous; state is
  * [NH][2][M][2][d] (see header).  `want` (length L, may be NULL) selects the
@@ -523,6 +598,24 @@ int orc_forward_decay(int NH, int L, int dk, int dv, int M, int S, double T, dou
         size_t ok = (size_t)h * L * dk, ov = (size_t)h * L * dv;
         head_decay(&c, A, B, delta, q + ok, k + ok, v + ov, o + ov, lse ? lse + (size_t)h * L : NULL,
                    state ? state + (size_t)h * S * (dk + dv) : NULL);
+    }
+    free(delta); free(A); free(B);
+    return 0;
+}
+
+/* VJP of orc_forward_decay from the zero state, tokens at absolute indices pos0 .. pos0+L-1. */
+int orc_backward_decay(int NH, int L, int dk, int dv, int M, int S, double T, double omega, double scale,
+                       long long pos0, const double *q, const double *k, const double *v, const double *dout,
+                       double *dq, double *dk_, double *dv_)
+{
+    if (NH < 0 || L < 0 || dk < 1 || dv < 1 || M < 1 || S < 1 || pos0 < 0) return 1;
+    orc_cfg c = make_cfg(L, dk, dv, M, S, T, omega, scale, pos0);
+    double *delta = malloc(sizeof(double) * S), *A = malloc(sizeof(double) * S * M), *B = malloc(sizeof(double) * S * M);
+    orc_tables(M, S, T, omega, delta, A, B);
+    #pragma omp parallel for schedule(dynamic, 1)
+    for (int h = 0; h < NH; ++h) {
+        size_t ok = (size_t)h * L * dk, ov = (size_t)h * L * dv;
+        head_backward_decay(&c, A, B, delta, q + ok, k + ok, v + ov, dout + ov, dq + ok, dk_ + ok, dv_ + ov);
     }
     free(delta); free(A); free(B);
     return 0;

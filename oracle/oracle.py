@@ -9,7 +9,7 @@ Forms (see the C header for the paper passage each follows):
   "modes"     same recurrence, read-out through the modes (Eq. conv exchange of sums)
   "parallel"  closed form of Eq. (states) with translated Dirichlet kernels
   "absolute"  Alg. 1 (efficient recurrent BLA, time-rolling slots); pins only
-  forward_decay: Alg. 1 with the state decay of Sec. 3.3 (slot-space state)
+  forward_decay, backward_decay: Alg. 1 with the state decay of Sec. 3.3 (slot-space state) and its VJP
 """
 import ctypes
 
@@ -40,6 +40,8 @@ def _configure(lib):
     lib.orc_backward.argtypes = [ctypes.c_int] * 7 + [ctypes.c_double] * 3 + [_dp] * 7
     lib.orc_forward_decay.restype = ctypes.c_int
     lib.orc_forward_decay.argtypes = [ctypes.c_int] * 6 + [ctypes.c_double] * 3 + [ctypes.c_longlong] + [_dp] * 6
+    lib.orc_backward_decay.restype = ctypes.c_int
+    lib.orc_backward_decay.argtypes = [ctypes.c_int] * 6 + [ctypes.c_double] * 3 + [ctypes.c_longlong] + [_dp] * 7
     lib.orc_max_threads.restype = ctypes.c_int
     return lib
 
@@ -177,3 +179,16 @@ def backward(q, k, v, dout, M, S, T, omega=0.0, scale=0.0, form="parallel"):
         raise ValueError("oracle backward rejected its arguments (code %d)" % rc)
     return dq, dkk, dvv
 
+
+def backward_decay(q, k, v, dout, M, S, T, omega=0.0, scale=0.0, pos0=0):
+    """Vector-Jacobian product (dq, dk, dv) of ``forward_decay`` from the zero state, tokens at
+    absolute indices pos0 .., for upstream gradient dout."""
+    q, k, v, dout = _f64(q), _f64(k), _f64(v), _f64(dout)
+    Bn, Hn, L, dk = q.shape
+    dv = v.shape[-1]
+    dq, dkk, dvv = np.zeros_like(q), np.zeros_like(k), np.zeros_like(v)
+    rc = _load().orc_backward_decay(Bn * Hn, L, dk, dv, int(M), int(S), float(T), float(omega), float(scale),
+                                    int(pos0), _ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(dq), _ptr(dkk), _ptr(dvv))
+    if rc != 0:
+        raise ValueError("oracle decay backward rejected its arguments (code %d)" % rc)
+    return dq, dkk, dvv

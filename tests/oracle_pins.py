@@ -412,6 +412,32 @@ def pin_decay_handoff(orc):
                   float(np.abs(a["o"] - full["o"][:, :, :L1]).max()))
 
 
+def pin_decay_backward_fd(orc, h=1e-6):
+    """The decayed form's VJP = central finite differences of its forward, loss = sum(dO * O), for
+    T above 2M-1, at T = 2M-1 (sliding window) and from a later start position."""
+    g = rng(59)
+    err = 0.0
+    for M, S, T, L, d, pos0 in ((3, 4, 10.0, 8, 3, 0), (2, 3, 3.0, 9, 2, 0), (2, 5, 11.0, 7, 2, 6)):
+        q, k, v, do = (g.standard_normal((1, 1, L, d)) for _ in range(4))
+        dq, dk, dv = orc.backward_decay(q, k, v, do, M, S, T, pos0=pos0)
+
+        def loss():
+            return float((orc.forward_decay(q, k, v, M, S, T, pos0=pos0)["o"] * do).sum())
+
+        for x, gx in ((q, dq), (k, dk), (v, dv)):
+            fd = np.zeros_like(x)
+            for idx in np.ndindex(x.shape):
+                x0 = x[idx]
+                x[idx] = x0 + h
+                lp = loss()
+                x[idx] = x0 - h
+                lm = loss()
+                x[idx] = x0
+                fd[idx] = (lp - lm) / (2 * h)
+            err = _worst(err, float(np.abs(fd - gx).max() / (np.abs(gx).max() + 1e-30)))
+    return err
+
+
 ALL_PINS = {
     "dirichlet_identity": (pin_dirichlet_identity, 1e-12),
     "dirichlet_samples": (pin_dirichlet_samples, 1e-13),
@@ -431,4 +457,5 @@ ALL_PINS = {
     "decay_closed_form": (pin_decay_closed_form, 1e-11),
     "decay_single_mode": (pin_decay_single_mode, 1e-13),
     "decay_handoff": (pin_decay_handoff, 1e-12),
+    "decay_backward_fd": (pin_decay_backward_fd, 1e-6),
 }

@@ -42,6 +42,8 @@ MUTANTS = {
                         "Kp[j * dk + e] = keep * (Kp[j * dk + e] + ip[j] * k[(size_t)i * dk + e]);"),
     "decay_relative_phase": ("double t = (double)(c->pos0 + i);", "double t = (double)i;"),
     "decay_factor_sign": ("double keep = 1.0 - ip[j];", "double keep = 1.0 + ip[j];"),
+    "decay_backward_product_inclusive": ("Wt[(size_t)u * S + j] = ip[(size_t)u * S + j] * prod;\n                prod *= 1.0 - ip[(size_t)u * S + j];",
+                                         "prod *= 1.0 - ip[(size_t)u * S + j];\n                Wt[(size_t)u * S + j] = ip[(size_t)u * S + j] * prod;"),
     "decay_value_not_decayed": ("Vp[j * dv + e] = keep * Vp[j * dv + e] + ip[j]", "Vp[j * dv + e] = Vp[j * dv + e] + ip[j]"),
 }
 
