@@ -170,6 +170,10 @@ bla_status check_decay(const bla_params *p, OpDims *d, bool forward) {
     if (d->S > 256) return fail(BLA_ERR_UNSUPPORTED, "the decay path needs S <= 256 (got %d)", d->S);
     if (forward && decay_table_entries(*d) > (size_t(1) << 30))
         return fail(BLA_ERR_UNSUPPORTED, "L + T too large for the decay table (L=%d, T=%g)", d->L, d->T);
+    // one-dimensional grids: heads x slot blocks (K scan), heads x column blocks (V scan), tokens / 256 (lse)
+    const long long bh = (long long)d->B * d->H, imax = (1ll << 31) - 1;
+    if (bh * ((d->S + 7) / 8) > imax || bh * (d->dv / 32) > imax || (forward && bh * d->L / 256 + 1 > imax))
+        return fail(BLA_ERR_UNSUPPORTED, "B*H too large for the decay kernels' grids (B*H=%lld)", bh);
     return BLA_OK;
 }
 

@@ -170,3 +170,5 @@ def test_decay_argument_checks(lib):
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_FORWARD) >= 2 * 3 * 8 * 100 * 4
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_DECODE) > 0
     assert lib.bla_workspace_bytes(ctypes.byref(_params()), bla.BLA_WS_DECAY_FORWARD) == 0
+    # grids that would exceed the launch limits are refused before any launch
+    assert fwd(_params(phase_mode=ab, B=1 << 20, H=1 << 10, S=64, window=64.0)) == bla.BLA_ERR_UNSUPPORTED
