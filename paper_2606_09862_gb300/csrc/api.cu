@@ -12,6 +12,7 @@
 
 #include "common.cuh"
 #include "bwd.cuh"
+#include "decay.cuh"
 #include "fwd_bf16.cuh"
 #include "tc.cuh"
 

@@ -25,7 +25,7 @@
 //                  V rows updated and accumulated; every state row is read and written once.
 #include <math.h>
 
-#include "common.cuh"
+#include "decay.cuh"
 
 namespace bla {
 

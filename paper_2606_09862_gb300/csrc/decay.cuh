@@ -1,0 +1,18 @@
+// decay.cuh -- launchers of the state-decay kernels (decay.cu).
+#pragma once
+
+#include "common.cuh"
+
+namespace bla {
+
+// State decay (Sec. 3.3) on Alg. 1's slot-space state.  The state is fp32
+// [B][H][2 (K~ then V~)][S][d]; the workspace holds the grid, the D_M table, the slot scores and,
+// when lse is NULL, the log-sum-exp of the forward.
+size_t decay_workspace_bytes(const OpDims &d, bool decode);
+size_t decay_table_entries(const OpDims &d);   // D_M values one forward call tabulates
+cudaError_t launch_decay_forward(const OpDims &d, long long pos0, const void *q, const void *k, const void *v, void *o,
+                                 float *lse, const float *state_in, float *state_out, void *ws, cudaStream_t st);
+cudaError_t launch_decay_decode(const OpDims &d, long long pos, const void *q, const void *k, const void *v,
+                                float *state, void *o, void *ws, cudaStream_t st);
+
+}  // namespace bla
