@@ -92,6 +92,34 @@ def tables(M: int, S: int, T: float, omega: float = 0.0):
     return delta, A, B
 
 
+def _per_head(T, H):
+    """The periods of Alg. 1 and Alg. 3 (T in R^H): None for one scalar period shared by every head,
+    else the array of H periods (each head's grid, omega, A and B follow its own period)."""
+    Ts = np.atleast_1d(np.asarray(T, dtype=np.float64))
+    if Ts.size == 1 and np.ndim(T) == 0:
+        return None
+    if Ts.shape != (H,):
+        raise ValueError("per-head periods need one value per head (%d), got shape %s" % (H, Ts.shape))
+    return Ts
+
+
+def _by_head(fn, Ts, arrays, H, **kw):
+    """Run ``fn`` on each head's slice [:, h:h+1] at period Ts[h]; returns the per-head results."""
+    out = []
+    for h in range(H):
+        sl = [None if a is None else np.asarray(a)[:, h:h + 1] for a in arrays]
+        out.append(fn(*sl, T=float(Ts[h]), **kw))
+    return out
+
+
+def _cat_dicts(parts):
+    res = {}
+    for key in parts[0]:
+        vals = [p[key] for p in parts]
+        res[key] = None if vals[0] is None else np.concatenate(vals, axis=1)
+    return res
+
+
 def forward(q, k, v, M, S, T, omega=0.0, scale=0.0, form="naive", state=None, pos0=0,
             want=None, return_state=False):
     """Run the oracle forward.
@@ -101,8 +129,15 @@ def forward(q, k, v, M, S, T, omega=0.0, scale=0.0, form="naive", state=None, po
     layout) and ``pos0`` the absolute index of token 0 (slot mask t >= Delta_j).
     ``want`` (bool [L]) restricts which tokens get an output (others are NaN);
     the state always advances over every token.
+    ``T`` is one period, or one per head (Alg. 1 and Alg. 3 take T in R^H).
     Returns dict(o=[B,H,L,dv], lse=[B,H,L], state=final state or None).
     """
+    Ts = _per_head(T, np.shape(q)[1])
+    if Ts is not None:
+        parts = _by_head(lambda q_, k_, v_, st_, T: forward(q_, k_, v_, M, S, T, omega, scale, form, st_, pos0, want,
+                                                             return_state),
+                         Ts, (q, k, v, state), len(Ts))
+        return _cat_dicts(parts)
     q, k, v = _f64(q), _f64(k), _f64(v)
     Bn, Hn, L, dk = q.shape
     dv = v.shape[-1]
@@ -140,8 +175,14 @@ def forward_decay(q, k, v, M, S, T, omega=0.0, scale=0.0, state=None, pos0=0, re
     q, k: [B, H, L, dk]; v: [B, H, L, dv].  ``state`` (optional) is the slot-space state
     [B, H, 2, S, d] (K~ then V~; any shape with S*(dk+dv) values per head) and ``pos0`` the
     absolute index of token 0.  Returns dict(o, lse, state) like ``forward``; the state is
-    [B, H, 2, S, d] when dk == dv.
+    [B, H, 2, S, d] when dk == dv.  ``T`` is one period or one per head.
     """
+    Ts = _per_head(T, np.shape(q)[1])
+    if Ts is not None:
+        parts = _by_head(lambda q_, k_, v_, st_, T: forward_decay(q_, k_, v_, M, S, T, omega, scale, st_, pos0,
+                                                                   return_state),
+                         Ts, (q, k, v, state), len(Ts))
+        return _cat_dicts(parts)
     q, k, v = _f64(q), _f64(k), _f64(v)
     Bn, Hn, L, dk = q.shape
     dv = v.shape[-1]
@@ -164,7 +205,13 @@ def forward_decay(q, k, v, M, S, T, omega=0.0, scale=0.0, state=None, pos0=0, re
 def backward(q, k, v, dout, M, S, T, omega=0.0, scale=0.0, form="parallel"):
     """Vector-Jacobian product (dq, dk, dv) of the forward for upstream gradient dout.
 
-    ``form`` "parallel" (any of the lag-form forwards; they agree) or "absolute" (Alg. 1)."""
+    ``form`` "parallel" (any of the lag-form forwards; they agree) or "absolute" (Alg. 1).
+    ``T`` is one period or one per head."""
+    Ts = _per_head(T, np.shape(q)[1])
+    if Ts is not None:
+        parts = _by_head(lambda q_, k_, v_, do_, T: backward(q_, k_, v_, do_, M, S, T, omega, scale, form),
+                         Ts, (q, k, v, dout), len(Ts))
+        return tuple(np.concatenate([p[i] for p in parts], axis=1) for i in range(3))
     if form not in ("parallel", "absolute"):
         raise ValueError("backward form must be 'parallel' or 'absolute', got %r" % (form,))
     q, k, v, dout = _f64(q), _f64(k), _f64(v), _f64(dout)
@@ -182,7 +229,12 @@ def backward(q, k, v, dout, M, S, T, omega=0.0, scale=0.0, form="parallel"):
 
 def backward_decay(q, k, v, dout, M, S, T, omega=0.0, scale=0.0, pos0=0):
     """Vector-Jacobian product (dq, dk, dv) of ``forward_decay`` from the zero state, tokens at
-    absolute indices pos0 .., for upstream gradient dout."""
+    absolute indices pos0 .., for upstream gradient dout.  ``T`` is one period or one per head."""
+    Ts = _per_head(T, np.shape(q)[1])
+    if Ts is not None:
+        parts = _by_head(lambda q_, k_, v_, do_, T: backward_decay(q_, k_, v_, do_, M, S, T, omega, scale, pos0),
+                         Ts, (q, k, v, dout), len(Ts))
+        return tuple(np.concatenate([p[i] for p in parts], axis=1) for i in range(3))
     q, k, v, dout = _f64(q), _f64(k), _f64(v), _f64(dout)
     Bn, Hn, L, dk = q.shape
     dv = v.shape[-1]

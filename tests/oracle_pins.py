@@ -438,6 +438,71 @@ def pin_decay_backward_fd(orc, h=1e-6):
     return err
 
 
+# --------------------------------------- NEXT: per-head periods (T in R^H)
+
+def pin_per_head_period(orc):
+    """Alg. 1 and Alg. 3 take one period per head: each head's grid round(j T_h / S), frequency
+    2 pi / T_h and coefficients follow its own period.  Every head of a per-head run is checked
+    against a brute force at its own period, computed here with the sine-ratio D_M: the lag form
+    (weight D_M(t - u - Delta_j)), the absolute form (D_M(u - Delta_j)) and the decayed form (the
+    unrolled product).  The periods differ per head, including T = 2M-1, so a head reading
+    another head's period fails."""
+    g = rng(61)
+    M, S, L, d = 3, 5, 14, 3
+    Ts = np.array([5.0, 13.0, 21.0])
+    q, k, v = (g.standard_normal((2, 3, L, d)) for _ in range(3))
+    lag = orc.forward(q, k, v, M, S, Ts, form="naive")
+    ab = orc.forward(q, k, v, M, S, Ts, form="absolute")
+    dec = orc.forward_decay(q, k, v, M, S, Ts)
+    err = 0.0
+    for h, T in enumerate(Ts):
+        w = 2 * np.pi / T
+        delta = np.round(np.arange(S) * T / S)
+        Dabs = dirichlet_sine_ratio(M, w, np.arange(L)[None, :] - delta[:, None])   # D_j(u), [S, L]
+        for b in range(2):
+            for t in range(L):
+                u = np.arange(t + 1)
+                Wd = np.zeros((S, t + 1))
+                for uu in range(t + 1):
+                    Wd[:, uu] = Dabs[:, uu] * np.prod(1.0 - Dabs[:, uu + 1: t + 1], axis=1)
+                for r, W in ((lag, dirichlet_sine_ratio(M, w, (t - u)[None, :] - delta[:, None])),
+                             (ab, Dabs[:, : t + 1]), (dec, Wd)):
+                    Ks, Vs = W @ k[b, h, : t + 1], W @ v[b, h, : t + 1]
+                    p, lse = _softmax_masked((Ks @ q[b, h, t] / np.sqrt(d))[None], (t >= delta)[None])
+                    err = _worst(err, float(np.abs(r["o"][b, h, t] - p[0] @ Vs).max()),
+                                 float(abs(r["lse"][b, h, t] - lse[0])))
+    return err
+
+
+def pin_per_head_period_backward(orc, h=1e-6):
+    """The VJPs with per-head periods (lag, absolute and decayed forms) = central differences of
+    the per-head forwards."""
+    g = rng(67)
+    M, S, L, d = 2, 3, 6, 2
+    Ts = np.array([3.0, 8.0])
+    q, k, v, do = (g.standard_normal((1, 2, L, d)) for _ in range(4))
+    err = 0.0
+    for fwd, bwd in ((lambda: orc.forward(q, k, v, M, S, Ts, form="parallel")["o"],
+                      lambda: orc.backward(q, k, v, do, M, S, Ts)),
+                     (lambda: orc.forward(q, k, v, M, S, Ts, form="absolute")["o"],
+                      lambda: orc.backward(q, k, v, do, M, S, Ts, form="absolute")),
+                     (lambda: orc.forward_decay(q, k, v, M, S, Ts)["o"],
+                      lambda: orc.backward_decay(q, k, v, do, M, S, Ts))):
+        grads = bwd()
+        for x, gx in zip((q, k, v), grads):
+            fd = np.zeros_like(x)
+            for idx in np.ndindex(x.shape):
+                x0 = x[idx]
+                x[idx] = x0 + h
+                lp = float((fwd() * do).sum())
+                x[idx] = x0 - h
+                lm = float((fwd() * do).sum())
+                x[idx] = x0
+                fd[idx] = (lp - lm) / (2 * h)
+            err = _worst(err, float(np.abs(fd - gx).max() / (np.abs(gx).max() + 1e-30)))
+    return err
+
+
 ALL_PINS = {
     "dirichlet_identity": (pin_dirichlet_identity, 1e-12),
     "dirichlet_samples": (pin_dirichlet_samples, 1e-13),
@@ -458,4 +523,6 @@ ALL_PINS = {
     "decay_single_mode": (pin_decay_single_mode, 1e-13),
     "decay_handoff": (pin_decay_handoff, 1e-12),
     "decay_backward_fd": (pin_decay_backward_fd, 1e-6),
+    "per_head_period": (pin_per_head_period, 1e-11),
+    "per_head_period_backward": (pin_per_head_period_backward, 1e-6),
 }

@@ -73,3 +73,17 @@ def test_mutant_is_caught(name, src_text, tmp_path, monkeypatch):
         if not err <= tol:
             failed.append(pname)
     assert failed, "planted mistake %r passed every pin" % name
+
+
+def test_per_head_period_mapping_mutant_is_caught(monkeypatch):
+    """A front end that hands each head another head's period (reversed order) fails the
+    per-head pins."""
+    import oracle
+    import oracle.oracle as oo
+    real = oo._by_head
+
+    def swapped(fn, Ts, arrays, H, **kw):
+        return real(fn, Ts[::-1].copy(), arrays, H, **kw)
+
+    monkeypatch.setattr(oo, "_by_head", swapped)
+    assert P.pin_per_head_period(oracle) > 1e-3
