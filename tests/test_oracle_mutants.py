@@ -54,6 +54,7 @@ def src_text():
         return f.read()
 
 
+@pytest.mark.filterwarnings("ignore::RuntimeWarning")   # a broken oracle may yield NaN; the pins count it as a failure
 @pytest.mark.parametrize("name", sorted(MUTANTS))
 def test_mutant_is_caught(name, src_text, tmp_path, monkeypatch):
     import oracle.oracle as oo
