@@ -438,6 +438,29 @@ def pin_decay_backward_fd(orc, h=1e-6):
     return err
 
 
+# ------------------------------------------------ token selection (want)
+
+def pin_token_selection(orc):
+    """Restricting the output to some tokens (``want``, used to sample long sequences) changes
+    nothing else: selected tokens equal the full run, the others are NaN, and the state advances
+    over every token (Eq. recurrence is applied to all of them)."""
+    g = rng(71)
+    M, S, T, L, d = 3, 4, 11.0, 19, 3
+    q, k, v = (g.standard_normal((1, 2, L, d)) for _ in range(3))
+    want = np.zeros(L, bool)
+    want[[0, 5, 6, 13, L - 1]] = True
+    err = 0.0
+    for form in ("naive", "modes"):
+        full = orc.forward(q, k, v, M, S, T, form=form, return_state=True)
+        part = orc.forward(q, k, v, M, S, T, form=form, want=want, return_state=True)
+        err = _worst(err, float(np.abs(part["o"][:, :, want] - full["o"][:, :, want]).max()),
+                     float(np.abs(part["lse"][:, :, want] - full["lse"][:, :, want]).max()),
+                     float(np.abs(part["state"] - full["state"]).max()))
+        if not (np.isnan(part["o"][:, :, ~want]).all() and np.isnan(part["lse"][:, :, ~want]).all()):
+            err = float("inf")
+    return err
+
+
 # --------------------------------------- NEXT: per-head periods (T in R^H)
 
 def pin_per_head_period(orc):
@@ -524,5 +547,6 @@ ALL_PINS = {
     "decay_handoff": (pin_decay_handoff, 1e-12),
     "decay_backward_fd": (pin_decay_backward_fd, 1e-6),
     "per_head_period": (pin_per_head_period, 1e-11),
+    "token_selection": (pin_token_selection, 0.0),
     "per_head_period_backward": (pin_per_head_period_backward, 1e-6),
 }

@@ -44,6 +44,8 @@ MUTANTS = {
     "decay_factor_sign": ("double keep = 1.0 - ip[j];", "double keep = 1.0 + ip[j];"),
     "decay_backward_product_inclusive": ("Wt[(size_t)u * S + j] = ip[(size_t)u * S + j] * prod;\n                prod *= 1.0 - ip[(size_t)u * S + j];",
                                          "prod *= 1.0 - ip[(size_t)u * S + j];\n                Wt[(size_t)u * S + j] = ip[(size_t)u * S + j] * prod;"),
+    "selection_skips_state": ("rotate_add(M, dk, c->w, Kc, Ks, k + (size_t)t * dk);\n        rotate_add(M, dv, c->w, Vc, Vs, v + (size_t)t * dv);\n        if (want && !want[t]) continue;\n        const double *qt",
+                              "if (want && !want[t]) continue;\n        rotate_add(M, dk, c->w, Kc, Ks, k + (size_t)t * dk);\n        rotate_add(M, dv, c->w, Vc, Vs, v + (size_t)t * dv);\n        const double *qt"),
     "decay_value_not_decayed": ("Vp[j * dv + e] = keep * Vp[j * dv + e] + ip[j]", "Vp[j * dv + e] = Vp[j * dv + e] + ip[j]"),
 }
 
