@@ -438,6 +438,31 @@ def pin_decay_backward_fd(orc, h=1e-6):
     return err
 
 
+# ------------------------------------ explicit frequency and softmax scale
+
+def pin_explicit_omega_scale(orc):
+    """An explicit mode frequency omega > 0 replaces 2 pi / T in D_M (Sec. 3.1) while the grid
+    stays round(j T / S), and an explicit scale replaces 1/sqrt(d_k) (Eq. output): the lag and
+    absolute forms against a sine-ratio brute force at that omega and scale."""
+    g = rng(73)
+    M, S, T, L, d, om, sc = 3, 4, 12.0, 15, 3, 0.37, 0.8
+    q, k, v = (g.standard_normal((1, 1, L, d)) for _ in range(3))
+    delta = np.round(np.arange(S) * T / S)
+    err = 0.0
+    for form, arg in (("naive", lambda t, u: (t - u)[None, :] - delta[:, None]),
+                      ("modes", lambda t, u: (t - u)[None, :] - delta[:, None]),
+                      ("absolute", lambda t, u: u[None, :] - delta[:, None])):
+        r = orc.forward(q, k, v, M, S, T, omega=om, scale=sc, form=form)
+        for t in range(L):
+            u = np.arange(t + 1)
+            W = dirichlet_sine_ratio(M, om, arg(t, u))
+            Ks, Vs = W @ k[0, 0, : t + 1], W @ v[0, 0, : t + 1]
+            p, lse = _softmax_masked((sc * (Ks @ q[0, 0, t]))[None], (t >= delta)[None])
+            err = _worst(err, float(np.abs(r["o"][0, 0, t] - p[0] @ Vs).max()),
+                         float(abs(r["lse"][0, 0, t] - lse[0])))
+    return err
+
+
 # ------------------------------------------------ token selection (want)
 
 def pin_token_selection(orc):
@@ -548,5 +573,6 @@ ALL_PINS = {
     "decay_backward_fd": (pin_decay_backward_fd, 1e-6),
     "per_head_period": (pin_per_head_period, 1e-11),
     "token_selection": (pin_token_selection, 0.0),
+    "explicit_omega_scale": (pin_explicit_omega_scale, 1e-11),
     "per_head_period_backward": (pin_per_head_period_backward, 1e-6),
 }

@@ -46,6 +46,10 @@ MUTANTS = {
                                          "prod *= 1.0 - ip[(size_t)u * S + j];\n                Wt[(size_t)u * S + j] = ip[(size_t)u * S + j] * prod;"),
     "selection_skips_state": ("rotate_add(M, dk, c->w, Kc, Ks, k + (size_t)t * dk);\n        rotate_add(M, dv, c->w, Vc, Vs, v + (size_t)t * dv);\n        if (want && !want[t]) continue;\n        const double *qt",
                               "if (want && !want[t]) continue;\n        rotate_add(M, dk, c->w, Kc, Ks, k + (size_t)t * dk);\n        rotate_add(M, dv, c->w, Vc, Vs, v + (size_t)t * dv);\n        const double *qt"),
+    "explicit_omega_ignored": ("return omega > 0.0 ? omega : 2.0 * ORC_PI / orc_period(M, T);",
+                               "return 2.0 * ORC_PI / orc_period(M, T);"),
+    "explicit_scale_ignored": ("c.scale = scale > 0.0 ? scale : 1.0 / sqrt((double)dk);",
+                               "c.scale = 1.0 / sqrt((double)dk);"),
     "decay_value_not_decayed": ("Vp[j * dv + e] = keep * Vp[j * dv + e] + ip[j]", "Vp[j * dv + e] = Vp[j * dv + e] + ip[j]"),
 }
 
