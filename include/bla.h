@@ -70,6 +70,13 @@ typedef struct {
     double scale;       /* softmax scale; <= 0: 1/sqrt(d_k) (Eq. output, per head) */
     int dtype;          /* bla_dtype of q, k, v, o, dout, dq, dk, dv */
     int phase_mode;     /* bla_phase_mode: how the slots index time (0 = the lag form) */
+    const double *periods;  /* NULL: every head uses `window`.  Else a HOST array of H periods, one
+                               per head (Alg. 1 and Alg. 3 take T in R^H): head h's grid, frequency
+                               (2*pi/T_h unless omega > 0) and coefficients follow periods[h], each
+                               clamped to max(T_h, 2M-1); S must not exceed any of them.  Read
+                               during the call only.  At most 256 heads.  Supported by the fp32
+                               forward, bla_decode_step and the state-decay entry points; the others
+                               return BLA_ERR_UNSUPPORTED. */
 } bla_params;
 
 /* How a slot reads the past (bla_params.phase_mode).

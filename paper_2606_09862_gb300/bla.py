@@ -41,7 +41,8 @@ class Params(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("H", ctypes.c_int), ("L", ctypes.c_int),
                 ("d_k", ctypes.c_int), ("d_v", ctypes.c_int), ("M", ctypes.c_int), ("S", ctypes.c_int),
                 ("window", ctypes.c_double), ("omega", ctypes.c_double), ("chunk", ctypes.c_int),
-                ("scale", ctypes.c_double), ("dtype", ctypes.c_int), ("phase_mode", ctypes.c_int)]
+                ("scale", ctypes.c_double), ("dtype", ctypes.c_int), ("phase_mode", ctypes.c_int),
+                ("periods", ctypes.POINTER(ctypes.c_double))]
 
 
 _lib = None
@@ -125,9 +126,22 @@ def _phase_code(phase_mode):
 
 def make_params(B, H, L, d_k, d_v, M, S, window, omega=0.0, chunk=0, scale=0.0, dtype=torch.bfloat16,
                 phase_mode="lag"):
-    """bla_params; phase_mode is "lag" (Alg. 2, the default) or "absolute" (Alg. 1), or its code."""
-    return Params(int(B), int(H), int(L), int(d_k), int(d_v), int(M), int(S), float(window), float(omega),
-                  int(chunk), float(scale), _dtype_code(dtype), _phase_code(phase_mode))
+    """bla_params; phase_mode is "lag" (Alg. 2, the default) or "absolute" (Alg. 1), or its code.
+
+    ``window`` is the period T, or a sequence of H periods, one per head (Alg. 1 and Alg. 3 take
+    T in R^H), passed as ``periods``."""
+    periods = None
+    if isinstance(window, (list, tuple)) or (hasattr(window, "__len__") and not isinstance(window, str)):
+        vals = [float(x) for x in window]
+        if len(vals) != int(H):
+            raise BlaError(BLA_ERR_INVALID, "per-head periods need %d values, got %d" % (int(H), len(vals)))
+        periods = (ctypes.c_double * len(vals))(*vals)
+        window = max(vals)
+    p = Params(int(B), int(H), int(L), int(d_k), int(d_v), int(M), int(S), float(window), float(omega),
+               int(chunk), float(scale), _dtype_code(dtype), _phase_code(phase_mode))
+    if periods is not None:
+        p.periods = periods       # ctypes keeps the array alive with the structure
+    return p
 
 
 def bla_workspace_bytes(params, which):

@@ -52,17 +52,26 @@ __device__ double dirichlet_closed(int M, double w, double x) {
 __device__ __forceinline__ int grid_delta(int j, double T, int S) { return (int)rint((double)j * T / (double)S); }
 
 // per_slot == 0: Dx[i] = D_M(x0 + i), i < n.   per_slot != 0: Dx[j] = D_M(x0 - Delta_j), j < S.
-// Both: delta[j] = round(j T / S) (round half to even, the default rounding mode).
-__global__ void k_decay_table(int M, double w, double T, int S, long long x0, int n, int per_slot, float *Dx,
-                              int *delta) {
-    const int total = (per_slot ? S : n) + S;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+// Both: delta[j] = round(j T / S) (round half to even, the default rounding mode).  With per-head
+// periods (hp.n > 0) head h writes its own Dx[h][...] and delta[h][S] at (T_h, w_h); otherwise the
+// single (T, w) is used.
+__global__ void k_decay_table(int M, HeadPeriods hp, double T, double w, int S, long long x0, int n, int per_slot,
+                              float *Dx, int *delta) {
+    const int nh = hp.n > 0 ? hp.n : 1;
+    const int per = (per_slot ? S : n) + S;
+    const long long total = (long long)per * nh;
+    for (long long ii = blockIdx.x * (long long)blockDim.x + threadIdx.x; ii < total;
+         ii += (long long)gridDim.x * blockDim.x) {
+        const int h = (int)(ii / per), i = (int)(ii % per);
+        const double Th = hp.n > 0 ? hp.T[h] : T, wh = hp.n > 0 ? hp.w[h] : w;
+        float *Dh = Dx + (size_t)h * (per_slot ? S : n);
+        int *dh = delta + (size_t)h * S;
         if (per_slot) {
-            if (i < S) Dx[i] = (float)dirichlet_closed(M, w, (double)(x0 - grid_delta(i, T, S)));
-            else delta[i - S] = grid_delta(i - S, T, S);
+            if (i < S) Dh[i] = (float)dirichlet_closed(M, wh, (double)(x0 - grid_delta(i, Th, S)));
+            else dh[i - S] = grid_delta(i - S, Th, S);
         } else {
-            if (i < n) Dx[i] = (float)dirichlet_closed(M, w, (double)(x0 + i));
-            else delta[i - n] = grid_delta(i - n, T, S);
+            if (i < n) Dh[i] = (float)dirichlet_closed(M, wh, (double)(x0 + i));
+            else dh[i - n] = grid_delta(i - n, Th, S);
         }
     }
 }
@@ -105,11 +114,15 @@ template <typename T, int CPL>
 __global__ void __launch_bounds__(256) k_decay_kscan(const T *__restrict__ q, const T *__restrict__ k,
                                                      const float *__restrict__ Dx, const int *__restrict__ delta,
                                                      int S, int L, int d, int dmax, int nsb, float scale,
+                                                     int H, int hs_dx, int hs_delta,
                                                      const float *state_in, float *state_out, float *__restrict__ sc) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long bh = blockIdx.x / nsb;
     const int j = (blockIdx.x % nsb) * 8 + warp;
     if (j >= S) return;                       // whole warps only; no block-level synchronisation below
+    const int hd = (int)(bh % H);             // this head's D_M table and grid (strides 0 when shared)
+    Dx += (size_t)hd * hs_dx;
+    delta += (size_t)hd * hs_delta;
     const int off = dmax - delta[j];          // Dx index of token t is t + off
     const size_t row0 = (size_t)bh * L * d + lane * CPL;
     const size_t st = (size_t)bh * S * 2 * d + (size_t)j * d + lane * CPL;   // K half, slot j
@@ -167,11 +180,12 @@ __global__ void __launch_bounds__(256) k_decay_kscan(const T *__restrict__ q, co
 
 // lse[head][t] = log sum_{j : pos0 + t >= Delta_j} exp(sc[head][j][t]).
 __global__ void k_decay_lse(const float *__restrict__ sc, const int *__restrict__ delta, int S, int L, long long pos0,
-                            long long n, float *__restrict__ lse) {
+                            long long n, int H, int hs_delta, float *__restrict__ lse) {
     const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
     if (i >= n) return;
     const long long bh = i / L;
     const int t = (int)(i % L);
+    delta += (size_t)(bh % H) * hs_delta;
     const float *col = sc + (size_t)bh * S * L + t;
     float m = -INFINITY, sum = 0.f;
     for (int j = 0; j < S; ++j) {
@@ -192,8 +206,8 @@ __global__ void k_decay_lse(const float *__restrict__ sc, const int *__restrict_
 template <typename T>
 __global__ void __launch_bounds__(1024) k_decay_vscan(const T *__restrict__ v, const float *__restrict__ Dx, const int *__restrict__ delta,
                               const float *__restrict__ sc, const float *__restrict__ lse, int S, int L, int dk, int dv,
-                              int dmax, int ncb, int ng, long long pos0, const float *state_in, float *state_out,
-                              T *__restrict__ o) {
+                              int dmax, int ncb, int ng, long long pos0, int H, int hs_dx, int hs_delta,
+                              const float *state_in, float *state_out, T *__restrict__ o) {
     constexpr int G = kSlotsPerWarpGroup, TT = kVTile;
     extern __shared__ float4 smem4[];
     const int spad = ng * G, sp = spad + 4;            // row stride: a multiple of 4 floats
@@ -205,6 +219,8 @@ __global__ void __launch_bounds__(1024) k_decay_vscan(const T *__restrict__ v, c
     const int g = threadIdx.x >> 5, lane = threadIdx.x & 31, nthr = blockDim.x;
     const long long bh = blockIdx.x / ncb;
     const int c = (blockIdx.x % ncb) * 32 + lane;
+    Dx += (size_t)(bh % H) * hs_dx;           // this head's D_M table and grid (strides 0 when shared)
+    delta += (size_t)(bh % H) * hs_delta;
     for (int i = threadIdx.x; i < spad; i += nthr) dl[i] = i < S ? delta[i] : 0;
     const size_t vst = (size_t)bh * S * (dk + dv) + (size_t)S * dk + c;   // V half, column c
     float V[G];
@@ -273,12 +289,15 @@ template <typename T, int CPL>
 __global__ void __launch_bounds__(256) k_decay_decode(const T *__restrict__ q, const T *__restrict__ k,
                                                       const T *__restrict__ v, const float *__restrict__ Dj,
                                                       const int *__restrict__ delta, int S, int d, long long pos,
-                                                      float scale, float *__restrict__ state, T *__restrict__ o) {
+                                                      float scale, int H, int hs, float *__restrict__ state,
+                                                      T *__restrict__ o) {
     __shared__ float s_sc[256];
     __shared__ float s_red[kDecodeWarps][128];
     __shared__ float s_stat[2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long bh = blockIdx.x;
+    Dj += (size_t)(bh % H) * hs;              // this head's weights D_j(pos) and grid (stride 0 when shared)
+    delta += (size_t)(bh % H) * hs;
     float *Ks = state + (size_t)bh * 2 * S * d + lane * CPL;
     float *Vs = Ks + (size_t)S * d;
     float qv[CPL], kv[CPL], vv[CPL];
@@ -365,10 +384,11 @@ __global__ void __launch_bounds__(256) k_decay_decode(const T *__restrict__ q, c
 int host_dmax(const OpDims &d) { return (int)rint((double)(d.S - 1) * d.T / (double)d.S); }
 
 struct DecayWs {
-    int *delta;
-    float *Dx;
+    int *delta;      // [nh][S]
+    float *Dx;       // [nh][S] (decode) or [nh][L + max Delta + 1] (forward)
     float *sc;
     float *lse;
+    int hs_dx, hs_delta;   // per-head strides of Dx and delta (0 when the heads share one period)
 };
 
 size_t decay_table_len(const OpDims &d) { return (size_t)d.L + (size_t)host_dmax(d) + 1; }
@@ -380,8 +400,12 @@ size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w)
         off += align_up(bytes, 256);
         return p;
     };
-    w->delta = reinterpret_cast<int *>(take(sizeof(int) * d.S));
-    w->Dx = reinterpret_cast<float *>(take(sizeof(float) * (decode ? (size_t)d.S : decay_table_len(d))));
+    const size_t nh = d.periods ? (size_t)d.H : 1;
+    const size_t per = decode ? (size_t)d.S : decay_table_len(d);
+    w->delta = reinterpret_cast<int *>(take(sizeof(int) * nh * d.S));
+    w->Dx = reinterpret_cast<float *>(take(sizeof(float) * nh * per));
+    w->hs_dx = d.periods ? (int)per : 0;
+    w->hs_delta = d.periods ? d.S : 0;
     w->sc = nullptr;
     w->lse = nullptr;
     if (!decode) {
@@ -401,11 +425,14 @@ cudaError_t kscan_dispatch(const OpDims &d, const DecayWs &w, const void *q, con
     ProfScope ps(BLA_K_DECAY, st);
     switch (d.dk) {
     case 32: k_decay_kscan<T, 1><<<(unsigned)blocks, 256, 0, st>>>(qq, kk, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
-                                                                    d.scale, state_in, state_out, w.sc); break;
+                                                                    d.scale, d.H, w.hs_dx, w.hs_delta, state_in,
+                                                                    state_out, w.sc); break;
     case 64: k_decay_kscan<T, 2><<<(unsigned)blocks, 256, 0, st>>>(qq, kk, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
-                                                                    d.scale, state_in, state_out, w.sc); break;
+                                                                    d.scale, d.H, w.hs_dx, w.hs_delta, state_in,
+                                                                    state_out, w.sc); break;
     default: k_decay_kscan<T, 4><<<(unsigned)blocks, 256, 0, st>>>(qq, kk, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
-                                                                    d.scale, state_in, state_out, w.sc); break;
+                                                                    d.scale, d.H, w.hs_dx, w.hs_delta, state_in,
+                                                                    state_out, w.sc); break;
     }
     return cudaGetLastError();
 }
@@ -427,17 +454,19 @@ cudaError_t vscan_dispatch(const OpDims &d, const DecayWs &w, const float *lse, 
     const long long blocks = (long long)d.B * d.H * ncb;
     ProfScope ps(BLA_K_DECAY, st);
     k_decay_vscan<T><<<(unsigned)blocks, 32 * ng, smem, st>>>(static_cast<const T *>(v), w.Dx, w.delta, w.sc, lse,
-                                                              d.S, d.L, d.dk, d.dv, dmax, ncb, ng, pos0, state_in,
-                                                              state_out, static_cast<T *>(o));
+                                                              d.S, d.L, d.dk, d.dv, dmax, ncb, ng, pos0, d.H, w.hs_dx,
+                                                              w.hs_delta, state_in, state_out, static_cast<T *>(o));
     return cudaGetLastError();
 }
 
 cudaError_t table_launch(const OpDims &d, long long x0, int n, int per_slot, const DecayWs &w, cudaStream_t st) {
-    const int total = (per_slot ? d.S : n) + d.S;
-    int blocks = (total + 255) / 256;
+    HeadPeriods hp;
+    head_periods(d, d.omega_in, &hp);   // hp.n = 0 when the heads share one period
+    const long long total = (long long)((per_slot ? d.S : n) + d.S) * (hp.n > 0 ? hp.n : 1);
+    long long blocks = (total + 255) / 256;
     if (blocks > 1024) blocks = 1024;
     ProfScope ps(BLA_K_DECAY, st);
-    k_decay_table<<<blocks, 256, 0, st>>>(d.M, d.w, d.T, d.S, x0, n, per_slot, w.Dx, w.delta);
+    k_decay_table<<<(int)blocks, 256, 0, st>>>(d.M, hp, d.T, d.w, d.S, x0, n, per_slot, w.Dx, w.delta);
     return cudaGetLastError();
 }
 
@@ -465,7 +494,7 @@ cudaError_t launch_decay_forward(const OpDims &d, long long pos0, const void *q,
     const long long nt = (long long)d.B * d.H * d.L;
     if (nt > 0) {
         ProfScope ps(BLA_K_DECAY, st);
-        k_decay_lse<<<(unsigned)((nt + 255) / 256), 256, 0, st>>>(w.sc, w.delta, d.S, d.L, pos0, nt, l);
+        k_decay_lse<<<(unsigned)((nt + 255) / 256), 256, 0, st>>>(w.sc, w.delta, d.S, d.L, pos0, nt, d.H, w.hs_delta, l);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     return d.dtype == BLA_BF16 ? vscan_dispatch<__nv_bfloat16>(d, w, l, v, o, dmax, pos0, state_in, state_out, st)
@@ -485,18 +514,18 @@ cudaError_t launch_decay_decode(const OpDims &d, long long pos, const void *q, c
         const T *qq = static_cast<const T *>(q), *kk = static_cast<const T *>(k), *vv = static_cast<const T *>(v);
         T *oo = static_cast<T *>(o);
         switch (d.dk) {
-        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
+        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
         }
     } else {
         using T = float;
         const T *qq = static_cast<const T *>(q), *kk = static_cast<const T *>(k), *vv = static_cast<const T *>(v);
         T *oo = static_cast<T *>(o);
         switch (d.dk) {
-        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
+        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
         }
     }
     return cudaGetLastError();
