@@ -95,7 +95,7 @@ typedef enum { BLA_PHASE_LAG = 0, BLA_PHASE_ABSOLUTE = 1 } bla_phase_mode;
 /* Which entry point a workspace size is asked for. */
 typedef enum {
     BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2, BLA_WS_FORWARD_HOST = 3,
-    BLA_WS_DECAY_FORWARD = 4, BLA_WS_DECAY_DECODE = 5
+    BLA_WS_DECAY_FORWARD = 4, BLA_WS_DECAY_DECODE = 5, BLA_WS_DECAY_BACKWARD = 6
 } bla_ws_kind;
 
 /*
@@ -225,6 +225,18 @@ bla_status bla_decay_forward(const bla_params *p, long long pos0, const void *q,
  */
 bla_status bla_decay_decode_step(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
                                  float *state, void *o, void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Backward of bla_decay_forward from the zero state (state_in = NULL), tokens at absolute indices
+ * pos0 ..: given dout = dL/do, writes dq, dk, dv (shapes and dtype of q, k, v).  o and lse are the
+ * forward's outputs.  The vector-Jacobian product of the decayed recurrence; the paper trains
+ * through it but prints no formula.
+ *   workspace  device scratch of >= bla_workspace_bytes(p, BLA_WS_DECAY_BACKWARD) bytes (two
+ *              B*H*S*L fp32 buffers and the D_M table).
+ */
+bla_status bla_decay_backward(const bla_params *p, long long pos0, const void *q, const void *k, const void *v,
+                              const void *o, const void *dout, const float *lse, void *dq, void *dk, void *dv,
+                              void *workspace, size_t ws_bytes, void *stream);
 
 /* ---------------------------------------------------------------- instrumentation
  * (no paper counterpart: measurement support for benchmarks and tests)

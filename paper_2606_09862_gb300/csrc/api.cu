@@ -340,6 +340,7 @@ size_t bla_workspace_bytes(const bla_params *p, int which) {
     case BLA_WS_BACKWARD: return bwd_workspace_bytes(d);
     case BLA_WS_DECAY_FORWARD: return check_decay(p, &d, true) == BLA_OK ? decay_workspace_bytes(d, false) : 0;
     case BLA_WS_DECAY_DECODE: return check_decay(p, &d, false) == BLA_OK ? decay_workspace_bytes(d, true) : 0;
+    case BLA_WS_DECAY_BACKWARD: return check_decay(p, &d, true) == BLA_OK ? decay_backward_workspace_bytes(d) : 0;
     default: return 0;
     }
 }
@@ -475,6 +476,27 @@ bla_status bla_decay_decode_step(const bla_params *p, long long pos, const void 
     if ((s = check_ws(workspace, ws_bytes, decay_workspace_bytes(d, true))) != BLA_OK) return s;
     cudaError_t e = launch_decay_decode(d, pos, q, k, v, state, o, workspace, reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "decay decode launch");
+    return BLA_OK;
+}
+
+bla_status bla_decay_backward(const bla_params *p, long long pos0, const void *q, const void *k, const void *v,
+                              const void *o, const void *dout, const float *lse, void *dq, void *dk, void *dv,
+                              void *workspace, size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    NvtxRange nvtx("bla_decay_backward");
+    OpDims d;
+    bla_status s = check_decay(p, &d, true);
+    if (s != BLA_OK) return s;
+    if (pos0 < 0) return fail(BLA_ERR_INVALID, "pos0 must be >= 0 (got %lld)", pos0);
+    if (d.L > 0 && (!q || !k || !v || !o || !dout || !lse || !dq || !dk || !dv))
+        return fail(BLA_ERR_INVALID, "q, k, v, o, dout, lse, dq, dk and dv must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(dout) || !aligned16(lse) ||
+        !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    if ((s = check_ws(workspace, ws_bytes, decay_backward_workspace_bytes(d))) != BLA_OK) return s;
+    cudaError_t e = launch_decay_backward(d, pos0, q, k, v, o, dout, lse, dq, dk, dv, workspace,
+                                          reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "decay backward launch");
     return BLA_OK;
 }
 

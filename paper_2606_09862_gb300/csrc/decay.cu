@@ -380,6 +380,136 @@ __global__ void __launch_bounds__(256) k_decay_decode(const T *__restrict__ q, c
     }
 }
 
+// ------------------------------------------------------------------ backward (VJP)
+// Unrolled, the decayed slot state is a fixed linear map of the tokens,
+//     K~_j(t) = sum_{u<=t} W_j(t,u) k_u,     W_j(t,u) = D_j(u) prod_{u<x<=t} (1 - D_j(x)),
+// so the chain rule through s = scale q . K~, the masked softmax and o = sum_j p V~ gives, with
+// upstream do:
+//     dp[t,j] = do_t . V~_j(t),     g[t,j] = scale p[t,j] (dp[t,j] - do_t . o_t)
+//     dq_t = sum_j g[t,j] K~_j(t)                                                  forward in time
+//     lK_j(t) = g[t,j] q_t + (1 - D_j(t+1)) lK_j(t+1),    dk_t = sum_j D_j(t) lK_j(t)    backward
+//     lV_j(t) = p[t,j] do_t + (1 - D_j(t+1)) lV_j(t+1),   dv_t = sum_j D_j(t) lV_j(t)    backward
+// dp comes from the K scan with (do, v) in place of (q, k); the three sums over slots run in
+// k_decay_rscan, the V scan's layout with the per-token factors (f, u, w) of
+//     X_j <- f X_j + u x_t,     out_t = sum_j w X_j
+// staged per tile: forward in time f = 1 - D_j(t), u = D_j(t), w = g; backward in time
+// f = 1 - D_j(t+1), u = g or p, w = D_j(t).
+
+// g[head][j][t] = scale p (dp - do_t . o_t), in place of dp; one thread per token.
+template <typename T>
+__global__ void k_decay_ds(const float *__restrict__ sc, const float *__restrict__ lse, float *__restrict__ g,
+                           const T *__restrict__ dout, const T *__restrict__ o, const int *__restrict__ delta, int S,
+                           int L, int dv, long long pos0, float scale, long long n, int H, int hs_delta) {
+    const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const long long bh = i / L;
+    const int t = (int)(i % L);
+    delta += (size_t)(bh % H) * hs_delta;
+    float rd = 0.f;
+    for (int c = 0; c < dv; ++c) rd = fmaf(load_elem<T>(dout, (size_t)i * dv + c), load_elem<T>(o, (size_t)i * dv + c), rd);
+    const size_t col = (size_t)bh * S * L + t;
+    const float l = lse[i];
+    for (int j = 0; j < S; ++j) {
+        const size_t e = col + (size_t)j * L;
+        g[e] = (pos0 + t >= delta[j]) ? scale * expf(sc[e] - l) * (g[e] - rd) : 0.f;
+    }
+}
+
+// Reduce scan over the slots for 32 columns of one head (layout of k_decay_vscan).  REV = false:
+// forward in time, f = 1 - D_j(t), u = D_j(t), w = wt(t, j).  REV = true: backward in time,
+// f = 1 - D_j(t+1), u = wt(t, j), w = D_j(t).  wt(t, j) = G[j][t] when lse is NULL, else the slot
+// probability exp(G[j][t] - lse[t]) (G holding scores; 0 on masked slots).
+template <typename T, bool REV>
+__global__ void __launch_bounds__(1024) k_decay_rscan(const T *__restrict__ x, const float *__restrict__ Dx,
+                                                      const int *__restrict__ delta, const float *__restrict__ G,
+                                                      const float *__restrict__ lse, int S, int L, int dx, int dmax,
+                                                      int ncb, int ng, long long pos0, int H, int hs_dx, int hs_delta,
+                                                      T *__restrict__ out) {
+    constexpr int G8 = kSlotsPerWarpGroup, TT = kVTile;
+    extern __shared__ float4 smem4[];
+    const int spad = ng * G8, sp = spad + 4;
+    float *Ft = reinterpret_cast<float *>(smem4);      // [TT][sp]
+    float *Ut = Ft + TT * sp;                          // [TT][sp]
+    float *Wt = Ut + TT * sp;                          // [TT][sp]
+    float *red = Wt + TT * sp;                         // [TT][ng][32]
+    float *Xt = red + TT * ng * 32;                    // [TT][32]
+    int *dl = reinterpret_cast<int *>(Xt + TT * 32);   // [spad]
+    const int g = threadIdx.x >> 5, lane = threadIdx.x & 31, nthr = blockDim.x;
+    const long long bh = blockIdx.x / ncb;
+    const int c = (blockIdx.x % ncb) * 32 + lane;
+    Dx += (size_t)(bh % H) * hs_dx;           // this head's D_M table and grid (strides 0 when shared)
+    delta += (size_t)(bh % H) * hs_delta;
+    for (int i = threadIdx.x; i < spad; i += nthr) dl[i] = i < S ? delta[i] : 0;
+    float X[G8];
+#pragma unroll
+    for (int jj = 0; jj < G8; ++jj) X[jj] = 0.f;
+    __syncthreads();
+    const T *xb = x + (size_t)bh * L * dx + (c - lane);
+    T *oh = out + (size_t)bh * L * dx + c;
+    const float *gh = G + (size_t)bh * S * L;
+    const float *lh = lse ? lse + (size_t)bh * L : nullptr;
+    for (int t0 = 0; t0 < L; t0 += TT) {
+        // tile position tt holds token t = t0 + tt (forward) or L - 1 - (t0 + tt) (backward)
+        for (int idx = threadIdx.x; idx < TT * spad; idx += nthr) {
+            const int tt = idx % TT, j = idx / TT, r = t0 + tt;
+            float f = 0.f, u = 0.f, w = 0.f;
+            if (j < S && r < L) {
+                const int t = REV ? L - 1 - r : r;
+                float wt;
+                if (lh) wt = (pos0 + t >= dl[j]) ? expf(gh[(size_t)j * L + t] - lh[t]) : 0.f;
+                else wt = gh[(size_t)j * L + t];
+                const float Dt = Dx[t + dmax - dl[j]];
+                if (REV) {
+                    f = 1.f - Dx[t + 1 + dmax - dl[j]];   // entry L + dmax - Delta_j < L + dmax + 1 at t = L - 1
+                    u = wt;
+                    w = Dt;
+                } else {
+                    f = 1.f - Dt;
+                    u = Dt;
+                    w = wt;
+                }
+            }
+            Ft[tt * sp + j] = f;
+            Ut[tt * sp + j] = u;
+            Wt[tt * sp + j] = w;
+        }
+        for (int idx = threadIdx.x; idx < TT * 32; idx += nthr) {
+            const int r = t0 + (idx >> 5);
+            const int t = REV ? L - 1 - r : r;
+            Xt[idx] = r < L ? load_elem<T>(xb, (size_t)t * dx + (idx & 31)) : 0.f;
+        }
+        __syncthreads();
+        const int nt = min(TT, L - t0);
+#pragma unroll 4
+        for (int tt = 0; tt < nt; ++tt) {
+            const float xv = Xt[tt * 32 + lane];
+            const float4 *f4 = reinterpret_cast<const float4 *>(Ft + tt * sp + g * G8);
+            const float4 *u4 = reinterpret_cast<const float4 *>(Ut + tt * sp + g * G8);
+            const float4 *w4 = reinterpret_cast<const float4 *>(Wt + tt * sp + g * G8);
+            const float4 fa = f4[0], fb = f4[1], ua = u4[0], ub = u4[1], wa = w4[0], wb = w4[1];
+            const float ff[G8] = {fa.x, fa.y, fa.z, fa.w, fb.x, fb.y, fb.z, fb.w};
+            const float uu[G8] = {ua.x, ua.y, ua.z, ua.w, ub.x, ub.y, ub.z, ub.w};
+            const float ww[G8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
+            float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll
+            for (int jj = 0; jj < G8; jj += 2) {
+                X[jj] = fmaf(ff[jj], X[jj], uu[jj] * xv);
+                X[jj + 1] = fmaf(ff[jj + 1], X[jj + 1], uu[jj + 1] * xv);
+                acc0 = fmaf(ww[jj], X[jj], acc0);
+                acc1 = fmaf(ww[jj + 1], X[jj + 1], acc1);
+            }
+            red[(tt * ng + g) * 32 + lane] = acc0 + acc1;
+        }
+        __syncthreads();
+        for (int tt = g; tt < nt; tt += ng) {
+            float sum = 0.f;
+            for (int gg = 0; gg < ng; ++gg) sum += red[(tt * ng + gg) * 32 + lane];
+            const int r = t0 + tt;
+            store_elem<T>(oh, (size_t)(REV ? L - 1 - r : r) * dx, sum);
+        }
+    }
+}
+
 // Largest Delta_j (the grid is non-decreasing in j), computed exactly as the device does.
 int host_dmax(const OpDims &d) { return (int)rint((double)(d.S - 1) * d.T / (double)d.S); }
 
@@ -389,11 +519,12 @@ struct DecayWs {
     float *sc;
     float *lse;
     int hs_dx, hs_delta;   // per-head strides of Dx and delta (0 when the heads share one period)
+    float *g = nullptr;    // backward: dp, then g = scale ds, [BH][S][L]
 };
 
 size_t decay_table_len(const OpDims &d) { return (size_t)d.L + (size_t)host_dmax(d) + 1; }
 
-size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w) {
+size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w, bool backward = false) {
     size_t off = 0;
     auto take = [&](size_t bytes) {
         char *p = base ? base + off : nullptr;
@@ -412,6 +543,8 @@ size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w)
         const size_t BH = (size_t)d.B * d.H;
         w->sc = reinterpret_cast<float *>(take(sizeof(float) * BH * d.S * (size_t)(d.L > 0 ? d.L : 1)));
         if (own_lse) w->lse = reinterpret_cast<float *>(take(sizeof(float) * BH * (size_t)(d.L > 0 ? d.L : 1)));
+        w->g = backward ? reinterpret_cast<float *>(take(sizeof(float) * BH * d.S * (size_t)(d.L > 0 ? d.L : 1)))
+                        : nullptr;
     }
     return off;
 }
@@ -470,7 +603,89 @@ cudaError_t table_launch(const OpDims &d, long long x0, int n, int per_slot, con
     return cudaGetLastError();
 }
 
+// K scan with explicit operands: out[head][j][t] = scale z_t . X_j(t), X_j <- (1 - D) X_j + D x_t.
+template <typename T>
+cudaError_t kscan_launch(const OpDims &d, const DecayWs &w, const void *z, const void *x, int dmax, float scale,
+                         float *out, cudaStream_t st) {
+    const int nsb = (d.S + 7) / 8;
+    const long long blocks = (long long)d.B * d.H * nsb;
+    const T *zz = static_cast<const T *>(z), *xx = static_cast<const T *>(x);
+    ProfScope ps(BLA_K_DECAY, st);
+    switch (d.dk) {
+    case 32: k_decay_kscan<T, 1><<<(unsigned)blocks, 256, 0, st>>>(zz, xx, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
+                                                                    scale, d.H, w.hs_dx, w.hs_delta, nullptr, nullptr,
+                                                                    out); break;
+    case 64: k_decay_kscan<T, 2><<<(unsigned)blocks, 256, 0, st>>>(zz, xx, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
+                                                                    scale, d.H, w.hs_dx, w.hs_delta, nullptr, nullptr,
+                                                                    out); break;
+    default: k_decay_kscan<T, 4><<<(unsigned)blocks, 256, 0, st>>>(zz, xx, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
+                                                                    scale, d.H, w.hs_dx, w.hs_delta, nullptr, nullptr,
+                                                                    out); break;
+    }
+    return cudaGetLastError();
+}
+
+size_t rscan_smem(int ng) {
+    const int spad = ng * kSlotsPerWarpGroup, sp = spad + 4;
+    return sizeof(float) * ((size_t)3 * kVTile * sp + (size_t)kVTile * ng * 32 + (size_t)kVTile * 32) +
+           sizeof(int) * (size_t)spad;
+}
+
+template <typename T, bool REV>
+cudaError_t rscan_launch(const OpDims &d, const DecayWs &w, const void *x, const float *G, const float *lse, int dmax,
+                         long long pos0, void *out, cudaStream_t st) {
+    const int ncb = d.dv / 32;
+    const int ng = (d.S + kSlotsPerWarpGroup - 1) / kSlotsPerWarpGroup;
+    const size_t smem = rscan_smem(ng);
+    cudaError_t e = cudaFuncSetAttribute(k_decay_rscan<T, REV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const long long blocks = (long long)d.B * d.H * ncb;
+    ProfScope ps(BLA_K_DECAY, st);
+    k_decay_rscan<T, REV><<<(unsigned)blocks, 32 * ng, smem, st>>>(static_cast<const T *>(x), w.Dx, w.delta, G, lse,
+                                                                   d.S, d.L, d.dv, dmax, ncb, ng, pos0, d.H, w.hs_dx,
+                                                                   w.hs_delta, static_cast<T *>(out));
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t backward_run(const OpDims &d, const DecayWs &w, long long pos0, const void *q, const void *k,
+                         const void *v, const void *o, const void *dout, const float *lse, void *dq, void *dk,
+                         void *dv, int dmax, cudaStream_t st) {
+    cudaError_t e;
+    if ((e = kscan_launch<T>(d, w, q, k, dmax, d.scale, w.sc, st)) != cudaSuccess) return e;    // scores
+    if ((e = kscan_launch<T>(d, w, dout, v, dmax, 1.f, w.g, st)) != cudaSuccess) return e;     // dp
+    const long long nt = (long long)d.B * d.H * d.L;
+    {
+        ProfScope ps(BLA_K_DECAY, st);
+        k_decay_ds<T><<<(unsigned)((nt + 255) / 256), 256, 0, st>>>(w.sc, lse, w.g, static_cast<const T *>(dout),
+                                                                    static_cast<const T *>(o), w.delta, d.S, d.L,
+                                                                    d.dv, pos0, d.scale, nt, d.H, w.hs_delta);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    if ((e = rscan_launch<T, false>(d, w, k, w.g, nullptr, dmax, pos0, dq, st)) != cudaSuccess) return e;
+    if ((e = rscan_launch<T, true>(d, w, q, w.g, nullptr, dmax, pos0, dk, st)) != cudaSuccess) return e;
+    return rscan_launch<T, true>(d, w, dout, w.sc, lse, dmax, pos0, dv, st);
+}
+
 }  // namespace
+
+size_t decay_backward_workspace_bytes(const OpDims &d) {
+    DecayWs w;
+    return carve(d, false, false, nullptr, &w, true);
+}
+
+cudaError_t launch_decay_backward(const OpDims &d, long long pos0, const void *q, const void *k, const void *v,
+                                  const void *o, const void *dout, const float *lse, void *dq, void *dk, void *dv,
+                                  void *ws, cudaStream_t st) {
+    if (d.L == 0) return cudaSuccess;
+    DecayWs w;
+    carve(d, false, false, static_cast<char *>(ws), &w, true);
+    const int dmax = host_dmax(d);
+    cudaError_t e = table_launch(d, pos0 - dmax, (int)decay_table_len(d), 0, w, st);
+    if (e != cudaSuccess) return e;
+    return d.dtype == BLA_BF16 ? backward_run<__nv_bfloat16>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st)
+                               : backward_run<float>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st);
+}
 
 size_t decay_table_entries(const OpDims &d) { return decay_table_len(d); }
 

@@ -170,6 +170,14 @@ def test_decay_argument_checks(lib):
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_FORWARD) >= 2 * 3 * 8 * 100 * 4
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_DECODE) > 0
     assert lib.bla_workspace_bytes(ctypes.byref(_params()), bla.BLA_WS_DECAY_FORWARD) == 0
+    bwd = lib.bla_decay_backward
+    assert bwd(ctypes.byref(_params()), 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30,
+               None) == bla.BLA_ERR_UNSUPPORTED                                       # lag form
+    assert bwd(ctypes.byref(_params(phase_mode=ab)), -1, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE,
+               1 << 30, None) == bla.BLA_ERR_INVALID
+    assert bwd(ctypes.byref(_params(phase_mode=ab)), 0, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE,
+               1 << 30, None) == bla.BLA_ERR_INVALID                                  # no lse
+    assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_BACKWARD) >= 2 * 2 * 3 * 8 * 100 * 4
     # grids that would exceed the launch limits are refused before any launch
     assert fwd(_params(phase_mode=ab, B=1 << 20, H=1 << 10, S=64, window=64.0)) == bla.BLA_ERR_UNSUPPORTED
 

@@ -85,3 +85,21 @@ def test_shared_period_unchanged(orc):
     b = bla.bla_forward_chunked(q, k, v, 4, 7, 16.0, chunk=16)[0]
     bla.bla_device_error()
     assert rel(a.cpu().numpy(), b.cpu().numpy()) <= 1e-6
+
+
+def test_decay_backward(orc):
+    """The decayed VJP with one period per head against the oracle's per-head VJP."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_dout, make_qkv
+    dev = require_cuda()
+    B, H, L, d, M, S = 1, 3, 60, 32, 4, 7
+    q, k, v = make_qkv(B, H, L, d, dtype="f32", seed=17)
+    do = make_dout(B, H, L, d, dtype="f32", seed=17)
+    tq, tk, tv, tdo = (to_dev(x, dev, torch.float32) for x in (q, k, v, do))
+    o, lse, _ = bla.bla_decay_forward(tq, tk, tv, M, S, TS)
+    got = bla.bla_decay_backward(tq, tk, tv, o, tdo, lse, M, S, TS)
+    bla.bla_device_error()
+    ref = orc.backward_decay(q, k, v, do, M, S, TS)
+    for name, a, b in zip(("dq", "dk", "dv"), got, ref):
+        assert rel(a.cpu().numpy(), b) <= 1e-4, (name, rel(a.cpu().numpy(), b))
