@@ -451,7 +451,7 @@ bla_status bla_decay_forward(const bla_params *p, long long pos0, const void *q,
     bla_status s = check_decay(p, &d, true);
     if (s != BLA_OK) return s;
     if (pos0 < 0) return fail(BLA_ERR_INVALID, "pos0 must be >= 0 (got %lld)", pos0);
-    if (!q || !k || !v || !o) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
+    if (d.L > 0 && (!q || !k || !v || !o)) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)) ||
         (state_in && !aligned16(state_in)) || (state_out && !aligned16(state_out)))
         return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");

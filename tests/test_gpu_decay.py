@@ -182,3 +182,19 @@ def test_backward_against_oracle_vjp(orc, dtype, B, H, L, d, M, S, T, pos0):
     tol = 1e-4 if dtype == "f32" else TOL_GRAD
     for name, a, b in zip(("dq", "dk", "dv"), got, ref):
         assert rel(a.float().cpu().numpy(), b) <= tol, (name, rel(a.float().cpu().numpy(), b))
+
+
+def test_empty_sequence_passes_state_through():
+    """L = 0: nothing to attend; the final state is the given one (or zero without one)."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    dev = require_cuda()
+    z = torch.zeros((1, 2, 0, 32), device=dev)
+    st0 = torch.randn((1, 2, 2, 5, 32), device=dev)
+    st = st0.clone()
+    o, _, out = bla.bla_decay_forward(z, z, z, 3, 5, 9.0, pos0=4, state=st, want_state=True)
+    _, _, zero = bla.bla_decay_forward(z, z, z, 3, 5, 9.0, want_state=True)
+    bla.bla_device_error()
+    assert o.shape == (1, 2, 0, 32)
+    assert torch.equal(out, st0)
+    assert float(zero.abs().max()) == 0.0
