@@ -556,7 +556,7 @@ def measure_decay(bla, torch, dev, timed, peaks):
     pos = 4096, from a random fp32 slot state.  The forward is a scan on the CUDA cores: its flops
     are 10 S d per token and head (state update 3 + score 2 for K and for V, FMA = 2); the decode
     reads and writes the whole slot state once."""
-    from paper_2606_09862_gb300.inputs import WORKLOADS, make_decode_step, make_qkv, make_slot_state
+    from paper_2606_09862_gb300.inputs import WORKLOADS, make_decode_step, make_dout, make_qkv, make_slot_state
     w = WORKLOADS["decay_bf16_lm"]
     q, k, v = (torch.from_numpy(x).to(torch.bfloat16).to(dev) for x in make_qkv(w.B, w.H, w.L, w.d, "bf16", seed=0))
     par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16, phase_mode="absolute")
@@ -569,7 +569,18 @@ def measure_decay(bla, torch, dev, timed, peaks):
                        "bound": "alu", "frac_alu": tf / FP32_SIMT_PEAK_TFLOPS,
                        "alu_peak_tflops": FP32_SIMT_PEAK_TFLOPS},
            "shape": "B=%d H=%d L=%d d=%d M=%d S=%d T=%d bf16 absolute+decay" % (w.B, w.H, w.L, w.d, w.M, w.S, w.T)}
-    del q, k, v, ws, o
+    # backward: two dot scans (scores, dp) and three reduce scans (dq, dk, dv), 25 S d flops per
+    # token-head (each scan 5 S d)
+    o, lse, _ = bla.bla_decay_forward(q, k, v, w.M, w.S, w.T, workspace=ws)
+    do = torch.from_numpy(make_dout(w.B, w.H, w.L, w.d, "bf16", seed=0)).to(torch.bfloat16).to(dev)
+    parb = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16, phase_mode="absolute")
+    wsb = torch.empty(bla.bla_workspace_bytes(parb, bla.BLA_WS_DECAY_BACKWARD), dtype=torch.uint8, device=dev)
+    ms_b = timed(lambda: bla.bla_decay_backward(q, k, v, o, do, lse, w.M, w.S, w.T, workspace=wsb))
+    fb = 25.0 * w.B * w.H * w.L * w.S * w.d
+    res["backward"] = {"ms": ms_b, "tokens_per_s": w.B * w.L / (ms_b / 1000.0),
+                       "tflops_fp32": fb / (ms_b / 1000.0) / 1e12, "flops": fb, "bound": "alu",
+                       "frac_alu": fb / (ms_b / 1000.0) / 1e12 / FP32_SIMT_PEAK_TFLOPS}
+    del q, k, v, ws, o, lse, do, wsb
     wd = WORKLOADS["decay_decode_bf16"]
     qd, kd, vd = (torch.from_numpy(x).to(torch.bfloat16).to(dev)
                   for x in make_decode_step(0, wd.B, wd.H, wd.d, "bf16", seed=0))

@@ -70,6 +70,13 @@ typedef struct {
     double scale;       /* softmax scale; <= 0: 1/sqrt(d_k) (Eq. output, per head) */
     int dtype;          /* bla_dtype of q, k, v, o, dout, dq, dk, dv */
     int phase_mode;     /* bla_phase_mode: how the slots index time (0 = the lag form) */
+    const double *periods;  /* NULL: every head uses `window`.  Else a HOST array of H periods, one
+                               per head (Alg. 1 and Alg. 3 take T in R^H): head h's grid, frequency
+                               (2*pi/T_h unless omega > 0) and coefficients follow periods[h], each
+                               clamped to max(T_h, 2M-1); S must not exceed any of them.  Read
+                               during the call only.  At most 256 heads.  Supported by the fp32
+                               forward, bla_decode_step and the state-decay entry points; the others
+                               return BLA_ERR_UNSUPPORTED. */
 } bla_params;
 
 /* How a slot reads the past (bla_params.phase_mode).
@@ -88,7 +95,7 @@ typedef enum { BLA_PHASE_LAG = 0, BLA_PHASE_ABSOLUTE = 1 } bla_phase_mode;
 /* Which entry point a workspace size is asked for. */
 typedef enum {
     BLA_WS_FORWARD = 0, BLA_WS_BACKWARD = 1, BLA_WS_DECODE = 2, BLA_WS_FORWARD_HOST = 3,
-    BLA_WS_DECAY_FORWARD = 4, BLA_WS_DECAY_DECODE = 5
+    BLA_WS_DECAY_FORWARD = 4, BLA_WS_DECAY_DECODE = 5, BLA_WS_DECAY_BACKWARD = 6
 } bla_ws_kind;
 
 /*
@@ -218,6 +225,18 @@ bla_status bla_decay_forward(const bla_params *p, long long pos0, const void *q,
  */
 bla_status bla_decay_decode_step(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
                                  float *state, void *o, void *workspace, size_t ws_bytes, void *stream);
+
+/*
+ * Backward of bla_decay_forward from the zero state (state_in = NULL), tokens at absolute indices
+ * pos0 ..: given dout = dL/do, writes dq, dk, dv (shapes and dtype of q, k, v).  o and lse are the
+ * forward's outputs.  The vector-Jacobian product of the decayed recurrence; the paper trains
+ * through it but prints no formula.
+ *   workspace  device scratch of >= bla_workspace_bytes(p, BLA_WS_DECAY_BACKWARD) bytes (two
+ *              B*H*S*L fp32 buffers and the D_M table).
+ */
+bla_status bla_decay_backward(const bla_params *p, long long pos0, const void *q, const void *k, const void *v,
+                              const void *o, const void *dout, const float *lse, void *dq, void *dk, void *dv,
+                              void *workspace, size_t ws_bytes, void *stream);
 
 /* ---------------------------------------------------------------- instrumentation
  * (no paper counterpart: measurement support for benchmarks and tests)

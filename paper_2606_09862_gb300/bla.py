@@ -17,14 +17,15 @@ LIB_PATH = os.path.join(_HERE, "libbla_gb300.so")
 BLA_OK, BLA_ERR_INVALID, BLA_ERR_UNSUPPORTED, BLA_ERR_CUDA, BLA_ERR_TIMEOUT = range(5)
 BLA_F32, BLA_BF16 = 0, 1
 BLA_WS_FORWARD, BLA_WS_BACKWARD, BLA_WS_DECODE, BLA_WS_FORWARD_HOST = 0, 1, 2, 3
-BLA_WS_DECAY_FORWARD, BLA_WS_DECAY_DECODE = 4, 5
+BLA_WS_DECAY_FORWARD, BLA_WS_DECAY_DECODE, BLA_WS_DECAY_BACKWARD = 4, 5, 6
 BLA_PHASE_LAG, BLA_PHASE_ABSOLUTE = 0, 1
 PHASE_MODES = {"lag": BLA_PHASE_LAG, "absolute": BLA_PHASE_ABSOLUTE}
 
 EXPORTED = ("bla_workspace_bytes", "bla_forward_chunked", "bla_decode_step", "bla_backward",
             "bla_device_error", "bla_status_string", "bla_last_error_string", "bla_kernel_launches",
             "bla_profile_enable", "bla_profile_collect", "bla_decode_step_noalloc", "bla_forward_chunked_host",
-            "bla_selftest_wait_timeout", "bla_decay_forward", "bla_decay_decode_step")
+            "bla_selftest_wait_timeout", "bla_decay_forward", "bla_decay_decode_step",
+            "bla_decay_backward")
 
 # bla_kernel_id
 KERNELS = ("tables", "tables_bf16", "prepass", "scan", "kpass", "vpass", "fwd_f32", "decode", "bwd", "decay")
@@ -41,7 +42,8 @@ class Params(ctypes.Structure):
     _fields_ = [("B", ctypes.c_int), ("H", ctypes.c_int), ("L", ctypes.c_int),
                 ("d_k", ctypes.c_int), ("d_v", ctypes.c_int), ("M", ctypes.c_int), ("S", ctypes.c_int),
                 ("window", ctypes.c_double), ("omega", ctypes.c_double), ("chunk", ctypes.c_int),
-                ("scale", ctypes.c_double), ("dtype", ctypes.c_int), ("phase_mode", ctypes.c_int)]
+                ("scale", ctypes.c_double), ("dtype", ctypes.c_int), ("phase_mode", ctypes.c_int),
+                ("periods", ctypes.POINTER(ctypes.c_double))]
 
 
 _lib = None
@@ -73,6 +75,8 @@ def load():
     lib.bla_decay_forward.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_decay_decode_step.restype = ctypes.c_int
     lib.bla_decay_decode_step.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bla_decay_backward.restype = ctypes.c_int
+    lib.bla_decay_backward.argtypes = [P, ctypes.c_longlong, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_backward.restype = ctypes.c_int
     lib.bla_backward.argtypes = [P, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bla_device_error.restype = ctypes.c_int
@@ -125,9 +129,22 @@ def _phase_code(phase_mode):
 
 def make_params(B, H, L, d_k, d_v, M, S, window, omega=0.0, chunk=0, scale=0.0, dtype=torch.bfloat16,
                 phase_mode="lag"):
-    """bla_params; phase_mode is "lag" (Alg. 2, the default) or "absolute" (Alg. 1), or its code."""
-    return Params(int(B), int(H), int(L), int(d_k), int(d_v), int(M), int(S), float(window), float(omega),
-                  int(chunk), float(scale), _dtype_code(dtype), _phase_code(phase_mode))
+    """bla_params; phase_mode is "lag" (Alg. 2, the default) or "absolute" (Alg. 1), or its code.
+
+    ``window`` is the period T, or a sequence of H periods, one per head (Alg. 1 and Alg. 3 take
+    T in R^H), passed as ``periods``."""
+    periods = None
+    if isinstance(window, (list, tuple)) or (hasattr(window, "__len__") and not isinstance(window, str)):
+        vals = [float(x) for x in window]
+        if len(vals) != int(H):
+            raise BlaError(BLA_ERR_INVALID, "per-head periods need %d values, got %d" % (int(H), len(vals)))
+        periods = (ctypes.c_double * len(vals))(*vals)
+        window = max(vals)
+    p = Params(int(B), int(H), int(L), int(d_k), int(d_v), int(M), int(S), float(window), float(omega),
+               int(chunk), float(scale), _dtype_code(dtype), _phase_code(phase_mode))
+    if periods is not None:
+        p.periods = periods       # ctypes keeps the array alive with the structure
+    return p
 
 
 def bla_workspace_bytes(params, which):
@@ -245,6 +262,21 @@ def bla_decay_decode_step(q, k, v, state, pos, M, S, window, omega=0.0, scale=0.
     _check(load().bla_decay_decode_step(ctypes.byref(p), int(pos), _ptr(q), _ptr(k), _ptr(v), _ptr(state), _ptr(o),
                                         _ptr(ws), n, _stream(stream)))
     return o
+
+
+def bla_decay_backward(q, k, v, o, dout, lse, M, S, window, omega=0.0, scale=0.0, pos0=0, workspace=None,
+                       stream=None, phase_mode="absolute"):
+    """Gradients (dq, dk, dv) of bla_decay_forward (zero initial state, tokens from pos0) for
+    upstream gradient dout; o and lse are the forward's outputs."""
+    _need_cuda(q, k, v, o, dout, lse)
+    B, H, L, dk = q.shape
+    dv = v.shape[-1]
+    p = make_params(B, H, L, dk, dv, M, S, window, omega, 0, scale, q.dtype, phase_mode)
+    dq, dkk, dvv = torch.empty_like(q), torch.empty_like(k), torch.empty_like(v)
+    ws, n = _workspace(p, BLA_WS_DECAY_BACKWARD, q.device, workspace)
+    _check(load().bla_decay_backward(ctypes.byref(p), int(pos0), _ptr(q), _ptr(k), _ptr(v), _ptr(o), _ptr(dout),
+                                     _ptr(lse), _ptr(dq), _ptr(dkk), _ptr(dvv), _ptr(ws), n, _stream(stream)))
+    return dq, dkk, dvv
 
 
 def bla_device_error(stream=None):

@@ -115,11 +115,29 @@ bla_status check_params(const bla_params *p, OpDims *d) {
     if (p->L < 0) return fail(BLA_ERR_INVALID, "L must be >= 0 (got %d)", p->L);
     if (p->d_k < 1 || p->d_v < 1) return fail(BLA_ERR_INVALID, "d_k and d_v must be >= 1");
     if (p->M < 1) return fail(BLA_ERR_INVALID, "M must be >= 1 (got %d)", p->M);
-    if (!(p->window > 0.0) || !isfinite(p->window)) return fail(BLA_ERR_INVALID, "window (period T) must be > 0");
+    if (!p->periods && (!(p->window > 0.0) || !isfinite(p->window)))
+        return fail(BLA_ERR_INVALID, "window (period T) must be > 0");
     if (!isfinite(p->omega) || !isfinite(p->scale)) return fail(BLA_ERR_INVALID, "omega and scale must be finite");
     if (p->dtype != BLA_F32 && p->dtype != BLA_BF16) return fail(BLA_ERR_INVALID, "dtype must be BLA_F32 or BLA_BF16");
-    const double Te = fmax(p->window, 2.0 * p->M - 1.0);
-    if (p->S < 1 || (double)p->S > Te) return fail(BLA_ERR_INVALID, "S must be in [1, T] (S=%d, T=%g)", p->S, Te);
+    double Te = fmax(p->window, 2.0 * p->M - 1.0);
+    if (p->periods) {
+        // one period per head (Alg. 1 and Alg. 3: T in R^H); S must fit under every one of them
+        if (p->H > kMaxHeadPeriods)
+            return fail(BLA_ERR_UNSUPPORTED, "per-head periods support at most %d heads (H=%d)", kMaxHeadPeriods, p->H);
+        double tmin = INFINITY, tmax = 0.0;
+        for (int h = 0; h < p->H; ++h) {
+            const double T = p->periods[h];
+            if (!(T > 0.0) || !isfinite(T)) return fail(BLA_ERR_INVALID, "periods[%d] must be > 0 and finite", h);
+            const double Th = fmax(T, 2.0 * p->M - 1.0);
+            tmin = fmin(tmin, Th);
+            tmax = fmax(tmax, Th);
+        }
+        if (p->S < 1 || (double)p->S > tmin)
+            return fail(BLA_ERR_INVALID, "S must be in [1, min_h T_h] (S=%d, min T_h=%g)", p->S, tmin);
+        Te = tmax;
+    } else if (p->S < 1 || (double)p->S > Te) {
+        return fail(BLA_ERR_INVALID, "S must be in [1, T] (S=%d, T=%g)", p->S, Te);
+    }
     if (p->chunk < 0) return fail(BLA_ERR_INVALID, "chunk must be >= 0");
     if (p->phase_mode != BLA_PHASE_LAG && p->phase_mode != BLA_PHASE_ABSOLUTE)
         return fail(BLA_ERR_INVALID, "phase_mode must be BLA_PHASE_LAG or BLA_PHASE_ABSOLUTE (got %d)", p->phase_mode);
@@ -131,6 +149,14 @@ bla_status check_params(const bla_params *p, OpDims *d) {
     d->scale = (float)(p->scale > 0.0 ? p->scale : 1.0 / sqrt((double)p->d_k));
     d->dtype = p->dtype;
     d->absolute = p->phase_mode == BLA_PHASE_ABSOLUTE;
+    d->periods = p->periods;
+    d->omega_in = p->omega;
+    return BLA_OK;
+}
+
+// Entry points whose kernels read one shared set of tables refuse per-head periods.
+bla_status no_per_head(const OpDims &d, const char *what) {
+    if (d.periods) return fail(BLA_ERR_UNSUPPORTED, "%s does not support per-head periods yet", what);
     return BLA_OK;
 }
 
@@ -169,7 +195,7 @@ bla_status check_decay(const bla_params *p, OpDims *d, bool forward) {
     if (d->dk != d->dv || (d->dk != 32 && d->dk != 64 && d->dk != 128))
         return fail(BLA_ERR_UNSUPPORTED, "the decay path needs d_k = d_v in {32, 64, 128} (got %d, %d)", d->dk, d->dv);
     if (d->S > 256) return fail(BLA_ERR_UNSUPPORTED, "the decay path needs S <= 256 (got %d)", d->S);
-    if (forward && decay_table_entries(*d) > (size_t(1) << 30))
+    if (forward && decay_table_entries(*d) * (d->periods ? (size_t)d->H : 1) > (size_t(1) << 30))
         return fail(BLA_ERR_UNSUPPORTED, "L + T too large for the decay table (L=%d, T=%g)", d->L, d->T);
     // one-dimensional grids: heads x slot blocks (K scan), heads x column blocks (V scan), tokens / 256 (lse)
     const long long bh = (long long)d->B * d->H, imax = (1ll << 31) - 1;
@@ -314,6 +340,7 @@ size_t bla_workspace_bytes(const bla_params *p, int which) {
     case BLA_WS_BACKWARD: return bwd_workspace_bytes(d);
     case BLA_WS_DECAY_FORWARD: return check_decay(p, &d, true) == BLA_OK ? decay_workspace_bytes(d, false) : 0;
     case BLA_WS_DECAY_DECODE: return check_decay(p, &d, false) == BLA_OK ? decay_workspace_bytes(d, true) : 0;
+    case BLA_WS_DECAY_BACKWARD: return check_decay(p, &d, true) == BLA_OK ? decay_backward_workspace_bytes(d) : 0;
     default: return 0;
     }
 }
@@ -330,6 +357,7 @@ bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k
         !aligned16(state_out))
         return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
     if (d.dtype == BLA_BF16) {
+        if ((s = no_per_head(d, "the bf16 forward")) != BLA_OK) return s;
         const char *why = fwd_bf16_unsupported(d);
         if (why) return fail(BLA_ERR_UNSUPPORTED, "bf16 forward: %s", why);
     }
@@ -344,6 +372,7 @@ bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const vo
     OpDims d;
     bla_status s = check_params(p, &d);
     if (s != BLA_OK) return s;
+    if ((s = no_per_head(d, "the host-buffer forward")) != BLA_OK) return s;
     if (d.L > 0 && (!q || !k || !v || !o)) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
     if (d.dtype == BLA_BF16) {
         const char *why = fwd_bf16_unsupported(d);
@@ -422,7 +451,7 @@ bla_status bla_decay_forward(const bla_params *p, long long pos0, const void *q,
     bla_status s = check_decay(p, &d, true);
     if (s != BLA_OK) return s;
     if (pos0 < 0) return fail(BLA_ERR_INVALID, "pos0 must be >= 0 (got %lld)", pos0);
-    if (!q || !k || !v || !o) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
+    if (d.L > 0 && (!q || !k || !v || !o)) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || (lse && !aligned16(lse)) ||
         (state_in && !aligned16(state_in)) || (state_out && !aligned16(state_out)))
         return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
@@ -450,6 +479,27 @@ bla_status bla_decay_decode_step(const bla_params *p, long long pos, const void 
     return BLA_OK;
 }
 
+bla_status bla_decay_backward(const bla_params *p, long long pos0, const void *q, const void *k, const void *v,
+                              const void *o, const void *dout, const float *lse, void *dq, void *dk, void *dv,
+                              void *workspace, size_t ws_bytes, void *stream) {
+    t_last_error[0] = 0;
+    NvtxRange nvtx("bla_decay_backward");
+    OpDims d;
+    bla_status s = check_decay(p, &d, true);
+    if (s != BLA_OK) return s;
+    if (pos0 < 0) return fail(BLA_ERR_INVALID, "pos0 must be >= 0 (got %lld)", pos0);
+    if (d.L > 0 && (!q || !k || !v || !o || !dout || !lse || !dq || !dk || !dv))
+        return fail(BLA_ERR_INVALID, "q, k, v, o, dout, lse, dq, dk and dv must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(dout) || !aligned16(lse) ||
+        !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    if ((s = check_ws(workspace, ws_bytes, decay_backward_workspace_bytes(d))) != BLA_OK) return s;
+    cudaError_t e = launch_decay_backward(d, pos0, q, k, v, o, dout, lse, dq, dk, dv, workspace,
+                                          reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "decay backward launch");
+    return BLA_OK;
+}
+
 bla_status bla_backward(const bla_params *p, const void *q, const void *k, const void *v, const void *o,
                         const void *dout, const float *lse, void *dq, void *dk, void *dv, void *workspace,
                         size_t ws_bytes, void *stream) {
@@ -463,6 +513,7 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(dout) || !aligned16(lse) ||
         !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
         return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    if ((s = no_per_head(d, "the backward")) != BLA_OK) return s;
     const char *why = bwd_unsupported(d);
     if (why) return fail(BLA_ERR_UNSUPPORTED, "backward: %s", why);
     size_t need = bwd_workspace_bytes(d);

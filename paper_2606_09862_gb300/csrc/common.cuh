@@ -24,7 +24,20 @@ struct OpDims {
     float scale;
     int dtype;
     int absolute;                    // 1: absolute-phase slots (Alg. 1), 0: lag form (Alg. 2)
+    const double *periods;           // host array of H per-head periods (raw, before the clamp), or
+                                     // NULL when every head uses T; never read on the device
+    double omega_in;                 // the caller's omega (> 0: the frequency of every head)
 };
+
+// Per-head periods handed to the table builders by value (Alg. 1 and Alg. 3: T in R^H).
+constexpr int kMaxHeadPeriods = 256;
+struct HeadPeriods {
+    int n;
+    double T[kMaxHeadPeriods];   // clamped periods
+    double w[kMaxHeadPeriods];   // mode frequencies
+};
+// Fill `hp` from d.periods (clamp to 2M-1; omega > 0 overrides every head's 2 pi / T_h).
+void head_periods(const OpDims &d, double omega, HeadPeriods *hp);
 
 // Table block (built on the device per call; lives in the caller's workspace).
 //   phi   [S][R2] fp32: phi[j][2m] = c_m cos(m w D_j), phi[j][2m+1] = sigma c_m sin(m w D_j)
@@ -34,13 +47,27 @@ struct OpDims {
 //   delta [S] int: dilated lags round(j T / S).
 //   rot1  [M][2] fp32: cos(m w), sin(m w) (Eq. recurrence, one step).
 //   erel  [C+1][M][2] fp32: cos(m w tau), sin(m w tau), tau = 0..C (chunk phases).
+//   With per-head periods each table is repeated per head; hs_* are the per-head element strides
+//   (0 when the heads share one period) and wh[H] holds each head's mode frequency (NULL when shared:
+//   kernels then use OpDims::w).
 struct Tables {
     float *phi;
     int *delta;
     float *rot1;
     float *erel;
     int C;
+    int hs_phi, hs_delta, hs_rot1, hs_erel;
+    double *wh;
 };
+
+// Point `t` at head h's tables; returns head h's mode frequency.
+__device__ __forceinline__ double tables_for_head(Tables &t, int h, double w_shared) {
+    t.phi += (size_t)h * t.hs_phi;
+    t.delta += (size_t)h * t.hs_delta;
+    t.rot1 += (size_t)h * t.hs_rot1;
+    t.erel += (size_t)h * t.hs_erel;
+    return t.wh ? t.wh[h] : w_shared;
+}
 
 // Bytes taken by the table block for a given chunk length (each part 256-aligned).
 size_t tables_bytes(const OpDims &d, int C);

@@ -52,17 +52,26 @@ __device__ double dirichlet_closed(int M, double w, double x) {
 __device__ __forceinline__ int grid_delta(int j, double T, int S) { return (int)rint((double)j * T / (double)S); }
 
 // per_slot == 0: Dx[i] = D_M(x0 + i), i < n.   per_slot != 0: Dx[j] = D_M(x0 - Delta_j), j < S.
-// Both: delta[j] = round(j T / S) (round half to even, the default rounding mode).
-__global__ void k_decay_table(int M, double w, double T, int S, long long x0, int n, int per_slot, float *Dx,
-                              int *delta) {
-    const int total = (per_slot ? S : n) + S;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+// Both: delta[j] = round(j T / S) (round half to even, the default rounding mode).  With per-head
+// periods (hp.n > 0) head h writes its own Dx[h][...] and delta[h][S] at (T_h, w_h); otherwise the
+// single (T, w) is used.
+__global__ void k_decay_table(int M, HeadPeriods hp, double T, double w, int S, long long x0, int n, int per_slot,
+                              float *Dx, int *delta) {
+    const int nh = hp.n > 0 ? hp.n : 1;
+    const int per = (per_slot ? S : n) + S;
+    const long long total = (long long)per * nh;
+    for (long long ii = blockIdx.x * (long long)blockDim.x + threadIdx.x; ii < total;
+         ii += (long long)gridDim.x * blockDim.x) {
+        const int h = (int)(ii / per), i = (int)(ii % per);
+        const double Th = hp.n > 0 ? hp.T[h] : T, wh = hp.n > 0 ? hp.w[h] : w;
+        float *Dh = Dx + (size_t)h * (per_slot ? S : n);
+        int *dh = delta + (size_t)h * S;
         if (per_slot) {
-            if (i < S) Dx[i] = (float)dirichlet_closed(M, w, (double)(x0 - grid_delta(i, T, S)));
-            else delta[i - S] = grid_delta(i - S, T, S);
+            if (i < S) Dh[i] = (float)dirichlet_closed(M, wh, (double)(x0 - grid_delta(i, Th, S)));
+            else dh[i - S] = grid_delta(i - S, Th, S);
         } else {
-            if (i < n) Dx[i] = (float)dirichlet_closed(M, w, (double)(x0 + i));
-            else delta[i - n] = grid_delta(i - n, T, S);
+            if (i < n) Dh[i] = (float)dirichlet_closed(M, wh, (double)(x0 + i));
+            else dh[i - n] = grid_delta(i - n, Th, S);
         }
     }
 }
@@ -105,11 +114,15 @@ template <typename T, int CPL>
 __global__ void __launch_bounds__(256) k_decay_kscan(const T *__restrict__ q, const T *__restrict__ k,
                                                      const float *__restrict__ Dx, const int *__restrict__ delta,
                                                      int S, int L, int d, int dmax, int nsb, float scale,
+                                                     int H, int hs_dx, int hs_delta,
                                                      const float *state_in, float *state_out, float *__restrict__ sc) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long bh = blockIdx.x / nsb;
     const int j = (blockIdx.x % nsb) * 8 + warp;
     if (j >= S) return;                       // whole warps only; no block-level synchronisation below
+    const int hd = (int)(bh % H);             // this head's D_M table and grid (strides 0 when shared)
+    Dx += (size_t)hd * hs_dx;
+    delta += (size_t)hd * hs_delta;
     const int off = dmax - delta[j];          // Dx index of token t is t + off
     const size_t row0 = (size_t)bh * L * d + lane * CPL;
     const size_t st = (size_t)bh * S * 2 * d + (size_t)j * d + lane * CPL;   // K half, slot j
@@ -167,11 +180,12 @@ __global__ void __launch_bounds__(256) k_decay_kscan(const T *__restrict__ q, co
 
 // lse[head][t] = log sum_{j : pos0 + t >= Delta_j} exp(sc[head][j][t]).
 __global__ void k_decay_lse(const float *__restrict__ sc, const int *__restrict__ delta, int S, int L, long long pos0,
-                            long long n, float *__restrict__ lse) {
+                            long long n, int H, int hs_delta, float *__restrict__ lse) {
     const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
     if (i >= n) return;
     const long long bh = i / L;
     const int t = (int)(i % L);
+    delta += (size_t)(bh % H) * hs_delta;
     const float *col = sc + (size_t)bh * S * L + t;
     float m = -INFINITY, sum = 0.f;
     for (int j = 0; j < S; ++j) {
@@ -192,8 +206,8 @@ __global__ void k_decay_lse(const float *__restrict__ sc, const int *__restrict_
 template <typename T>
 __global__ void __launch_bounds__(1024) k_decay_vscan(const T *__restrict__ v, const float *__restrict__ Dx, const int *__restrict__ delta,
                               const float *__restrict__ sc, const float *__restrict__ lse, int S, int L, int dk, int dv,
-                              int dmax, int ncb, int ng, long long pos0, const float *state_in, float *state_out,
-                              T *__restrict__ o) {
+                              int dmax, int ncb, int ng, long long pos0, int H, int hs_dx, int hs_delta,
+                              const float *state_in, float *state_out, T *__restrict__ o) {
     constexpr int G = kSlotsPerWarpGroup, TT = kVTile;
     extern __shared__ float4 smem4[];
     const int spad = ng * G, sp = spad + 4;            // row stride: a multiple of 4 floats
@@ -205,6 +219,8 @@ __global__ void __launch_bounds__(1024) k_decay_vscan(const T *__restrict__ v, c
     const int g = threadIdx.x >> 5, lane = threadIdx.x & 31, nthr = blockDim.x;
     const long long bh = blockIdx.x / ncb;
     const int c = (blockIdx.x % ncb) * 32 + lane;
+    Dx += (size_t)(bh % H) * hs_dx;           // this head's D_M table and grid (strides 0 when shared)
+    delta += (size_t)(bh % H) * hs_delta;
     for (int i = threadIdx.x; i < spad; i += nthr) dl[i] = i < S ? delta[i] : 0;
     const size_t vst = (size_t)bh * S * (dk + dv) + (size_t)S * dk + c;   // V half, column c
     float V[G];
@@ -273,12 +289,15 @@ template <typename T, int CPL>
 __global__ void __launch_bounds__(256) k_decay_decode(const T *__restrict__ q, const T *__restrict__ k,
                                                       const T *__restrict__ v, const float *__restrict__ Dj,
                                                       const int *__restrict__ delta, int S, int d, long long pos,
-                                                      float scale, float *__restrict__ state, T *__restrict__ o) {
+                                                      float scale, int H, int hs, float *__restrict__ state,
+                                                      T *__restrict__ o) {
     __shared__ float s_sc[256];
     __shared__ float s_red[kDecodeWarps][128];
     __shared__ float s_stat[2];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long bh = blockIdx.x;
+    Dj += (size_t)(bh % H) * hs;              // this head's weights D_j(pos) and grid (stride 0 when shared)
+    delta += (size_t)(bh % H) * hs;
     float *Ks = state + (size_t)bh * 2 * S * d + lane * CPL;
     float *Vs = Ks + (size_t)S * d;
     float qv[CPL], kv[CPL], vv[CPL];
@@ -361,33 +380,171 @@ __global__ void __launch_bounds__(256) k_decay_decode(const T *__restrict__ q, c
     }
 }
 
+// ------------------------------------------------------------------ backward (VJP)
+// Unrolled, the decayed slot state is a fixed linear map of the tokens,
+//     K~_j(t) = sum_{u<=t} W_j(t,u) k_u,     W_j(t,u) = D_j(u) prod_{u<x<=t} (1 - D_j(x)),
+// so the chain rule through s = scale q . K~, the masked softmax and o = sum_j p V~ gives, with
+// upstream do:
+//     dp[t,j] = do_t . V~_j(t),     g[t,j] = scale p[t,j] (dp[t,j] - do_t . o_t)
+//     dq_t = sum_j g[t,j] K~_j(t)                                                  forward in time
+//     lK_j(t) = g[t,j] q_t + (1 - D_j(t+1)) lK_j(t+1),    dk_t = sum_j D_j(t) lK_j(t)    backward
+//     lV_j(t) = p[t,j] do_t + (1 - D_j(t+1)) lV_j(t+1),   dv_t = sum_j D_j(t) lV_j(t)    backward
+// dp comes from the K scan with (do, v) in place of (q, k); the three sums over slots run in
+// k_decay_rscan, the V scan's layout with the per-token factors (f, u, w) of
+//     X_j <- f X_j + u x_t,     out_t = sum_j w X_j
+// staged per tile: forward in time f = 1 - D_j(t), u = D_j(t), w = g; backward in time
+// f = 1 - D_j(t+1), u = g or p, w = D_j(t).
+
+// g[head][j][t] = scale p (dp - do_t . o_t), in place of dp; one thread per token.
+template <typename T>
+__global__ void k_decay_ds(const float *__restrict__ sc, const float *__restrict__ lse, float *__restrict__ g,
+                           const T *__restrict__ dout, const T *__restrict__ o, const int *__restrict__ delta, int S,
+                           int L, int dv, long long pos0, float scale, long long n, int H, int hs_delta) {
+    const long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+    if (i >= n) return;
+    const long long bh = i / L;
+    const int t = (int)(i % L);
+    delta += (size_t)(bh % H) * hs_delta;
+    float rd = 0.f;
+    for (int c = 0; c < dv; ++c) rd = fmaf(load_elem<T>(dout, (size_t)i * dv + c), load_elem<T>(o, (size_t)i * dv + c), rd);
+    const size_t col = (size_t)bh * S * L + t;
+    const float l = lse[i];
+    for (int j = 0; j < S; ++j) {
+        const size_t e = col + (size_t)j * L;
+        g[e] = (pos0 + t >= delta[j]) ? scale * expf(sc[e] - l) * (g[e] - rd) : 0.f;
+    }
+}
+
+// Reduce scan over the slots for 32 columns of one head (layout of k_decay_vscan).  REV = false:
+// forward in time, f = 1 - D_j(t), u = D_j(t), w = wt(t, j).  REV = true: backward in time,
+// f = 1 - D_j(t+1), u = wt(t, j), w = D_j(t).  wt(t, j) = G[j][t] when lse is NULL, else the slot
+// probability exp(G[j][t] - lse[t]) (G holding scores; 0 on masked slots).
+template <typename T, bool REV>
+__global__ void __launch_bounds__(1024) k_decay_rscan(const T *__restrict__ x, const float *__restrict__ Dx,
+                                                      const int *__restrict__ delta, const float *__restrict__ G,
+                                                      const float *__restrict__ lse, int S, int L, int dx, int dmax,
+                                                      int ncb, int ng, long long pos0, int H, int hs_dx, int hs_delta,
+                                                      T *__restrict__ out) {
+    constexpr int G8 = kSlotsPerWarpGroup, TT = kVTile;
+    extern __shared__ float4 smem4[];
+    const int spad = ng * G8, sp = spad + 4;
+    float *Ft = reinterpret_cast<float *>(smem4);      // [TT][sp]
+    float *Ut = Ft + TT * sp;                          // [TT][sp]
+    float *Wt = Ut + TT * sp;                          // [TT][sp]
+    float *red = Wt + TT * sp;                         // [TT][ng][32]
+    float *Xt = red + TT * ng * 32;                    // [TT][32]
+    int *dl = reinterpret_cast<int *>(Xt + TT * 32);   // [spad]
+    const int g = threadIdx.x >> 5, lane = threadIdx.x & 31, nthr = blockDim.x;
+    const long long bh = blockIdx.x / ncb;
+    const int c = (blockIdx.x % ncb) * 32 + lane;
+    Dx += (size_t)(bh % H) * hs_dx;           // this head's D_M table and grid (strides 0 when shared)
+    delta += (size_t)(bh % H) * hs_delta;
+    for (int i = threadIdx.x; i < spad; i += nthr) dl[i] = i < S ? delta[i] : 0;
+    float X[G8];
+#pragma unroll
+    for (int jj = 0; jj < G8; ++jj) X[jj] = 0.f;
+    __syncthreads();
+    const T *xb = x + (size_t)bh * L * dx + (c - lane);
+    T *oh = out + (size_t)bh * L * dx + c;
+    const float *gh = G + (size_t)bh * S * L;
+    const float *lh = lse ? lse + (size_t)bh * L : nullptr;
+    for (int t0 = 0; t0 < L; t0 += TT) {
+        // tile position tt holds token t = t0 + tt (forward) or L - 1 - (t0 + tt) (backward)
+        for (int idx = threadIdx.x; idx < TT * spad; idx += nthr) {
+            const int tt = idx % TT, j = idx / TT, r = t0 + tt;
+            float f = 0.f, u = 0.f, w = 0.f;
+            if (j < S && r < L) {
+                const int t = REV ? L - 1 - r : r;
+                float wt;
+                if (lh) wt = (pos0 + t >= dl[j]) ? expf(gh[(size_t)j * L + t] - lh[t]) : 0.f;
+                else wt = gh[(size_t)j * L + t];
+                const float Dt = Dx[t + dmax - dl[j]];
+                if (REV) {
+                    f = 1.f - Dx[t + 1 + dmax - dl[j]];   // entry L + dmax - Delta_j < L + dmax + 1 at t = L - 1
+                    u = wt;
+                    w = Dt;
+                } else {
+                    f = 1.f - Dt;
+                    u = Dt;
+                    w = wt;
+                }
+            }
+            Ft[tt * sp + j] = f;
+            Ut[tt * sp + j] = u;
+            Wt[tt * sp + j] = w;
+        }
+        for (int idx = threadIdx.x; idx < TT * 32; idx += nthr) {
+            const int r = t0 + (idx >> 5);
+            const int t = REV ? L - 1 - r : r;
+            Xt[idx] = r < L ? load_elem<T>(xb, (size_t)t * dx + (idx & 31)) : 0.f;
+        }
+        __syncthreads();
+        const int nt = min(TT, L - t0);
+#pragma unroll 4
+        for (int tt = 0; tt < nt; ++tt) {
+            const float xv = Xt[tt * 32 + lane];
+            const float4 *f4 = reinterpret_cast<const float4 *>(Ft + tt * sp + g * G8);
+            const float4 *u4 = reinterpret_cast<const float4 *>(Ut + tt * sp + g * G8);
+            const float4 *w4 = reinterpret_cast<const float4 *>(Wt + tt * sp + g * G8);
+            const float4 fa = f4[0], fb = f4[1], ua = u4[0], ub = u4[1], wa = w4[0], wb = w4[1];
+            const float ff[G8] = {fa.x, fa.y, fa.z, fa.w, fb.x, fb.y, fb.z, fb.w};
+            const float uu[G8] = {ua.x, ua.y, ua.z, ua.w, ub.x, ub.y, ub.z, ub.w};
+            const float ww[G8] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w};
+            float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll
+            for (int jj = 0; jj < G8; jj += 2) {
+                X[jj] = fmaf(ff[jj], X[jj], uu[jj] * xv);
+                X[jj + 1] = fmaf(ff[jj + 1], X[jj + 1], uu[jj + 1] * xv);
+                acc0 = fmaf(ww[jj], X[jj], acc0);
+                acc1 = fmaf(ww[jj + 1], X[jj + 1], acc1);
+            }
+            red[(tt * ng + g) * 32 + lane] = acc0 + acc1;
+        }
+        __syncthreads();
+        for (int tt = g; tt < nt; tt += ng) {
+            float sum = 0.f;
+            for (int gg = 0; gg < ng; ++gg) sum += red[(tt * ng + gg) * 32 + lane];
+            const int r = t0 + tt;
+            store_elem<T>(oh, (size_t)(REV ? L - 1 - r : r) * dx, sum);
+        }
+    }
+}
+
 // Largest Delta_j (the grid is non-decreasing in j), computed exactly as the device does.
 int host_dmax(const OpDims &d) { return (int)rint((double)(d.S - 1) * d.T / (double)d.S); }
 
 struct DecayWs {
-    int *delta;
-    float *Dx;
+    int *delta;      // [nh][S]
+    float *Dx;       // [nh][S] (decode) or [nh][L + max Delta + 1] (forward)
     float *sc;
     float *lse;
+    int hs_dx, hs_delta;   // per-head strides of Dx and delta (0 when the heads share one period)
+    float *g = nullptr;    // backward: dp, then g = scale ds, [BH][S][L]
 };
 
 size_t decay_table_len(const OpDims &d) { return (size_t)d.L + (size_t)host_dmax(d) + 1; }
 
-size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w) {
+size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w, bool backward = false) {
     size_t off = 0;
     auto take = [&](size_t bytes) {
         char *p = base ? base + off : nullptr;
         off += align_up(bytes, 256);
         return p;
     };
-    w->delta = reinterpret_cast<int *>(take(sizeof(int) * d.S));
-    w->Dx = reinterpret_cast<float *>(take(sizeof(float) * (decode ? (size_t)d.S : decay_table_len(d))));
+    const size_t nh = d.periods ? (size_t)d.H : 1;
+    const size_t per = decode ? (size_t)d.S : decay_table_len(d);
+    w->delta = reinterpret_cast<int *>(take(sizeof(int) * nh * d.S));
+    w->Dx = reinterpret_cast<float *>(take(sizeof(float) * nh * per));
+    w->hs_dx = d.periods ? (int)per : 0;
+    w->hs_delta = d.periods ? d.S : 0;
     w->sc = nullptr;
     w->lse = nullptr;
     if (!decode) {
         const size_t BH = (size_t)d.B * d.H;
         w->sc = reinterpret_cast<float *>(take(sizeof(float) * BH * d.S * (size_t)(d.L > 0 ? d.L : 1)));
         if (own_lse) w->lse = reinterpret_cast<float *>(take(sizeof(float) * BH * (size_t)(d.L > 0 ? d.L : 1)));
+        w->g = backward ? reinterpret_cast<float *>(take(sizeof(float) * BH * d.S * (size_t)(d.L > 0 ? d.L : 1)))
+                        : nullptr;
     }
     return off;
 }
@@ -401,11 +558,14 @@ cudaError_t kscan_dispatch(const OpDims &d, const DecayWs &w, const void *q, con
     ProfScope ps(BLA_K_DECAY, st);
     switch (d.dk) {
     case 32: k_decay_kscan<T, 1><<<(unsigned)blocks, 256, 0, st>>>(qq, kk, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
-                                                                    d.scale, state_in, state_out, w.sc); break;
+                                                                    d.scale, d.H, w.hs_dx, w.hs_delta, state_in,
+                                                                    state_out, w.sc); break;
     case 64: k_decay_kscan<T, 2><<<(unsigned)blocks, 256, 0, st>>>(qq, kk, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
-                                                                    d.scale, state_in, state_out, w.sc); break;
+                                                                    d.scale, d.H, w.hs_dx, w.hs_delta, state_in,
+                                                                    state_out, w.sc); break;
     default: k_decay_kscan<T, 4><<<(unsigned)blocks, 256, 0, st>>>(qq, kk, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
-                                                                    d.scale, state_in, state_out, w.sc); break;
+                                                                    d.scale, d.H, w.hs_dx, w.hs_delta, state_in,
+                                                                    state_out, w.sc); break;
     }
     return cudaGetLastError();
 }
@@ -427,21 +587,105 @@ cudaError_t vscan_dispatch(const OpDims &d, const DecayWs &w, const float *lse, 
     const long long blocks = (long long)d.B * d.H * ncb;
     ProfScope ps(BLA_K_DECAY, st);
     k_decay_vscan<T><<<(unsigned)blocks, 32 * ng, smem, st>>>(static_cast<const T *>(v), w.Dx, w.delta, w.sc, lse,
-                                                              d.S, d.L, d.dk, d.dv, dmax, ncb, ng, pos0, state_in,
-                                                              state_out, static_cast<T *>(o));
+                                                              d.S, d.L, d.dk, d.dv, dmax, ncb, ng, pos0, d.H, w.hs_dx,
+                                                              w.hs_delta, state_in, state_out, static_cast<T *>(o));
     return cudaGetLastError();
 }
 
 cudaError_t table_launch(const OpDims &d, long long x0, int n, int per_slot, const DecayWs &w, cudaStream_t st) {
-    const int total = (per_slot ? d.S : n) + d.S;
-    int blocks = (total + 255) / 256;
+    HeadPeriods hp;
+    head_periods(d, d.omega_in, &hp);   // hp.n = 0 when the heads share one period
+    const long long total = (long long)((per_slot ? d.S : n) + d.S) * (hp.n > 0 ? hp.n : 1);
+    long long blocks = (total + 255) / 256;
     if (blocks > 1024) blocks = 1024;
     ProfScope ps(BLA_K_DECAY, st);
-    k_decay_table<<<blocks, 256, 0, st>>>(d.M, d.w, d.T, d.S, x0, n, per_slot, w.Dx, w.delta);
+    k_decay_table<<<(int)blocks, 256, 0, st>>>(d.M, hp, d.T, d.w, d.S, x0, n, per_slot, w.Dx, w.delta);
     return cudaGetLastError();
 }
 
+// K scan with explicit operands: out[head][j][t] = scale z_t . X_j(t), X_j <- (1 - D) X_j + D x_t.
+template <typename T>
+cudaError_t kscan_launch(const OpDims &d, const DecayWs &w, const void *z, const void *x, int dmax, float scale,
+                         float *out, cudaStream_t st) {
+    const int nsb = (d.S + 7) / 8;
+    const long long blocks = (long long)d.B * d.H * nsb;
+    const T *zz = static_cast<const T *>(z), *xx = static_cast<const T *>(x);
+    ProfScope ps(BLA_K_DECAY, st);
+    switch (d.dk) {
+    case 32: k_decay_kscan<T, 1><<<(unsigned)blocks, 256, 0, st>>>(zz, xx, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
+                                                                    scale, d.H, w.hs_dx, w.hs_delta, nullptr, nullptr,
+                                                                    out); break;
+    case 64: k_decay_kscan<T, 2><<<(unsigned)blocks, 256, 0, st>>>(zz, xx, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
+                                                                    scale, d.H, w.hs_dx, w.hs_delta, nullptr, nullptr,
+                                                                    out); break;
+    default: k_decay_kscan<T, 4><<<(unsigned)blocks, 256, 0, st>>>(zz, xx, w.Dx, w.delta, d.S, d.L, d.dk, dmax, nsb,
+                                                                    scale, d.H, w.hs_dx, w.hs_delta, nullptr, nullptr,
+                                                                    out); break;
+    }
+    return cudaGetLastError();
+}
+
+size_t rscan_smem(int ng) {
+    const int spad = ng * kSlotsPerWarpGroup, sp = spad + 4;
+    return sizeof(float) * ((size_t)3 * kVTile * sp + (size_t)kVTile * ng * 32 + (size_t)kVTile * 32) +
+           sizeof(int) * (size_t)spad;
+}
+
+template <typename T, bool REV>
+cudaError_t rscan_launch(const OpDims &d, const DecayWs &w, const void *x, const float *G, const float *lse, int dmax,
+                         long long pos0, void *out, cudaStream_t st) {
+    const int ncb = d.dv / 32;
+    const int ng = (d.S + kSlotsPerWarpGroup - 1) / kSlotsPerWarpGroup;
+    const size_t smem = rscan_smem(ng);
+    cudaError_t e = cudaFuncSetAttribute(k_decay_rscan<T, REV>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const long long blocks = (long long)d.B * d.H * ncb;
+    ProfScope ps(BLA_K_DECAY, st);
+    k_decay_rscan<T, REV><<<(unsigned)blocks, 32 * ng, smem, st>>>(static_cast<const T *>(x), w.Dx, w.delta, G, lse,
+                                                                   d.S, d.L, d.dv, dmax, ncb, ng, pos0, d.H, w.hs_dx,
+                                                                   w.hs_delta, static_cast<T *>(out));
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t backward_run(const OpDims &d, const DecayWs &w, long long pos0, const void *q, const void *k,
+                         const void *v, const void *o, const void *dout, const float *lse, void *dq, void *dk,
+                         void *dv, int dmax, cudaStream_t st) {
+    cudaError_t e;
+    if ((e = kscan_launch<T>(d, w, q, k, dmax, d.scale, w.sc, st)) != cudaSuccess) return e;    // scores
+    if ((e = kscan_launch<T>(d, w, dout, v, dmax, 1.f, w.g, st)) != cudaSuccess) return e;     // dp
+    const long long nt = (long long)d.B * d.H * d.L;
+    {
+        ProfScope ps(BLA_K_DECAY, st);
+        k_decay_ds<T><<<(unsigned)((nt + 255) / 256), 256, 0, st>>>(w.sc, lse, w.g, static_cast<const T *>(dout),
+                                                                    static_cast<const T *>(o), w.delta, d.S, d.L,
+                                                                    d.dv, pos0, d.scale, nt, d.H, w.hs_delta);
+        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+    }
+    if ((e = rscan_launch<T, false>(d, w, k, w.g, nullptr, dmax, pos0, dq, st)) != cudaSuccess) return e;
+    if ((e = rscan_launch<T, true>(d, w, q, w.g, nullptr, dmax, pos0, dk, st)) != cudaSuccess) return e;
+    return rscan_launch<T, true>(d, w, dout, w.sc, lse, dmax, pos0, dv, st);
+}
+
 }  // namespace
+
+size_t decay_backward_workspace_bytes(const OpDims &d) {
+    DecayWs w;
+    return carve(d, false, false, nullptr, &w, true);
+}
+
+cudaError_t launch_decay_backward(const OpDims &d, long long pos0, const void *q, const void *k, const void *v,
+                                  const void *o, const void *dout, const float *lse, void *dq, void *dk, void *dv,
+                                  void *ws, cudaStream_t st) {
+    if (d.L == 0) return cudaSuccess;
+    DecayWs w;
+    carve(d, false, false, static_cast<char *>(ws), &w, true);
+    const int dmax = host_dmax(d);
+    cudaError_t e = table_launch(d, pos0 - dmax, (int)decay_table_len(d), 0, w, st);
+    if (e != cudaSuccess) return e;
+    return d.dtype == BLA_BF16 ? backward_run<__nv_bfloat16>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st)
+                               : backward_run<float>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st);
+}
 
 size_t decay_table_entries(const OpDims &d) { return decay_table_len(d); }
 
@@ -465,7 +709,7 @@ cudaError_t launch_decay_forward(const OpDims &d, long long pos0, const void *q,
     const long long nt = (long long)d.B * d.H * d.L;
     if (nt > 0) {
         ProfScope ps(BLA_K_DECAY, st);
-        k_decay_lse<<<(unsigned)((nt + 255) / 256), 256, 0, st>>>(w.sc, w.delta, d.S, d.L, pos0, nt, l);
+        k_decay_lse<<<(unsigned)((nt + 255) / 256), 256, 0, st>>>(w.sc, w.delta, d.S, d.L, pos0, nt, d.H, w.hs_delta, l);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     return d.dtype == BLA_BF16 ? vscan_dispatch<__nv_bfloat16>(d, w, l, v, o, dmax, pos0, state_in, state_out, st)
@@ -485,18 +729,18 @@ cudaError_t launch_decay_decode(const OpDims &d, long long pos, const void *q, c
         const T *qq = static_cast<const T *>(q), *kk = static_cast<const T *>(k), *vv = static_cast<const T *>(v);
         T *oo = static_cast<T *>(o);
         switch (d.dk) {
-        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
+        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
         }
     } else {
         using T = float;
         const T *qq = static_cast<const T *>(q), *kk = static_cast<const T *>(k), *vv = static_cast<const T *>(v);
         T *oo = static_cast<T *>(o);
         switch (d.dk) {
-        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
-        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, state, oo); break;
+        case 32: k_decay_decode<T, 1><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        case 64: k_decay_decode<T, 2><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
+        default: k_decay_decode<T, 4><<<blocks, 256, 0, st>>>(qq, kk, vv, w.Dx, w.delta, d.S, d.dk, pos, d.scale, d.H, w.hs_delta, state, oo); break;
         }
     }
     return cudaGetLastError();

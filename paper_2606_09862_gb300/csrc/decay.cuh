@@ -14,5 +14,10 @@ cudaError_t launch_decay_forward(const OpDims &d, long long pos0, const void *q,
                                  float *lse, const float *state_in, float *state_out, void *ws, cudaStream_t st);
 cudaError_t launch_decay_decode(const OpDims &d, long long pos, const void *q, const void *k, const void *v,
                                 float *state, void *o, void *ws, cudaStream_t st);
+// Vector-Jacobian product of the decayed forward from the zero state (dq, dk, dv in the input dtype).
+size_t decay_backward_workspace_bytes(const OpDims &d);
+cudaError_t launch_decay_backward(const OpDims &d, long long pos0, const void *q, const void *k, const void *v,
+                                  const void *o, const void *dout, const float *lse, void *dq, void *dk, void *dv,
+                                  void *ws, cudaStream_t st);
 
 }  // namespace bla

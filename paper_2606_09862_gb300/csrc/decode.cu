@@ -78,6 +78,7 @@ __global__ void __launch_bounds__(kThreads) k_decode(OpDims d, long long pos, Ta
     const int M = d.M, R2 = d.R2, S = d.S;
     const int bh = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const double w = tables_for_head(tb, bh % d.H, d.w);   // this head's tables and mode frequency
     extern __shared__ float sm[];
     float *y = sm;                 // [R2]: q . Z rows, later u
     float *ps = y + R2;            // [S]: scores, later probabilities
@@ -138,7 +139,7 @@ __global__ void __launch_bounds__(kThreads) k_decode(OpDims d, long long pos, Ta
     // absolute form: y_m <- e^{-i m w pos} y_m
     if (d.absolute) {
         for (int m = threadIdx.x; m < M; m += kThreads) {
-            const float2 f = pos_phase(m, pos, d.w);
+            const float2 f = pos_phase(m, pos, w);
             const float yc = y[2 * m], ys = y[2 * m + 1];
             y[2 * m] = f.x * yc + f.y * ys;
             y[2 * m + 1] = f.x * ys - f.y * yc;
@@ -182,7 +183,7 @@ __global__ void __launch_bounds__(kThreads) k_decode(OpDims d, long long pos, Ta
     // absolute form: the coefficient uc - i us is multiplied by e^{-i m w pos}
     if (d.absolute) {
         for (int m = threadIdx.x; m < M; m += kThreads) {
-            const float2 f = pos_phase(m, pos, d.w);
+            const float2 f = pos_phase(m, pos, w);
             const float uc = y[2 * m], us = y[2 * m + 1];
             y[2 * m] = f.x * uc - f.y * us;
             y[2 * m + 1] = f.y * uc + f.x * us;

@@ -74,6 +74,7 @@ extern "C" bla_status bla_decode_step_noalloc(const bla_params *p, long long pos
     const double Te = fmax(p->window, 2.0 * p->M - 1.0);
     if (p->S < 1 || (double)p->S > Te) return reject(BLA_ERR_INVALID, "S must be in [1, T] (S=%lld)", p->S);
     if (pos < 0) return reject(BLA_ERR_INVALID, "pos must be >= 0 (got %lld)", pos);
+    if (p->periods) return reject(BLA_ERR_UNSUPPORTED, "the no-alloc decode does not support per-head periods yet");
     if (!q || !k || !v || !state || !o) return reject(BLA_ERR_INVALID, "q, k, v, state and o must be non-NULL");
     const uintptr_t mis = reinterpret_cast<uintptr_t>(q) | reinterpret_cast<uintptr_t>(k) |
                           reinterpret_cast<uintptr_t>(v) | reinterpret_cast<uintptr_t>(state) |
@@ -92,6 +93,8 @@ extern "C" bla_status bla_decode_step_noalloc(const bla_params *p, long long pos
     d.scale = (float)(p->scale > 0.0 ? p->scale : 1.0 / sqrt((double)p->d_k));
     d.dtype = p->dtype;
     d.absolute = p->phase_mode == BLA_PHASE_ABSOLUTE;
+    d.periods = nullptr;
+    d.omega_in = p->omega;
     const size_t need = tables_bytes(d, 0);
     if (need > kNoAllocScratchBytes)
         return reject(BLA_ERR_UNSUPPORTED,

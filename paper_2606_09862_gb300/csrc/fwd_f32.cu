@@ -45,6 +45,7 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
     const int QS = dk + 1, VS = dv + 1;   // padded row strides of the q/k and v tiles
     const int bh = blockIdx.x;
     const int tid = threadIdx.x, nt = blockDim.x;
+    const double w = tables_for_head(tb, bh % d.H, d.w);   // this head's tables and mode frequency
     F32Smem sm;
     sm.Q = smem;
     sm.K = sm.Q + C * QS;
@@ -106,7 +107,7 @@ __global__ void __launch_bounds__(256) k_forward_f32(OpDims d, int C, Tables tb,
         if (d.absolute) {
             for (int m = tid; m < M; m += nt) {
                 double sn, cs;
-                sincos((double)m * d.w * (double)t0, &sn, &cs);
+                sincos((double)m * w * (double)t0, &sn, &cs);
                 sm.Ph[2 * m] = (float)cs;
                 sm.Ph[2 * m + 1] = (float)-sn;
             }

@@ -170,5 +170,46 @@ def test_decay_argument_checks(lib):
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_FORWARD) >= 2 * 3 * 8 * 100 * 4
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_DECODE) > 0
     assert lib.bla_workspace_bytes(ctypes.byref(_params()), bla.BLA_WS_DECAY_FORWARD) == 0
+    bwd = lib.bla_decay_backward
+    assert bwd(ctypes.byref(_params()), 0, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30,
+               None) == bla.BLA_ERR_UNSUPPORTED                                       # lag form
+    assert bwd(ctypes.byref(_params(phase_mode=ab)), -1, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE,
+               1 << 30, None) == bla.BLA_ERR_INVALID
+    assert bwd(ctypes.byref(_params(phase_mode=ab)), 0, FAKE, FAKE, FAKE, FAKE, FAKE, None, FAKE, FAKE, FAKE, FAKE,
+               1 << 30, None) == bla.BLA_ERR_INVALID                                  # no lse
+    assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECAY_BACKWARD) >= 2 * 2 * 3 * 8 * 100 * 4
     # grids that would exceed the launch limits are refused before any launch
     assert fwd(_params(phase_mode=ab, B=1 << 20, H=1 << 10, S=64, window=64.0)) == bla.BLA_ERR_UNSUPPORTED
+
+
+def test_per_head_periods_checked_on_host(lib):
+    """Per-head periods (Alg. 1 and Alg. 3: T in R^H): each must be > 0, S must fit under all of
+    them, at most 256 heads, and the paths without per-head tables refuse them before any launch."""
+    from paper_2606_09862_gb300 import bla
+
+    def params(periods, **kw):
+        p = _params(H=len(periods), **kw)
+        p.periods = (ctypes.c_double * len(periods))(*periods)
+        return p
+
+    def fwd(p):
+        return lib.bla_forward_chunked(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, None, None, FAKE, 1 << 30, None)
+
+    assert fwd(params([16.0, -1.0])) == bla.BLA_ERR_INVALID
+    assert fwd(params([16.0, float("nan")])) == bla.BLA_ERR_INVALID
+    assert fwd(params([16.0, 3.0], S=8, M=2)) == bla.BLA_ERR_INVALID          # S above one head's period
+    assert fwd(params([16.0] * 257)) == bla.BLA_ERR_UNSUPPORTED
+    assert fwd(params([16.0, 32.0], dtype=bla.BLA_BF16, d_k=64, d_v=64)) == bla.BLA_ERR_UNSUPPORTED
+    p = params([16.0, 32.0])
+    assert lib.bla_backward(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30,
+                            None) == bla.BLA_ERR_UNSUPPORTED
+    assert lib.bla_decode_step_noalloc(ctypes.byref(p), 0, FAKE, FAKE, FAKE, FAKE, FAKE, None) == \
+        bla.BLA_ERR_UNSUPPORTED
+    assert lib.bla_forward_chunked_host(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30, None) == \
+        bla.BLA_ERR_UNSUPPORTED
+    # the tables repeat per head, so the workspace grows with H
+    shared = lib.bla_workspace_bytes(ctypes.byref(_params(H=2)), bla.BLA_WS_DECODE)
+    assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECODE) > shared
+    assert bla.make_params(1, 2, 8, 32, 32, 4, 4, [9.0, 20.0]).periods[1] == 20.0
+    with pytest.raises(bla.BlaError):
+        bla.make_params(1, 3, 8, 32, 32, 4, 4, [9.0, 20.0])

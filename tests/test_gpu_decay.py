@@ -3,7 +3,7 @@ added) on the GPU, through the C ABI, against the oracle's decayed Alg. 1."""
 import numpy as np
 import pytest
 
-from gpu_util import TOL_BF16, TOL_F32, rel, require_cuda, to_dev
+from gpu_util import TOL_BF16, TOL_F32, TOL_GRAD, rel, require_cuda, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -157,3 +157,44 @@ def test_lag_form_rejected():
     with pytest.raises(bla.BlaError) as e:
         bla.bla_decay_forward(x, x, x, 4, 4, 16.0, phase_mode="lag")
     assert e.value.status == bla.BLA_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("dtype,B,H,L,d,M,S,T,pos0", [
+    ("f32", 1, 2, 70, 32, 8, 12, 40.0, 0),       # ragged 16-token tiles, T > 2M-1
+    ("f32", 1, 1, 50, 64, 4, 7, 7.0, 0),         # T = S = 2M-1 (sliding window)
+    ("f32", 2, 1, 33, 32, 4, 5, 20.0, 9),        # later start position
+    ("bf16", 1, 2, 300, 128, 64, 64, 1024.0, 0), # the LM-layer (M, S, T), shortened
+])
+def test_backward_against_oracle_vjp(orc, dtype, B, H, L, d, M, S, T, pos0):
+    """dq, dk, dv of the decayed forward against the oracle's VJP of Alg. 1 with decay."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_dout, make_qkv
+    dev = require_cuda()
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    q, k, v = make_qkv(B, H, L, d, dtype=dtype, seed=L + S)
+    do = make_dout(B, H, L, d, dtype=dtype, seed=L + S)
+    tq, tk, tv, tdo = (to_dev(x, dev, tdt) for x in (q, k, v, do))
+    o, lse, _ = bla.bla_decay_forward(tq, tk, tv, M, S, T, pos0=pos0)
+    got = bla.bla_decay_backward(tq, tk, tv, o, tdo, lse, M, S, T, pos0=pos0)
+    bla.bla_device_error()
+    ref = orc.backward_decay(q, k, v, do, M, S, T, pos0=pos0)
+    tol = 1e-4 if dtype == "f32" else TOL_GRAD
+    for name, a, b in zip(("dq", "dk", "dv"), got, ref):
+        assert rel(a.float().cpu().numpy(), b) <= tol, (name, rel(a.float().cpu().numpy(), b))
+
+
+def test_empty_sequence_passes_state_through():
+    """L = 0: nothing to attend; the final state is the given one (or zero without one)."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    dev = require_cuda()
+    z = torch.zeros((1, 2, 0, 32), device=dev)
+    st0 = torch.randn((1, 2, 2, 5, 32), device=dev)
+    st = st0.clone()
+    o, _, out = bla.bla_decay_forward(z, z, z, 3, 5, 9.0, pos0=4, state=st, want_state=True)
+    _, _, zero = bla.bla_decay_forward(z, z, z, 3, 5, 9.0, want_state=True)
+    bla.bla_device_error()
+    assert o.shape == (1, 2, 0, 32)
+    assert torch.equal(out, st0)
+    assert float(zero.abs().max()) == 0.0

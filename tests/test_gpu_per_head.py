@@ -1,0 +1,105 @@
+"""Per-head periods (Alg. 1 and Alg. 3 take T in R^H) on the paths with per-head tables: the fp32
+forward, the decode step and the state-decay entry points, against the oracle run at each head's
+own period."""
+import numpy as np
+import pytest
+
+from gpu_util import TOL_BF16, TOL_F32, rel, require_cuda, to_dev
+
+pytestmark = pytest.mark.gpu
+
+TS = [7.0, 16.0, 40.0]   # one head at T = 2M-1 = S (M = 4, S = 7), two blurry ones
+
+
+@pytest.mark.parametrize("phase_mode", ["lag", "absolute"])
+def test_f32_forward(orc, phase_mode):
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    B, H, L, d, M, S = 2, 3, 150, 32, 4, 7
+    q, k, v = make_qkv(B, H, L, d, dtype="f32", seed=5)
+    o, lse, st = bla.bla_forward_chunked(*(to_dev(x, dev, torch.float32) for x in (q, k, v)), M, S, TS, chunk=32,
+                                         want_state=True, phase_mode=phase_mode)
+    bla.bla_device_error()
+    form = "naive" if phase_mode == "lag" else "absolute"
+    ref = orc.forward(q, k, v, M, S, TS, form=form)
+    assert rel(o.cpu().numpy(), ref["o"]) <= TOL_F32
+    assert np.abs(lse.cpu().numpy() - ref["lse"]).max() <= 1e-4
+    st_ref = orc.forward(q, k, v, M, S, TS, form="modes", return_state=True)["state"]
+    assert rel(st.cpu().numpy(), st_ref) <= TOL_F32
+
+
+@pytest.mark.parametrize("dtype,phase_mode", [("f32", "lag"), ("bf16", "lag"), ("bf16", "absolute")])
+def test_decode_from_zero_state(orc, dtype, phase_mode):
+    """Decode steps from the zero state at pos = 0, 1, ... reproduce the forward over the sequence."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    B, H, L, d, M, S = 2, 3, 40, 64, 4, 7
+    q, k, v = make_qkv(B, H, L, d, dtype=dtype, seed=9)
+    st = torch.zeros((B, H, 2, M, 2, d), dtype=torch.float32, device=dev)
+    outs = []
+    for t in range(L):
+        o = bla.bla_decode_step(to_dev(q[:, :, t], dev, tdt), to_dev(k[:, :, t], dev, tdt), to_dev(v[:, :, t], dev, tdt),
+                                st, t, M, S, TS, phase_mode=phase_mode)
+        outs.append(o.float().cpu().numpy())
+    bla.bla_device_error()
+    form = "naive" if phase_mode == "lag" else "absolute"
+    ref = orc.forward(q, k, v, M, S, TS, form=form)
+    assert rel(np.stack(outs, 2), ref["o"]) <= (TOL_F32 if dtype == "f32" else TOL_BF16)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_decay_forward_and_decode(orc, dtype):
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    tdt = torch.float32 if dtype == "f32" else torch.bfloat16
+    tol = TOL_F32 if dtype == "f32" else TOL_BF16
+    B, H, L, L1, d, M, S = 2, 3, 120, 90, 64, 4, 7
+    q, k, v = make_qkv(B, H, L, d, dtype=dtype, seed=13)
+    full = orc.forward_decay(q, k, v, M, S, TS, return_state=True)
+    o1, _, st = bla.bla_decay_forward(*(to_dev(x[:, :, :L1], dev, tdt) for x in (q, k, v)), M, S, TS, want_state=True)
+    outs = [o1.float().cpu().numpy()]
+    for t in range(L1, L):
+        o = bla.bla_decay_decode_step(to_dev(q[:, :, t], dev, tdt), to_dev(k[:, :, t], dev, tdt),
+                                      to_dev(v[:, :, t], dev, tdt), st, t, M, S, TS)
+        outs.append(o.float().cpu().numpy()[:, :, None])
+    bla.bla_device_error()
+    assert rel(np.concatenate(outs, 2), full["o"]) <= tol
+    assert rel(st.cpu().numpy(), full["state"]) <= tol
+
+
+def test_shared_period_unchanged(orc):
+    """Equal per-head periods give the shared-period result."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    q, k, v = (to_dev(x, dev, torch.float32) for x in make_qkv(1, 3, 70, 32, dtype="f32", seed=2))
+    a = bla.bla_forward_chunked(q, k, v, 4, 7, [16.0] * 3, chunk=16)[0]
+    b = bla.bla_forward_chunked(q, k, v, 4, 7, 16.0, chunk=16)[0]
+    bla.bla_device_error()
+    assert rel(a.cpu().numpy(), b.cpu().numpy()) <= 1e-6
+
+
+def test_decay_backward(orc):
+    """The decayed VJP with one period per head against the oracle's per-head VJP."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_dout, make_qkv
+    dev = require_cuda()
+    B, H, L, d, M, S = 1, 3, 60, 32, 4, 7
+    q, k, v = make_qkv(B, H, L, d, dtype="f32", seed=17)
+    do = make_dout(B, H, L, d, dtype="f32", seed=17)
+    tq, tk, tv, tdo = (to_dev(x, dev, torch.float32) for x in (q, k, v, do))
+    o, lse, _ = bla.bla_decay_forward(tq, tk, tv, M, S, TS)
+    got = bla.bla_decay_backward(tq, tk, tv, o, tdo, lse, M, S, TS)
+    bla.bla_device_error()
+    ref = orc.backward_decay(q, k, v, do, M, S, TS)
+    for name, a, b in zip(("dq", "dk", "dv"), got, ref):
+        assert rel(a.cpu().numpy(), b) <= 1e-4, (name, rel(a.cpu().numpy(), b))
