@@ -10,7 +10,8 @@ own independent batch; there is no collective on the data path).
 Printed (rank 0, one JSON line): the device-timed throughput with inputs resident in HBM,
 the roofline of the dominant kernel (per-launch CUDA-event time on its launch stream, against
 the measured bf16 peak), the end-to-end throughput through host buffers (H2D of q,k,v and D2H
-of o inside the timed region), SM clocks sampled during the timed region, the number of this
+of o inside the timed region), SM clocks sampled during timed work (the K steps and a sustained
+leg of the same step looped for >= 1.5 s, reported beside them), the number of this
 library's kernel launches in the timed region, the decode step's HBM roofline, and the float64
 oracle timed on the host cores on a bounded sample of the same workload.
 
@@ -18,6 +19,7 @@ oracle timed on the host cores on a bounded sample of the same workload.
 on bounded samples of the same workload and prints the same line with "impl": "reference".
 """
 import argparse
+import math
 import json
 import os
 import statistics
@@ -84,10 +86,11 @@ class ClockSampler:
         self.thread.start()
 
     def _read(self):
+        # nvidia-smi prints each sample as it takes it: the read time stamps the sample
         for line in self.proc.stdout:
             parts = [x.strip() for x in line.split(",")]
             if len(parts) >= 8:
-                self.rows.append(parts)
+                self.rows.append((time.perf_counter(), parts))
 
     def stop(self):
         if self.proc is not None:
@@ -99,10 +102,14 @@ class ClockSampler:
         if self.thread is not None:
             self.thread.join(timeout=2)
 
-    def summary(self):
+    def summary(self, t0=None, t1=None):
+        """Median SM clock, max clock and throttle reasons of the samples taken in [t0, t1]
+        (perf_counter seconds; all samples when not given)."""
         sm, mx, reasons = [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for r in self.rows:
+        for ts, r in self.rows:
+            if (t0 is not None and ts < t0) or (t1 is not None and ts > t1):
+                continue
             try:
                 sm.append(float(r[0]))
                 mx.append(float(r[1]))
@@ -252,6 +259,7 @@ def main():
     ap.add_argument("--configs-only", default="",
                     help="comma-separated parity configs to time alone (profiling captures); prints their JSON")
     ap.add_argument("--configs-iters", type=int, default=20, help="timed calls per parity config")
+    ap.add_argument("--no-sustained", action="store_true", help="skip the >= 1.5 s sustained leg (profiling captures)")
     args = ap.parse_args()
     if args.impl == "reference":
         return run_reference(args)
@@ -302,6 +310,14 @@ def main():
     launches = bla.bla_kernel_launches() - n0
     if world > 1:
         torch.distributed.barrier()
+    # ---- sustained leg: the same step back to back for >= 1.5 s, so that the clock samples (every
+    # 200 ms) fall inside timed work and the power-capped clock is seen; reported beside the K steps
+    sus_steps = 0 if args.no_sustained else max(steps, int(math.ceil(1500.0 / max(ms, 1e-3))))
+    t_sus0 = time.perf_counter()
+    sus_ms = time_steps(step, sus_steps, stream) if sus_steps else float("nan")
+    t_sus1 = time.perf_counter()
+    if world > 1:
+        torch.distributed.barrier()
     sampler.stop()
     bla.bla_device_error()
     ms = barrier_max(ms, world)
@@ -331,6 +347,13 @@ def main():
                 "flops_per_launch": dom_flops, "ms_per_launch": dom_ms,
                 "kernels_ms_per_launch": per_launch,
                 "step_frac_of_peak": flops["total"] * w.B * w.H * w.L / (ms / 1000.0) / 1e12 / peak}
+    sus_ms = barrier_max(sus_ms, world) if sus_steps else None
+    sustained_leg = None if not sus_steps else {"steps": sus_steps, "seconds": t_sus1 - t_sus0, "ms_per_step": sus_ms,
+                     "value": whole_job_rate(world, tokens_per_step, sus_ms), "unit": "tokens/s",
+                     "peak": peaks["bf16_tflops_sustained"],
+                     "step_frac_of_sustained_peak": flops["total"] * w.B * w.H * w.L / (sus_ms / 1000.0) / 1e12 /
+                     peaks["bf16_tflops_sustained"],
+                     "clocks": sampler.summary(t_sus0, t_sus1)}
 
     # ---- end to end through host buffers (pinned), copies inside the timed region
     e2e = None
@@ -407,7 +430,8 @@ def main():
                            "inputs": "q,k,v bf16 805 MB resident, larger than the 129 MB L2 (no flush)",
                            "accumulate": "fp32 (TMEM), state fp32"},
                 "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches,
-                "clocks": sampler.summary(), "decode": decode, "configs": configs}
+                "clocks": dict(sampler.summary(t_wall0, t_sus1), window="timed steps and the sustained leg"),
+                "sustained": sustained_leg, "decode": decode, "configs": configs}
         print(json.dumps(line))
     if world > 1:
         torch.distributed.destroy_process_group()

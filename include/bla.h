@@ -154,7 +154,9 @@ bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const vo
  *              includes this token.
  *   o          [B][H][d_v] (device), dtype p->dtype.
  *   workspace  device scratch of >= bla_workspace_bytes(p, BLA_WS_DECODE) bytes.
- * p->L is ignored.  Requires d_k = d_v in {32, 64, 128} and S <= 256.
+ * p->L is ignored.  Requires d_k = d_v in {32, 64, 128}, S <= 256, and
+ * 4 (2M + S + 8 d_k) bytes of shared memory at most 227 KB (M up to about 28,000);
+ * other sizes return BLA_ERR_UNSUPPORTED before any launch.
  */
 bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, const void *k,
                            const void *v, float *state, void *o, void *workspace, size_t ws_bytes,
@@ -164,13 +166,18 @@ bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, co
  * bla_decode_step for callers that may not allocate device memory (the paper has no
  * counterpart; this is a deployment convenience).  Same arguments and results as
  * bla_decode_step, without the workspace: the step's tables live in a fixed 512 KiB
- * device array owned by the library (reserved on every GPU that loads it, until exit).
- * Meant for callers that run within a fixed, pre-reserved memory budget or must not
- * call the allocator mid-step (cudaMalloc can synchronise the device).
+ * device array owned by the library.  Meant for callers that run within a fixed,
+ * pre-reserved memory budget or must not call the allocator mid-step (cudaMalloc can
+ * synchronise the device).
+ *   - The array takes its 512 KiB of device memory when the library's module is loaded
+ *     on a device (with lazy module loading, the CUDA default, at the first use of the
+ *     module there, at the latest on the first call) and keeps it until exit.  Make the
+ *     first call before reserving a fixed memory budget and before any stream capture.
  *   - Parameters whose tables exceed the array are rejected with BLA_ERR_UNSUPPORTED
- *     before any launch.
- *   - The array's device address is looked up on the first call made on each device;
- *     make that first call before any stream capture.
+ *     before any launch; the argument checks are those of bla_decode_step.
+ *   - The array's device address is looked up on the first call made on each device and
+ *     kept for the life of that device's primary context: do not call this entry point
+ *     on a device after cudaDeviceReset.
  *   - All calls share the array (it keeps the last call's tables, rewritten in full by
  *     every call): calls that overlap on the GPU race and must be ordered by the caller.
  */

@@ -59,19 +59,26 @@ ProfScope::~ProfScope() {
     if (slot < (int)g_prof_recs.size()) cudaEventRecord(g_prof_recs[slot].b, stream);
 }
 
+NvtxRange::NvtxRange(const char *name) { nvtxRangePushA(name); }
+NvtxRange::~NvtxRange() { nvtxRangePop(); }
+
 __device__ int g_dev_error = 0;
 
+// The address is cached per device for the life of the device's primary context (host threads
+// may race on the first lookup; both store the same value).
 int *device_error_word() {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
-    static int *cache[64] = {nullptr};
+    static std::atomic<int *> cache[64];
     if (dev < 0 || dev >= 64) return nullptr;
-    if (!cache[dev]) {
+    int *w = cache[dev].load(std::memory_order_acquire);
+    if (!w) {
         void *ptr = nullptr;
         if (cudaGetSymbolAddress(&ptr, g_dev_error) != cudaSuccess) return nullptr;
-        cache[dev] = static_cast<int *>(ptr);
+        w = static_cast<int *>(ptr);
+        cache[dev].store(w, std::memory_order_release);
     }
-    return cache[dev];
+    return w;
 }
 
 namespace {
@@ -101,12 +108,6 @@ constexpr double kPi = 3.14159265358979323846;
 constexpr int kDefaultChunkF32 = 64;
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
-
-// An NVTX range around each entry point (visible in Nsight timelines; free when no tool listens).
-struct NvtxRange {
-    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
-    ~NvtxRange() { nvtxRangePop(); }
-};
 
 // Common parameter checks; fills the derived dimensions.
 bla_status check_params(const bla_params *p, OpDims *d) {
@@ -311,6 +312,24 @@ bla_status forward_device(const bla_params *p, const OpDims &d, const void *q, c
 }
 
 }  // namespace
+
+bla_status check_decode(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
+                        const float *state, const void *o, OpDims *d) {
+    bla_status s = check_params(p, d);
+    if (s != BLA_OK) return s;
+    if (pos < 0) return fail(BLA_ERR_INVALID, "pos must be >= 0 (got %lld)", pos);
+    if (!q || !k || !v || !state || !o) return fail(BLA_ERR_INVALID, "q, k, v, state and o must be non-NULL");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(state) || !aligned16(o))
+        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
+    if (d->dk != d->dv || (d->dk != 32 && d->dk != 64 && d->dk != 128))
+        return fail(BLA_ERR_UNSUPPORTED, "decode needs d_k = d_v in {32, 64, 128} (got %d, %d)", d->dk, d->dv);
+    if (d->S > 256) return fail(BLA_ERR_UNSUPPORTED, "decode needs S <= 256 (got %d)", d->S);
+    if (decode_smem_bytes(*d) > 227 * 1024)
+        return fail(BLA_ERR_UNSUPPORTED, "decode needs %d bytes of shared memory (M=%d), more than 227 KB",
+                    decode_smem_bytes(*d), d->M);
+    return BLA_OK;
+}
+
 }  // namespace bla
 
 using namespace bla;
@@ -421,15 +440,8 @@ bla_status bla_decode_step(const bla_params *p, long long pos, const void *q, co
     t_last_error[0] = 0;
     NvtxRange nvtx("bla_decode_step");
     OpDims d;
-    bla_status s = check_params(p, &d);
+    bla_status s = check_decode(p, pos, q, k, v, state, o, &d);
     if (s != BLA_OK) return s;
-    if (pos < 0) return fail(BLA_ERR_INVALID, "pos must be >= 0 (got %lld)", pos);
-    if (!q || !k || !v || !state || !o) return fail(BLA_ERR_INVALID, "q, k, v, state and o must be non-NULL");
-    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(state) || !aligned16(o))
-        return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
-    if (d.dk != d.dv || (d.dk != 32 && d.dk != 64 && d.dk != 128))
-        return fail(BLA_ERR_UNSUPPORTED, "decode needs d_k = d_v in {32, 64, 128} (got %d, %d)", d.dk, d.dv);
-    if (d.S > 256) return fail(BLA_ERR_UNSUPPORTED, "decode needs S <= 256 (got %d)", d.S);
     size_t need = ws_decode(d);
     if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);

@@ -140,5 +140,19 @@ int forward_f32_smem_bytes(const OpDims &d, int C);
 
 cudaError_t launch_decode(const OpDims &d, long long pos, const Tables &t, const void *q, const void *k,
                           const void *v, float *state, void *o, cudaStream_t st);
+// Dynamic shared memory of one decode launch (the launcher opts in above 48 KB).
+int decode_smem_bytes(const OpDims &d);
+
+// Checks shared by both decode entry points (api.cu): the common parameter checks, pos >= 0,
+// non-NULL 16-byte-aligned tensors, d_k = d_v in {32, 64, 128}, S <= 256 and the decode's shared
+// memory; fills `d`.  Sets the thread's last-error text on failure.
+bla_status check_decode(const bla_params *p, long long pos, const void *q, const void *k, const void *v,
+                        const float *state, const void *o, OpDims *d);
+
+// An NVTX range around an entry point (visible in Nsight timelines; free when no tool listens).
+struct NvtxRange {
+    explicit NvtxRange(const char *name);
+    ~NvtxRange();
+};
 
 }  // namespace bla

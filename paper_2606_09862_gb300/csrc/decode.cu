@@ -241,7 +241,11 @@ __global__ void __launch_bounds__(kThreads) k_decode(OpDims d, long long pos, Ta
 template <typename T, int D>
 cudaError_t launch_decode_t(const OpDims &d, long long pos, const Tables &t, const void *q, const void *k,
                             const void *v, float *state, void *o, cudaStream_t st) {
-    int smem = (int)(sizeof(float) * (d.R2 + d.S + kWarps * D));
+    const int smem = decode_smem_bytes(d);
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(k_decode<T, D>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+    }
     ProfScope ps(BLA_K_DECODE, st);
     k_decode<T, D><<<d.B * d.H, kThreads, smem, st>>>(d, pos, t, (const T *)q, (const T *)k, (const T *)v, state,
                                                      (T *)o);
@@ -249,6 +253,10 @@ cudaError_t launch_decode_t(const OpDims &d, long long pos, const Tables &t, con
 }
 
 }  // namespace
+
+int decode_smem_bytes(const OpDims &d) {
+    return (int)(sizeof(float) * ((size_t)d.R2 + d.S + (size_t)kWarps * d.dk));
+}
 
 cudaError_t launch_decode(const OpDims &d, long long pos, const Tables &t, const void *q, const void *k,
                           const void *v, float *state, void *o, cudaStream_t st) {

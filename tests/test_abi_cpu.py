@@ -89,6 +89,24 @@ def test_decode_argument_checks(lib):
         bla.BLA_ERR_UNSUPPORTED
 
 
+def test_both_decode_entry_points_share_their_checks(lib):
+    """bla_decode_step and bla_decode_step_noalloc reject the same arguments on the host, before any
+    launch: B*H beyond the int grid, a negative position, an unsupported head size, and a mode count
+    whose decode needs more shared memory than a CTA has."""
+    from paper_2606_09862_gb300 import bla
+
+    def both(p, pos=0):
+        a = lib.bla_decode_step(ctypes.byref(p), pos, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30, None)
+        b = lib.bla_decode_step_noalloc(ctypes.byref(p), pos, FAKE, FAKE, FAKE, FAKE, FAKE, None)
+        return a, b
+
+    assert both(_params(B=1 << 16, H=1 << 16)) == (bla.BLA_ERR_INVALID,) * 2
+    assert both(_params(), pos=-1) == (bla.BLA_ERR_INVALID,) * 2
+    assert both(_params(d_k=48, d_v=48)) == (bla.BLA_ERR_UNSUPPORTED,) * 2
+    assert both(_params(M=30000, S=64, window=1e5)) == (bla.BLA_ERR_UNSUPPORTED,) * 2
+    assert b"shared memory" in lib.bla_last_error_string()
+
+
 def test_workspace_sizes_positive(lib):
     from paper_2606_09862_gb300 import bla
     p = _params()

@@ -2,7 +2,7 @@
 import numpy as np
 import pytest
 
-from gpu_util import TOL_GRAD, rel, require_cuda, to_dev
+from gpu_util import TOL_GRAD, TOL_ROW_SHARP_GRAD, rel, require_cuda, row_errors, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -45,6 +45,23 @@ def test_gradients_sharp_softmax(orc):
         assert rel(a, b) <= TOL_GRAD, (name, rel(a, b))
 
 
+def test_lm_layer_workload_gradients_sharp_sampled_heads(orc):
+    """The LM-layer shape (B=8, H=8, L=4096, d=128, M=64, S=64, T=1024) with sharp q, k ~ N(0,1):
+    the full-size backward recomputes p from an lse taken at |s| up to ~30; every gradient of three
+    sampled (batch, head) pairs against the oracle, pooled and per row."""
+    from paper_2606_09862_gb300.inputs import WORKLOADS, workload_inputs
+    w = WORKLOADS["fwdbwd_bf16_lm"]
+    x = workload_inputs(w, seed=0, sharp=True)
+    got = run(x["q"], x["k"], x["v"], x["dout"], w.M, w.S, w.T)
+    for b, h in ((0, 0), (3, 5), (7, 7)):
+        sl = (slice(b, b + 1), slice(h, h + 1))
+        ref = orc.backward(x["q"][sl], x["k"][sl], x["v"][sl], x["dout"][sl], w.M, w.S, w.T)
+        for name, a, r in zip(("dq", "dk", "dv"), got, ref):
+            pooled, worst = row_errors(a[sl], r)
+            assert pooled <= TOL_GRAD, (name, b, h, pooled)
+            assert worst <= TOL_ROW_SHARP_GRAD, (name, b, h, worst)
+
+
 def test_lm_layer_workload_gradients_sampled_heads(orc):
     """B=8, H=8, L=4096, d=128, M=64, S=64, T=1024, dO ~ N(0,1): the full-size backward on the GPU;
     every gradient of three sampled (batch, head) pairs against the oracle (heads are independent)."""
@@ -56,4 +73,6 @@ def test_lm_layer_workload_gradients_sampled_heads(orc):
         sl = (slice(b, b + 1), slice(h, h + 1))
         ref = orc.backward(x["q"][sl], x["k"][sl], x["v"][sl], x["dout"][sl], w.M, w.S, w.T)
         for name, a, r in zip(("dq", "dk", "dv"), got, ref):
-            assert rel(a[sl], r) <= TOL_GRAD, (name, b, h, rel(a[sl], r))
+            pooled, worst = row_errors(a[sl], r)
+            assert pooled <= TOL_GRAD, (name, b, h, pooled)
+            assert worst <= TOL_GRAD, (name, b, h, worst)

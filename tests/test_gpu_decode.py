@@ -2,7 +2,7 @@
 import numpy as np
 import pytest
 
-from gpu_util import TOL_BF16, TOL_F32, rel, require_cuda, to_dev
+from gpu_util import TOL_BF16, TOL_F32, TOL_ROW_BF16, rel, require_cuda, row_errors, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -98,4 +98,7 @@ def test_decode_workload_1024_steps(orc):
                       return_state=True)
     worst = max(rel(outs[:, 0, s], ref["o"][:, 0, s]) for s in range(nsteps))
     assert worst <= TOL_BF16, worst
+    # every (head, step) output row on its own
+    pooled, worst_row = row_errors(outs, ref["o"])
+    assert pooled <= TOL_BF16 and worst_row <= TOL_ROW_BF16, (pooled, worst_row)
     assert rel(tst.cpu().numpy()[bi, hi], ref["state"][:, 0]) <= TOL_F32

@@ -2,7 +2,7 @@
 import numpy as np
 import pytest
 
-from gpu_util import TOL_BF16, rel, require_cuda, to_dev
+from gpu_util import TOL_BF16, TOL_ROW_BF16, TOL_ROW_SHARP, lse_bound, rel, require_cuda, row_errors, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -36,12 +36,20 @@ def test_shapes_against_oracle(orc, B, H, L, d, M, S, T):
     assert rel(st, ref["state"]) <= TOL_BF16
 
 
-def test_sharp_softmax(orc):
+@pytest.mark.parametrize("B,H,L,d,M,S,T", [
+    (1, 2, 2000, 128, 128, 128, 4096.0),   # 2M = 256, two segments' worth of sharp scores
+    (1, 2, 4096, 128, 64, 64, 1024.0),     # the LM-layer shape per head (2M = 128)
+])
+def test_sharp_softmax(orc, B, H, L, d, M, S, T):
+    """q, k ~ N(0,1): peaked softmax rows (|s| up to ~30).  o pooled and per row, lse per token, state."""
     from paper_2606_09862_gb300.inputs import make_qkv
-    q, k, v = make_qkv(1, 2, 2000, 128, dtype="bf16", seed=3, sharp=True)
-    o, lse, st = run(q, k, v, 128, 128, 4096.0)
-    ref = orc.forward(q, k, v, 128, 128, 4096.0, form="modes", return_state=True)
-    assert rel(o, ref["o"]) <= TOL_BF16, rel(o, ref["o"])
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=3 + L, sharp=True)
+    o, lse, st = run(q, k, v, M, S, T)
+    ref = orc.forward(q, k, v, M, S, T, form="modes", return_state=True)
+    pooled, worst = row_errors(o, ref["o"])
+    assert pooled <= TOL_BF16, pooled
+    assert worst <= TOL_ROW_SHARP, worst
+    assert np.all(np.abs(lse - ref["lse"]) <= lse_bound(ref["lse"])), np.abs(lse - ref["lse"]).max()
     assert rel(st, ref["state"]) <= TOL_BF16
 
 
@@ -52,7 +60,10 @@ def test_recall_workload_full(orc):
     x = workload_inputs(w, seed=0)
     o, lse, st = run(x["q"], x["k"], x["v"], w.M, w.S, w.T)
     ref = orc.forward(x["q"], x["k"], x["v"], w.M, w.S, w.T, form="modes", return_state=True)
-    assert rel(o, ref["o"]) <= TOL_BF16, rel(o, ref["o"])
+    pooled, worst = row_errors(o, ref["o"])
+    assert pooled <= TOL_BF16, pooled
+    assert worst <= TOL_ROW_BF16, worst
+    assert np.all(np.abs(lse - ref["lse"]) <= lse_bound(ref["lse"]))
     assert rel(st, ref["state"]) <= TOL_BF16
 
 
@@ -63,7 +74,10 @@ def test_lm_layer_workload_forward_full(orc):
     x = workload_inputs(w, seed=0)
     o, lse, st = run(x["q"], x["k"], x["v"], w.M, w.S, w.T)
     ref = orc.forward(x["q"], x["k"], x["v"], w.M, w.S, w.T, form="modes", return_state=True)
-    assert rel(o, ref["o"]) <= TOL_BF16, rel(o, ref["o"])
+    pooled, worst = row_errors(o, ref["o"])
+    assert pooled <= TOL_BF16, pooled
+    assert worst <= TOL_ROW_BF16, worst
+    assert np.all(np.abs(lse - ref["lse"]) <= lse_bound(ref["lse"]))
     assert rel(st, ref["state"]) <= TOL_BF16
 
 
@@ -81,7 +95,9 @@ def test_long_prefill_workload_sampled(orc):
     want[128::128] = True
     want[-5:] = True
     ref = orc.forward(x["q"], x["k"], x["v"], w.M, w.S, w.T, form="modes", want=want, return_state=True)
-    assert rel(o[:, :, want], ref["o"][:, :, want]) <= TOL_BF16, rel(o[:, :, want], ref["o"][:, :, want])
+    pooled, worst = row_errors(o[:, :, want], ref["o"][:, :, want])
+    assert pooled <= TOL_BF16, pooled
+    assert worst <= TOL_ROW_BF16, worst
     assert np.abs(lse[:, :, want] - ref["lse"][:, :, want]).max() <= 5e-2
     assert rel(st, ref["state"]) <= TOL_BF16
 
