@@ -75,8 +75,9 @@ typedef struct {
                                (2*pi/T_h unless omega > 0) and coefficients follow periods[h], each
                                clamped to max(T_h, 2M-1); S must not exceed any of them.  Read
                                during the call only.  At most 256 heads.  Supported by the fp32
-                               forward, bla_decode_step and the state-decay entry points; the others
-                               return BLA_ERR_UNSUPPORTED. */
+                               and bf16 forwards (device and host buffers), both decode entry
+                               points and the state-decay entry points; bla_backward returns
+                               BLA_ERR_UNSUPPORTED. */
 } bla_params;
 
 /* How a slot reads the past (bla_params.phase_mode).

@@ -376,7 +376,6 @@ bla_status bla_forward_chunked(const bla_params *p, const void *q, const void *k
         !aligned16(state_out))
         return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
     if (d.dtype == BLA_BF16) {
-        if ((s = no_per_head(d, "the bf16 forward")) != BLA_OK) return s;
         const char *why = fwd_bf16_unsupported(d);
         if (why) return fail(BLA_ERR_UNSUPPORTED, "bf16 forward: %s", why);
     }
@@ -391,7 +390,6 @@ bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const vo
     OpDims d;
     bla_status s = check_params(p, &d);
     if (s != BLA_OK) return s;
-    if ((s = no_per_head(d, "the host-buffer forward")) != BLA_OK) return s;
     if (d.L > 0 && (!q || !k || !v || !o)) return fail(BLA_ERR_INVALID, "q, k, v and o must be non-NULL");
     if (d.dtype == BLA_BF16) {
         const char *why = fwd_bf16_unsupported(d);
@@ -423,8 +421,17 @@ bla_status bla_forward_chunked_host(const bla_params *p, const void *q, const vo
             (e = cudaMemcpyAsync(vd + h0 * rv, vh + h0 * rv, nh * rv, cudaMemcpyHostToDevice, hp->h2d)) != cudaSuccess ||
             (e = cudaEventRecord(hp->in[g], hp->h2d)) != cudaSuccess || (e = cudaStreamWaitEvent(st, hp->in[g], 0)) != cudaSuccess)
             return cuda_fail(e, "host-to-device copy");
-        if ((s = forward_device(p, host_group_dims(d, nh), qd + h0 * rq, kd + h0 * rq, vd + h0 * rv, od + h0 * rv, nullptr,
-                                nullptr, ws, st)) != BLA_OK)
+        // the group's heads as one batch; with per-head periods, their periods in the group's order
+        // (read on the host only, during the launch)
+        OpDims gd = host_group_dims(d, nh);
+        std::vector<double> gper;
+        if (d.periods) {
+            gper.resize((size_t)nh);
+            for (long long i = 0; i < nh; ++i) gper[(size_t)i] = d.periods[(h0 + i) % d.H];
+            gd.periods = gper.data();
+        }
+        if ((s = forward_device(p, gd, qd + h0 * rq, kd + h0 * rq, vd + h0 * rv, od + h0 * rv, nullptr, nullptr, ws,
+                                st)) != BLA_OK)
             return s;
         if ((e = cudaEventRecord(hp->out[g], st)) != cudaSuccess || (e = cudaStreamWaitEvent(hp->d2h, hp->out[g], 0)) != cudaSuccess ||
             (e = cudaMemcpyAsync(oh + h0 * rv, od + h0 * rv, nh * rv, cudaMemcpyDeviceToHost, hp->d2h)) != cudaSuccess)

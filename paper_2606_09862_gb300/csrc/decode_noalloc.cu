@@ -75,7 +75,6 @@ extern "C" bla_status bla_decode_step_noalloc(const bla_params *p, long long pos
     OpDims d;
     const bla_status s = check_decode(p, pos, q, k, v, state, o, &d);
     if (s != BLA_OK) return s;
-    if (d.periods) return reject(BLA_ERR_UNSUPPORTED, "the no-alloc decode does not support per-head periods yet");
     const size_t need = tables_bytes(d, 0);
     if (need > kNoAllocScratchBytes)
         return reject(BLA_ERR_UNSUPPORTED,

@@ -103,16 +103,21 @@ Geo make_geo(const OpDims &d) {
 }
 
 struct WsLayout {
-    size_t delta, eb, phi, fseg, deltas, win, pbuf, total;
+    size_t delta, eb, phi, fseg, hw, htint, deltas, win, pbuf, total;
 };
 
+// With per-head periods every table is repeated per head (nh = H), plus each head's mode frequency
+// and integer period; with one shared period nh = 1 and the head arrays are absent.
 WsLayout ws_layout(const OpDims &d, const Geo &g) {
     WsLayout w;
+    const size_t nh = d.periods ? (size_t)d.H : 1;
     size_t off = 0;
-    w.delta = off;  off += align_up(sizeof(int) * (size_t)g.S, 1024);
-    w.eb = off;     off += align_up(sizeof(bf16) * (size_t)g.nchunks * g.RP * kC, 1024);   // EB per chunk
-    w.phi = off;    off += align_up(sizeof(bf16) * (size_t)g.SP * g.R2, 1024);
-    w.fseg = off;   off += g.G > 1 ? align_up(sizeof(bf16) * (size_t)g.RP * g.Lseg, 1024) : 0;
+    w.delta = off;  off += align_up(sizeof(int) * nh * g.S, 1024);
+    w.eb = off;     off += align_up(sizeof(bf16) * nh * g.nchunks * g.RP * kC, 1024);   // EB per chunk
+    w.phi = off;    off += align_up(sizeof(bf16) * nh * g.SP * g.R2, 1024);
+    w.fseg = off;   off += g.G > 1 ? align_up(sizeof(bf16) * nh * g.RP * g.Lseg, 1024) : 0;
+    w.hw = off;     off += d.periods ? align_up(sizeof(double) * nh, 256) : 0;
+    w.htint = off;  off += d.periods ? align_up(sizeof(int) * nh, 256) : 0;
     w.deltas = off; off += g.G > 1 ? align_up(sizeof(float) * (size_t)g.BH * g.G * 2 * g.RP * g.D, 1024) : 0;
     w.win = off;    off += g.G > 1 ? align_up(sizeof(float) * (size_t)g.BH * g.G * 2 * g.RP * g.D, 1024) : 0;
     w.pbuf = off;   off += align_up(sizeof(bf16) * (size_t)g.BH * (g.L > 0 ? g.L : 1) * g.SP, 1024);
@@ -146,16 +151,38 @@ __device__ __forceinline__ void mode_phase(long long mu, double w, int tint, flo
 //   delta [S] (optional): the slot lags D_j
 // EB is written by one thread per (c, m, 8 consecutive u), u fastest so that a warp writes whole
 // rows: the first phase is reduced exactly, the next seven follow by products with e^{i m w}.
-__global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, double T, double w, int tint,
-                              float sin_sign, bf16 *eb, bf16 *phi, bf16 *fseg, int *delta) {
+// Per-head periods (Alg. 1 and Alg. 3: T in R^H; hp.n = H > 0): head h writes its own copy of every
+// table at (T_h, w_h, tint_h), one table block after the other, and hw[h], htint[h]; with hp.n = 0
+// the single (T, w, tint) is used.
+struct HeadTint {
+    int t[kMaxHeadPeriods];   // each head's integer period for exact phase reduction (0: fp64 phases)
+};
+
+__global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, HeadPeriods hp, HeadTint ht, double T0,
+                              double w0, int tint0, float sin_sign, bf16 *eb0, bf16 *phi0, bf16 *fseg0, int *delta0,
+                              double *hw, int *htint) {
     const int R2 = 2 * M, MP = RP / 2;
     const long long n_eb = (long long)nch * MP * (kC / 8), n_phi = (long long)SP * R2;
-    const long long n_f = fseg ? (long long)MP * ((Lseg + 7) / 8) : 0, n_d = delta ? S : 0;
-    const long long total = n_eb + n_phi + n_f + n_d;
+    const long long n_f = fseg0 ? (long long)MP * ((Lseg + 7) / 8) : 0, n_d = delta0 ? S : 0;
+    const long long per = n_eb + n_phi + n_f + n_d + 1;
+    const int nh = hp.n > 0 ? hp.n : 1;
+    const long long total = per * nh;
     const double n = 2.0 * M - 1.0;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        if (i < n_eb) {
+    for (long long ii = blockIdx.x * (long long)blockDim.x + threadIdx.x; ii < total;
+         ii += (long long)gridDim.x * blockDim.x) {
+        const int h = hp.n > 0 ? (int)(ii / per) : 0;   // (one shared period: ii < per)
+        const long long i = ii - (long long)h * per;
+        const double T = hp.n > 0 ? hp.T[h] : T0, w = hp.n > 0 ? hp.w[h] : w0;
+        const int tint = hp.n > 0 ? ht.t[h] : tint0;
+        bf16 *eb = eb0 + (size_t)h * nch * RP * kC, *phi = phi0 + (size_t)h * SP * R2;
+        bf16 *fseg = fseg0 ? fseg0 + (size_t)h * RP * Lseg : nullptr;
+        int *delta = delta0 ? delta0 + (size_t)h * S : nullptr;
+        if (i == per - 1) {
+            if (hp.n > 0) {
+                hw[h] = w;
+                htint[h] = tint;
+            }
+        } else if (i < n_eb) {
             // (32-bit index arithmetic: n_eb = 16 L < 2^31 for L <= 2^26, which the host checks)
             const unsigned per_c = (unsigned)MP * (kC / 8), ui = (unsigned)i;
             const int c = (int)(ui / per_c), rem = (int)(ui - (unsigned)c * per_c);
@@ -235,7 +262,26 @@ struct Args {
     int tint;            // integer period for exact phase reduction (0: use fp64 phases)
     int absolute;        // absolute form (Alg. 1): the drains do not rotate rows by e^{i m w t}
     int *err;
+    // Per-head periods (Alg. 1 and Alg. 3: T in R^H): head h = bh % H reads its own tables at these
+    // per-head strides (rows of the EB, PHI and FSEG tensor maps; entries of delta) and its own w and
+    // integer period; all four strides are 0 and hw, htint null when the heads share one period.
+    int H;
+    int eb_rows_h, phi_rows_h, f_rows_h, delta_h;
+    const double *hw;
+    const int *htint;
 };
+
+// Mode frequency and integer period of head bh % H (written by the tables kernel: read them only
+// after the programmatic-launch wait).
+struct HeadW {
+    double w;
+    int tint;
+};
+__device__ __forceinline__ HeadW head_w(const Args &a, int bh) {
+    if (!a.hw) return HeadW{a.w, a.tint};
+    const int hd = bh % a.H;
+    return HeadW{a.hw[hd], a.htint[hd]};
+}
 
 // Bounded-wait bookkeeping shared by the roles of one CTA.
 struct Ctl {
@@ -516,13 +562,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int t_seg = seg * g.Lseg;
 
     if (warp == 4 && lane == 0) {
+        const int fy = (bh % a.H) * a.f_rows_h;   // this head's FSEG rows
         uint32_t ph[kPreStages] = {0, 0, 0};
         for (int it = 0; it < steps; ++it) {
             const int st = it % kPreStages;
             if (it >= kPreStages && !wait_bar(&empty[st], ph[st], ctl, a.err)) break;
             uint8_t *base = stage0 + st * stage_bytes;
             tc::mbar_arrive_expect_tx(&full[st], (uint32_t)stage_bytes);
-            for (int b = 0; b < NB; ++b) tc::tma_load_2d(base + b * 128 * 128, &tm_f, &full[st], it * 64, b * 128);
+            for (int b = 0; b < NB; ++b)
+                tc::tma_load_2d(base + b * 128 * 128, &tm_f, &full[st], it * 64, fy + b * 128);
             for (int db = 0; db < D / 64; ++db) {
                 tc::tma_load_3d(base + f_bytes + db * 64 * 128, &tm_k, &full[st], db * 64, t_seg + it * 64, bh);
                 tc::tma_load_3d(base + f_bytes + x_bytes + db * 64 * 128, &tm_v, &full[st], db * 64, t_seg + it * 64,
@@ -587,7 +635,8 @@ __global__ void k_scan(Args a) {
         const int x = (int)(r % 2);
         const int bh = (int)(r / 2);
         float c, s;
-        mode_phase((long long)m * g.Lseg, a.w, a.tint, &c, &s);
+        const HeadW hw = head_w(a, bh);
+        mode_phase((long long)m * g.Lseg, hw.w, hw.tint, &c, &s);
         float re = 0.f, im = 0.f;
         // the deltas of eight segments are loaded before they are used, so that their latencies overlap
         for (int s0 = 0; s0 < g.G; s0 += 8) {
@@ -691,7 +740,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     if (warp == 9) { tc::tmem_alloc(tslot, ncols); tc::tmem_relinquish(); }
     // the tables and the entering states come from the kernels before this one
     tc::pdl_wait();
-    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[j];
+    for (int j = threadIdx.x; j < S; j += blockDim.x) sdelta[j] = a.delta[(bh % a.H) * a.delta_h + j];
+    const HeadW hph = head_w(a, bh);                      // this head's w and integer period
+    const int eby = (bh % a.H) * a.eb_rows_h, phy = (bh % a.H) * a.phi_rows_h;   // its table rows
     tc::tc_fence_before();
     __syncthreads();
     tc::tc_fence_after();
@@ -727,12 +778,13 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         first_eb = false;
                         tc::mbar_arrive_expect_tx(&bar[KB_EB_FULL], (uint32_t)(128 * kC * 2));
                         for (int kb = 0; kb < 2; ++kb)
-                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[KB_EB_FULL], kb * 64, c * g.RP + h * 128);
+                            tc::tma_load_2d(sEB + kb * 128 * 128, &tm_eb, &bar[KB_EB_FULL], kb * 64,
+                                            eby + c * g.RP + h * 128);
                         if (!first_phi && !wait_bar(&bar[KB_PHI_FREE], ph_phi, ctl, a.err)) break;
                         first_phi = false;
                         tc::mbar_arrive_expect_tx(&bar[KB_PHI_FULL], (uint32_t)(SP * RH * 2));
                         for (int kb = 0; kb < RH / 64; ++kb)
-                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[KB_PHI_FULL], h * RH + kb * 64, 0);
+                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[KB_PHI_FULL], h * RH + kb * 64, phy);
                     }
                 }
             }
@@ -861,8 +913,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             // the drain phases of this row: exact at the CTA's first chunk, then advanced per chunk
             const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
             // (the absolute form reads the absolute-frame products as they are: every phase is 1)
-            RowPhases rp = row_phases(a.absolute ? 0 : (long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
-            const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, a.w, a.tint);
+            RowPhases rp = row_phases(a.absolute ? 0 : (long long)c_begin * kC + row, m00, m10, NH == 2, hph.w,
+                                      hph.tint);
+            const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, hph.w, hph.tint);
             // the state is kept in the absolute frame, A = sum_{u < t0} e^{-i m w u} k_u: it needs no
             // rotation between chunks; the carried-in lag-frame state is rotated once
             if (g.NB > 1 && g.G > 1)
@@ -870,7 +923,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                                        g.R2 - 128, D);
             for (int b = 0; b < g.NB; ++b) {
                 const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 0) * g.RP + b * 128) * D : nullptr;
-                const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
+                const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, hph.w, hph.tint);
                 state_init_abs<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D, f.x, f.y);
             }
             // W_h: state block h after the previous chunk's update, packed to bf16 in registers
@@ -1080,7 +1133,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     for (int b = 0; b < g.NB; ++b) {
                         const int r = b * 128 + row, m = r >> 1;
                         float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + r) * D : nullptr;
-                        const float2 f = (m < M) ? abs_phase((long long)m * (g.L - 1), a.w, a.tint) : make_float2(1.f, 0.f);
+                        const float2 f =
+                            (m < M) ? abs_phase((long long)m * (g.L - 1), hph.w, hph.tint) : make_float2(1.f, 0.f);
                         state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
                     }
                 }
@@ -1176,6 +1230,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
     tc::tc_fence_after();
     const uint32_t tb = *tslot;
     tc::pdl_wait();      // p from the K pass, and the tables and states before it
+    const HeadW hph = head_w(a, bh);                      // this head's w and integer period
+    const int eby = (bh % a.H) * a.eb_rows_h, phy = (bh % a.H) * a.phi_rows_h;   // its table rows
 
     if (warp >= 8) {
         if (warp == 8) {
@@ -1196,12 +1252,12 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     if (!first && !wait_bar(&bar[VB_PH_FREE], ph_ph, ctl, a.err)) break;
                     tc::mbar_arrive_expect_tx(&bar[VB_PH_FULL], (uint32_t)(SP * RH * 2));
                     for (int kb = 0; kb < RH / 64; ++kb)
-                        tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PH_FULL], kb * 64, 0);
+                        tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PH_FULL], kb * 64, phy);
                     // EB_0 into the buffer of the previous chunk's p/G (freed once G V has read it)
                     if (!first && !wait_bar(&bar[VB_EB_FREE], ph_eb, ctl, a.err)) break;
                     tc::mbar_arrive_expect_tx(&bar[VB_EB_FULL], (uint32_t)(128 * kC * 2));
                     for (int kb = 0; kb < 2; ++kb)
-                        tc::tma_load_2d(ebuf(i) + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, c * g.RP);
+                        tc::tma_load_2d(ebuf(i) + kb * 128 * 128, &tm_eb, &bar[VB_EB_FULL], kb * 64, eby + c * g.RP);
                     if (!first && !wait_bar(&bar[VB_V_FREE], ph_v, ctl, a.err)) break;
                     tc::mbar_arrive_expect_tx(&bar[VB_V_FULL], (uint32_t)(kC * D * 2));
                     for (int db = 0; db < D / 64; ++db)
@@ -1211,11 +1267,12 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         if (!wait_bar(&bar[VB_PH_FREE], ph_ph, ctl, a.err)) break;
                         tc::mbar_arrive_expect_tx(&bar[VB_PH_FULL], (uint32_t)(SP * RH * 2));
                         for (int kb = 0; kb < RH / 64; ++kb)
-                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PH_FULL], RH + kb * 64, 0);
+                            tc::tma_load_2d(sPHI + kb * SP * 128, &tm_phi, &bar[VB_PH_FULL], RH + kb * 64, phy);
                         if (!wait_bar(&bar[VB_PH_FREE], ph_ph, ctl, a.err)) break;
                         tc::mbar_arrive_expect_tx(&bar[VB_PH_FULL], (uint32_t)(128 * kC * 2));
                         for (int kb = 0; kb < 2; ++kb)
-                            tc::tma_load_2d(sPHI + kb * 128 * 128, &tm_eb, &bar[VB_PH_FULL], kb * 64, c * g.RP + 128);
+                            tc::tma_load_2d(sPHI + kb * 128 * 128, &tm_eb, &bar[VB_PH_FULL], kb * 64,
+                                            eby + c * g.RP + 128);
                     }
                 }
             }
@@ -1326,15 +1383,16 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             uint32_t ph_states = 0;   // bit h: phase parity of STATE_DONE + h
             // first mode of this thread's range in each half, and the drain phases of this row
             const int m00 = wg * (XH / 2), m10 = RH / 2 + wg * (XH / 2);
-            RowPhases rp = row_phases(a.absolute ? 0 : (long long)c_begin * kC + row, m00, m10, NH == 2, a.w, a.tint);
-            const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, a.w, a.tint);
+            RowPhases rp = row_phases(a.absolute ? 0 : (long long)c_begin * kC + row, m00, m10, NH == 2, hph.w,
+                                      hph.tint);
+            const RowPhases rp_step = row_phases(a.absolute ? 0 : kC, m00, m10, NH == 2, hph.w, hph.tint);
             // V state in the absolute frame (see the K pass)
             if (g.NB > 1 && g.G > 1)
                 state_prefetch_row<DH>(a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + 128) * D + wg * DH, row,
                                        g.R2 - 128, D);
             for (int b = 0; b < g.NB; ++b) {
                 const float *src = (g.G > 1) ? a.win + ((((size_t)bh * g.G + seg) * 2 + 1) * g.RP + b * 128) * D : nullptr;
-                const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, a.w, a.tint);
+                const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, hph.w, hph.tint);
                 state_init_abs<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D, f.x, f.y);
             }
             // W_0 goes to the W tile once the previous chunk's O = A'_0 W_0 has read it; W_1 goes to the
@@ -1444,7 +1502,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     for (int b = 0; b < g.NB; ++b) {
                         const int r = b * 128 + row, m = r >> 1;
                         float *dst = (r < g.R2) ? a.state_out + ((size_t)bh * 2 * g.R2 + g.R2 + r) * D : nullptr;
-                        const float2 f = (m < M) ? abs_phase((long long)m * (g.L - 1), a.w, a.tint) : make_float2(1.f, 0.f);
+                        const float2 f =
+                            (m < M) ? abs_phase((long long)m * (g.L - 1), hph.w, hph.tint) : make_float2(1.f, 0.f);
                         state_pass<DH>(tb, b * D + wg * DH, row, true, f.x, f.y, false, nullptr, 0, dst, wg * DH);
                     }
                 }
@@ -1465,20 +1524,24 @@ __global__ void __launch_bounds__(kPassThreads, 1)
 
 // The period as an integer when w = 2 pi / T and T is a whole number below 2^24 (exact phase
 // reduction applies), else 0.
-static int integer_period(const OpDims &d) {
+static int integer_period(double T, double w) {
     const double kPi2 = 6.283185307179586;
-    if (d.T >= 16777216.0 || d.T != floor(d.T)) return 0;
-    if (fabs(d.w - kPi2 / d.T) > 1e-15 * kPi2 / d.T) return 0;
-    return (int)d.T;
+    if (T >= 16777216.0 || T != floor(T)) return 0;
+    if (fabs(w - kPi2 / T) > 1e-15 * kPi2 / T) return 0;
+    return (int)T;
 }
+static int integer_period(const OpDims &d) { return integer_period(d.T, d.w); }
 
 cudaError_t build_bf16_tables(const OpDims &d, int RP, int SP, bf16 *eb, bf16 *phi, cudaStream_t st) {
-    long long total = (long long)(RP / 2) * (kC / 8) + (long long)SP * d.R2;
+    long long total = (long long)(RP / 2) * (kC / 8) + (long long)SP * d.R2 + 1;
     int blocks = (int)((total + 255) / 256);
     if (blocks > 2048) blocks = 2048;
+    HeadPeriods hp;
+    hp.n = 0;
+    HeadTint ht;
     ProfScope ps(BLA_K_TABLES_BF16, st);
-    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, 1, d.T, d.w, integer_period(d), d.absolute ? -1.f : 1.f,
-                                          eb, phi, nullptr, nullptr);
+    k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, 1, hp, ht, d.T, d.w, integer_period(d),
+                                          d.absolute ? -1.f : 1.f, eb, phi, nullptr, nullptr, nullptr, nullptr);
     return cudaGetLastError();
 }
 
@@ -1608,14 +1671,23 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     bf16 *eb = reinterpret_cast<bf16 *>(ws + wl.eb), *phi = reinterpret_cast<bf16 *>(ws + wl.phi);
     bf16 *fseg = g.G > 1 ? reinterpret_cast<bf16 *>(ws + wl.fseg) : nullptr;
     int *delta = reinterpret_cast<int *>(ws + wl.delta);
+    double *hw = d.periods ? reinterpret_cast<double *>(ws + wl.hw) : nullptr;
+    int *htint = d.periods ? reinterpret_cast<int *>(ws + wl.htint) : nullptr;
+    // per-head periods: every head's (T_h, w_h) and integer period; nh tables
+    HeadPeriods hp;
+    head_periods(d, d.omega_in, &hp);
+    HeadTint ht;
+    for (int h = 0; h < hp.n; ++h) ht.t[h] = integer_period(hp.T[h], hp.w[h]);
+    const int nh = hp.n > 0 ? hp.n : 1;
     {
         // EB of every chunk (absolute phases), PHI, FSEG and the slot lags in one launch
-        const long long total = (long long)g.nchunks * (g.RP / 2) * (kC / 8) + (long long)g.SP * g.R2 +
-                                (fseg ? (long long)(g.RP / 2) * ((g.Lseg + 7) / 8) : 0) + g.S;
+        const long long total = nh * ((long long)g.nchunks * (g.RP / 2) * (kC / 8) + (long long)g.SP * g.R2 +
+                                      (fseg ? (long long)(g.RP / 2) * ((g.Lseg + 7) / 8) : 0) + g.S + 1);
         const int blocks = (int)(total < 4096 * 256 ? (total + 255) / 256 : 4096);
         ProfScope ps(BLA_K_TABLES_BF16, st);
-        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, g.nchunks, d.T, d.w, integer_period(d),
-                                              d.absolute ? -1.f : 1.f, eb, phi, fseg, delta);
+        k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, g.nchunks, hp, ht, d.T, d.w,
+                                              integer_period(d), d.absolute ? -1.f : 1.f, eb, phi, fseg, delta, hw,
+                                              htint);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     Args a;
@@ -1633,6 +1705,13 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     a.tint = integer_period(d);
     a.absolute = d.absolute;
     a.err = device_error_word();
+    a.H = d.H;
+    a.eb_rows_h = hp.n > 0 ? g.nchunks * g.RP : 0;
+    a.phi_rows_h = hp.n > 0 ? g.SP : 0;
+    a.f_rows_h = hp.n > 0 ? g.RP : 0;
+    a.delta_h = hp.n > 0 ? g.S : 0;
+    a.hw = hw;
+    a.htint = htint;
 
     // tensor maps
     CUtensorMap tq, tk, tv, tp, teb, tphi, tf;
@@ -1642,9 +1721,9 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     const uint32_t bx[3] = {64, 64, 1};
     const uint64_t dp[3] = {(uint64_t)g.SP, (uint64_t)g.L, (uint64_t)g.BH};
     const uint64_t sp[2] = {(uint64_t)g.SP * 2, (uint64_t)g.L * g.SP * 2};
-    const uint64_t deb[2] = {(uint64_t)kC, (uint64_t)g.nchunks * g.RP}, seb[1] = {(uint64_t)kC * 2};
+    const uint64_t deb[2] = {(uint64_t)kC, (uint64_t)nh * g.nchunks * g.RP}, seb[1] = {(uint64_t)kC * 2};
     const uint32_t beb[2] = {64, 128};
-    const uint64_t dph[2] = {(uint64_t)g.R2, (uint64_t)g.SP}, sph[1] = {(uint64_t)g.R2 * 2};
+    const uint64_t dph[2] = {(uint64_t)g.R2, (uint64_t)nh * g.SP}, sph[1] = {(uint64_t)g.R2 * 2};
     const uint32_t bph[2] = {64, (uint32_t)g.SP};
     if (!make_tmap_bf16(&tq, q, 3, dq, sq, bq) || !make_tmap_bf16(&tp, a.pbuf, 3, dp, sp, bq) ||
         !make_tmap_bf16(&teb, eb, 2, deb, seb, beb) || !make_tmap_bf16(&tphi, phi, 2, dph, sph, bph))
@@ -1653,7 +1732,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     if (g.G > 1) {
         // prepass uses half-chunk boxes (64 rows) for K and V
         if (!make_tmap_bf16(&tk, k, 3, dq, sq, bx) || !make_tmap_bf16(&tv, v, 3, dq, sq, bx)) return cudaErrorInvalidValue;
-        const uint64_t df[2] = {(uint64_t)g.Lseg, (uint64_t)g.RP}, sf[1] = {(uint64_t)g.Lseg * 2};
+        const uint64_t df[2] = {(uint64_t)g.Lseg, (uint64_t)nh * g.RP}, sf[1] = {(uint64_t)g.Lseg * 2};
         const uint32_t bf[2] = {64, 128};
         if (!make_tmap_bf16(&tf, fseg, 2, df, sf, bf)) return cudaErrorInvalidValue;
         const size_t stage_bytes = (size_t)g.NB * 128 * 64 * 2 + 2 * (size_t)64 * g.D * 2;

@@ -217,17 +217,17 @@ def test_per_head_periods_checked_on_host(lib):
     assert fwd(params([16.0, float("nan")])) == bla.BLA_ERR_INVALID
     assert fwd(params([16.0, 3.0], S=8, M=2)) == bla.BLA_ERR_INVALID          # S above one head's period
     assert fwd(params([16.0] * 257)) == bla.BLA_ERR_UNSUPPORTED
-    assert fwd(params([16.0, 32.0], dtype=bla.BLA_BF16, d_k=64, d_v=64)) == bla.BLA_ERR_UNSUPPORTED
     p = params([16.0, 32.0])
     assert lib.bla_backward(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30,
                             None) == bla.BLA_ERR_UNSUPPORTED
-    assert lib.bla_decode_step_noalloc(ctypes.byref(p), 0, FAKE, FAKE, FAKE, FAKE, FAKE, None) == \
-        bla.BLA_ERR_UNSUPPORTED
-    assert lib.bla_forward_chunked_host(ctypes.byref(p), FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 30, None) == \
-        bla.BLA_ERR_UNSUPPORTED
-    # the tables repeat per head, so the workspace grows with H
+    # the tables repeat per head, so the workspace grows with H (decode, and the bf16 forward's
+    # per-chunk EB tables)
     shared = lib.bla_workspace_bytes(ctypes.byref(_params(H=2)), bla.BLA_WS_DECODE)
     assert lib.bla_workspace_bytes(ctypes.byref(p), bla.BLA_WS_DECODE) > shared
+    kw = dict(dtype=bla.BLA_BF16, d_k=64, d_v=64, M=32, S=32, L=4096)
+    shared = lib.bla_workspace_bytes(ctypes.byref(_params(H=2, window=256.0, **kw)), bla.BLA_WS_FORWARD)
+    per = lib.bla_workspace_bytes(ctypes.byref(params([256.0, 300.0], window=300.0, **kw)), bla.BLA_WS_FORWARD)
+    assert per >= shared + 32 * 64 * 128 * 2      # a second copy of the 32 chunks' EB tables
     assert bla.make_params(1, 2, 8, 32, 32, 4, 4, [9.0, 20.0]).periods[1] == 20.0
     with pytest.raises(bla.BlaError):
         bla.make_params(1, 3, 8, 32, 32, 4, 4, [9.0, 20.0])

@@ -1,10 +1,10 @@
 """Per-head periods (Alg. 1 and Alg. 3 take T in R^H) on the paths with per-head tables: the fp32
-forward, the decode step and the state-decay entry points, against the oracle run at each head's
-own period."""
+forward, the bf16 tensor-core forward (device and host buffers), both decode entry points and the
+state-decay entry points, against the oracle run at each head's own period."""
 import numpy as np
 import pytest
 
-from gpu_util import TOL_BF16, TOL_F32, rel, require_cuda, to_dev
+from gpu_util import TOL_BF16, TOL_F32, lse_bound, rel, require_cuda, row_errors, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -103,3 +103,80 @@ def test_decay_backward(orc):
     ref = orc.backward_decay(q, k, v, do, M, S, TS)
     for name, a, b in zip(("dq", "dk", "dv"), got, ref):
         assert rel(a.cpu().numpy(), b) <= 1e-4, (name, rel(a.cpu().numpy(), b))
+
+
+@pytest.mark.parametrize("B,H,L,d,M,S,TH,phase_mode", [
+    # 2M = 64: an integer, a clamped (T < 2M-1) and a fractional period (fp64 phases)
+    (2, 3, 700, 64, 32, 32, [256.0, 40.0, 1000.5], "lag"),
+    (2, 3, 700, 64, 32, 32, [256.0, 40.0, 1000.5], "absolute"),
+    # 2M = 256 (two mode halves), one-chunk segments: per-head FSEG tables in the prepass and scan
+    (1, 2, 3000, 128, 128, 128, [4096.0, 1500.0], "lag"),
+    # 2M = 128 with S = 64, ragged tail, three heads of one batch element each
+    (3, 2, 333, 128, 64, 64, [1024.0, 200.0], "lag"),
+])
+def test_bf16_forward(orc, B, H, L, d, M, S, TH, phase_mode):
+    """The tensor-core passes with one EB, PHI, FSEG and slot-lag table per head, against the oracle."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=L + H)
+    o, lse, st = bla.bla_forward_chunked(*(to_dev(x, dev, torch.bfloat16) for x in (q, k, v)), M, S, TH,
+                                         want_state=True, phase_mode=phase_mode)
+    bla.bla_device_error()
+    form = "modes" if phase_mode == "lag" else "absolute"
+    ref = orc.forward(q, k, v, M, S, TH, form=form)
+    pooled, worst = row_errors(o.float().cpu().numpy(), ref["o"])
+    assert pooled <= TOL_BF16 and worst <= TOL_BF16, (pooled, worst)
+    lse = lse.cpu().numpy()
+    assert np.all(np.abs(lse - ref["lse"]) <= lse_bound(ref["lse"])), np.abs(lse - ref["lse"]).max()
+    st_ref = orc.forward(q, k, v, M, S, TH, form="modes", return_state=True)["state"]
+    assert rel(st.cpu().numpy(), st_ref) <= TOL_BF16
+    # each head alone at its own scalar period gives the same result (tables indexed per head)
+    for h in range(H):
+        oh = bla.bla_forward_chunked(*(to_dev(x[:, h:h + 1], dev, torch.bfloat16) for x in (q, k, v)), M, S, TH[h],
+                                     phase_mode=phase_mode)[0]
+        assert rel(oh.float().cpu().numpy(), o[:, h:h + 1].float().cpu().numpy()) <= 1e-2
+
+
+def test_bf16_host_buffer_forward_groups_cross_batches(orc):
+    """B=3, H=5, L=12000, d=128 (184 MB: two pipelined head groups that split a batch element) with one
+    period per head: equals the device-buffer forward, whose heads the oracle checks above."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_qkv
+    dev = require_cuda()
+    TH = [1024.0, 300.0, 700.0, 2048.0, 129.0]
+    q, k, v = make_qkv(3, 5, 12000, 128, dtype="bf16", seed=31)
+    hq, hk, hv = (torch.from_numpy(x).to(torch.bfloat16).pin_memory() for x in (q, k, v))
+    o_host = bla.bla_forward_chunked_host(hq, hk, hv, 64, 64, TH)
+    torch.cuda.synchronize()
+    bla.bla_device_error()
+    o_dev = bla.bla_forward_chunked(hq.to(dev), hk.to(dev), hv.to(dev), 64, 64, TH)[0].cpu()
+    assert rel(o_host.float().numpy(), o_dev.float().numpy()) <= 1e-2
+    want = np.zeros(12000, bool)
+    want[::101] = True
+    want[-2:] = True
+    ref = orc.forward(q[1:2], k[1:2], v[1:2], 64, 64, TH, form="modes", want=want)
+    got = o_host.float().numpy()[1:2]
+    assert rel(got[:, :, want], ref["o"][:, :, want]) <= TOL_BF16
+
+
+def test_noalloc_decode_matches_workspace_decode():
+    """The no-alloc decode builds every head's tables in its fixed scratch and matches bla_decode_step."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_decode_step, make_state
+    dev = require_cuda()
+    B, H, d, M, S = 4, 3, 128, 32, 32
+    TH = [64.0, 256.0, 1000.5]
+    st0 = torch.from_numpy(make_state(B, H, M, d, std=0.1, seed=7)).to(dev)
+    sa, sb = st0.clone(), st0.clone()
+    for step in range(3):
+        q, k, v = (to_dev(x, dev, torch.bfloat16) for x in make_decode_step(step, B, H, d, "bf16", seed=7))
+        oa = bla.bla_decode_step(q, k, v, sa, 1100 + step, M, S, TH)
+        ob = bla.bla_decode_step_noalloc(q, k, v, sb, 1100 + step, M, S, TH)
+        torch.cuda.synchronize()
+        assert rel(ob.float().cpu().numpy(), oa.float().cpu().numpy()) <= 1e-6
+    assert rel(sb.cpu().numpy(), sa.cpu().numpy()) <= 1e-6
+    bla.bla_device_error()
