@@ -54,6 +54,50 @@ def test_bf16_forward(orc, B, H, L, d, M, S, T):
           TOL_BF16, 5e-2)
 
 
+@pytest.mark.parametrize("B,H,L,d,M,S,T", [
+    (1, 2, 500, 64, 17, 32, 33.0),      # T = 2M-1: the decay factors reach exact zeros
+    (16, 10, 130, 64, 32, 32, 256.0),   # 160 heads: one segment per head
+    (1, 1, 1000, 128, 64, 64, 1024.0),  # 16 one-chunk segments
+    (2, 1, 63, 128, 32, 64, 512.0),     # one ragged chunk
+])
+def test_bf16_chunked_forward(orc, B, H, L, d, M, S, T):
+    """The chunked tensor-core form (d in {64, 128}, S in {32, 64}): o per row, lse and state."""
+    from paper_2606_09862_gb300.inputs import make_qkv
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=L + S)
+    o, lse, st = gpu_forward(q, k, v, M, S, T, "bf16")
+    ref = orc.forward_decay(q, k, v, M, S, T, return_state=True)
+    pooled, worst = row_errors(o, ref["o"])
+    assert pooled <= TOL_BF16 and worst <= TOL_ROW_BF16, (pooled, worst)
+    assert np.abs(lse - ref["lse"]).max() <= 5e-2
+    assert rel(st, ref["state"]) <= TOL_BF16, rel(st, ref["state"])
+
+
+def test_bf16_chunked_continues_from_state(orc):
+    """A chunked forward from a random slot state at pos0 = 777 (mid-chunk phases, every slot visible
+    from the start) equals the oracle continued from the same state; and a prefill split in two
+    calls equals one call."""
+    from paper_2606_09862_gb300.inputs import make_qkv, make_slot_state
+    B, H, L, d, M, S, T = 2, 2, 300, 64, 16, 32, 100.0
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=19)
+    st0 = make_slot_state(B, H, S, d, 0.1, seed=19)
+    got = gpu_forward(q, k, v, M, S, T, "bf16", pos0=777, state=st0)
+    check(got, orc.forward_decay(q, k, v, M, S, T, state=st0, pos0=777, return_state=True), TOL_BF16, 5e-2)
+    full = orc.forward_decay(q, k, v, M, S, T, return_state=True)
+    o1, _, st1 = gpu_forward(q[:, :, :130], k[:, :, :130], v[:, :, :130], M, S, T, "bf16")
+    o2, _, st2 = gpu_forward(q[:, :, 130:], k[:, :, 130:], v[:, :, 130:], M, S, T, "bf16", pos0=130, state=st1)
+    assert rel(np.concatenate([o1, o2], 2), full["o"]) <= TOL_BF16
+    assert rel(st2, full["state"]) <= TOL_BF16
+
+
+def test_bf16_chunked_per_head_periods(orc):
+    """Per-head periods on the chunked form: one D_M table and grid per head."""
+    from paper_2606_09862_gb300.inputs import make_qkv
+    TH = [33.0, 256.0, 1000.5]
+    q, k, v = make_qkv(2, 3, 200, 64, dtype="bf16", seed=23)
+    check(gpu_forward(q, k, v, 17, 32, TH, "bf16"), orc.forward_decay(q, k, v, 17, 32, TH, return_state=True),
+          TOL_BF16, 5e-2)
+
+
 def test_bf16_sharp_softmax(orc):
     from paper_2606_09862_gb300.inputs import make_qkv
     q, k, v = make_qkv(1, 2, 400, 128, dtype="bf16", seed=3, sharp=True)
