@@ -110,19 +110,24 @@ struct DcLayout {
     static constexpr int kst = v1 + kTile;                  // bf16 [S][D]: K~ at the chunk start
     static constexpr int vst = kst + S * D * 2;             // bf16 [S][D]: V~ at the chunk start
     static constexpr int wend = vst + S * D * 2;            // bf16 [S][64]: Wend
-    static constexpr int pa = wend + S * 128;               // bf16 [64][64]: p o A (columns >= S zero)
+    static constexpr int beta = wend + S * 128;             // bf16 [S][64]: beta_j(u)
+    static constexpr int pa = beta + S * 128;               // bf16 [64][64]: p o A (columns >= S zero)
     static constexpr int gm = pa + kDC * 128;               // bf16 [64][64]: G (upper triangle zero)
     static constexpr int pf = gm + kDC * 128;               // fp32 [64][kFS]: P; then bf16 [64][D]: O
     static constexpr int yf = pf + kDC * kFS * 4;           // fp32 [64][kFS]: Y, s, then p
     static constexpr int df = yf + kDC * kFS * 4;           // fp32 [64][kFS]: D_j(t0 + u)
-    static constexpr int af = df + kDC * kFS * 4;           // fp32 [64][kFS]: A_j(tau)
-    static constexpr int aend = af + kDC * kFS * 4;         // fp32 [S]: A_j(63)
+    static constexpr int af = df + kDC * kFS * 4;           // fp32 [64][kFS]: alpha_j(tau)
+    static constexpr int g4 = af + kDC * kFS * 4;           // fp32 [4][S]: sub-block products g_j(B)
+    static constexpr int gpre = g4 + 4 * S * 4;             // fp32 [4][S]: prod_{B' < B} g_j(B')
+    static constexpr int aend = gpre + 4 * S * 4;           // fp32 [S]: A_j(63)
     static constexpr int delta = aend + S * 4;              // int [S]
     static constexpr int tot = delta + S * 4;               // fp32 [kDThreads / S][S]: segment products
     static constexpr int bars = tot + kDThreads * 4;        // 3 mbarriers (q, kv stage 0, kv stage 1)
     static constexpr int total = bars + 64;
-    static_assert(pf % 1024 == 0 && kst % 1024 == 0 && wend % 1024 == 0 && pa % 1024 == 0 && gm % 1024 == 0,
+    static_assert(pf % 1024 == 0 && kst % 1024 == 0 && wend % 1024 == 0 && beta % 1024 == 0 && pa % 1024 == 0 &&
+                      gm % 1024 == 0,
                   "swizzled tiles need 1024-byte alignment");
+    static_assert(total <= 227 * 1024, "shared memory of one CTA");
     static_assert(kDC * D * 2 <= kDC * kFS * 4, "the O tile reuses the P tile");
 };
 
@@ -168,15 +173,18 @@ __global__ void __launch_bounds__(kDThreads, 1)
     const bool outputs = a.mode == 1;
 
     uint8_t *sQ = dsm + Lay::q, *sKst = dsm + Lay::kst, *sVst = dsm + Lay::vst, *sW = dsm + Lay::wend;
+    uint8_t *sBeta = dsm + Lay::beta;
     uint8_t *sPA = dsm + Lay::pa, *sGm = dsm + Lay::gm, *sO = dsm + Lay::pf;
     float *sP = reinterpret_cast<float *>(dsm + Lay::pf), *sY = reinterpret_cast<float *>(dsm + Lay::yf);
-    float *sD = reinterpret_cast<float *>(dsm + Lay::df), *sA = reinterpret_cast<float *>(dsm + Lay::af);
+    float *sD = reinterpret_cast<float *>(dsm + Lay::df), *sAl = reinterpret_cast<float *>(dsm + Lay::af);
+    float *sG4 = reinterpret_cast<float *>(dsm + Lay::g4), *sGpre = reinterpret_cast<float *>(dsm + Lay::gpre);
     float *sAend = reinterpret_cast<float *>(dsm + Lay::aend);
     int *sdelta = reinterpret_cast<int *>(dsm + Lay::delta);
     float *sTot = reinterpret_cast<float *>(dsm + Lay::tot);
     uint64_t *bar = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
     const uint32_t uQ = tc::smem_u32(sQ), uKst = tc::smem_u32(sKst), uVst = tc::smem_u32(sVst);
     const uint32_t uW = tc::smem_u32(sW), uPA = tc::smem_u32(sPA), uGm = tc::smem_u32(sGm);
+    const uint32_t uBeta = tc::smem_u32(sBeta);
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
@@ -267,9 +275,13 @@ __global__ void __launch_bounds__(kDThreads, 1)
         const int t0 = c * kDC, n = min(kDC, a.L - t0), s = (c - c_begin) & 1;
         const uint8_t *sK = dsm + (s ? Lay::k1 : Lay::k0), *sV = dsm + (s ? Lay::v1 : Lay::v0);
         const uint32_t uK = tc::smem_u32(sK), uV = tc::smem_u32(sV);
-        // ---- D_j(t0 + u) (0 past the end of the sequence: those steps leave the state as it is), the
-        // prefix products A_j(tau) and Wend[j][u] = D_j(u) prod_{x > u} a_j(x): each thread's run of UPS
-        // tokens forms its local products; the runs' totals combine through shared memory
+        // ---- D_j(t0 + u) (0 past the end of the sequence: those steps leave the state as it is) and the
+        // products built from a_j = 1 - D_j, per 16-token sub-block B of the chunk:
+        //   alpha_j(tau) = prod_{B start <= x <= tau} a_j,   beta_j(u) = D_j(u) prod_{u < x <= B end} a_j,
+        //   g_j(B) = prod_{x in B} a_j,   Gpre_j(B) = prod_{B' < B} g_j(B')   (A_j(tau) = Gpre_j alpha_j),
+        //   Wend[j][u] = D_j(u) prod_{x > u} a_j.
+        // Each thread's run of UPS tokens forms its local products; the runs' totals combine through
+        // shared memory.
         {
             float pf[UPS], tot = 1.f;
 #pragma unroll
@@ -279,27 +291,43 @@ __global__ void __launch_bounds__(kDThreads, 1)
                 pf[i] = tot;
             }
             sTot[trun * S + tj] = tot;
+            if (threadIdx.x == 0) tc::bulk_wait_read0();   // the last chunk's o has left the P tile
             __syncthreads();
-            float pre = 1.f, suf = 1.f;
+            constexpr int RPB = 16 / UPS;   // runs per sub-block
+            const int rb0 = (trun / RPB) * RPB;
+            float pre = 1.f, suf = 1.f, pre_b = 1.f, suf_b = 1.f;
             for (int r2 = 0; r2 < NRUN; ++r2) {
                 const float x = sTot[r2 * S + tj];
-                if (r2 < trun) pre *= x;
-                else if (r2 > trun) suf *= x;
+                if (r2 < trun) {
+                    pre *= x;
+                    if (r2 >= rb0) pre_b *= x;
+                } else if (r2 > trun) {
+                    suf *= x;
+                    if (r2 < rb0 + RPB) suf_b *= x;
+                }
             }
 #pragma unroll
-            for (int i = 0; i < UPS; ++i) sA[(tu0 + i) * kFS + tj] = pre * pf[i];
+            for (int i = 0; i < UPS; ++i) sAl[(tu0 + i) * kFS + tj] = pre_b * pf[i];
+            if (trun == rb0) {
+                // this sub-block's product and the product of the sub-blocks before it
+                float gb = tot;
+                for (int r2 = trun + 1; r2 < rb0 + RPB; ++r2) gb *= sTot[r2 * S + tj];
+                sG4[(trun / RPB) * S + tj] = gb;
+                sGpre[(trun / RPB) * S + tj] = pre;
+            }
             if (trun == NRUN - 1) {
                 sAend[tj] = pre * tot;
                 seg_dec *= pre * tot;
             }
-            float r = suf;   // prod of a over the tokens after this one, to the end of the chunk
+            float r = 1.f;   // prod of a over this run's tokens after the current one
 #pragma unroll
             for (int i = UPS - 1; i >= 1; i -= 2) {
                 const float w1 = dl[i] * r;
                 r -= r * dl[i];
                 const float w0 = dl[i - 1] * r;
                 r -= r * dl[i - 1];
-                st_bf16x2(sW, S, tj, tu0 + i - 1, w0, w1);
+                st_bf16x2(sW, S, tj, tu0 + i - 1, w0 * suf, w1 * suf);
+                st_bf16x2(sBeta, S, tj, tu0 + i - 1, w0 * suf_b, w1 * suf_b);
             }
         }
         if (c + 1 < c_end) load_d(c + 1);
@@ -309,43 +337,78 @@ __global__ void __launch_bounds__(kDThreads, 1)
             ph_q ^= 1;
             if (!tc::mbar_wait(&bar[1 + s], ph_kv[s] & 1)) { report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (16 << 4)); ok = false; }
             if (!ok) break;
+            // warp (sub-block bt, 16 columns): P's block, and Y's block where the columns are slots; the
+            // two share Q's fragments.  Y = Q K~^T stays in registers until P is complete.
+            const int bt = warp >> 2, yn0 = (warp & 3) * 16, ym0 = bt * 16;
+            const bool has_y = (warp & 3) < SB;
+            float yacc[2][4] = {};
             {
-                const int m0 = (warp >> 2) * 16, n0 = (warp & 3) * 16;
                 float acc[2][4] = {};
-                mma_block<true>(uQ, kDC, uK, kDC, m0, n0, D, acc);
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int col = n0 + h * 8 + 2 * t4;
-                    *reinterpret_cast<float2 *>(&sP[(m0 + g8) * kFS + col]) = make_float2(acc[h][0], acc[h][1]);
-                    *reinterpret_cast<float2 *>(&sP[(m0 + g8 + 8) * kFS + col]) = make_float2(acc[h][2], acc[h][3]);
+                for (int k0 = 0; k0 < D; k0 += 16) {
+                    uint32_t af[4], b[4];
+                    load_a(uQ, kDC, ym0, k0, af);
+                    load_b_nk(uK, kDC, yn0, k0, b);
+                    mma16816(acc[0], af, b[0], b[1]);
+                    mma16816(acc[1], af, b[2], b[3]);
+                    if (has_y) {
+                        load_b_nk(uKst, S, yn0, k0, b);
+                        mma16816(yacc[0], af, b[0], b[1]);
+                        mma16816(yacc[1], af, b[2], b[3]);
+                    }
                 }
-            }
-            if (warp < 4 * SB) {
-                const int m0 = (warp / SB) * 16, n0 = (warp % SB) * 16;
-                float acc[2][4] = {};
-                mma_block<true>(uQ, kDC, uKst, S, m0, n0, D, acc);
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
-                    const int col = n0 + h * 8 + 2 * t4;
-                    *reinterpret_cast<float2 *>(&sY[(m0 + g8) * kFS + col]) = make_float2(acc[h][0], acc[h][1]);
-                    *reinterpret_cast<float2 *>(&sY[(m0 + g8 + 8) * kFS + col]) = make_float2(acc[h][2], acc[h][3]);
+                    const int col = yn0 + h * 8 + 2 * t4;
+                    *reinterpret_cast<float2 *>(&sP[(ym0 + g8) * kFS + col]) = make_float2(acc[h][0], acc[h][1]);
+                    *reinterpret_cast<float2 *>(&sP[(ym0 + g8 + 8) * kFS + col]) = make_float2(acc[h][2], acc[h][3]);
                 }
             }
             __syncthreads();
             // the next chunk's q may load now (its tile has been read)
             if (threadIdx.x == 0 && c + 1 < c_end) issue_q(c + 1);
-            // ---- s[tau, j] = scale (A_j(tau) Y[tau, j] + sum_{u <= tau} P[tau, u] D_j(u) r_j(tau, u)):
-            // thread (pair pi, slot group sg) takes rows pi and 63 - pi (65 steps together) and SPT slots
-            const int sg = threadIdx.x & 15, pi = threadIdx.x >> 4;
+            // ---- s[tau, j] = scale (A_j(tau) Y[tau, j] + sum_{u <= tau} P[tau, u] W_j(tau, u)).  For u in a
+            // sub-block B_u before tau's, W = alpha_j(tau) gamma_j beta_j(u), gamma_j the product of g_j over
+            // the sub-blocks between, so those terms are alpha_j(tau) F with
+            //   F = sum_{B_u < B_tau} gamma_j P_blk beta_blk   (Horner over B_u: F <- g_j(B_u) F + P_blk beta_blk)
+            // on the tensor cores; with A = Gpre alpha the warp leaves alpha (Gpre Y + F) in sY.
+            if (has_y) {
+                float facc[2][4] = {};
+                for (int kb = 0; kb < bt; ++kb) {
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const float2 gk = *reinterpret_cast<const float2 *>(&sG4[kb * S + yn0 + h * 8 + 2 * t4]);
+                        facc[h][0] *= gk.x; facc[h][1] *= gk.y; facc[h][2] *= gk.x; facc[h][3] *= gk.y;
+                    }
+                    const float *p0 = sP + (ym0 + g8) * kFS + kb * 16 + 2 * t4, *p1 = p0 + 8 * kFS;
+                    const uint32_t af[4] = {tc::pack_bf16x2(p0[0], p0[1]), tc::pack_bf16x2(p1[0], p1[1]),
+                                            tc::pack_bf16x2(p0[8], p0[9]), tc::pack_bf16x2(p1[8], p1[9])};
+                    uint32_t b[4];
+                    load_b_nk(uBeta, S, yn0, kb * 16, b);
+                    mma16816(facc[0], af, b[0], b[1]);
+                    mma16816(facc[1], af, b[2], b[3]);
+                }
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int row = ym0 + g8 + ((q >> 1) << 3), j = yn0 + h * 8 + 2 * t4 + (q & 1);
+                        sY[row * kFS + j] = sAl[row * kFS + j] * fmaf(sGpre[bt * S + j], yacc[h][q], facc[h][q]);
+                    }
+            }
+            __syncthreads();
+            // ---- the diagonal sub-blocks on the CUDA cores: thread (pair ip of sub-block sb, slot group sg)
+            // walks rows 16 sb + ip and 16 sb + 15 - ip (17 steps together) down to the sub-block's start,
+            // with the running product r_j
+            const int sg = threadIdx.x & 15, rp = threadIdx.x >> 4, sb = rp >> 3, ip = rp & 7;
 #pragma unroll 1
             for (int rr = 0; rr < 2; ++rr) {
-                const int row = rr ? kDC - 1 - pi : pi;
+                const int row = sb * 16 + (rr ? 15 - ip : ip), lo = sb * 16;
                 float acc[SPT], r[SPT];
 #pragma unroll
                 for (int k = 0; k < SPT; ++k) { acc[k] = 0.f; r[k] = 1.f; }
                 const float *prow = sP + row * kFS;
 #pragma unroll 4
-                for (int u = row; u >= 0; --u) {
+                for (int u = row; u >= lo; --u) {
                     const float pv = prow[u];
                     float dv[SPT];
                     if constexpr (SPT == 4) {
@@ -365,7 +428,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
 #pragma unroll
                 for (int k = 0; k < SPT; ++k) {
                     const int j = sg * SPT + k;
-                    const float sc = a.scale * fmaf(sA[row * kFS + j], sY[row * kFS + j], acc[k]);
+                    const float sc = a.scale * (sY[row * kFS + j] + acc[k]);
                     sY[row * kFS + j] = (t >= sdelta[j]) ? sc : -INFINITY;
                 }
             }
@@ -397,55 +460,126 @@ __global__ void __launch_bounds__(kDThreads, 1)
                     const float p0 = v[k] * inv, p1 = v[k + 1] * inv;
                     sY[row * kFS + j] = p0;
                     sY[row * kFS + j + 1] = p1;
-                    st_bf16x2(sPA, kDC, row, j, p0 * sA[row * kFS + j], p1 * sA[row * kFS + j + 1]);
+                    const float g0 = sGpre[(row >> 4) * S + j], g1 = sGpre[(row >> 4) * S + j + 1];
+                    st_bf16x2(sPA, kDC, row, j, p0 * g0 * sAl[row * kFS + j], p1 * g1 * sAl[row * kFS + j + 1]);
                 }
                 if (sub == 0 && row < n) a.lse[(size_t)bh * a.L + t0 + row] = mx + __logf(sum);
             }
             __syncthreads();
-            // ---- G[tau, u] = sum_j p[tau, j] D_j(u) r_j(tau, u): the same walk with q_j = p_j r_j; the
-            // 16 slot groups of a row sit in one half-warp and add their partial sums by shuffles within
-            // it (the two half-warps of a warp walk rows of different lengths)
+            // ---- G[tau, u] = sum_j p[tau, j] W_j(tau, u).  Diagonal sub-blocks on the CUDA cores: the walk
+            // above with q_j = p_j r_j, the 16 slot groups of a row adding their partial sums by shuffles
+            // within their half-warp (the two half-warps of a warp walk rows of different lengths).
             const unsigned hmask = 0xffffu << (lane & 16);
 #pragma unroll 1
             for (int rr = 0; rr < 2; ++rr) {
-                const int row = rr ? kDC - 1 - pi : pi;
-                float qv[SPT];
+                const int row = sb * 16 + (rr ? 15 - ip : ip), span = row - sb * 16;   // u = row - i, i <= span
+                float qv[SPT], gp[16];
 #pragma unroll
                 for (int k = 0; k < SPT; ++k) qv[k] = sY[row * kFS + sg * SPT + k];
-#pragma unroll 4
-                for (int u = row; u >= 0; --u) {
-                    float dv[SPT];
-                    if constexpr (SPT == 4) {
-                        const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kFS + sg * 4]);
-                        dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
-                    } else {
-                        const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kFS + sg * 2]);
-                        dv[0] = d2.x; dv[1] = d2.y;
-                    }
-                    float part = 0.f;
 #pragma unroll
-                    for (int k = 0; k < SPT; ++k) {
-                        part = fmaf(qv[k], dv[k], part);
-                        qv[k] = fmaf(-qv[k], dv[k], qv[k]);
-                    }
+                for (int i = 0; i < 16; ++i) {
+                    gp[i] = 0.f;
+                    if (i <= span) {
+                        const int u = row - i;
+                        float dv[SPT];
+                        if constexpr (SPT == 4) {
+                            const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kFS + sg * 4]);
+                            dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
+                        } else {
+                            const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kFS + sg * 2]);
+                            dv[0] = d2.x; dv[1] = d2.y;
+                        }
 #pragma unroll
-                    for (int o = 8; o >= 1; o >>= 1) part += __shfl_xor_sync(hmask, part, o);
-                    if (sg == 0) *reinterpret_cast<__nv_bfloat16 *>(sGm + sw_off(kDC, row, u)) = __float2bfloat16_rn(part);
+                        for (int k = 0; k < SPT; ++k) {
+                            gp[i] = fmaf(qv[k], dv[k], gp[i]);
+                            qv[k] = fmaf(-qv[k], dv[k], qv[k]);
+                        }
+                    }
+                }
+                // transposing butterfly over the 16 slot groups: after the stage of width o a lane with bit
+                // o set holds in gp[i] the sums of entries i + o; at the end lane sg holds entry sg
+#pragma unroll
+                for (int o = 8; o >= 1; o >>= 1) {
+                    const bool up = (sg & o) != 0;
+#pragma unroll
+                    for (int i = 0; i < o; ++i) {
+                        const float send = up ? gp[i] : gp[i + o];
+                        const float mine = up ? gp[i + o] : gp[i];
+                        gp[i] = mine + __shfl_xor_sync(hmask, send, o);
+                    }
+                }
+                if (sg <= span)
+                    *reinterpret_cast<__nv_bfloat16 *>(sGm + sw_off(kDC, row, row - sg)) = __float2bfloat16_rn(gp[0]);
+            }
+            // sub-blocks B_u < B_tau on the tensor cores: G_blk = (p o alpha o gamma) beta_blk^T, the
+            // contraction running over the slots; warp w < 6 takes the pair (bt, bu) of w
+            if (warp < 6) {
+                const int gbt = 1 + (warp >= 1) + (warp >= 3), gbu = warp - gbt * (gbt - 1) / 2, m0 = gbt * 16;
+                float acc[2][4] = {};
+#pragma unroll
+                for (int kk = 0; kk < S / 16; ++kk) {
+                    float x[2][2][2];   // [row g8 / g8 + 8][column half][pair]
+#pragma unroll
+                    for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const int j = kk * 16 + ch * 8 + 2 * t4 + e;
+                            float gam = 1.f;
+                            for (int b2 = gbu + 1; b2 < gbt; ++b2) gam *= sG4[b2 * S + j];
+#pragma unroll
+                            for (int rh = 0; rh < 2; ++rh) {
+                                const int row = m0 + g8 + rh * 8;
+                                x[rh][ch][e] = sY[row * kFS + j] * sAl[row * kFS + j] * gam;
+                            }
+                        }
+                    const uint32_t af[4] = {tc::pack_bf16x2(x[0][0][0], x[0][0][1]), tc::pack_bf16x2(x[1][0][0], x[1][0][1]),
+                                            tc::pack_bf16x2(x[0][1][0], x[0][1][1]), tc::pack_bf16x2(x[1][1][0], x[1][1][1])};
+                    uint32_t b[4];
+                    load_b_kn(uBeta, S, gbu * 16, kk * 16, b);
+                    mma16816(acc[0], af, b[0], b[1]);
+                    mma16816(acc[1], af, b[2], b[3]);
+                }
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int col = gbu * 16 + h * 8 + 2 * t4;
+                    st_bf16x2(sGm, kDC, m0 + g8, col, acc[h][0], acc[h][1]);
+                    st_bf16x2(sGm, kDC, m0 + g8 + 8, col, acc[h][2], acc[h][3]);
                 }
             }
             __syncthreads();
             // ---- O = (p o A) V~ + G V_c into the O tile (over the dead P tile)
-            for (int blk = warp; blk < 4 * DB; blk += kDWarps) {
-                const int m0 = (blk / DB) * 16, n0 = (blk % DB) * 16;
-                float acc[2][4] = {};
-                mma_block<false>(uPA, kDC, uVst, S, m0, n0, S, acc);
-                mma_block<false>(uGm, kDC, uV, kDC, m0, n0, kDC, acc);
+            {
+                constexpr int ONB = D / 64;                      // 16-column blocks per warp
+                const int m0 = (warp >> 2) * 16, nb0 = (warp & 3) * ONB * 16;
+                float acc[ONB][2][4] = {};
+                for (int k0 = 0; k0 < S; k0 += 16) {
+                    uint32_t af[4], b[4];
+                    load_a(uPA, kDC, m0, k0, af);
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int col = n0 + h * 8 + 2 * t4;
-                    st_bf16x2(sO, kDC, m0 + g8, col, acc[h][0], acc[h][1]);
-                    st_bf16x2(sO, kDC, m0 + g8 + 8, col, acc[h][2], acc[h][3]);
+                    for (int nb = 0; nb < ONB; ++nb) {
+                        load_b_kn(uVst, S, nb0 + nb * 16, k0, b);
+                        mma16816(acc[nb][0], af, b[0], b[1]);
+                        mma16816(acc[nb][1], af, b[2], b[3]);
+                    }
                 }
+                for (int k0 = 0; k0 < kDC; k0 += 16) {
+                    uint32_t af[4], b[4];
+                    load_a(uGm, kDC, m0, k0, af);
+#pragma unroll
+                    for (int nb = 0; nb < ONB; ++nb) {
+                        load_b_kn(uV, kDC, nb0 + nb * 16, k0, b);
+                        mma16816(acc[nb][0], af, b[0], b[1]);
+                        mma16816(acc[nb][1], af, b[2], b[3]);
+                    }
+                }
+#pragma unroll
+                for (int nb = 0; nb < ONB; ++nb)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        const int col = nb0 + nb * 16 + h * 8 + 2 * t4;
+                        st_bf16x2(sO, kDC, m0 + g8, col, acc[nb][h][0], acc[nb][h][1]);
+                        st_bf16x2(sO, kDC, m0 + g8 + 8, col, acc[nb][h][2], acc[nb][h][3]);
+                    }
             }
         } else {
             if (!tc::mbar_wait(&bar[1 + s], ph_kv[s] & 1)) {
@@ -456,18 +590,30 @@ __global__ void __launch_bounds__(kDThreads, 1)
             __syncthreads();   // A_end and Wend of this chunk
         }
         ph_kv[s] ^= 1;
-        // ---- state update: X~ <- A_end o X~ + Wend X_c (every warp: its NU state blocks)
-#pragma unroll
-        for (int i = 0; i < NU; ++i) {
-            const int b = warp * NU + i, kv = b / (SB * DB), rem = b % (SB * DB);
-            const int j0 = (rem / DB) * 16, e0 = (rem % DB) * 16;
+        // ---- state update: X~ <- A_end o X~ + Wend X_c (every warp: its NU state blocks, which share
+        // their slot rows and so Wend's fragments)
+        {
+            const int b0 = warp * NU, kv = b0 / (SB * DB), rem0 = b0 % (SB * DB);
+            const int j0 = (rem0 / DB) * 16, e00 = (rem0 % DB) * 16;
             const float f0 = sAend[j0 + g8], f1 = sAend[j0 + g8 + 8];
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                st[i][h][0] *= f0; st[i][h][1] *= f0;
-                st[i][h][2] *= f1; st[i][h][3] *= f1;
+            for (int i = 0; i < NU; ++i)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    st[i][h][0] *= f0; st[i][h][1] *= f0;
+                    st[i][h][2] *= f1; st[i][h][3] *= f1;
+                }
+            const uint32_t ux = kv ? uV : uK;
+            for (int k0 = 0; k0 < kDC; k0 += 16) {
+                uint32_t af[4], b[4];
+                load_a(uW, S, j0, k0, af);
+#pragma unroll
+                for (int i = 0; i < NU; ++i) {
+                    load_b_kn(ux, kDC, e00 + i * 16, k0, b);
+                    mma16816(st[i][0], af, b[0], b[1]);
+                    mma16816(st[i][1], af, b[2], b[3]);
+                }
             }
-            mma_block<false>(uW, S, kv ? uV : uK, kDC, j0, e0, kDC, st[i]);
         }
         __syncthreads();   // Y and O have read the old state copy; every warp is done with this stage
         if (threadIdx.x == 0 && c + 2 < c_end) issue_kv(c + 2);
@@ -478,8 +624,7 @@ __global__ void __launch_bounds__(kDThreads, 1)
             __syncthreads();
             if (threadIdx.x == 0) {
                 for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sO + db * kDC * 128, db * 64, t0, bh);
-                tc::bulk_commit();
-                tc::bulk_wait_read0();   // the O tile is the next chunk's P tile
+                tc::bulk_commit();   // the store's read of the O tile is awaited before P is written over it
             }
         }
     }
