@@ -343,7 +343,9 @@ def forward_from_host(q_host, k_host, v_host, M, S, window, omega=0.0, scale=0.0
     bufs = {} if bufs is None else bufs
     B, H, L, dk = q_host.shape
     dv = v_host.shape[-1]
-    key = (B, H, L, dk, dv, M, S, float(window), q_host.dtype, phase_mode)
+    # every argument the workspace size may depend on (per-head periods as a tuple)
+    per = tuple(float(x) for x in window) if hasattr(window, "__len__") else float(window)
+    key = (B, H, L, dk, dv, M, S, per, float(omega), float(scale), q_host.dtype, phase_mode)
     if bufs.get("key") != key:
         p = make_params(B, H, L, dk, dv, M, S, window, omega, 0, scale, q_host.dtype, phase_mode)
         bufs["ws"] = torch.empty(max(bla_workspace_bytes(p, BLA_WS_FORWARD_HOST), 1), dtype=torch.uint8, device=dev)
