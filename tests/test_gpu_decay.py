@@ -210,6 +210,11 @@ def test_lag_form_rejected():
     ("f32", 1, 1, 50, 64, 4, 7, 7.0, 0),         # T = S = 2M-1 (sliding window)
     ("f32", 2, 1, 33, 32, 4, 5, 20.0, 9),        # later start position
     ("bf16", 1, 2, 300, 128, 64, 64, 1024.0, 0), # the LM-layer (M, S, T), shortened
+    # the chunked backward (32-token chunks, d in {64, 128}, S in {32, 64}):
+    ("bf16", 1, 2, 150, 64, 17, 32, 33.0, 0),    # T = 2M-1: exact zeros of 1 - D
+    ("bf16", 2, 1, 77, 128, 32, 64, 512.0, 45),  # ragged last chunk, later start position
+    ("bf16", 1, 1, 1000, 64, 64, 64, 1024.0, 0), # 32 chunks
+    ("bf16", 3, 1, 16, 128, 16, 32, 64.0, 0),    # half a chunk
 ])
 def test_backward_against_oracle_vjp(orc, dtype, B, H, L, d, M, S, T, pos0):
     """dq, dk, dv of the decayed forward against the oracle's VJP of Alg. 1 with decay."""
@@ -244,3 +249,23 @@ def test_empty_sequence_passes_state_through():
     assert o.shape == (1, 2, 0, 32)
     assert torch.equal(out, st0)
     assert float(zero.abs().max()) == 0.0
+
+
+def test_chunked_backward_per_head_periods(orc):
+    """The chunked backward with one period per head (one D_M table and grid per head)."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_dout, make_qkv
+    dev = require_cuda()
+    TH = [33.0, 256.0, 700.5]
+    B, H, L, d, M, S = 2, 3, 130, 64, 17, 32
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=41)
+    do = make_dout(B, H, L, d, dtype="bf16", seed=41)
+    tq, tk, tv, tdo = (to_dev(x, dev, torch.bfloat16) for x in (q, k, v, do))
+    o, lse, _ = bla.bla_decay_forward(tq, tk, tv, M, S, TH)
+    got = bla.bla_decay_backward(tq, tk, tv, o, tdo, lse, M, S, TH)
+    bla.bla_device_error()
+    ref = orc.backward_decay(q, k, v, do, M, S, TH)
+    for name, a, b in zip(("dq", "dk", "dv"), got, ref):
+        pooled, worst = row_errors(a.float().cpu().numpy(), b)
+        assert pooled <= TOL_GRAD and worst <= TOL_GRAD * 2, (name, pooled, worst)
