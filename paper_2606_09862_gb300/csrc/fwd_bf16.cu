@@ -1015,6 +1015,13 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 tc::tc_fence_after();
                 y_drain(0, colB, rp);
                 epi_arrive(&bar[KB_ACC_FREE_B]);
+                // W_0 of the next chunk (the state after this chunk's first update), stored once Q W_1^T (with
+                // one half Q W_0^T) has read the W tile: between the two Y drains, where the epilogue would
+                // otherwise wait for P EB_1^T and s_0
+                if (more) {
+                    uint32_t pk0[DH / 2];
+                    if (!w_compute(0, true, pk0) || !w_store(true, pk0)) { bad = true; break; }
+                }
                 if (NH == 2) {
                     // Y_1 from A once s_0 has read Y_0
                     if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
@@ -1022,19 +1029,9 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     tc::tc_fence_after();
                     y_drain(1, colA, rp);
                     epi_arrive(&bar[KB_ACC_FREE_A]);
+                    // W_1 of the next chunk into registers while s_1 runs
+                    if (more && !w_compute(1, true, pk1)) { bad = true; break; }
                 }
-                // W_0 of the next chunk (stored once Q W_1^T, or with one half Q W_0^T, has read the W
-                // tile) and W_1 of the next chunk into registers, while the last s MMA runs
-                if (more) {
-                    uint32_t pk0[DH / 2];
-                    if (!w_compute(0, true, pk0) || !w_store(true, pk0) || (NH == 2 && !w_compute(1, true, pk1))) {
-                        bad = true;
-                        break;
-                    }
-                }
-                // two halves: the next chunk's P (A is free once Y_1 is drained) before this chunk's
-                // softmax, so that the next chunk's X MMAs run during the softmax
-                if (NH == 2 && more && !p_drain()) { bad = true; break; }
                 // masked softmax over the S slots; the two warpgroups exchange their (max, sum) pairs once
                 constexpr bool sB = NH == 2;
                 if (sB ? !wait_bar(&bar[KB_ACC_FULL_B], ph_fullB, ctl, a.err)
@@ -1121,8 +1118,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     tc::fence_proxy_async_smem();
                     epi_arrive(&bar[KB_P_SMEM]);
                 }
-                // one half: the scores occupy A until the softmax has loaded them
-                if (NH == 1 && more && !p_drain()) { bad = true; break; }
+                // the next chunk's P once the softmax has loaded the scores (they free the next chunk's Q W_0^T
+                // at once; with one half they also occupy A until then)
+                if (more && !p_drain()) { bad = true; break; }
+
             }
             // final K state (lag frame at t = L-1) after the last chunk of the last segment
             if (!bad && seg == g.G - 1 && a.state_out && c_end > c_begin) {
