@@ -8,7 +8,7 @@
 // Given dO and the adjoints mu_K, mu_V of the states at the chunk's end (zero after the last
 // chunk: the final state is not differentiated), the chain rule gives, with PV = dO V^T and
 // YV = dO V0^T,
-//     dp = A o YV + sum_u PV o W,   delta = rowsum(dO o o),   g = scale p o (dp - delta),
+//     dp = A o YV + sum_u PV o W,   delta = sum_j p dp,   g = scale p o (dp - delta),
 //     G^ = sum_j g W,
 //     dQ = (g o A) K0 + G^ K,   dK = G^T Q + Wend^T mu_K,   dV = G^T dO + Wend^T mu_V,
 //     mu_K <- (g o A)^T Q + A_end o mu_K,   mu_V <- (p o A)^T dO + A_end o mu_V   (the previous chunk's).
@@ -35,14 +35,14 @@ using namespace wmma16;
 
 constexpr int kBC = 32;          // tokens per chunk
 constexpr int kBT = 256;         // threads (8 warps)
-constexpr int kBW = kBT / 32;
 constexpr int kBFS = kBC + 4;    // fp32 row stride of [32][32] tiles
 constexpr int kBSS = 64 + 4;     // fp32 row stride of [32][S] tiles (S <= 64)
 
 template <int D, int S>
 struct BwLayout {
     static constexpr int kTile = kBC * D * 2;          // one [32][D] bf16 tile
-    static constexpr int q = 0, k = q + kTile, v = k + kTile, dout = v + kTile, o = dout + kTile;
+    static constexpr int q = 0, k = q + kTile, v = k + kTile, dout = v + kTile;
+    static constexpr int o = dout + kTile;              // bf16 [32][D]: dK staging (dQ is staged over v)
     static constexpr int ost = o + kTile;               // bf16 [32][D]: dV staging
     static constexpr int k0 = ost + kTile;              // bf16 [S][D]: K~ entering the chunk
     static constexpr int v0 = k0 + S * D * 2;           // bf16 [S][D]: V~ entering the chunk
@@ -65,9 +65,8 @@ struct BwLayout {
     static constexpr int aend = gpre + 2 * S * 4;       // fp32 [S]
     static constexpr int tot = aend + S * 4;            // fp32 [kBT / S][S]: run products
     static constexpr int delta = tot + kBT * 4;         // int [S]
-    static constexpr int dl = delta + S * 4;            // fp32 [32]: rowsum(dO o o)
-    static constexpr int lse = dl + kBC * 4;            // fp32 [32]
-    static constexpr int bars = lse + kBC * 4;          // 2 mbarriers (forward sweep, reverse sweep)
+    static constexpr int lse = delta + S * 4;           // fp32 [32]
+    static constexpr int bars = lse + kBC * 4;          // mbarriers: forward-sweep stages 0 and 1, reverse sweep
     static constexpr int total = bars + 64;
     static_assert(k0 % 1024 == 0 && wend % 1024 == 0 && beta % 1024 == 0 && pa % 1024 == 0 && gh % 1024 == 0 &&
                       pf % 16 == 0,
@@ -105,7 +104,7 @@ template <int D, int S>
 __global__ void __launch_bounds__(kBT, 1)
     k_dchunk_bwd(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
                  const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                 const __grid_constant__ CUtensorMap tm_o, const __grid_constant__ CUtensorMap tm_st,
+                 const __grid_constant__ CUtensorMap tm_st,
                  const __grid_constant__ CUtensorMap tm_dq, const __grid_constant__ CUtensorMap tm_dk,
                  const __grid_constant__ CUtensorMap tm_dv, DbArgs a) {
     using Lay = BwLayout<D, S>;
@@ -131,7 +130,7 @@ __global__ void __launch_bounds__(kBT, 1)
     float *sG4 = reinterpret_cast<float *>(dsm + Lay::g4), *sGpre = reinterpret_cast<float *>(dsm + Lay::gpre);
     float *sAend = reinterpret_cast<float *>(dsm + Lay::aend), *sTot = reinterpret_cast<float *>(dsm + Lay::tot);
     int *sdelta = reinterpret_cast<int *>(dsm + Lay::delta);
-    float *sDl = reinterpret_cast<float *>(dsm + Lay::dl), *sLse = reinterpret_cast<float *>(dsm + Lay::lse);
+    float *sLse = reinterpret_cast<float *>(dsm + Lay::lse);
     uint64_t *bar = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
     const uint32_t uQ = tc::smem_u32(sQ), uK = tc::smem_u32(sK), uV = tc::smem_u32(sV), uDO = tc::smem_u32(sDO);
     const uint32_t uK0 = tc::smem_u32(sK0), uV0 = tc::smem_u32(sV0), uMuK = tc::smem_u32(sMuK);
@@ -141,6 +140,7 @@ __global__ void __launch_bounds__(kBT, 1)
     if (threadIdx.x == 0) {
         tc::mbar_init(&bar[0], 1);
         tc::mbar_init(&bar[1], 1);
+        tc::mbar_init(&bar[2], 1);
         tc::fence_barrier_init();
     }
     for (int j = threadIdx.x; j < S; j += kBT) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
@@ -239,19 +239,28 @@ __global__ void __launch_bounds__(kBT, 1)
         }
     };
 
-    // ================= forward sweep: the state entering every chunk, to the workspace (bf16)
-    uint32_t ph0 = 0, ph1 = 0;
+    // ================= forward sweep: the state entering every chunk, to the workspace (bf16).  k and
+    // v arrive in two stages: (k, v tiles) and (q, dO tiles), which the reverse sweep uses later.
+    uint32_t ph0 = 0, ph1 = 0, phs[2] = {0, 0};
     bool ok = true;
-    if (nch > 0) load_d(0);
-    for (int c = 0; c < nch && ok; ++c) {
-        const int t0 = c * kBC;
-        if (threadIdx.x == 0) {
-            tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(2 * Lay::kTile));
-            for (int db = 0; db < D / 64; ++db) {
-                tc::tma_load_3d(sK + db * kBC * 128, &tm_k, &bar[0], db * 64, t0, bh);
-                tc::tma_load_3d(sV + db * kBC * 128, &tm_v, &bar[0], db * 64, t0, bh);
-            }
+    auto issue_kv = [&](int c) {
+        const int st2 = c & 1, t0 = c * kBC;
+        uint8_t *kb = st2 ? sQ : sK, *vb = st2 ? sDO : sV;
+        uint64_t *b = &bar[st2 ? 2 : 0];
+        tc::mbar_arrive_expect_tx(b, (uint32_t)(2 * Lay::kTile));
+        for (int db = 0; db < D / 64; ++db) {
+            tc::tma_load_3d(kb + db * kBC * 128, &tm_k, b, db * 64, t0, bh);
+            tc::tma_load_3d(vb + db * kBC * 128, &tm_v, b, db * 64, t0, bh);
         }
+    };
+    if (nch > 0) {
+        load_d(0);
+        if (threadIdx.x == 0) issue_kv(0);
+    }
+    for (int c = 0; c < nch && ok; ++c) {
+        const int st2 = c & 1;
+        // the other stage was last read by the previous chunk (before the barrier that ended it)
+        if (threadIdx.x == 0 && c + 1 < nch) issue_kv(c + 1);
         build_tables();
         if (c + 1 < nch) load_d(c + 1);
         {
@@ -266,15 +275,16 @@ __global__ void __launch_bounds__(kBT, 1)
                         tc::pack_bf16x2(st[i][h][2], st[i][h][3]);
                 }
         }
-        if (!tc::mbar_wait(&bar[0], ph0)) {
+        if (!tc::mbar_wait(&bar[st2 ? 2 : 0], phs[st2])) {
             report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (17 << 4));
             ok = false;
             break;
         }
-        ph0 ^= 1;
-        state_update(skv ? uV : uK, uW, false);
+        phs[st2] ^= 1;
+        state_update(skv ? (st2 ? uDO : uV) : (st2 ? uQ : uK), uW, false);
         __syncthreads();   // the chunk's tiles and tables are read before the next chunk's arrive
     }
+    (void)ph0;
     if (!ok) return;
     // the states were written through the generic proxy; the reverse sweep reads them by TMA
     fence_proxy_async_global();
@@ -307,18 +317,28 @@ __global__ void __launch_bounds__(kBT, 1)
         const int t0 = c * kBC, n = min(kBC, L - t0);
         if (threadIdx.x == 0) {
             tc::bulk_wait_read0();   // the later chunk's dQ, dK, dV stores have read their staging tiles
-            tc::mbar_arrive_expect_tx(&bar[1], (uint32_t)(5 * Lay::kTile + 2 * S * D * 2));
+            tc::mbar_arrive_expect_tx(&bar[1], (uint32_t)(4 * Lay::kTile + 2 * S * D * 2));
             for (int db = 0; db < D / 64; ++db) {
                 const int x = db * 64;
                 tc::tma_load_3d(sQ + db * kBC * 128, &tm_q, &bar[1], x, t0, bh);
                 tc::tma_load_3d(sK + db * kBC * 128, &tm_k, &bar[1], x, t0, bh);
                 tc::tma_load_3d(sV + db * kBC * 128, &tm_v, &bar[1], x, t0, bh);
                 tc::tma_load_3d(sDO + db * kBC * 128, &tm_do, &bar[1], x, t0, bh);
-                tc::tma_load_3d(sO + db * kBC * 128, &tm_o, &bar[1], x, t0, bh);
                 const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
                 tc::tma_load_2d(sK0 + db * S * 128, &tm_st, &bar[1], x, srow);
                 tc::tma_load_2d(sV0 + db * S * 128, &tm_st, &bar[1], x, srow + S);
             }
+        }
+        // the chunk before this one (processed next) into L2 meanwhile
+        if (threadIdx.x == 0 && c > 0) {
+            for (int db = 0; db < D / 64; ++db) {
+                const int x = db * 64, tp = t0 - kBC;
+                tc::tma_prefetch_3d(&tm_q, x, tp, bh);
+                tc::tma_prefetch_3d(&tm_k, x, tp, bh);
+                tc::tma_prefetch_3d(&tm_v, x, tp, bh);
+                tc::tma_prefetch_3d(&tm_do, x, tp, bh);
+            }
+            tc::bulk_prefetch_l2(a.states + (((size_t)bh * nch + c - 1) * 2) * S * D, (uint32_t)(2 * S * D * 2));
         }
         if (threadIdx.x < kBC) sLse[threadIdx.x] = threadIdx.x < n ? a.lse[(size_t)bh * L + t0 + threadIdx.x] : 0.f;
         build_tables();
@@ -329,21 +349,6 @@ __global__ void __launch_bounds__(kBT, 1)
             break;
         }
         ph1 ^= 1;
-        // ---- delta = rowsum(dO o o): warp w takes rows 4w .. 4w + 3
-#pragma unroll
-        for (int rr = 0; rr < kBC / kBW; ++rr) {
-            const int row = warp * (kBC / kBW) + rr;
-            float acc = 0.f;
-#pragma unroll
-            for (int e = lane; e < D; e += 32) {
-                const uint32_t off = sw_off(kBC, row, e);
-                acc = fmaf(__bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(sDO + off)),
-                           __bfloat162float(*reinterpret_cast<const __nv_bfloat16 *>(sO + off)), acc);
-            }
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
-            if (lane == 0) sDl[row] = acc;
-        }
         // ---- (a) P = Q K^T, Y = Q K0^T (warps 0-3), PV = dO V^T, YV = dO V0^T (warps 4-7): warp takes
         // row block m0 and half hh of the columns; Y / YV stay in registers
         const int side = warp >> 2, m0 = ((warp >> 1) & 1) * 16, hh = warp & 1, bt = m0 >> 4;
@@ -406,7 +411,9 @@ __global__ void __launch_bounds__(kBT, 1)
         }
         __syncthreads();
         // ---- (c) the diagonal sub-blocks of s and dp on the CUDA cores (one walk, the same weights),
-        // then p = exp(s - lse), g = scale p (dp - delta), and p o A, g o A in bf16
+        // then p = exp(s - lse), delta = sum_j p dp (the 16 slot groups of the row add theirs by shuffles:
+        // exact for the p and dp at hand, so a row whose softmax sees one slot gets g = 0), g = scale p
+        // (dp - delta), and p o A, g o A in bf16
 #pragma unroll 1
         for (int rr = 0; rr < 2; ++rr) {
             const int row = sb * 16 + (rr ? 15 - ip : ip), lo = sb * 16;
@@ -434,16 +441,22 @@ __global__ void __launch_bounds__(kBT, 1)
             }
             const long long t = a.pos0 + t0 + row;
             const bool live = row < n;
-            const float lr = sLse[row], dr = sDl[row];
-            float pj[SPT], gj[SPT];
+            const float lr = sLse[row];
+            float pj[SPT], dpj[SPT], gj[SPT], pdp = 0.f;
 #pragma unroll
             for (int k = 0; k < SPT; ++k) {
                 const int j = sg * SPT + k;
                 const float s = a.scale * (sS[row * kBSS + j] + as[k]);
-                const float p = (live && t >= sdelta[j]) ? __expf(s - lr) : 0.f;
-                const float dp = sDP[row * kBSS + j] + ad[k];
-                pj[k] = p;
-                gj[k] = a.scale * p * (dp - dr);
+                pj[k] = (live && t >= sdelta[j]) ? __expf(s - lr) : 0.f;
+                dpj[k] = sDP[row * kBSS + j] + ad[k];
+                pdp = fmaf(pj[k], dpj[k], pdp);
+            }
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1) pdp += __shfl_xor_sync(hmask, pdp, o);
+#pragma unroll
+            for (int k = 0; k < SPT; ++k) {
+                const int j = sg * SPT + k;
+                gj[k] = a.scale * pj[k] * (dpj[k] - pdp);
                 sS[row * kBSS + j] = pj[k];
                 sDP[row * kBSS + j] = gj[k];
             }
@@ -624,9 +637,9 @@ __global__ void __launch_bounds__(kBT, 1)
 }
 
 template <int D, int S>
-cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v, const void *o,
+cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v,
                           const void *dout, void *dq, void *dk, void *dv, cudaStream_t st) {
-    CUtensorMap tq, tk, tv, tdo, to, tst, tdq, tdk, tdv;
+    CUtensorMap tq, tk, tv, tdo, tst, tdq, tdk, tdv;
     const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
     const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
     const uint32_t box[3] = {64, (uint32_t)kBC, 1};
@@ -636,7 +649,7 @@ cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const
     const uint32_t sbox[2] = {64, (uint32_t)S};
     if (!make_tmap_bf16(&tq, q, 3, dims, strides, box) || !make_tmap_bf16(&tk, k, 3, dims, strides, box) ||
         !make_tmap_bf16(&tv, v, 3, dims, strides, box) || !make_tmap_bf16(&tdo, dout, 3, dims, strides, box) ||
-        !make_tmap_bf16(&to, o, 3, dims, strides, box) || !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) ||
+        !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) ||
         !make_tmap_bf16(&tdq, dq, 3, dims, strides, box) || !make_tmap_bf16(&tdk, dk, 3, dims, strides, box) ||
         !make_tmap_bf16(&tdv, dv, 3, dims, strides, box))
         return cudaErrorInvalidValue;
@@ -644,7 +657,7 @@ cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const
     cudaError_t e = cudaFuncSetAttribute(k_dchunk_bwd<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_DECAY, st);
-    k_dchunk_bwd<D, S><<<(unsigned)((long long)d.B * d.H), kBT, smem, st>>>(tq, tk, tv, tdo, to, tst, tdq, tdk, tdv, a);
+    k_dchunk_bwd<D, S><<<(unsigned)((long long)d.B * d.H), kBT, smem, st>>>(tq, tk, tv, tdo, tst, tdq, tdk, tdv, a);
     return cudaGetLastError();
 }
 
@@ -665,10 +678,10 @@ cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, co
     a.lse = lse;
     a.states = static_cast<__nv_bfloat16 *>(states);
     a.err = device_error_word();
-    if (d.dk == 64) return d.S == 32 ? launch_dbwd_t<64, 32>(d, a, q, k, v, o, dout, dq, dk, dv, st)
-                                     : launch_dbwd_t<64, 64>(d, a, q, k, v, o, dout, dq, dk, dv, st);
-    return d.S == 32 ? launch_dbwd_t<128, 32>(d, a, q, k, v, o, dout, dq, dk, dv, st)
-                     : launch_dbwd_t<128, 64>(d, a, q, k, v, o, dout, dq, dk, dv, st);
+    if (d.dk == 64) return d.S == 32 ? launch_dbwd_t<64, 32>(d, a, q, k, v, dout, dq, dk, dv, st)
+                                     : launch_dbwd_t<64, 64>(d, a, q, k, v, dout, dq, dk, dv, st);
+    return d.S == 32 ? launch_dbwd_t<128, 32>(d, a, q, k, v, dout, dq, dk, dv, st)
+                     : launch_dbwd_t<128, 64>(d, a, q, k, v, dout, dq, dk, dv, st);
 }
 
 }  // namespace bla

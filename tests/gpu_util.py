@@ -33,7 +33,8 @@ def row_errors(a, b):
 
     The floor at the median row norm matters only for rows whose exact value vanishes (dq of the
     first token, whose softmax has one visible slot; dk of the last key): their absolute error is of
-    the size of a typical row's, so it is measured against a typical row."""
+    the size of a typical row's, so it is measured against a typical row.  Pass one head at a time
+    where heads differ in scale (per-head periods)."""
     a = np.asarray(a, dtype=np.float64)
     b = np.asarray(b, dtype=np.float64)
     d = a.shape[-1]

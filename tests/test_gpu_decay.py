@@ -170,6 +170,29 @@ def test_full_size_forward_sampled(orc):
     assert worst <= TOL_ROW_BF16, worst
 
 
+def test_full_size_backward_sampled(orc):
+    """The bench's decay workload (B=8, H=8, L=4096, d=128, M=64, S=64, T=1024, bf16): the full
+    backward in one call (the chunked form); heads (0, 0) and (7, 7) against the oracle's VJP,
+    pooled and per row."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import WORKLOADS, make_dout, make_qkv
+    dev = require_cuda()
+    w = WORKLOADS["decay_bf16_lm"]
+    q, k, v = make_qkv(w.B, w.H, w.L, w.d, dtype="bf16", seed=0)
+    do = make_dout(w.B, w.H, w.L, w.d, dtype="bf16", seed=0)
+    tq, tk, tv, tdo = (to_dev(x, dev, torch.bfloat16) for x in (q, k, v, do))
+    o, lse, _ = bla.bla_decay_forward(tq, tk, tv, w.M, w.S, w.T)
+    got = [x.float().cpu().numpy() for x in bla.bla_decay_backward(tq, tk, tv, o, tdo, lse, w.M, w.S, w.T)]
+    bla.bla_device_error()
+    for b, h in ((0, 0), (7, 7)):
+        sl = (slice(b, b + 1), slice(h, h + 1))
+        ref = orc.backward_decay(q[sl], k[sl], v[sl], do[sl], w.M, w.S, w.T)
+        for name, a, r in zip(("dq", "dk", "dv"), got, ref):
+            pooled, worst = row_errors(a[sl], r)
+            assert pooled <= TOL_GRAD and worst <= TOL_GRAD, (name, b, h, pooled, worst)
+
+
 def test_full_size_decode_sampled(orc):
     """The decay decode workload (B=256, H=16, d=128, M=128, S=128, T=4096, pos = 4096, random slot
     state) in one call; three heads against the oracle's one-token forward from the same state."""
@@ -266,6 +289,11 @@ def test_chunked_backward_per_head_periods(orc):
     got = bla.bla_decay_backward(tq, tk, tv, o, tdo, lse, M, S, TH)
     bla.bla_device_error()
     ref = orc.backward_decay(q, k, v, do, M, S, TH)
-    for name, a, b in zip(("dq", "dk", "dv"), got, ref):
-        pooled, worst = row_errors(a.float().cpu().numpy(), b)
-        assert pooled <= TOL_GRAD and worst <= TOL_GRAD * 2, (name, pooled, worst)
+    for name, a, r in zip(("dq", "dk", "dv"), got, ref):
+        a = a.float().cpu().numpy()
+        assert rel(a, r) <= TOL_GRAD, (name, rel(a, r))
+        # rows are compared within their head: heads at different periods have gradients of different sizes
+        for b in range(B):
+            for h in range(H):
+                worst = row_errors(a[b, h], r[b, h])[1]
+                assert worst <= TOL_GRAD, (name, b, h, worst)
