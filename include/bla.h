@@ -74,10 +74,9 @@ typedef struct {
                                per head (Alg. 1 and Alg. 3 take T in R^H): head h's grid, frequency
                                (2*pi/T_h unless omega > 0) and coefficients follow periods[h], each
                                clamped to max(T_h, 2M-1); S must not exceed any of them.  Read
-                               during the call only.  At most 256 heads.  Supported by the fp32
-                               and bf16 forwards (device and host buffers), both decode entry
-                               points and the state-decay entry points; bla_backward returns
-                               BLA_ERR_UNSUPPORTED. */
+                               during the call only.  At most 256 heads.  Supported by every
+                               entry point; bla_backward then runs the (batch, head) slices one
+                               after the other, each at its own period. */
 } bla_params;
 
 /* How a slot reads the past (bla_params.phase_mode).

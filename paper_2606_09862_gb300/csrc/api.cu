@@ -155,11 +155,6 @@ bla_status check_params(const bla_params *p, OpDims *d) {
     return BLA_OK;
 }
 
-// Entry points whose kernels read one shared set of tables refuse per-head periods.
-bla_status no_per_head(const OpDims &d, const char *what) {
-    if (d.periods) return fail(BLA_ERR_UNSUPPORTED, "%s does not support per-head periods yet", what);
-    return BLA_OK;
-}
 
 int f32_chunk(const bla_params *p, const OpDims &d) {
     int C = p->chunk > 0 ? p->chunk : kDefaultChunkF32;
@@ -185,6 +180,25 @@ size_t ws_forward(const bla_params *p, const OpDims &d) {
 }
 
 size_t ws_decode(const OpDims &d) { return tables_bytes(d, 0); }
+
+// One (batch, head) slice at head h's own period (per-head periods, Alg. 1 and Alg. 3: T in R^H), as a
+// problem of one head with a shared period.
+OpDims one_head(const OpDims &d, int h) {
+    HeadPeriods hp;
+    head_periods(d, d.omega_in, &hp);
+    OpDims o = d;
+    o.B = 1;
+    o.H = 1;
+    o.periods = nullptr;
+    if (hp.n > 0) {
+        o.T = hp.T[h];
+        o.w = hp.w[h];
+    }
+    return o;
+}
+
+// The backward's workspace: with per-head periods the heads run one at a time on one head's workspace.
+size_t ws_backward(const OpDims &d) { return bwd_workspace_bytes(d.periods ? one_head(d, 0) : d); }
 
 // Checks shared by the state-decay entry points (Sec. 3.3 on Alg. 1's slot state).
 bla_status check_decay(const bla_params *p, OpDims *d, bool forward) {
@@ -356,7 +370,7 @@ size_t bla_workspace_bytes(const bla_params *p, int which) {
     case BLA_WS_FORWARD: return ws_forward(p, d);
     case BLA_WS_DECODE: return ws_decode(d);
     case BLA_WS_FORWARD_HOST: return ws_forward_host(p, d);
-    case BLA_WS_BACKWARD: return bwd_workspace_bytes(d);
+    case BLA_WS_BACKWARD: return ws_backward(d);
     case BLA_WS_DECAY_FORWARD: return check_decay(p, &d, true) == BLA_OK ? decay_workspace_bytes(d, false) : 0;
     case BLA_WS_DECAY_DECODE: return check_decay(p, &d, false) == BLA_OK ? decay_workspace_bytes(d, true) : 0;
     case BLA_WS_DECAY_BACKWARD: return check_decay(p, &d, true) == BLA_OK ? decay_backward_workspace_bytes(d) : 0;
@@ -532,13 +546,30 @@ bla_status bla_backward(const bla_params *p, const void *q, const void *k, const
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(o) || !aligned16(dout) || !aligned16(lse) ||
         !aligned16(dq) || !aligned16(dk) || !aligned16(dv))
         return fail(BLA_ERR_INVALID, "tensor pointers must be 16-byte aligned");
-    if ((s = no_per_head(d, "the backward")) != BLA_OK) return s;
-    const char *why = bwd_unsupported(d);
+    const char *why = bwd_unsupported(d.periods ? one_head(d, 0) : d);
     if (why) return fail(BLA_ERR_UNSUPPORTED, "backward: %s", why);
-    size_t need = bwd_workspace_bytes(d);
-    if ((s = check_ws(workspace, ws_bytes, need)) != BLA_OK) return s;
-    cudaError_t e = bwd_run(d, q, k, v, o, dout, lse, dq, dk, dv, workspace, reinterpret_cast<cudaStream_t>(stream));
-    if (e != cudaSuccess) return cuda_fail(e, "backward");
+    if ((s = check_ws(workspace, ws_bytes, ws_backward(d))) != BLA_OK) return s;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (!d.periods) {
+        cudaError_t e = bwd_run(d, q, k, v, o, dout, lse, dq, dk, dv, workspace, st);
+        if (e != cudaSuccess) return cuda_fail(e, "backward");
+        return BLA_OK;
+    }
+    // per-head periods: every (batch, head) slice of the tensors is contiguous; run them one after the
+    // other at their own periods on the one-head workspace (stream order keeps the workspace's uses apart)
+    const size_t e_sz = d.dtype == BLA_BF16 ? 2 : 4;
+    const size_t sq = (size_t)d.L * d.dk * e_sz, sv = (size_t)d.L * d.dv * e_sz;
+    for (int b = 0; b < d.B; ++b)
+        for (int h = 0; h < d.H; ++h) {
+            const size_t i = (size_t)b * d.H + h;
+            const OpDims d1 = one_head(d, h);
+            cudaError_t e = bwd_run(d1, static_cast<const char *>(q) + i * sq, static_cast<const char *>(k) + i * sq,
+                                    static_cast<const char *>(v) + i * sv, static_cast<const char *>(o) + i * sv,
+                                    static_cast<const char *>(dout) + i * sv, lse + i * d.L,
+                                    static_cast<char *>(dq) + i * sq, static_cast<char *>(dk) + i * sq,
+                                    static_cast<char *>(dv) + i * sv, workspace, st);
+            if (e != cudaSuccess) return cuda_fail(e, "backward");
+        }
     return BLA_OK;
 }
 

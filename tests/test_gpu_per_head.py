@@ -1,10 +1,10 @@
-"""Per-head periods (Alg. 1 and Alg. 3 take T in R^H) on the paths with per-head tables: the fp32
-forward, the bf16 tensor-core forward (device and host buffers), both decode entry points and the
-state-decay entry points, against the oracle run at each head's own period."""
+"""Per-head periods (Alg. 1 and Alg. 3 take T in R^H): the fp32 forward, the bf16 tensor-core forward
+(device and host buffers) and backward, both decode entry points and the state-decay entry points,
+against the oracle run at each head's own period."""
 import numpy as np
 import pytest
 
-from gpu_util import TOL_BF16, TOL_F32, lse_bound, rel, require_cuda, row_errors, to_dev
+from gpu_util import TOL_BF16, TOL_F32, TOL_GRAD, lse_bound, rel, require_cuda, row_errors, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -180,3 +180,28 @@ def test_noalloc_decode_matches_workspace_decode():
         assert rel(ob.float().cpu().numpy(), oa.float().cpu().numpy()) <= 1e-6
     assert rel(sb.cpu().numpy(), sa.cpu().numpy()) <= 1e-6
     bla.bla_device_error()
+
+
+@pytest.mark.parametrize("phase_mode", ["lag", "absolute"])
+def test_bf16_backward(orc, phase_mode):
+    """The bf16 backward with one period per head (the heads run one at a time, each at its period),
+    against the oracle's VJP; rows compared within their head."""
+    import torch
+    from paper_2606_09862_gb300 import bla
+    from paper_2606_09862_gb300.inputs import make_dout, make_qkv
+    dev = require_cuda()
+    B, H, L, d, M, S = 2, 3, 300, 64, 32, 32
+    TH = [256.0, 40.0, 1000.5]
+    q, k, v = make_qkv(B, H, L, d, dtype="bf16", seed=51)
+    do = make_dout(B, H, L, d, dtype="bf16", seed=51)
+    tq, tk, tv, tdo = (to_dev(x, dev, torch.bfloat16) for x in (q, k, v, do))
+    o, lse, _ = bla.bla_forward_chunked(tq, tk, tv, M, S, TH, phase_mode=phase_mode)
+    got = bla.bla_backward(tq, tk, tv, o, tdo, lse, M, S, TH, phase_mode=phase_mode)
+    bla.bla_device_error()
+    ref = orc.backward(q, k, v, do, M, S, TH, form="parallel" if phase_mode == "lag" else "absolute")
+    for name, a, r in zip(("dq", "dk", "dv"), got, ref):
+        a = a.float().cpu().numpy()
+        assert rel(a, r) <= TOL_GRAD, (name, rel(a, r))
+        for b in range(B):
+            for h in range(H):
+                assert row_errors(a[b, h], r[b, h])[1] <= TOL_GRAD, (name, b, h)
