@@ -522,8 +522,8 @@ struct DecayWs {
     float *g = nullptr;    // backward: dp, then g = scale ds, [BH][S][L]
     // chunked forward (decay_chunk.cu): per-segment state deltas and decay products, entering states
     float *seg_delta = nullptr, *seg_decay = nullptr, *win = nullptr;
-    // chunked backward (decay_chunk_bwd.cu): the state entering every 32-token chunk (bf16)
-    void *states = nullptr;
+    // chunked backward (decay_chunk_bwd.cu): chunk states, adjoint contributions and tables
+    void *chunk_bwd = nullptr;
 };
 
 size_t decay_table_len(const OpDims &d) { return (size_t)d.L + (size_t)host_dmax(d) + 1; }
@@ -544,7 +544,7 @@ size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w,
     w->sc = nullptr;
     w->lse = nullptr;
     if (!decode && backward && decay_chunk_supported(d)) {
-        w->states = take(decay_chunk_bwd_state_bytes(d));
+        w->chunk_bwd = take(decay_chunk_bwd_ws_bytes(d));
     } else if (!decode && !backward && decay_chunk_supported(d)) {
         // the chunked forward keeps its scores on chip: only the segment states travel
         const size_t BH = (size_t)d.B * d.H, G = (size_t)decay_chunk_plan(d).G;
@@ -699,8 +699,8 @@ cudaError_t launch_decay_backward(const OpDims &d, long long pos0, const void *q
     cudaError_t e = table_launch(d, pos0 - dmax, (int)decay_table_len(d), 0, w, st);
     if (e != cudaSuccess) return e;
     if (decay_chunk_supported(d))
-        return launch_decay_chunk_bwd(d, pos0, dmax, w.Dx, w.delta, w.hs_dx, w.hs_delta, q, k, v, o, dout, lse, dq, dk,
-                                      dv, w.states, st);
+        return launch_decay_chunk_bwd(d, pos0, dmax, w.Dx, w.delta, w.hs_dx, w.hs_delta, q, k, v, dout, lse, dq, dk,
+                                      dv, w.chunk_bwd, st);
     return d.dtype == BLA_BF16 ? backward_run<__nv_bfloat16>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st)
                                : backward_run<float>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st);
 }

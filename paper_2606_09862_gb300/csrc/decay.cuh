@@ -26,12 +26,14 @@ cudaError_t launch_decay_chunk(const OpDims &d, long long pos0, int dmax, const 
                                int hs_dx, int hs_delta, const void *q, const void *k, const void *v, void *o,
                                float *lse, const float *state_in, float *state_out, float *seg_delta,
                                float *seg_decay, float *win, cudaStream_t st);
-// Its backward (decay_chunk_bwd.cu), for the same shapes: one CTA per head, 32-token chunks; the
-// state entering each chunk is kept in `states` (decay_chunk_bwd_state_bytes, bf16).
-size_t decay_chunk_bwd_state_bytes(const OpDims &d);
+// Its backward (decay_chunk_bwd.cu), for the same shapes, in 32-token chunks: tables, a pass for the
+// state entering every chunk, the per-chunk chains in parallel, and a reverse pass for the adjoint
+// states; the workspace (decay_chunk_bwd_ws_bytes) holds the chunk states, the chunks' adjoint
+// contributions (both bf16) and the tables.
+size_t decay_chunk_bwd_ws_bytes(const OpDims &d);
 cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, const float *Dx, const int *delta,
-                                   int hs_dx, int hs_delta, const void *q, const void *k, const void *v, const void *o,
-                                   const void *dout, const float *lse, void *dq, void *dk, void *dv, void *states,
+                                   int hs_dx, int hs_delta, const void *q, const void *k, const void *v,
+                                   const void *dout, const float *lse, void *dq, void *dk, void *dv, void *ws,
                                    cudaStream_t st);
 // Vector-Jacobian product of the decayed forward from the zero state (dq, dk, dv in the input dtype).
 size_t decay_backward_workspace_bytes(const OpDims &d);

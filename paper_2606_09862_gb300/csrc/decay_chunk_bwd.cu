@@ -14,12 +14,21 @@
 //     mu_K <- (g o A)^T Q + A_end o mu_K,   mu_V <- (p o A)^T dO + A_end o mu_V   (the previous chunk's).
 // (A numpy emulation of these lines matched the oracle's decayed VJP to 1e-15.)
 //
-// One CTA per head: a forward sweep runs the state updates alone and stores the state entering
-// every chunk (bf16); a reverse sweep then takes the chunks from last to first with mu in the
-// accumulator registers of the MMAs that update it.  As in the forward, the triangle sums (s, dp, G,
-// G^) are split at 16-token sub-blocks: the off-diagonal block is a contraction on the tensor cores
-// (W = alpha_j(tau) beta_j(u) across adjacent sub-blocks), the diagonal blocks walk u on the CUDA
-// cores.  All contractions are warp-level bf16 MMAs (m16n8k16).
+// Both recurrences are linear with a per-slot diagonal decay, so only two thin passes run along the
+// sequence; everything else runs one chunk at a time, in parallel:
+//   1. k_dbtab: Wend and A_end of every (head, chunk) from the D_M table (they depend on the
+//      period and the positions only, not on the batch);
+//   2. k_dbstate: per (head, 64-column strip of K~ or V~): K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c,
+//      the state entering every chunk stored in bf16;
+//   3. k_dbchain: one work item per (head, chunk), over persistent CTAs: s, p, dp, g, G, G^, then dQ
+//      (final), the chunk's own parts G^T Q and G^T dO of dK and dV, and its adjoint contributions
+//      Z_K = (g o A)^T Q, Z_V = (p o A)^T dO (bf16);
+//   4. k_dbadj: per (head, strip), from the last chunk back: dK += Wend^T mu_K (dV likewise), then
+//      mu <- A_end o mu + Z.
+// In the chain the triangle sums (s, dp, G, G^) are split at 16-token sub-blocks as in the forward:
+// the off-diagonal block is a contraction on the tensor cores (W = alpha_j(tau) beta_j(u) across
+// adjacent sub-blocks), the diagonal blocks walk u on the CUDA cores.  All contractions are
+// warp-level bf16 MMAs (m16n8k16).
 #include <math.h>
 
 #include "decay.cuh"
@@ -44,12 +53,9 @@ struct BwLayout {
     static constexpr int q = 0, k = q + kTile, v = k + kTile, dout = v + kTile;
     static constexpr int o = dout + kTile;              // bf16 [32][D]: dK staging (dQ is staged over v)
     static constexpr int ost = o + kTile;               // bf16 [32][D]: dV staging
-    static constexpr int k0 = ost + kTile;              // bf16 [S][D]: K~ entering the chunk
-    static constexpr int v0 = k0 + S * D * 2;           // bf16 [S][D]: V~ entering the chunk
-    static constexpr int muk = v0 + S * D * 2;          // bf16 [S][D]: adjoint of K~ at the chunk's end
-    static constexpr int muv = muk + S * D * 2;         // bf16 [S][D]: adjoint of V~
-    static constexpr int wend = muv + S * D * 2;        // bf16 [S][64] (u < 32 used): Wend
-    static constexpr int beta = wend + S * 128;         // bf16 [S][64]: beta_j(u)
+    static constexpr int k0 = ost + kTile;              // bf16 [S][D]: K~ entering the chunk, then Z_K
+    static constexpr int v0 = k0 + S * D * 2;           // bf16 [S][D]: V~ entering the chunk, then Z_V
+    static constexpr int beta = v0 + S * D * 2;         // bf16 [S][64] (u < 32 used): beta_j(u)
     static constexpr int pa = beta + S * 128;           // bf16 [32][64]: p o A
     static constexpr int ga = pa + kBC * 128;           // bf16 [32][64]: g o A
     static constexpr int gm = ga + kBC * 128;           // bf16 [32][64] (u < 32): G
@@ -62,20 +68,19 @@ struct BwLayout {
     static constexpr int af = df + kBC * kBSS * 4;      // fp32 [32][kBSS]: alpha_j(tau)
     static constexpr int g4 = af + kBC * kBSS * 4;      // fp32 [2][S]: sub-block products
     static constexpr int gpre = g4 + 2 * S * 4;         // fp32 [2][S]: product of the sub-blocks before
-    static constexpr int aend = gpre + 2 * S * 4;       // fp32 [S]
-    static constexpr int tot = aend + S * 4;            // fp32 [kBT / S][S]: run products
+    static constexpr int tot = gpre + 2 * S * 4;        // fp32 [kBT / S][S]: run products
     static constexpr int delta = tot + kBT * 4;         // int [S]
     static constexpr int lse = delta + S * 4;           // fp32 [32]
-    static constexpr int bars = lse + kBC * 4;          // mbarriers: forward-sweep stages 0 and 1, reverse sweep
+    static constexpr int bars = lse + kBC * 4;          // mbarrier: the item's tiles
     static constexpr int total = bars + 64;
-    static_assert(k0 % 1024 == 0 && wend % 1024 == 0 && beta % 1024 == 0 && pa % 1024 == 0 && gh % 1024 == 0 &&
+    static_assert(k0 % 1024 == 0 && beta % 1024 == 0 && pa % 1024 == 0 && gh % 1024 == 0 &&
                       pf % 16 == 0,
                   "swizzled tiles need 1024-byte alignment");
     static_assert(total <= 227 * 1024, "shared memory of one CTA");
 };
 
 struct DbArgs {
-    int L, H;
+    int L, H, BH;
     long long pos0;
     float scale;
     int dmax;
@@ -83,7 +88,11 @@ struct DbArgs {
     const int *delta;           // [S]
     int hs_dx, hs_delta;        // per-head strides (0: one shared period)
     const float *lse;           // [BH][L], from the forward
+    int ntab;                   // heads with their own tables (1 when the heads share one period)
+    __nv_bfloat16 *wtab;        // [ntab][nch][S][64] bf16, 128-byte swizzled (u < 32 used): Wend
+    float *atab;                // [ntab][nch][S]: A_end
     __nv_bfloat16 *states;      // [BH][nch][2][S][D]: the state entering each chunk
+    __nv_bfloat16 *zbuf;        // [BH][nch][2][S][D]: each chunk's adjoint contributions (g o A)^T Q, (p o A)^T dO
     int *err;
 };
 
@@ -98,15 +107,13 @@ struct StateMap {
     __device__ static int cb0(int w) { return ((w & 3) * NB2) % DB; }
 };
 
-__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
-
 template <int D, int S>
 __global__ void __launch_bounds__(kBT, 1)
-    k_dchunk_bwd(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-                 const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
-                 const __grid_constant__ CUtensorMap tm_st,
-                 const __grid_constant__ CUtensorMap tm_dq, const __grid_constant__ CUtensorMap tm_dk,
-                 const __grid_constant__ CUtensorMap tm_dv, DbArgs a) {
+    k_dbchain(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+              const __grid_constant__ CUtensorMap tm_st, const __grid_constant__ CUtensorMap tm_z,
+              const __grid_constant__ CUtensorMap tm_dq, const __grid_constant__ CUtensorMap tm_dk,
+              const __grid_constant__ CUtensorMap tm_dv, DbArgs a) {
     using Lay = BwLayout<D, S>;
     using SMap = StateMap<D, S>;
     constexpr int SPT = S / 16, NB2 = SMap::NB2, SB = S / 16, DB = D / 16;
@@ -117,33 +124,27 @@ __global__ void __launch_bounds__(kBT, 1)
         if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (17 << 4) | ((int)blockIdx.x << 16));
         return;
     }
-    const int bh = blockIdx.x, hd = bh % a.H;
-    const float *Dx = a.Dx + (size_t)hd * a.hs_dx;
     const int L = a.L, nch = (L + kBC - 1) / kBC;
+    const long long nitems = (long long)a.BH * nch;
     uint8_t *sQ = dsm + Lay::q, *sK = dsm + Lay::k, *sV = dsm + Lay::v, *sDO = dsm + Lay::dout, *sO = dsm + Lay::o;
-    uint8_t *sOst = dsm + Lay::ost, *sK0 = dsm + Lay::k0, *sV0 = dsm + Lay::v0;
-    uint8_t *sMuK = dsm + Lay::muk, *sMuV = dsm + Lay::muv, *sW = dsm + Lay::wend, *sBeta = dsm + Lay::beta;
+    uint8_t *sOst = dsm + Lay::ost, *sK0 = dsm + Lay::k0, *sV0 = dsm + Lay::v0, *sBeta = dsm + Lay::beta;
     uint8_t *sPA = dsm + Lay::pa, *sGA = dsm + Lay::ga, *sGm = dsm + Lay::gm, *sGh = dsm + Lay::gh;
     float *sP = reinterpret_cast<float *>(dsm + Lay::pf), *sPV = reinterpret_cast<float *>(dsm + Lay::pvf);
     float *sS = reinterpret_cast<float *>(dsm + Lay::sf), *sDP = reinterpret_cast<float *>(dsm + Lay::dpf);
     float *sD = reinterpret_cast<float *>(dsm + Lay::df), *sAl = reinterpret_cast<float *>(dsm + Lay::af);
     float *sG4 = reinterpret_cast<float *>(dsm + Lay::g4), *sGpre = reinterpret_cast<float *>(dsm + Lay::gpre);
-    float *sAend = reinterpret_cast<float *>(dsm + Lay::aend), *sTot = reinterpret_cast<float *>(dsm + Lay::tot);
+    float *sTot = reinterpret_cast<float *>(dsm + Lay::tot);
     int *sdelta = reinterpret_cast<int *>(dsm + Lay::delta);
     float *sLse = reinterpret_cast<float *>(dsm + Lay::lse);
     uint64_t *bar = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
     const uint32_t uQ = tc::smem_u32(sQ), uK = tc::smem_u32(sK), uV = tc::smem_u32(sV), uDO = tc::smem_u32(sDO);
-    const uint32_t uK0 = tc::smem_u32(sK0), uV0 = tc::smem_u32(sV0), uMuK = tc::smem_u32(sMuK);
-    const uint32_t uMuV = tc::smem_u32(sMuV), uW = tc::smem_u32(sW), uBeta = tc::smem_u32(sBeta);
+    const uint32_t uK0 = tc::smem_u32(sK0), uV0 = tc::smem_u32(sV0), uBeta = tc::smem_u32(sBeta);
     const uint32_t uPA = tc::smem_u32(sPA), uGA = tc::smem_u32(sGA), uGm = tc::smem_u32(sGm), uGh = tc::smem_u32(sGh);
 
     if (threadIdx.x == 0) {
         tc::mbar_init(&bar[0], 1);
-        tc::mbar_init(&bar[1], 1);
-        tc::mbar_init(&bar[2], 1);
         tc::fence_barrier_init();
     }
-    for (int j = threadIdx.x; j < S; j += kBT) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
     // the upper triangles of G and G^, and the columns past S of p o A and g o A, stay zero
     for (int i = threadIdx.x; i < kBC * 64 / 2; i += kBT) {
         reinterpret_cast<uint32_t *>(sGm)[i] = 0u;
@@ -156,13 +157,14 @@ __global__ void __launch_bounds__(kBT, 1)
     // ---- the decay tables of a chunk (as in the forward): thread (slot tj, run trun) holds UPS tokens
     const int tj = threadIdx.x % S, trun = threadIdx.x / S, tu0 = trun * UPS;
     float dl[UPS];
-    auto load_d = [&](int c) {
+    auto load_d = [&](long long it) {
+        const int c = (int)(it / a.BH), hd = (int)(it % a.BH) % a.H;
         const int t0 = c * kBC, n = min(kBC, L - t0);
-        const float *src = Dx + t0 + tu0 + a.dmax - sdelta[tj];
+        const float *src = a.Dx + (size_t)hd * a.hs_dx + t0 + tu0 + a.dmax - a.delta[(size_t)hd * a.hs_delta + tj];
 #pragma unroll
         for (int i = 0; i < UPS; ++i) dl[i] = (tu0 + i < n) ? src[i] : 0.f;
     };
-    // D_j(u), alpha_j(tau), the sub-block products g and their prefixes Gpre, A_end, Wend and beta
+    // D_j(u), alpha_j(tau), the sub-block products g and their prefixes Gpre, and beta
     auto build_tables = [&]() {
         float pf[UPS], tot = 1.f;
 #pragma unroll
@@ -174,15 +176,14 @@ __global__ void __launch_bounds__(kBT, 1)
         sTot[trun * S + tj] = tot;
         __syncthreads();
         const int rb0 = (trun / RPB) * RPB;
-        float pre = 1.f, suf = 1.f, pre_b = 1.f, suf_b = 1.f;
+        float pre = 1.f, pre_b = 1.f, suf_b = 1.f;
         for (int r2 = 0; r2 < NRUN; ++r2) {
             const float x = sTot[r2 * S + tj];
             if (r2 < trun) {
                 pre *= x;
                 if (r2 >= rb0) pre_b *= x;
-            } else if (r2 > trun) {
-                suf *= x;
-                if (r2 < rb0 + RPB) suf_b *= x;
+            } else if (r2 > trun && r2 < rb0 + RPB) {
+                suf_b *= x;
             }
         }
 #pragma unroll
@@ -193,7 +194,6 @@ __global__ void __launch_bounds__(kBT, 1)
             sG4[(trun / RPB) * S + tj] = gb;
             sGpre[(trun / RPB) * S + tj] = pre;
         }
-        if (trun == NRUN - 1) sAend[tj] = pre * tot;
         float r = 1.f;
 #pragma unroll
         for (int i = UPS - 1; i >= 1; i -= 2) {
@@ -201,35 +201,25 @@ __global__ void __launch_bounds__(kBT, 1)
             r -= r * dl[i];
             const float w0 = dl[i - 1] * r;
             r -= r * dl[i - 1];
-            st_bf16x2(sW, S, tj, tu0 + i - 1, w0 * suf, w1 * suf);
             st_bf16x2(sBeta, S, tj, tu0 + i - 1, w0 * suf_b, w1 * suf_b);
         }
     };
 
-    // ---- the state (forward sweep) and later its adjoint (reverse sweep), in the accumulator layout
-    // of the MMAs that update them: warp w holds NB2 blocks of half kv, row block rb, column blocks cb0..
+    // ---- the chunk's adjoint contributions Z, in the accumulator layout of the MMAs that form them:
+    // warp w holds NB2 blocks of half kv, row block rb, column blocks cb0..
     const int skv = SMap::kv(warp), sj0 = SMap::rb(warp) * 16, se0 = SMap::cb0(warp) * 16;
     float st[NB2][2][4];
-#pragma unroll
-    for (int i = 0; i < NB2; ++i)
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) st[i][h][q] = 0.f;
-    // X <- A_end o X + Wend^T' X_c: A = Wend (rows S), B = the chunk's k or v (kn)
-    auto state_update = [&](uint32_t ux, uint32_t uw, bool transposed_a) {
-        const float f0 = sAend[sj0 + g8], f1 = sAend[sj0 + g8 + 8];
+    // Z = X_a^T X (A = the transposed p o A or g o A tile, B = the chunk's q or dO)
+    auto z_product = [&](uint32_t ux, uint32_t uw) {
 #pragma unroll
         for (int i = 0; i < NB2; ++i)
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                st[i][h][0] *= f0; st[i][h][1] *= f0;
-                st[i][h][2] *= f1; st[i][h][3] *= f1;
-            }
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) st[i][h][q] = 0.f;
         for (int k0 = 0; k0 < kBC; k0 += 16) {
             uint32_t af[4], b[4];
-            if (transposed_a) load_a_t(uw, kBC, sj0, k0, af);
-            else load_a(uw, S, sj0, k0, af);
+            load_a_t(uw, kBC, sj0, k0, af);
 #pragma unroll
             for (int i = 0; i < NB2; ++i) {
                 load_b_kn(ux, kBC, se0 + i * 16, k0, b);
@@ -239,111 +229,47 @@ __global__ void __launch_bounds__(kBT, 1)
         }
     };
 
-    // ================= forward sweep: the state entering every chunk, to the workspace (bf16).  k and
-    // v arrive in two stages: (k, v tiles) and (q, dO tiles), which the reverse sweep uses later.
-    uint32_t ph0 = 0, ph1 = 0, phs[2] = {0, 0};
+    uint32_t ph1 = 0;
     bool ok = true;
-    auto issue_kv = [&](int c) {
-        const int st2 = c & 1, t0 = c * kBC;
-        uint8_t *kb = st2 ? sQ : sK, *vb = st2 ? sDO : sV;
-        uint64_t *b = &bar[st2 ? 2 : 0];
-        tc::mbar_arrive_expect_tx(b, (uint32_t)(2 * Lay::kTile));
-        for (int db = 0; db < D / 64; ++db) {
-            tc::tma_load_3d(kb + db * kBC * 128, &tm_k, b, db * 64, t0, bh);
-            tc::tma_load_3d(vb + db * kBC * 128, &tm_v, b, db * 64, t0, bh);
-        }
-    };
-    if (nch > 0) {
-        load_d(0);
-        if (threadIdx.x == 0) issue_kv(0);
-    }
-    for (int c = 0; c < nch && ok; ++c) {
-        const int st2 = c & 1;
-        // the other stage was last read by the previous chunk (before the barrier that ended it)
-        if (threadIdx.x == 0 && c + 1 < nch) issue_kv(c + 1);
-        build_tables();
-        if (c + 1 < nch) load_d(c + 1);
-        {
-            __nv_bfloat16 *dst = a.states + (((size_t)bh * nch + c) * 2 + skv) * S * D;
-#pragma unroll
-            for (int i = 0; i < NB2; ++i)
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int e = se0 + i * 16 + h * 8 + 2 * t4;
-                    *reinterpret_cast<uint32_t *>(dst + (size_t)(sj0 + g8) * D + e) = tc::pack_bf16x2(st[i][h][0], st[i][h][1]);
-                    *reinterpret_cast<uint32_t *>(dst + (size_t)(sj0 + g8 + 8) * D + e) =
-                        tc::pack_bf16x2(st[i][h][2], st[i][h][3]);
-                }
-        }
-        if (!tc::mbar_wait(&bar[st2 ? 2 : 0], phs[st2])) {
-            report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (17 << 4));
-            ok = false;
-            break;
-        }
-        phs[st2] ^= 1;
-        state_update(skv ? (st2 ? uDO : uV) : (st2 ? uQ : uK), uW, false);
-        __syncthreads();   // the chunk's tiles and tables are read before the next chunk's arrive
-    }
-    (void)ph0;
-    if (!ok) return;
-    // the states were written through the generic proxy; the reverse sweep reads them by TMA
-    fence_proxy_async_global();
-    __syncthreads();
-
-    // ================= reverse sweep
-#pragma unroll
-    for (int i = 0; i < NB2; ++i)
-#pragma unroll
-        for (int h = 0; h < 2; ++h)
-#pragma unroll
-            for (int q = 0; q < 4; ++q) st[i][h][q] = 0.f;
-    // bf16 copy of the adjoint for the next (earlier) chunk's Wend^T mu
-    auto store_mu_copy = [&]() {
-        uint8_t *tile = skv ? sMuV : sMuK;
-#pragma unroll
-        for (int i = 0; i < NB2; ++i)
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int e = se0 + i * 16 + h * 8 + 2 * t4;
-                st_bf16x2(tile, S, sj0 + g8, e, st[i][h][0], st[i][h][1]);
-                st_bf16x2(tile, S, sj0 + g8 + 8, e, st[i][h][2], st[i][h][3]);
-            }
-    };
-    store_mu_copy();
-    if (nch > 0) load_d(nch - 1);
     const int sg = threadIdx.x & 15, rp = threadIdx.x >> 4, sb = rp >> 3, ip = rp & 7;
     const unsigned hmask = 0xffffu << (lane & 16);
-    for (int c = nch - 1; c >= 0 && ok; --c) {
+    if (blockIdx.x < nitems) load_d(blockIdx.x);
+    for (long long it = blockIdx.x; it < nitems && ok; it += gridDim.x) {
+        const int c = (int)(it / a.BH), bh = (int)(it % a.BH), hd = bh % a.H;
         const int t0 = c * kBC, n = min(kBC, L - t0);
+        const long long nx = it + gridDim.x;
         if (threadIdx.x == 0) {
-            tc::bulk_wait_read0();   // the later chunk's dQ, dK, dV stores have read their staging tiles
-            tc::mbar_arrive_expect_tx(&bar[1], (uint32_t)(4 * Lay::kTile + 2 * S * D * 2));
+            tc::bulk_wait_read0();   // the previous item's stores have read their staging tiles
+            tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(4 * Lay::kTile + 2 * S * D * 2));
+            const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
             for (int db = 0; db < D / 64; ++db) {
                 const int x = db * 64;
-                tc::tma_load_3d(sQ + db * kBC * 128, &tm_q, &bar[1], x, t0, bh);
-                tc::tma_load_3d(sK + db * kBC * 128, &tm_k, &bar[1], x, t0, bh);
-                tc::tma_load_3d(sV + db * kBC * 128, &tm_v, &bar[1], x, t0, bh);
-                tc::tma_load_3d(sDO + db * kBC * 128, &tm_do, &bar[1], x, t0, bh);
-                const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
-                tc::tma_load_2d(sK0 + db * S * 128, &tm_st, &bar[1], x, srow);
-                tc::tma_load_2d(sV0 + db * S * 128, &tm_st, &bar[1], x, srow + S);
+                tc::tma_load_3d(sQ + db * kBC * 128, &tm_q, &bar[0], x, t0, bh);
+                tc::tma_load_3d(sK + db * kBC * 128, &tm_k, &bar[0], x, t0, bh);
+                tc::tma_load_3d(sV + db * kBC * 128, &tm_v, &bar[0], x, t0, bh);
+                tc::tma_load_3d(sDO + db * kBC * 128, &tm_do, &bar[0], x, t0, bh);
+                tc::tma_load_2d(sK0 + db * S * 128, &tm_st, &bar[0], x, srow);
+                tc::tma_load_2d(sV0 + db * S * 128, &tm_st, &bar[0], x, srow + S);
+            }
+            // the next item's tiles into L2 meanwhile
+            if (nx < nitems) {
+                const int cn = (int)(nx / a.BH), bn = (int)(nx % a.BH), tn = cn * kBC;
+                for (int db = 0; db < D / 64; ++db) {
+                    const int x = db * 64;
+                    tc::tma_prefetch_3d(&tm_q, x, tn, bn);
+                    tc::tma_prefetch_3d(&tm_k, x, tn, bn);
+                    tc::tma_prefetch_3d(&tm_v, x, tn, bn);
+                    tc::tma_prefetch_3d(&tm_do, x, tn, bn);
+                }
+                tc::bulk_prefetch_l2(a.states + (((size_t)bn * nch + cn) * 2) * S * D, (uint32_t)(2 * S * D * 2));
             }
         }
-        // the chunk before this one (processed next) into L2 meanwhile
-        if (threadIdx.x == 0 && c > 0) {
-            for (int db = 0; db < D / 64; ++db) {
-                const int x = db * 64, tp = t0 - kBC;
-                tc::tma_prefetch_3d(&tm_q, x, tp, bh);
-                tc::tma_prefetch_3d(&tm_k, x, tp, bh);
-                tc::tma_prefetch_3d(&tm_v, x, tp, bh);
-                tc::tma_prefetch_3d(&tm_do, x, tp, bh);
-            }
-            tc::bulk_prefetch_l2(a.states + (((size_t)bh * nch + c - 1) * 2) * S * D, (uint32_t)(2 * S * D * 2));
-        }
+        // sdelta and sLse were last read before the previous item's closing barriers
+        for (int j = threadIdx.x; j < S; j += kBT) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
         if (threadIdx.x < kBC) sLse[threadIdx.x] = threadIdx.x < n ? a.lse[(size_t)bh * L + t0 + threadIdx.x] : 0.f;
         build_tables();
-        if (c > 0) load_d(c - 1);
-        if (!tc::mbar_wait(&bar[1], ph1)) {
+        if (nx < nitems) load_d(nx);
+        if (!tc::mbar_wait(&bar[0], ph1)) {
             report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (17 << 4));
             ok = false;
             break;
@@ -582,21 +508,11 @@ __global__ void __launch_bounds__(kBT, 1)
                     }
                 } else {
                     const uint32_t ug = which == 1 ? uGh : uGm, ux = which == 1 ? uQ : uDO;
-                    const uint32_t umu = which == 1 ? uMuK : uMuV;
                     for (int k0 = 0; k0 < kBC; k0 += 16) {
                         load_a_t(ug, kBC, om0, k0, af);
 #pragma unroll
                         for (int cb = 0; cb < OCB; ++cb) {
                             load_b_kn(ux, kBC, on0 + cb * 16, k0, b);
-                            mma16816(acc[cb][0], af, b[0], b[1]);
-                            mma16816(acc[cb][1], af, b[2], b[3]);
-                        }
-                    }
-                    for (int k0 = 0; k0 < S; k0 += 16) {
-                        load_a_t(uW, S, om0, k0, af);
-#pragma unroll
-                        for (int cb = 0; cb < OCB; ++cb) {
-                            load_b_kn(umu, S, on0 + cb * 16, k0, b);
                             mma16816(acc[cb][0], af, b[0], b[1]);
                             mma16816(acc[cb][1], af, b[2], b[3]);
                         }
@@ -612,34 +528,266 @@ __global__ void __launch_bounds__(kBT, 1)
                         st_bf16x2(dst, kBC, om0 + g8 + 8, col, acc[cb][h][2], acc[cb][h][3]);
                     }
             };
-            // dQ reads K0 and K, dK reads Q and mu_K, dV reads dO and mu_V: none of them reads the v or o
-            // tile, which the stores overwrite (V was read by PV, o by delta, before the barriers above)
+            // dQ reads K0 and K, dK reads Q, dV reads dO: none of them reads the v or o tile, which the
+            // stores overwrite (V was read by PV, o by delta, before the barriers above)
             out3(0);
             out3(1);
             out3(2);
         }
-        // ---- the adjoints of the previous chunk: mu_K <- (g o A)^T Q + A_end o mu_K,
-        // mu_V <- (p o A)^T dO + A_end o mu_V (registers; read after dK and dV used the old copies)
-        state_update(skv ? uDO : uQ, skv ? uPA : uGA, true);
+        // ---- the chunk's adjoint contributions Z_K = (g o A)^T Q, Z_V = (p o A)^T dO, staged over the
+        // K0 and V0 tiles once every warp has finished dQ
+        z_product(skv ? uDO : uQ, skv ? uPA : uGA);
+        __syncthreads();
+        {
+            uint8_t *tile = skv ? sV0 : sK0;
+#pragma unroll
+            for (int i = 0; i < NB2; ++i)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int e = se0 + i * 16 + h * 8 + 2 * t4;
+                    st_bf16x2(tile, S, sj0 + g8, e, st[i][h][0], st[i][h][1]);
+                    st_bf16x2(tile, S, sj0 + g8 + 8, e, st[i][h][2], st[i][h][3]);
+                }
+        }
         tc::fence_proxy_async_smem();
         __syncthreads();
         if (threadIdx.x == 0) {
+            const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
             for (int db = 0; db < D / 64; ++db) {
                 tc::tma_store_3d(&tm_dq, sV + db * kBC * 128, db * 64, t0, bh);
                 tc::tma_store_3d(&tm_dk, sO + db * kBC * 128, db * 64, t0, bh);
                 tc::tma_store_3d(&tm_dv, sOst + db * kBC * 128, db * 64, t0, bh);
+                tc::tma_store_2d(&tm_z, sK0 + db * S * 128, db * 64, srow);
+                tc::tma_store_2d(&tm_z, sV0 + db * S * 128, db * 64, srow + S);
             }
             tc::bulk_commit();
         }
-        store_mu_copy();
     }
     if (threadIdx.x == 0) tc::bulk_wait0();
+}
+
+// ---- Wend and A_end of every (head, chunk): thread j walks the chunk's tokens from the last back.
+// D_j(t0 + u) = Dx[t0 + u + dmax - Delta_j]; tokens past L contribute nothing (D = 0).
+template <int S>
+__global__ void __launch_bounds__(S) k_dbtab(DbArgs a) {
+    const int c = blockIdx.x, h = blockIdx.y, j = threadIdx.x, nch = (a.L + kBC - 1) / kBC;
+    const int t0 = c * kBC, n = min(kBC, a.L - t0);
+    const float *src = a.Dx + (size_t)h * a.hs_dx + t0 + a.dmax - a.delta[(size_t)h * a.hs_delta + j];
+    uint8_t *w = reinterpret_cast<uint8_t *>(a.wtab + ((size_t)h * nch + c) * S * 64);
+    float r = 1.f;
+#pragma unroll 4
+    for (int u = kBC - 2; u >= 0; u -= 2) {
+        const float d1 = (u + 1 < n) ? src[u + 1] : 0.f, d0 = (u < n) ? src[u] : 0.f;
+        const float w1 = d1 * r;
+        r -= r * d1;
+        const float w0 = d0 * r;
+        r -= r * d0;
+        *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = tc::pack_bf16x2(w0, w1);
+    }
+    for (int u = kBC; u < 64; u += 2) *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = 0u;
+    a.atab[((size_t)h * nch + c) * S + j] = r;
+}
+
+// ---- the two thin passes along the sequence.  One CTA per (64-column strip, K~ or V~, head) with
+// 4 warps; the strip [S][64] (fp32) lives in the accumulator registers of the MMAs that update it.
+constexpr int kSW = 4;           // warps
+constexpr int kNS = 4;           // pipeline stages
+
+template <int S>
+struct StripMap {
+    static constexpr int WR = S / 16, WC = kSW / WR, NC = 64 / WC, NB = NC / 16;
+    static_assert(WR * WC == kSW && NB >= 1, "strip blocks per warp");
+};
+
+template <int S>
+struct ScanLayout {
+    static constexpr int kT = kBC * 128;                    // [32][64] bf16 tile
+    static constexpr int kW = S * 128;                      // [S][64] bf16 tile (Wend image, state strip)
+    static constexpr int stage = kW + kW + kT;              // z (reverse only) | Wend | k or dk
+    static constexpr int mu = kNS * stage;                  // bf16 [S][64]: mu (reverse)
+    static constexpr int out = mu + kW;                     // 2 staging tiles: [S][64] (state) or [32][64]
+    static constexpr int ae = out + 2 * kW;                 // fp32 [kNS][S]: A_end of each stage
+    static constexpr int bars = ae + kNS * S * 4;
+    static constexpr int total = bars + 8 * kNS;
+    static_assert(stage % 1024 == 0 && mu % 1024 == 0 && out % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+};
+
+// REV = false: K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c from the zero state; the state entering chunk c
+// goes to `states` (bf16).  REV = true: from the last chunk back, dK_c += Wend(c)^T mu_c (bf16 MMA on a
+// copy of mu), then mu_{c-1} = A_end(c) o mu_c + Z_c.
+template <int D, int S, bool REV>
+__global__ void __launch_bounds__(kSW * 32)
+    k_dbscan(const __grid_constant__ CUtensorMap tm_x0, const __grid_constant__ CUtensorMap tm_x1,
+             const __grid_constant__ CUtensorMap tm_st, DbArgs a) {
+    using Lay = ScanLayout<S>;
+    using M = StripMap<S>;
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g8 = lane >> 2, t4 = lane & 3;
+    if (tc::smem_u32(dsm) & 1023u) {
+        if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (18 << 4) | ((int)blockIdx.x << 16));
+        return;
+    }
+    const int strip = blockIdx.x, kv = blockIdx.y, bh = blockIdx.z;
+    const int tab = a.ntab > 1 ? bh % a.H : 0;
+    const int nch = (a.L + kBC - 1) / kBC, x = strip * 64;
+    const CUtensorMap *tx = kv ? &tm_x1 : &tm_x0;   // k / v (forward) or dk / dv (reverse)
+    uint64_t *full = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
+    uint8_t *sMu = dsm + Lay::mu, *sOut = dsm + Lay::out;
+    // stage s: Z strip (reverse) at +0, Wend at +kW, the [32][64] tile at +2 kW; its A_end apart
+    auto sz = [&](int s) { return dsm + s * Lay::stage; };
+    auto sw = [&](int s) { return dsm + s * Lay::stage + Lay::kW; };
+    auto sx = [&](int s) { return dsm + s * Lay::stage + 2 * Lay::kW; };
+    auto sa = [&](int s) { return reinterpret_cast<float *>(dsm + Lay::ae + s * S * 4); };
+    auto chunk_of = [&](int i) { return REV ? nch - 1 - i : i; };
+    auto issue = [&](int i) {
+        const int s = i % kNS, c = chunk_of(i);
+        const size_t ti = (size_t)tab * nch + c;
+        const uint32_t bytes = (uint32_t)(Lay::kW + Lay::kT + S * 4 + (REV ? Lay::kW : 0));
+        tc::mbar_arrive_expect_tx(&full[s], bytes);
+        if (REV) tc::tma_load_2d(sz(s), &tm_st, &full[s], x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
+        tc::bulk_load(sw(s), a.wtab + ti * S * 64, (uint32_t)Lay::kW, &full[s]);
+        tc::tma_load_3d(sx(s), tx, &full[s], x, c * kBC, bh);
+        tc::bulk_load(sa(s), a.atab + ti * S, (uint32_t)(S * 4), &full[s]);
+    };
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kNS; ++s) tc::mbar_init(&full[s], 1);
+        tc::fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+        for (int i = 0; i < kNS && i < nch; ++i) issue(i);
+
+    const int r0 = (warp % M::WR) * 16, c0 = (warp / M::WR) * M::NC;
+    float acc[M::NB][2][4];
+#pragma unroll
+    for (int i = 0; i < M::NB; ++i)
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc[i][h][q] = 0.f;
+    auto put = [&](uint8_t *tile) {   // acc (bf16) into a swizzled [S][64] tile
+#pragma unroll
+        for (int i = 0; i < M::NB; ++i)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int e = c0 + i * 16 + h * 8 + 2 * t4;
+                st_bf16x2(tile, S, r0 + g8, e, acc[i][h][0], acc[i][h][1]);
+                st_bf16x2(tile, S, r0 + g8 + 8, e, acc[i][h][2], acc[i][h][3]);
+            }
+    };
+    bool ok = true;
+    for (int i = 0; i < nch; ++i) {
+        const int s = i % kNS, c = chunk_of(i), ob = i & 1;
+        if (threadIdx.x == 0) tc::bulk_wait_read1();   // the store that used staging tile ob has read it
+        if (!REV) {
+            __syncthreads();
+            put(sOut + ob * Lay::kW);   // the state entering chunk c
+        }
+        if (!tc::mbar_wait(&full[s], (uint32_t)((i / kNS) & 1))) {
+            report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (18 << 4));
+            ok = false;
+        }
+        if (__syncthreads_or(!ok)) break;
+        const float *ae = sa(s);
+        const float f0 = ae[r0 + g8], f1 = ae[r0 + g8 + 8];
+        const uint32_t uW = tc::smem_u32(sw(s)), uX = tc::smem_u32(sx(s));
+        if (!REV) {
+            // acc <- A_end o acc + Wend K_c: A = Wend [S][32 tokens], B = the chunk's strip [32][64]
+#pragma unroll
+            for (int b = 0; b < M::NB; ++b)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    acc[b][h][0] *= f0; acc[b][h][1] *= f0;
+                    acc[b][h][2] *= f1; acc[b][h][3] *= f1;
+                }
+#pragma unroll
+            for (int k0 = 0; k0 < kBC; k0 += 16) {
+                uint32_t af[4], bf[4];
+                load_a(uW, S, r0, k0, af);
+#pragma unroll
+                for (int b = 0; b < M::NB; ++b) {
+                    load_b_kn(uX, kBC, c0 + b * 16, k0, bf);
+                    mma16816(acc[b][0], af, bf[0], bf[1]);
+                    mma16816(acc[b][1], af, bf[2], bf[3]);
+                }
+            }
+        } else {
+            // dK_c [32][64] += Wend^T mu: warp takes token rows om0.. and 32 columns on0..
+            const bool live = i > 0;   // mu is zero after the last chunk
+            if (live) {
+                put(sMu);
+                __syncthreads();
+                const int om0 = (warp & 1) * 16, on0 = (warp >> 1) * 32;
+                float o[2][2][4] = {};
+                const uint32_t uMu = tc::smem_u32(sMu);
+#pragma unroll
+                for (int k0 = 0; k0 < S; k0 += 16) {
+                    uint32_t af[4], bf[4];
+                    load_a_t(uW, S, om0, k0, af);
+#pragma unroll
+                    for (int b = 0; b < 2; ++b) {
+                        load_b_kn(uMu, S, on0 + b * 16, k0, bf);
+                        mma16816(o[b][0], af, bf[0], bf[1]);
+                        mma16816(o[b][1], af, bf[2], bf[3]);
+                    }
+                }
+                const uint8_t *dk = sx(s);
+                uint8_t *dst = sOut + ob * Lay::kW;
+#pragma unroll
+                for (int b = 0; b < 2; ++b)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int rh = 0; rh < 2; ++rh) {
+                            const int row = om0 + g8 + rh * 8, col = on0 + b * 16 + h * 8 + 2 * t4;
+                            const float2 l = __bfloat1622float2(
+                                *reinterpret_cast<const __nv_bfloat162 *>(dk + sw_off(kBC, row, col)));
+                            st_bf16x2(dst, kBC, row, col, o[b][h][2 * rh] + l.x, o[b][h][2 * rh + 1] + l.y);
+                        }
+            }
+            // mu <- A_end o mu + Z_c
+            const uint8_t *z = sz(s);
+#pragma unroll
+            for (int b = 0; b < M::NB; ++b)
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int rh = 0; rh < 2; ++rh) {
+                        const int row = r0 + g8 + rh * 8, col = c0 + b * 16 + h * 8 + 2 * t4;
+                        const float f = rh ? f1 : f0;
+                        const float2 zz =
+                            __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(z + sw_off(S, row, col)));
+                        acc[b][h][2 * rh] = fmaf(f, acc[b][h][2 * rh], zz.x);
+                        acc[b][h][2 * rh + 1] = fmaf(f, acc[b][h][2 * rh + 1], zz.y);
+                    }
+        }
+        tc::fence_proxy_async_smem();
+        __syncthreads();   // stage s and the staging tile are complete
+        if (threadIdx.x == 0) {
+            if (!REV) {
+                tc::tma_store_2d(&tm_st, sOut + ob * Lay::kW, x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
+                tc::bulk_commit();
+            } else if (i > 0) {
+                tc::tma_store_3d(tx, sOut + ob * Lay::kW, x, c * kBC, bh);
+                tc::bulk_commit();
+            }
+            if (i + kNS < nch) issue(i + kNS);
+        }
+    }
+    if (threadIdx.x == 0) tc::bulk_wait0();
+}
+
+int sm_count_db() {
+    int dev = 0, n = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 152;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 152;
+    return n;
 }
 
 template <int D, int S>
 cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v,
                           const void *dout, void *dq, void *dk, void *dv, cudaStream_t st) {
-    CUtensorMap tq, tk, tv, tdo, tst, tdq, tdk, tdv;
+    CUtensorMap tq, tk, tv, tdo, tst, tz, tdq, tdk, tdv;
     const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
     const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
     const uint32_t box[3] = {64, (uint32_t)kBC, 1};
@@ -649,34 +797,65 @@ cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const
     const uint32_t sbox[2] = {64, (uint32_t)S};
     if (!make_tmap_bf16(&tq, q, 3, dims, strides, box) || !make_tmap_bf16(&tk, k, 3, dims, strides, box) ||
         !make_tmap_bf16(&tv, v, 3, dims, strides, box) || !make_tmap_bf16(&tdo, dout, 3, dims, strides, box) ||
-        !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) ||
+        !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) || !make_tmap_bf16(&tz, a.zbuf, 2, sdims, sstr, sbox) ||
         !make_tmap_bf16(&tdq, dq, 3, dims, strides, box) || !make_tmap_bf16(&tdk, dk, 3, dims, strides, box) ||
         !make_tmap_bf16(&tdv, dv, 3, dims, strides, box))
         return cudaErrorInvalidValue;
-    const int smem = BwLayout<D, S>::total;
-    cudaError_t e = cudaFuncSetAttribute(k_dchunk_bwd<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    const int smem = BwLayout<D, S>::total, ssm = ScanLayout<S>::total;
+    cudaError_t e = cudaFuncSetAttribute(k_dbchain<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_dbscan<D, S, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_dbscan<D, S, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_DECAY, st);
-    k_dchunk_bwd<D, S><<<(unsigned)((long long)d.B * d.H), kBT, smem, st>>>(tq, tk, tv, tdo, tst, tdq, tdk, tdv, a);
+    k_dbtab<S><<<dim3((unsigned)nch, (unsigned)a.ntab), S, 0, st>>>(a);
+    const dim3 sgrid((unsigned)(D / 64), 2u, (unsigned)a.BH);
+    k_dbscan<D, S, false><<<sgrid, kSW * 32, ssm, st>>>(tk, tv, tst, a);
+    const long long items = (long long)a.BH * nch;
+    const int grid = (int)(items < sm_count_db() ? items : sm_count_db());
+    k_dbchain<D, S><<<(unsigned)grid, kBT, smem, st>>>(tq, tk, tv, tdo, tst, tz, tdq, tdk, tdv, a);
+    k_dbscan<D, S, true><<<sgrid, kSW * 32, ssm, st>>>(tdk, tdv, tz, a);
     return cudaGetLastError();
+}
+
+// the pieces of the backward's workspace: states, Z, Wend tables, A_end tables
+struct DbWs {
+    size_t states, z, wtab, atab, total;
+};
+
+DbWs db_ws(const OpDims &d) {
+    const size_t nch = (size_t)(d.L + kBC - 1) / kBC, ntab = d.periods ? (size_t)d.H : 1;
+    const size_t per = align_up((size_t)d.B * d.H * nch * 2 * d.S * d.dk * sizeof(__nv_bfloat16), 256);
+    DbWs w;
+    w.states = 0;
+    w.z = per;
+    w.wtab = 2 * per;
+    w.atab = w.wtab + align_up(ntab * nch * d.S * 64 * sizeof(__nv_bfloat16), 256);
+    w.total = w.atab + align_up(ntab * nch * d.S * sizeof(float), 256);
+    return w;
 }
 
 }  // namespace
 
-size_t decay_chunk_bwd_state_bytes(const OpDims &d) {
-    const size_t nch = (size_t)(d.L + kBC - 1) / kBC;
-    return (size_t)d.B * d.H * nch * 2 * d.S * d.dk * sizeof(__nv_bfloat16);
-}
+size_t decay_chunk_bwd_ws_bytes(const OpDims &d) { return db_ws(d).total; }
 
 cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, const float *Dx, const int *delta,
-                                   int hs_dx, int hs_delta, const void *q, const void *k, const void *v, const void *o,
-                                   const void *dout, const float *lse, void *dq, void *dk, void *dv, void *states,
+                                   int hs_dx, int hs_delta, const void *q, const void *k, const void *v,
+                                   const void *dout, const float *lse, void *dq, void *dk, void *dv, void *ws,
                                    cudaStream_t st) {
+    const DbWs w = db_ws(d);
+    char *base = static_cast<char *>(ws);
     DbArgs a;
-    a.L = d.L; a.H = d.H; a.pos0 = pos0; a.scale = d.scale; a.dmax = dmax;
+    a.L = d.L; a.H = d.H; a.BH = d.B * d.H; a.pos0 = pos0; a.scale = d.scale; a.dmax = dmax;
     a.Dx = Dx; a.delta = delta; a.hs_dx = hs_dx; a.hs_delta = hs_delta;
     a.lse = lse;
-    a.states = static_cast<__nv_bfloat16 *>(states);
+    a.ntab = (hs_dx != 0 || hs_delta != 0) ? d.H : 1;
+    if (a.ntab > 1 && !d.periods) return cudaErrorInvalidValue;   // the tables are sized per head only then
+    a.states = reinterpret_cast<__nv_bfloat16 *>(base + w.states);
+    a.zbuf = reinterpret_cast<__nv_bfloat16 *>(base + w.z);
+    a.wtab = reinterpret_cast<__nv_bfloat16 *>(base + w.wtab);
+    a.atab = reinterpret_cast<float *>(base + w.atab);
     a.err = device_error_word();
     if (d.dk == 64) return d.S == 32 ? launch_dbwd_t<64, 32>(d, a, q, k, v, dout, dq, dk, dv, st)
                                      : launch_dbwd_t<64, 64>(d, a, q, k, v, dout, dq, dk, dv, st);
