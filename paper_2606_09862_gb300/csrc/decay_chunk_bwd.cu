@@ -20,7 +20,7 @@
 //      period and the positions only, not on the batch);
 //   2. k_dbstate: per (head, 64-column strip of K~ or V~): K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c,
 //      the state entering every chunk stored in bf16;
-//   3. k_dbchain: one work item per (head, chunk), over persistent CTAs: s, p, dp, g, G, G^, then dQ
+//   3. k_dbchain: one work item per (head, chunk), each CTA a run of consecutive chunks: s, p, dp, g, G, G^, then dQ
 //      (final), the chunk's own parts G^T Q and G^T dO of dK and dV, and its adjoint contributions
 //      Z_K = (g o A)^T Q, Z_V = (p o A)^T dO (bf16);
 //   4. k_dbadj: per (head, strip), from the last chunk back: dK += Wend^T mu_K (dV likewise), then
@@ -47,40 +47,50 @@ constexpr int kBT = 256;         // threads (8 warps)
 constexpr int kBFS = kBC + 4;    // fp32 row stride of [32][32] tiles
 constexpr int kBSS = 64 + 4;     // fp32 row stride of [32][S] tiles (S <= 64)
 
+// The chain's tables of one (head, chunk), built by k_dbtab and copied whole into shared memory:
+// beta_j(u) (bf16, swizzled [S][64], u < 32 used), D_j(t0 + u) and alpha_j(tau) (fp32 [32][kBSS]),
+// and Gpre (fp32 [2][S]: the decay of the sub-blocks before sub-block 0, 1).
+template <int S>
+struct ChunkTab {
+    static constexpr int beta = 0, d = S * 128, alpha = d + kBC * kBSS * 4, gpre = alpha + kBC * kBSS * 4;
+    static constexpr int bytes = gpre + 2 * S * 4;
+    static_assert(bytes % 16 == 0, "bulk copies move multiples of 16 bytes");
+};
+
 template <int D, int S>
 struct BwLayout {
     static constexpr int kTile = kBC * D * 2;          // one [32][D] bf16 tile
-    static constexpr int q = 0, k = q + kTile, v = k + kTile, dout = v + kTile;
-    static constexpr int o = dout + kTile;              // bf16 [32][D]: dK staging (dQ is staged over v)
+    static constexpr int q = 0;                         // bf16 [2][32][D]: q of this item and the next
+    static constexpr int dout = q + 2 * kTile;          // bf16 [2][32][D]: dO likewise
+    static constexpr int k = dout + 2 * kTile, v = k + kTile;
+    static constexpr int o = v + kTile;                 // bf16 [32][D]: dK staging
     static constexpr int ost = o + kTile;               // bf16 [32][D]: dV staging
-    static constexpr int k0 = ost + kTile;              // bf16 [S][D]: K~ entering the chunk, then Z_K
-    static constexpr int v0 = k0 + S * D * 2;           // bf16 [S][D]: V~ entering the chunk, then Z_V
-    static constexpr int beta = v0 + S * D * 2;         // bf16 [S][64] (u < 32 used): beta_j(u)
-    static constexpr int pa = beta + S * 128;           // bf16 [32][64]: p o A
+    static constexpr int k0 = ost + kTile;              // bf16 [S][D]: K~ entering the chunk
+    static constexpr int v0 = k0 + S * D * 2;           // bf16 [S][D]: V~ entering the chunk
+    static constexpr int zk = v0 + S * D * 2;           // bf16 [S][D]: Z_K staging
+    static constexpr int zv = zk + S * D * 2;           // bf16 [S][D]: Z_V staging
+    static constexpr int tab = zv + S * D * 2;          // the chunk's tables (ChunkTab)
+    static constexpr int pa = tab + ((ChunkTab<S>::bytes + 1023) / 1024) * 1024;   // bf16 [32][64]: p o A
     static constexpr int ga = pa + kBC * 128;           // bf16 [32][64]: g o A
     static constexpr int gm = ga + kBC * 128;           // bf16 [32][64] (u < 32): G
     static constexpr int gh = gm + kBC * 128;           // bf16 [32][64]: G^
-    static constexpr int pf = gh + kBC * 128;           // fp32 [32][kBFS]: P
+    static constexpr int sf = gh + kBC * 128;           // fp32 [32][kBSS]: s, then p, then dQ staging (bf16)
+    static constexpr int pf = sf + kBC * kBSS * 4;      // fp32 [32][kBFS]: P
     static constexpr int pvf = pf + kBC * kBFS * 4;     // fp32 [32][kBFS]: PV
-    static constexpr int sf = pvf + kBC * kBFS * 4;     // fp32 [32][kBSS]: s, then p
-    static constexpr int dpf = sf + kBC * kBSS * 4;     // fp32 [32][kBSS]: dp, then g
-    static constexpr int df = dpf + kBC * kBSS * 4;     // fp32 [32][kBSS]: D_j(t0 + u)
-    static constexpr int af = df + kBC * kBSS * 4;      // fp32 [32][kBSS]: alpha_j(tau)
-    static constexpr int g4 = af + kBC * kBSS * 4;      // fp32 [2][S]: sub-block products
-    static constexpr int gpre = g4 + 2 * S * 4;         // fp32 [2][S]: product of the sub-blocks before
-    static constexpr int tot = gpre + 2 * S * 4;        // fp32 [kBT / S][S]: run products
-    static constexpr int delta = tot + kBT * 4;         // int [S]
+    static constexpr int dpf = pvf + kBC * kBFS * 4;    // fp32 [32][kBSS]: dp, then g
+    static constexpr int delta = dpf + kBC * kBSS * 4;  // int [S]
     static constexpr int lse = delta + S * 4;           // fp32 [32]
     static constexpr int bars = lse + kBC * 4;          // mbarrier: the item's tiles
     static constexpr int total = bars + 64;
-    static_assert(k0 % 1024 == 0 && beta % 1024 == 0 && pa % 1024 == 0 && gh % 1024 == 0 &&
-                      pf % 16 == 0,
+    static_assert(k0 % 1024 == 0 && tab % 1024 == 0 && pa % 1024 == 0 && gh % 1024 == 0 && sf % 1024 == 0 &&
+                      kBC * kBSS * 4 >= kTile && pf % 16 == 0,
                   "swizzled tiles need 1024-byte alignment");
     static_assert(total <= 227 * 1024, "shared memory of one CTA");
 };
 
 struct DbArgs {
     int L, H, BH;
+    int ipc;                    // chain items (chunks) per CTA: CTA b takes items [b ipc, (b + 1) ipc), chunk fastest
     long long pos0;
     float scale;
     int dmax;
@@ -89,6 +99,7 @@ struct DbArgs {
     int hs_dx, hs_delta;        // per-head strides (0: one shared period)
     const float *lse;           // [BH][L], from the forward
     int ntab;                   // heads with their own tables (1 when the heads share one period)
+    uint8_t *ctab;              // [ntab][nch] ChunkTab records of the chain
     __nv_bfloat16 *wtab;        // [ntab][nch][S][64] bf16, 128-byte swizzled (u < 32 used): Wend
     float *atab;                // [ntab][nch][S]: A_end
     __nv_bfloat16 *states;      // [BH][nch][2][S][D]: the state entering each chunk
@@ -117,7 +128,6 @@ __global__ void __launch_bounds__(kBT, 1)
     using Lay = BwLayout<D, S>;
     using SMap = StateMap<D, S>;
     constexpr int SPT = S / 16, NB2 = SMap::NB2, SB = S / 16, DB = D / 16;
-    constexpr int NRUN = kBT / S, UPS = kBC / NRUN, RPB = 16 / UPS;
     extern __shared__ __align__(1024) uint8_t dsm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g8 = lane >> 2, t4 = lane & 3;
     if (tc::smem_u32(dsm) & 1023u) {
@@ -126,18 +136,19 @@ __global__ void __launch_bounds__(kBT, 1)
     }
     const int L = a.L, nch = (L + kBC - 1) / kBC;
     const long long nitems = (long long)a.BH * nch;
-    uint8_t *sQ = dsm + Lay::q, *sK = dsm + Lay::k, *sV = dsm + Lay::v, *sDO = dsm + Lay::dout, *sO = dsm + Lay::o;
-    uint8_t *sOst = dsm + Lay::ost, *sK0 = dsm + Lay::k0, *sV0 = dsm + Lay::v0, *sBeta = dsm + Lay::beta;
+    uint8_t *sK = dsm + Lay::k, *sV = dsm + Lay::v, *sO = dsm + Lay::o;
+    using Tab = ChunkTab<S>;
+    uint8_t *sOst = dsm + Lay::ost, *sK0 = dsm + Lay::k0, *sV0 = dsm + Lay::v0, *sTab = dsm + Lay::tab;
+    uint8_t *sZK = dsm + Lay::zk, *sZV = dsm + Lay::zv, *sBeta = sTab + Tab::beta;
     uint8_t *sPA = dsm + Lay::pa, *sGA = dsm + Lay::ga, *sGm = dsm + Lay::gm, *sGh = dsm + Lay::gh;
     float *sP = reinterpret_cast<float *>(dsm + Lay::pf), *sPV = reinterpret_cast<float *>(dsm + Lay::pvf);
     float *sS = reinterpret_cast<float *>(dsm + Lay::sf), *sDP = reinterpret_cast<float *>(dsm + Lay::dpf);
-    float *sD = reinterpret_cast<float *>(dsm + Lay::df), *sAl = reinterpret_cast<float *>(dsm + Lay::af);
-    float *sG4 = reinterpret_cast<float *>(dsm + Lay::g4), *sGpre = reinterpret_cast<float *>(dsm + Lay::gpre);
-    float *sTot = reinterpret_cast<float *>(dsm + Lay::tot);
+    float *sD = reinterpret_cast<float *>(sTab + Tab::d), *sAl = reinterpret_cast<float *>(sTab + Tab::alpha);
+    float *sGpre = reinterpret_cast<float *>(sTab + Tab::gpre);
     int *sdelta = reinterpret_cast<int *>(dsm + Lay::delta);
     float *sLse = reinterpret_cast<float *>(dsm + Lay::lse);
     uint64_t *bar = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
-    const uint32_t uQ = tc::smem_u32(sQ), uK = tc::smem_u32(sK), uV = tc::smem_u32(sV), uDO = tc::smem_u32(sDO);
+    const uint32_t uK = tc::smem_u32(sK), uV = tc::smem_u32(sV);
     const uint32_t uK0 = tc::smem_u32(sK0), uV0 = tc::smem_u32(sV0), uBeta = tc::smem_u32(sBeta);
     const uint32_t uPA = tc::smem_u32(sPA), uGA = tc::smem_u32(sGA), uGm = tc::smem_u32(sGm), uGh = tc::smem_u32(sGh);
 
@@ -153,57 +164,6 @@ __global__ void __launch_bounds__(kBT, 1)
         reinterpret_cast<uint32_t *>(sGA)[i] = 0u;
     }
     __syncthreads();
-
-    // ---- the decay tables of a chunk (as in the forward): thread (slot tj, run trun) holds UPS tokens
-    const int tj = threadIdx.x % S, trun = threadIdx.x / S, tu0 = trun * UPS;
-    float dl[UPS];
-    auto load_d = [&](long long it) {
-        const int c = (int)(it / a.BH), hd = (int)(it % a.BH) % a.H;
-        const int t0 = c * kBC, n = min(kBC, L - t0);
-        const float *src = a.Dx + (size_t)hd * a.hs_dx + t0 + tu0 + a.dmax - a.delta[(size_t)hd * a.hs_delta + tj];
-#pragma unroll
-        for (int i = 0; i < UPS; ++i) dl[i] = (tu0 + i < n) ? src[i] : 0.f;
-    };
-    // D_j(u), alpha_j(tau), the sub-block products g and their prefixes Gpre, and beta
-    auto build_tables = [&]() {
-        float pf[UPS], tot = 1.f;
-#pragma unroll
-        for (int i = 0; i < UPS; ++i) {
-            sD[(tu0 + i) * kBSS + tj] = dl[i];
-            tot *= 1.f - dl[i];
-            pf[i] = tot;
-        }
-        sTot[trun * S + tj] = tot;
-        __syncthreads();
-        const int rb0 = (trun / RPB) * RPB;
-        float pre = 1.f, pre_b = 1.f, suf_b = 1.f;
-        for (int r2 = 0; r2 < NRUN; ++r2) {
-            const float x = sTot[r2 * S + tj];
-            if (r2 < trun) {
-                pre *= x;
-                if (r2 >= rb0) pre_b *= x;
-            } else if (r2 > trun && r2 < rb0 + RPB) {
-                suf_b *= x;
-            }
-        }
-#pragma unroll
-        for (int i = 0; i < UPS; ++i) sAl[(tu0 + i) * kBSS + tj] = pre_b * pf[i];
-        if (trun == rb0) {
-            float gb = tot;
-            for (int r2 = trun + 1; r2 < rb0 + RPB; ++r2) gb *= sTot[r2 * S + tj];
-            sG4[(trun / RPB) * S + tj] = gb;
-            sGpre[(trun / RPB) * S + tj] = pre;
-        }
-        float r = 1.f;
-#pragma unroll
-        for (int i = UPS - 1; i >= 1; i -= 2) {
-            const float w1 = dl[i] * r;
-            r -= r * dl[i];
-            const float w0 = dl[i - 1] * r;
-            r -= r * dl[i - 1];
-            st_bf16x2(sBeta, S, tj, tu0 + i - 1, w0 * suf_b, w1 * suf_b);
-        }
-    };
 
     // ---- the chunk's adjoint contributions Z, in the accumulator layout of the MMAs that form them:
     // warp w holds NB2 blocks of half kv, row block rb, column blocks cb0..
@@ -233,42 +193,63 @@ __global__ void __launch_bounds__(kBT, 1)
     bool ok = true;
     const int sg = threadIdx.x & 15, rp = threadIdx.x >> 4, sb = rp >> 3, ip = rp & 7;
     const unsigned hmask = 0xffffu << (lane & 16);
-    if (blockIdx.x < nitems) load_d(blockIdx.x);
-    for (long long it = blockIdx.x; it < nitems && ok; it += gridDim.x) {
-        const int c = (int)(it / a.BH), bh = (int)(it % a.BH), hd = bh % a.H;
-        const int t0 = c * kBC, n = min(kBC, L - t0);
-        const long long nx = it + gridDim.x;
+    const int i0 = (int)blockIdx.x * a.ipc, i1 = (int)min(nitems, (long long)i0 + a.ipc);
+    // the next item's lse (threads < 32) travels in a register
+    float lse_nx = 0.f;
+    auto load_lse = [&](int it) {
+        const int c = (int)(it % nch), bh = (int)(it / nch), t = c * kBC + (int)threadIdx.x;
+        if (threadIdx.x < kBC) lse_nx = t < L ? a.lse[(size_t)bh * L + t] : 0.f;
+    };
+    auto tab_of = [&](int it) {
+        const int tb = a.ntab > 1 ? (int)(it / nch) % a.H : 0;
+        return a.ctab + ((size_t)tb * nch + (size_t)(it % nch)) * Tab::bytes;
+    };
+    // Item it + 1's loads are issued while item it runs, each once its place is free: v, q and dO
+    // (the other of the two q / dO buffers) after (a), the tables after (d), k, K0 and V0 after dQ.
+    auto issue_vqo = [&](int it, int buf) {
+        const int c = (int)(it % nch), bh = (int)(it / nch), t0 = c * kBC;
+        tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(4 * Lay::kTile + 2 * S * D * 2 + Tab::bytes));
+        tc::tma_load_4d(sV, &tm_v, &bar[0], 0, t0, 0, bh);
+        tc::tma_load_4d(dsm + Lay::q + buf * Lay::kTile, &tm_q, &bar[0], 0, t0, 0, bh);
+        tc::tma_load_4d(dsm + Lay::dout + buf * Lay::kTile, &tm_do, &bar[0], 0, t0, 0, bh);
+    };
+    auto issue_tab = [&](int it) { tc::bulk_load(sTab, tab_of(it), (uint32_t)Tab::bytes, &bar[0]); };
+    auto issue_k = [&](int it) {
+        const int c = (int)(it % nch), bh = (int)(it / nch);
+        const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
+        tc::tma_load_4d(sK, &tm_k, &bar[0], 0, c * kBC, 0, bh);
+        tc::tma_load_3d(sK0, &tm_st, &bar[0], 0, srow, 0);
+        tc::tma_load_3d(sV0, &tm_st, &bar[0], 0, srow + S, 0);
+    };
+    if (i0 < i1) {
+        load_lse(i0);
         if (threadIdx.x == 0) {
-            tc::bulk_wait_read0();   // the previous item's stores have read their staging tiles
-            tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(4 * Lay::kTile + 2 * S * D * 2));
-            const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
-            for (int db = 0; db < D / 64; ++db) {
-                const int x = db * 64;
-                tc::tma_load_3d(sQ + db * kBC * 128, &tm_q, &bar[0], x, t0, bh);
-                tc::tma_load_3d(sK + db * kBC * 128, &tm_k, &bar[0], x, t0, bh);
-                tc::tma_load_3d(sV + db * kBC * 128, &tm_v, &bar[0], x, t0, bh);
-                tc::tma_load_3d(sDO + db * kBC * 128, &tm_do, &bar[0], x, t0, bh);
-                tc::tma_load_2d(sK0 + db * S * 128, &tm_st, &bar[0], x, srow);
-                tc::tma_load_2d(sV0 + db * S * 128, &tm_st, &bar[0], x, srow + S);
-            }
-            // the next item's tiles into L2 meanwhile
-            if (nx < nitems) {
-                const int cn = (int)(nx / a.BH), bn = (int)(nx % a.BH), tn = cn * kBC;
-                for (int db = 0; db < D / 64; ++db) {
-                    const int x = db * 64;
-                    tc::tma_prefetch_3d(&tm_q, x, tn, bn);
-                    tc::tma_prefetch_3d(&tm_k, x, tn, bn);
-                    tc::tma_prefetch_3d(&tm_v, x, tn, bn);
-                    tc::tma_prefetch_3d(&tm_do, x, tn, bn);
-                }
-                tc::bulk_prefetch_l2(a.states + (((size_t)bn * nch + cn) * 2) * S * D, (uint32_t)(2 * S * D * 2));
-            }
+            issue_vqo(i0, 0);
+            issue_tab(i0);
+            issue_k(i0);
+        }
+    }
+    int cur_hd = -1;
+    for (int it = i0; it < i1 && ok; ++it) {
+        const int c = (int)(it % nch), bh = (int)(it / nch), hd = bh % a.H;
+        const int t0 = c * kBC, n = min(kBC, L - t0);
+        const int nx = it + 1;
+        const int buf = (int)((it - i0) & 1);
+        const uint32_t uQ = tc::smem_u32(dsm + Lay::q + buf * Lay::kTile);
+        const uint32_t uDO = tc::smem_u32(dsm + Lay::dout + buf * Lay::kTile);
+        if (threadIdx.x == kBT - 32 && nx < i1) {
+            // the next item's k and states into L2 (their loads follow dQ)
+            const int cn = (int)(nx % nch), bn = (int)(nx / nch);
+            tc::tma_prefetch_4d(&tm_k, 0, cn * kBC, 0, bn);
+            tc::bulk_prefetch_l2(a.states + (((size_t)bn * nch + cn) * 2) * S * D, (uint32_t)(2 * S * D * 2));
         }
         // sdelta and sLse were last read before the previous item's closing barriers
-        for (int j = threadIdx.x; j < S; j += kBT) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
-        if (threadIdx.x < kBC) sLse[threadIdx.x] = threadIdx.x < n ? a.lse[(size_t)bh * L + t0 + threadIdx.x] : 0.f;
-        build_tables();
-        if (nx < nitems) load_d(nx);
+        if (hd != cur_hd) {
+            for (int j = threadIdx.x; j < S; j += kBT) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
+            cur_hd = hd;
+        }
+        if (threadIdx.x < kBC) sLse[threadIdx.x] = lse_nx;
+        if (nx < i1) load_lse(nx);
         if (!tc::mbar_wait(&bar[0], ph1)) {
             report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (17 << 4));
             ok = false;
@@ -306,7 +287,12 @@ __global__ void __launch_bounds__(kBT, 1)
                 *reinterpret_cast<float2 *>(&dst[(m0 + g8 + 8) * kBFS + col]) = make_float2(pacc[h][2], pacc[h][3]);
             }
         }
+        // the previous item's stores have read their staging tiles (s, where dQ was staged, is written
+        // next; the dK, dV and Z staging tiles later)
+        if (threadIdx.x == 0) tc::bulk_wait_read0();
         __syncthreads();
+        // v, q and dO are read: the next item's go in (q and dO into the other buffer)
+        if (threadIdx.x == 0 && nx < i1) issue_vqo(nx, buf ^ 1);
         // ---- (b) the off-diagonal block of sub-block 1 over sub-block 0 (W = alpha beta there), and
         // alpha (Gpre Y + F) into s (warps 0-3) or dp (warps 4-7)
         {
@@ -340,80 +326,23 @@ __global__ void __launch_bounds__(kBT, 1)
         // then p = exp(s - lse), delta = sum_j p dp (the 16 slot groups of the row add theirs by shuffles:
         // exact for the p and dp at hand, so a row whose softmax sees one slot gets g = 0), g = scale p
         // (dp - delta), and p o A, g o A in bf16
-#pragma unroll 1
-        for (int rr = 0; rr < 2; ++rr) {
-            const int row = sb * 16 + (rr ? 15 - ip : ip), lo = sb * 16;
-            float as[SPT], ad[SPT], r[SPT];
+        // Each thread takes rows lo + ip and lo + 15 - ip of its sub-block (walks of ip + 1 and 16 - ip
+        // steps) side by side.
+        {
+            const int lo = sb * 16, nA = ip + 1, nB = 16 - ip;
+            const int rowx[2] = {lo + ip, lo + 15 - ip};
+            float as[2][SPT], ad[2][SPT], r[2][SPT];
 #pragma unroll
-            for (int k = 0; k < SPT; ++k) { as[k] = 0.f; ad[k] = 0.f; r[k] = 1.f; }
-#pragma unroll 4
-            for (int u = row; u >= lo; --u) {
-                const float pv = sP[row * kBFS + u], pw = sPV[row * kBFS + u];
-                float dv[SPT];
-                if constexpr (SPT == 4) {
-                    const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kBSS + sg * 4]);
-                    dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
-                } else {
-                    const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kBSS + sg * 2]);
-                    dv[0] = d2.x; dv[1] = d2.y;
-                }
+            for (int x = 0; x < 2; ++x)
 #pragma unroll
-                for (int k = 0; k < SPT; ++k) {
-                    const float w = dv[k] * r[k];
-                    as[k] = fmaf(pv, w, as[k]);
-                    ad[k] = fmaf(pw, w, ad[k]);
-                    r[k] = fmaf(-r[k], dv[k], r[k]);
-                }
-            }
-            const long long t = a.pos0 + t0 + row;
-            const bool live = row < n;
-            const float lr = sLse[row];
-            float pj[SPT], dpj[SPT], gj[SPT], pdp = 0.f;
-#pragma unroll
-            for (int k = 0; k < SPT; ++k) {
-                const int j = sg * SPT + k;
-                const float s = a.scale * (sS[row * kBSS + j] + as[k]);
-                pj[k] = (live && t >= sdelta[j]) ? __expf(s - lr) : 0.f;
-                dpj[k] = sDP[row * kBSS + j] + ad[k];
-                pdp = fmaf(pj[k], dpj[k], pdp);
-            }
-#pragma unroll
-            for (int o = 8; o >= 1; o >>= 1) pdp += __shfl_xor_sync(hmask, pdp, o);
-#pragma unroll
-            for (int k = 0; k < SPT; ++k) {
-                const int j = sg * SPT + k;
-                gj[k] = a.scale * pj[k] * (dpj[k] - pdp);
-                sS[row * kBSS + j] = pj[k];
-                sDP[row * kBSS + j] = gj[k];
-            }
-#pragma unroll
-            for (int k = 0; k < SPT; k += 2) {
-                const int j = sg * SPT + k;
-                const float A0 = sGpre[sb * S + j] * sAl[row * kBSS + j];
-                const float A1 = sGpre[sb * S + j + 1] * sAl[row * kBSS + j + 1];
-                st_bf16x2(sPA, kBC, row, j, pj[k] * A0, pj[k + 1] * A1);
-                st_bf16x2(sGA, kBC, row, j, gj[k] * A0, gj[k + 1] * A1);
-            }
-        }
-        __syncthreads();
-        // ---- (d) G = sum_j p W and G^ = sum_j g W: diagonal sub-blocks by the walk (partials per step in
-        // registers, one transposing butterfly over the 16 slot groups each), the block of sub-block 1
-        // over sub-block 0 on the tensor cores (warp 0: G, warp 1: G^)
-#pragma unroll 1
-        for (int rr = 0; rr < 2; ++rr) {
-            const int row = sb * 16 + (rr ? 15 - ip : ip), span = row - sb * 16;
-            float qv[SPT], hv[SPT], gp[16], hp[16];
-#pragma unroll
-            for (int k = 0; k < SPT; ++k) {
-                qv[k] = sS[row * kBSS + sg * SPT + k];
-                hv[k] = sDP[row * kBSS + sg * SPT + k];
-            }
+                for (int k = 0; k < SPT; ++k) { as[x][k] = 0.f; ad[x][k] = 0.f; r[x][k] = 1.f; }
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
-                gp[i] = 0.f;
-                hp[i] = 0.f;
-                if (i <= span) {
-                    const int u = row - i;
+#pragma unroll
+                for (int x = 1; x >= 0; --x) {
+                    if (i >= (x ? nB : nA)) continue;
+                    const int row = rowx[x], u = row - i;
+                    const float pv = sP[row * kBFS + u], pw = sPV[row * kBFS + u];
                     float dv[SPT];
                     if constexpr (SPT == 4) {
                         const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kBSS + sg * 4]);
@@ -424,10 +353,94 @@ __global__ void __launch_bounds__(kBT, 1)
                     }
 #pragma unroll
                     for (int k = 0; k < SPT; ++k) {
-                        gp[i] = fmaf(qv[k], dv[k], gp[i]);
-                        hp[i] = fmaf(hv[k], dv[k], hp[i]);
-                        qv[k] = fmaf(-qv[k], dv[k], qv[k]);
-                        hv[k] = fmaf(-hv[k], dv[k], hv[k]);
+                        const float w = dv[k] * r[x][k];
+                        as[x][k] = fmaf(pv, w, as[x][k]);
+                        ad[x][k] = fmaf(pw, w, ad[x][k]);
+                        r[x][k] = fmaf(-r[x][k], dv[k], r[x][k]);
+                    }
+                }
+            }
+            float pj[2][SPT], dpj[2][SPT], pdp[2] = {0.f, 0.f};
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                const int row = rowx[x];
+                const long long t = a.pos0 + t0 + row;
+                const bool live = row < n;
+                const float lr = sLse[row];
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) {
+                    const int j = sg * SPT + k;
+                    const float sv = a.scale * (sS[row * kBSS + j] + as[x][k]);
+                    pj[x][k] = (live && t >= sdelta[j]) ? __expf(sv - lr) : 0.f;
+                    dpj[x][k] = sDP[row * kBSS + j] + ad[x][k];
+                    pdp[x] = fmaf(pj[x][k], dpj[x][k], pdp[x]);
+                }
+            }
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1) {
+                pdp[0] += __shfl_xor_sync(hmask, pdp[0], o);
+                pdp[1] += __shfl_xor_sync(hmask, pdp[1], o);
+            }
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                const int row = rowx[x];
+                float gj[SPT];
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) {
+                    const int j = sg * SPT + k;
+                    gj[k] = a.scale * pj[x][k] * (dpj[x][k] - pdp[x]);
+                    sS[row * kBSS + j] = pj[x][k];
+                    sDP[row * kBSS + j] = gj[k];
+                }
+#pragma unroll
+                for (int k = 0; k < SPT; k += 2) {
+                    const int j = sg * SPT + k;
+                    const float A0 = sGpre[sb * S + j] * sAl[row * kBSS + j];
+                    const float A1 = sGpre[sb * S + j + 1] * sAl[row * kBSS + j + 1];
+                    st_bf16x2(sPA, kBC, row, j, pj[x][k] * A0, pj[x][k + 1] * A1);
+                    st_bf16x2(sGA, kBC, row, j, gj[k] * A0, gj[k + 1] * A1);
+                }
+            }
+        }
+        __syncthreads();
+        // ---- (d) G = sum_j p W and G^ = sum_j g W: diagonal sub-blocks by the walk (partials per step in
+        // registers, one transposing butterfly over the 16 slot groups each), the block of sub-block 1
+        // over sub-block 0 on the tensor cores (warp 0: G, warp 1: G^)
+        // (rows lo + ip and lo + 15 - ip side by side, as above)
+        {
+            const int lo = sb * 16;
+            const int rowx[2] = {lo + ip, lo + 15 - ip}, spanx[2] = {ip, 15 - ip};
+            float qv[2][SPT], hv[2][SPT], gp[2][16], hp[2][16];
+#pragma unroll
+            for (int x = 0; x < 2; ++x)
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) {
+                    qv[x][k] = sS[rowx[x] * kBSS + sg * SPT + k];
+                    hv[x][k] = sDP[rowx[x] * kBSS + sg * SPT + k];
+                }
+#pragma unroll
+            for (int i = 0; i < 16; ++i) {
+#pragma unroll
+                for (int x = 0; x < 2; ++x) {
+                    gp[x][i] = 0.f;
+                    hp[x][i] = 0.f;
+                    if (i <= spanx[x]) {
+                        const int u = rowx[x] - i;
+                        float dv[SPT];
+                        if constexpr (SPT == 4) {
+                            const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kBSS + sg * 4]);
+                            dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
+                        } else {
+                            const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kBSS + sg * 2]);
+                            dv[0] = d2.x; dv[1] = d2.y;
+                        }
+#pragma unroll
+                        for (int k = 0; k < SPT; ++k) {
+                            gp[x][i] = fmaf(qv[x][k], dv[k], gp[x][i]);
+                            hp[x][i] = fmaf(hv[x][k], dv[k], hp[x][i]);
+                            qv[x][k] = fmaf(-qv[x][k], dv[k], qv[x][k]);
+                            hv[x][k] = fmaf(-hv[x][k], dv[k], hv[x][k]);
+                        }
                     }
                 }
             }
@@ -435,18 +448,22 @@ __global__ void __launch_bounds__(kBT, 1)
             for (int o = 8; o >= 1; o >>= 1) {
                 const bool up = (sg & o) != 0;
 #pragma unroll
-                for (int i = 0; i < o; ++i) {
-                    const float s1 = up ? gp[i] : gp[i + o], m1 = up ? gp[i + o] : gp[i];
-                    const float s2 = up ? hp[i] : hp[i + o], m2 = up ? hp[i + o] : hp[i];
-                    gp[i] = m1 + __shfl_xor_sync(hmask, s1, o);
-                    hp[i] = m2 + __shfl_xor_sync(hmask, s2, o);
+                for (int i = 0; i < o; ++i)
+#pragma unroll
+                    for (int x = 0; x < 2; ++x) {
+                        const float s1 = up ? gp[x][i] : gp[x][i + o], m1 = up ? gp[x][i + o] : gp[x][i];
+                        const float s2 = up ? hp[x][i] : hp[x][i + o], m2 = up ? hp[x][i + o] : hp[x][i];
+                        gp[x][i] = m1 + __shfl_xor_sync(hmask, s1, o);
+                        hp[x][i] = m2 + __shfl_xor_sync(hmask, s2, o);
+                    }
+            }
+#pragma unroll
+            for (int x = 0; x < 2; ++x)
+                if (sg <= spanx[x]) {
+                    const uint32_t off = sw_off(kBC, rowx[x], rowx[x] - sg);
+                    *reinterpret_cast<__nv_bfloat16 *>(sGm + off) = __float2bfloat16_rn(gp[x][0]);
+                    *reinterpret_cast<__nv_bfloat16 *>(sGh + off) = __float2bfloat16_rn(hp[x][0]);
                 }
-            }
-            if (sg <= span) {
-                const uint32_t off = sw_off(kBC, row, row - sg);
-                *reinterpret_cast<__nv_bfloat16 *>(sGm + off) = __float2bfloat16_rn(gp[0]);
-                *reinterpret_cast<__nv_bfloat16 *>(sGh + off) = __float2bfloat16_rn(hp[0]);
-            }
         }
         if (warp < 2) {
             const float *src = warp ? sDP : sS;
@@ -479,8 +496,10 @@ __global__ void __launch_bounds__(kBT, 1)
             }
         }
         __syncthreads();
-        // ---- (e) dQ = (g o A) K0 + G^ K into the v tile, dK = G^T Q + Wend^T mu_K into the o tile,
-        // dV = G^T dO + Wend^T mu_V into the staging tile: warp takes row block orb and OCB column blocks
+        // the tables are read: the next item's go in
+        if (threadIdx.x == 0 && nx < i1) issue_tab(nx);
+        // ---- (e) dQ = (g o A) K0 + G^ K (staged over s), the chunk's parts G^T Q of dK and G^T dO of dV:
+        // warp takes row block om0 and OCB column blocks
         {
             constexpr int OCB = DB / 4;
             const int om0 = (warp & 1) * 16, on0 = (warp >> 1) * OCB * 16;
@@ -518,7 +537,7 @@ __global__ void __launch_bounds__(kBT, 1)
                         }
                     }
                 }
-                uint8_t *dst = which == 0 ? sV : which == 1 ? sO : sOst;
+                uint8_t *dst = which == 0 ? reinterpret_cast<uint8_t *>(sS) : which == 1 ? sO : sOst;
 #pragma unroll
                 for (int cb = 0; cb < OCB; ++cb)
 #pragma unroll
@@ -528,18 +547,22 @@ __global__ void __launch_bounds__(kBT, 1)
                         st_bf16x2(dst, kBC, om0 + g8 + 8, col, acc[cb][h][2], acc[cb][h][3]);
                     }
             };
-            // dQ reads K0 and K, dK reads Q, dV reads dO: none of them reads the v or o tile, which the
-            // stores overwrite (V was read by PV, o by delta, before the barriers above)
+            // dQ first: k, K0 and V0 are then free for the next item
             out3(0);
+            tc::fence_proxy_async_smem();
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                tc::tma_store_4d(&tm_dq, sS, 0, t0, 0, bh);
+                tc::bulk_commit();
+                if (nx < i1) issue_k(nx);
+            }
             out3(1);
             out3(2);
         }
-        // ---- the chunk's adjoint contributions Z_K = (g o A)^T Q, Z_V = (p o A)^T dO, staged over the
-        // K0 and V0 tiles once every warp has finished dQ
+        // ---- the chunk's adjoint contributions Z_K = (g o A)^T Q, Z_V = (p o A)^T dO
         z_product(skv ? uDO : uQ, skv ? uPA : uGA);
-        __syncthreads();
         {
-            uint8_t *tile = skv ? sV0 : sK0;
+            uint8_t *tile = skv ? sZV : sZK;
 #pragma unroll
             for (int i = 0; i < NB2; ++i)
 #pragma unroll
@@ -553,39 +576,72 @@ __global__ void __launch_bounds__(kBT, 1)
         __syncthreads();
         if (threadIdx.x == 0) {
             const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
-            for (int db = 0; db < D / 64; ++db) {
-                tc::tma_store_3d(&tm_dq, sV + db * kBC * 128, db * 64, t0, bh);
-                tc::tma_store_3d(&tm_dk, sO + db * kBC * 128, db * 64, t0, bh);
-                tc::tma_store_3d(&tm_dv, sOst + db * kBC * 128, db * 64, t0, bh);
-                tc::tma_store_2d(&tm_z, sK0 + db * S * 128, db * 64, srow);
-                tc::tma_store_2d(&tm_z, sV0 + db * S * 128, db * 64, srow + S);
-            }
+            tc::tma_store_4d(&tm_dk, sO, 0, t0, 0, bh);
+            tc::tma_store_4d(&tm_dv, sOst, 0, t0, 0, bh);
+            tc::tma_store_3d(&tm_z, sZK, 0, srow, 0);
+            tc::tma_store_3d(&tm_z, sZV, 0, srow + S, 0);
             tc::bulk_commit();
         }
     }
     if (threadIdx.x == 0) tc::bulk_wait0();
 }
 
-// ---- Wend and A_end of every (head, chunk): thread j walks the chunk's tokens from the last back.
-// D_j(t0 + u) = Dx[t0 + u + dmax - Delta_j]; tokens past L contribute nothing (D = 0).
+// ---- the tables of every (head, chunk), one thread per slot j: Wend and A_end for the thin passes,
+// and the chain's ChunkTab record (D, alpha, beta, Gpre).  D_j(t0 + u) = Dx[t0 + u + dmax - Delta_j];
+// tokens past L contribute nothing (D = 0).
 template <int S>
 __global__ void __launch_bounds__(S) k_dbtab(DbArgs a) {
+    using Tab = ChunkTab<S>;
     const int c = blockIdx.x, h = blockIdx.y, j = threadIdx.x, nch = (a.L + kBC - 1) / kBC;
     const int t0 = c * kBC, n = min(kBC, a.L - t0);
     const float *src = a.Dx + (size_t)h * a.hs_dx + t0 + a.dmax - a.delta[(size_t)h * a.hs_delta + j];
-    uint8_t *w = reinterpret_cast<uint8_t *>(a.wtab + ((size_t)h * nch + c) * S * 64);
-    float r = 1.f;
-#pragma unroll 4
+    const size_t ti = (size_t)h * nch + c;
+    uint8_t *w = reinterpret_cast<uint8_t *>(a.wtab + ti * S * 64);
+    uint8_t *rec = a.ctab + ti * Tab::bytes;
+    float *rd = reinterpret_cast<float *>(rec + Tab::d), *ral = reinterpret_cast<float *>(rec + Tab::alpha);
+    float *rg = reinterpret_cast<float *>(rec + Tab::gpre);
+    float dv[kBC];
+#pragma unroll
+    for (int u = 0; u < kBC; ++u) {
+        dv[u] = u < n ? src[u] : 0.f;
+        rd[u * kBSS + j] = dv[u];
+        for (int col = S + j; col < kBSS; col += S) rd[u * kBSS + col] = 0.f, ral[u * kBSS + col] = 0.f;
+    }
+    // alpha_j(tau): the decay from the start of tau's 16-token sub-block through tau; Gpre: before it
+    float p = 1.f;
+    rg[j] = 1.f;
+#pragma unroll
+    for (int u = 0; u < kBC; ++u) {
+        if (u == 16) {
+            rg[S + j] = p;
+            p = 1.f;
+        }
+        p *= 1.f - dv[u];
+        ral[u * kBSS + j] = p;
+    }
+    // Wend_j(u) = D_j(u) x the decay after u to the chunk's end; beta_j(u) the same to the end of u's
+    // sub-block
+    float r = 1.f, rb = 1.f;
+#pragma unroll
     for (int u = kBC - 2; u >= 0; u -= 2) {
-        const float d1 = (u + 1 < n) ? src[u + 1] : 0.f, d0 = (u < n) ? src[u] : 0.f;
+        if (u == 14) rb = 1.f;
+        const float d1 = dv[u + 1], d0 = dv[u];
         const float w1 = d1 * r;
         r -= r * d1;
         const float w0 = d0 * r;
         r -= r * d0;
+        const float b1 = d1 * rb;
+        rb -= rb * d1;
+        const float b0 = d0 * rb;
+        rb -= rb * d0;
         *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = tc::pack_bf16x2(w0, w1);
+        *reinterpret_cast<uint32_t *>(rec + Tab::beta + wmma16::sw_off(S, j, u)) = tc::pack_bf16x2(b0, b1);
     }
-    for (int u = kBC; u < 64; u += 2) *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = 0u;
-    a.atab[((size_t)h * nch + c) * S + j] = r;
+    for (int u = kBC; u < 64; u += 2) {
+        *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = 0u;
+        *reinterpret_cast<uint32_t *>(rec + Tab::beta + wmma16::sw_off(S, j, u)) = 0u;
+    }
+    a.atab[ti * S + j] = r;
 }
 
 // ---- the two thin passes along the sequence.  One CTA per (64-column strip, K~ or V~, head) with
@@ -787,7 +843,7 @@ int sm_count_db() {
 template <int D, int S>
 cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v,
                           const void *dout, void *dq, void *dk, void *dv, cudaStream_t st) {
-    CUtensorMap tq, tk, tv, tdo, tst, tz, tdq, tdk, tdv;
+    CUtensorMap tk, tv, tst, tz, tdk, tdv;
     const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
     const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
     const uint32_t box[3] = {64, (uint32_t)kBC, 1};
@@ -795,11 +851,24 @@ cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const
     const uint64_t sdims[2] = {(uint64_t)D, (uint64_t)d.B * d.H * nch * 2 * S};
     const uint64_t sstr[1] = {(uint64_t)D * 2};
     const uint32_t sbox[2] = {64, (uint32_t)S};
-    if (!make_tmap_bf16(&tq, q, 3, dims, strides, box) || !make_tmap_bf16(&tk, k, 3, dims, strides, box) ||
-        !make_tmap_bf16(&tv, v, 3, dims, strides, box) || !make_tmap_bf16(&tdo, dout, 3, dims, strides, box) ||
+    if (!make_tmap_bf16(&tk, k, 3, dims, strides, box) || !make_tmap_bf16(&tv, v, 3, dims, strides, box) ||
         !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) || !make_tmap_bf16(&tz, a.zbuf, 2, sdims, sstr, sbox) ||
-        !make_tmap_bf16(&tdq, dq, 3, dims, strides, box) || !make_tmap_bf16(&tdk, dk, 3, dims, strides, box) ||
-        !make_tmap_bf16(&tdv, dv, 3, dims, strides, box))
+        !make_tmap_bf16(&tdk, dk, 3, dims, strides, box) || !make_tmap_bf16(&tdv, dv, 3, dims, strides, box))
+        return cudaErrorInvalidValue;
+    // the chain moves whole [32][D] and [S][D] tiles in one copy each: the 64-column blocks are a
+    // further dimension of the maps (128 bytes apart), so a box lands as [D / 64][rows][64]
+    CUtensorMap cq, ck, cv, cdo, cst, cz, cdq, cdk, cdv;
+    const uint64_t cdims[4] = {64, (uint64_t)d.L, (uint64_t)(D / 64), (uint64_t)d.B * d.H};
+    const uint64_t cstr[3] = {(uint64_t)D * 2, 128, (uint64_t)d.L * D * 2};
+    const uint32_t cbox[4] = {64, (uint32_t)kBC, (uint32_t)(D / 64), 1};
+    const uint64_t csdims[3] = {64, (uint64_t)d.B * d.H * nch * 2 * S, (uint64_t)(D / 64)};
+    const uint64_t csstr[2] = {(uint64_t)D * 2, 128};
+    const uint32_t csbox[3] = {64, (uint32_t)S, (uint32_t)(D / 64)};
+    if (!make_tmap_bf16(&cq, q, 4, cdims, cstr, cbox) || !make_tmap_bf16(&ck, k, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&cv, v, 4, cdims, cstr, cbox) || !make_tmap_bf16(&cdo, dout, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&cst, a.states, 3, csdims, csstr, csbox) ||
+        !make_tmap_bf16(&cz, a.zbuf, 3, csdims, csstr, csbox) || !make_tmap_bf16(&cdq, dq, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&cdk, dk, 4, cdims, cstr, cbox) || !make_tmap_bf16(&cdv, dv, 4, cdims, cstr, cbox))
         return cudaErrorInvalidValue;
     const int smem = BwLayout<D, S>::total, ssm = ScanLayout<S>::total;
     cudaError_t e = cudaFuncSetAttribute(k_dbchain<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
@@ -813,15 +882,18 @@ cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const
     const dim3 sgrid((unsigned)(D / 64), 2u, (unsigned)a.BH);
     k_dbscan<D, S, false><<<sgrid, kSW * 32, ssm, st>>>(tk, tv, tst, a);
     const long long items = (long long)a.BH * nch;
-    const int grid = (int)(items < sm_count_db() ? items : sm_count_db());
-    k_dbchain<D, S><<<(unsigned)grid, kBT, smem, st>>>(tq, tk, tv, tdo, tst, tz, tdq, tdk, tdv, a);
+    if (items > 0x7fffffffLL) return cudaErrorInvalidValue;   // the chain indexes its items in 32 bits
+    DbArgs ac = a;
+    ac.ipc = (int)((items + sm_count_db() - 1) / sm_count_db());
+    const int grid = (int)((items + ac.ipc - 1) / ac.ipc);
+    k_dbchain<D, S><<<(unsigned)grid, kBT, smem, st>>>(cq, ck, cv, cdo, cst, cz, cdq, cdk, cdv, ac);
     k_dbscan<D, S, true><<<sgrid, kSW * 32, ssm, st>>>(tdk, tdv, tz, a);
     return cudaGetLastError();
 }
 
 // the pieces of the backward's workspace: states, Z, Wend tables, A_end tables
 struct DbWs {
-    size_t states, z, wtab, atab, total;
+    size_t states, z, wtab, atab, ctab, total;
 };
 
 DbWs db_ws(const OpDims &d) {
@@ -832,7 +904,9 @@ DbWs db_ws(const OpDims &d) {
     w.z = per;
     w.wtab = 2 * per;
     w.atab = w.wtab + align_up(ntab * nch * d.S * 64 * sizeof(__nv_bfloat16), 256);
-    w.total = w.atab + align_up(ntab * nch * d.S * sizeof(float), 256);
+    w.ctab = w.atab + align_up(ntab * nch * d.S * sizeof(float), 256);
+    const size_t tab_bytes = d.S == 32 ? (size_t)ChunkTab<32>::bytes : (size_t)ChunkTab<64>::bytes;
+    w.total = w.ctab + align_up(ntab * nch * tab_bytes, 256);
     return w;
 }
 
@@ -847,7 +921,7 @@ cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, co
     const DbWs w = db_ws(d);
     char *base = static_cast<char *>(ws);
     DbArgs a;
-    a.L = d.L; a.H = d.H; a.BH = d.B * d.H; a.pos0 = pos0; a.scale = d.scale; a.dmax = dmax;
+    a.L = d.L; a.H = d.H; a.BH = d.B * d.H; a.ipc = 1; a.pos0 = pos0; a.scale = d.scale; a.dmax = dmax;
     a.Dx = Dx; a.delta = delta; a.hs_dx = hs_dx; a.hs_delta = hs_delta;
     a.lse = lse;
     a.ntab = (hs_dx != 0 || hs_delta != 0) ? d.H : 1;
@@ -856,6 +930,7 @@ cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, co
     a.zbuf = reinterpret_cast<__nv_bfloat16 *>(base + w.z);
     a.wtab = reinterpret_cast<__nv_bfloat16 *>(base + w.wtab);
     a.atab = reinterpret_cast<float *>(base + w.atab);
+    a.ctab = reinterpret_cast<uint8_t *>(base + w.ctab);
     a.err = device_error_word();
     if (d.dk == 64) return d.S == 32 ? launch_dbwd_t<64, 32>(d, a, q, k, v, dout, dq, dk, dv, st)
                                      : launch_dbwd_t<64, 64>(d, a, q, k, v, dout, dq, dk, dv, st);
