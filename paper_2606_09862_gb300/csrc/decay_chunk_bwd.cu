@@ -118,6 +118,32 @@ struct StateMap {
     __device__ static int cb0(int w) { return ((w & 3) * NB2) % DB; }
 };
 
+// N (2 or 4) consecutive 32-bit words of shared memory in one access (16- or 8-byte aligned)
+template <typename T, int N>
+__device__ __forceinline__ void lds_vec(const T *p, T (&v)[N]) {
+    static_assert(N == 2 || N == 4, "vector width");
+    if constexpr (N == 4) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(p);
+        v[0] = __builtin_bit_cast(T, x.x); v[1] = __builtin_bit_cast(T, x.y);
+        v[2] = __builtin_bit_cast(T, x.z); v[3] = __builtin_bit_cast(T, x.w);
+    } else {
+        const uint2 x = *reinterpret_cast<const uint2 *>(p);
+        v[0] = __builtin_bit_cast(T, x.x); v[1] = __builtin_bit_cast(T, x.y);
+    }
+}
+template <int N>
+__device__ __forceinline__ void sts_vec(float *p, const float (&v)[N]) {
+    if constexpr (N == 4) *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    else *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+}
+// N bf16 (rounded from fp32) to consecutive columns of a swizzled tile row (within one 16-byte chunk)
+template <int N>
+__device__ __forceinline__ void st_bf16_vec(uint8_t *p, const float (&v)[N]) {
+    if constexpr (N == 4)
+        *reinterpret_cast<uint2 *>(p) = make_uint2(tc::pack_bf16x2(v[0], v[1]), tc::pack_bf16x2(v[2], v[3]));
+    else *reinterpret_cast<uint32_t *>(p) = tc::pack_bf16x2(v[0], v[1]);
+}
+
 template <int D, int S>
 __global__ void __launch_bounds__(kBT, 1)
     k_dbchain(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
@@ -326,53 +352,62 @@ __global__ void __launch_bounds__(kBT, 1)
         // then p = exp(s - lse), delta = sum_j p dp (the 16 slot groups of the row add theirs by shuffles:
         // exact for the p and dp at hand, so a row whose softmax sees one slot gets g = 0), g = scale p
         // (dp - delta), and p o A, g o A in bf16
-        // Each thread takes rows lo + ip and lo + 15 - ip of its sub-block (walks of ip + 1 and 16 - ip
-        // steps) side by side.
+        // Each thread takes rows lo + ip and lo + 15 - ip of its sub-block and walks u down from the
+        // sub-block's last token: one load of D_j(u) serves both rows (and both half-warps, which share
+        // the sub-block), and P, PV come four tokens at a time.
         {
-            const int lo = sb * 16, nA = ip + 1, nB = 16 - ip;
-            const int rowx[2] = {lo + ip, lo + 15 - ip};
+            const int lo = sb * 16;
+            const int rowx[2] = {lo + ip, lo + 15 - ip}, spanx[2] = {ip, 15 - ip};
             float as[2][SPT], ad[2][SPT], r[2][SPT];
 #pragma unroll
             for (int x = 0; x < 2; ++x)
 #pragma unroll
                 for (int k = 0; k < SPT; ++k) { as[x][k] = 0.f; ad[x][k] = 0.f; r[x][k] = 1.f; }
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
+            for (int q4 = 3; q4 >= 0; --q4) {
+                if (4 * q4 > spanx[1]) continue;
+                float pq[2][4], wq[2][4];
 #pragma unroll
-                for (int x = 1; x >= 0; --x) {
-                    if (i >= (x ? nB : nA)) continue;
-                    const int row = rowx[x], u = row - i;
-                    const float pv = sP[row * kBFS + u], pw = sPV[row * kBFS + u];
+                for (int x = 0; x < 2; ++x) {
+                    lds_vec(&sP[rowx[x] * kBFS + lo + 4 * q4], pq[x]);
+                    lds_vec(&sPV[rowx[x] * kBFS + lo + 4 * q4], wq[x]);
+                }
+#pragma unroll
+                for (int e = 3; e >= 0; --e) {
+                    const int uo = 4 * q4 + e;
+                    if (uo > spanx[1]) continue;
                     float dv[SPT];
-                    if constexpr (SPT == 4) {
-                        const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kBSS + sg * 4]);
-                        dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
-                    } else {
-                        const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kBSS + sg * 2]);
-                        dv[0] = d2.x; dv[1] = d2.y;
-                    }
+                    lds_vec(&sD[(lo + uo) * kBSS + sg * SPT], dv);
 #pragma unroll
-                    for (int k = 0; k < SPT; ++k) {
-                        const float w = dv[k] * r[x][k];
-                        as[x][k] = fmaf(pv, w, as[x][k]);
-                        ad[x][k] = fmaf(pw, w, ad[x][k]);
-                        r[x][k] = fmaf(-r[x][k], dv[k], r[x][k]);
+                    for (int x = 0; x < 2; ++x) {
+                        if (uo > spanx[x]) continue;
+#pragma unroll
+                        for (int k = 0; k < SPT; ++k) {
+                            const float w = dv[k] * r[x][k];
+                            as[x][k] = fmaf(pq[x][e], w, as[x][k]);
+                            ad[x][k] = fmaf(wq[x][e], w, ad[x][k]);
+                            r[x][k] = fmaf(-r[x][k], dv[k], r[x][k]);
+                        }
                     }
                 }
             }
             float pj[2][SPT], dpj[2][SPT], pdp[2] = {0.f, 0.f};
+            int dlt[SPT];
+            lds_vec(&sdelta[sg * SPT], dlt);
 #pragma unroll
             for (int x = 0; x < 2; ++x) {
                 const int row = rowx[x];
                 const long long t = a.pos0 + t0 + row;
                 const bool live = row < n;
                 const float lr = sLse[row];
+                float sv[SPT], dpv[SPT];
+                lds_vec(&sS[row * kBSS + sg * SPT], sv);
+                lds_vec(&sDP[row * kBSS + sg * SPT], dpv);
 #pragma unroll
                 for (int k = 0; k < SPT; ++k) {
-                    const int j = sg * SPT + k;
-                    const float sv = a.scale * (sS[row * kBSS + j] + as[x][k]);
-                    pj[x][k] = (live && t >= sdelta[j]) ? __expf(sv - lr) : 0.f;
-                    dpj[x][k] = sDP[row * kBSS + j] + ad[x][k];
+                    const float sc = a.scale * (sv[k] + as[x][k]);
+                    pj[x][k] = (live && t >= dlt[k]) ? __expf(sc - lr) : 0.f;
+                    dpj[x][k] = dpv[k] + ad[x][k];
                     pdp[x] = fmaf(pj[x][k], dpj[x][k], pdp[x]);
                 }
             }
@@ -381,69 +416,63 @@ __global__ void __launch_bounds__(kBT, 1)
                 pdp[0] += __shfl_xor_sync(hmask, pdp[0], o);
                 pdp[1] += __shfl_xor_sync(hmask, pdp[1], o);
             }
+            float gpre[SPT];
+            lds_vec(&sGpre[sb * S + sg * SPT], gpre);
 #pragma unroll
             for (int x = 0; x < 2; ++x) {
                 const int row = rowx[x];
-                float gj[SPT];
+                float gj[SPT], al[SPT], pa[SPT], ga[SPT];
+                lds_vec(&sAl[row * kBSS + sg * SPT], al);
 #pragma unroll
                 for (int k = 0; k < SPT; ++k) {
-                    const int j = sg * SPT + k;
                     gj[k] = a.scale * pj[x][k] * (dpj[x][k] - pdp[x]);
-                    sS[row * kBSS + j] = pj[x][k];
-                    sDP[row * kBSS + j] = gj[k];
+                    const float A = gpre[k] * al[k];
+                    pa[k] = pj[x][k] * A;
+                    ga[k] = gj[k] * A;
                 }
-#pragma unroll
-                for (int k = 0; k < SPT; k += 2) {
-                    const int j = sg * SPT + k;
-                    const float A0 = sGpre[sb * S + j] * sAl[row * kBSS + j];
-                    const float A1 = sGpre[sb * S + j + 1] * sAl[row * kBSS + j + 1];
-                    st_bf16x2(sPA, kBC, row, j, pj[x][k] * A0, pj[x][k + 1] * A1);
-                    st_bf16x2(sGA, kBC, row, j, gj[k] * A0, gj[k + 1] * A1);
-                }
+                sts_vec(&sS[row * kBSS + sg * SPT], pj[x]);
+                sts_vec(&sDP[row * kBSS + sg * SPT], gj);
+                st_bf16_vec(sPA + sw_off(kBC, row, sg * SPT), pa);
+                st_bf16_vec(sGA + sw_off(kBC, row, sg * SPT), ga);
             }
         }
         __syncthreads();
         // ---- (d) G = sum_j p W and G^ = sum_j g W: diagonal sub-blocks by the walk (partials per step in
         // registers, one transposing butterfly over the 16 slot groups each), the block of sub-block 1
         // over sub-block 0 on the tensor cores (warp 0: G, warp 1: G^)
-        // (rows lo + ip and lo + 15 - ip side by side, as above)
+        // (rows lo + ip and lo + 15 - ip walk u down together, as above; the partial sums are kept by u)
         {
             const int lo = sb * 16;
             const int rowx[2] = {lo + ip, lo + 15 - ip}, spanx[2] = {ip, 15 - ip};
             float qv[2][SPT], hv[2][SPT], gp[2][16], hp[2][16];
 #pragma unroll
-            for (int x = 0; x < 2; ++x)
+            for (int x = 0; x < 2; ++x) {
+                lds_vec(&sS[rowx[x] * kBSS + sg * SPT], qv[x]);
+                lds_vec(&sDP[rowx[x] * kBSS + sg * SPT], hv[x]);
+            }
 #pragma unroll
-                for (int k = 0; k < SPT; ++k) {
-                    qv[x][k] = sS[rowx[x] * kBSS + sg * SPT + k];
-                    hv[x][k] = sDP[rowx[x] * kBSS + sg * SPT + k];
-                }
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
+            for (int uo = 15; uo >= 0; --uo) {
 #pragma unroll
                 for (int x = 0; x < 2; ++x) {
-                    gp[x][i] = 0.f;
-                    hp[x][i] = 0.f;
-                    if (i <= spanx[x]) {
-                        const int u = rowx[x] - i;
-                        float dv[SPT];
-                        if constexpr (SPT == 4) {
-                            const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kBSS + sg * 4]);
-                            dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
-                        } else {
-                            const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kBSS + sg * 2]);
-                            dv[0] = d2.x; dv[1] = d2.y;
-                        }
+                    gp[x][uo] = 0.f;
+                    hp[x][uo] = 0.f;
+                }
+                if (uo > spanx[1]) continue;
+                float dv[SPT];
+                lds_vec(&sD[(lo + uo) * kBSS + sg * SPT], dv);
 #pragma unroll
-                        for (int k = 0; k < SPT; ++k) {
-                            gp[x][i] = fmaf(qv[x][k], dv[k], gp[x][i]);
-                            hp[x][i] = fmaf(hv[x][k], dv[k], hp[x][i]);
-                            qv[x][k] = fmaf(-qv[x][k], dv[k], qv[x][k]);
-                            hv[x][k] = fmaf(-hv[x][k], dv[k], hv[x][k]);
-                        }
+                for (int x = 0; x < 2; ++x) {
+                    if (uo > spanx[x]) continue;
+#pragma unroll
+                    for (int k = 0; k < SPT; ++k) {
+                        gp[x][uo] = fmaf(qv[x][k], dv[k], gp[x][uo]);
+                        hp[x][uo] = fmaf(hv[x][k], dv[k], hp[x][uo]);
+                        qv[x][k] = fmaf(-qv[x][k], dv[k], qv[x][k]);
+                        hv[x][k] = fmaf(-hv[x][k], dv[k], hv[x][k]);
                     }
                 }
             }
+            // transposing butterfly: slot group sg ends with the row's total at u = lo + sg
 #pragma unroll
             for (int o = 8; o >= 1; o >>= 1) {
                 const bool up = (sg & o) != 0;
@@ -460,7 +489,7 @@ __global__ void __launch_bounds__(kBT, 1)
 #pragma unroll
             for (int x = 0; x < 2; ++x)
                 if (sg <= spanx[x]) {
-                    const uint32_t off = sw_off(kBC, rowx[x], rowx[x] - sg);
+                    const uint32_t off = sw_off(kBC, rowx[x], lo + sg);
                     *reinterpret_cast<__nv_bfloat16 *>(sGm + off) = __float2bfloat16_rn(gp[x][0]);
                     *reinterpret_cast<__nv_bfloat16 *>(sGh + off) = __float2bfloat16_rn(hp[x][0]);
                 }
