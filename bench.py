@@ -571,39 +571,45 @@ def measure_block(bla, torch, dev, timed):
 
 
 # Nominal fp32 SIMT peak of the part: 152 SMs x 128 fp32 lanes x 2 flops (FMA) x 2.07 GHz.
-FP32_SIMT_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 
 
 def measure_decay(bla, torch, dev, timed, peaks):
     """The state decay of Sec. 3.3 (absolute form): the LM-layer prefill (B=8, H=8, L=4096, d=128,
-    M=64, S=64, T=1024, bf16) and one decode step at B=256, H=16, d=128, M=128, S=128, T=4096,
-    pos = 4096, from a random fp32 slot state.  The forward is a scan on the CUDA cores: its flops
-    are 10 S d per token and head (state update 3 + score 2 for K and for V, FMA = 2); the decode
-    reads and writes the whole slot state once."""
+    M=64, S=64, T=1024, bf16), its backward, and one decode step at B=256, H=16, d=128, M=128, S=128,
+    T=4096, pos = 4096, from a random fp32 slot state.
+
+    The forward and backward run the chunked kernels (warp-level bf16 MMAs for the contractions,
+    triangle walks on the CUDA cores); they are bound by latency, not by a roof, so both fractions
+    are reported.  FLOPs count the contractions per token and head (c = chunk length, S slots):
+    forward (c = 64) P, Y, O and the two state updates, 4 c d + 8 S d; backward (c = 32) P, Y, PV,
+    YV, dQ, the chunk parts of dK and dV, Z, the state pass and the adjoint pass,
+    10 c d + 18 S d.  Bytes are the tensors a call must read and write once: q, k, v, o and lse
+    forward; q, k, v, dO, lse, dq, dk, dv backward.  The decode reads and writes the whole slot
+    state once."""
     from paper_2606_09862_gb300.inputs import WORKLOADS, make_decode_step, make_dout, make_qkv, make_slot_state
     w = WORKLOADS["decay_bf16_lm"]
     q, k, v = (torch.from_numpy(x).to(torch.bfloat16).to(dev) for x in make_qkv(w.B, w.H, w.L, w.d, "bf16", seed=0))
     par = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16, phase_mode="absolute")
     ws = torch.empty(bla.bla_workspace_bytes(par, bla.BLA_WS_DECAY_FORWARD), dtype=torch.uint8, device=dev)
     o = torch.empty_like(v)
+    units = w.B * w.H * w.L
+
+    def entry(ms, flops, nbytes):
+        tf = flops / (ms / 1000.0) / 1e12
+        gbs = nbytes / (ms / 1000.0) / 1e9
+        return {"ms": ms, "tokens_per_s": w.B * w.L / (ms / 1000.0), "tflops": tf, "flops": flops, "gbs": gbs,
+                "bytes": nbytes, "bound": "latency", "frac_tensor": tf / peaks["bf16_tflops"],
+                "frac_hbm": gbs / peaks["hbm_gbs"]}
+
     ms = timed(lambda: bla.bla_decay_forward(q, k, v, w.M, w.S, w.T, workspace=ws, out=o))
-    flops = 10.0 * w.B * w.H * w.L * w.S * w.d
-    tf = flops / (ms / 1000.0) / 1e12
-    res = {"forward": {"ms": ms, "tokens_per_s": w.B * w.L / (ms / 1000.0), "tflops_fp32": tf, "flops": flops,
-                       "bound": "alu", "frac_alu": tf / FP32_SIMT_PEAK_TFLOPS,
-                       "alu_peak_tflops": FP32_SIMT_PEAK_TFLOPS},
+    res = {"forward": entry(ms, float(units) * (4 * 64 * w.d + 8 * w.S * w.d), float(units) * (8 * w.d + 4)),
            "shape": "B=%d H=%d L=%d d=%d M=%d S=%d T=%d bf16 absolute+decay" % (w.B, w.H, w.L, w.d, w.M, w.S, w.T)}
-    # backward: two dot scans (scores, dp) and three reduce scans (dq, dk, dv), 25 S d flops per
-    # token-head (each scan 5 S d)
     o, lse, _ = bla.bla_decay_forward(q, k, v, w.M, w.S, w.T, workspace=ws)
     do = torch.from_numpy(make_dout(w.B, w.H, w.L, w.d, "bf16", seed=0)).to(torch.bfloat16).to(dev)
     parb = bla.make_params(w.B, w.H, w.L, w.d, w.d, w.M, w.S, w.T, dtype=torch.bfloat16, phase_mode="absolute")
     wsb = torch.empty(bla.bla_workspace_bytes(parb, bla.BLA_WS_DECAY_BACKWARD), dtype=torch.uint8, device=dev)
     ms_b = timed(lambda: bla.bla_decay_backward(q, k, v, o, do, lse, w.M, w.S, w.T, workspace=wsb))
-    fb = 25.0 * w.B * w.H * w.L * w.S * w.d
-    res["backward"] = {"ms": ms_b, "tokens_per_s": w.B * w.L / (ms_b / 1000.0),
-                       "tflops_fp32": fb / (ms_b / 1000.0) / 1e12, "flops": fb, "bound": "alu",
-                       "frac_alu": fb / (ms_b / 1000.0) / 1e12 / FP32_SIMT_PEAK_TFLOPS}
+    res["backward"] = entry(ms_b, float(units) * (10 * 32 * w.d + 18 * w.S * w.d), float(units) * (14 * w.d + 4))
     del q, k, v, ws, o, lse, do, wsb
     wd = WORKLOADS["decay_decode_bf16"]
     qd, kd, vd = (torch.from_numpy(x).to(torch.bfloat16).to(dev)

@@ -57,6 +57,14 @@ struct ChunkTab {
     static_assert(bytes % 16 == 0, "bulk copies move multiples of 16 bytes");
 };
 
+// The thin passes' tables of one (head, chunk): Wend (bf16, swizzled [S][64], u < 32 used), then
+// A_end (fp32 [S]), one bulk copy.
+template <int S>
+struct EndTab {
+    static constexpr int wend = 0, aend = S * 128, bytes = aend + S * 4;
+    static_assert(bytes % 16 == 0, "bulk copies move multiples of 16 bytes");
+};
+
 template <int D, int S>
 struct BwLayout {
     static constexpr int kTile = kBC * D * 2;          // one [32][D] bf16 tile
@@ -100,8 +108,7 @@ struct DbArgs {
     const float *lse;           // [BH][L], from the forward
     int ntab;                   // heads with their own tables (1 when the heads share one period)
     uint8_t *ctab;              // [ntab][nch] ChunkTab records of the chain
-    __nv_bfloat16 *wtab;        // [ntab][nch][S][64] bf16, 128-byte swizzled (u < 32 used): Wend
-    float *atab;                // [ntab][nch][S]: A_end
+    uint8_t *etab;              // [ntab][nch] EndTab records of the thin passes
     __nv_bfloat16 *states;      // [BH][nch][2][S][D]: the state entering each chunk
     __nv_bfloat16 *zbuf;        // [BH][nch][2][S][D]: each chunk's adjoint contributions (g o A)^T Q, (p o A)^T dO
     int *err;
@@ -625,7 +632,7 @@ __global__ void __launch_bounds__(S) k_dbtab(DbArgs a) {
     const int t0 = c * kBC, n = min(kBC, a.L - t0);
     const float *src = a.Dx + (size_t)h * a.hs_dx + t0 + a.dmax - a.delta[(size_t)h * a.hs_delta + j];
     const size_t ti = (size_t)h * nch + c;
-    uint8_t *w = reinterpret_cast<uint8_t *>(a.wtab + ti * S * 64);
+    uint8_t *w = a.etab + ti * EndTab<S>::bytes + EndTab<S>::wend;
     uint8_t *rec = a.ctab + ti * Tab::bytes;
     float *rd = reinterpret_cast<float *>(rec + Tab::d), *ral = reinterpret_cast<float *>(rec + Tab::alpha);
     float *rg = reinterpret_cast<float *>(rec + Tab::gpre);
@@ -670,7 +677,7 @@ __global__ void __launch_bounds__(S) k_dbtab(DbArgs a) {
         *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = 0u;
         *reinterpret_cast<uint32_t *>(rec + Tab::beta + wmma16::sw_off(S, j, u)) = 0u;
     }
-    a.atab[ti * S + j] = r;
+    reinterpret_cast<float *>(a.etab + ti * EndTab<S>::bytes + EndTab<S>::aend)[j] = r;
 }
 
 // ---- the two thin passes along the sequence.  One CTA per (64-column strip, K~ or V~, head) with
@@ -688,11 +695,11 @@ template <int S>
 struct ScanLayout {
     static constexpr int kT = kBC * 128;                    // [32][64] bf16 tile
     static constexpr int kW = S * 128;                      // [S][64] bf16 tile (Wend image, state strip)
-    static constexpr int stage = kW + kW + kT;              // z (reverse only) | Wend | k or dk
+    // a stage: z (reverse only) | k or dk | the EndTab record, rounded up to whole 1024-byte blocks
+    static constexpr int stage = ((kW + kT + EndTab<S>::bytes) + 1023) / 1024 * 1024;
     static constexpr int mu = kNS * stage;                  // bf16 [S][64]: mu (reverse)
     static constexpr int out = mu + kW;                     // 2 staging tiles: [S][64] (state) or [32][64]
-    static constexpr int ae = out + 2 * kW;                 // fp32 [kNS][S]: A_end of each stage
-    static constexpr int bars = ae + kNS * S * 4;
+    static constexpr int bars = out + 2 * kW;
     static constexpr int total = bars + 8 * kNS;
     static_assert(stage % 1024 == 0 && mu % 1024 == 0 && out % 1024 == 0, "swizzled tiles need 1024-byte alignment");
 };
@@ -718,28 +725,29 @@ __global__ void __launch_bounds__(kSW * 32)
     const CUtensorMap *tx = kv ? &tm_x1 : &tm_x0;   // k / v (forward) or dk / dv (reverse)
     uint64_t *full = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
     uint8_t *sMu = dsm + Lay::mu, *sOut = dsm + Lay::out;
-    // stage s: Z strip (reverse) at +0, Wend at +kW, the [32][64] tile at +2 kW; its A_end apart
+    // stage s: Z strip (reverse) at +0, the [32][64] tile at +kW, the EndTab record at +kW + kT
     auto sz = [&](int s) { return dsm + s * Lay::stage; };
-    auto sw = [&](int s) { return dsm + s * Lay::stage + Lay::kW; };
-    auto sx = [&](int s) { return dsm + s * Lay::stage + 2 * Lay::kW; };
-    auto sa = [&](int s) { return reinterpret_cast<float *>(dsm + Lay::ae + s * S * 4); };
+    auto sx = [&](int s) { return dsm + s * Lay::stage + Lay::kW; };
+    auto sw = [&](int s) { return dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::wend; };
+    auto sa = [&](int s) {
+        return reinterpret_cast<float *>(dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::aend);
+    };
     auto chunk_of = [&](int i) { return REV ? nch - 1 - i : i; };
     auto issue = [&](int i) {
         const int s = i % kNS, c = chunk_of(i);
         const size_t ti = (size_t)tab * nch + c;
-        const uint32_t bytes = (uint32_t)(Lay::kW + Lay::kT + S * 4 + (REV ? Lay::kW : 0));
+        const uint32_t bytes = (uint32_t)(Lay::kT + EndTab<S>::bytes + (REV ? Lay::kW : 0));
         tc::mbar_arrive_expect_tx(&full[s], bytes);
         if (REV) tc::tma_load_2d(sz(s), &tm_st, &full[s], x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
-        tc::bulk_load(sw(s), a.wtab + ti * S * 64, (uint32_t)Lay::kW, &full[s]);
         tc::tma_load_3d(sx(s), tx, &full[s], x, c * kBC, bh);
-        tc::bulk_load(sa(s), a.atab + ti * S, (uint32_t)(S * 4), &full[s]);
+        tc::bulk_load(sw(s), a.etab + ti * EndTab<S>::bytes, (uint32_t)EndTab<S>::bytes, &full[s]);
     };
     if (threadIdx.x == 0) {
         for (int s = 0; s < kNS; ++s) tc::mbar_init(&full[s], 1);
         tc::fence_barrier_init();
     }
     __syncthreads();
-    if (threadIdx.x == 0)
+    if (threadIdx.x == 32)
         for (int i = 0; i < kNS && i < nch; ++i) issue(i);
 
     const int r0 = (warp % M::WR) * 16, c0 = (warp / M::WR) * M::NC;
@@ -856,8 +864,9 @@ __global__ void __launch_bounds__(kSW * 32)
                 tc::tma_store_3d(tx, sOut + ob * Lay::kW, x, c * kBC, bh);
                 tc::bulk_commit();
             }
-            if (i + kNS < nch) issue(i + kNS);
         }
+        // the loads come from another warp: each TMA issue holds its thread for a while
+        if (threadIdx.x == 32 && i + kNS < nch) issue(i + kNS);
     }
     if (threadIdx.x == 0) tc::bulk_wait0();
 }
@@ -922,7 +931,7 @@ cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const
 
 // the pieces of the backward's workspace: states, Z, Wend tables, A_end tables
 struct DbWs {
-    size_t states, z, wtab, atab, ctab, total;
+    size_t states, z, etab, ctab, total;
 };
 
 DbWs db_ws(const OpDims &d) {
@@ -931,9 +940,9 @@ DbWs db_ws(const OpDims &d) {
     DbWs w;
     w.states = 0;
     w.z = per;
-    w.wtab = 2 * per;
-    w.atab = w.wtab + align_up(ntab * nch * d.S * 64 * sizeof(__nv_bfloat16), 256);
-    w.ctab = w.atab + align_up(ntab * nch * d.S * sizeof(float), 256);
+    w.etab = 2 * per;
+    const size_t end_bytes = d.S == 32 ? (size_t)EndTab<32>::bytes : (size_t)EndTab<64>::bytes;
+    w.ctab = w.etab + align_up(ntab * nch * end_bytes, 256);
     const size_t tab_bytes = d.S == 32 ? (size_t)ChunkTab<32>::bytes : (size_t)ChunkTab<64>::bytes;
     w.total = w.ctab + align_up(ntab * nch * tab_bytes, 256);
     return w;
@@ -957,8 +966,7 @@ cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, co
     if (a.ntab > 1 && !d.periods) return cudaErrorInvalidValue;   // the tables are sized per head only then
     a.states = reinterpret_cast<__nv_bfloat16 *>(base + w.states);
     a.zbuf = reinterpret_cast<__nv_bfloat16 *>(base + w.z);
-    a.wtab = reinterpret_cast<__nv_bfloat16 *>(base + w.wtab);
-    a.atab = reinterpret_cast<float *>(base + w.atab);
+    a.etab = reinterpret_cast<uint8_t *>(base + w.etab);
     a.ctab = reinterpret_cast<uint8_t *>(base + w.ctab);
     a.err = device_error_word();
     if (d.dk == 64) return d.S == 32 ? launch_dbwd_t<64, 32>(d, a, q, k, v, dout, dq, dk, dv, st)
