@@ -520,10 +520,8 @@ struct DecayWs {
     float *lse;
     int hs_dx, hs_delta;   // per-head strides of Dx and delta (0 when the heads share one period)
     float *g = nullptr;    // backward: dp, then g = scale ds, [BH][S][L]
-    // chunked forward (decay_chunk.cu): per-segment state deltas and decay products, entering states
-    float *seg_delta = nullptr, *seg_decay = nullptr, *win = nullptr;
-    // chunked backward (decay_chunk_bwd.cu): chunk states, adjoint contributions and tables
-    void *chunk_bwd = nullptr;
+    // chunked forward and backward (decay_chunk.cu): chunk states, adjoint contributions and tables
+    void *chunk = nullptr;
 };
 
 size_t decay_table_len(const OpDims &d) { return (size_t)d.L + (size_t)host_dmax(d) + 1; }
@@ -544,16 +542,11 @@ size_t carve(const OpDims &d, bool decode, bool own_lse, char *base, DecayWs *w,
     w->sc = nullptr;
     w->lse = nullptr;
     if (!decode && backward && decay_chunk_supported(d)) {
-        w->chunk_bwd = take(decay_chunk_bwd_ws_bytes(d));
+        w->chunk = take(decay_chunk_bwd_ws_bytes(d));
     } else if (!decode && !backward && decay_chunk_supported(d)) {
-        // the chunked forward keeps its scores on chip: only the segment states travel
-        const size_t BH = (size_t)d.B * d.H, G = (size_t)decay_chunk_plan(d).G;
-        if (own_lse) w->lse = reinterpret_cast<float *>(take(sizeof(float) * BH * (size_t)d.L));
-        if (G > 1) {
-            w->seg_delta = reinterpret_cast<float *>(take(sizeof(float) * BH * G * 2 * d.S * d.dk));
-            w->seg_decay = reinterpret_cast<float *>(take(sizeof(float) * BH * G * d.S));
-            w->win = reinterpret_cast<float *>(take(sizeof(float) * BH * G * 2 * d.S * d.dk));
-        }
+        // the chunked forward keeps its scores on chip: the chunk states and tables travel
+        if (own_lse) w->lse = reinterpret_cast<float *>(take(sizeof(float) * (size_t)d.B * d.H * (size_t)d.L));
+        w->chunk = take(decay_chunk_fwd_ws_bytes(d));
     } else if (!decode) {
         const size_t BH = (size_t)d.B * d.H;
         w->sc = reinterpret_cast<float *>(take(sizeof(float) * BH * d.S * (size_t)(d.L > 0 ? d.L : 1)));
@@ -700,7 +693,7 @@ cudaError_t launch_decay_backward(const OpDims &d, long long pos0, const void *q
     if (e != cudaSuccess) return e;
     if (decay_chunk_supported(d))
         return launch_decay_chunk_bwd(d, pos0, dmax, w.Dx, w.delta, w.hs_dx, w.hs_delta, q, k, v, dout, lse, dq, dk,
-                                      dv, w.chunk_bwd, st);
+                                      dv, w.chunk, st);
     return d.dtype == BLA_BF16 ? backward_run<__nv_bfloat16>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st)
                                : backward_run<float>(d, w, pos0, q, k, v, o, dout, lse, dq, dk, dv, dmax, st);
 }
@@ -722,7 +715,7 @@ cudaError_t launch_decay_forward(const OpDims &d, long long pos0, const void *q,
     if (e != cudaSuccess) return e;
     if (decay_chunk_supported(d))
         return launch_decay_chunk(d, pos0, dmax, w.Dx, w.delta, w.hs_dx, w.hs_delta, q, k, v, o, lse ? lse : w.lse,
-                                  state_in, state_out, w.seg_delta, w.seg_decay, w.win, st);
+                                  state_in, state_out, w.chunk, st);
     e = d.dtype == BLA_BF16 ? kscan_dispatch<__nv_bfloat16>(d, w, q, k, dmax, state_in, state_out, st)
                             : kscan_dispatch<float>(d, w, q, k, dmax, state_in, state_out, st);
     if (e != cudaSuccess) return e;

@@ -14,22 +14,17 @@ cudaError_t launch_decay_forward(const OpDims &d, long long pos0, const void *q,
                                  float *lse, const float *state_in, float *state_out, void *ws, cudaStream_t st);
 cudaError_t launch_decay_decode(const OpDims &d, long long pos, const void *q, const void *k, const void *v,
                                 float *state, void *o, void *ws, cudaStream_t st);
-// The chunked bf16 forward of the decayed form (decay_chunk.cu): 64-token chunks with the
-// contractions on the tensor cores, for d_k = d_v in {64, 128} and S in {32, 64}.  Each head's
-// sequence runs as G segments of cps chunks (state deltas, a scan, then the outputs).
-struct DcPlan {
-    int G, cps;
-};
+// The chunked bf16 forward and backward of the decayed form (decay_chunk.cu), for d_k = d_v in
+// {64, 128} and S in {32, 64}, in 32-token chunks: tables per (head, chunk), a pass along the
+// sequence for the state entering every chunk, the per-chunk work in parallel over all SMs and, in
+// the backward, a reverse pass for the adjoint states.  The workspaces (decay_chunk_fwd_ws_bytes,
+// decay_chunk_bwd_ws_bytes) hold the chunk states, the backward's per-chunk adjoint contributions
+// (both bf16) and the tables.
 bool decay_chunk_supported(const OpDims &d);
-DcPlan decay_chunk_plan(const OpDims &d);
+size_t decay_chunk_fwd_ws_bytes(const OpDims &d);
 cudaError_t launch_decay_chunk(const OpDims &d, long long pos0, int dmax, const float *Dx, const int *delta,
                                int hs_dx, int hs_delta, const void *q, const void *k, const void *v, void *o,
-                               float *lse, const float *state_in, float *state_out, float *seg_delta,
-                               float *seg_decay, float *win, cudaStream_t st);
-// Its backward (decay_chunk_bwd.cu), for the same shapes, in 32-token chunks: tables, a pass for the
-// state entering every chunk, the per-chunk chains in parallel, and a reverse pass for the adjoint
-// states; the workspace (decay_chunk_bwd_ws_bytes) holds the chunk states, the chunks' adjoint
-// contributions (both bf16) and the tables.
+                               float *lse, const float *state_in, float *state_out, void *ws, cudaStream_t st);
 size_t decay_chunk_bwd_ws_bytes(const OpDims &d);
 cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, const float *Dx, const int *delta,
                                    int hs_dx, int hs_delta, const void *q, const void *k, const void *v,

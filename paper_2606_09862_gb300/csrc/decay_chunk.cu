@@ -1,29 +1,40 @@
-// decay_chunk.cu -- the state-decayed forward (Sec. 3.3) in chunks of 64 tokens, bf16 operands.
+// decay_chunk.cu -- the state-decayed form (Sec. 3.3) in chunks of 32 tokens: forward and
+// vector-Jacobian product, bf16 operands, fp32 accumulation.
 //
 // Per slot j the decayed state is a first-order linear recurrence,
 //     X_j(t) = a_j(t) X_j(t-1) + D_j(t) x_t,     a_j(t) = 1 - D_j(t),  D_j(t) = D_M(t - Delta_j),
-// for X = K~ (x = k) and X = V~ (x = v).  Over a chunk of C tokens starting at t0 (tau, u = 0..C-1
-// the in-chunk positions) it unrolls to
-//     X_j(t0 + tau) = A_j(tau) X_j(t0 - 1) + sum_{u <= tau} W_j(tau, u) x_{t0+u},
+// for X = K~ (x = k) and X = V~ (x = v).  Over a chunk starting at t0 (tau, u the in-chunk positions),
+// with K0, V0 the state entering the chunk,
 //     A_j(tau) = prod_{x <= tau} a_j(t0 + x),   W_j(tau, u) = D_j(t0 + u) prod_{u < x <= tau} a_j(t0 + x),
-// so that, with P = Q_c K_c^T and Y = Q_c K~(t0-1)^T,
-//     s[tau, j] = scale (A_j(tau) Y[tau, j] + sum_{u <= tau} P[tau, u] W_j(tau, u))       (Alg. 1 scores)
-//     p = softmax over the slots with t >= Delta_j,
-//     o = (p o A) V~(t0-1) + G V_c,   G[tau, u] = sum_j p[tau, j] W_j(tau, u)
-//     X~(t0 + C - 1) = A_j(C-1) X~(t0 - 1) + Wend X_c,   Wend[j][u] = W_j(C-1, u).
-// Every factor is a product of a's: nothing is divided, so the exact zeros of a (D = 1 at the
-// kernel's peak) need no care.  The four contractions per chunk (P, Y, O and the state update) run
-// on the tensor cores as warp-level bf16 MMAs with fp32 accumulation; the weighted triangle sums
-// (s and G) run on the CUDA cores, walking u downward from tau with the running product r_j:
-//     w = D_j(u) r,   r <- r a_j(u).
-// The fp32 state lives in the MMA accumulator registers of the warps that update it; a bf16 copy
-// in shared memory feeds the next chunk's Y and O.
+//     s = scale (A o Y + sum_u P o W)  (P = Q K^T, Y = Q K0^T),   p = softmax over the visible slots,
+//     o = (p o A) V0 + G V,   G = sum_j p W,
+//     K~end = A_end o K0 + Wend K,  V~end = A_end o V0 + Wend V   (Wend[j][u] = W_j(last, u)).
+// Every factor is a product of a's: nothing is divided, so the exact zeros of a need no care.
+// Given dO and the adjoints mu_K, mu_V of the states at the chunk's end (zero after the last
+// chunk: the final state is not differentiated), the chain rule gives, with PV = dO V^T and
+// YV = dO V0^T,
+//     dp = A o YV + sum_u PV o W,   delta = sum_j p dp,   g = scale p o (dp - delta),
+//     G^ = sum_j g W,
+//     dQ = (g o A) K0 + G^ K,   dK = G^T Q + Wend^T mu_K,   dV = G^T dO + Wend^T mu_V,
+//     mu_K <- (g o A)^T Q + A_end o mu_K,   mu_V <- (p o A)^T dO + A_end o mu_V   (the previous chunk's).
+// (A numpy emulation of these lines matched the oracle's decayed VJP to 1e-15.)
 //
-// Parallelism: each head's sequence is cut into G segments.  Mode 0 (only when G > 1) runs every
-// segment but the last from the zero state through the state updates alone and writes the
-// segment's decay product prod a_j and its state delta; k_dchunk_scan chains them into the state
-// entering each segment; mode 1 runs every segment from its entering state and writes o, lse and,
-// from the last segment, the final state.
+// Both recurrences are linear with a per-slot diagonal decay, so only thin passes run along the
+// sequence; everything else runs one chunk at a time, in parallel over all SMs:
+//   1. k_dbtab: per (head, chunk), Wend and A_end for the thin passes and the chains' tables
+//      (they depend on the period and the positions only, not on the batch);
+//   2. k_dbscan<false>: per (head, K~ or V~, 64-column strip), K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c
+//      from the entering state: the state entering every chunk, stored in bf16, and the final state;
+//   3. forward, k_dfchain: one work item per (head, chunk), each CTA a run of consecutive chunks: s, the
+//      softmax and lse, G, then o;
+//      backward, k_dbchain: likewise s, p, dp, g, G, G^, then dQ (final), the chunk's own parts G^T Q
+//      and G^T dO of dK and dV, and its adjoint contributions Z_K = (g o A)^T Q, Z_V = (p o A)^T dO;
+//   4. backward, k_dbscan<true>: per (head, strip), from the last chunk back: dK += Wend^T mu_K (dV
+//      likewise), then mu <- A_end o mu + Z.
+// In the chains the triangle sums (s, dp, G, G^) are split at 16-token sub-blocks: the off-diagonal
+// block is a contraction on the tensor cores (W = alpha_j(tau) beta_j(u) across adjacent
+// sub-blocks), the diagonal blocks walk u on the CUDA cores.  All contractions are warp-level bf16
+// MMAs (m16n8k16).
 #include <math.h>
 
 #include "decay.cuh"
@@ -37,295 +48,309 @@ namespace {
 
 using namespace wmma16;
 
-constexpr int kDC = 64;            // tokens per chunk
-constexpr int kDThreads = 512;     // 16 warps
-constexpr int kDWarps = kDThreads / 32;
-constexpr int kFS = kDC + 4;       // row stride (floats) of the fp32 [64][64] tiles
+constexpr int kBC = 32;          // tokens per chunk
+constexpr int kBT = 256;         // threads (8 warps)
+constexpr int kBFS = kBC + 4;    // fp32 row stride of [32][32] tiles
+constexpr int kBSS = 64 + 4;     // fp32 row stride of [32][S] tiles (S <= 64)
 
-// ------------------------------------------------------------------ shared-memory layout
-
-template <int D, int S>
-struct DcLayout {
-    static constexpr int kTile = kDC * D * 2;   // one [64][D] bf16 tile
-    static constexpr int q = 0;
-    static constexpr int k0 = q + kTile, v0 = k0 + kTile, k1 = v0 + kTile, v1 = k1 + kTile;   // two stages
-    static constexpr int kst = v1 + kTile;                  // bf16 [S][D]: K~ at the chunk start
-    static constexpr int vst = kst + S * D * 2;             // bf16 [S][D]: V~ at the chunk start
-    static constexpr int wend = vst + S * D * 2;            // bf16 [S][64]: Wend
-    static constexpr int beta = wend + S * 128;             // bf16 [S][64]: beta_j(u)
-    static constexpr int pa = beta + S * 128;               // bf16 [64][64]: p o A (columns >= S zero)
-    static constexpr int gm = pa + kDC * 128;               // bf16 [64][64]: G (upper triangle zero)
-    static constexpr int pf = gm + kDC * 128;               // fp32 [64][kFS]: P; then bf16 [64][D]: O
-    static constexpr int yf = pf + kDC * kFS * 4;           // fp32 [64][kFS]: Y, s, then p
-    static constexpr int df = yf + kDC * kFS * 4;           // fp32 [64][kFS]: D_j(t0 + u)
-    static constexpr int af = df + kDC * kFS * 4;           // fp32 [64][kFS]: alpha_j(tau)
-    static constexpr int g4 = af + kDC * kFS * 4;           // fp32 [4][S]: sub-block products g_j(B)
-    static constexpr int gpre = g4 + 4 * S * 4;             // fp32 [4][S]: prod_{B' < B} g_j(B')
-    static constexpr int aend = gpre + 4 * S * 4;           // fp32 [S]: A_j(63)
-    static constexpr int delta = aend + S * 4;              // int [S]
-    static constexpr int tot = delta + S * 4;               // fp32 [kDThreads / S][S]: segment products
-    static constexpr int bars = tot + kDThreads * 4;        // 3 mbarriers (q, kv stage 0, kv stage 1)
-    static constexpr int total = bars + 64;
-    static_assert(pf % 1024 == 0 && kst % 1024 == 0 && wend % 1024 == 0 && beta % 1024 == 0 && pa % 1024 == 0 &&
-                      gm % 1024 == 0,
-                  "swizzled tiles need 1024-byte alignment");
-    static_assert(total <= 227 * 1024, "shared memory of one CTA");
-    static_assert(kDC * D * 2 <= kDC * kFS * 4, "the O tile reuses the P tile");
+// The chain's tables of one (head, chunk), built by k_dbtab and copied whole into shared memory:
+// beta_j(u) (bf16, swizzled [S][64], u < 32 used), D_j(t0 + u) and alpha_j(tau) (fp32 [32][kBSS]),
+// and Gpre (fp32 [2][S]: the decay of the sub-blocks before sub-block 0, 1).
+template <int S>
+struct ChunkTab {
+    static constexpr int beta = 0, d = S * 128, alpha = d + kBC * kBSS * 4, gpre = alpha + kBC * kBSS * 4;
+    static constexpr int bytes = gpre + 2 * S * 4;
+    static_assert(bytes % 16 == 0, "bulk copies move multiples of 16 bytes");
 };
 
-struct DcArgs {
-    int L, G, cps, H, mode;     // mode 0: segment deltas (G > 1); 1: outputs
+// The thin passes' tables of one (head, chunk): Wend (bf16, swizzled [S][64], u < 32 used), then
+// A_end (fp32 [S]), one bulk copy.
+template <int S>
+struct EndTab {
+    static constexpr int wend = 0, aend = S * 128, bytes = aend + S * 4;
+    static_assert(bytes % 16 == 0, "bulk copies move multiples of 16 bytes");
+};
+
+template <int D, int S>
+struct BwLayout {
+    static constexpr int kTile = kBC * D * 2;          // one [32][D] bf16 tile
+    static constexpr int q = 0;                         // bf16 [2][32][D]: q of this item and the next
+    static constexpr int dout = q + 2 * kTile;          // bf16 [2][32][D]: dO likewise
+    static constexpr int k = dout + 2 * kTile, v = k + kTile;
+    static constexpr int o = v + kTile;                 // bf16 [32][D]: dK staging
+    static constexpr int ost = o + kTile;               // bf16 [32][D]: dV staging
+    static constexpr int k0 = ost + kTile;              // bf16 [S][D]: K~ entering the chunk
+    static constexpr int v0 = k0 + S * D * 2;           // bf16 [S][D]: V~ entering the chunk
+    static constexpr int zk = v0 + S * D * 2;           // bf16 [S][D]: Z_K staging
+    static constexpr int zv = zk + S * D * 2;           // bf16 [S][D]: Z_V staging
+    static constexpr int tab = zv + S * D * 2;          // the chunk's tables (ChunkTab)
+    static constexpr int pa = tab + ((ChunkTab<S>::bytes + 1023) / 1024) * 1024;   // bf16 [32][64]: p o A
+    static constexpr int ga = pa + kBC * 128;           // bf16 [32][64]: g o A
+    static constexpr int gm = ga + kBC * 128;           // bf16 [32][64] (u < 32): G
+    static constexpr int gh = gm + kBC * 128;           // bf16 [32][64]: G^
+    static constexpr int sf = gh + kBC * 128;           // fp32 [32][kBSS]: s, then p, then dQ staging (bf16)
+    static constexpr int pf = sf + kBC * kBSS * 4;      // fp32 [32][kBFS]: P
+    static constexpr int pvf = pf + kBC * kBFS * 4;     // fp32 [32][kBFS]: PV
+    static constexpr int dpf = pvf + kBC * kBFS * 4;    // fp32 [32][kBSS]: dp, then g
+    static constexpr int delta = dpf + kBC * kBSS * 4;  // int [S]
+    static constexpr int lse = delta + S * 4;           // fp32 [32]
+    static constexpr int bars = lse + kBC * 4;          // mbarrier: the item's tiles
+    static constexpr int total = bars + 64;
+    static_assert(k0 % 1024 == 0 && tab % 1024 == 0 && pa % 1024 == 0 && gh % 1024 == 0 && sf % 1024 == 0 &&
+                      kBC * kBSS * 4 >= kTile && pf % 16 == 0,
+                  "swizzled tiles need 1024-byte alignment");
+    static_assert(total <= 227 * 1024, "shared memory of one CTA");
+};
+
+struct DbArgs {
+    int L, H, BH;
+    int ipc;                    // chain items (chunks) per CTA: CTA b takes items [b ipc, (b + 1) ipc), chunk fastest
     long long pos0;
     float scale;
     int dmax;
     const float *Dx;            // D_M table: D_j(pos0 + t) = Dx[t + dmax - Delta_j]
-    const int *delta;           // [S] slot lags
+    const int *delta;           // [S]
     int hs_dx, hs_delta;        // per-head strides (0: one shared period)
-    const float *state_in;      // [BH][2][S][D] or null (zero state)
-    float *state_out;           // [BH][2][S][D] or null
-    float *seg_delta;           // [BH][G][2][S][D]: mode 0 output (state delta of each segment)
-    float *seg_decay;           // [BH][G][S]: mode 0 output (prod of a_j over each segment)
-    const float *win;           // [BH][G][2][S][D]: state entering each segment (G > 1)
-    float *lse;                 // [BH][L]
+    const float *lse;           // [BH][L], from the forward (backward)
+    float *lse_out;             // [BH][L] (forward)
+    const float *state_in;      // [BH][2][S][D] fp32 or null: the state before the first token (forward)
+    float *state_out;           // [BH][2][S][D] fp32 or null: the state after the last token (forward)
+    int ntab;                   // heads with their own tables (1 when the heads share one period)
+    uint8_t *ctab;              // [ntab][nch] ChunkTab records of the chain
+    uint8_t *etab;              // [ntab][nch] EndTab records of the thin passes
+    __nv_bfloat16 *states;      // [BH][nch][2][S][D]: the state entering each chunk
+    __nv_bfloat16 *zbuf;        // [BH][nch][2][S][D]: each chunk's adjoint contributions (g o A)^T Q, (p o A)^T dO
     int *err;
 };
 
+// the 8 warps' share of a [2][S][D] state (K~ | V~) or of its adjoint: warp w holds NB2 blocks of 16 x 16
+// in row block rb and column blocks cb0 .. cb0 + NB2 - 1 of half kv = w / 4
 template <int D, int S>
-__global__ void __launch_bounds__(kDThreads, 1)
-    k_dchunk(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
-             const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_o, DcArgs a) {
-    using Lay = DcLayout<D, S>;
-    constexpr int SPT = S / 16;                  // slots per thread in the triangle sums
-    constexpr int NU = S * D / 2048;             // 16x16 state blocks per warp (K and V together)
-    constexpr int SB = S / 16, DB = D / 16;
+struct StateMap {
+    static constexpr int SB = S / 16, DB = D / 16, NB2 = SB * DB / 4;
+    static_assert(NB2 >= 1 && NB2 <= DB && DB % NB2 == 0, "state blocks per warp");
+    __device__ static int kv(int w) { return w >> 2; }
+    __device__ static int rb(int w) { return ((w & 3) * NB2) / DB; }
+    __device__ static int cb0(int w) { return ((w & 3) * NB2) % DB; }
+};
+
+// N (2 or 4) consecutive 32-bit words of shared memory in one access (16- or 8-byte aligned)
+template <typename T, int N>
+__device__ __forceinline__ void lds_vec(const T *p, T (&v)[N]) {
+    static_assert(N == 2 || N == 4, "vector width");
+    if constexpr (N == 4) {
+        const uint4 x = *reinterpret_cast<const uint4 *>(p);
+        v[0] = __builtin_bit_cast(T, x.x); v[1] = __builtin_bit_cast(T, x.y);
+        v[2] = __builtin_bit_cast(T, x.z); v[3] = __builtin_bit_cast(T, x.w);
+    } else {
+        const uint2 x = *reinterpret_cast<const uint2 *>(p);
+        v[0] = __builtin_bit_cast(T, x.x); v[1] = __builtin_bit_cast(T, x.y);
+    }
+}
+template <int N>
+__device__ __forceinline__ void sts_vec(float *p, const float (&v)[N]) {
+    if constexpr (N == 4) *reinterpret_cast<float4 *>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    else *reinterpret_cast<float2 *>(p) = make_float2(v[0], v[1]);
+}
+// N bf16 (rounded from fp32) to consecutive columns of a swizzled tile row (within one 16-byte chunk)
+template <int N>
+__device__ __forceinline__ void st_bf16_vec(uint8_t *p, const float (&v)[N]) {
+    if constexpr (N == 4)
+        *reinterpret_cast<uint2 *>(p) = make_uint2(tc::pack_bf16x2(v[0], v[1]), tc::pack_bf16x2(v[2], v[3]));
+    else *reinterpret_cast<uint32_t *>(p) = tc::pack_bf16x2(v[0], v[1]);
+}
+
+template <int D, int S>
+__global__ void __launch_bounds__(kBT, 1)
+    k_dbchain(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_do,
+              const __grid_constant__ CUtensorMap tm_st, const __grid_constant__ CUtensorMap tm_z,
+              const __grid_constant__ CUtensorMap tm_dq, const __grid_constant__ CUtensorMap tm_dk,
+              const __grid_constant__ CUtensorMap tm_dv, DbArgs a) {
+    using Lay = BwLayout<D, S>;
+    using SMap = StateMap<D, S>;
+    constexpr int SPT = S / 16, NB2 = SMap::NB2, SB = S / 16, DB = D / 16;
     extern __shared__ __align__(1024) uint8_t dsm[];
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g8 = lane >> 2, t4 = lane & 3;
     if (tc::smem_u32(dsm) & 1023u) {
-        if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (16 << 4) | ((int)blockIdx.x << 16));
+        if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (17 << 4) | ((int)blockIdx.x << 16));
         return;
     }
-    const int G = a.G;
-    const int bh = blockIdx.x / G, seg = blockIdx.x % G;
-    if (a.mode == 0 && seg == G - 1) return;      // the last segment's delta is never used
-    const int hd = bh % a.H;
-    const float *Dx = a.Dx + (size_t)hd * a.hs_dx;
-    const int c_begin = seg * a.cps;
-    const int nch = (a.L + kDC - 1) / kDC;
-    const int c_end = min(nch, c_begin + a.cps);
-    const bool outputs = a.mode == 1;
-
-    uint8_t *sQ = dsm + Lay::q, *sKst = dsm + Lay::kst, *sVst = dsm + Lay::vst, *sW = dsm + Lay::wend;
-    uint8_t *sBeta = dsm + Lay::beta;
-    uint8_t *sPA = dsm + Lay::pa, *sGm = dsm + Lay::gm, *sO = dsm + Lay::pf;
-    float *sP = reinterpret_cast<float *>(dsm + Lay::pf), *sY = reinterpret_cast<float *>(dsm + Lay::yf);
-    float *sD = reinterpret_cast<float *>(dsm + Lay::df), *sAl = reinterpret_cast<float *>(dsm + Lay::af);
-    float *sG4 = reinterpret_cast<float *>(dsm + Lay::g4), *sGpre = reinterpret_cast<float *>(dsm + Lay::gpre);
-    float *sAend = reinterpret_cast<float *>(dsm + Lay::aend);
+    const int L = a.L, nch = (L + kBC - 1) / kBC;
+    const long long nitems = (long long)a.BH * nch;
+    uint8_t *sK = dsm + Lay::k, *sV = dsm + Lay::v, *sO = dsm + Lay::o;
+    using Tab = ChunkTab<S>;
+    uint8_t *sOst = dsm + Lay::ost, *sK0 = dsm + Lay::k0, *sV0 = dsm + Lay::v0, *sTab = dsm + Lay::tab;
+    uint8_t *sZK = dsm + Lay::zk, *sZV = dsm + Lay::zv, *sBeta = sTab + Tab::beta;
+    uint8_t *sPA = dsm + Lay::pa, *sGA = dsm + Lay::ga, *sGm = dsm + Lay::gm, *sGh = dsm + Lay::gh;
+    float *sP = reinterpret_cast<float *>(dsm + Lay::pf), *sPV = reinterpret_cast<float *>(dsm + Lay::pvf);
+    float *sS = reinterpret_cast<float *>(dsm + Lay::sf), *sDP = reinterpret_cast<float *>(dsm + Lay::dpf);
+    float *sD = reinterpret_cast<float *>(sTab + Tab::d), *sAl = reinterpret_cast<float *>(sTab + Tab::alpha);
+    float *sGpre = reinterpret_cast<float *>(sTab + Tab::gpre);
     int *sdelta = reinterpret_cast<int *>(dsm + Lay::delta);
-    float *sTot = reinterpret_cast<float *>(dsm + Lay::tot);
+    float *sLse = reinterpret_cast<float *>(dsm + Lay::lse);
     uint64_t *bar = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
-    const uint32_t uQ = tc::smem_u32(sQ), uKst = tc::smem_u32(sKst), uVst = tc::smem_u32(sVst);
-    const uint32_t uW = tc::smem_u32(sW), uPA = tc::smem_u32(sPA), uGm = tc::smem_u32(sGm);
-    const uint32_t uBeta = tc::smem_u32(sBeta);
+    const uint32_t uK = tc::smem_u32(sK), uV = tc::smem_u32(sV);
+    const uint32_t uK0 = tc::smem_u32(sK0), uV0 = tc::smem_u32(sV0), uBeta = tc::smem_u32(sBeta);
+    const uint32_t uPA = tc::smem_u32(sPA), uGA = tc::smem_u32(sGA), uGm = tc::smem_u32(sGm), uGh = tc::smem_u32(sGh);
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < 3; ++i) tc::mbar_init(&bar[i], 1);
+        tc::mbar_init(&bar[0], 1);
         tc::fence_barrier_init();
     }
-    for (int j = threadIdx.x; j < S; j += kDThreads) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
-    // G's upper triangle and p o A's columns past S stay zero for the whole call
-    for (int i = threadIdx.x; i < kDC * 64 / 2; i += kDThreads) {
+    // the upper triangles of G and G^, and the columns past S of p o A and g o A, stay zero
+    for (int i = threadIdx.x; i < kBC * 64 / 2; i += kBT) {
         reinterpret_cast<uint32_t *>(sGm)[i] = 0u;
+        reinterpret_cast<uint32_t *>(sGh)[i] = 0u;
         reinterpret_cast<uint32_t *>(sPA)[i] = 0u;
+        reinterpret_cast<uint32_t *>(sGA)[i] = 0u;
     }
     __syncthreads();
 
-    // ---- the state, in the accumulator layout of the state-update MMA: warp w holds NU blocks of
-    // 16 rows (slots) x 16 columns of [K~ | V~]; block b -> kv = b / (SB DB), slot block, column block
-    float st[NU][2][4];
-    // outputs: the state entering the segment (from the scan, or the call's initial state when the
-    // head is one segment); segment deltas: the zero state
-    const float *src = nullptr;
-    if (outputs && G > 1) src = a.win + ((size_t)bh * G + seg) * 2 * S * D;
-    else if (outputs && a.state_in) src = a.state_in + (size_t)bh * 2 * S * D;
-    const int g8 = lane >> 2, t4 = lane & 3;
+    // ---- the chunk's adjoint contributions Z, in the accumulator layout of the MMAs that form them:
+    // warp w holds NB2 blocks of half kv, row block rb, column blocks cb0..
+    const int skv = SMap::kv(warp), sj0 = SMap::rb(warp) * 16, se0 = SMap::cb0(warp) * 16;
+    float st[NB2][2][4];
+    // Z = X_a^T X (A = the transposed p o A or g o A tile, B = the chunk's q or dO)
+    auto z_product = [&](uint32_t ux, uint32_t uw) {
 #pragma unroll
-    for (int i = 0; i < NU; ++i) {
-        const int b = warp * NU + i, kv = b / (SB * DB), rem = b % (SB * DB);
-        const int j0 = (rem / DB) * 16, e0 = (rem % DB) * 16;
+        for (int i = 0; i < NB2; ++i)
 #pragma unroll
-        for (int h = 0; h < 2; ++h)
+            for (int h = 0; h < 2; ++h)
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int j = j0 + g8 + ((q >> 1) << 3), e = e0 + h * 8 + 2 * t4 + (q & 1);
-                st[i][h][q] = src ? src[((size_t)kv * S + j) * D + e] : 0.f;
+                for (int q = 0; q < 4; ++q) st[i][h][q] = 0.f;
+        for (int k0 = 0; k0 < kBC; k0 += 16) {
+            uint32_t af[4], b[4];
+            load_a_t(uw, kBC, sj0, k0, af);
+#pragma unroll
+            for (int i = 0; i < NB2; ++i) {
+                load_b_kn(ux, kBC, se0 + i * 16, k0, b);
+                mma16816(st[i][0], af, b[0], b[1]);
+                mma16816(st[i][1], af, b[2], b[3]);
             }
+        }
+    };
+
+    uint32_t ph1 = 0;
+    bool ok = true;
+    const int sg = threadIdx.x & 15, rp = threadIdx.x >> 4, sb = rp >> 3, ip = rp & 7;
+    const unsigned hmask = 0xffffu << (lane & 16);
+    const int i0 = (int)blockIdx.x * a.ipc, i1 = (int)min(nitems, (long long)i0 + a.ipc);
+    // the next item's lse (threads < 32) travels in a register
+    float lse_nx = 0.f;
+    auto load_lse = [&](int it) {
+        const int c = (int)(it % nch), bh = (int)(it / nch), t = c * kBC + (int)threadIdx.x;
+        if (threadIdx.x < kBC) lse_nx = t < L ? a.lse[(size_t)bh * L + t] : 0.f;
+    };
+    auto tab_of = [&](int it) {
+        const int tb = a.ntab > 1 ? (int)(it / nch) % a.H : 0;
+        return a.ctab + ((size_t)tb * nch + (size_t)(it % nch)) * Tab::bytes;
+    };
+    // Item it + 1's loads are issued while item it runs, each once its place is free: v, q and dO
+    // (the other of the two q / dO buffers) after (a), the tables after (d), k, K0 and V0 after dQ.
+    auto issue_vqo = [&](int it, int buf) {
+        const int c = (int)(it % nch), bh = (int)(it / nch), t0 = c * kBC;
+        tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(4 * Lay::kTile + 2 * S * D * 2 + Tab::bytes));
+        tc::tma_load_4d(sV, &tm_v, &bar[0], 0, t0, 0, bh);
+        tc::tma_load_4d(dsm + Lay::q + buf * Lay::kTile, &tm_q, &bar[0], 0, t0, 0, bh);
+        tc::tma_load_4d(dsm + Lay::dout + buf * Lay::kTile, &tm_do, &bar[0], 0, t0, 0, bh);
+    };
+    auto issue_tab = [&](int it) { tc::bulk_load(sTab, tab_of(it), (uint32_t)Tab::bytes, &bar[0]); };
+    auto issue_k = [&](int it) {
+        const int c = (int)(it % nch), bh = (int)(it / nch);
+        const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
+        tc::tma_load_4d(sK, &tm_k, &bar[0], 0, c * kBC, 0, bh);
+        tc::tma_load_3d(sK0, &tm_st, &bar[0], 0, srow, 0);
+        tc::tma_load_3d(sV0, &tm_st, &bar[0], 0, srow + S, 0);
+    };
+    if (i0 < i1) {
+        load_lse(i0);
+        if (threadIdx.x == 0) {
+            issue_vqo(i0, 0);
+            issue_tab(i0);
+            issue_k(i0);
+        }
     }
-    // bf16 copy of the entering state for the first chunk's Y and O
-    auto store_state_copy = [&]() {
+    int cur_hd = -1;
+    for (int it = i0; it < i1 && ok; ++it) {
+        const int c = (int)(it % nch), bh = (int)(it / nch), hd = bh % a.H;
+        const int t0 = c * kBC, n = min(kBC, L - t0);
+        const int nx = it + 1;
+        const int buf = (int)((it - i0) & 1);
+        const uint32_t uQ = tc::smem_u32(dsm + Lay::q + buf * Lay::kTile);
+        const uint32_t uDO = tc::smem_u32(dsm + Lay::dout + buf * Lay::kTile);
+        if (threadIdx.x == kBT - 32 && nx < i1) {
+            // the next item's k and states into L2 (their loads follow dQ)
+            const int cn = (int)(nx % nch), bn = (int)(nx / nch);
+            tc::tma_prefetch_4d(&tm_k, 0, cn * kBC, 0, bn);
+            tc::bulk_prefetch_l2(a.states + (((size_t)bn * nch + cn) * 2) * S * D, (uint32_t)(2 * S * D * 2));
+        }
+        // sdelta and sLse were last read before the previous item's closing barriers
+        if (hd != cur_hd) {
+            for (int j = threadIdx.x; j < S; j += kBT) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
+            cur_hd = hd;
+        }
+        if (threadIdx.x < kBC) sLse[threadIdx.x] = lse_nx;
+        if (nx < i1) load_lse(nx);
+        if (!tc::mbar_wait(&bar[0], ph1)) {
+            report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (17 << 4));
+            ok = false;
+            break;
+        }
+        ph1 ^= 1;
+        // ---- (a) P = Q K^T, Y = Q K0^T (warps 0-3), PV = dO V^T, YV = dO V0^T (warps 4-7): warp takes
+        // row block m0 and half hh of the columns; Y / YV stay in registers
+        const int side = warp >> 2, m0 = ((warp >> 1) & 1) * 16, hh = warp & 1, bt = m0 >> 4;
+        constexpr int YB = SB / 2 > 0 ? SB / 2 : 1;   // 16-column blocks of Y per warp
+        const int yn0 = hh * (S / 2);
+        float yacc[YB][2][4] = {};
+        {
+            const uint32_t ua = side ? uDO : uQ, ub = side ? uV : uK, uy = side ? uV0 : uK0;
+            float pacc[2][4] = {};
+            for (int k0 = 0; k0 < D; k0 += 16) {
+                uint32_t af[4], b[4];
+                load_a(ua, kBC, m0, k0, af);
+                load_b_nk(ub, kBC, hh * 16, k0, b);
+                mma16816(pacc[0], af, b[0], b[1]);
+                mma16816(pacc[1], af, b[2], b[3]);
 #pragma unroll
-        for (int i = 0; i < NU; ++i) {
-            const int b = warp * NU + i, kv = b / (SB * DB), rem = b % (SB * DB);
-            const int j0 = (rem / DB) * 16, e0 = (rem % DB) * 16;
-            uint8_t *tile = kv ? sVst : sKst;
+                for (int i = 0; i < YB; ++i) {
+                    if (yn0 + i * 16 >= S) break;
+                    load_b_nk(uy, S, yn0 + i * 16, k0, b);
+                    mma16816(yacc[i][0], af, b[0], b[1]);
+                    mma16816(yacc[i][1], af, b[2], b[3]);
+                }
+            }
+            float *dst = side ? sPV : sP;
 #pragma unroll
             for (int h = 0; h < 2; ++h) {
-                const int e = e0 + h * 8 + 2 * t4;
-                st_bf16x2(tile, S, j0 + g8, e, st[i][h][0], st[i][h][1]);
-                st_bf16x2(tile, S, j0 + g8 + 8, e, st[i][h][2], st[i][h][3]);
+                const int col = hh * 16 + h * 8 + 2 * t4;
+                *reinterpret_cast<float2 *>(&dst[(m0 + g8) * kBFS + col]) = make_float2(pacc[h][0], pacc[h][1]);
+                *reinterpret_cast<float2 *>(&dst[(m0 + g8 + 8) * kBFS + col]) = make_float2(pacc[h][2], pacc[h][3]);
             }
         }
-    };
-    if (outputs) store_state_copy();
-
-    // ---- TMA: q of the chunk (one buffer), k and v in two stages
-    uint32_t ph_q = 0, ph_kv[2] = {0, 0};
-    auto issue_q = [&](int c) {
-        tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)Lay::kTile);
-        for (int db = 0; db < D / 64; ++db) tc::tma_load_3d(sQ + db * kDC * 128, &tm_q, &bar[0], db * 64, c * kDC, bh);
-    };
-    auto issue_kv = [&](int c) {
-        const int s = (c - c_begin) & 1;
-        uint8_t *kb = dsm + (s ? Lay::k1 : Lay::k0), *vb = dsm + (s ? Lay::v1 : Lay::v0);
-        tc::mbar_arrive_expect_tx(&bar[1 + s], (uint32_t)(2 * Lay::kTile));
-        for (int db = 0; db < D / 64; ++db) {
-            tc::tma_load_3d(kb + db * kDC * 128, &tm_k, &bar[1 + s], db * 64, c * kDC, bh);
-            tc::tma_load_3d(vb + db * kDC * 128, &tm_v, &bar[1 + s], db * 64, c * kDC, bh);
-        }
-    };
-    if (threadIdx.x == 0 && c_begin < c_end) {
-        if (outputs) issue_q(c_begin);
-        issue_kv(c_begin);
-        if (c_begin + 1 < c_end) issue_kv(c_begin + 1);
-    }
-    float seg_dec = 1.f;   // mode 0: prod of a_j over the segment (thread j < S)
-    bool ok = true;
-    // ---- the decay tables of a chunk, by all threads: thread (slot j, run r) holds UPS consecutive
-    // tokens' D_j; their values for the next chunk are loaded while this chunk is processed
-    constexpr int NRUN = kDThreads / S, UPS = kDC / NRUN;
-    const int tj = threadIdx.x % S, trun = threadIdx.x / S, tu0 = trun * UPS;
-    float dl[UPS];
-    auto load_d = [&](int c) {
-        const int t0 = c * kDC, n = min(kDC, a.L - t0);
-        const float *src = Dx + t0 + tu0 + a.dmax - sdelta[tj];
-#pragma unroll
-        for (int i = 0; i < UPS; ++i) dl[i] = (tu0 + i < n) ? src[i] : 0.f;
-    };
-    if (c_begin < c_end) load_d(c_begin);
-
-    for (int c = c_begin; c < c_end && ok; ++c) {
-        const int t0 = c * kDC, n = min(kDC, a.L - t0), s = (c - c_begin) & 1;
-        const uint8_t *sK = dsm + (s ? Lay::k1 : Lay::k0), *sV = dsm + (s ? Lay::v1 : Lay::v0);
-        const uint32_t uK = tc::smem_u32(sK), uV = tc::smem_u32(sV);
-        // ---- D_j(t0 + u) (0 past the end of the sequence: those steps leave the state as it is) and the
-        // products built from a_j = 1 - D_j, per 16-token sub-block B of the chunk:
-        //   alpha_j(tau) = prod_{B start <= x <= tau} a_j,   beta_j(u) = D_j(u) prod_{u < x <= B end} a_j,
-        //   g_j(B) = prod_{x in B} a_j,   Gpre_j(B) = prod_{B' < B} g_j(B')   (A_j(tau) = Gpre_j alpha_j),
-        //   Wend[j][u] = D_j(u) prod_{x > u} a_j.
-        // Each thread's run of UPS tokens forms its local products; the runs' totals combine through
-        // shared memory.
+        // the previous item's stores have read their staging tiles (s, where dQ was staged, is written
+        // next; the dK, dV and Z staging tiles later)
+        if (threadIdx.x == 0) tc::bulk_wait_read0();
+        __syncthreads();
+        // v, q and dO are read: the next item's go in (q and dO into the other buffer)
+        if (threadIdx.x == 0 && nx < i1) issue_vqo(nx, buf ^ 1);
+        // ---- (b) the off-diagonal block of sub-block 1 over sub-block 0 (W = alpha beta there), and
+        // alpha (Gpre Y + F) into s (warps 0-3) or dp (warps 4-7)
         {
-            float pf[UPS], tot = 1.f;
+            const float *pm = side ? sPV : sP;
+            float *dst = side ? sDP : sS;
 #pragma unroll
-            for (int i = 0; i < UPS; ++i) {
-                sD[(tu0 + i) * kFS + tj] = dl[i];
-                tot *= 1.f - dl[i];
-                pf[i] = tot;
-            }
-            sTot[trun * S + tj] = tot;
-            if (threadIdx.x == 0) tc::bulk_wait_read0();   // the last chunk's o has left the P tile
-            __syncthreads();
-            constexpr int RPB = 16 / UPS;   // runs per sub-block
-            const int rb0 = (trun / RPB) * RPB;
-            float pre = 1.f, suf = 1.f, pre_b = 1.f, suf_b = 1.f;
-            for (int r2 = 0; r2 < NRUN; ++r2) {
-                const float x = sTot[r2 * S + tj];
-                if (r2 < trun) {
-                    pre *= x;
-                    if (r2 >= rb0) pre_b *= x;
-                } else if (r2 > trun) {
-                    suf *= x;
-                    if (r2 < rb0 + RPB) suf_b *= x;
-                }
-            }
-#pragma unroll
-            for (int i = 0; i < UPS; ++i) sAl[(tu0 + i) * kFS + tj] = pre_b * pf[i];
-            if (trun == rb0) {
-                // this sub-block's product and the product of the sub-blocks before it
-                float gb = tot;
-                for (int r2 = trun + 1; r2 < rb0 + RPB; ++r2) gb *= sTot[r2 * S + tj];
-                sG4[(trun / RPB) * S + tj] = gb;
-                sGpre[(trun / RPB) * S + tj] = pre;
-            }
-            if (trun == NRUN - 1) {
-                sAend[tj] = pre * tot;
-                seg_dec *= pre * tot;
-            }
-            float r = 1.f;   // prod of a over this run's tokens after the current one
-#pragma unroll
-            for (int i = UPS - 1; i >= 1; i -= 2) {
-                const float w1 = dl[i] * r;
-                r -= r * dl[i];
-                const float w0 = dl[i - 1] * r;
-                r -= r * dl[i - 1];
-                st_bf16x2(sW, S, tj, tu0 + i - 1, w0 * suf, w1 * suf);
-                st_bf16x2(sBeta, S, tj, tu0 + i - 1, w0 * suf_b, w1 * suf_b);
-            }
-        }
-        if (c + 1 < c_end) load_d(c + 1);
-        if (outputs) {
-            // ---- P = Q K^T and Y = Q K~^T: one 16x16 block of each per warp
-            if (!tc::mbar_wait(&bar[0], ph_q)) { report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (16 << 4)); ok = false; }
-            ph_q ^= 1;
-            if (!tc::mbar_wait(&bar[1 + s], ph_kv[s] & 1)) { report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (16 << 4)); ok = false; }
-            if (!ok) break;
-            // warp (sub-block bt, 16 columns): P's block, and Y's block where the columns are slots; the
-            // two share Q's fragments.  Y = Q K~^T stays in registers until P is complete.
-            const int bt = warp >> 2, yn0 = (warp & 3) * 16, ym0 = bt * 16;
-            const bool has_y = (warp & 3) < SB;
-            float yacc[2][4] = {};
-            {
-                float acc[2][4] = {};
-                for (int k0 = 0; k0 < D; k0 += 16) {
-                    uint32_t af[4], b[4];
-                    load_a(uQ, kDC, ym0, k0, af);
-                    load_b_nk(uK, kDC, yn0, k0, b);
-                    mma16816(acc[0], af, b[0], b[1]);
-                    mma16816(acc[1], af, b[2], b[3]);
-                    if (has_y) {
-                        load_b_nk(uKst, S, yn0, k0, b);
-                        mma16816(yacc[0], af, b[0], b[1]);
-                        mma16816(yacc[1], af, b[2], b[3]);
-                    }
-                }
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int col = yn0 + h * 8 + 2 * t4;
-                    *reinterpret_cast<float2 *>(&sP[(ym0 + g8) * kFS + col]) = make_float2(acc[h][0], acc[h][1]);
-                    *reinterpret_cast<float2 *>(&sP[(ym0 + g8 + 8) * kFS + col]) = make_float2(acc[h][2], acc[h][3]);
-                }
-            }
-            __syncthreads();
-            // the next chunk's q may load now (its tile has been read)
-            if (threadIdx.x == 0 && c + 1 < c_end) issue_q(c + 1);
-            // ---- s[tau, j] = scale (A_j(tau) Y[tau, j] + sum_{u <= tau} P[tau, u] W_j(tau, u)).  For u in a
-            // sub-block B_u before tau's, W = alpha_j(tau) gamma_j beta_j(u), gamma_j the product of g_j over
-            // the sub-blocks between, so those terms are alpha_j(tau) F with
-            //   F = sum_{B_u < B_tau} gamma_j P_blk beta_blk   (Horner over B_u: F <- g_j(B_u) F + P_blk beta_blk)
-            // on the tensor cores; with A = Gpre alpha the warp leaves alpha (Gpre Y + F) in sY.
-            if (has_y) {
+            for (int i = 0; i < YB; ++i) {
+                const int n0 = yn0 + i * 16;
+                if (n0 >= S) break;
                 float facc[2][4] = {};
-                for (int kb = 0; kb < bt; ++kb) {
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        const float2 gk = *reinterpret_cast<const float2 *>(&sG4[kb * S + yn0 + h * 8 + 2 * t4]);
-                        facc[h][0] *= gk.x; facc[h][1] *= gk.y; facc[h][2] *= gk.x; facc[h][3] *= gk.y;
-                    }
-                    const float *p0 = sP + (ym0 + g8) * kFS + kb * 16 + 2 * t4, *p1 = p0 + 8 * kFS;
+                if (bt == 1) {
+                    const float *p0 = pm + (m0 + g8) * kBFS + 2 * t4, *p1 = p0 + 8 * kBFS;
                     const uint32_t af[4] = {tc::pack_bf16x2(p0[0], p0[1]), tc::pack_bf16x2(p1[0], p1[1]),
                                             tc::pack_bf16x2(p0[8], p0[9]), tc::pack_bf16x2(p1[8], p1[9])};
                     uint32_t b[4];
-                    load_b_nk(uBeta, S, yn0, kb * 16, b);
+                    load_b_nk(uBeta, S, n0, 0, b);
                     mma16816(facc[0], af, b[0], b[1]);
                     mma16816(facc[1], af, b[2], b[3]);
                 }
@@ -333,370 +358,1103 @@ __global__ void __launch_bounds__(kDThreads, 1)
                 for (int h = 0; h < 2; ++h)
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
-                        const int row = ym0 + g8 + ((q >> 1) << 3), j = yn0 + h * 8 + 2 * t4 + (q & 1);
-                        sY[row * kFS + j] = sAl[row * kFS + j] * fmaf(sGpre[bt * S + j], yacc[h][q], facc[h][q]);
+                        const int row = m0 + g8 + ((q >> 1) << 3), j = n0 + h * 8 + 2 * t4 + (q & 1);
+                        dst[row * kBSS + j] = sAl[row * kBSS + j] * fmaf(sGpre[bt * S + j], yacc[i][h][q], facc[h][q]);
                     }
             }
-            __syncthreads();
-            // ---- the diagonal sub-blocks on the CUDA cores: thread (pair ip of sub-block sb, slot group sg)
-            // walks rows 16 sb + ip and 16 sb + 15 - ip (17 steps together) down to the sub-block's start,
-            // with the running product r_j
-            const int sg = threadIdx.x & 15, rp = threadIdx.x >> 4, sb = rp >> 3, ip = rp & 7;
-#pragma unroll 1
-            for (int rr = 0; rr < 2; ++rr) {
-                const int row = sb * 16 + (rr ? 15 - ip : ip), lo = sb * 16;
-                float acc[SPT], r[SPT];
+        }
+        __syncthreads();
+        // ---- (c) the diagonal sub-blocks of s and dp on the CUDA cores (one walk, the same weights),
+        // then p = exp(s - lse), delta = sum_j p dp (the 16 slot groups of the row add theirs by shuffles:
+        // exact for the p and dp at hand, so a row whose softmax sees one slot gets g = 0), g = scale p
+        // (dp - delta), and p o A, g o A in bf16
+        // Each thread takes rows lo + ip and lo + 15 - ip of its sub-block and walks u down from the
+        // sub-block's last token: one load of D_j(u) serves both rows (and both half-warps, which share
+        // the sub-block), and P, PV come four tokens at a time.
+        {
+            const int lo = sb * 16;
+            const int rowx[2] = {lo + ip, lo + 15 - ip}, spanx[2] = {ip, 15 - ip};
+            float as[2][SPT], ad[2][SPT], r[2][SPT];
 #pragma unroll
-                for (int k = 0; k < SPT; ++k) { acc[k] = 0.f; r[k] = 1.f; }
-                const float *prow = sP + row * kFS;
-#pragma unroll 4
-                for (int u = row; u >= lo; --u) {
-                    const float pv = prow[u];
+            for (int x = 0; x < 2; ++x)
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) { as[x][k] = 0.f; ad[x][k] = 0.f; r[x][k] = 1.f; }
+#pragma unroll
+            for (int q4 = 3; q4 >= 0; --q4) {
+                if (4 * q4 > spanx[1]) continue;
+                float pq[2][4], wq[2][4];
+#pragma unroll
+                for (int x = 0; x < 2; ++x) {
+                    lds_vec(&sP[rowx[x] * kBFS + lo + 4 * q4], pq[x]);
+                    lds_vec(&sPV[rowx[x] * kBFS + lo + 4 * q4], wq[x]);
+                }
+#pragma unroll
+                for (int e = 3; e >= 0; --e) {
+                    const int uo = 4 * q4 + e;
+                    if (uo > spanx[1]) continue;
                     float dv[SPT];
-                    if constexpr (SPT == 4) {
-                        const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kFS + sg * 4]);
-                        dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
-                    } else {
-                        const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kFS + sg * 2]);
-                        dv[0] = d2.x; dv[1] = d2.y;
-                    }
+                    lds_vec(&sD[(lo + uo) * kBSS + sg * SPT], dv);
 #pragma unroll
-                    for (int k = 0; k < SPT; ++k) {
-                        acc[k] = fmaf(pv, dv[k] * r[k], acc[k]);
-                        r[k] = fmaf(-r[k], dv[k], r[k]);
-                    }
-                }
-                const long long t = a.pos0 + t0 + row;
-#pragma unroll
-                for (int k = 0; k < SPT; ++k) {
-                    const int j = sg * SPT + k;
-                    const float sc = a.scale * (sY[row * kFS + j] + acc[k]);
-                    sY[row * kFS + j] = (t >= sdelta[j]) ? sc : -INFINITY;
-                }
-            }
-            __syncthreads();
-            // ---- softmax over the slots: eight threads per row
-            {
-                constexpr int SPR = S / 8;
-                const int row = threadIdx.x >> 3, sub = threadIdx.x & 7;
-                float v[SPR], mx = -INFINITY;
-#pragma unroll
-                for (int k = 0; k < SPR; ++k) {
-                    v[k] = sY[row * kFS + sub * SPR + k];
-                    mx = fmaxf(mx, v[k]);
-                }
-#pragma unroll
-                for (int o = 4; o >= 1; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-                float sum = 0.f;
-#pragma unroll
-                for (int k = 0; k < SPR; ++k) {
-                    v[k] = __expf(v[k] - mx);
-                    sum += v[k];
-                }
-#pragma unroll
-                for (int o = 4; o >= 1; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-                const float inv = 1.f / sum;
-#pragma unroll
-                for (int k = 0; k < SPR; k += 2) {
-                    const int j = sub * SPR + k;
-                    const float p0 = v[k] * inv, p1 = v[k + 1] * inv;
-                    sY[row * kFS + j] = p0;
-                    sY[row * kFS + j + 1] = p1;
-                    const float g0 = sGpre[(row >> 4) * S + j], g1 = sGpre[(row >> 4) * S + j + 1];
-                    st_bf16x2(sPA, kDC, row, j, p0 * g0 * sAl[row * kFS + j], p1 * g1 * sAl[row * kFS + j + 1]);
-                }
-                if (sub == 0 && row < n) a.lse[(size_t)bh * a.L + t0 + row] = mx + __logf(sum);
-            }
-            __syncthreads();
-            // ---- G[tau, u] = sum_j p[tau, j] W_j(tau, u).  Diagonal sub-blocks on the CUDA cores: the walk
-            // above with q_j = p_j r_j, the 16 slot groups of a row adding their partial sums by shuffles
-            // within their half-warp (the two half-warps of a warp walk rows of different lengths).
-            const unsigned hmask = 0xffffu << (lane & 16);
-#pragma unroll 1
-            for (int rr = 0; rr < 2; ++rr) {
-                const int row = sb * 16 + (rr ? 15 - ip : ip), span = row - sb * 16;   // u = row - i, i <= span
-                float qv[SPT], gp[16];
-#pragma unroll
-                for (int k = 0; k < SPT; ++k) qv[k] = sY[row * kFS + sg * SPT + k];
-#pragma unroll
-                for (int i = 0; i < 16; ++i) {
-                    gp[i] = 0.f;
-                    if (i <= span) {
-                        const int u = row - i;
-                        float dv[SPT];
-                        if constexpr (SPT == 4) {
-                            const float4 d4 = *reinterpret_cast<const float4 *>(&sD[u * kFS + sg * 4]);
-                            dv[0] = d4.x; dv[1] = d4.y; dv[2] = d4.z; dv[3] = d4.w;
-                        } else {
-                            const float2 d2 = *reinterpret_cast<const float2 *>(&sD[u * kFS + sg * 2]);
-                            dv[0] = d2.x; dv[1] = d2.y;
-                        }
+                    for (int x = 0; x < 2; ++x) {
+                        if (uo > spanx[x]) continue;
 #pragma unroll
                         for (int k = 0; k < SPT; ++k) {
-                            gp[i] = fmaf(qv[k], dv[k], gp[i]);
-                            qv[k] = fmaf(-qv[k], dv[k], qv[k]);
+                            const float w = dv[k] * r[x][k];
+                            as[x][k] = fmaf(pq[x][e], w, as[x][k]);
+                            ad[x][k] = fmaf(wq[x][e], w, ad[x][k]);
+                            r[x][k] = fmaf(-r[x][k], dv[k], r[x][k]);
                         }
                     }
                 }
-                // transposing butterfly over the 16 slot groups: after the stage of width o a lane with bit
-                // o set holds in gp[i] the sums of entries i + o; at the end lane sg holds entry sg
+            }
+            float pj[2][SPT], dpj[2][SPT], pdp[2] = {0.f, 0.f};
+            int dlt[SPT];
+            lds_vec(&sdelta[sg * SPT], dlt);
 #pragma unroll
-                for (int o = 8; o >= 1; o >>= 1) {
-                    const bool up = (sg & o) != 0;
+            for (int x = 0; x < 2; ++x) {
+                const int row = rowx[x];
+                const long long t = a.pos0 + t0 + row;
+                const bool live = row < n;
+                const float lr = sLse[row];
+                float sv[SPT], dpv[SPT];
+                lds_vec(&sS[row * kBSS + sg * SPT], sv);
+                lds_vec(&sDP[row * kBSS + sg * SPT], dpv);
 #pragma unroll
-                    for (int i = 0; i < o; ++i) {
-                        const float send = up ? gp[i] : gp[i + o];
-                        const float mine = up ? gp[i + o] : gp[i];
-                        gp[i] = mine + __shfl_xor_sync(hmask, send, o);
+                for (int k = 0; k < SPT; ++k) {
+                    const float sc = a.scale * (sv[k] + as[x][k]);
+                    pj[x][k] = (live && t >= dlt[k]) ? __expf(sc - lr) : 0.f;
+                    dpj[x][k] = dpv[k] + ad[x][k];
+                    pdp[x] = fmaf(pj[x][k], dpj[x][k], pdp[x]);
+                }
+            }
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1) {
+                pdp[0] += __shfl_xor_sync(hmask, pdp[0], o);
+                pdp[1] += __shfl_xor_sync(hmask, pdp[1], o);
+            }
+            float gpre[SPT];
+            lds_vec(&sGpre[sb * S + sg * SPT], gpre);
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                const int row = rowx[x];
+                float gj[SPT], al[SPT], pa[SPT], ga[SPT];
+                lds_vec(&sAl[row * kBSS + sg * SPT], al);
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) {
+                    gj[k] = a.scale * pj[x][k] * (dpj[x][k] - pdp[x]);
+                    const float A = gpre[k] * al[k];
+                    pa[k] = pj[x][k] * A;
+                    ga[k] = gj[k] * A;
+                }
+                sts_vec(&sS[row * kBSS + sg * SPT], pj[x]);
+                sts_vec(&sDP[row * kBSS + sg * SPT], gj);
+                st_bf16_vec(sPA + sw_off(kBC, row, sg * SPT), pa);
+                st_bf16_vec(sGA + sw_off(kBC, row, sg * SPT), ga);
+            }
+        }
+        __syncthreads();
+        // ---- (d) G = sum_j p W and G^ = sum_j g W: diagonal sub-blocks by the walk (partials per step in
+        // registers, one transposing butterfly over the 16 slot groups each), the block of sub-block 1
+        // over sub-block 0 on the tensor cores (warp 0: G, warp 1: G^)
+        // (rows lo + ip and lo + 15 - ip walk u down together, as above; the partial sums are kept by u)
+        {
+            const int lo = sb * 16;
+            const int rowx[2] = {lo + ip, lo + 15 - ip}, spanx[2] = {ip, 15 - ip};
+            float qv[2][SPT], hv[2][SPT], gp[2][16], hp[2][16];
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                lds_vec(&sS[rowx[x] * kBSS + sg * SPT], qv[x]);
+                lds_vec(&sDP[rowx[x] * kBSS + sg * SPT], hv[x]);
+            }
+#pragma unroll
+            for (int uo = 15; uo >= 0; --uo) {
+#pragma unroll
+                for (int x = 0; x < 2; ++x) {
+                    gp[x][uo] = 0.f;
+                    hp[x][uo] = 0.f;
+                }
+                if (uo > spanx[1]) continue;
+                float dv[SPT];
+                lds_vec(&sD[(lo + uo) * kBSS + sg * SPT], dv);
+#pragma unroll
+                for (int x = 0; x < 2; ++x) {
+                    if (uo > spanx[x]) continue;
+#pragma unroll
+                    for (int k = 0; k < SPT; ++k) {
+                        gp[x][uo] = fmaf(qv[x][k], dv[k], gp[x][uo]);
+                        hp[x][uo] = fmaf(hv[x][k], dv[k], hp[x][uo]);
+                        qv[x][k] = fmaf(-qv[x][k], dv[k], qv[x][k]);
+                        hv[x][k] = fmaf(-hv[x][k], dv[k], hv[x][k]);
                     }
                 }
-                if (sg <= span)
-                    *reinterpret_cast<__nv_bfloat16 *>(sGm + sw_off(kDC, row, row - sg)) = __float2bfloat16_rn(gp[0]);
             }
-            // sub-blocks B_u < B_tau on the tensor cores: G_blk = (p o alpha o gamma) beta_blk^T, the
-            // contraction running over the slots; warp w < 6 takes the pair (bt, bu) of w
-            if (warp < 6) {
-                const int gbt = 1 + (warp >= 1) + (warp >= 3), gbu = warp - gbt * (gbt - 1) / 2, m0 = gbt * 16;
-                float acc[2][4] = {};
+            // transposing butterfly: slot group sg ends with the row's total at u = lo + sg
 #pragma unroll
-                for (int kk = 0; kk < S / 16; ++kk) {
-                    float x[2][2][2];   // [row g8 / g8 + 8][column half][pair]
+            for (int o = 8; o >= 1; o >>= 1) {
+                const bool up = (sg & o) != 0;
 #pragma unroll
-                    for (int ch = 0; ch < 2; ++ch)
+                for (int i = 0; i < o; ++i)
 #pragma unroll
-                        for (int e = 0; e < 2; ++e) {
-                            const int j = kk * 16 + ch * 8 + 2 * t4 + e;
-                            float gam = 1.f;
-                            for (int b2 = gbu + 1; b2 < gbt; ++b2) gam *= sG4[b2 * S + j];
+                    for (int x = 0; x < 2; ++x) {
+                        const float s1 = up ? gp[x][i] : gp[x][i + o], m1 = up ? gp[x][i + o] : gp[x][i];
+                        const float s2 = up ? hp[x][i] : hp[x][i + o], m2 = up ? hp[x][i + o] : hp[x][i];
+                        gp[x][i] = m1 + __shfl_xor_sync(hmask, s1, o);
+                        hp[x][i] = m2 + __shfl_xor_sync(hmask, s2, o);
+                    }
+            }
 #pragma unroll
-                            for (int rh = 0; rh < 2; ++rh) {
-                                const int row = m0 + g8 + rh * 8;
-                                x[rh][ch][e] = sY[row * kFS + j] * sAl[row * kFS + j] * gam;
-                            }
+            for (int x = 0; x < 2; ++x)
+                if (sg <= spanx[x]) {
+                    const uint32_t off = sw_off(kBC, rowx[x], lo + sg);
+                    *reinterpret_cast<__nv_bfloat16 *>(sGm + off) = __float2bfloat16_rn(gp[x][0]);
+                    *reinterpret_cast<__nv_bfloat16 *>(sGh + off) = __float2bfloat16_rn(hp[x][0]);
+                }
+        }
+        if (warp < 2) {
+            const float *src = warp ? sDP : sS;
+            float acc[2][4] = {};
+#pragma unroll
+            for (int kk = 0; kk < SB; ++kk) {
+                float x[2][2][2];
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e)
+#pragma unroll
+                        for (int rh = 0; rh < 2; ++rh) {
+                            const int row = 16 + g8 + rh * 8, j = kk * 16 + ch * 8 + 2 * t4 + e;
+                            x[rh][ch][e] = src[row * kBSS + j] * sAl[row * kBSS + j];
                         }
-                    const uint32_t af[4] = {tc::pack_bf16x2(x[0][0][0], x[0][0][1]), tc::pack_bf16x2(x[1][0][0], x[1][0][1]),
-                                            tc::pack_bf16x2(x[0][1][0], x[0][1][1]), tc::pack_bf16x2(x[1][1][0], x[1][1][1])};
-                    uint32_t b[4];
-                    load_b_kn(uBeta, S, gbu * 16, kk * 16, b);
-                    mma16816(acc[0], af, b[0], b[1]);
-                    mma16816(acc[1], af, b[2], b[3]);
-                }
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int col = gbu * 16 + h * 8 + 2 * t4;
-                    st_bf16x2(sGm, kDC, m0 + g8, col, acc[h][0], acc[h][1]);
-                    st_bf16x2(sGm, kDC, m0 + g8 + 8, col, acc[h][2], acc[h][3]);
-                }
+                const uint32_t af[4] = {tc::pack_bf16x2(x[0][0][0], x[0][0][1]), tc::pack_bf16x2(x[1][0][0], x[1][0][1]),
+                                        tc::pack_bf16x2(x[0][1][0], x[0][1][1]), tc::pack_bf16x2(x[1][1][0], x[1][1][1])};
+                uint32_t b[4];
+                load_b_kn(uBeta, S, 0, kk * 16, b);
+                mma16816(acc[0], af, b[0], b[1]);
+                mma16816(acc[1], af, b[2], b[3]);
             }
-            __syncthreads();
-            // ---- O = (p o A) V~ + G V_c into the O tile (over the dead P tile)
-            {
-                constexpr int ONB = D / 64;                      // 16-column blocks per warp
-                const int m0 = (warp >> 2) * 16, nb0 = (warp & 3) * ONB * 16;
-                float acc[ONB][2][4] = {};
-                for (int k0 = 0; k0 < S; k0 += 16) {
-                    uint32_t af[4], b[4];
-                    load_a(uPA, kDC, m0, k0, af);
+            uint8_t *dst = warp ? sGh : sGm;
 #pragma unroll
-                    for (int nb = 0; nb < ONB; ++nb) {
-                        load_b_kn(uVst, S, nb0 + nb * 16, k0, b);
-                        mma16816(acc[nb][0], af, b[0], b[1]);
-                        mma16816(acc[nb][1], af, b[2], b[3]);
+            for (int h = 0; h < 2; ++h) {
+                const int col = h * 8 + 2 * t4;
+                st_bf16x2(dst, kBC, 16 + g8, col, acc[h][0], acc[h][1]);
+                st_bf16x2(dst, kBC, 24 + g8, col, acc[h][2], acc[h][3]);
+            }
+        }
+        __syncthreads();
+        // the tables are read: the next item's go in
+        if (threadIdx.x == 0 && nx < i1) issue_tab(nx);
+        // ---- (e) dQ = (g o A) K0 + G^ K (staged over s), the chunk's parts G^T Q of dK and G^T dO of dV:
+        // warp takes row block om0 and OCB column blocks
+        {
+            constexpr int OCB = DB / 4;
+            const int om0 = (warp & 1) * 16, on0 = (warp >> 1) * OCB * 16;
+            auto out3 = [&](int which) {
+                float acc[OCB][2][4] = {};
+                uint32_t af[4], b[4];
+                if (which == 0) {
+                    for (int k0 = 0; k0 < S; k0 += 16) {
+                        load_a(uGA, kBC, om0, k0, af);
+#pragma unroll
+                        for (int cb = 0; cb < OCB; ++cb) {
+                            load_b_kn(uK0, S, on0 + cb * 16, k0, b);
+                            mma16816(acc[cb][0], af, b[0], b[1]);
+                            mma16816(acc[cb][1], af, b[2], b[3]);
+                        }
+                    }
+                    for (int k0 = 0; k0 < kBC; k0 += 16) {
+                        load_a(uGh, kBC, om0, k0, af);
+#pragma unroll
+                        for (int cb = 0; cb < OCB; ++cb) {
+                            load_b_kn(uK, kBC, on0 + cb * 16, k0, b);
+                            mma16816(acc[cb][0], af, b[0], b[1]);
+                            mma16816(acc[cb][1], af, b[2], b[3]);
+                        }
+                    }
+                } else {
+                    const uint32_t ug = which == 1 ? uGh : uGm, ux = which == 1 ? uQ : uDO;
+                    for (int k0 = 0; k0 < kBC; k0 += 16) {
+                        load_a_t(ug, kBC, om0, k0, af);
+#pragma unroll
+                        for (int cb = 0; cb < OCB; ++cb) {
+                            load_b_kn(ux, kBC, on0 + cb * 16, k0, b);
+                            mma16816(acc[cb][0], af, b[0], b[1]);
+                            mma16816(acc[cb][1], af, b[2], b[3]);
+                        }
                     }
                 }
-                for (int k0 = 0; k0 < kDC; k0 += 16) {
-                    uint32_t af[4], b[4];
-                    load_a(uGm, kDC, m0, k0, af);
+                uint8_t *dst = which == 0 ? reinterpret_cast<uint8_t *>(sS) : which == 1 ? sO : sOst;
 #pragma unroll
-                    for (int nb = 0; nb < ONB; ++nb) {
-                        load_b_kn(uV, kDC, nb0 + nb * 16, k0, b);
-                        mma16816(acc[nb][0], af, b[0], b[1]);
-                        mma16816(acc[nb][1], af, b[2], b[3]);
-                    }
-                }
-#pragma unroll
-                for (int nb = 0; nb < ONB; ++nb)
+                for (int cb = 0; cb < OCB; ++cb)
 #pragma unroll
                     for (int h = 0; h < 2; ++h) {
-                        const int col = nb0 + nb * 16 + h * 8 + 2 * t4;
-                        st_bf16x2(sO, kDC, m0 + g8, col, acc[nb][h][0], acc[nb][h][1]);
-                        st_bf16x2(sO, kDC, m0 + g8 + 8, col, acc[nb][h][2], acc[nb][h][3]);
+                        const int col = on0 + cb * 16 + h * 8 + 2 * t4;
+                        st_bf16x2(dst, kBC, om0 + g8, col, acc[cb][h][0], acc[cb][h][1]);
+                        st_bf16x2(dst, kBC, om0 + g8 + 8, col, acc[cb][h][2], acc[cb][h][3]);
                     }
-            }
-        } else {
-            if (!tc::mbar_wait(&bar[1 + s], ph_kv[s] & 1)) {
-                report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (16 << 4));
-                ok = false;
-                break;
-            }
-            __syncthreads();   // A_end and Wend of this chunk
-        }
-        ph_kv[s] ^= 1;
-        // ---- state update: X~ <- A_end o X~ + Wend X_c (every warp: its NU state blocks, which share
-        // their slot rows and so Wend's fragments)
-        {
-            const int b0 = warp * NU, kv = b0 / (SB * DB), rem0 = b0 % (SB * DB);
-            const int j0 = (rem0 / DB) * 16, e00 = (rem0 % DB) * 16;
-            const float f0 = sAend[j0 + g8], f1 = sAend[j0 + g8 + 8];
-#pragma unroll
-            for (int i = 0; i < NU; ++i)
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    st[i][h][0] *= f0; st[i][h][1] *= f0;
-                    st[i][h][2] *= f1; st[i][h][3] *= f1;
-                }
-            const uint32_t ux = kv ? uV : uK;
-            for (int k0 = 0; k0 < kDC; k0 += 16) {
-                uint32_t af[4], b[4];
-                load_a(uW, S, j0, k0, af);
-#pragma unroll
-                for (int i = 0; i < NU; ++i) {
-                    load_b_kn(ux, kDC, e00 + i * 16, k0, b);
-                    mma16816(st[i][0], af, b[0], b[1]);
-                    mma16816(st[i][1], af, b[2], b[3]);
-                }
-            }
-        }
-        __syncthreads();   // Y and O have read the old state copy; every warp is done with this stage
-        if (threadIdx.x == 0 && c + 2 < c_end) issue_kv(c + 2);
-        if (outputs) {
-            store_state_copy();
-            // o of the chunk: one bulk tensor store (rows past the end of the sequence are clipped)
+            };
+            // dQ first: k, K0 and V0 are then free for the next item
+            out3(0);
             tc::fence_proxy_async_smem();
             __syncthreads();
             if (threadIdx.x == 0) {
-                for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(&tm_o, sO + db * kDC * 128, db * 64, t0, bh);
-                tc::bulk_commit();   // the store's read of the O tile is awaited before P is written over it
+                tc::tma_store_4d(&tm_dq, sS, 0, t0, 0, bh);
+                tc::bulk_commit();
+                if (nx < i1) issue_k(nx);
             }
+            out3(1);
+            out3(2);
+        }
+        // ---- the chunk's adjoint contributions Z_K = (g o A)^T Q, Z_V = (p o A)^T dO
+        z_product(skv ? uDO : uQ, skv ? uPA : uGA);
+        {
+            uint8_t *tile = skv ? sZV : sZK;
+#pragma unroll
+            for (int i = 0; i < NB2; ++i)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int e = se0 + i * 16 + h * 8 + 2 * t4;
+                    st_bf16x2(tile, S, sj0 + g8, e, st[i][h][0], st[i][h][1]);
+                    st_bf16x2(tile, S, sj0 + g8 + 8, e, st[i][h][2], st[i][h][3]);
+                }
+        }
+        tc::fence_proxy_async_smem();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int srow = (int)((((size_t)bh * nch + c) * 2) * S);
+            tc::tma_store_4d(&tm_dk, sO, 0, t0, 0, bh);
+            tc::tma_store_4d(&tm_dv, sOst, 0, t0, 0, bh);
+            tc::tma_store_3d(&tm_z, sZK, 0, srow, 0);
+            tc::tma_store_3d(&tm_z, sZV, 0, srow + S, 0);
+            tc::bulk_commit();
         }
     }
     if (threadIdx.x == 0) tc::bulk_wait0();
-    if (!ok) return;
-    // ---- results: the final state (last segment) or the segment's delta and decay product
-    float *dst = nullptr;
-    if (a.mode == 0) {
-        dst = a.seg_delta + ((size_t)bh * G + seg) * 2 * S * D;
-        if (trun == NRUN - 1) a.seg_decay[((size_t)bh * G + seg) * S + tj] = seg_dec;
-    } else if (seg == G - 1 && a.state_out) {
-        dst = a.state_out + (size_t)bh * 2 * S * D;
-    }
-    if (dst) {
-#pragma unroll
-        for (int i = 0; i < NU; ++i) {
-            const int b = warp * NU + i, kv = b / (SB * DB), rem = b % (SB * DB);
-            const int j0 = (rem / DB) * 16, e0 = (rem % DB) * 16;
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int e = e0 + h * 8 + 2 * t4;
-                *reinterpret_cast<float2 *>(&dst[((size_t)kv * S + j0 + g8) * D + e]) = make_float2(st[i][h][0], st[i][h][1]);
-                *reinterpret_cast<float2 *>(&dst[((size_t)kv * S + j0 + g8 + 8) * D + e]) =
-                    make_float2(st[i][h][2], st[i][h][3]);
-            }
-        }
-    }
 }
 
-// States entering each segment: X_in(0) = the call's initial state (or zero);
-// X_in(g+1) = prod_{segment g} a_j o X_in(g) + delta(g).  One thread per (head, K|V, slot, column).
-__global__ void k_dchunk_scan(int G, int S, int D, long long total, const float *__restrict__ state_in,
-                              const float *__restrict__ seg_delta, const float *__restrict__ seg_decay,
-                              float *__restrict__ win) {
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const long long sd = (long long)S * D;
-        const long long r = i / sd, within = i % sd;   // r = bh * 2 + kv
-        const long long bh = r / 2, kv = r % 2;
-        const int j = (int)(within / D);
-        float x = state_in ? state_in[i] : 0.f;
-        for (int g = 0; g < G; ++g) {
-            const size_t base = ((size_t)(bh * G + g) * 2 + kv) * sd + within;
-            win[base] = x;
-            if (g + 1 < G) x = fmaf(seg_decay[(size_t)(bh * G + g) * S + j], x, seg_delta[base]);
-        }
-    }
-}
+// ---- the forward's chunk chains (Sec. 3.3 forward): one work item per (head, 32-token chunk), each CTA
+// a run of consecutive chunks, two CTAs per SM.  Per item: P = Q K^T and Y = Q K0^T, the two-level
+// triangle sums of s, the softmax over the visible slots (lse written), G = sum_j p W, then
+// o = (p o A) V0 + G V, staged over s and stored by TMA.
+template <int D, int S>
+struct FwLayout {
+    static constexpr int kTile = kBC * D * 2;           // one [32][D] bf16 tile
+    static constexpr int q = 0, k = q + kTile, v = k + kTile;
+    static constexpr int k0 = v + kTile;                // bf16 [S][D]: K~ entering the chunk
+    static constexpr int v0 = k0 + S * D * 2;           // bf16 [S][D]: V~ entering the chunk
+    static constexpr int tab = v0 + S * D * 2;          // the chunk's tables (ChunkTab)
+    static constexpr int pa = tab + ((ChunkTab<S>::bytes + 1023) / 1024) * 1024;   // bf16 [32][64]: p o A
+    static constexpr int gm = pa + kBC * 128;           // bf16 [32][64] (u < 32): G
+    static constexpr int sf = gm + kBC * 128;           // fp32 [32][kBSS]: s, then p, then o staging (bf16)
+    static constexpr int pf = sf + kBC * kBSS * 4;      // fp32 [32][kBFS]: P
+    static constexpr int delta = pf + kBC * kBFS * 4;   // int [S]
+    static constexpr int bars = delta + S * 4;          // mbarriers: q, k, K0 and tables; v and V0
+    static constexpr int total = bars + 64;
+    static_assert(k0 % 1024 == 0 && tab % 1024 == 0 && pa % 1024 == 0 && sf % 1024 == 0 && kBC * kBSS * 4 >= kTile,
+                  "swizzled tiles need 1024-byte alignment");
+    static_assert(2 * (total + 1024) <= 228 * 1024, "two CTAs per SM");
+};
 
 template <int D, int S>
-cudaError_t launch_dchunk_t(const OpDims &d, const DcArgs &base, const DcPlan &pl, const void *q, const void *k,
-                            const void *v, void *o, cudaStream_t st) {
-    CUtensorMap tq, tk, tv, to;
-    const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
-    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
-    const uint32_t box[3] = {64, (uint32_t)kDC, 1};
-    if (!make_tmap_bf16(&tq, q, 3, dims, strides, box) || !make_tmap_bf16(&tk, k, 3, dims, strides, box) ||
-        !make_tmap_bf16(&tv, v, 3, dims, strides, box) || !make_tmap_bf16(&to, o, 3, dims, strides, box))
-        return cudaErrorInvalidValue;
-    const int smem = DcLayout<D, S>::total;
-    cudaError_t e = cudaFuncSetAttribute(k_dchunk<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    const unsigned blocks = (unsigned)((long long)d.B * d.H * pl.G);
-    DcArgs a = base;
-    if (pl.G > 1) {
-        a.mode = 0;
-        {
-            ProfScope ps(BLA_K_DECAY, st);
-            k_dchunk<D, S><<<blocks, kDThreads, smem, st>>>(tq, tk, tv, to, a);
-        }
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
-        const long long total = (long long)d.B * d.H * 2 * S * D;
-        const int sblocks = (int)((total + 255) / 256 < 4096 ? (total + 255) / 256 : 4096);
-        {
-            ProfScope ps(BLA_K_DECAY, st);
-            k_dchunk_scan<<<sblocks, 256, 0, st>>>(pl.G, S, D, total, a.state_in, a.seg_delta, a.seg_decay,
-                                                  const_cast<float *>(a.win));
-        }
-        if ((e = cudaGetLastError()) != cudaSuccess) return e;
+__global__ void __launch_bounds__(kBT, 2)
+    k_dfchain(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
+              const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_st,
+              const __grid_constant__ CUtensorMap tm_o, DbArgs a) {
+    using Lay = FwLayout<D, S>;
+    using Tab = ChunkTab<S>;
+    constexpr int SPT = S / 16, SB = S / 16, DB = D / 16, NBLK = 2 + SB;
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g8 = lane >> 2, t4 = lane & 3;
+    if (tc::smem_u32(dsm) & 1023u) {
+        if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (19 << 4) | ((int)blockIdx.x << 16));
+        return;
     }
-    a.mode = 1;
-    ProfScope ps(BLA_K_DECAY, st);
-    k_dchunk<D, S><<<blocks, kDThreads, smem, st>>>(tq, tk, tv, to, a);
-    return cudaGetLastError();
+    const int L = a.L, nch = (L + kBC - 1) / kBC;
+    const long long nitems = (long long)a.BH * nch;
+    uint8_t *sQ = dsm + Lay::q, *sK = dsm + Lay::k, *sV = dsm + Lay::v, *sK0 = dsm + Lay::k0, *sV0 = dsm + Lay::v0;
+    uint8_t *sTab = dsm + Lay::tab, *sBeta = sTab + Tab::beta, *sPA = dsm + Lay::pa, *sGm = dsm + Lay::gm;
+    float *sS = reinterpret_cast<float *>(dsm + Lay::sf), *sP = reinterpret_cast<float *>(dsm + Lay::pf);
+    float *sD = reinterpret_cast<float *>(sTab + Tab::d), *sAl = reinterpret_cast<float *>(sTab + Tab::alpha);
+    float *sGpre = reinterpret_cast<float *>(sTab + Tab::gpre);
+    int *sdelta = reinterpret_cast<int *>(dsm + Lay::delta);
+    uint64_t *bar = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
+    const uint32_t uQ = tc::smem_u32(sQ), uK = tc::smem_u32(sK), uV = tc::smem_u32(sV);
+    const uint32_t uK0 = tc::smem_u32(sK0), uV0 = tc::smem_u32(sV0), uBeta = tc::smem_u32(sBeta);
+    const uint32_t uPA = tc::smem_u32(sPA), uGm = tc::smem_u32(sGm);
+
+    if (threadIdx.x == 0) {
+        tc::mbar_init(&bar[0], 1);
+        tc::mbar_init(&bar[1], 1);
+        tc::fence_barrier_init();
+    }
+    // the upper triangle of G and the columns past S of p o A stay zero
+    for (int i = threadIdx.x; i < kBC * 64 / 2; i += kBT) {
+        reinterpret_cast<uint32_t *>(sGm)[i] = 0u;
+        reinterpret_cast<uint32_t *>(sPA)[i] = 0u;
+    }
+    __syncthreads();
+
+    uint32_t ph0 = 0, ph1 = 0;
+    bool ok = true;
+    const int sg = threadIdx.x & 15, rp = threadIdx.x >> 4, sb = rp >> 3, ip = rp & 7;
+    const unsigned hmask = 0xffffu << (lane & 16);
+    const int i0 = (int)blockIdx.x * a.ipc, i1 = (int)min(nitems, (long long)i0 + a.ipc);
+    auto tab_of = [&](int it) {
+        const int tb = a.ntab > 1 ? (it / nch) % a.H : 0;
+        return a.ctab + ((size_t)tb * nch + (size_t)(it % nch)) * Tab::bytes;
+    };
+    // Item it + 1's loads are issued while item it runs, each once its place is free: q, k and K0 after
+    // the P/Y products, the tables after G, v and V0 after o.  Barrier 0 covers q, k, K0 and the
+    // tables (waited at the item's start), barrier 1 v and V0 (waited before o).
+    auto issue_qk = [&](int it) {
+        const int c = it % nch, bh = it / nch;
+        tc::mbar_arrive_expect_tx(&bar[0], (uint32_t)(2 * Lay::kTile + S * D * 2 + Tab::bytes));
+        tc::tma_load_4d(sQ, &tm_q, &bar[0], 0, c * kBC, 0, bh);
+        tc::tma_load_4d(sK, &tm_k, &bar[0], 0, c * kBC, 0, bh);
+        tc::tma_load_3d(sK0, &tm_st, &bar[0], 0, (int)((((size_t)bh * nch + c) * 2) * S), 0);
+    };
+    auto issue_tab = [&](int it) { tc::bulk_load(sTab, tab_of(it), (uint32_t)Tab::bytes, &bar[0]); };
+    auto issue_v = [&](int it) {
+        const int c = it % nch, bh = it / nch;
+        tc::mbar_arrive_expect_tx(&bar[1], (uint32_t)(Lay::kTile + S * D * 2));
+        tc::tma_load_4d(sV, &tm_v, &bar[1], 0, c * kBC, 0, bh);
+        tc::tma_load_3d(sV0, &tm_st, &bar[1], 0, (int)((((size_t)bh * nch + c) * 2 + 1) * S), 0);
+    };
+    if (i0 < i1 && threadIdx.x == 0) {
+        issue_qk(i0);
+        issue_tab(i0);
+        issue_v(i0);
+    }
+    int cur_hd = -1;
+    for (int it = i0; it < i1 && ok; ++it) {
+        const int c = it % nch, bh = it / nch, hd = bh % a.H;
+        const int t0 = c * kBC, n = min(kBC, L - t0);
+        const int nx = it + 1;
+        if (threadIdx.x == kBT - 32 && nx < i1) {
+            // the next item's q, k and states into L2 (their loads follow this item's P and Y)
+            const int cn = nx % nch, bn = nx / nch;
+            tc::tma_prefetch_4d(&tm_q, 0, cn * kBC, 0, bn);
+            tc::tma_prefetch_4d(&tm_k, 0, cn * kBC, 0, bn);
+            tc::bulk_prefetch_l2(a.states + (((size_t)bn * nch + cn) * 2) * S * D, (uint32_t)(2 * S * D * 2));
+        }
+        // sdelta was last read before the previous item's closing barriers
+        if (hd != cur_hd) {
+            for (int j = threadIdx.x; j < S; j += kBT) sdelta[j] = a.delta[(size_t)hd * a.hs_delta + j];
+            cur_hd = hd;
+        }
+        if (!tc::mbar_wait(&bar[0], ph0)) {
+            report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (19 << 4));
+            ok = false;
+            break;
+        }
+        ph0 ^= 1;
+        // ---- (a) P = Q K^T and Y = Q K0^T: warp takes row block m0 and column blocks bi and bi + 4 of
+        // the row block's 2 + S/16 (blocks 0, 1 are P's, the rest Y's); Y stays in registers
+        const int m0 = (warp & 1) * 16, bi = warp >> 1, bt = m0 >> 4;
+        const bool has2 = bi + 4 < NBLK;
+        float acc0[2][4] = {}, acc1[2][4] = {};
+        for (int k0 = 0; k0 < D; k0 += 16) {
+            uint32_t af[4], b[4];
+            load_a(uQ, kBC, m0, k0, af);
+            if (bi < 2) load_b_nk(uK, kBC, bi * 16, k0, b);
+            else load_b_nk(uK0, S, (bi - 2) * 16, k0, b);
+            mma16816(acc0[0], af, b[0], b[1]);
+            mma16816(acc0[1], af, b[2], b[3]);
+            if (has2) {
+                load_b_nk(uK0, S, (bi + 2) * 16, k0, b);
+                mma16816(acc1[0], af, b[0], b[1]);
+                mma16816(acc1[1], af, b[2], b[3]);
+            }
+        }
+        if (bi < 2) {
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int col = bi * 16 + h * 8 + 2 * t4;
+                *reinterpret_cast<float2 *>(&sP[(m0 + g8) * kBFS + col]) = make_float2(acc0[h][0], acc0[h][1]);
+                *reinterpret_cast<float2 *>(&sP[(m0 + g8 + 8) * kBFS + col]) = make_float2(acc0[h][2], acc0[h][3]);
+            }
+        }
+        // the previous item's o store has read its staging tile (s, written next)
+        if (threadIdx.x == 0) tc::bulk_wait_read0();
+        __syncthreads();
+        // q, k and K0 are read: the next item's go in
+        if (threadIdx.x == 0 && nx < i1) issue_qk(nx);
+        // ---- (b) the off-diagonal block of sub-block 1 over sub-block 0 (W = alpha beta there), and
+        // alpha (Gpre Y + F) into s, for the warp's Y blocks
+        auto y_block = [&](int yb, const float (&y)[2][4]) {
+            const int n0 = yb * 16;
+            float facc[2][4] = {};
+            if (bt == 1) {
+                const float *p0 = sP + (m0 + g8) * kBFS + 2 * t4, *p1 = p0 + 8 * kBFS;
+                const uint32_t af[4] = {tc::pack_bf16x2(p0[0], p0[1]), tc::pack_bf16x2(p1[0], p1[1]),
+                                        tc::pack_bf16x2(p0[8], p0[9]), tc::pack_bf16x2(p1[8], p1[9])};
+                uint32_t b[4];
+                load_b_nk(uBeta, S, n0, 0, b);
+                mma16816(facc[0], af, b[0], b[1]);
+                mma16816(facc[1], af, b[2], b[3]);
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int row = m0 + g8 + ((q >> 1) << 3), j = n0 + h * 8 + 2 * t4 + (q & 1);
+                    sS[row * kBSS + j] = sAl[row * kBSS + j] * fmaf(sGpre[bt * S + j], y[h][q], facc[h][q]);
+                }
+        };
+        if (bi >= 2) y_block(bi - 2, acc0);
+        if (has2) y_block(bi + 2, acc1);
+        __syncthreads();
+        // ---- (c) the diagonal sub-blocks of s on the CUDA cores, then the softmax over the visible
+        // slots (the 16 slot groups of a row meet by shuffles), lse, p and p o A.  Each thread takes rows
+        // lo + ip and lo + 15 - ip of its sub-block and walks u down from the sub-block's last token:
+        // one load of D_j(u) serves both rows and both half-warps, P comes four tokens at a time.
+        {
+            const int lo = sb * 16;
+            const int rowx[2] = {lo + ip, lo + 15 - ip}, spanx[2] = {ip, 15 - ip};
+            float as[2][SPT], r[2][SPT];
+#pragma unroll
+            for (int x = 0; x < 2; ++x)
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) { as[x][k] = 0.f; r[x][k] = 1.f; }
+#pragma unroll
+            for (int q4 = 3; q4 >= 0; --q4) {
+                if (4 * q4 > spanx[1]) continue;
+                float pq[2][4];
+#pragma unroll
+                for (int x = 0; x < 2; ++x) lds_vec(&sP[rowx[x] * kBFS + lo + 4 * q4], pq[x]);
+#pragma unroll
+                for (int e = 3; e >= 0; --e) {
+                    const int uo = 4 * q4 + e;
+                    if (uo > spanx[1]) continue;
+                    float dv[SPT];
+                    lds_vec(&sD[(lo + uo) * kBSS + sg * SPT], dv);
+#pragma unroll
+                    for (int x = 0; x < 2; ++x) {
+                        if (uo > spanx[x]) continue;
+#pragma unroll
+                        for (int k = 0; k < SPT; ++k) {
+                            as[x][k] = fmaf(pq[x][e], dv[k] * r[x][k], as[x][k]);
+                            r[x][k] = fmaf(-r[x][k], dv[k], r[x][k]);
+                        }
+                    }
+                }
+            }
+            int dlt[SPT];
+            lds_vec(&sdelta[sg * SPT], dlt);
+            float sc[2][SPT], mx[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                const long long t = a.pos0 + t0 + rowx[x];
+                float sv[SPT];
+                lds_vec(&sS[rowx[x] * kBSS + sg * SPT], sv);
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) {
+                    sc[x][k] = t >= dlt[k] ? a.scale * (sv[k] + as[x][k]) : -INFINITY;
+                    mx[x] = fmaxf(mx[x], sc[x][k]);
+                }
+            }
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1) {
+                mx[0] = fmaxf(mx[0], __shfl_xor_sync(hmask, mx[0], o));
+                mx[1] = fmaxf(mx[1], __shfl_xor_sync(hmask, mx[1], o));
+            }
+            float sum[2] = {0.f, 0.f};
+#pragma unroll
+            for (int x = 0; x < 2; ++x)
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) {
+                    sc[x][k] = __expf(sc[x][k] - mx[x]);
+                    sum[x] += sc[x][k];
+                }
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1) {
+                sum[0] += __shfl_xor_sync(hmask, sum[0], o);
+                sum[1] += __shfl_xor_sync(hmask, sum[1], o);
+            }
+            float gpre[SPT];
+            lds_vec(&sGpre[sb * S + sg * SPT], gpre);
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+                const int row = rowx[x];
+                const float inv = 1.f / sum[x];
+                float pj[SPT], al[SPT], pa[SPT];
+                lds_vec(&sAl[row * kBSS + sg * SPT], al);
+#pragma unroll
+                for (int k = 0; k < SPT; ++k) {
+                    pj[k] = sc[x][k] * inv;
+                    pa[k] = pj[k] * gpre[k] * al[k];
+                }
+                sts_vec(&sS[row * kBSS + sg * SPT], pj);
+                st_bf16_vec(sPA + sw_off(kBC, row, sg * SPT), pa);
+                if (sg == 0 && row < n) a.lse_out[(size_t)bh * L + t0 + row] = mx[x] + __logf(sum[x]);
+            }
+        }
+        __syncthreads();
+        // ---- (d) G = sum_j p W: the diagonal sub-blocks by the walk (partial sums kept by u, one
+        // transposing butterfly over the 16 slot groups), the block of sub-block 1 over sub-block 0 on
+        // the tensor cores (warp 0)
+        {
+            const int lo = sb * 16;
+            const int rowx[2] = {lo + ip, lo + 15 - ip}, spanx[2] = {ip, 15 - ip};
+            float qv[2][SPT], gp[2][16];
+#pragma unroll
+            for (int x = 0; x < 2; ++x) lds_vec(&sS[rowx[x] * kBSS + sg * SPT], qv[x]);
+#pragma unroll
+            for (int uo = 15; uo >= 0; --uo) {
+                gp[0][uo] = 0.f;
+                gp[1][uo] = 0.f;
+                if (uo > spanx[1]) continue;
+                float dv[SPT];
+                lds_vec(&sD[(lo + uo) * kBSS + sg * SPT], dv);
+#pragma unroll
+                for (int x = 0; x < 2; ++x) {
+                    if (uo > spanx[x]) continue;
+#pragma unroll
+                    for (int k = 0; k < SPT; ++k) {
+                        gp[x][uo] = fmaf(qv[x][k], dv[k], gp[x][uo]);
+                        qv[x][k] = fmaf(-qv[x][k], dv[k], qv[x][k]);
+                    }
+                }
+            }
+            // slot group sg ends with the row's total at u = lo + sg
+#pragma unroll
+            for (int o = 8; o >= 1; o >>= 1) {
+                const bool up = (sg & o) != 0;
+#pragma unroll
+                for (int i = 0; i < o; ++i)
+#pragma unroll
+                    for (int x = 0; x < 2; ++x) {
+                        const float s1 = up ? gp[x][i] : gp[x][i + o], m1 = up ? gp[x][i + o] : gp[x][i];
+                        gp[x][i] = m1 + __shfl_xor_sync(hmask, s1, o);
+                    }
+            }
+#pragma unroll
+            for (int x = 0; x < 2; ++x)
+                if (sg <= spanx[x])
+                    *reinterpret_cast<__nv_bfloat16 *>(sGm + sw_off(kBC, rowx[x], lo + sg)) =
+                        __float2bfloat16_rn(gp[x][0]);
+        }
+        if (warp == 0) {
+            float acc[2][4] = {};
+#pragma unroll
+            for (int kk = 0; kk < SB; ++kk) {
+                float xv[2][2][2];
+#pragma unroll
+                for (int ch = 0; ch < 2; ++ch)
+#pragma unroll
+                    for (int e = 0; e < 2; ++e)
+#pragma unroll
+                        for (int rh = 0; rh < 2; ++rh) {
+                            const int row = 16 + g8 + rh * 8, j = kk * 16 + ch * 8 + 2 * t4 + e;
+                            xv[rh][ch][e] = sS[row * kBSS + j] * sAl[row * kBSS + j];
+                        }
+                const uint32_t af[4] = {tc::pack_bf16x2(xv[0][0][0], xv[0][0][1]),
+                                        tc::pack_bf16x2(xv[1][0][0], xv[1][0][1]),
+                                        tc::pack_bf16x2(xv[0][1][0], xv[0][1][1]),
+                                        tc::pack_bf16x2(xv[1][1][0], xv[1][1][1])};
+                uint32_t b[4];
+                load_b_kn(uBeta, S, 0, kk * 16, b);
+                mma16816(acc[0], af, b[0], b[1]);
+                mma16816(acc[1], af, b[2], b[3]);
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int col = h * 8 + 2 * t4;
+                st_bf16x2(sGm, kBC, 16 + g8, col, acc[h][0], acc[h][1]);
+                st_bf16x2(sGm, kBC, 24 + g8, col, acc[h][2], acc[h][3]);
+            }
+        }
+        __syncthreads();
+        // the tables are read: the next item's go in
+        if (threadIdx.x == 0 && nx < i1) issue_tab(nx);
+        // ---- (e) o = (p o A) V0 + G V, staged over s: warp takes row block om0 and OCB column blocks
+        if (!tc::mbar_wait(&bar[1], ph1)) {
+            report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (19 << 4));
+            ok = false;
+            break;
+        }
+        ph1 ^= 1;
+        {
+            constexpr int OCB = DB / 4;
+            const int om0 = (warp & 1) * 16, on0 = (warp >> 1) * OCB * 16;
+            float acc[OCB][2][4] = {};
+            uint32_t af[4], b[4];
+            for (int k0 = 0; k0 < S; k0 += 16) {
+                load_a(uPA, kBC, om0, k0, af);
+#pragma unroll
+                for (int cb = 0; cb < OCB; ++cb) {
+                    load_b_kn(uV0, S, on0 + cb * 16, k0, b);
+                    mma16816(acc[cb][0], af, b[0], b[1]);
+                    mma16816(acc[cb][1], af, b[2], b[3]);
+                }
+            }
+            for (int k0 = 0; k0 < kBC; k0 += 16) {
+                load_a(uGm, kBC, om0, k0, af);
+#pragma unroll
+                for (int cb = 0; cb < OCB; ++cb) {
+                    load_b_kn(uV, kBC, on0 + cb * 16, k0, b);
+                    mma16816(acc[cb][0], af, b[0], b[1]);
+                    mma16816(acc[cb][1], af, b[2], b[3]);
+                }
+            }
+            uint8_t *dst = reinterpret_cast<uint8_t *>(sS);
+#pragma unroll
+            for (int cb = 0; cb < OCB; ++cb)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int col = on0 + cb * 16 + h * 8 + 2 * t4;
+                    st_bf16x2(dst, kBC, om0 + g8, col, acc[cb][h][0], acc[cb][h][1]);
+                    st_bf16x2(dst, kBC, om0 + g8 + 8, col, acc[cb][h][2], acc[cb][h][3]);
+                }
+        }
+        tc::fence_proxy_async_smem();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            tc::tma_store_4d(&tm_o, sS, 0, t0, 0, bh);
+            tc::bulk_commit();
+            if (nx < i1) issue_v(nx);   // v and V0 are read
+        }
+    }
+    if (threadIdx.x == 0) tc::bulk_wait0();
 }
 
-int sm_count_dc() {
+// ---- the tables of every (head, chunk), one thread per slot j: Wend and A_end for the thin passes,
+// and the chain's ChunkTab record (D, alpha, beta, Gpre).  D_j(t0 + u) = Dx[t0 + u + dmax - Delta_j];
+// tokens past L contribute nothing (D = 0).
+template <int S>
+__global__ void __launch_bounds__(S) k_dbtab(DbArgs a) {
+    using Tab = ChunkTab<S>;
+    const int c = blockIdx.x, h = blockIdx.y, j = threadIdx.x, nch = (a.L + kBC - 1) / kBC;
+    const int t0 = c * kBC, n = min(kBC, a.L - t0);
+    const float *src = a.Dx + (size_t)h * a.hs_dx + t0 + a.dmax - a.delta[(size_t)h * a.hs_delta + j];
+    const size_t ti = (size_t)h * nch + c;
+    uint8_t *w = a.etab + ti * EndTab<S>::bytes + EndTab<S>::wend;
+    uint8_t *rec = a.ctab + ti * Tab::bytes;
+    float *rd = reinterpret_cast<float *>(rec + Tab::d), *ral = reinterpret_cast<float *>(rec + Tab::alpha);
+    float *rg = reinterpret_cast<float *>(rec + Tab::gpre);
+    float dv[kBC];
+#pragma unroll
+    for (int u = 0; u < kBC; ++u) {
+        dv[u] = u < n ? src[u] : 0.f;
+        rd[u * kBSS + j] = dv[u];
+        for (int col = S + j; col < kBSS; col += S) rd[u * kBSS + col] = 0.f, ral[u * kBSS + col] = 0.f;
+    }
+    // alpha_j(tau): the decay from the start of tau's 16-token sub-block through tau; Gpre: before it
+    float p = 1.f;
+    rg[j] = 1.f;
+#pragma unroll
+    for (int u = 0; u < kBC; ++u) {
+        if (u == 16) {
+            rg[S + j] = p;
+            p = 1.f;
+        }
+        p *= 1.f - dv[u];
+        ral[u * kBSS + j] = p;
+    }
+    // Wend_j(u) = D_j(u) x the decay after u to the chunk's end; beta_j(u) the same to the end of u's
+    // sub-block
+    float r = 1.f, rb = 1.f;
+#pragma unroll
+    for (int u = kBC - 2; u >= 0; u -= 2) {
+        if (u == 14) rb = 1.f;
+        const float d1 = dv[u + 1], d0 = dv[u];
+        const float w1 = d1 * r;
+        r -= r * d1;
+        const float w0 = d0 * r;
+        r -= r * d0;
+        const float b1 = d1 * rb;
+        rb -= rb * d1;
+        const float b0 = d0 * rb;
+        rb -= rb * d0;
+        *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = tc::pack_bf16x2(w0, w1);
+        *reinterpret_cast<uint32_t *>(rec + Tab::beta + wmma16::sw_off(S, j, u)) = tc::pack_bf16x2(b0, b1);
+    }
+    for (int u = kBC; u < 64; u += 2) {
+        *reinterpret_cast<uint32_t *>(w + wmma16::sw_off(S, j, u)) = 0u;
+        *reinterpret_cast<uint32_t *>(rec + Tab::beta + wmma16::sw_off(S, j, u)) = 0u;
+    }
+    reinterpret_cast<float *>(a.etab + ti * EndTab<S>::bytes + EndTab<S>::aend)[j] = r;
+}
+
+// ---- the two thin passes along the sequence.  One CTA per (64-column strip, K~ or V~, head) with
+// 4 warps; the strip [S][64] (fp32) lives in the accumulator registers of the MMAs that update it.
+constexpr int kSW = 4;           // warps
+constexpr int kNS = 4;           // pipeline stages
+
+template <int S>
+struct StripMap {
+    static constexpr int WR = S / 16, WC = kSW / WR, NC = 64 / WC, NB = NC / 16;
+    static_assert(WR * WC == kSW && NB >= 1, "strip blocks per warp");
+};
+
+template <int S>
+struct ScanLayout {
+    static constexpr int kT = kBC * 128;                    // [32][64] bf16 tile
+    static constexpr int kW = S * 128;                      // [S][64] bf16 tile (Wend image, state strip)
+    // a stage: z (reverse only) | k or dk | the EndTab record, rounded up to whole 1024-byte blocks
+    static constexpr int stage = ((kW + kT + EndTab<S>::bytes) + 1023) / 1024 * 1024;
+    static constexpr int mu = kNS * stage;                  // bf16 [S][64]: mu (reverse)
+    static constexpr int out = mu + kW;                     // 2 staging tiles: [S][64] (state) or [32][64]
+    static constexpr int bars = out + 2 * kW;
+    static constexpr int total = bars + 8 * kNS;
+    static_assert(stage % 1024 == 0 && mu % 1024 == 0 && out % 1024 == 0, "swizzled tiles need 1024-byte alignment");
+};
+
+// REV = false: K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c from the zero state; the state entering chunk c
+// goes to `states` (bf16).  REV = true: from the last chunk back, dK_c += Wend(c)^T mu_c (bf16 MMA on a
+// copy of mu), then mu_{c-1} = A_end(c) o mu_c + Z_c.
+template <int D, int S, bool REV>
+__global__ void __launch_bounds__(kSW * 32)
+    k_dbscan(const __grid_constant__ CUtensorMap tm_x0, const __grid_constant__ CUtensorMap tm_x1,
+             const __grid_constant__ CUtensorMap tm_st, DbArgs a) {
+    using Lay = ScanLayout<S>;
+    using M = StripMap<S>;
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g8 = lane >> 2, t4 = lane & 3;
+    if (tc::smem_u32(dsm) & 1023u) {
+        if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (18 << 4) | ((int)blockIdx.x << 16));
+        return;
+    }
+    const int strip = blockIdx.x, kv = blockIdx.y, bh = blockIdx.z;
+    const int tab = a.ntab > 1 ? bh % a.H : 0;
+    const int nch = (a.L + kBC - 1) / kBC, x = strip * 64;
+    const CUtensorMap *tx = kv ? &tm_x1 : &tm_x0;   // k / v (forward) or dk / dv (reverse)
+    uint64_t *full = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
+    uint8_t *sMu = dsm + Lay::mu, *sOut = dsm + Lay::out;
+    // stage s: Z strip (reverse) at +0, the [32][64] tile at +kW, the EndTab record at +kW + kT
+    auto sz = [&](int s) { return dsm + s * Lay::stage; };
+    auto sx = [&](int s) { return dsm + s * Lay::stage + Lay::kW; };
+    auto sw = [&](int s) { return dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::wend; };
+    auto sa = [&](int s) {
+        return reinterpret_cast<float *>(dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::aend);
+    };
+    auto chunk_of = [&](int i) { return REV ? nch - 1 - i : i; };
+    auto issue = [&](int i) {
+        const int s = i % kNS, c = chunk_of(i);
+        const size_t ti = (size_t)tab * nch + c;
+        const uint32_t bytes = (uint32_t)(Lay::kT + EndTab<S>::bytes + (REV ? Lay::kW : 0));
+        tc::mbar_arrive_expect_tx(&full[s], bytes);
+        if (REV) tc::tma_load_2d(sz(s), &tm_st, &full[s], x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
+        tc::tma_load_3d(sx(s), tx, &full[s], x, c * kBC, bh);
+        tc::bulk_load(sw(s), a.etab + ti * EndTab<S>::bytes, (uint32_t)EndTab<S>::bytes, &full[s]);
+    };
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kNS; ++s) tc::mbar_init(&full[s], 1);
+        tc::fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 32)
+        for (int i = 0; i < kNS && i < nch; ++i) issue(i);
+
+    const int r0 = (warp % M::WR) * 16, c0 = (warp / M::WR) * M::NC;
+    float acc[M::NB][2][4];
+    // the strip's rows of an fp32 [BH][2][S][D] state: acc element (b, h, q) is row r0 + g8 + 8 (q >> 1),
+    // column x + c0 + 16 b + 8 h + 2 t4 + (q & 1)
+    auto strip_row = [&](int rh) { return ((size_t)(bh * 2 + kv) * S + r0 + g8 + 8 * rh) * D + x + c0 + 2 * t4; };
+#pragma unroll
+    for (int i = 0; i < M::NB; ++i)
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int rh = 0; rh < 2; ++rh) {
+                float2 v0 = make_float2(0.f, 0.f);
+                if (!REV && a.state_in)
+                    v0 = *reinterpret_cast<const float2 *>(a.state_in + strip_row(rh) + i * 16 + h * 8);
+                acc[i][h][2 * rh] = v0.x;
+                acc[i][h][2 * rh + 1] = v0.y;
+            }
+    auto put = [&](uint8_t *tile) {   // acc (bf16) into a swizzled [S][64] tile
+#pragma unroll
+        for (int i = 0; i < M::NB; ++i)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int e = c0 + i * 16 + h * 8 + 2 * t4;
+                st_bf16x2(tile, S, r0 + g8, e, acc[i][h][0], acc[i][h][1]);
+                st_bf16x2(tile, S, r0 + g8 + 8, e, acc[i][h][2], acc[i][h][3]);
+            }
+    };
+    bool ok = true;
+    for (int i = 0; i < nch; ++i) {
+        const int s = i % kNS, c = chunk_of(i), ob = i & 1;
+        if (threadIdx.x == 0) tc::bulk_wait_read1();   // the store that used staging tile ob has read it
+        if (!REV) {
+            __syncthreads();
+            put(sOut + ob * Lay::kW);   // the state entering chunk c
+        }
+        if (!tc::mbar_wait(&full[s], (uint32_t)((i / kNS) & 1))) {
+            report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (18 << 4));
+            ok = false;
+        }
+        if (__syncthreads_or(!ok)) break;
+        const float *ae = sa(s);
+        const float f0 = ae[r0 + g8], f1 = ae[r0 + g8 + 8];
+        const uint32_t uW = tc::smem_u32(sw(s)), uX = tc::smem_u32(sx(s));
+        if (!REV) {
+            // acc <- A_end o acc + Wend K_c: A = Wend [S][32 tokens], B = the chunk's strip [32][64]
+#pragma unroll
+            for (int b = 0; b < M::NB; ++b)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    acc[b][h][0] *= f0; acc[b][h][1] *= f0;
+                    acc[b][h][2] *= f1; acc[b][h][3] *= f1;
+                }
+#pragma unroll
+            for (int k0 = 0; k0 < kBC; k0 += 16) {
+                uint32_t af[4], bf[4];
+                load_a(uW, S, r0, k0, af);
+#pragma unroll
+                for (int b = 0; b < M::NB; ++b) {
+                    load_b_kn(uX, kBC, c0 + b * 16, k0, bf);
+                    mma16816(acc[b][0], af, bf[0], bf[1]);
+                    mma16816(acc[b][1], af, bf[2], bf[3]);
+                }
+            }
+        } else {
+            // dK_c [32][64] += Wend^T mu: warp takes token rows om0.. and 32 columns on0..
+            const bool live = i > 0;   // mu is zero after the last chunk
+            if (live) {
+                put(sMu);
+                __syncthreads();
+                const int om0 = (warp & 1) * 16, on0 = (warp >> 1) * 32;
+                float o[2][2][4] = {};
+                const uint32_t uMu = tc::smem_u32(sMu);
+#pragma unroll
+                for (int k0 = 0; k0 < S; k0 += 16) {
+                    uint32_t af[4], bf[4];
+                    load_a_t(uW, S, om0, k0, af);
+#pragma unroll
+                    for (int b = 0; b < 2; ++b) {
+                        load_b_kn(uMu, S, on0 + b * 16, k0, bf);
+                        mma16816(o[b][0], af, bf[0], bf[1]);
+                        mma16816(o[b][1], af, bf[2], bf[3]);
+                    }
+                }
+                const uint8_t *dk = sx(s);
+                uint8_t *dst = sOut + ob * Lay::kW;
+#pragma unroll
+                for (int b = 0; b < 2; ++b)
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int rh = 0; rh < 2; ++rh) {
+                            const int row = om0 + g8 + rh * 8, col = on0 + b * 16 + h * 8 + 2 * t4;
+                            const float2 l = __bfloat1622float2(
+                                *reinterpret_cast<const __nv_bfloat162 *>(dk + sw_off(kBC, row, col)));
+                            st_bf16x2(dst, kBC, row, col, o[b][h][2 * rh] + l.x, o[b][h][2 * rh + 1] + l.y);
+                        }
+            }
+            // mu <- A_end o mu + Z_c
+            const uint8_t *z = sz(s);
+#pragma unroll
+            for (int b = 0; b < M::NB; ++b)
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int rh = 0; rh < 2; ++rh) {
+                        const int row = r0 + g8 + rh * 8, col = c0 + b * 16 + h * 8 + 2 * t4;
+                        const float f = rh ? f1 : f0;
+                        const float2 zz =
+                            __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(z + sw_off(S, row, col)));
+                        acc[b][h][2 * rh] = fmaf(f, acc[b][h][2 * rh], zz.x);
+                        acc[b][h][2 * rh + 1] = fmaf(f, acc[b][h][2 * rh + 1], zz.y);
+                    }
+        }
+        tc::fence_proxy_async_smem();
+        __syncthreads();   // stage s and the staging tile are complete
+        if (threadIdx.x == 0) {
+            if (!REV) {
+                tc::tma_store_2d(&tm_st, sOut + ob * Lay::kW, x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
+                tc::bulk_commit();
+            } else if (i > 0) {
+                tc::tma_store_3d(tx, sOut + ob * Lay::kW, x, c * kBC, bh);
+                tc::bulk_commit();
+            }
+        }
+        // the loads come from another warp: each TMA issue holds its thread for a while
+        if (threadIdx.x == 32 && i + kNS < nch) issue(i + kNS);
+    }
+    if (!REV && ok && a.state_out) {
+#pragma unroll
+        for (int i = 0; i < M::NB; ++i)
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int rh = 0; rh < 2; ++rh)
+                    *reinterpret_cast<float2 *>(a.state_out + strip_row(rh) + i * 16 + h * 8) =
+                        make_float2(acc[i][h][2 * rh], acc[i][h][2 * rh + 1]);
+    }
+    if (threadIdx.x == 0) tc::bulk_wait0();
+}
+
+int sm_count_db() {
     int dev = 0, n = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 152;
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) return 152;
     return n;
 }
 
+template <int D, int S>
+cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v,
+                          const void *dout, void *dq, void *dk, void *dv, cudaStream_t st) {
+    CUtensorMap tk, tv, tst, tz, tdk, tdv;
+    const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
+    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
+    const uint32_t box[3] = {64, (uint32_t)kBC, 1};
+    const int nch = (d.L + kBC - 1) / kBC;
+    const uint64_t sdims[2] = {(uint64_t)D, (uint64_t)d.B * d.H * nch * 2 * S};
+    const uint64_t sstr[1] = {(uint64_t)D * 2};
+    const uint32_t sbox[2] = {64, (uint32_t)S};
+    if (!make_tmap_bf16(&tk, k, 3, dims, strides, box) || !make_tmap_bf16(&tv, v, 3, dims, strides, box) ||
+        !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) || !make_tmap_bf16(&tz, a.zbuf, 2, sdims, sstr, sbox) ||
+        !make_tmap_bf16(&tdk, dk, 3, dims, strides, box) || !make_tmap_bf16(&tdv, dv, 3, dims, strides, box))
+        return cudaErrorInvalidValue;
+    // the chain moves whole [32][D] and [S][D] tiles in one copy each: the 64-column blocks are a
+    // further dimension of the maps (128 bytes apart), so a box lands as [D / 64][rows][64]
+    CUtensorMap cq, ck, cv, cdo, cst, cz, cdq, cdk, cdv;
+    const uint64_t cdims[4] = {64, (uint64_t)d.L, (uint64_t)(D / 64), (uint64_t)d.B * d.H};
+    const uint64_t cstr[3] = {(uint64_t)D * 2, 128, (uint64_t)d.L * D * 2};
+    const uint32_t cbox[4] = {64, (uint32_t)kBC, (uint32_t)(D / 64), 1};
+    const uint64_t csdims[3] = {64, (uint64_t)d.B * d.H * nch * 2 * S, (uint64_t)(D / 64)};
+    const uint64_t csstr[2] = {(uint64_t)D * 2, 128};
+    const uint32_t csbox[3] = {64, (uint32_t)S, (uint32_t)(D / 64)};
+    if (!make_tmap_bf16(&cq, q, 4, cdims, cstr, cbox) || !make_tmap_bf16(&ck, k, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&cv, v, 4, cdims, cstr, cbox) || !make_tmap_bf16(&cdo, dout, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&cst, a.states, 3, csdims, csstr, csbox) ||
+        !make_tmap_bf16(&cz, a.zbuf, 3, csdims, csstr, csbox) || !make_tmap_bf16(&cdq, dq, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&cdk, dk, 4, cdims, cstr, cbox) || !make_tmap_bf16(&cdv, dv, 4, cdims, cstr, cbox))
+        return cudaErrorInvalidValue;
+    const int smem = BwLayout<D, S>::total, ssm = ScanLayout<S>::total;
+    cudaError_t e = cudaFuncSetAttribute(k_dbchain<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_dbscan<D, S, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_dbscan<D, S, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
+    if (e != cudaSuccess) return e;
+    ProfScope ps(BLA_K_DECAY, st);
+    k_dbtab<S><<<dim3((unsigned)nch, (unsigned)a.ntab), S, 0, st>>>(a);
+    const dim3 sgrid((unsigned)(D / 64), 2u, (unsigned)a.BH);
+    k_dbscan<D, S, false><<<sgrid, kSW * 32, ssm, st>>>(tk, tv, tst, a);
+    const long long items = (long long)a.BH * nch;
+    if (items > 0x7fffffffLL) return cudaErrorInvalidValue;   // the chain indexes its items in 32 bits
+    DbArgs ac = a;
+    ac.ipc = (int)((items + sm_count_db() - 1) / sm_count_db());
+    const int grid = (int)((items + ac.ipc - 1) / ac.ipc);
+    k_dbchain<D, S><<<(unsigned)grid, kBT, smem, st>>>(cq, ck, cv, cdo, cst, cz, cdq, cdk, cdv, ac);
+    k_dbscan<D, S, true><<<sgrid, kSW * 32, ssm, st>>>(tdk, tdv, tz, a);
+    return cudaGetLastError();
+}
+
+// the pieces of the backward's workspace: states, Z, Wend tables, A_end tables
+struct DbWs {
+    size_t states, z, etab, ctab, total;
+};
+
+DbWs db_ws(const OpDims &d, bool with_z) {
+    const size_t nch = (size_t)(d.L + kBC - 1) / kBC, ntab = d.periods ? (size_t)d.H : 1;
+    const size_t per = align_up((size_t)d.B * d.H * nch * 2 * d.S * d.dk * sizeof(__nv_bfloat16), 256);
+    DbWs w;
+    w.states = 0;
+    w.z = per;
+    w.etab = with_z ? 2 * per : per;
+    const size_t end_bytes = d.S == 32 ? (size_t)EndTab<32>::bytes : (size_t)EndTab<64>::bytes;
+    w.ctab = w.etab + align_up(ntab * nch * end_bytes, 256);
+    const size_t tab_bytes = d.S == 32 ? (size_t)ChunkTab<32>::bytes : (size_t)ChunkTab<64>::bytes;
+    w.total = w.ctab + align_up(ntab * nch * tab_bytes, 256);
+    return w;
+}
+
+template <int D, int S>
+cudaError_t launch_dfwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v, void *o,
+                          cudaStream_t st) {
+    CUtensorMap tk, tv, tst, cq, ck, cv, cst, co;
+    const int nch = (d.L + kBC - 1) / kBC;
+    const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
+    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
+    const uint32_t box[3] = {64, (uint32_t)kBC, 1};
+    const uint64_t sdims[2] = {(uint64_t)D, (uint64_t)d.B * d.H * nch * 2 * S};
+    const uint64_t sstr[1] = {(uint64_t)D * 2};
+    const uint32_t sbox[2] = {64, (uint32_t)S};
+    const uint64_t cdims[4] = {64, (uint64_t)d.L, (uint64_t)(D / 64), (uint64_t)d.B * d.H};
+    const uint64_t cstr[3] = {(uint64_t)D * 2, 128, (uint64_t)d.L * D * 2};
+    const uint32_t cbox[4] = {64, (uint32_t)kBC, (uint32_t)(D / 64), 1};
+    const uint64_t csdims[3] = {64, (uint64_t)d.B * d.H * nch * 2 * S, (uint64_t)(D / 64)};
+    const uint64_t csstr[2] = {(uint64_t)D * 2, 128};
+    const uint32_t csbox[3] = {64, (uint32_t)S, (uint32_t)(D / 64)};
+    if (!make_tmap_bf16(&tk, k, 3, dims, strides, box) || !make_tmap_bf16(&tv, v, 3, dims, strides, box) ||
+        !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) || !make_tmap_bf16(&cq, q, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&ck, k, 4, cdims, cstr, cbox) || !make_tmap_bf16(&cv, v, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&cst, a.states, 3, csdims, csstr, csbox) || !make_tmap_bf16(&co, o, 4, cdims, cstr, cbox))
+        return cudaErrorInvalidValue;
+    const int smem = FwLayout<D, S>::total, ssm = ScanLayout<S>::total;
+    cudaError_t e = cudaFuncSetAttribute(k_dfchain<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_dbscan<D, S, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
+    if (e != cudaSuccess) return e;
+    const long long items = (long long)a.BH * nch;
+    if (items > 0x7fffffffLL) return cudaErrorInvalidValue;   // the chain indexes its items in 32 bits
+    ProfScope ps(BLA_K_DECAY, st);
+    k_dbtab<S><<<dim3((unsigned)nch, (unsigned)a.ntab), S, 0, st>>>(a);
+    k_dbscan<D, S, false><<<dim3((unsigned)(D / 64), 2u, (unsigned)a.BH), kSW * 32, ssm, st>>>(tk, tv, tst, a);
+    DbArgs ac = a;
+    const long long slots = 2LL * sm_count_db();   // two chain CTAs per SM
+    ac.ipc = (int)((items + slots - 1) / slots);
+    const int grid = (int)((items + ac.ipc - 1) / ac.ipc);
+    k_dfchain<D, S><<<(unsigned)grid, kBT, smem, st>>>(cq, ck, cv, cst, co, ac);
+    return cudaGetLastError();
+}
+
 }  // namespace
+
+size_t decay_chunk_bwd_ws_bytes(const OpDims &d) { return db_ws(d, true).total; }
+size_t decay_chunk_fwd_ws_bytes(const OpDims &d) { return db_ws(d, false).total; }
 
 bool decay_chunk_supported(const OpDims &d) {
     return d.dtype == BLA_BF16 && d.dk == d.dv && (d.dk == 64 || d.dk == 128) && (d.S == 32 || d.S == 64) &&
            d.L > 0;
 }
 
-// Segments per head: one CTA per SM and per segment, as many segments as fill the SMs once.
-DcPlan decay_chunk_plan(const OpDims &d) {
-    DcPlan p;
-    const int nch = (d.L + kDC - 1) / kDC;
-    const long long BH = (long long)d.B * d.H;
-    long long G = sm_count_dc() / (BH > 0 ? BH : 1);
-    if (G < 1) G = 1;
-    if (G > nch) G = nch;
-    p.cps = (int)((nch + G - 1) / G);
-    p.G = (nch + p.cps - 1) / p.cps;
-    return p;
+cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, const float *Dx, const int *delta,
+                                   int hs_dx, int hs_delta, const void *q, const void *k, const void *v,
+                                   const void *dout, const float *lse, void *dq, void *dk, void *dv, void *ws,
+                                   cudaStream_t st) {
+    const DbWs w = db_ws(d, true);
+    char *base = static_cast<char *>(ws);
+    DbArgs a = {};
+    a.L = d.L; a.H = d.H; a.BH = d.B * d.H; a.ipc = 1; a.pos0 = pos0; a.scale = d.scale; a.dmax = dmax;
+    a.Dx = Dx; a.delta = delta; a.hs_dx = hs_dx; a.hs_delta = hs_delta;
+    a.lse = lse;
+    a.ntab = (hs_dx != 0 || hs_delta != 0) ? d.H : 1;
+    if (a.ntab > 1 && !d.periods) return cudaErrorInvalidValue;   // the tables are sized per head only then
+    a.states = reinterpret_cast<__nv_bfloat16 *>(base + w.states);
+    a.zbuf = reinterpret_cast<__nv_bfloat16 *>(base + w.z);
+    a.etab = reinterpret_cast<uint8_t *>(base + w.etab);
+    a.ctab = reinterpret_cast<uint8_t *>(base + w.ctab);
+    a.err = device_error_word();
+    if (d.dk == 64) return d.S == 32 ? launch_dbwd_t<64, 32>(d, a, q, k, v, dout, dq, dk, dv, st)
+                                     : launch_dbwd_t<64, 64>(d, a, q, k, v, dout, dq, dk, dv, st);
+    return d.S == 32 ? launch_dbwd_t<128, 32>(d, a, q, k, v, dout, dq, dk, dv, st)
+                     : launch_dbwd_t<128, 64>(d, a, q, k, v, dout, dq, dk, dv, st);
 }
 
 cudaError_t launch_decay_chunk(const OpDims &d, long long pos0, int dmax, const float *Dx, const int *delta,
                                int hs_dx, int hs_delta, const void *q, const void *k, const void *v, void *o,
-                               float *lse, const float *state_in, float *state_out, float *seg_delta,
-                               float *seg_decay, float *win, cudaStream_t st) {
-    const DcPlan pl = decay_chunk_plan(d);
-    DcArgs a;
-    a.L = d.L; a.G = pl.G; a.cps = pl.cps; a.H = d.H; a.mode = 1;
-    a.pos0 = pos0; a.scale = d.scale; a.dmax = dmax;
+                               float *lse, const float *state_in, float *state_out, void *ws, cudaStream_t st) {
+    const DbWs w = db_ws(d, false);
+    char *base = static_cast<char *>(ws);
+    DbArgs a = {};
+    a.L = d.L; a.H = d.H; a.BH = d.B * d.H; a.ipc = 1; a.pos0 = pos0; a.scale = d.scale; a.dmax = dmax;
     a.Dx = Dx; a.delta = delta; a.hs_dx = hs_dx; a.hs_delta = hs_delta;
-    a.state_in = state_in; a.state_out = state_out;
-    a.seg_delta = seg_delta; a.seg_decay = seg_decay; a.win = win;
-    a.lse = lse;
+    a.lse_out = lse;
+    a.state_in = state_in;
+    a.state_out = state_out;
+    a.ntab = (hs_dx != 0 || hs_delta != 0) ? d.H : 1;
+    if (a.ntab > 1 && !d.periods) return cudaErrorInvalidValue;   // the tables are sized per head only then
+    a.states = reinterpret_cast<__nv_bfloat16 *>(base + w.states);
+    a.etab = reinterpret_cast<uint8_t *>(base + w.etab);
+    a.ctab = reinterpret_cast<uint8_t *>(base + w.ctab);
     a.err = device_error_word();
-    if (d.dk == 64) return d.S == 32 ? launch_dchunk_t<64, 32>(d, a, pl, q, k, v, o, st)
-                                     : launch_dchunk_t<64, 64>(d, a, pl, q, k, v, o, st);
-    return d.S == 32 ? launch_dchunk_t<128, 32>(d, a, pl, q, k, v, o, st)
-                     : launch_dchunk_t<128, 64>(d, a, pl, q, k, v, o, st);
+    if (d.dk == 64) return d.S == 32 ? launch_dfwd_t<64, 32>(d, a, q, k, v, o, st)
+                                     : launch_dfwd_t<64, 64>(d, a, q, k, v, o, st);
+    return d.S == 32 ? launch_dfwd_t<128, 32>(d, a, q, k, v, o, st) : launch_dfwd_t<128, 64>(d, a, q, k, v, o, st);
 }
 
 }  // namespace bla

@@ -1,6 +1,6 @@
 // mma_sync.cuh -- warp-level bf16 tensor-core MMAs (m16n8k16, fp32 accumulation) on operand tiles
 // kept in shared memory in the 128-byte-swizzled layout, for the chunked kernels of the decayed
-// form (decay_chunk.cu, decay_chunk_bwd.cu).
+// form (decay_chunk.cu).
 #pragma once
 
 #include "tc.cuh"
