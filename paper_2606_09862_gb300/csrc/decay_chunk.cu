@@ -23,13 +23,13 @@
 // sequence; everything else runs one chunk at a time, in parallel over all SMs:
 //   1. k_dbtab: per (head, chunk), Wend and A_end for the thin passes and the chains' tables
 //      (they depend on the period and the positions only, not on the batch);
-//   2. k_dbscan<false>: per (head, K~ or V~, 64-column strip), K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c
+//   2. k_dstate: per (head, K~ or V~, 64-column strip), K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c
 //      from the entering state: the state entering every chunk, stored in bf16, and the final state;
 //   3. forward, k_dfchain: one work item per (head, chunk), each CTA a run of consecutive chunks: s, the
 //      softmax and lse, G, then o;
 //      backward, k_dbchain: likewise s, p, dp, g, G, G^, then dQ (final), the chunk's own parts G^T Q
 //      and G^T dO of dK and dV, and its adjoint contributions Z_K = (g o A)^T Q, Z_V = (p o A)^T dO;
-//   4. backward, k_dbscan<true>: per (head, strip), from the last chunk back: dK += Wend^T mu_K (dV
+//   4. backward, k_dadj: per (head, strip), from the last chunk back: dK += Wend^T mu_K (dV
 //      likewise), then mu <- A_end o mu + Z.
 // In the chains the triangle sums (s, dp, G, G^) are split at 16-token sub-blocks: the off-diagonal
 // block is a contraction on the tensor cores (W = alpha_j(tau) beta_j(u) across adjacent
@@ -1075,39 +1075,33 @@ __global__ void __launch_bounds__(S) k_dbtab(DbArgs a) {
     reinterpret_cast<float *>(a.etab + ti * EndTab<S>::bytes + EndTab<S>::aend)[j] = r;
 }
 
-// ---- the two thin passes along the sequence.  One CTA per (64-column strip, K~ or V~, head) with
-// 4 warps; the strip [S][64] (fp32) lives in the accumulator registers of the MMAs that update it.
-constexpr int kSW = 4;           // warps
+// ---- the thin passes along the sequence.  One CTA per (64-column strip, K~ or V~, head): compute
+// warps that never wait for one another, and a producer warp that keeps kNS stages of loads in
+// flight (a stage is released when every compute warp has arrived on its empty barrier).
 constexpr int kNS = 4;           // pipeline stages
 
 template <int S>
-struct StripMap {
-    static constexpr int WR = S / 16, WC = kSW / WR, NC = 64 / WC, NB = NC / 16;
-    static_assert(WR * WC == kSW && NB >= 1, "strip blocks per warp");
-};
-
-template <int S>
-struct ScanLayout {
+struct ThinLayout {
     static constexpr int kT = kBC * 128;                    // [32][64] bf16 tile
-    static constexpr int kW = S * 128;                      // [S][64] bf16 tile (Wend image, state strip)
-    // a stage: z (reverse only) | k or dk | the EndTab record, rounded up to whole 1024-byte blocks
+    static constexpr int kW = S * 128;                      // [S][64] bf16 tile
+    // a stage: Z (adjoint pass only) | k, v, dK or dV | the EndTab record, in whole 1024-byte blocks
     static constexpr int stage = ((kW + kT + EndTab<S>::bytes) + 1023) / 1024 * 1024;
-    static constexpr int mu = kNS * stage;                  // bf16 [S][64]: mu (reverse)
-    static constexpr int out = mu + kW;                     // 2 staging tiles: [S][64] (state) or [32][64]
-    static constexpr int bars = out + 2 * kW;
-    static constexpr int total = bars + 8 * kNS;
+    static constexpr int mu = kNS * stage;                  // bf16 [S][64]: mu (adjoint pass)
+    static constexpr int out = mu + kW;                     // per compute warp two 2 KB staging tiles
+    static constexpr int bars = out + 4 * 2 * 2048;         // full[kNS], empty[kNS]
+    static constexpr int total = bars + 16 * kNS;
     static_assert(stage % 1024 == 0 && mu % 1024 == 0 && out % 1024 == 0, "swizzled tiles need 1024-byte alignment");
 };
 
-// REV = false: K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c from the zero state; the state entering chunk c
-// goes to `states` (bf16).  REV = true: from the last chunk back, dK_c += Wend(c)^T mu_c (bf16 MMA on a
-// copy of mu), then mu_{c-1} = A_end(c) o mu_c + Z_c.
-template <int D, int S, bool REV>
-__global__ void __launch_bounds__(kSW * 32)
-    k_dbscan(const __grid_constant__ CUtensorMap tm_x0, const __grid_constant__ CUtensorMap tm_x1,
-             const __grid_constant__ CUtensorMap tm_st, DbArgs a) {
-    using Lay = ScanLayout<S>;
-    using M = StripMap<S>;
+// K~_{c+1} = A_end(c) o K~_c + Wend(c) K_c from the entering state (or zero): the state entering every
+// chunk goes to `states` (bf16), the final one to state_out.  Compute warp w owns rows 16 w .. 16 w + 15
+// of the strip (S / 16 warps); each stores its rows of every chunk's state by its own TMA store.
+template <int D, int S>
+__global__ void __launch_bounds__((S / 16 + 1) * 32)
+    k_dstate(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
+             const __grid_constant__ CUtensorMap tm_st16, DbArgs a) {
+    using Lay = ThinLayout<S>;
+    constexpr int NW = S / 16;
     extern __shared__ __align__(1024) uint8_t dsm[];
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g8 = lane >> 2, t4 = lane & 3;
     if (tc::smem_u32(dsm) & 1023u) {
@@ -1117,172 +1111,262 @@ __global__ void __launch_bounds__(kSW * 32)
     const int strip = blockIdx.x, kv = blockIdx.y, bh = blockIdx.z;
     const int tab = a.ntab > 1 ? bh % a.H : 0;
     const int nch = (a.L + kBC - 1) / kBC, x = strip * 64;
-    const CUtensorMap *tx = kv ? &tm_x1 : &tm_x0;   // k / v (forward) or dk / dv (reverse)
-    uint64_t *full = reinterpret_cast<uint64_t *>(dsm + Lay::bars);
-    uint8_t *sMu = dsm + Lay::mu, *sOut = dsm + Lay::out;
-    // stage s: Z strip (reverse) at +0, the [32][64] tile at +kW, the EndTab record at +kW + kT
-    auto sz = [&](int s) { return dsm + s * Lay::stage; };
+    uint64_t *full = reinterpret_cast<uint64_t *>(dsm + Lay::bars), *empty = full + kNS;
     auto sx = [&](int s) { return dsm + s * Lay::stage + Lay::kW; };
     auto sw = [&](int s) { return dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::wend; };
     auto sa = [&](int s) {
-        return reinterpret_cast<float *>(dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::aend);
-    };
-    auto chunk_of = [&](int i) { return REV ? nch - 1 - i : i; };
-    auto issue = [&](int i) {
-        const int s = i % kNS, c = chunk_of(i);
-        const size_t ti = (size_t)tab * nch + c;
-        const uint32_t bytes = (uint32_t)(Lay::kT + EndTab<S>::bytes + (REV ? Lay::kW : 0));
-        tc::mbar_arrive_expect_tx(&full[s], bytes);
-        if (REV) tc::tma_load_2d(sz(s), &tm_st, &full[s], x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
-        tc::tma_load_3d(sx(s), tx, &full[s], x, c * kBC, bh);
-        tc::bulk_load(sw(s), a.etab + ti * EndTab<S>::bytes, (uint32_t)EndTab<S>::bytes, &full[s]);
+        return reinterpret_cast<const float *>(dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::aend);
     };
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kNS; ++s) tc::mbar_init(&full[s], 1);
+        for (int s = 0; s < kNS; ++s) {
+            tc::mbar_init(&full[s], 1);
+            tc::mbar_init(&empty[s], NW);
+        }
         tc::fence_barrier_init();
     }
     __syncthreads();
-    if (threadIdx.x == 32)
-        for (int i = 0; i < kNS && i < nch; ++i) issue(i);
-
-    const int r0 = (warp % M::WR) * 16, c0 = (warp / M::WR) * M::NC;
-    float acc[M::NB][2][4];
-    // the strip's rows of an fp32 [BH][2][S][D] state: acc element (b, h, q) is row r0 + g8 + 8 (q >> 1),
-    // column x + c0 + 16 b + 8 h + 2 t4 + (q & 1)
-    auto strip_row = [&](int rh) { return ((size_t)(bh * 2 + kv) * S + r0 + g8 + 8 * rh) * D + x + c0 + 2 * t4; };
+    if (warp == NW) {
+        // producer: chunk i into stage i % kNS once the compute warps have released it
+        if (lane == 0) {
+            const CUtensorMap *tx = kv ? &tm_v : &tm_k;
+            for (int i = 0; i < nch; ++i) {
+                const int s = i % kNS;
+                if (i >= kNS && !tc::mbar_wait(&empty[s], (uint32_t)((i / kNS - 1) & 1))) {
+                    report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (18 << 4));
+                    break;
+                }
+                tc::mbar_arrive_expect_tx(&full[s], (uint32_t)(Lay::kT + EndTab<S>::bytes));
+                tc::tma_load_3d(sx(s), tx, &full[s], x, i * kBC, bh);
+                tc::bulk_load(sw(s), a.etab + ((size_t)tab * nch + i) * EndTab<S>::bytes, (uint32_t)EndTab<S>::bytes,
+                              &full[s]);
+            }
+        }
+        return;
+    }
+    const int r0 = warp * 16;
+    float acc[4][2][4];
+    // the warp's rows of an fp32 [BH][2][S][D] state: acc element (b, h, q) is row r0 + g8 + 8 (q >> 1),
+    // column x + 16 b + 8 h + 2 t4 + (q & 1)
+    auto state_at = [&](int rh) { return ((size_t)(bh * 2 + kv) * S + r0 + g8 + 8 * rh) * D + x + 2 * t4; };
 #pragma unroll
-    for (int i = 0; i < M::NB; ++i)
+    for (int b = 0; b < 4; ++b)
 #pragma unroll
         for (int h = 0; h < 2; ++h)
 #pragma unroll
             for (int rh = 0; rh < 2; ++rh) {
                 float2 v0 = make_float2(0.f, 0.f);
-                if (!REV && a.state_in)
-                    v0 = *reinterpret_cast<const float2 *>(a.state_in + strip_row(rh) + i * 16 + h * 8);
-                acc[i][h][2 * rh] = v0.x;
-                acc[i][h][2 * rh + 1] = v0.y;
+                if (a.state_in) v0 = *reinterpret_cast<const float2 *>(a.state_in + state_at(rh) + b * 16 + h * 8);
+                acc[b][h][2 * rh] = v0.x;
+                acc[b][h][2 * rh + 1] = v0.y;
             }
-    auto put = [&](uint8_t *tile) {   // acc (bf16) into a swizzled [S][64] tile
-#pragma unroll
-        for (int i = 0; i < M::NB; ++i)
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                const int e = c0 + i * 16 + h * 8 + 2 * t4;
-                st_bf16x2(tile, S, r0 + g8, e, acc[i][h][0], acc[i][h][1]);
-                st_bf16x2(tile, S, r0 + g8 + 8, e, acc[i][h][2], acc[i][h][3]);
-            }
-    };
+    uint8_t *stg = dsm + Lay::out + warp * 2 * 2048;
     bool ok = true;
     for (int i = 0; i < nch; ++i) {
-        const int s = i % kNS, c = chunk_of(i), ob = i & 1;
-        if (threadIdx.x == 0) tc::bulk_wait_read1();   // the store that used staging tile ob has read it
-        if (!REV) {
-            __syncthreads();
-            put(sOut + ob * Lay::kW);   // the state entering chunk c
+        const int s = i % kNS, ob = i & 1;
+        // the state entering chunk i: the warp's 16 rows, by its own store
+        if (lane == 0) tc::bulk_wait_read1();   // the store from staging tile ob two chunks ago has read it
+        __syncwarp();
+        uint8_t *tile = stg + ob * 2048;
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int col = b * 16 + h * 8 + 2 * t4;
+                st_bf16x2(tile, 16, g8, col, acc[b][h][0], acc[b][h][1]);
+                st_bf16x2(tile, 16, g8 + 8, col, acc[b][h][2], acc[b][h][3]);
+            }
+        tc::fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) {
+            tc::tma_store_2d(&tm_st16, tile, x, (int)((((size_t)bh * nch + i) * 2 + kv) * S + r0));
+            tc::bulk_commit();
         }
         if (!tc::mbar_wait(&full[s], (uint32_t)((i / kNS) & 1))) {
             report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (18 << 4));
             ok = false;
+            break;
         }
-        if (__syncthreads_or(!ok)) break;
+        // acc <- A_end o acc + Wend K_i: A = the Wend rows r0.. (tokens as K), B = the chunk's strip
         const float *ae = sa(s);
         const float f0 = ae[r0 + g8], f1 = ae[r0 + g8 + 8];
+#pragma unroll
+        for (int b = 0; b < 4; ++b)
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                acc[b][h][0] *= f0; acc[b][h][1] *= f0;
+                acc[b][h][2] *= f1; acc[b][h][3] *= f1;
+            }
         const uint32_t uW = tc::smem_u32(sw(s)), uX = tc::smem_u32(sx(s));
-        if (!REV) {
-            // acc <- A_end o acc + Wend K_c: A = Wend [S][32 tokens], B = the chunk's strip [32][64]
 #pragma unroll
-            for (int b = 0; b < M::NB; ++b)
+        for (int k0 = 0; k0 < kBC; k0 += 16) {
+            uint32_t af[4], bf[4];
+            load_a(uW, S, r0, k0, af);
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    acc[b][h][0] *= f0; acc[b][h][1] *= f0;
-                    acc[b][h][2] *= f1; acc[b][h][3] *= f1;
-                }
-#pragma unroll
-            for (int k0 = 0; k0 < kBC; k0 += 16) {
-                uint32_t af[4], bf[4];
-                load_a(uW, S, r0, k0, af);
-#pragma unroll
-                for (int b = 0; b < M::NB; ++b) {
-                    load_b_kn(uX, kBC, c0 + b * 16, k0, bf);
-                    mma16816(acc[b][0], af, bf[0], bf[1]);
-                    mma16816(acc[b][1], af, bf[2], bf[3]);
-                }
-            }
-        } else {
-            // dK_c [32][64] += Wend^T mu: warp takes token rows om0.. and 32 columns on0..
-            const bool live = i > 0;   // mu is zero after the last chunk
-            if (live) {
-                put(sMu);
-                __syncthreads();
-                const int om0 = (warp & 1) * 16, on0 = (warp >> 1) * 32;
-                float o[2][2][4] = {};
-                const uint32_t uMu = tc::smem_u32(sMu);
-#pragma unroll
-                for (int k0 = 0; k0 < S; k0 += 16) {
-                    uint32_t af[4], bf[4];
-                    load_a_t(uW, S, om0, k0, af);
-#pragma unroll
-                    for (int b = 0; b < 2; ++b) {
-                        load_b_kn(uMu, S, on0 + b * 16, k0, bf);
-                        mma16816(o[b][0], af, bf[0], bf[1]);
-                        mma16816(o[b][1], af, bf[2], bf[3]);
-                    }
-                }
-                const uint8_t *dk = sx(s);
-                uint8_t *dst = sOut + ob * Lay::kW;
-#pragma unroll
-                for (int b = 0; b < 2; ++b)
-#pragma unroll
-                    for (int h = 0; h < 2; ++h)
-#pragma unroll
-                        for (int rh = 0; rh < 2; ++rh) {
-                            const int row = om0 + g8 + rh * 8, col = on0 + b * 16 + h * 8 + 2 * t4;
-                            const float2 l = __bfloat1622float2(
-                                *reinterpret_cast<const __nv_bfloat162 *>(dk + sw_off(kBC, row, col)));
-                            st_bf16x2(dst, kBC, row, col, o[b][h][2 * rh] + l.x, o[b][h][2 * rh + 1] + l.y);
-                        }
-            }
-            // mu <- A_end o mu + Z_c
-            const uint8_t *z = sz(s);
-#pragma unroll
-            for (int b = 0; b < M::NB; ++b)
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-#pragma unroll
-                    for (int rh = 0; rh < 2; ++rh) {
-                        const int row = r0 + g8 + rh * 8, col = c0 + b * 16 + h * 8 + 2 * t4;
-                        const float f = rh ? f1 : f0;
-                        const float2 zz =
-                            __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(z + sw_off(S, row, col)));
-                        acc[b][h][2 * rh] = fmaf(f, acc[b][h][2 * rh], zz.x);
-                        acc[b][h][2 * rh + 1] = fmaf(f, acc[b][h][2 * rh + 1], zz.y);
-                    }
-        }
-        tc::fence_proxy_async_smem();
-        __syncthreads();   // stage s and the staging tile are complete
-        if (threadIdx.x == 0) {
-            if (!REV) {
-                tc::tma_store_2d(&tm_st, sOut + ob * Lay::kW, x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
-                tc::bulk_commit();
-            } else if (i > 0) {
-                tc::tma_store_3d(tx, sOut + ob * Lay::kW, x, c * kBC, bh);
-                tc::bulk_commit();
+            for (int b = 0; b < 4; ++b) {
+                load_b_kn(uX, kBC, b * 16, k0, bf);
+                mma16816(acc[b][0], af, bf[0], bf[1]);
+                mma16816(acc[b][1], af, bf[2], bf[3]);
             }
         }
-        // the loads come from another warp: each TMA issue holds its thread for a while
-        if (threadIdx.x == 32 && i + kNS < nch) issue(i + kNS);
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&empty[s]);
     }
-    if (!REV && ok && a.state_out) {
+    if (ok && a.state_out) {
 #pragma unroll
-        for (int i = 0; i < M::NB; ++i)
+        for (int b = 0; b < 4; ++b)
 #pragma unroll
             for (int h = 0; h < 2; ++h)
 #pragma unroll
                 for (int rh = 0; rh < 2; ++rh)
-                    *reinterpret_cast<float2 *>(a.state_out + strip_row(rh) + i * 16 + h * 8) =
-                        make_float2(acc[i][h][2 * rh], acc[i][h][2 * rh + 1]);
+                    *reinterpret_cast<float2 *>(a.state_out + state_at(rh) + b * 16 + h * 8) =
+                        make_float2(acc[b][h][2 * rh], acc[b][h][2 * rh + 1]);
     }
-    if (threadIdx.x == 0) tc::bulk_wait0();
+    if (lane == 0) tc::bulk_wait0();
+}
+
+// From the last chunk back: dK_c += Wend(c)^T mu_c (a bf16 copy of mu as the MMA operand), then
+// mu_{c-1} = A_end(c) o mu_c + Z_c.  Compute warp w (4 of them) owns columns 16 w .. 16 w + 15 of the
+// strip for all S rows of mu, so the contraction over the slots needs no other warp's data; each
+// stores its [32][16] block of dK by its own TMA store (unswizzled box).
+template <int D, int S>
+__global__ void __launch_bounds__(5 * 32)
+    k_dadj(const __grid_constant__ CUtensorMap tm_dk, const __grid_constant__ CUtensorMap tm_dv,
+           const __grid_constant__ CUtensorMap tm_dk16, const __grid_constant__ CUtensorMap tm_dv16,
+           const __grid_constant__ CUtensorMap tm_z, DbArgs a) {
+    using Lay = ThinLayout<S>;
+    constexpr int NW = 4, SB = S / 16;
+    extern __shared__ __align__(1024) uint8_t dsm[];
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, g8 = lane >> 2, t4 = lane & 3;
+    if (tc::smem_u32(dsm) & 1023u) {
+        if (threadIdx.x == 0) report_device_error(a.err, DEVERR_SMEM_ALIGN | (18 << 4) | ((int)blockIdx.x << 16));
+        return;
+    }
+    const int strip = blockIdx.x, kv = blockIdx.y, bh = blockIdx.z;
+    const int tab = a.ntab > 1 ? bh % a.H : 0;
+    const int nch = (a.L + kBC - 1) / kBC, x = strip * 64;
+    uint64_t *full = reinterpret_cast<uint64_t *>(dsm + Lay::bars), *empty = full + kNS;
+    auto sz = [&](int s) { return dsm + s * Lay::stage; };
+    auto sx = [&](int s) { return dsm + s * Lay::stage + Lay::kW; };
+    auto sw = [&](int s) { return dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::wend; };
+    auto sa = [&](int s) {
+        return reinterpret_cast<const float *>(dsm + s * Lay::stage + Lay::kW + Lay::kT + EndTab<S>::aend);
+    };
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kNS; ++s) {
+            tc::mbar_init(&full[s], 1);
+            tc::mbar_init(&empty[s], NW);
+        }
+        tc::fence_barrier_init();
+    }
+    __syncthreads();
+    if (warp == NW) {
+        // producer: step i (chunk nch - 1 - i) into stage i % kNS: Z, the chain's dK (or dV) part, EndTab
+        if (lane == 0) {
+            const CUtensorMap *tx = kv ? &tm_dv : &tm_dk;
+            for (int i = 0; i < nch; ++i) {
+                const int s = i % kNS, c = nch - 1 - i;
+                if (i >= kNS && !tc::mbar_wait(&empty[s], (uint32_t)((i / kNS - 1) & 1))) {
+                    report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (18 << 4));
+                    break;
+                }
+                tc::mbar_arrive_expect_tx(&full[s], (uint32_t)(Lay::kW + Lay::kT + EndTab<S>::bytes));
+                tc::tma_load_2d(sz(s), &tm_z, &full[s], x, (int)((((size_t)bh * nch + c) * 2 + kv) * S));
+                tc::tma_load_3d(sx(s), tx, &full[s], x, c * kBC, bh);
+                tc::bulk_load(sw(s), a.etab + ((size_t)tab * nch + c) * EndTab<S>::bytes, (uint32_t)EndTab<S>::bytes,
+                              &full[s]);
+            }
+        }
+        return;
+    }
+    const int n0 = warp * 16;
+    const CUtensorMap *tout = kv ? &tm_dv16 : &tm_dk16;
+    float mu[SB][2][4];
+#pragma unroll
+    for (int rb = 0; rb < SB; ++rb)
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) mu[rb][h][q] = 0.f;
+    uint8_t *sMu = dsm + Lay::mu;
+    const uint32_t uMu = tc::smem_u32(sMu);
+    __nv_bfloat16 *stg = reinterpret_cast<__nv_bfloat16 *>(dsm + Lay::out + warp * 2 * 2048);
+    for (int i = 0; i < nch; ++i) {
+        const int s = i % kNS, c = nch - 1 - i, ob = i & 1;
+        if (!tc::mbar_wait(&full[s], (uint32_t)((i / kNS) & 1))) {
+            report_device_error(a.err, DEVERR_MBAR_TIMEOUT | (18 << 4));
+            break;
+        }
+        if (i > 0) {   // mu is zero after the last chunk
+            // the warp's columns of mu in bf16, as the B operand
+#pragma unroll
+            for (int rb = 0; rb < SB; ++rb)
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int col = n0 + h * 8 + 2 * t4;
+                    st_bf16x2(sMu, S, rb * 16 + g8, col, mu[rb][h][0], mu[rb][h][1]);
+                    st_bf16x2(sMu, S, rb * 16 + g8 + 8, col, mu[rb][h][2], mu[rb][h][3]);
+                }
+            __syncwarp();
+            float o[2][2][4] = {};
+            const uint32_t uW = tc::smem_u32(sw(s));
+#pragma unroll
+            for (int k0 = 0; k0 < S; k0 += 16) {
+                uint32_t bf[4];
+                load_b_kn(uMu, S, n0, k0, bf);
+#pragma unroll
+                for (int tb = 0; tb < 2; ++tb) {
+                    uint32_t af[4];
+                    load_a_t(uW, S, tb * 16, k0, af);
+                    mma16816(o[tb][0], af, bf[0], bf[1]);
+                    mma16816(o[tb][1], af, bf[2], bf[3]);
+                }
+            }
+            // + the chain's part, into the warp's dense [32][16] staging tile
+            if (lane == 0) tc::bulk_wait_read1();
+            __syncwarp();
+            __nv_bfloat16 *tile = stg + ob * (kBC * 16);
+            const uint8_t *dk = sx(s);
+#pragma unroll
+            for (int tb = 0; tb < 2; ++tb)
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+#pragma unroll
+                    for (int rh = 0; rh < 2; ++rh) {
+                        const int row = tb * 16 + g8 + rh * 8, cl = h * 8 + 2 * t4;
+                        const float2 l = __bfloat1622float2(
+                            *reinterpret_cast<const __nv_bfloat162 *>(dk + sw_off(kBC, row, n0 + cl)));
+                        *reinterpret_cast<uint32_t *>(tile + row * 16 + cl) =
+                            tc::pack_bf16x2(o[tb][h][2 * rh] + l.x, o[tb][h][2 * rh + 1] + l.y);
+                    }
+            tc::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                tc::tma_store_3d(tout, tile, x + n0, c * kBC, bh);
+                tc::bulk_commit();
+            }
+        }
+        // mu <- A_end o mu + Z_c
+        const float *ae = sa(s);
+        const uint8_t *z = sz(s);
+#pragma unroll
+        for (int rb = 0; rb < SB; ++rb) {
+            const float f0 = ae[rb * 16 + g8], f1 = ae[rb * 16 + g8 + 8];
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int rh = 0; rh < 2; ++rh) {
+                    const int row = rb * 16 + g8 + rh * 8, col = n0 + h * 8 + 2 * t4;
+                    const float2 zz =
+                        __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(z + sw_off(S, row, col)));
+                    const float f = rh ? f1 : f0;
+                    mu[rb][h][2 * rh] = fmaf(f, mu[rb][h][2 * rh], zz.x);
+                    mu[rb][h][2 * rh + 1] = fmaf(f, mu[rb][h][2 * rh + 1], zz.y);
+                }
+        }
+        __syncwarp();
+        if (lane == 0) tc::mbar_arrive(&empty[s]);
+    }
+    if (lane == 0) tc::bulk_wait0();
 }
 
 int sm_count_db() {
@@ -1295,17 +1379,22 @@ int sm_count_db() {
 template <int D, int S>
 cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v,
                           const void *dout, void *dq, void *dk, void *dv, cudaStream_t st) {
-    CUtensorMap tk, tv, tst, tz, tdk, tdv;
+    // the thin passes: [32][64] strips of k, v and of the chain's dK, dV parts, [16][64] blocks of the
+    // states (one per warp), [S][64] strips of Z, and the [32][16] blocks of dK and dV each warp stores
+    CUtensorMap tk, tv, tst16, tz, tdk, tdv, tdk16, tdv16;
     const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
     const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
-    const uint32_t box[3] = {64, (uint32_t)kBC, 1};
+    const uint32_t box[3] = {64, (uint32_t)kBC, 1}, box16[3] = {16, (uint32_t)kBC, 1};
     const int nch = (d.L + kBC - 1) / kBC;
     const uint64_t sdims[2] = {(uint64_t)D, (uint64_t)d.B * d.H * nch * 2 * S};
     const uint64_t sstr[1] = {(uint64_t)D * 2};
-    const uint32_t sbox[2] = {64, (uint32_t)S};
+    const uint32_t sbox[2] = {64, (uint32_t)S}, sbox16[2] = {64, 16};
     if (!make_tmap_bf16(&tk, k, 3, dims, strides, box) || !make_tmap_bf16(&tv, v, 3, dims, strides, box) ||
-        !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) || !make_tmap_bf16(&tz, a.zbuf, 2, sdims, sstr, sbox) ||
-        !make_tmap_bf16(&tdk, dk, 3, dims, strides, box) || !make_tmap_bf16(&tdv, dv, 3, dims, strides, box))
+        !make_tmap_bf16(&tst16, a.states, 2, sdims, sstr, sbox16) ||
+        !make_tmap_bf16(&tz, a.zbuf, 2, sdims, sstr, sbox) || !make_tmap_bf16(&tdk, dk, 3, dims, strides, box) ||
+        !make_tmap_bf16(&tdv, dv, 3, dims, strides, box) ||
+        !make_tmap_bf16(&tdk16, dk, 3, dims, strides, box16, false) ||
+        !make_tmap_bf16(&tdv16, dv, 3, dims, strides, box16, false))
         return cudaErrorInvalidValue;
     // the chain moves whole [32][D] and [S][D] tiles in one copy each: the 64-column blocks are a
     // further dimension of the maps (128 bytes apart), so a box lands as [D / 64][rows][64]
@@ -1322,24 +1411,22 @@ cudaError_t launch_dbwd_t(const OpDims &d, const DbArgs &a, const void *q, const
         !make_tmap_bf16(&cz, a.zbuf, 3, csdims, csstr, csbox) || !make_tmap_bf16(&cdq, dq, 4, cdims, cstr, cbox) ||
         !make_tmap_bf16(&cdk, dk, 4, cdims, cstr, cbox) || !make_tmap_bf16(&cdv, dv, 4, cdims, cstr, cbox))
         return cudaErrorInvalidValue;
-    const int smem = BwLayout<D, S>::total, ssm = ScanLayout<S>::total;
+    const int smem = BwLayout<D, S>::total, ssm = ThinLayout<S>::total;
     cudaError_t e = cudaFuncSetAttribute(k_dbchain<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_dbscan<D, S, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_dbscan<D, S, true>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_dstate<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_dadj<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_DECAY, st);
     k_dbtab<S><<<dim3((unsigned)nch, (unsigned)a.ntab), S, 0, st>>>(a);
     const dim3 sgrid((unsigned)(D / 64), 2u, (unsigned)a.BH);
-    k_dbscan<D, S, false><<<sgrid, kSW * 32, ssm, st>>>(tk, tv, tst, a);
+    k_dstate<D, S><<<sgrid, (S / 16 + 1) * 32, ssm, st>>>(tk, tv, tst16, a);
     const long long items = (long long)a.BH * nch;
     if (items > 0x7fffffffLL) return cudaErrorInvalidValue;   // the chain indexes its items in 32 bits
     DbArgs ac = a;
     ac.ipc = (int)((items + sm_count_db() - 1) / sm_count_db());
     const int grid = (int)((items + ac.ipc - 1) / ac.ipc);
     k_dbchain<D, S><<<(unsigned)grid, kBT, smem, st>>>(cq, ck, cv, cdo, cst, cz, cdq, cdk, cdv, ac);
-    k_dbscan<D, S, true><<<sgrid, kSW * 32, ssm, st>>>(tdk, tdv, tz, a);
+    k_dadj<D, S><<<sgrid, 5 * 32, ssm, st>>>(tdk, tdv, tdk16, tdv16, tz, a);
     return cudaGetLastError();
 }
 
@@ -1365,14 +1452,14 @@ DbWs db_ws(const OpDims &d, bool with_z) {
 template <int D, int S>
 cudaError_t launch_dfwd_t(const OpDims &d, const DbArgs &a, const void *q, const void *k, const void *v, void *o,
                           cudaStream_t st) {
-    CUtensorMap tk, tv, tst, cq, ck, cv, cst, co;
+    CUtensorMap tk, tv, tst16, cq, ck, cv, cst, co;
     const int nch = (d.L + kBC - 1) / kBC;
     const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d.L, (uint64_t)d.B * d.H};
     const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d.L * D * 2};
     const uint32_t box[3] = {64, (uint32_t)kBC, 1};
     const uint64_t sdims[2] = {(uint64_t)D, (uint64_t)d.B * d.H * nch * 2 * S};
     const uint64_t sstr[1] = {(uint64_t)D * 2};
-    const uint32_t sbox[2] = {64, (uint32_t)S};
+    const uint32_t sbox16[2] = {64, 16};
     const uint64_t cdims[4] = {64, (uint64_t)d.L, (uint64_t)(D / 64), (uint64_t)d.B * d.H};
     const uint64_t cstr[3] = {(uint64_t)D * 2, 128, (uint64_t)d.L * D * 2};
     const uint32_t cbox[4] = {64, (uint32_t)kBC, (uint32_t)(D / 64), 1};
@@ -1380,20 +1467,19 @@ cudaError_t launch_dfwd_t(const OpDims &d, const DbArgs &a, const void *q, const
     const uint64_t csstr[2] = {(uint64_t)D * 2, 128};
     const uint32_t csbox[3] = {64, (uint32_t)S, (uint32_t)(D / 64)};
     if (!make_tmap_bf16(&tk, k, 3, dims, strides, box) || !make_tmap_bf16(&tv, v, 3, dims, strides, box) ||
-        !make_tmap_bf16(&tst, a.states, 2, sdims, sstr, sbox) || !make_tmap_bf16(&cq, q, 4, cdims, cstr, cbox) ||
+        !make_tmap_bf16(&tst16, a.states, 2, sdims, sstr, sbox16) || !make_tmap_bf16(&cq, q, 4, cdims, cstr, cbox) ||
         !make_tmap_bf16(&ck, k, 4, cdims, cstr, cbox) || !make_tmap_bf16(&cv, v, 4, cdims, cstr, cbox) ||
         !make_tmap_bf16(&cst, a.states, 3, csdims, csstr, csbox) || !make_tmap_bf16(&co, o, 4, cdims, cstr, cbox))
         return cudaErrorInvalidValue;
-    const int smem = FwLayout<D, S>::total, ssm = ScanLayout<S>::total;
+    const int smem = FwLayout<D, S>::total, ssm = ThinLayout<S>::total;
     cudaError_t e = cudaFuncSetAttribute(k_dfchain<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_dbscan<D, S, false>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(k_dstate<D, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, ssm);
     if (e != cudaSuccess) return e;
     const long long items = (long long)a.BH * nch;
     if (items > 0x7fffffffLL) return cudaErrorInvalidValue;   // the chain indexes its items in 32 bits
     ProfScope ps(BLA_K_DECAY, st);
     k_dbtab<S><<<dim3((unsigned)nch, (unsigned)a.ntab), S, 0, st>>>(a);
-    k_dbscan<D, S, false><<<dim3((unsigned)(D / 64), 2u, (unsigned)a.BH), kSW * 32, ssm, st>>>(tk, tv, tst, a);
+    k_dstate<D, S><<<dim3((unsigned)(D / 64), 2u, (unsigned)a.BH), (S / 16 + 1) * 32, ssm, st>>>(tk, tv, tst16, a);
     DbArgs ac = a;
     const long long slots = 2LL * sm_count_db();   // two chain CTAs per SM
     ac.ipc = (int)((items + slots - 1) / slots);
