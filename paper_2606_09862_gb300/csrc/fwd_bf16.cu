@@ -625,15 +625,17 @@ __global__ void __launch_bounds__(kThreads, 1)
 __global__ void k_scan(Args a) {
     tc::pdl_wait();      // the segment deltas
     const Geo &g = a.g;
-    const long long total = (long long)g.BH * 2 * g.M * g.D;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
-         i += (long long)gridDim.x * blockDim.x) {
-        const int e = (int)(i % g.D);
-        long long r = i / g.D;
-        const int m = (int)(r % g.M);
-        r /= g.M;
-        const int x = (int)(r % 2);
-        const int bh = (int)(r / 2);
+    // 32-bit index arithmetic (the host checks that the element count fits): 64-bit divisions made
+    // this kernel instruction-bound
+    const unsigned total = (unsigned)g.BH * 2u * (unsigned)g.M * (unsigned)g.D;
+    const unsigned uD = (unsigned)g.D, uM = (unsigned)g.M;
+    for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+        const int e = (int)(i % uD);
+        unsigned r = i / uD;
+        const int m = (int)(r % uM);
+        r /= uM;
+        const int x = (int)(r & 1u);
+        const int bh = (int)(r >> 1);
         float c, s;
         const HeadW hw = head_w(a, bh);
         mode_phase((long long)m * g.Lseg, hw.w, hw.tint, &c, &s);
@@ -1745,6 +1747,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
         }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
         long long tot = (long long)g.BH * 2 * g.M * g.D;
+        if (tot > 0x7fffffffLL) return cudaErrorInvalidValue;   // k_scan indexes in 32 bits
         int blocks = (int)((tot + 255) / 256);
         if (blocks > 4096) blocks = 4096;
         {
