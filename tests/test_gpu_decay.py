@@ -59,6 +59,8 @@ def test_bf16_forward(orc, B, H, L, d, M, S, T):
     (16, 10, 130, 64, 32, 32, 256.0),   # 160 heads: one segment per head
     (1, 1, 1000, 128, 64, 64, 1024.0),  # 16 one-chunk segments
     (2, 1, 63, 128, 32, 64, 512.0),     # one ragged chunk
+    (1, 1, 1, 64, 8, 32, 64.0),         # a single token: one item, one state update
+    (1, 2, 33, 128, 16, 64, 100.0),     # one chunk and one token
 ])
 def test_bf16_chunked_forward(orc, B, H, L, d, M, S, T):
     """The chunked tensor-core form (d in {64, 128}, S in {32, 64}): o per row, lse and state."""
