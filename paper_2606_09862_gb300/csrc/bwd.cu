@@ -417,18 +417,28 @@ enum FsBar { FS_EB, FS_FULL0, FS_EMPTY0 = FS_FULL0 + 4, FS_DFULL0 = FS_EMPTY0 + 
              FS_COUNT = FS_DEMPTY0 + 2 };
 constexpr int kFsStages = 3;
 
+// The chunk states W_c leave through shared memory: the eight epilogue warps write their rows into a
+// staging tile ([D/64][RP rows][64], 128-byte swizzled; two tiles when they fit) and thread 0 stores it
+// by TMA, instead of every thread storing its own row (32 rows per warp store, half-filled sectors).
+template <int NB>
+struct FsStaging {
+    static constexpr int buffers = NB == 1 ? 2 : 1;
+};
+
 template <int D, int NB>
 __global__ void __launch_bounds__(kSeqThreads, 1)
     k_fwd_states(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-                 const __grid_constant__ CUtensorMap tm_eb, SeqArgs a) {
+                 const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_w, SeqArgs a) {
     constexpr int DH = D / 2, RP = NB * 128;
+    constexpr int SBUF = FsStaging<NB>::buffers, w_bytes = RP * D * 2;
     const int x = blockIdx.x & 1, bh = blockIdx.x >> 1;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t *sEB = sm;                                   // [2][RP][64] K-major A (rows r, K = u)
     uint8_t *sX = sEB + RP * 256;                        // kFsStages x [D/64][128 u][64] MN-major B
     constexpr int x_bytes = 128 * D * 2;
-    uint64_t *bar = reinterpret_cast<uint64_t *>(sX + kFsStages * x_bytes);
+    uint8_t *sWst = sX + kFsStages * x_bytes;            // SBUF x [D/64][RP][64]: W_c staging
+    uint64_t *bar = reinterpret_cast<uint64_t *>(sWst + SBUF * w_bytes);
     uint32_t *tslot = reinterpret_cast<uint32_t *>(bar + FS_COUNT);
     Ctl *ctl = reinterpret_cast<Ctl *>(bar + FS_COUNT + 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -498,12 +508,27 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
         }
         uint32_t ph_df[2] = {0, 0};
         for (int c = 0; c < a.nch; ++c) {
-            // W_c
+            // W_c, by thread 0's TMA store of the staging tile (the one two chunks back has been read)
+            uint8_t *stile = sWst + (SBUF == 2 ? (c & 1) : 0) * w_bytes;
+            if (threadIdx.x == 0) {
+                if (SBUF == 2) tc::bulk_wait_read1();
+                else tc::bulk_wait_read0();
+            }
+            tc::named_bar(1, kSeqEpiWarps * 32);
 #pragma unroll
             for (int b = 0; b < NB; ++b) {
                 const int r = b * 128 + row;
-                if (r < a.R2)
-                    st_row_global<DH>(a.wout + ((((size_t)bh * a.nch + c) * 2 + x) * a.R2 + r) * D + wg * DH, s[b]);
+                if (r < a.R2) {
+#pragma unroll
+                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16_seq(stile, RP, r, wg * DH + g0, s[b] + g0);
+                }
+            }
+            tc::fence_proxy_async_smem();
+            tc::named_bar(1, kSeqEpiWarps * 32);
+            if (threadIdx.x == 0) {
+                for (int db = 0; db < D / 64; ++db)
+                    tc::tma_store_3d(&tm_w, stile + db * RP * 128, db * 64, 0, (bh * a.nch + c) * 2 + x);
+                tc::bulk_commit();
             }
             if (c == nupd) break;
             const int buf = c & 1;
@@ -522,6 +547,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 #pragma unroll
             for (int b = 0; b < NB; ++b) rot_rows<DH>(s[b], odd, cs[b], sn[b], 1.f);
         }
+        if (threadIdx.x == 0) tc::bulk_wait0();
     }
     tc::tc_fence_before();
     __syncthreads();
@@ -535,7 +561,9 @@ enum AsBar { AS_EB, AS_FULL0, AS_FREE0 = AS_FULL0 + 2, AS_CFULL0 = AS_FREE0 + 2,
              AS_LB = AS_CEMPTY0 + 2, AS_DKFULL, AS_DKEMPTY, AS_COUNT };
 
 // Shared memory of k_adj_states: EB, then `stages` x (Xa [RP/64][128 t][64], Bq [D/64][128 t][64],
-// Pa [2][128 t][64]); L_c (bf16, [D/64][R2][64]) is written over the stage's Xa once its MMA is done.
+// Pa [2][128 t][64]); L_c (bf16, [D/64][R2][64]) is written over the stage's Xa once its MMA is done,
+// and the chunk's dK or dV rows over its Pa once the gradient MMAs are done.  Thread 0 stores those
+// rows by TMA and releases the stage to the producer once the store has read them.
 __host__ __device__ inline int adj_stage_bytes(int RP, int D) { return RP * 256 + D * 256 + 2 * 128 * 128; }
 
 template <int D, int NB>
@@ -543,7 +571,8 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
     k_adj_states(const __grid_constant__ CUtensorMap tm_dx, const __grid_constant__ CUtensorMap tm_ap,
                  const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_do,
                  const __grid_constant__ CUtensorMap tm_dp, const __grid_constant__ CUtensorMap tm_g,
-                 const __grid_constant__ CUtensorMap tm_eb, SeqArgs a, int stages) {
+                 const __grid_constant__ CUtensorMap tm_eb, const __grid_constant__ CUtensorMap tm_gk,
+                 const __grid_constant__ CUtensorMap tm_gv, SeqArgs a, int stages) {
     constexpr int DH = D / 2, RP = NB * 128;
     constexpr int NCB = NB == 1 ? 2 : 1;                 // contribution buffers in TMEM
     const int x = blockIdx.x & 1, bh = blockIdx.x >> 1;
@@ -601,6 +630,14 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
                     tc::tma_load_3d(base + RP * 256 + db * 128 * 128, mb, &bar[AS_FULL0 + st], db * 64, c * kC, bh);
                 for (int ub = 0; ub < 2; ++ub)
                     tc::tma_load_3d(base + RP * 256 + D * 256 + ub * 128 * 128, mp, &bar[AS_FULL0 + st], ub * 64, 0, z);
+                // the chunk `stages` steps later into L2 now: with at most `stages` 96 KB stages in shared
+                // memory the loads alone would keep too few bytes in flight
+                if (i + stages < nch) {
+                    const int cn = c - stages, zn = bh * nch + cn;
+                    for (int rb = 0; rb < RP / 64; ++rb) tc::tma_prefetch_3d(ma, rb * 64, 0, zn);
+                    for (int db = 0; db < D / 64; ++db) tc::tma_prefetch_3d(mb, db * 64, cn * kC, bh);
+                    for (int ub = 0; ub < 2; ++ub) tc::tma_prefetch_3d(mp, ub * 64, 0, zn);
+                }
             }
         }
     } else if (warp == 9) {
@@ -631,8 +668,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
                 tc::tc_fence_after();
                 for (int k = 0; k < R2 / 16; ++k)
                     tc::mma_bf16(tb + colDK, seq_mnmaj(es, RP, 0, k), seq_mnmaj(xa, R2, 0, k), id_c, 1u);
-                tc::mma_commit(&bar[AS_DKFULL]);
-                tc::mma_commit(&bar[AS_FREE0 + st]);
+                tc::mma_commit(&bar[AS_DKFULL]);   // (the epilogue releases the stage after the dK store)
                 ok = true;
             }
         }
@@ -650,7 +686,7 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
             for (int i = 0; i < DH; ++i) s[b][i] = 0.f;
         }
         uint32_t ph_cf[2] = {0, 0}, ph_dkf = 0;
-        bf16 *gout = a.gout[x];
+        const CUtensorMap *tg = x ? &tm_gv : &tm_gk;
         for (int i = 0; i < nch; ++i) {
             const int c = nch - 1 - i, st = i % stages, cb = i % NCB;
             // L_c (bf16) over the stage's Xa once the contribution MMA has read it
@@ -685,19 +721,37 @@ __global__ void __launch_bounds__(kSeqThreads, 1)
 #pragma unroll
                 for (int b = 0; b < NB; ++b) rot_rows<DH>(s[b], odd, cs[b], sn[b], -1.f);
             }
-            // the chunk's gradient rows
+            // the chunk's gradient rows, staged over the stage's dP / G tile (its MMAs are done) and
+            // stored by thread 0 (rows past L are clipped by the tensor map)
             if (!wait_bar(&bar[AS_DKFULL], ph_dkf, ctl, a.err, 27)) break;
             tc::tc_fence_after();
+            uint8_t *gt = sStage + st * sbytes + RP * 256 + D * 256;
             {
                 float v[DH];
                 tc::tmem_ld<DH>(tb + ((uint32_t)lane_base << 16) + colDK + (uint32_t)(wg * DH), v);
-                const int t = c * kC + row;
-                if (t < a.L) st_row_global<DH>(gout + ((size_t)bh * a.L + t) * D + wg * DH, v);
+#pragma unroll
+                for (int g0 = 0; g0 < DH; g0 += 32) st_row32_bf16_seq(gt, 128, row, wg * DH + g0, v + g0);
             }
             tc::tc_fence_before();
             __syncwarp();
             if (lane == 0) tc::mbar_arrive(&bar[AS_DKEMPTY]);
+            tc::fence_proxy_async_smem();
+            tc::named_bar(1, kSeqEpiWarps * 32);
+            if (threadIdx.x == 0) {
+                for (int db = 0; db < D / 64; ++db) tc::tma_store_3d(tg, gt + db * 128 * 128, db * 64, c * kC, bh);
+                tc::bulk_commit();
+                // a stage goes back to the producer once its rows are read: with two stages the previous
+                // step's (this step's store may still be reading), with one this step's own
+                if (stages == 1) {
+                    tc::bulk_wait_read0();
+                    tc::mbar_arrive(&bar[AS_FREE0]);
+                } else if (i > 0) {
+                    tc::bulk_wait_read1();
+                    tc::mbar_arrive(&bar[AS_FREE0 + (i - 1) % stages]);
+                }
+            }
         }
+        if (threadIdx.x == 0) tc::bulk_wait0();
     }
     tc::tc_fence_before();
     __syncthreads();
@@ -1472,31 +1526,33 @@ cudaError_t gemm(const BwdGeo &g, int mtiles, int N, const CUtensorMap &a0, cons
 
 template <int D, int NB>
 cudaError_t launch_fwd_states_t(const BwdGeo &g, const CUtensorMap &mk, const CUtensorMap &mv, const CUtensorMap &meb,
-                                const SeqArgs &sa, cudaStream_t st) {
+                                const CUtensorMap &mw, const SeqArgs &sa, cudaStream_t st) {
     // (both chunk kernels allocate all 512 TMEM columns: at least 120 KB of shared memory keeps a
     //  second CTA off the SM, so an allocation never waits for another CTA to finish)
-    int smem = NB * 128 * 256 + kFsStages * 128 * D * 2 + 256 + 1024;
+    int smem = NB * 128 * 256 + kFsStages * 128 * D * 2 + FsStaging<NB>::buffers * NB * 128 * D * 2 + 256 + 1024;
+    if (smem > 227 * 1024) return cudaErrorInvalidValue;
     if (smem < 120 * 1024) smem = 120 * 1024;
     cudaError_t e = cudaFuncSetAttribute(k_fwd_states<D, NB>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_BWD, st);
-    return launch_pdl(k_fwd_states<D, NB>, dim3(g.BH * 2), dim3(kSeqThreads), (size_t)smem, st, mk, mv, meb, sa);
+    return launch_pdl(k_fwd_states<D, NB>, dim3(g.BH * 2), dim3(kSeqThreads), (size_t)smem, st, mk, mv, meb, mw, sa);
 }
 
 cudaError_t launch_fwd_states(const BwdGeo &g, const CUtensorMap &mk, const CUtensorMap &mv, const CUtensorMap &meb,
-                              const SeqArgs &sa, cudaStream_t st) {
+                              const CUtensorMap &mw, const SeqArgs &sa, cudaStream_t st) {
     const int NB = g.RP / 128;
-    if (g.D == 128) return NB == 1 ? launch_fwd_states_t<128, 1>(g, mk, mv, meb, sa, st)
-                                   : launch_fwd_states_t<128, 2>(g, mk, mv, meb, sa, st);
-    if (g.D == 64) return NB == 1 ? launch_fwd_states_t<64, 1>(g, mk, mv, meb, sa, st)
-                                  : launch_fwd_states_t<64, 2>(g, mk, mv, meb, sa, st);
+    if (g.D == 128) return NB == 1 ? launch_fwd_states_t<128, 1>(g, mk, mv, meb, mw, sa, st)
+                                   : launch_fwd_states_t<128, 2>(g, mk, mv, meb, mw, sa, st);
+    if (g.D == 64) return NB == 1 ? launch_fwd_states_t<64, 1>(g, mk, mv, meb, mw, sa, st)
+                                  : launch_fwd_states_t<64, 2>(g, mk, mv, meb, mw, sa, st);
     return cudaErrorInvalidValue;
 }
 
 template <int D, int NB>
 cudaError_t launch_adj_states_t(const BwdGeo &g, const CUtensorMap &mdx, const CUtensorMap &map_, const CUtensorMap &mq,
                                 const CUtensorMap &mdo, const CUtensorMap &mdp, const CUtensorMap &mg,
-                                const CUtensorMap &meb, const SeqArgs &sa, cudaStream_t st) {
+                                const CUtensorMap &meb, const CUtensorMap &mgk, const CUtensorMap &mgv,
+                                const SeqArgs &sa, cudaStream_t st) {
     const int RP = NB * 128, sbytes = adj_stage_bytes(RP, D);
     int stages = (227 * 1024 - 1024 - 256 - RP * 256) / sbytes;
     if (stages > 2) stages = 2;
@@ -1507,17 +1563,18 @@ cudaError_t launch_adj_states_t(const BwdGeo &g, const CUtensorMap &mdx, const C
     if (e != cudaSuccess) return e;
     ProfScope ps(BLA_K_BWD, st);
     return launch_pdl(k_adj_states<D, NB>, dim3(g.BH * 2), dim3(kSeqThreads), (size_t)smem, st, mdx, map_, mq, mdo,
-                      mdp, mg, meb, sa, stages);
+                      mdp, mg, meb, mgk, mgv, sa, stages);
 }
 
 cudaError_t launch_adj_states(const BwdGeo &g, const CUtensorMap &mdx, const CUtensorMap &map_, const CUtensorMap &mq,
                               const CUtensorMap &mdo, const CUtensorMap &mdp, const CUtensorMap &mg,
-                              const CUtensorMap &meb, const SeqArgs &sa, cudaStream_t st) {
+                              const CUtensorMap &meb, const CUtensorMap &mgk, const CUtensorMap &mgv, const SeqArgs &sa,
+                              cudaStream_t st) {
     const int NB = g.RP / 128;
-    if (g.D == 128) return NB == 1 ? launch_adj_states_t<128, 1>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st)
-                                   : launch_adj_states_t<128, 2>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st);
-    if (g.D == 64) return NB == 1 ? launch_adj_states_t<64, 1>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st)
-                                  : launch_adj_states_t<64, 2>(g, mdx, map_, mq, mdo, mdp, mg, meb, sa, st);
+    if (g.D == 128) return NB == 1 ? launch_adj_states_t<128, 1>(g, mdx, map_, mq, mdo, mdp, mg, meb, mgk, mgv, sa, st)
+                                   : launch_adj_states_t<128, 2>(g, mdx, map_, mq, mdo, mdp, mg, meb, mgk, mgv, sa, st);
+    if (g.D == 64) return NB == 1 ? launch_adj_states_t<64, 1>(g, mdx, map_, mq, mdo, mdp, mg, meb, mgk, mgv, sa, st)
+                                  : launch_adj_states_t<64, 2>(g, mdx, map_, mq, mdo, mdp, mg, meb, mgk, mgv, sa, st);
     return cudaErrorInvalidValue;
 }
 
@@ -1606,7 +1663,7 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
 
     // ---- tensor maps
     CUtensorMap qK, kK, kM, vK, dOK, ebK128, ebKR, ebM, phiK, phiM;
-    CUtensorMap wbK, wbM, PK, YK, pK, AK, GK, dGK, dUK, dsK, dXK, dPK;
+    CUtensorMap wbK, wbM, PK, YK, pK, AK, GK, dGK, dUK, dsK, dXK, dPK, dkS, dvS;
     bool ok = map_seq(&qK, q, g, D, true, kC) && map_seq(&kK, k, g, D, true, kC) && map_seq(&kM, k, g, D, false, 0) &&
               map_seq(&vK, v, g, D, true, kC) && map_seq(&dOK, dout, g, D, true, kC) &&
               map_2d(&ebK128, eb, kC, g.RP, true, 128) && map_2d(&ebKR, eb, kC, g.RP, true, R2) &&
@@ -1617,7 +1674,8 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
               map_z(&pK, pb, SP, kC, Z, true, kC) && map_z(&AK, Ab, R2, kC, Z, true, kC) &&
               map_z(&GK, Gb, kC, kC, Z, true, kC) && map_z(&dGK, dGb, kC, kC, Z, true, kC) &&
               map_z(&dUK, dUb, R2, kC, Z, true, kC) && map_z(&dsK, dsb, SP, kC, Z, true, kC) &&
-              map_z(&dXK, dXb, R2, kC, Z, true, kC) && map_z(&dPK, dPb, kC, kC, Z, true, kC);
+              map_z(&dXK, dXb, R2, kC, Z, true, kC) && map_z(&dPK, dPb, kC, kC, Z, true, kC) &&
+              map_seq(&dkS, dk, g, D, true, kC) && map_seq(&dvS, dv, g, D, true, kC);
     if (!ok) return cudaErrorInvalidValue;
     const Operand SEQK = opnd(OP_SEQ, 1), SEQM = opnd(OP_SEQ, 0);
     const Operand ZK = opnd(OP_Z, 1), ZM = opnd(OP_Z, 0);
@@ -1630,7 +1688,7 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     sa.BH = g.BH; sa.L = g.L; sa.nch = g.nch; sa.M = g.M; sa.R2 = R2; sa.RP = g.RP; sa.D = D;
     sa.erel = t.erel; sa.wout = wb; sa.gout[0] = static_cast<bf16 *>(dk); sa.gout[1] = static_cast<bf16 *>(dv);
     sa.err = device_error_word();
-    if ((e = launch_fwd_states(g, kK, vK, ebK128, sa, st)) != cudaSuccess) return e;
+    if ((e = launch_fwd_states(g, kK, vK, ebK128, wbK, sa, st)) != cudaSuccess) return e;
     if (chain_fits(g)) {
         // ---- 1-2. the chunk-local chains, fused
         ChainArgs ca;
@@ -1642,7 +1700,7 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
         if (!map_seq(&dqK, dq, g, D, true, kC)) return cudaErrorInvalidValue;
         if ((e = launch_chains(g, ca, qK, kK, vK, dOK, wbK, pK, ebKR, phiK, AK, GK, dXK, dPK, dqK, st)) != cudaSuccess)
             return e;
-        if ((e = launch_adj_states(g, dXK, AK, qK, dOK, dPK, GK, ebK128, sa, st)) != cudaSuccess) return e;
+        if ((e = launch_adj_states(g, dXK, AK, qK, dOK, dPK, GK, ebK128, dkS, dvS, sa, st)) != cudaSuccess) return e;
         return cudaSuccess;
     }
     Epi ep;
@@ -1682,7 +1740,7 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     if ((e = gemm(g, 1, D, dPK, ZK, kM, SEQM, kC, &dXK, &ZK, &wbM, &WK_M, R2, ep, st))) return e;
     // ---- 3. adjoint states backwards over the chunks, with dK = dP^T Q + EB^T Lk and
     //         dV = G^T dO + EB^T Lv for every chunk on the way
-    if ((e = launch_adj_states(g, dXK, AK, qK, dOK, dPK, GK, ebK128, sa, st)) != cudaSuccess) return e;
+    if ((e = launch_adj_states(g, dXK, AK, qK, dOK, dPK, GK, ebK128, dkS, dvS, sa, st)) != cudaSuccess) return e;
     return cudaSuccess;
 }
 
