@@ -621,17 +621,18 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // ================================================================== segment scan
-// W_in(0) = 0; W_in(g+1) = e^{i m w Lseg} W_in(g) + delta(g).  One thread per (head, K|V, mode, d).
+// W_in(0) = 0; W_in(g+1) = e^{i m w Lseg} W_in(g) + delta(g).  One thread per (head, K|V, mode, four
+// consecutive state columns): the index arithmetic and the mode's phase are paid once per four
+// columns, and every access is 16 bytes wide.
 __global__ void k_scan(Args a) {
     tc::pdl_wait();      // the segment deltas
     const Geo &g = a.g;
-    // 32-bit index arithmetic (the host checks that the element count fits): 64-bit divisions made
-    // this kernel instruction-bound
-    const unsigned total = (unsigned)g.BH * 2u * (unsigned)g.M * (unsigned)g.D;
-    const unsigned uD = (unsigned)g.D, uM = (unsigned)g.M;
+    const int vsh = g.D == 128 ? 5 : 4;   // float4 per state row: D / 4 = 32 or 16
+    // (the host checks that the thread count fits 32 bits)
+    const unsigned total = ((unsigned)g.BH * 2u * (unsigned)g.M) << vsh, uM = (unsigned)g.M;
     for (unsigned i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
-        const int e = (int)(i % uD);
-        unsigned r = i / uD;
+        const int e = (int)(i & ((1u << vsh) - 1u)) * 4;
+        unsigned r = i >> vsh;
         const int m = (int)(r % uM);
         r /= uM;
         const int x = (int)(r & 1u);
@@ -639,29 +640,32 @@ __global__ void k_scan(Args a) {
         float c, s;
         const HeadW hw = head_w(a, bh);
         mode_phase((long long)m * g.Lseg, hw.w, hw.tint, &c, &s);
-        float re = 0.f, im = 0.f;
+        float4 re = make_float4(0.f, 0.f, 0.f, 0.f), im = re;
+        // rows 2m (Re) and 2m+1 (Im) of segment seg: base + seg * seg_stride
+        const size_t seg_stride = (size_t)2 * g.RP * g.D;
+        const size_t base = (((size_t)bh * g.G * 2 + x) * g.RP + 2 * m) * g.D + e;
         // the deltas of eight segments are loaded before they are used, so that their latencies overlap
         for (int s0 = 0; s0 < g.G; s0 += 8) {
-            float dre[8], dim[8];
+            float4 dre[8], dim[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int seg = s0 + j;
-                dre[j] = dim[j] = 0.f;
+                dre[j] = dim[j] = make_float4(0.f, 0.f, 0.f, 0.f);
                 if (seg + 1 < g.G) {
-                    const size_t base = (((size_t)bh * g.G + seg) * 2 + x) * g.RP;
-                    dre[j] = a.deltas[(base + 2 * m) * g.D + e];
-                    dim[j] = a.deltas[(base + 2 * m + 1) * g.D + e];
+                    dre[j] = *reinterpret_cast<const float4 *>(a.deltas + base + seg * seg_stride);
+                    dim[j] = *reinterpret_cast<const float4 *>(a.deltas + base + seg * seg_stride + g.D);
                 }
             }
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const int seg = s0 + j;
                 if (seg >= g.G) break;
-                const size_t base = (((size_t)bh * g.G + seg) * 2 + x) * g.RP;
-                a.win[(base + 2 * m) * g.D + e] = re;
-                a.win[(base + 2 * m + 1) * g.D + e] = im;
-                const float nre = c * re - s * im + dre[j];
-                const float nim = s * re + c * im + dim[j];
+                *reinterpret_cast<float4 *>(a.win + base + seg * seg_stride) = re;
+                *reinterpret_cast<float4 *>(a.win + base + seg * seg_stride + g.D) = im;
+                const float4 nre = make_float4(c * re.x - s * im.x + dre[j].x, c * re.y - s * im.y + dre[j].y,
+                                               c * re.z - s * im.z + dre[j].z, c * re.w - s * im.w + dre[j].w);
+                const float4 nim = make_float4(s * re.x + c * im.x + dim[j].x, s * re.y + c * im.y + dim[j].y,
+                                               s * re.z + c * im.z + dim[j].z, s * re.w + c * im.w + dim[j].w);
                 re = nre;
                 im = nim;
             }
@@ -1746,8 +1750,8 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
                 return e;
         }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
-        long long tot = (long long)g.BH * 2 * g.M * g.D;
-        if (tot > 0x7fffffffLL) return cudaErrorInvalidValue;   // k_scan indexes in 32 bits
+        long long tot = (long long)g.BH * 2 * g.M * (g.D / 4);   // k_scan: four state columns per thread
+        if (tot > 0x7fffffffLL) return cudaErrorInvalidValue;        // (indexed in 32 bits)
         int blocks = (int)((tot + 255) / 256);
         if (blocks > 4096) blocks = 4096;
         {
