@@ -158,11 +158,43 @@ struct HeadTint {
     int t[kMaxHeadPeriods];   // each head's integer period for exact phase reduction (0: fp64 phases)
 };
 
+// One EB item of one head's table `eb` ([nch][RP][C]): rows 2m and 2m+1 of chunk c for 8 consecutive u,
+// item ui = (c MP + m) (C / 8) + u0 / 8 (u fastest, so that a warp writes whole rows).
+__device__ __forceinline__ void eb_item(bf16 *eb, int M, int RP, unsigned ui, double w, int tint) {
+    // (32-bit index arithmetic: nch MP C / 8 = 16 L < 2^31 for L <= 2^26, which the host checks)
+    const unsigned per_c = (unsigned)(RP / 2) * (kC / 8);
+    const int c = (int)(ui / per_c), rem = (int)(ui - (unsigned)c * per_c);
+    const int m = rem / (kC / 8), u0 = (rem % (kC / 8)) * 8;
+    bf16 *rc = eb + ((size_t)c * RP + 2 * m) * kC + u0, *rs = rc + kC;
+    uint32_t wc[4] = {0u, 0u, 0u, 0u}, ws[4] = {0u, 0u, 0u, 0u};
+    if (m < M) {
+        float bc, bs, ec, es;
+        mode_phase((long long)m * ((long long)c * kC + u0), w, tint, &bc, &bs);
+        mode_phase((long long)m, w, tint, &ec, &es);
+#pragma unroll
+        for (int j = 0; j < 8; j += 2) {
+            const float c0 = bc, s0 = bs;
+            float t = bc * ec - bs * es;
+            bs = bc * es + bs * ec;
+            bc = t;
+            wc[j / 2] = tc::pack_bf16x2(c0, bc);
+            ws[j / 2] = tc::pack_bf16x2(-s0, -bs);
+            t = bc * ec - bs * es;
+            bs = bc * es + bs * ec;
+            bc = t;
+        }
+    }
+    *reinterpret_cast<uint4 *>(rc) = make_uint4(wc[0], wc[1], wc[2], wc[3]);
+    *reinterpret_cast<uint4 *>(rs) = make_uint4(ws[0], ws[1], ws[2], ws[3]);
+}
+
+// With eb_skip the EB tables are left to the segment prepass (whose epilogue warps are idle while
+// its MMAs stream K and V); everything else is written here.
 __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, HeadPeriods hp, HeadTint ht, double T0,
                               double w0, int tint0, float sin_sign, bf16 *eb0, bf16 *phi0, bf16 *fseg0, int *delta0,
-                              double *hw, int *htint) {
+                              double *hw, int *htint, int eb_skip) {
     const int R2 = 2 * M, MP = RP / 2;
-    const long long n_eb = (long long)nch * MP * (kC / 8), n_phi = (long long)SP * R2;
+    const long long n_eb = eb_skip ? 0 : (long long)nch * MP * (kC / 8), n_phi = (long long)SP * R2;
     const long long n_f = fseg0 ? (long long)MP * ((Lseg + 7) / 8) : 0, n_d = delta0 ? S : 0;
     const long long per = n_eb + n_phi + n_f + n_d + 1;
     const int nh = hp.n > 0 ? hp.n : 1;
@@ -183,31 +215,7 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, H
                 htint[h] = tint;
             }
         } else if (i < n_eb) {
-            // (32-bit index arithmetic: n_eb = 16 L < 2^31 for L <= 2^26, which the host checks)
-            const unsigned per_c = (unsigned)MP * (kC / 8), ui = (unsigned)i;
-            const int c = (int)(ui / per_c), rem = (int)(ui - (unsigned)c * per_c);
-            const int m = rem / (kC / 8), u0 = (rem % (kC / 8)) * 8;
-            bf16 *rc = eb + ((size_t)c * RP + 2 * m) * kC + u0, *rs = rc + kC;
-            uint32_t wc[4] = {0u, 0u, 0u, 0u}, ws[4] = {0u, 0u, 0u, 0u};
-            if (m < M) {
-                float bc, bs, ec, es;
-                mode_phase((long long)m * ((long long)c * kC + u0), w, tint, &bc, &bs);
-                mode_phase((long long)m, w, tint, &ec, &es);
-#pragma unroll
-                for (int j = 0; j < 8; j += 2) {
-                    const float c0 = bc, s0 = bs;
-                    float t = bc * ec - bs * es;
-                    bs = bc * es + bs * ec;
-                    bc = t;
-                    wc[j / 2] = tc::pack_bf16x2(c0, bc);
-                    ws[j / 2] = tc::pack_bf16x2(-s0, -bs);
-                    t = bc * ec - bs * es;
-                    bs = bc * es + bs * ec;
-                    bc = t;
-                }
-            }
-            *reinterpret_cast<uint4 *>(rc) = make_uint4(wc[0], wc[1], wc[2], wc[3]);
-            *reinterpret_cast<uint4 *>(rs) = make_uint4(ws[0], ws[1], ws[2], ws[3]);
+            eb_item(eb, M, RP, (unsigned)i, w, tint);
         } else if (i < n_eb + n_phi) {
             const int e = (int)(i - n_eb);
             const int j = e / R2, r = e % R2, m = r >> 1;
@@ -231,12 +239,25 @@ __global__ void k_tables_bf16(int M, int S, int SP, int RP, int Lseg, int nch, H
                 mode_phase((long long)m * (Lseg - u0), w, tint, &bc, &bs);
                 mode_phase((long long)m, w, tint, &ec, &es);
             }
-            for (int j = 0; j < 8 && u0 + j < Lseg; ++j) {
-                rc[j] = __float2bfloat16_rn(bc);
-                rs[j] = __float2bfloat16_rn(bs);
+            float vc[8], vs[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                vc[j] = bc;
+                vs[j] = bs;
                 const float t = bc * ec + bs * es;   // times e^{-i m w}
                 bs = bs * ec - bc * es;
                 bc = t;
+            }
+            if (u0 + 8 <= Lseg && (Lseg & 7) == 0) {   // whole 16-byte pieces of 16-byte aligned rows
+                *reinterpret_cast<uint4 *>(rc) = make_uint4(tc::pack_bf16x2(vc[0], vc[1]), tc::pack_bf16x2(vc[2], vc[3]),
+                                                            tc::pack_bf16x2(vc[4], vc[5]), tc::pack_bf16x2(vc[6], vc[7]));
+                *reinterpret_cast<uint4 *>(rs) = make_uint4(tc::pack_bf16x2(vs[0], vs[1]), tc::pack_bf16x2(vs[2], vs[3]),
+                                                            tc::pack_bf16x2(vs[4], vs[5]), tc::pack_bf16x2(vs[6], vs[7]));
+            } else {
+                for (int j = 0; j < 8 && u0 + j < Lseg; ++j) {
+                    rc[j] = __float2bfloat16_rn(vc[j]);
+                    rs[j] = __float2bfloat16_rn(vs[j]);
+                }
             }
         } else {
             const int j = (int)(i - n_eb - n_phi - n_f);
@@ -269,6 +290,10 @@ struct Args {
     int eb_rows_h, phi_rows_h, f_rows_h, delta_h;
     const double *hw;
     const int *htint;
+    // EB tables written by the prepass's epilogue warps while its MMAs run (null: the tables kernel
+    // wrote them); eb_nh heads of [nchunks][RP][C] each
+    bf16 *eb_gen;
+    int eb_nh;
 };
 
 // Mode frequency and integer period of head bh % H (written by the tables kernel: read them only
@@ -597,6 +622,18 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc::mma_commit(done);
     } else if (warp < 4) {
+        if (a.eb_gen) {
+            // this CTA's share of the EB tables (the CTAs of every segment but the last get here)
+            const unsigned n_eb = (unsigned)g.nchunks * (unsigned)(g.RP / 2) * (kC / 8);
+            const unsigned nct = (unsigned)g.BH * (unsigned)(g.G - 1), ci = (unsigned)bh * (g.G - 1) + seg;
+            const unsigned nitems = n_eb * (unsigned)a.eb_nh;
+            for (unsigned i = ci * 128u + threadIdx.x; i < nitems; i += nct * 128u) {
+                const int h = (int)(i / n_eb);
+                const double w = a.hw ? a.hw[h] : a.w;
+                const int tint = a.hw ? a.htint[h] : a.tint;
+                eb_item(a.eb_gen + (size_t)h * g.nchunks * g.RP * kC, g.M, g.RP, i - (unsigned)h * n_eb, w, tint);
+            }
+        }
         uint32_t ph = 0;
         bool ok = wait_bar(done, ph, ctl, a.err);
         tc::tc_fence_after();
@@ -1543,10 +1580,10 @@ cudaError_t build_bf16_tables(const OpDims &d, int RP, int SP, bf16 *eb, bf16 *p
     if (blocks > 2048) blocks = 2048;
     HeadPeriods hp;
     hp.n = 0;
-    HeadTint ht;
+    HeadTint ht = {};
     ProfScope ps(BLA_K_TABLES_BF16, st);
     k_tables_bf16<<<blocks, 256, 0, st>>>(d.M, d.S, SP, RP, 1, 1, hp, ht, d.T, d.w, integer_period(d),
-                                          d.absolute ? -1.f : 1.f, eb, phi, nullptr, nullptr, nullptr, nullptr);
+                                          d.absolute ? -1.f : 1.f, eb, phi, nullptr, nullptr, nullptr, nullptr, 0);
     return cudaGetLastError();
 }
 
@@ -1685,14 +1722,17 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     for (int h = 0; h < hp.n; ++h) ht.t[h] = integer_period(hp.T[h], hp.w[h]);
     const int nh = hp.n > 0 ? hp.n : 1;
     {
-        // EB of every chunk (absolute phases), PHI, FSEG and the slot lags in one launch
-        const long long total = nh * ((long long)g.nchunks * (g.RP / 2) * (kC / 8) + (long long)g.SP * g.R2 +
+        // EB of every chunk (absolute phases), PHI, FSEG and the slot lags in one launch; with segments
+        // the prepass writes EB instead
+        const int eb_skip = g.G > 1 ? 1 : 0;
+        const long long total = nh * ((eb_skip ? 0 : (long long)g.nchunks * (g.RP / 2) * (kC / 8)) +
+                                      (long long)g.SP * g.R2 +
                                       (fseg ? (long long)(g.RP / 2) * ((g.Lseg + 7) / 8) : 0) + g.S + 1);
         const int blocks = (int)(total < 4096 * 256 ? (total + 255) / 256 : 4096);
         ProfScope ps(BLA_K_TABLES_BF16, st);
         k_tables_bf16<<<blocks, 256, 0, st>>>(g.M, g.S, g.SP, g.RP, g.Lseg, g.nchunks, hp, ht, d.T, d.w,
                                               integer_period(d), d.absolute ? -1.f : 1.f, eb, phi, fseg, delta, hw,
-                                              htint);
+                                              htint, eb_skip);
         if ((e = cudaGetLastError()) != cudaSuccess) return e;
     }
     Args a;
@@ -1717,6 +1757,8 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     a.delta_h = hp.n > 0 ? g.S : 0;
     a.hw = hw;
     a.htint = htint;
+    a.eb_gen = g.G > 1 ? eb : nullptr;
+    a.eb_nh = nh;
 
     // tensor maps
     CUtensorMap tq, tk, tv, tp, teb, tphi, tf;
