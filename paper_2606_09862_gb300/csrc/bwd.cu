@@ -1659,7 +1659,6 @@ cudaError_t bwd_run(const OpDims &d, const void *q, const void *k, const void *v
     bf16 *dUb = reinterpret_cast<bf16 *>(ws + w.dU), *dsb = reinterpret_cast<bf16 *>(ws + w.ds);
     bf16 *dXb = reinterpret_cast<bf16 *>(ws + w.dX), *dPb = reinterpret_cast<bf16 *>(ws + w.dP);
     const int D = g.D, R2 = g.R2, S = g.S, SP = g.SP, Z = g.Z;
-    const int rt = g.R2 <= 128 ? 1 : g.R2 / 128;   // 128-row tiles of an [R2 x D] result
 
     // ---- tensor maps
     CUtensorMap qK, kK, kM, vK, dOK, ebK128, ebKR, ebM, phiK, phiM;
