@@ -61,6 +61,8 @@ def test_bf16_forward(orc, B, H, L, d, M, S, T):
     (2, 1, 63, 128, 32, 64, 512.0),     # one ragged chunk
     (1, 1, 1, 64, 8, 32, 64.0),         # a single token: one item, one state update
     (1, 2, 33, 128, 16, 64, 100.0),     # one chunk and one token
+    (1, 2, 97, 128, 16, 32, 64.0),      # S = 32 with d = 128
+    (2, 1, 161, 64, 32, 64, 300.0),     # S = 64 with d = 64
 ])
 def test_bf16_chunked_forward(orc, B, H, L, d, M, S, T):
     """The chunked tensor-core form (d in {64, 128}, S in {32, 64}): o per row, lse and state."""
