@@ -550,7 +550,7 @@ constexpr int kPreStages = 3;
 
 __global__ void __launch_bounds__(kThreads, 1)
     k_prepass(const __grid_constant__ CUtensorMap tm_k, const __grid_constant__ CUtensorMap tm_v,
-              const __grid_constant__ CUtensorMap tm_f, Args a) {
+              const __grid_constant__ CUtensorMap tm_f, const __grid_constant__ CUtensorMap tm_d, Args a) {
     const Geo &g = a.g;
     const int seg = blockIdx.x % g.G, bh = blockIdx.x / g.G;
     if (seg >= g.G - 1) return;   // the last segment's delta is never used
@@ -638,15 +638,37 @@ __global__ void __launch_bounds__(kThreads, 1)
         bool ok = wait_bar(done, ph, ctl, a.err);
         tc::tc_fence_after();
         if (ok) {
-            const int row = threadIdx.x;
-            for (int x = 0; x < 2; ++x)
-                for (int b = 0; b < NB; ++b) {
-                    float *dst = a.deltas_out + ((((size_t)bh * g.G + seg) * 2 + x) * g.RP + b * 128 + row) * D;
-                    if (D == 128)
-                        state_pass<128>(tb, (b * 2 + x) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
-                    else
-                        state_pass<64>(tb, (b * 2 + x) * D, row, false, 1.f, 0.f, false, nullptr, 0, dst);
+            // The deltas leave through the (now idle) pipeline stages: thread = state row writes its
+            // row into [NB][D/32][128 rows][32] fp32 boxes (128-byte swizzled), and thread 0 stores
+            // them by TMA, K first, then V
+            const int row = threadIdx.x, lane_base = (row >> 5) << 5;
+            for (int x = 0; x < 2; ++x) {
+                if (x > 0) {
+                    if (row == 0) tc::bulk_wait_read0();   // the K boxes have been read
+                    tc::named_bar(1, 128);
                 }
+                for (int b = 0; b < NB; ++b)
+                    for (int cb = 0; cb < D / 32; ++cb) {
+                        float v[32];
+                        tc::tmem_ld<32>(tmem_addr(tb, lane_base, (b * 2 + x) * D + cb * 32), v);
+                        uint8_t *box = stage0 + (size_t)(b * (D / 32) + cb) * 128 * 128;
+#pragma unroll
+                        for (int q = 0; q < 8; ++q)
+                            *reinterpret_cast<float4 *>(box + row * 128 + ((q ^ (row & 7)) << 4)) =
+                                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                    }
+                tc::fence_proxy_async_smem();
+                tc::named_bar(1, 128);
+                if (row == 0) {
+                    const int r0 = (int)((((size_t)bh * g.G + seg) * 2 + x) * g.RP);
+                    for (int b = 0; b < NB; ++b)
+                        for (int cb = 0; cb < D / 32; ++cb)
+                            tc::tma_store_2d(&tm_d, stage0 + (size_t)(b * (D / 32) + cb) * 128 * 128, cb * 32,
+                                             r0 + b * 128);
+                    tc::bulk_commit();
+                }
+            }
+            if (row == 0) tc::bulk_wait0();
         }
     }
     tc::tc_fence_before();
@@ -1761,7 +1783,7 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
     a.eb_nh = nh;
 
     // tensor maps
-    CUtensorMap tq, tk, tv, tp, teb, tphi, tf;
+    CUtensorMap tq, tk, tv, tp, teb, tphi, tf, tdl;
     const uint64_t dq[3] = {(uint64_t)g.D, (uint64_t)g.L, (uint64_t)g.BH};
     const uint64_t sq[2] = {(uint64_t)g.D * 2, (uint64_t)g.L * g.D * 2};
     const uint32_t bq[3] = {64, (uint32_t)kC, 1};
@@ -1782,13 +1804,18 @@ cudaError_t fwd_bf16_run(const OpDims &d, const void *q, const void *k, const vo
         const uint64_t df[2] = {(uint64_t)g.Lseg, (uint64_t)nh * g.RP}, sf[1] = {(uint64_t)g.Lseg * 2};
         const uint32_t bf[2] = {64, 128};
         if (!make_tmap_bf16(&tf, fseg, 2, df, sf, bf)) return cudaErrorInvalidValue;
+        // the segment deltas, fp32 [BH][G][2][RP][D], stored by the prepass in [128 rows][32] boxes
+        const uint64_t dd[2] = {(uint64_t)g.D, (uint64_t)g.BH * g.G * 2 * g.RP}, sd[1] = {(uint64_t)g.D * 4};
+        const uint32_t bd[2] = {32, 128};
+        if (!make_tmap_f32(&tdl, a.deltas_out, 2, dd, sd, bd)) return cudaErrorInvalidValue;
         const size_t stage_bytes = (size_t)g.NB * 128 * 64 * 2 + 2 * (size_t)64 * g.D * 2;
         const int smem = smem_request(kPreStages * stage_bytes + 256 + 1024, pow2_cols(2 * g.NB * g.D));
         if ((e = cudaFuncSetAttribute(k_prepass, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
             return e;
         {
             ProfScope ps(BLA_K_PREPASS, st);
-            if ((e = launch_pdl(k_prepass, dim3(nblk), dim3(kThreads), (size_t)smem, st, tk, tv, tf, a)) != cudaSuccess)
+            if ((e = launch_pdl(k_prepass, dim3(nblk), dim3(kThreads), (size_t)smem, st, tk, tv, tf, tdl, a)) !=
+                cudaSuccess)
                 return e;
         }
         if ((e = cudaGetLastError()) != cudaSuccess) return e;

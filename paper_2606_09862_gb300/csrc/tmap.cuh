@@ -1,4 +1,4 @@
-// tmap.cuh -- host-side construction of TMA tensor maps (bf16, 128-byte swizzle or none).
+// tmap.cuh -- host-side construction of TMA tensor maps (bf16 with 128-byte swizzle or none; fp32).
 #pragma once
 #include <cuda.h>
 #include <stdint.h>
@@ -13,5 +13,8 @@ namespace bla {
 // Returns false if the driver entry point is unavailable or the encode fails.
 bool make_tmap_bf16(CUtensorMap *map, const void *base, int rank, const uint64_t *dims,
                     const uint64_t *strides_bytes, const uint32_t *box, bool swizzle128 = true);
+// The same for fp32 tensors, 128-byte swizzle: box[0] is 32 (128 bytes).
+bool make_tmap_f32(CUtensorMap *map, const void *base, int rank, const uint64_t *dims,
+                   const uint64_t *strides_bytes, const uint32_t *box);
 
 }  // namespace bla
