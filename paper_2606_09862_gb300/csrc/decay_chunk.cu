@@ -1494,8 +1494,9 @@ size_t decay_chunk_bwd_ws_bytes(const OpDims &d) { return db_ws(d, true).total; 
 size_t decay_chunk_fwd_ws_bytes(const OpDims &d) { return db_ws(d, false).total; }
 
 bool decay_chunk_supported(const OpDims &d) {
+    // (the thin passes put the heads on the grid's z dimension: at most 65535 of them)
     return d.dtype == BLA_BF16 && d.dk == d.dv && (d.dk == 64 || d.dk == 128) && (d.S == 32 || d.S == 64) &&
-           d.L > 0;
+           d.L > 0 && (long long)d.B * d.H <= 65535;
 }
 
 cudaError_t launch_decay_chunk_bwd(const OpDims &d, long long pos0, int dmax, const float *Dx, const int *delta,
