@@ -41,10 +41,11 @@ constexpr int kThreads = 192;
 // 10 issues the bulk stores of finished output tiles (K pass), 11 only completes the third
 // warpgroup.  In the K pass the third warpgroup hands registers to the first two: launched with
 // kLaunchRegs each (65536 / 384 rounded down to the allocation granule), it drops to kCtlRegs and
-// the epilogue warpgroups rise to kEpiRegs, within the launch's total.  (The V pass measured
-// slower with the same split and keeps kLaunchRegs everywhere.)
+// the epilogue warpgroups rise to kEpiRegs, within the launch's total (the MMA issuer spills less at
+// 56 than at 40, which measured faster).  (The V pass measured slower with the same split and keeps
+// kLaunchRegs everywhere.)
 constexpr int kPassThreads = 384;
-constexpr int kLaunchRegs = 168, kCtlRegs = 40, kEpiRegs = 232;
+constexpr int kLaunchRegs = 168, kCtlRegs = 56, kEpiRegs = 224;
 static_assert(128 * kCtlRegs + 256 * kEpiRegs <= kPassThreads * kLaunchRegs, "register split exceeds the launch");
 constexpr int kPassEpiWarps = 8;
 
@@ -732,6 +733,30 @@ __global__ void k_scan(Args a) {
     }
 }
 
+// Packed fp32 pairs (f32x2): one instruction for two elementwise operations, each rounded as the scalar
+// operation would be.  The softmax uses them for its scale, exponent argument, sums and normalisation,
+// which shortens the epilogue's instruction stream per chunk.
+__device__ __forceinline__ void mul2_bcast(float &x, float &y, float s) {
+    asm("{\n\t.reg .b64 a, b;\n\tmov.b64 a, {%0, %1};\n\tmov.b64 b, {%2, %2};\n\tmul.rn.f32x2 a, a, b;\n\t"
+        "mov.b64 {%0, %1}, a;\n\t}"
+        : "+f"(x), "+f"(y)
+        : "f"(s));
+}
+__device__ __forceinline__ float2 sub2_bcast(float x, float y, float s) {
+    float2 r;
+    asm("{\n\t.reg .b64 a, b;\n\tmov.b64 a, {%2, %3};\n\tmov.b64 b, {%4, %4};\n\tsub.rn.f32x2 a, a, b;\n\t"
+        "mov.b64 {%0, %1}, a;\n\t}"
+        : "=f"(r.x), "=f"(r.y)
+        : "f"(x), "f"(y), "f"(s));
+    return r;
+}
+__device__ __forceinline__ void add2(float &x, float &y, float a, float b) {
+    asm("{\n\t.reg .b64 u, w;\n\tmov.b64 u, {%0, %1};\n\tmov.b64 w, {%2, %3};\n\tadd.rn.f32x2 u, u, w;\n\t"
+        "mov.b64 {%0, %1}, u;\n\t}"
+        : "+f"(x), "+f"(y)
+        : "f"(a), "f"(b));
+}
+
 // ================================================================== K pass
 
 struct KLayout {
@@ -991,19 +1016,22 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 const float2 f = abs_phase((long long)((b * 128 + row) >> 1) * c_begin * kC, hph.w, hph.tint);
                 state_init_abs<DH>(tb, b * D + wg * DH, row, src ? src + wg * DH : nullptr, g.R2 - b * 128, D, f.x, f.y);
             }
-            // W_h: state block h after the previous chunk's update, packed to bf16 in registers
-            // (w_compute); copied into the W tile once the MMA that read the previous W is done (w_store).
-            auto w_compute = [&](int h, bool wait_update, uint32_t *pk) -> bool {
+            // W_h: state block h after the previous chunk's update (once that update is done), copied from
+            // TMEM into the W tile as bf16 once the MMA that read the previous W is done.  Read just before it
+            // is stored (nothing waits for it sooner), in 32-column blocks, so that no packed copy is held in
+            // registers across the chunk.
+            auto w_copy = [&](int h, bool wait_update, bool wait_free) -> bool {
                 if (wait_update && !wait_bar(&bar[KB_STATE_DONE + h], ph_states, h, ctl, a.err)) return false;
-                tc::tc_fence_after();
-                state_pack<DH>(tb, h * D + wg * DH, row, pk);
-                return true;
-            };
-            auto w_store = [&](bool wait_free, const uint32_t *pk) -> bool {
                 if (wait_free && !wait_bar(&bar[KB_W_FREE], ph_wfree, ctl, a.err)) return false;
-                if (row < RH) {
+                tc::tc_fence_after();
+#pragma unroll 1
+                for (int g0 = 0; g0 < DH; g0 += 32) {
+                    float v[32];
+                    tc::tmem_ld<32>(tmem_addr(tb, lane_base, h * D + wg * DH + g0), v);
+                    uint32_t pk[16];
 #pragma unroll
-                    for (int g0 = 0; g0 < DH; g0 += 32) st_row32_packed(sW, RH, row, wg * DH + g0, pk + g0 / 2);
+                    for (int i = 0; i < 32; i += 2) pk[i / 2] = tc::pack_bf16x2(v[i], v[i + 1]);
+                    if (row < RH) st_row32_packed(sW, RH, row, wg * DH + g0, pk);
                 }
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
@@ -1013,29 +1041,33 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             // Y_h = e^{i m w t} X_h (t = absolute token of this row) from accumulator region `col`,
             // two interleaved mode chains
             auto y_drain = [&](int h, int col, const RowPhases &rp) {
-                float v[XH];
-                tc::tmem_ld<XH>(tmem_addr(tb, lane_base, col + wg * XH), v);
                 const float2 pa = h ? rp.h1 : rp.h0, pb = cmul(pa, rp.e1), e2 = rp.e2;
                 float ca = pa.x, sa = pa.y, cb = pb.x, sb = pb.y;
+                // 32-column blocks in a rolled loop: the epilogue's code per chunk has to stay within the
+                // instruction cache, and the phases carry from block to block
+#pragma unroll 1
+                for (int g0 = 0; g0 < XH; g0 += 32) {
+                    float v[32];
+                    tc::tmem_ld<32>(tmem_addr(tb, lane_base, col + wg * XH + g0), v);
 #pragma unroll
-                for (int i = 0; i < XH; i += 4) {
-                    float xr = v[i], xi = v[i + 1];
-                    v[i] = ca * xr - sa * xi;
-                    v[i + 1] = sa * xr + ca * xi;
-                    xr = v[i + 2];
-                    xi = v[i + 3];
-                    v[i + 2] = cb * xr - sb * xi;
-                    v[i + 3] = sb * xr + cb * xi;
-                    float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
-                    ca = t1;
-                    sa = t2;
-                    t1 = cb * e2.x - sb * e2.y;
-                    t2 = sb * e2.x + cb * e2.y;
-                    cb = t1;
-                    sb = t2;
+                    for (int i = 0; i < 32; i += 4) {
+                        float xr = v[i], xi = v[i + 1];
+                        v[i] = ca * xr - sa * xi;
+                        v[i + 1] = sa * xr + ca * xi;
+                        xr = v[i + 2];
+                        xi = v[i + 3];
+                        v[i + 2] = cb * xr - sb * xi;
+                        v[i + 3] = sb * xr + cb * xi;
+                        float t1 = ca * e2.x - sa * e2.y, t2 = sa * e2.x + ca * e2.y;
+                        ca = t1;
+                        sa = t2;
+                        t1 = cb * e2.x - sb * e2.y;
+                        t2 = sb * e2.x + cb * e2.y;
+                        cb = t1;
+                        sb = t2;
+                    }
+                    st_row32_bf16(sY, kC, row, wg * XH + g0, v);
                 }
-#pragma unroll
-                for (int g0 = 0; g0 < XH; g0 += 32) st_row32_bf16(sY, kC, row, wg * XH + g0, v + g0);
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
                 epi_arrive(&bar[KB_Y_READY]);
@@ -1044,14 +1076,14 @@ __global__ void __launch_bounds__(kPassThreads, 1)
             auto p_drain = [&]() -> bool {
                 if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) return false;
                 tc::tc_fence_after();
-                {
-                    float v[64];
-                    tc::tmem_ld<64>(tmem_addr(tb, lane_base, colA + wg * 64), v);
+#pragma unroll 1
+                for (int g0 = 0; g0 < 64; g0 += 32) {
+                    float v[32];
+                    tc::tmem_ld<32>(tmem_addr(tb, lane_base, colA + wg * 64 + g0), v);
 #pragma unroll
-                    for (int i = 0; i < 64; ++i)
-                        if (wg * 64 + i > row) v[i] = 0.f;
-#pragma unroll
-                    for (int g0 = 0; g0 < 64; g0 += 32) st_row32_bf16(sP, kC, row, wg * 64 + g0, v + g0);
+                    for (int i = 0; i < 32; ++i)
+                        if (wg * 64 + g0 + i > row) v[i] = 0.f;
+                    st_row32_bf16(sP, kC, row, wg * 64 + g0, v);
                 }
                 tc::fence_proxy_async_smem();
                 tc::tc_fence_before();
@@ -1060,20 +1092,16 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 return true;
             };
             // W_0 and W_1 of the first chunk (the carried-in state as it is) and its P
-            uint32_t pk1[DH / 2];   // W_1 of the coming chunk, stored once that chunk's Q W_0^T is done
             bool bad = false;
-            if (c_begin < c_end) {
-                uint32_t pk0[DH / 2];
-                bad = !w_compute(0, false, pk0) || !w_store(false, pk0) || (NH == 2 && !w_compute(1, false, pk1)) ||
-                      !p_drain();
-            }
+            if (c_begin < c_end) bad = !w_copy(0, false, false) || !p_drain();
             for (int c = c_begin; c < c_end && !bad; ++c) {
                 const int t0 = c * kC;
                 const int n = min(kC, g.L - t0);
                 const bool rot = c > c_begin, more = c + 1 < c_end;
                 if (rot) advance(rp, rp_step);
-                // W_1 (computed at the end of the previous chunk) once Q W_0^T has read W_0
-                if (NH == 2 && !w_store(true, pk1)) { bad = true; break; }
+                // W_1 once Q W_0^T has read W_0 (state_1 of the previous chunk's update: this chunk's state_1
+                // update waits for W_1, since Q W_1^T reads it)
+                if (NH == 2 && !w_copy(1, rot, true)) { bad = true; break; }
                 // Y_0 from B; the previous chunk's probabilities must have left the Y tile
                 if (!wait_bar(&bar[KB_ACC_FULL_B], ph_fullB, ctl, a.err)) { bad = true; break; }
                 if (rot && !wait_bar(&bar[KB_Y_STORED], ph_ystored, ctl, a.err)) { bad = true; break; }
@@ -1083,10 +1111,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 // W_0 of the next chunk (the state after this chunk's first update), stored once Q W_1^T (with
                 // one half Q W_0^T) has read the W tile: between the two Y drains, where the epilogue would
                 // otherwise wait for P EB_1^T and s_0
-                if (more) {
-                    uint32_t pk0[DH / 2];
-                    if (!w_compute(0, true, pk0) || !w_store(true, pk0)) { bad = true; break; }
-                }
+                if (more && !w_copy(0, true, true)) { bad = true; break; }
                 if (NH == 2) {
                     // Y_1 from A once s_0 has read Y_0
                     if (!wait_bar(&bar[KB_ACC_FULL_A], ph_fullA, ctl, a.err)) { bad = true; break; }
@@ -1094,8 +1119,6 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     tc::tc_fence_after();
                     y_drain(1, colA, rp);
                     epi_arrive(&bar[KB_ACC_FREE_A]);
-                    // W_1 of the next chunk into registers while s_1 runs
-                    if (more && !w_compute(1, true, pk1)) { bad = true; break; }
                 }
                 // masked softmax over the S slots; the two warpgroups exchange their (max, sum) pairs once
                 constexpr bool sB = NH == 2;
@@ -1122,9 +1145,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         float m4[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
                         if (all_visible) {
 #pragma unroll
-                            for (int j = 0; j < SH; ++j) {
-                                v[j] *= sl2;
+                            for (int j = 0; j < SH; j += 2) {
+                                mul2_bcast(v[j], v[j + 1], sl2);
                                 m4[j & 3] = fmaxf(m4[j & 3], v[j]);
+                                m4[(j + 1) & 3] = fmaxf(m4[(j + 1) & 3], v[j + 1]);
                             }
                         } else {
                             // the lags D_j do not decrease, so the visible slots are j < nvis(t): one
@@ -1150,11 +1174,11 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                         // bf16, whose resolution (2^-8) is coarser than the fp16 path's error
 #pragma unroll
                         for (int j = 0; j < SH; j += 2) {
-                            const float2 e2 = tc::exp2_pair_f16(v[j] - mref, v[j + 1] - mref);   // -inf -> 0
+                            const float2 d2 = sub2_bcast(v[j], v[j + 1], mref);
+                            const float2 e2 = tc::exp2_pair_f16(d2.x, d2.y);   // -inf -> 0
                             v[j] = e2.x;
                             v[j + 1] = e2.y;
-                            s4[j & 3] += e2.x;
-                            s4[(j + 1) & 3] += e2.y;
+                            add2(s4[j & 3], s4[(j + 1) & 3], e2.x, e2.y);
                         }
                         sum = (s4[0] + s4[1]) + (s4[2] + s4[3]);
                     }
@@ -1170,7 +1194,7 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     if (active) {
                         const float f = exp2f(mx - gmx) / gsum;
 #pragma unroll
-                        for (int j = 0; j < SH; ++j) v[j] *= f;
+                        for (int j = 0; j < SH; j += 2) mul2_bcast(v[j], v[j + 1], f);
 #pragma unroll
                         for (int g0 = 0; g0 < SH; g0 += 32) st_row32_bf16(sY, kC, row, j0 + g0, v + g0);
                     } else if (SP > S) {
