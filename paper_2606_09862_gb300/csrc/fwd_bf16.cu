@@ -41,11 +41,11 @@ constexpr int kThreads = 192;
 // 10 issues the bulk stores of finished output tiles (K pass), 11 only completes the third
 // warpgroup.  In the K pass the third warpgroup hands registers to the first two: launched with
 // kLaunchRegs each (65536 / 384 rounded down to the allocation granule), it drops to kCtlRegs and
-// the epilogue warpgroups rise to kEpiRegs, within the launch's total (the MMA issuer spills less at
-// 56 than at 40, which measured faster).  (The V pass measured slower with the same split and keeps
-// kLaunchRegs everywhere.)
+// the epilogue warpgroups rise to kEpiRegs, within the launch's total.  At 88 the control warps do not
+// spill (at 40 the MMA issuer did, which measured slower), and the epilogue's rolled drains fit in 208.
+// (The V pass measured slower with the same split and keeps kLaunchRegs everywhere.)
 constexpr int kPassThreads = 384;
-constexpr int kLaunchRegs = 168, kCtlRegs = 56, kEpiRegs = 224;
+constexpr int kLaunchRegs = 168, kCtlRegs = 88, kEpiRegs = 208;
 static_assert(128 * kCtlRegs + 256 * kEpiRegs <= kPassThreads * kLaunchRegs, "register split exceeds the launch");
 constexpr int kPassEpiWarps = 8;
 
