@@ -1365,8 +1365,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 }
             }
         } else if (warp == 9) {
-            // ---------------- MMA issuer.  Per chunk: U_0; U_1 (once A'_0 is drained); G = A'_0 EB_0;
-            // state_0 += EB_0 V; G += A'_1 EB_1; state_1 += EB_1 V; O = A'_0 W_0 (+ A'_1 W_1); O += G V.
+            // ---------------- MMA issuer.  Per chunk: U_0; state_0 += EB_0 V; U_1 (once A'_0 is drained);
+            // G = A'_0 EB_0; G += A'_1 EB_1; state_1 += EB_1 V; O = A'_0 W_0 (+ A'_1 W_1); O += G V.
             if (lane == 0) {
                 uint32_t ph_p = 0, ph_v = 0, ph_eb = 0, ph_ph = 0, ph_ufree = 0, ph_gfree = 0, ph_a0 = 0, ph_a1 = 0, ph_gready = 0;
                 uint32_t ph_w0 = 0, ph_w1 = 0, ph_sread = 0;
@@ -1386,6 +1386,14 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     mma_steps<true>(accU, sP, kC, sPHI, SP, id_U, SP / 16, false);
                     tc::mma_commit(&bar[VB_U_FULL]);
                     tc::mma_commit(&bar[VB_PH_FREE]);
+                    // state_0 += EB_0 V once this chunk's W tiles have been read from the state: it needs
+                    // neither A' nor G, so it runs while A'_0 is drained
+                    if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_STATE_READ], ph_sread, ctl, a.err)) break;
+                    if (!wait_bar(&bar[VB_V_FULL], ph_v, ctl, a.err)) break;
+                    tc::tc_fence_after();
+                    mma_steps<true>(tb, sE0, 128, sV, kC, id_O, kC / 16, true);
+                    tc::mma_commit(&bar[VB_STATE_DONE]);
                     if (NH == 2) {
                         // U_1 -> U once A'_0 is drained
                         if (!wait_bar(&bar[VB_PH_FULL], ph_ph, ctl, a.err)) break;
@@ -1397,17 +1405,10 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                     }
                     // G = A'_0 EB_0 -> G (last read by the previous chunk's G drain)
                     if (!wait_bar(&bar[VB_A_READY], ph_a0, ctl, a.err)) break;
-                    if (!wait_bar(&bar[VB_EB_FULL], ph_eb, ctl, a.err)) break;
                     if (!first && !wait_bar(&bar[VB_G_FREE], ph_gfree, ctl, a.err)) break;
                     tc::tc_fence_after();
                     mma_steps<true>(accG, sY0, kC, sE0, 128, id_G, RH / 16, false);
                     if (NH == 1) tc::mma_commit(&bar[VB_G_FULL]);
-                    // state_0 += EB_0 V once this chunk's W tiles have been read from the state
-                    if (!wait_bar(&bar[VB_STATE_READ], ph_sread, ctl, a.err)) break;
-                    if (!wait_bar(&bar[VB_V_FULL], ph_v, ctl, a.err)) break;
-                    tc::tc_fence_after();
-                    mma_steps<true>(tb, sE0, 128, sV, kC, id_O, kC / 16, true);
-                    tc::mma_commit(&bar[VB_STATE_DONE]);
                     tc::mma_commit(&bar[VB_P_FREE]);   // EB_0's buffer takes the next chunk's p
                     if (NH == 2) {
                         // G += A'_1 EB_1 (EB_1 in the PHI tile); state_1 += EB_1 V
