@@ -988,8 +988,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
         {
             // ---------------- epilogue warps 0-7: thread = TMEM lane = token row / state row;
             // warpgroup wg handles columns [wg*N/2, (wg+1)*N/2) of every N-column drain.
-            // Per chunk: W_1; Y_0; Y_1; W_0 (and W_1 into registers) of the next chunk; P of the next
-            // chunk; softmax (one half: softmax, then P).
+            // Per chunk: W_1; Y_0; W_0 of the next chunk; Y_1; softmax; P of the next chunk (one half:
+            // Y_0, W_0, softmax, P).
             const int row = threadIdx.x & 127, wg = threadIdx.x >> 7, lane_base = (warp & 3) * 32;
             // softmax partials [2 (max, sum)][2 (warpgroup)][128 rows] in the control area
             float *red = reinterpret_cast<float *>(sm + lay.bars + 1024);
