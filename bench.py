@@ -654,16 +654,40 @@ def stored_traffic(kernel, L):
 PASS_SOURCES = ("common.cuh", "fwd_bf16.cu", "fwd_bf16.cuh", "tc.cuh", "tmap.cu", "tmap.cuh")
 
 
+def _strip_comments(src):
+    """C/C++ source without its // and /* */ comments (string and character literals kept)."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        elif src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+        else:
+            out.append(c)
+            i += 1
+    return "".join(out)
+
+
 def _source_digest():
-    """Digest of the sources of the chunked passes; a stored DRAM-traffic figure of a pass is used
-    only if it matches (any change to those files may change the pass kernels)."""
+    """Digest of the sources of the chunked passes, comments removed; a stored DRAM-traffic figure
+    of a pass is used only if it matches (any change to the code of those files may change the
+    pass kernels, a change to a comment does not)."""
     import hashlib
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2606_09862_gb300", "csrc")
     for fn in PASS_SOURCES:
-        with open(os.path.join(d, fn), "rb") as f:
+        with open(os.path.join(d, fn), encoding="utf-8") as f:
             h.update(fn.encode())
-            h.update(f.read())
+            h.update(_strip_comments(f.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -62,3 +62,37 @@ def test_reference_arm_non_zero_rank_exits_quietly():
                         "--steps", "1", "--warmup", "0"], env=env, capture_output=True, text=True, timeout=120)
     assert r.returncode == 0, r.stderr
     assert r.stdout.strip() == ""
+
+
+def _bench_module():
+    import importlib.util
+    spec = importlib.util.spec_from_file_location("bench_for_digest", os.path.join(ROOT, "bench.py"))
+    mod = importlib.util.module_from_spec(spec)
+    argv = sys.argv
+    sys.argv = ["bench.py"]
+    try:
+        spec.loader.exec_module(mod)
+    finally:
+        sys.argv = argv
+    return mod
+
+
+def test_source_digest_ignores_comments_only():
+    b = _bench_module()
+    src = 'int a = 1; // note\nconst char *s = "//kept"; /* block\n comment */ char c = \'/\';\n'
+    assert b._strip_comments(src) == 'int a = 1; \nconst char *s = "//kept";  char c = \'/\';\n'
+    # a comment edit keeps the stripped text, a code edit changes it
+    assert b._strip_comments(src.replace("note", "other note")) == b._strip_comments(src)
+    assert b._strip_comments(src.replace("a = 1", "a = 2")) != b._strip_comments(src)
+
+
+def test_stored_traffic_is_plausible_when_current():
+    # bench.py reports a pass's DRAM traffic only while the figure under profiles/ was captured from
+    # the current pass kernels; such a figure lies near the pass's algorithmic bytes (809.5 MB)
+    b = _bench_module()
+    for kern in ("kpass", "vpass"):
+        t = b.stored_traffic(kern, 65536)
+        if t is None:
+            pytest.skip("the %s traffic figure predates the current sources" % kern)
+        assert 7e8 < t < 1e9, (kern, t)
+        assert b.stored_traffic(kern, 32768) == t / 2
