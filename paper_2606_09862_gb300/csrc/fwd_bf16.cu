@@ -1091,7 +1091,8 @@ __global__ void __launch_bounds__(kPassThreads, 1)
                 epi_arrive(&bar[KB_ACC_FREE_A]);
                 return true;
             };
-            // W_0 and W_1 of the first chunk (the carried-in state as it is) and its P
+            // W_0 of the first chunk (the carried-in state as it is) and its P; every W_1 is copied at the
+            // start of its chunk
             bool bad = false;
             if (c_begin < c_end) bad = !w_copy(0, false, false) || !p_drain();
             for (int c = c_begin; c < c_end && !bad; ++c) {
