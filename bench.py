@@ -678,16 +678,17 @@ def _strip_comments(src):
 
 
 def _source_digest():
-    """Digest of the sources of the chunked passes, comments removed; a stored DRAM-traffic figure
-    of a pass is used only if it matches (any change to the code of those files may change the
-    pass kernels, a change to a comment does not)."""
+    """Digest of the sources of the chunked passes with comments removed and whitespace runs
+    collapsed; a stored DRAM-traffic figure of a pass is used only if it matches (any change to the
+    code of those files may change the pass kernels, a change to a comment or a line break does
+    not)."""
     import hashlib
     h = hashlib.sha256()
     d = os.path.join(ROOT, "paper_2606_09862_gb300", "csrc")
     for fn in PASS_SOURCES:
         with open(os.path.join(d, fn), encoding="utf-8") as f:
             h.update(fn.encode())
-            h.update(_strip_comments(f.read()).encode())
+            h.update(" ".join(_strip_comments(f.read()).split()).encode())
     return h.hexdigest()[:16]
 
 

@@ -84,6 +84,10 @@ def test_source_digest_ignores_comments_only():
     # a comment edit keeps the stripped text, a code edit changes it
     assert b._strip_comments(src.replace("note", "other note")) == b._strip_comments(src)
     assert b._strip_comments(src.replace("a = 1", "a = 2")) != b._strip_comments(src)
+    # the digest also ignores line breaks and indentation (a comment that grows by a line)
+    def digest(text):
+        return " ".join(b._strip_comments(text).split())
+    assert digest(src.replace("// note", "// note\n    // more")) == digest(src)
 
 
 def test_stored_traffic_is_plausible_when_current():
