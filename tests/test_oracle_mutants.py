@@ -51,6 +51,15 @@ MUTANTS = {
     "explicit_scale_ignored": ("c.scale = scale > 0.0 ? scale : 1.0 / sqrt((double)dk);",
                                "c.scale = 1.0 / sqrt((double)dk);"),
     "decay_value_not_decayed": ("Vp[j * dv + e] = keep * Vp[j * dv + e] + ip[j]", "Vp[j * dv + e] = Vp[j * dv + e] + ip[j]"),
+    # the VJPs: a transposed operand, a dropped weight, an off-by-one causal range, a dropped centering
+    "backward_dk_transposed_operand": ("dk_[(size_t)u * dk + i] += dP * qt[i];\n            }\n            for (int i = 0; i < dv; ++i) dv_[(size_t)u * dv + i] += g * dot[i];\n        }\n    }\n    free(Dt);",
+                                       "dk_[(size_t)u * dk + i] += dP * k[(size_t)u * dk + i];\n            }\n            for (int i = 0; i < dv; ++i) dv_[(size_t)u * dv + i] += g * dot[i];\n        }\n    }\n    free(Dt);"),
+    "backward_dv_unweighted": ("double wgt = Dt[weight_arg(absolute, t, u, (int)delta[j]) + off];\n                g += p[j] * wgt;",
+                               "double wgt = Dt[weight_arg(absolute, t, u, (int)delta[j]) + off];\n                g += p[j];"),
+    "backward_excludes_current_token": ("for (int u = 0; u <= t; ++u) {\n            double g = 0.0, dP = 0.0;\n            for (int j = 0; j < S; ++j) {\n                double wgt = Dt[",
+                                        "for (int u = 0; u < t; ++u) {\n            double g = 0.0, dP = 0.0;\n            for (int j = 0; j < S; ++j) {\n                double wgt = Dt["),
+    "decay_backward_no_centering": ("double wgt = Wt[(size_t)u * S + j];\n                g += p[j] * wgt;\n                dP += p[j] * (dp[j] - pdp) * wgt;",
+                                    "double wgt = Wt[(size_t)u * S + j];\n                g += p[j] * wgt;\n                dP += p[j] * dp[j] * wgt;"),
 }
 
 
