@@ -51,6 +51,14 @@ MUTANTS = {
     "explicit_scale_ignored": ("c.scale = scale > 0.0 ? scale : 1.0 / sqrt((double)dk);",
                                "c.scale = 1.0 / sqrt((double)dk);"),
     "decay_value_not_decayed": ("Vp[j * dv + e] = keep * Vp[j * dv + e] + ip[j]", "Vp[j * dv + e] = Vp[j * dv + e] + ip[j]"),
+    # state layout on the way in and out, the mode read-out, the log-sum-exp
+    "store_state_swapped_rows": ("memcpy(sk + (size_t)(2 * m) * dk, Kc + m * dk, sizeof(double) * dk);\n        memcpy(sk + (size_t)(2 * m + 1) * dk, Ks + m * dk, sizeof(double) * dk);",
+                                 "memcpy(sk + (size_t)(2 * m) * dk, Ks + m * dk, sizeof(double) * dk);\n        memcpy(sk + (size_t)(2 * m + 1) * dk, Kc + m * dk, sizeof(double) * dk);"),
+    "load_state_value_rows_swapped": ("memcpy(Vc + m * dv, sv + (size_t)(2 * m) * dv, sizeof(double) * dv);\n        memcpy(Vs + m * dv, sv + (size_t)(2 * m + 1) * dv, sizeof(double) * dv);",
+                                      "memcpy(Vc + m * dv, sv + (size_t)(2 * m + 1) * dv, sizeof(double) * dv);\n        memcpy(Vs + m * dv, sv + (size_t)(2 * m) * dv, sizeof(double) * dv);"),
+    "modes_readout_swapped": ("acc += uc[m] * Vc[m * dv + i] + us[m] * Vs[m * dv + i];", "acc += uc[m] * Vs[m * dv + i] + us[m] * Vc[m * dv + i];"),
+    "lse_without_max": ("return mx + log(sum);", "return log(sum);"),
+    "lse_base2": ("return mx + log(sum);", "return mx + log2(sum);"),
     # the VJPs: a transposed operand, a dropped weight, an off-by-one causal range, a dropped centering
     "backward_dk_transposed_operand": ("dk_[(size_t)u * dk + i] += dP * qt[i];\n            }\n            for (int i = 0; i < dv; ++i) dv_[(size_t)u * dv + i] += g * dot[i];\n        }\n    }\n    free(Dt);",
                                        "dk_[(size_t)u * dk + i] += dP * k[(size_t)u * dk + i];\n            }\n            for (int i = 0; i < dv; ++i) dv_[(size_t)u * dv + i] += g * dot[i];\n        }\n    }\n    free(Dt);"),
